@@ -1,0 +1,263 @@
+/*
+ * omq.h — C ABI of libomq: one OmniQuant block-calibration step on a GB300 (sm_103a).
+ *
+ * The step is the inner loop of Algorithm 1 (Appendix A): apply the learnable
+ * equivalent transformation (LET, Eq. 3-5) and learnable weight clipping (LWC,
+ * Eq. 2) to a transformer block, run the quantized block on a calibration sample,
+ * take the MSE against the full-precision block output (Eq. 1), and back-propagate
+ * with the straight-through estimator to gamma, beta (Theta1) and s, delta, s_a
+ * (Theta2).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Memory: every tensor pointer is a DEVICE pointer owned by the caller.  The
+ *    library never allocates, frees or synchronises; every call only enqueues
+ *    work on `stream` and returns.  Scratch memory is a caller-provided workspace
+ *    whose size is queried first.
+ *  - Layouts are row-major.  A weight W is [Cout, Cin] (the transpose of the
+ *    paper's C_in x C_out notation in Sec. 3.3); activations are [T, C].
+ *  - Dtypes: frozen weights bf16; activations, learnable parameters, per-group /
+ *    per-token scales and all gradients fp32; zero points and argmax/argmin
+ *    indices int32; integer codes uint8.
+ *  - Alignment: every pointer must be 16-byte aligned and every inner dimension a
+ *    multiple of 8 elements, else OMQ_ERR_ALIGN.  There is no slow path.
+ *  - Errors: argument errors are found on the host before any launch, and then
+ *    nothing is written.  Device-side failures (a bounded wait that expired) are
+ *    written to the optional `dev_status` word of omq_qcfg and read back with
+ *    omq_stream_status.  The library never aborts, traps or prints.
+ *  - Gradient outputs are overwritten unless cfg->accumulate is 1, in which case
+ *    they are added to.
+ *  - Rounding: round() of Eq. 2 is round-half-to-even; every matrix-product operand
+ *    is rounded to bf16 (nearest-even) and accumulated in fp32.
+ */
+#ifndef OMQ_H
+#define OMQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* omq_stream_t;   /* same type as cudaStream_t; NULL = legacy default stream */
+
+typedef enum {
+  OMQ_OK = 0,
+  OMQ_ERR_INVALID_ARG = 1,   /* null where required, bad enum value */
+  OMQ_ERR_SHAPE = 2,         /* zero or negative size, group does not divide Cin, heads do not divide */
+  OMQ_ERR_ALIGN = 3,         /* pointer not 16-byte aligned or inner dimension not a multiple of 8 */
+  OMQ_ERR_UNSUPPORTED = 4,   /* bit width outside [2, 8] (or 16 = off); device is not sm_103 */
+  OMQ_ERR_CUDA = 5,          /* a launch failed */
+  OMQ_ERR_TIMEOUT = 6,       /* a device-side bounded wait expired (reported through dev_status) */
+  OMQ_ERR_WORKSPACE = 7      /* workspace smaller than the queried size */
+} omq_status;
+
+/* Quantization configuration (Sec. 4.1 "Quantization"). */
+typedef struct {
+  int32_t wbits;       /* weight bits N of Eq. 2: 2..8, or 16 = weights not quantized            */
+  int32_t abits;       /* per-token activation bits: 2..8, or 16 = activations not quantized     */
+  int32_t group;       /* weight group size along Cin; 0 = one group per output channel          */
+  int32_t let;         /* 1 = learnable equivalent transformation on (Eq. 3, Eq. 5)               */
+  float   h_eps;       /* floor of the quantizer step h (1e-5); a floored h has zero gradient    */
+  int32_t accumulate;  /* 1 = add into gradient outputs instead of overwriting them              */
+  int32_t* dev_status; /* optional device int32: 0 = ok, else an omq_status set by a kernel      */
+} omq_qcfg;
+
+/* ------------------------------------------------------------------------------------------
+ * Kernel-level entry points
+ * ------------------------------------------------------------------------------------------ */
+
+/* Eq. 3.  X~ = (X - delta) / s per input channel, W~ = W diag(s), B~ = B + W delta.
+ *   X [T, Cin] fp32, W [Cout, Cin] bf16, B [Cout] fp32 or NULL (= 0), s, delta [Cin] fp32.
+ *   Xt [T, Cin] fp32 (NULL = skip), Wt [Cout, Cin] fp32 (NULL = skip), Bt [Cout] fp32 (NULL = skip). */
+omq_status omq_let_apply(omq_stream_t stream, int64_t T, int64_t Cin, int64_t Cout,
+                         const float* X, const void* W, const float* B, const float* s,
+                         const float* delta, float* Xt, float* Wt, float* Bt, const omq_qcfg* cfg);
+
+/* Eq. 2 (LWC) on W~ = r_o * W_oi * s_i, per group of cfg->group input channels of one output row.
+ *   W [Cout, Cin] bf16; s [Cin] (NULL = 1: LET scale of Eq. 3); r [Cout] (NULL = 1: row scale, the
+ *   1/s_o that the [v, out] LET pair puts on v_proj's rows).  gamma_logit, beta_logit
+ *   [Cout, ngroups] fp32 with gamma = sigmoid(gamma_logit).
+ *   Outputs: Wq [Cout, Cin] bf16 fake-quantized value (q - z) h (NULL = skip); codes [Cout, Cin]
+ *   uint8 (NULL = skip); h [Cout, ngroups] fp32; z int32; argmax / argmin int32 = column index
+ *   (in 0..Cin-1) of the first max / min of each group.
+ *   bias_delta [Cin] (NULL = skip) and bias_shift [Cout] (NULL = 0): when bias_delta is given, also
+ *   writes Bt[o] = r_o * (sum_i W_oi bias_delta_i - bias_shift_o) (the B~ of Eq. 3). */
+omq_status omq_lwc_fakequant_fwd(omq_stream_t stream, int64_t Cout, int64_t Cin, const void* W,
+                                 const float* s, const float* r, const float* gamma_logit,
+                                 const float* beta_logit, void* Wq, uint8_t* codes, float* h,
+                                 int32_t* z, int32_t* argmax, int32_t* argmin,
+                                 const float* bias_delta, const float* bias_shift, float* Bt,
+                                 const omq_qcfg* cfg);
+
+/* Straight-through backward of omq_lwc_fakequant_fwd, given dWq = dL/dWq [Cout, Cin] fp32 and the
+ * saved h, z, argmax, argmin.  Every round() has derivative 1; clamp passes the gradient for
+ * 0 <= code <= 2^N-1; max/min route theirs to the saved first index; h is not detached.
+ *   dgamma, dbeta [Cout, ngroups] fp32.  dWt [Cout, Cin] fp32 = dL/dW~ (NULL = skip).
+ *   ds [Cin] (NULL = skip) = sum_o dWt_oi W_oi r_o;  dr [Cout] (NULL = skip) = sum_i dWt_oi W_oi s_i.
+ *   dBt [Cout] (NULL = none) with ddelta [Cin] (NULL = skip): ddelta_i = sum_o dBt_o r_o W_oi, the
+ *   bias path of Eq. 3.  A scratch workspace of omq_lwc_bwd_workspace_size bytes is required when
+ *   ds or ddelta is requested. */
+omq_status omq_lwc_fakequant_bwd(omq_stream_t stream, int64_t Cout, int64_t Cin, const void* W,
+                                 const float* s, const float* r, const float* gamma_logit,
+                                 const float* beta_logit, const float* h, const int32_t* z,
+                                 const int32_t* argmax, const int32_t* argmin, const float* dWq,
+                                 float* dgamma, float* dbeta, float* dWt, float* ds, float* dr,
+                                 const float* dBt, float* ddelta, void* workspace, size_t ws_bytes,
+                                 const omq_qcfg* cfg);
+size_t omq_lwc_bwd_workspace_size(int64_t Cout, int64_t Cin);
+
+/* LET on activations (Eq. 3, X~ = (X - delta)/s; s, delta NULL = identity) followed by Q_a, the
+ * per-token MinMax quantizer (Eq. 2 with gamma = beta = 1, one group per row, N = cfg->abits).
+ *   X [T, C] fp32 -> Xq [T, C] bf16 = (q - z) h (or bf16(X~) when abits = 16);
+ *   codes [T, C] uint8 (NULL = skip); h [T] fp32, z [T], argmax [T], argmin [T] int32
+ *   (all NULL allowed when abits = 16). */
+omq_status omq_act_quant_per_token(omq_stream_t stream, int64_t T, int64_t C, const float* X,
+                                   const float* s, const float* delta, void* Xq, uint8_t* codes,
+                                   float* h, int32_t* z, int32_t* argmax, int32_t* argmin,
+                                   const omq_qcfg* cfg);
+
+/* Straight-through backward of omq_act_quant_per_token, given dXq [T, C] fp32 and the saved
+ * per-token state.  dX [T, C] fp32 = dL/dX; ds, ddelta [C] (NULL = skip) are the LET column sums
+ * ds_i = -sum_t dX~_ti X~_ti / s_i and ddelta_i = -sum_t dX~_ti / s_i.  Needs a workspace of
+ * omq_act_bwd_workspace_size bytes when ds or ddelta is requested. */
+omq_status omq_act_quant_per_token_bwd(omq_stream_t stream, int64_t T, int64_t C, const float* X,
+                                       const float* s, const float* delta, const float* h,
+                                       const int32_t* z, const int32_t* argmax,
+                                       const int32_t* argmin, const float* dXq, float* dX,
+                                       float* ds, float* ddelta, void* workspace, size_t ws_bytes,
+                                       const omq_qcfg* cfg);
+size_t omq_act_bwd_workspace_size(int64_t T, int64_t C);
+
+/* Block loss of Eq. 1 / Algorithm 1, read as the mean over the n elements of (Yq - Yfp)^2.
+ *   loss: device fp32 scalar (overwritten).  dY [n] fp32 = 2 (Yq - Yfp) / n (NULL = skip);
+ *   dY_bf16 [n] bf16 copy of dY (NULL = skip).  Needs omq_loss_workspace_size bytes. */
+omq_status omq_block_loss(omq_stream_t stream, int64_t n, const float* Yq, const float* Yfp,
+                          float* loss, float* dY, void* dY_bf16, void* workspace, size_t ws_bytes);
+size_t omq_loss_workspace_size(int64_t n);
+
+/* Dense bf16 tensor-core matrix product used by every linear and attention product:
+ *   C[b, m, n] = alpha * sum_k A[b, m, k] B[b, n, k] (+ bias[n]) (+ R[b, m, n]) (+ beta_acc * C)
+ * A element (b, m, k) is at A + b*a_bs + (a_kmajor ? m*a_ld + k : k*a_ld + m); B likewise with n.
+ * Operands bf16, accumulation fp32 in tensor memory (tcgen05).  Cf [b, m, n] fp32 at
+ * Cf + b*c_bs + m*ldc + n (NULL = skip); Cb the same positions in bf16 (NULL = skip).
+ * causal: 0 none; 1 = skip output tiles with n-start > m-end (scores); 2 = k < m-tile end only
+ * (P V, dS K); 3 = k >= m-tile start only (P^T dO, dS^T Q).  Causal tiles assume square 128 tiles. */
+omq_status omq_gemm_bf16(omq_stream_t stream, int64_t M, int64_t N, int64_t K, int64_t batch,
+                         const void* A, int64_t a_ld, int64_t a_bs, int32_t a_kmajor,
+                         const void* B, int64_t b_ld, int64_t b_bs, int32_t b_kmajor,
+                         float* Cf, void* Cb, int64_t ldc, int64_t c_bs, float alpha,
+                         const float* bias, const float* R, int64_t ldr, float beta_acc,
+                         int32_t causal, int32_t* dev_status);
+
+/* ------------------------------------------------------------------------------------------
+ * Single quantized linear (Eq. 4): Y = Q_a(X~) Q_w(W~)^T + B~, and its STE backward.
+ * ------------------------------------------------------------------------------------------ */
+typedef struct {
+  void*    w_hat;   /* [Cout, Cin] bf16 fake-quantized W~                                    */
+  float*   h_w;     /* [Cout, ngroups] */
+  int32_t* z_w;
+  int32_t* imax_w;
+  int32_t* imin_w;
+  void*    x_hat;   /* [T, Cin] bf16 quantized (or rounded) X~                               */
+  float*   h_a;     /* [T] (unused when abits = 16) */
+  int32_t* z_a;
+  int32_t* imax_a;
+  int32_t* imin_a;
+  float*   b_tilde; /* [Cout] fp32 B~ */
+} omq_qlinear_saved;
+
+omq_status omq_qlinear_fwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t Cout,
+                           const float* X, const void* W, const float* B, const float* s,
+                           const float* delta, const float* gamma_logit, const float* beta_logit,
+                           float* Y, const omq_qlinear_saved* saved, const omq_qcfg* cfg);
+/* dY [T, Cout] fp32.  dX [T, Cin] fp32 (NULL = skip).  dgamma, dbeta [Cout, ngroups];
+ * ds, ddelta [Cin] (required when cfg->let). */
+omq_status omq_qlinear_bwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t Cout,
+                           const float* X, const void* W, const float* s, const float* delta,
+                           const float* gamma_logit, const float* beta_logit,
+                           const omq_qlinear_saved* saved, const float* dY, float* dX,
+                           float* dgamma, float* dbeta, float* ds, float* ddelta,
+                           void* workspace, size_t ws_bytes, const omq_qcfg* cfg);
+size_t omq_qlinear_workspace_size(int64_t T, int64_t Cin, int64_t Cout, const omq_qcfg* cfg);
+
+/* ------------------------------------------------------------------------------------------
+ * One LLaMA decoder block (RMSNorm -> RoPE causal attention -> RMSNorm -> SwiGLU FFN), the
+ * block F of Eq. 1.  LET pairs (Sec. 3.3 and the appendix ablation of LET positions):
+ * [ln1, (q, k, v)] with s1, d1 [d]; [v, out] with so, do [n_kv*hd] moved into v_proj;
+ * [Q, K] with sa [n_kv*hd] applied after RoPE; [ln2, (gate, up)] with s2, d2 [d]; none on down.
+ * With grouped KV heads so, do, sa are broadcast to the query heads of each group.
+ * ------------------------------------------------------------------------------------------ */
+typedef struct {
+  int32_t T;          /* tokens of one calibration sample */
+  int32_t d;          /* hidden size */
+  int32_t n_heads;    /* query heads */
+  int32_t n_kv;       /* key/value heads (divides n_heads) */
+  int32_t head_dim;   /* must be 128 */
+  int32_t ffn;        /* SwiGLU inner size */
+  float   rms_eps;
+  float   rope_theta;
+} omq_block_shape;
+
+/* Frozen bf16 weights, [Cout, Cin].  wqkv stacks the rows of q_proj [n_heads*hd, d], k_proj
+ * [n_kv*hd, d] and v_proj [n_kv*hd, d]; wgu stacks gate_proj [ffn, d] then up_proj [ffn, d]. */
+typedef struct {
+  const void* wqkv;
+  const void* wo;     /* [d, n_heads*hd] */
+  const void* wgu;
+  const void* wd;     /* [d, ffn] */
+} omq_block_weights;
+
+/* LWC logits [Cout, ngroups] fp32 stacked like the weights, and the LET vectors (NULL when
+ * cfg->let = 0).  The gradient struct has the same layout. */
+typedef struct {
+  float* gamma_qkv; float* beta_qkv;
+  float* gamma_o;   float* beta_o;
+  float* gamma_gu;  float* beta_gu;
+  float* gamma_d;   float* beta_d;
+  float* s1; float* d1;   /* [d] */
+  float* so; float* do_;  /* [n_kv*hd] */
+  float* sa;              /* [n_kv*hd] */
+  float* s2; float* d2;   /* [d] */
+} omq_block_params;
+
+size_t omq_block_workspace_size(const omq_block_shape* shape, const omq_qcfg* cfg);
+
+/* Forward of the quantized block on x [T, d] fp32 (y [T, d] fp32 out).  With wbits = abits = 16
+ * and let = 0 this is the full-precision block that produces the Eq. 1 target. */
+omq_status omq_block_forward(omq_stream_t stream, const omq_block_shape* shape,
+                             const omq_block_weights* w, const omq_block_params* theta,
+                             const float* x, float* y, void* workspace, size_t ws_bytes,
+                             const omq_qcfg* cfg);
+
+/* One calibration step without the parameter update: forward, loss = mean((y - y_fp)^2) written
+ * to the device scalar `loss`, and the STE gradients of every learnable parameter into `grads`.
+ * y (NULL = not returned) receives the quantized block output. */
+omq_status omq_block_step(omq_stream_t stream, const omq_block_shape* shape,
+                          const omq_block_weights* w, const omq_block_params* theta,
+                          const float* x, const float* y_fp, float* y, float* loss,
+                          const omq_block_params* grads, void* workspace, size_t ws_bytes,
+                          const omq_qcfg* cfg);
+
+/* AdamW update of one fp32 parameter vector (Sec. 4.1 "Training": AdamW, weight decay 0):
+ * m = b1 m + (1-b1) g; v = b2 v + (1-b2) g^2; p -= lr * (m / (1-b1^t)) / (sqrt(v / (1-b2^t)) + eps)
+ * - lr * wd * p.  step t >= 1. */
+omq_status omq_adamw_update(omq_stream_t stream, int64_t n, float* p, const float* g, float* m,
+                            float* v, float lr, float beta1, float beta2, float eps,
+                            float weight_decay, int32_t step);
+
+/* Reads the device status word written by kernels (synchronises `stream`).  *host_out receives
+ * the word (0 = ok); the return value is OMQ_OK or OMQ_ERR_CUDA if the copy failed. */
+omq_status omq_stream_status(omq_stream_t stream, const int32_t* dev_status, int32_t* host_out);
+
+/* Human-readable name of a status code (static string). */
+const char* omq_status_string(omq_status s);
+
+/* Library version, for the bindings' sanity check. */
+int32_t omq_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* OMQ_H */

@@ -48,6 +48,11 @@ notes of the repository):
      its transform into v_proj: W_v' = diag(1/s_o) W_v diag(s1),
      b_v' = (W_v delta1 - delta_o) / s_o, and the out_proj input is P V'
      (Sec. 3.3, last paragraph).
+ R15 where floating point decides an integer (a code, a zero point, a max/min
+     index, the floor of h) the decision is taken in the precision of the
+     kernels, IEEE single precision with one rounding per product, difference and
+     quotient, and the sigmoid rounded once from double; everything else stays
+     float64.  ("emulate" mode; "exact" mode decides in float64.)
 """
 from __future__ import annotations
 
@@ -107,25 +112,57 @@ def _first_argmin(w: torch.Tensor) -> torch.Tensor:
 # Eq. 2, explicit forward and STE backward of one quantizer over groups on the last axis
 # ----------------------------------------------------------------------------------------------
 
-def quant_fwd(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5) -> Dict[str, torch.Tensor]:
+def _decide_fp32(w: torch.Tensor, a, b, Q: float, eps: float):
+    """The integer decisions of Eq. 2 taken in IEEE single precision (R15).
+
+    Inputs are rounded to fp32 and every product, difference and quotient is rounded to fp32:
+    h = (a*M - b*m)/Q, u = (b*m)/h, x = w/h.  Returns the first argmax/argmin of the fp32
+    group, the floor flag and h, u, x as fp32 values."""
+    f32 = torch.float32
+    w32 = w.detach().to(f32)
+    a32 = torch.as_tensor(a).detach().to(f32)
+    b32 = torch.as_tensor(b).detach().to(f32)
+    imax = _first_argmax(w32)
+    imin = _first_argmin(w32)
+    M32 = torch.gather(w32, -1, imax[..., None])[..., 0]
+    m32 = torch.gather(w32, -1, imin[..., None])[..., 0]
+    aM = a32 * M32
+    bm = b32 * m32
+    hr = (aM - bm) / Q
+    floored = hr < eps
+    h32 = torch.where(floored, torch.full_like(hr, eps), hr)
+    u32 = bm / h32
+    x32 = w32 / h32[..., None]
+    return imax, imin, floored, h32, u32, x32
+
+
+def quant_fwd(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5, decide: str = "fp64") -> Dict[str, torch.Tensor]:
     """Eq. 2 over groups laid out on the last axis of `w` (shape [..., g]).
 
     a, b are the clipping strengths gamma, beta (tensors of shape [...] or floats; 1.0 gives
-    MinMax, the special case stated after Eq. 2).  Returns every intermediate."""
+    MinMax, the special case stated after Eq. 2).  decide = "fp64" takes every decision in
+    float64; "fp32" takes max/min, h, z and the codes in IEEE single precision (R15).
+    Returns every intermediate."""
     w = w.to(F64)
     Q = float(2 ** nbits - 1)
     a = torch.as_tensor(a, dtype=F64)
     b = torch.as_tensor(b, dtype=F64)
-    imax = _first_argmax(w)
-    imin = _first_argmin(w)
-    M = torch.gather(w, -1, imax[..., None])[..., 0]
-    m = torch.gather(w, -1, imin[..., None])[..., 0]
-    h_raw = (a * M - b * m) / Q
-    floored = h_raw < eps                                  # R3
-    h = torch.where(floored, torch.full_like(h_raw, eps), h_raw)
-    u = b * m / h
+    if decide == "fp32":
+        imax, imin, floored, h32, u32, x32 = _decide_fp32(w, a, b, Q, eps)
+        M = torch.gather(w, -1, imax[..., None])[..., 0]
+        m = torch.gather(w, -1, imin[..., None])[..., 0]
+        h, u, x = h32.to(F64), u32.to(F64), x32.to(F64)
+    else:
+        imax = _first_argmax(w)
+        imin = _first_argmin(w)
+        M = torch.gather(w, -1, imax[..., None])[..., 0]
+        m = torch.gather(w, -1, imin[..., None])[..., 0]
+        h_raw = (a * M - b * m) / Q
+        floored = h_raw < eps                              # R3
+        h = torch.where(floored, torch.full_like(h_raw, eps), h_raw)
+        u = b * m / h
+        x = w / h[..., None]
     z = -rne(u)
-    x = w / h[..., None]
     c = rne(x) + z[..., None]
     q = torch.clamp(c, 0.0, Q)
     what = (q - z[..., None]) * h[..., None]               # R1
@@ -211,11 +248,14 @@ class use_tape:
         _TAPE = self.prev
 
 
-def quant_ste(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5) -> torch.Tensor:
+def quant_ste(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5, decide: str = "fp64",
+              w_dec: Optional[torch.Tensor] = None) -> torch.Tensor:
     """Eq. 2 fake quantization as an autograd graph whose gradient is the STE of R7.
 
     Groups on the last axis; a, b broadcast against w[..., 0] (tensors that may require
-    grad, or floats for Q_a)."""
+    grad, or floats for Q_a).  With decide = "fp32" the max/min, the floor, the value of h and
+    every round() are taken in IEEE single precision from `w_dec` (default: w rounded to
+    fp32), as the kernels take them (R15); the gradient is the same STE."""
     Q = float(2 ** nbits - 1)
     tape = _TAPE
     if tape is not None and tape.mode == "replay":
@@ -229,6 +269,21 @@ def quant_ste(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5) -> torch.Ten
         z = -(u + r["ru"])
         c = w / h[..., None] + r["rx"] + z[..., None]
         q = torch.where(r["inr"], c, torch.where(r["below"], torch.zeros_like(c), torch.full_like(c, Q)))
+        return (q - z[..., None]) * h[..., None]
+    if decide == "fp32":
+        assert tape is None, "the frozen-offset surrogate is defined for float64 decisions"
+        with torch.no_grad():
+            imax, imin, floored, h32, u32, x32 = _decide_fp32(w if w_dec is None else w_dec, a, b, Q, eps)
+        M = torch.gather(w, -1, imax[..., None])[..., 0]
+        m = torch.gather(w, -1, imin[..., None])[..., 0]
+        h_raw = (a * M - b * m) / Q
+        h = torch.where(floored, torch.full_like(h_raw, eps), h_raw)     # R3: no gradient when floored
+        h = h + (h32.to(F64) - h).detach()                                 # value of the fp32 step
+        u = b * m / h
+        z = -(u + (rne(u32.to(F64)) - u).detach())
+        x = w / h[..., None]
+        c = x + (rne(x32.to(F64)) - x).detach() + z[..., None]
+        q = torch.clamp(c, 0.0, Q)
         return (q - z[..., None]) * h[..., None]
     imax = _first_argmax(w.detach())
     imin = _first_argmin(w.detach())
@@ -274,23 +329,37 @@ def _groups(W: torch.Tensor, group: int) -> torch.Tensor:
     return W.reshape(cout, cin // g, g)                    # R6
 
 
+def _wt_fp32(W, s, row_scale):
+    """W~ = fl32(fl32(W * s) * r), the kernels' single-precision quantizer input (R15)."""
+    wt = W.to(torch.float32)
+    if s is not None:
+        wt = wt * s.to(torch.float32)[None, :]
+    if row_scale is not None:
+        wt = wt * row_scale.to(torch.float32)[:, None]
+    return wt
+
+
 def lwc_fakequant_fwd(W, gamma_logit, beta_logit, nbits: int, group: int,
                       s: Optional[torch.Tensor] = None, eps: float = 1e-5,
-                      row_scale: Optional[torch.Tensor] = None) -> Dict[str, torch.Tensor]:
+                      row_scale: Optional[torch.Tensor] = None, decide: str = "fp64") -> Dict[str, torch.Tensor]:
     """LWC of Eq. 2 on W~ = s (.) W (Eq. 3) for W [Cout, Cin].
 
     row_scale (optional, [Cout]) multiplies each output row before quantization; it is how
     the [v, out] LET pair divides v_proj's rows by s_o (R14).  Returns h, z [Cout, ngroups],
     the first argmax/argmin inside each group (as column indices into Cin), integer codes,
-    W_hat [Cout, Cin] and the quantizer input Wt."""
+    W_hat [Cout, Cin] and the quantizer input Wt.  decide = "fp32" forms W~ and takes the
+    quantizer's decisions in single precision (R15)."""
     W = W.to(F64)
-    Wt = W if s is None else W * s.to(F64)[None, :]
-    if row_scale is not None:
-        Wt = Wt * row_scale.to(F64)[:, None]
+    if decide == "fp32":
+        Wt = _wt_fp32(W, s, row_scale).to(F64)
+    else:
+        Wt = W if s is None else W * s.to(F64)[None, :]
+        if row_scale is not None:
+            Wt = Wt * row_scale.to(F64)[:, None]
     G = _groups(Wt, group)
     a = sigmoid(gamma_logit.to(F64))
     b = sigmoid(beta_logit.to(F64))
-    st = quant_fwd(G, a, b, nbits, eps)
+    st = quant_fwd(G, a, b, nbits, eps, decide)
     gsz = G.shape[-1]
     base = torch.arange(G.shape[1], dtype=torch.int64)[None, :] * gsz
     return dict(st=st, Wt=Wt, h=st["h"], z=st["z"], argmax=st["imax"] + base, argmin=st["imin"] + base,
@@ -318,16 +387,19 @@ def lwc_fakequant_bwd(fwd: Dict[str, torch.Tensor], W, dWhat, s: Optional[torch.
 
 
 def act_quant_per_token(X, nbits: int, s: Optional[torch.Tensor] = None,
-                        delta: Optional[torch.Tensor] = None, eps: float = 1e-5) -> Dict[str, torch.Tensor]:
+                        delta: Optional[torch.Tensor] = None, eps: float = 1e-5,
+                        decide: str = "fp64") -> Dict[str, torch.Tensor]:
     """LET on activations (Eq. 3: X~ = (X - delta)/s) followed by Q_a, the per-token MinMax
-    quantizer (gamma = beta = 1 in Eq. 2; one group per token row)."""
-    X = X.to(F64)
-    Xt = X
+    quantizer (gamma = beta = 1 in Eq. 2; one group per token row).  decide = "fp32" forms X~
+    and takes the quantizer's decisions in single precision (R15)."""
+    dt = torch.float32 if decide == "fp32" else F64
+    Xt = X.to(dt)
     if delta is not None:
-        Xt = Xt - delta.to(F64)[None, :]
+        Xt = Xt - delta.to(dt)[None, :]
     if s is not None:
-        Xt = Xt / s.to(F64)[None, :]
-    st = quant_fwd(Xt, 1.0, 1.0, nbits, eps)
+        Xt = Xt / s.to(dt)[None, :]
+    Xt = Xt.to(F64)
+    st = quant_fwd(Xt, 1.0, 1.0, nbits, eps, decide)
     return dict(st=st, Xt=Xt, Xq=st["what"], codes=st["q"].to(torch.int64), h=st["h"], z=st["z"],
                 argmax=st["imax"], argmin=st["imin"])
 
@@ -416,10 +488,17 @@ def qlinear_step(X, W, B, gamma_logit, beta_logit, Yfp, wbits: int, group: int, 
     Bt = (torch.zeros(W.shape[0], dtype=F64) if B is None else B.to(F64))
     if sv is not None:
         Bt = Bt + W @ dv
-    Xh = Xt if abits >= 16 else quant_ste(Xt, 1.0, 1.0, abits, eps)
+    decide = "fp32" if mode == "emulate" else "fp64"
+    with torch.no_grad():
+        xd = X.to(torch.float32)
+        if sv is not None:
+            xd = (xd - dv.detach().to(torch.float32)) / sv.detach().to(torch.float32)
+    Xh = Xt if abits >= 16 else quant_ste(Xt, 1.0, 1.0, abits, eps, decide, xd)
     cout, cin = W.shape
     gsz = cin if group == 0 else group
-    Wh = quant_ste(Wt.reshape(cout, cin // gsz, gsz), sigmoid(gl), sigmoid(bl), wbits, eps).reshape(cout, cin)
+    wd = _dec32(W, sv).reshape(cout, cin // gsz, gsz)
+    Wh = quant_ste(Wt.reshape(cout, cin // gsz, gsz), sigmoid(gl), sigmoid(bl), wbits, eps, decide,
+                   wd).reshape(cout, cin)
     Y = _mm(Xh, Wh, mode) + Bt
     loss, _ = block_loss(Y, Yfp)
     grads = torch.autograd.grad(loss, leaves)
@@ -487,19 +566,31 @@ def _expand_kv(vec, cfg: BlockCfg):
     return vec.reshape(cfg.n_kv, 1, cfg.head_dim).expand(cfg.n_kv, rep, cfg.head_dim).reshape(-1)
 
 
-def _qw(Wt, gl, bl, cfg: BlockCfg):
+def _decide(cfg: BlockCfg) -> str:
+    return "fp32" if cfg.mode == "emulate" else "fp64"
+
+
+def _qw(Wt, gl, bl, cfg: BlockCfg, w_dec=None):
+    """LWC fake quantization of a (LET-scaled) weight; w_dec is its fp32 quantizer input."""
     if cfg.wbits >= 16:
         return Wt
     cout, cin = Wt.shape
     gsz = cin if cfg.group == 0 else cfg.group
+    dec = None if w_dec is None else w_dec.reshape(cout, cin // gsz, gsz)
     return quant_ste(Wt.reshape(cout, cin // gsz, gsz), sigmoid(gl), sigmoid(bl),
-                     cfg.wbits, cfg.h_eps).reshape(cout, cin)
+                     cfg.wbits, cfg.h_eps, _decide(cfg), dec).reshape(cout, cin)
 
 
 def _qa(X, cfg: BlockCfg):
     if cfg.abits >= 16:
         return X
-    return quant_ste(X, 1.0, 1.0, cfg.abits, cfg.h_eps)
+    return quant_ste(X, 1.0, 1.0, cfg.abits, cfg.h_eps, _decide(cfg))
+
+
+def _dec32(W, s=None, r=None):
+    """fp32 quantizer input of a scaled weight, formed as the kernels form it (R15)."""
+    with torch.no_grad():
+        return _wt_fp32(W, None if s is None else s.detach(), None if r is None else r.detach())
 
 
 def block_forward(x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], cfg: BlockCfg,
@@ -529,9 +620,15 @@ def block_forward(x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], c
         at, wq_t, wk_t, wv_t = a, wq, wk, wv
         bq = bk = bv = None
     ah = _qa(at, cfg)
-    q = _mm(ah, _qw(wq_t, th.get("gamma_q"), th.get("beta_q"), cfg), mode)
-    k = _mm(ah, _qw(wk_t, th.get("gamma_k"), th.get("beta_k"), cfg), mode)
-    v = _mm(ah, _qw(wv_t, th.get("gamma_v"), th.get("beta_v"), cfg), mode)
+    if let:
+        with torch.no_grad():
+            r_o = (1.0 / so.detach().to(torch.float32)).to(F64)
+        dq_, dk_, dv_ = _dec32(wq, s1), _dec32(wk, s1), _dec32(wv, s1, r_o)
+    else:
+        dq_ = dk_ = dv_ = None
+    q = _mm(ah, _qw(wq_t, th.get("gamma_q"), th.get("beta_q"), cfg, dq_), mode)
+    k = _mm(ah, _qw(wk_t, th.get("gamma_k"), th.get("beta_k"), cfg, dk_), mode)
+    v = _mm(ah, _qw(wv_t, th.get("gamma_v"), th.get("beta_v"), cfg, dv_), mode)
     if let:
         q, k, v = q + bq, k + bk, v + bv
     q = rope(q, H, hd, cfg.rope_theta)
@@ -556,7 +653,8 @@ def block_forward(x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], c
         bo = wo @ _expand_kv(do_, cfg)
     else:
         wo_t, bo = wo, None
-    o = _mm(oh, _qw(wo_t, th.get("gamma_o"), th.get("beta_o"), cfg), mode)
+    o = _mm(oh, _qw(wo_t, th.get("gamma_o"), th.get("beta_o"), cfg,
+                    _dec32(wo, _expand_kv(so, cfg)) if let else None), mode)
     if bo is not None:
         o = o + bo
     h1 = x + o
@@ -571,8 +669,8 @@ def block_forward(x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], c
     else:
         bt, wg_t, wu_t, bg, bu = b_, wg, wu, None, None
     bh = _qa(bt, cfg)
-    gt = _mm(bh, _qw(wg_t, th.get("gamma_g"), th.get("beta_g"), cfg), mode)
-    up = _mm(bh, _qw(wu_t, th.get("gamma_u"), th.get("beta_u"), cfg), mode)
+    gt = _mm(bh, _qw(wg_t, th.get("gamma_g"), th.get("beta_g"), cfg, _dec32(wg, s2) if let else None), mode)
+    up = _mm(bh, _qw(wu_t, th.get("gamma_u"), th.get("beta_u"), cfg, _dec32(wu, s2) if let else None), mode)
     if let:
         gt, up = gt + bg, up + bu
     m = silu(gt) * up

@@ -1,0 +1,112 @@
+"""Device-resident state of one decoder block for libomq's block entry points.
+
+PyTorch only allocates: this module stacks the frozen weights and the learnable parameters in
+the layout include/omq.h documents (q|k|v rows in one matrix, gate|up rows in another), holds
+the gradient buffers and the workspace, and passes pointers to omq_block_step /
+omq_block_forward.  All arithmetic of the step runs in libomq's kernels.
+"""
+from __future__ import annotations
+
+from typing import Dict, Optional
+
+import numpy as np
+
+from . import _lib
+
+LWC_PARTS = {"qkv": ("q", "k", "v"), "o": ("o",), "gu": ("g", "u"), "d": ("d",)}
+LET_NAMES = {"s1": "s1", "d1": "d1", "so": "so", "do": "do_", "sa": "sa", "s2": "s2", "d2": "d2"}
+
+
+class BlockState:
+    """Weights, parameters, gradients and workspace of one block on the current CUDA device."""
+
+    def __init__(self, shape, weights: Dict[str, np.ndarray], theta: Dict[str, np.ndarray], device: str = "cuda",
+                 wbits: Optional[int] = None, abits: Optional[int] = None, group: Optional[int] = None,
+                 let: Optional[int] = None):
+        import torch
+        self.torch = torch
+        self.shape = shape
+        self.device = device
+        self.wbits = shape.wbits if wbits is None else wbits
+        self.abits = shape.abits if abits is None else abits
+        self.group = shape.group if group is None else group
+        self.let = shape.let if let is None else let
+        bf = torch.bfloat16
+
+        def dev_bf16(a):
+            return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(device=device).to(bf).contiguous()
+
+        def dev_f32(a):
+            return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(device=device).contiguous()
+
+        self.W = dict(
+            qkv=dev_bf16(np.concatenate([weights["wq"], weights["wk"], weights["wv"]], 0)),
+            o=dev_bf16(weights["wo"]),
+            gu=dev_bf16(np.concatenate([weights["wg"], weights["wu"]], 0)),
+            d=dev_bf16(weights["wd"]))
+        self.theta = {}
+        self.grads = {}
+        if self.wbits < 16:
+            for key, parts in LWC_PARTS.items():
+                for gb in ("gamma", "beta"):
+                    v = np.concatenate([theta[f"{gb}_{p}"] for p in parts], 0)
+                    self.theta[f"{gb}_{key}"] = dev_f32(v)
+                    self.grads[f"{gb}_{key}"] = torch.zeros_like(self.theta[f"{gb}_{key}"])
+        if self.let:
+            for k in LET_NAMES:
+                self.theta[k] = dev_f32(theta[k])
+                self.grads[k] = torch.zeros_like(self.theta[k])
+        self.c_shape = _lib.omq_block_shape(shape.T, shape.d, shape.n_heads, shape.n_kv, shape.head_dim, shape.ffn,
+                                            shape.rms_eps, shape.rope_theta)
+        self.c_w = _lib.omq_block_weights(*[self.W[k].data_ptr() for k in ("qkv", "o", "gu", "d")])
+        self.c_theta = self._params(self.theta)
+        self.c_grads = self._params(self.grads)
+        self.status = torch.zeros(1, dtype=torch.int32, device=device)
+        self.cfg = _lib.make_cfg(self.wbits, self.abits, self.group, self.let, 1e-5, 0, self.status)
+        ws = _lib.omq_block_workspace_size(self.c_shape, self.cfg)
+        if ws == 0:
+            raise ValueError("block shape or configuration rejected by libomq")
+        self.workspace = torch.empty(ws, dtype=torch.uint8, device=device)
+        self.loss = torch.zeros(1, dtype=torch.float32, device=device)
+
+    @staticmethod
+    def _params(d) -> "_lib.omq_block_params":
+        p = _lib.omq_block_params()
+        for k, v in d.items():
+            setattr(p, LET_NAMES.get(k, k), v.data_ptr())
+        return p
+
+    def step(self, x, y_fp, y=None, stream=None):
+        """One calibration step: forward, loss (device scalar self.loss) and gradients (self.grads)."""
+        _lib.omq_block_step(self.c_shape, self.c_w, self.c_theta, x, y_fp, y, self.loss, self.c_grads,
+                            self.workspace, self.cfg, stream)
+        return self.loss
+
+    def forward(self, x, y, stream=None, cfg=None):
+        _lib.omq_block_forward(self.c_shape, self.c_w, self.c_theta, x, y, self.workspace, cfg or self.cfg, stream)
+        return y
+
+    def fp_forward(self, x, y, stream=None):
+        """Full-precision block (quantization and LET off): the target of Eq. 1."""
+        cfg = _lib.make_cfg(16, 16, 0, 0, 1e-5, 0, self.status)
+        return self.forward(x, y, stream, cfg)
+
+    def split_grads(self) -> Dict[str, np.ndarray]:
+        """Gradients on the host, named like the oracle's parameters."""
+        out = {}
+        sh = self.shape
+        sizes = dict(qkv=[sh.dq, sh.dkv, sh.dkv], o=[sh.d], gu=[sh.ffn, sh.ffn], d=[sh.d])
+        for key, parts in LWC_PARTS.items():
+            for gb in ("gamma", "beta"):
+                name = f"{gb}_{key}"
+                if name not in self.grads:
+                    continue
+                g = self.grads[name].float().cpu().numpy()
+                off = 0
+                for p, n in zip(parts, sizes[key]):
+                    out[f"d{gb}_{p}"] = g[off:off + n]
+                    off += n
+        for k in LET_NAMES:
+            if k in self.grads:
+                out["d" + k] = self.grads[k].float().cpu().numpy()
+        return out

@@ -1,0 +1,611 @@
+// One quantized decoder-block calibration step (Algorithm 1, inner loop) and the single quantized
+// linear of Eq. 4, enqueued kernel by kernel on one stream.  All scratch lives in the caller's
+// workspace, carved by the same routine that reports its size.
+#include "attn.cuh"
+#include "gemm.cuh"
+#include "quant.cuh"
+
+namespace {
+
+struct Carve {
+  uint8_t* base;
+  size_t off;
+  template <class T>
+  T* take(size_t n) {
+    off = (off + 255) & ~size_t(255);
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off += n * sizeof(T);
+    return p;
+  }
+};
+
+typedef __nv_bfloat16 bf16;
+
+struct QState4 { float* h; int32_t* z; int32_t* imax; int32_t* imin; };
+
+QState4 take_qstate(Carve& c, size_t n) {
+  QState4 q;
+  q.h = c.take<float>(n); q.z = c.take<int32_t>(n); q.imax = c.take<int32_t>(n); q.imin = c.take<int32_t>(n);
+  return q;
+}
+
+struct BlockWS {
+  // fake-quantized weights and their per-group state
+  bf16 *Wqkv_h, *Wo_h, *Wgu_h, *Wd_h;
+  QState4 sq_qkv, sq_o, sq_gu, sq_d;
+  float *B_qkv, *B_o, *B_gu;
+  float *r_qkv, *shift_qkv, *so_exp, *do_exp, *sa_exp;
+  float* cs;
+  // forward activations
+  bf16* a_h; float* rstd1; QState4 sa;
+  float* Yqkv; bf16 *Qh, *Kh, *Vh; QState4 sqkv;
+  float* S; bf16* P;
+  float* O; bf16* O_h; QState4 so;
+  float* h1; bf16* b_h; float* rstd2; QState4 sb;
+  float* Ygu; bf16* m_h; QState4 sm;
+  float* y;
+  // backward
+  float* loss_part;
+  float* dy; bf16* dy_b;
+  float* dm;
+  float* dW;
+  float* dYgu; bf16* dYgu_b;
+  float* db;
+  float* dh1; bf16* dh1_b;
+  float* dOh; bf16* dO_b;
+  bf16* dS;
+  float* dQKV; float* dYqkv; bf16* dYqkv_b;
+  float* da;
+  float *dB_qkv, *dB_o, *dB_gu, *dr_qkv;
+  float *vtmp0, *vtmp1, *vtmp2;     // [max(d, dq)] scratch vectors
+  float* part;                      // shared partial-sum scratch
+  size_t part_elems;
+};
+
+int64_t imax64(int64_t a, int64_t b) { return a > b ? a : b; }
+
+void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockWS& w, bool with_bwd) {
+  const int64_t T = s.T, d = s.d, hd = s.head_dim, H = s.n_heads, Hkv = s.n_kv, f = s.ffn;
+  const int64_t dq = H * hd, dkv = Hkv * hd, nqkv = dq + 2 * dkv;
+  auto ng = [&](int64_t cin) { return cfg.group == 0 ? (int64_t)1 : cin / cfg.group; };
+  w.Wqkv_h = c.take<bf16>(nqkv * d);
+  w.Wo_h = c.take<bf16>(d * dq);
+  w.Wgu_h = c.take<bf16>(2 * f * d);
+  w.Wd_h = c.take<bf16>(d * f);
+  w.sq_qkv = take_qstate(c, nqkv * ng(d));
+  w.sq_o = take_qstate(c, d * ng(dq));
+  w.sq_gu = take_qstate(c, 2 * f * ng(d));
+  w.sq_d = take_qstate(c, d * ng(f));
+  w.B_qkv = c.take<float>(nqkv);
+  w.B_o = c.take<float>(d);
+  w.B_gu = c.take<float>(2 * f);
+  w.r_qkv = c.take<float>(nqkv);
+  w.shift_qkv = c.take<float>(nqkv);
+  w.so_exp = c.take<float>(dq);
+  w.do_exp = c.take<float>(dq);
+  w.sa_exp = c.take<float>(dq);
+  w.cs = c.take<float>(T * hd);
+  w.a_h = c.take<bf16>(T * d);
+  w.rstd1 = c.take<float>(T);
+  w.sa = take_qstate(c, T);
+  w.Yqkv = c.take<float>(T * nqkv);
+  w.Qh = c.take<bf16>(T * dq);
+  w.Kh = c.take<bf16>(T * dkv);
+  w.Vh = c.take<bf16>(T * dkv);
+  w.sqkv = take_qstate(c, 3 * T);
+  w.S = c.take<float>(H * T * T);
+  w.P = c.take<bf16>(H * T * T);
+  w.O = c.take<float>(T * dq);
+  w.O_h = c.take<bf16>(T * dq);
+  w.so = take_qstate(c, T);
+  w.h1 = c.take<float>(T * d);
+  w.b_h = c.take<bf16>(T * d);
+  w.rstd2 = c.take<float>(T);
+  w.sb = take_qstate(c, T);
+  w.Ygu = c.take<float>(T * 2 * f);
+  w.m_h = c.take<bf16>(T * f);
+  w.sm = take_qstate(c, T);
+  w.y = c.take<float>(T * d);
+  w.loss_part = c.take<float>(loss_parts(T * d) + 64);
+  if (!with_bwd) return;
+  w.dy = c.take<float>(T * d);
+  w.dy_b = c.take<bf16>(T * d);
+  w.dm = c.take<float>(T * f);
+  w.dW = c.take<float>(imax64(imax64(nqkv * d, d * dq), imax64(2 * f * d, d * f)));
+  w.dYgu = c.take<float>(T * 2 * f);
+  w.dYgu_b = c.take<bf16>(T * 2 * f);
+  w.db = c.take<float>(T * d);
+  w.dh1 = c.take<float>(T * d);
+  w.dh1_b = c.take<bf16>(T * d);
+  w.dOh = c.take<float>(T * dq);
+  w.dO_b = c.take<bf16>(T * dq);
+  w.dS = c.take<bf16>(H * T * T);
+  w.dQKV = c.take<float>(T * nqkv);
+  w.dYqkv = c.take<float>(T * nqkv);
+  w.dYqkv_b = c.take<bf16>(T * nqkv);
+  w.da = c.take<float>(T * d);
+  w.dB_qkv = c.take<float>(nqkv);
+  w.dB_o = c.take<float>(d);
+  w.dB_gu = c.take<float>(2 * f);
+  w.dr_qkv = c.take<float>(nqkv);
+  const int64_t vmax = imax64(d, dq);
+  w.vtmp0 = c.take<float>(vmax);
+  w.vtmp1 = c.take<float>(vmax);
+  w.vtmp2 = c.take<float>(vmax);
+  int64_t pe = 0;
+  pe = imax64(pe, 2 * lwc_bwd_nslab(nqkv) * d);
+  pe = imax64(pe, 2 * lwc_bwd_nslab(d) * dq);
+  pe = imax64(pe, 2 * lwc_bwd_nslab(2 * f) * d);
+  pe = imax64(pe, 2 * ((T + 3) / 4) * imax64(d, dq));
+  pe = imax64(pe, qkv_bwd_nslab((int)T) * (dq + dkv));
+  pe = imax64(pe, colsum_rows_parts(T) * imax64(2 * f, nqkv));
+  w.part_elems = (size_t)pe;
+  w.part = c.take<float>(pe);
+}
+
+omq_status check_block(const omq_block_shape* s, const omq_qcfg* cfg) {
+  OMQ_REQUIRE(s, OMQ_ERR_INVALID_ARG);
+  OMQ_TRY(omq_check_cfg(cfg));
+  OMQ_REQUIRE(s->T > 0 && s->d > 0 && s->n_heads > 0 && s->n_kv > 0 && s->ffn > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(s->head_dim == 128, OMQ_ERR_UNSUPPORTED);
+  OMQ_REQUIRE(s->n_heads % s->n_kv == 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(s->T % 8 == 0 && s->d % 8 == 0 && s->ffn % 8 == 0, OMQ_ERR_ALIGN);
+  if (cfg->group > 0) {
+    OMQ_REQUIRE(s->d % cfg->group == 0 && s->ffn % cfg->group == 0 && ((int64_t)s->n_heads * 128) % cfg->group == 0,
+                OMQ_ERR_SHAPE);
+  }
+  return OMQ_OK;
+}
+
+// C = alpha * A B^T with A [M, K] and B [N, K] both stored K-major
+omq_status gemm_kk(cudaStream_t st, int64_t M, int64_t N, int64_t K, const bf16* A, int64_t lda, const bf16* B,
+                   int64_t ldb, float* Cf, bf16* Cb, int64_t ldc, const float* bias, const float* R, int32_t* status) {
+  GemmOperand a{A, lda, 0, 1}, b{B, ldb, 0, 1};
+  GemmEpilogue ep{Cf, Cb, ldc, 0, 1.f, bias, R, ldc, 0.f};
+  return gemm_launch(st, M, N, K, 1, a, b, ep, 0, status);
+}
+
+// dX = dY W  with dY [T, Cout] and W [Cout, Cin]: B[n = i, k = o] = W[o, i] is MN-major
+omq_status gemm_dx(cudaStream_t st, int64_t T, int64_t Cout, int64_t Cin, const bf16* dY, const bf16* W, float* dX,
+                   int32_t* status) {
+  GemmOperand a{dY, Cout, 0, 1}, b{W, Cin, 0, 0};
+  GemmEpilogue ep{dX, nullptr, Cin, 0, 1.f, nullptr, nullptr, 0, 0.f};
+  return gemm_launch(st, T, Cin, Cout, 1, a, b, ep, 0, status);
+}
+
+// dW = dY^T X with dY [T, Cout], X [T, Cin]: both operands MN-major, K = T
+omq_status gemm_dw(cudaStream_t st, int64_t T, int64_t Cout, int64_t Cin, const bf16* dY, const bf16* X, float* dW,
+                   int32_t* status) {
+  GemmOperand a{dY, Cout, 0, 0}, b{X, Cin, 0, 0};
+  GemmEpilogue ep{dW, nullptr, Cin, 0, 1.f, nullptr, nullptr, 0, 0.f};
+  return gemm_launch(st, Cout, Cin, T, 1, a, b, ep, 0, status);
+}
+
+LwcFwdArgs lwc_args(const bf16* W, int64_t Cout, int64_t Cin, const omq_qcfg& cfg, const float* s, const float* r,
+                    const float* gl, const float* bl, bf16* Wq, const QState4& q, const float* bias_delta,
+                    const float* bias_shift, float* Bt) {
+  LwcFwdArgs a{};
+  a.W = W; a.Cout = Cout; a.Cin = Cin; a.group = cfg.group == 0 ? (int)Cin : cfg.group;
+  a.s = s; a.r = r; a.gl = gl; a.bl = bl; a.lwc = 1; a.Wq = Wq; a.codes = nullptr;
+  a.h = q.h; a.z = q.z; a.imax = q.imax; a.imin = q.imin;
+  a.bias_delta = bias_delta; a.bias_shift = bias_shift; a.Bt = Bt;
+  a.wbits = cfg.wbits; a.eps = cfg.h_eps; a.status = cfg.dev_status;
+  return a;
+}
+
+omq_status lwc_bwd_full(cudaStream_t st, const bf16* W, int64_t Cout, int64_t Cin, const omq_qcfg& cfg,
+                        const float* s, const float* r, const float* gl, const float* bl, const QState4& q,
+                        const float* dW, float* dgl, float* dbl, float* dr, const float* dBt, float* ds,
+                        float* ddelta, int accumulate_sd, float* part) {
+  LwcBwdArgs a{};
+  a.W = W; a.Cout = Cout; a.Cin = Cin; a.group = cfg.group == 0 ? (int)Cin : cfg.group;
+  a.s = s; a.r = r; a.gl = gl; a.bl = bl; a.lwc = 1;
+  a.h = q.h; a.z = q.z; a.imax = q.imax; a.imin = q.imin;
+  a.dWq = dW; a.ld_dwq = Cin; a.dgl = dgl; a.dbl = dbl; a.dWt = nullptr; a.dr = dr; a.dBt = dBt;
+  const int64_t ns = lwc_bwd_nslab(Cout);
+  a.part_s = ds ? part : nullptr;
+  a.part_d = ddelta ? part + ns * Cin : nullptr;
+  a.wbits = cfg.wbits; a.eps = cfg.h_eps; a.accumulate = cfg.accumulate; a.accumulate_dr = 0;
+  int64_t n = 0;
+  OMQ_TRY(lwc_bwd_launch(st, a, &n));
+  if (ds) OMQ_TRY(omq_colsum_partials(st, a.part_s, n, Cin, ds, 1.f, accumulate_sd));
+  if (ddelta) OMQ_TRY(omq_colsum_partials(st, a.part_d, n, Cin, ddelta, 1.f, accumulate_sd));
+  return OMQ_OK;
+}
+
+struct Ctx {
+  cudaStream_t st;
+  omq_block_shape s;
+  omq_qcfg cfg;
+  const omq_block_weights* w;
+  const omq_block_params* th;
+  BlockWS ws;
+  int64_t T, d, hd, H, Hkv, rep, f, dq, dkv, nqkv;
+  bool let, wq, aq;
+};
+
+omq_status block_fwd(Ctx& c, const float* x, float* y) {
+  cudaStream_t st = c.st;
+  BlockWS& w = c.ws;
+  const omq_qcfg& cfg = c.cfg;
+  const omq_block_params* th = c.th;
+  int32_t* status = cfg.dev_status;
+  const bf16* Wqkv = (const bf16*)c.w->wqkv;
+  const bf16* Wo = (const bf16*)c.w->wo;
+  const bf16* Wgu = (const bf16*)c.w->wgu;
+  const bf16* Wd = (const bf16*)c.w->wd;
+
+  OMQ_TRY(rope_table(st, (int)c.T, (int)c.hd, c.s.rope_theta, w.cs));
+  if (c.let) {
+    OMQ_TRY(qkv_row_vectors(st, (int)c.dq, (int)c.dkv, th->so, th->do_, w.r_qkv, w.shift_qkv));
+    OMQ_TRY(gqa_expand(st, th->so, w.so_exp, (int)c.Hkv, (int)c.rep, (int)c.hd, 0));
+    OMQ_TRY(gqa_expand(st, th->do_, w.do_exp, (int)c.Hkv, (int)c.rep, (int)c.hd, 0));
+    OMQ_TRY(gqa_expand(st, th->sa, w.sa_exp, (int)c.Hkv, (int)c.rep, (int)c.hd, 0));
+  }
+  // ---- LET (Eq. 3) + LWC (Eq. 2) on every weight ------------------------------------------------
+  OMQ_TRY(lwc_fwd_launch(st, lwc_args(Wqkv, c.nqkv, c.d, cfg, c.let ? th->s1 : nullptr, c.let ? w.r_qkv : nullptr,
+                                      th->gamma_qkv, th->beta_qkv, w.Wqkv_h, w.sq_qkv, c.let ? th->d1 : nullptr,
+                                      c.let ? w.shift_qkv : nullptr, c.let ? w.B_qkv : nullptr)));
+  OMQ_TRY(lwc_fwd_launch(st, lwc_args(Wo, c.d, c.dq, cfg, c.let ? w.so_exp : nullptr, nullptr, th->gamma_o, th->beta_o,
+                                      w.Wo_h, w.sq_o, c.let ? w.do_exp : nullptr, nullptr, c.let ? w.B_o : nullptr)));
+  OMQ_TRY(lwc_fwd_launch(st, lwc_args(Wgu, 2 * c.f, c.d, cfg, c.let ? th->s2 : nullptr, nullptr, th->gamma_gu,
+                                      th->beta_gu, w.Wgu_h, w.sq_gu, c.let ? th->d2 : nullptr, nullptr,
+                                      c.let ? w.B_gu : nullptr)));
+  OMQ_TRY(lwc_fwd_launch(st, lwc_args(Wd, c.d, c.f, cfg, nullptr, nullptr, th->gamma_d, th->beta_d, w.Wd_h, w.sq_d,
+                                      nullptr, nullptr, nullptr)));
+
+  // ---- attention half ---------------------------------------------------------------------------
+  ActFwdArgs af{};
+  af.producer = AP_RMS_LET; af.X = x; af.ldx = c.d; af.s = c.let ? th->s1 : nullptr; af.delta = c.let ? th->d1 : nullptr;
+  af.rms_eps = c.s.rms_eps; af.rstd = w.rstd1; af.T = c.T; af.C = c.d; af.Xq = w.a_h; af.ldq = c.d;
+  af.h = w.sa.h; af.z = w.sa.z; af.imax = w.sa.imax; af.imin = w.sa.imin; af.abits = cfg.abits; af.eps = cfg.h_eps;
+  OMQ_TRY(act_fwd_launch(st, af));
+  OMQ_TRY(gemm_kk(st, c.T, c.nqkv, c.d, w.a_h, c.d, w.Wqkv_h, c.d, w.Yqkv, nullptr, c.nqkv, c.let ? w.B_qkv : nullptr,
+                  nullptr, status));
+  QkvArgs qa{};
+  qa.T = (int)c.T; qa.H = (int)c.H; qa.Hkv = (int)c.Hkv; qa.hd = (int)c.hd; qa.Y = w.Yqkv; qa.ldy = c.nqkv; qa.cs = w.cs;
+  qa.sa_exp = c.let ? w.sa_exp : nullptr; qa.sa = c.let ? th->sa : nullptr;
+  qa.Qh = w.Qh; qa.Kh = w.Kh; qa.Vh = w.Vh;
+  qa.h = w.sqkv.h; qa.z = w.sqkv.z; qa.imax = w.sqkv.imax; qa.imin = w.sqkv.imin; qa.abits = cfg.abits; qa.eps = cfg.h_eps;
+  OMQ_TRY(qkv_fwd_launch(st, qa));
+  const float scale = 1.0f / sqrtf((float)c.hd);
+  const int64_t TT = c.T * c.T;
+  for (int64_t r = 0; r < c.rep; ++r) {     // query heads kv*rep + r share KV head kv
+    GemmOperand a{w.Qh + r * c.hd, c.dq, c.rep * c.hd, 1}, b{w.Kh, c.dkv, c.hd, 1};
+    GemmEpilogue ep{w.S + r * TT, nullptr, c.T, c.rep * TT, scale, nullptr, nullptr, 0, 0.f};
+    OMQ_TRY(gemm_launch(st, c.T, c.T, c.hd, c.Hkv, a, b, ep, 1, status));
+  }
+  OMQ_TRY(softmax_fwd_launch(st, (int)c.H, (int)c.T, w.S, w.P));
+  for (int64_t r = 0; r < c.rep; ++r) {
+    GemmOperand a{w.P + r * TT, c.T, c.rep * TT, 1}, b{w.Vh, c.dkv, c.hd, 0};
+    GemmEpilogue ep{w.O + r * c.hd, nullptr, c.dq, c.rep * c.hd, 1.f, nullptr, nullptr, 0, 0.f};
+    OMQ_TRY(gemm_launch(st, c.T, c.hd, c.T, c.Hkv, a, b, ep, 2, status));
+  }
+  ActFwdArgs ao{};
+  ao.producer = AP_PLAIN; ao.X = w.O; ao.ldx = c.dq; ao.T = c.T; ao.C = c.dq; ao.Xq = w.O_h; ao.ldq = c.dq;
+  ao.h = w.so.h; ao.z = w.so.z; ao.imax = w.so.imax; ao.imin = w.so.imin; ao.abits = cfg.abits; ao.eps = cfg.h_eps;
+  OMQ_TRY(act_fwd_launch(st, ao));
+  OMQ_TRY(gemm_kk(st, c.T, c.d, c.dq, w.O_h, c.dq, w.Wo_h, c.dq, w.h1, nullptr, c.d, c.let ? w.B_o : nullptr, x, status));
+
+  // ---- FFN half ---------------------------------------------------------------------------------
+  ActFwdArgs ab = af;
+  ab.X = w.h1; ab.s = c.let ? th->s2 : nullptr; ab.delta = c.let ? th->d2 : nullptr; ab.rstd = w.rstd2; ab.Xq = w.b_h;
+  ab.h = w.sb.h; ab.z = w.sb.z; ab.imax = w.sb.imax; ab.imin = w.sb.imin;
+  OMQ_TRY(act_fwd_launch(st, ab));
+  OMQ_TRY(gemm_kk(st, c.T, 2 * c.f, c.d, w.b_h, c.d, w.Wgu_h, c.d, w.Ygu, nullptr, 2 * c.f, c.let ? w.B_gu : nullptr,
+                  nullptr, status));
+  ActFwdArgs am{};
+  am.producer = AP_SWIGLU; am.X = w.Ygu; am.ldx = 2 * c.f; am.U = w.Ygu + c.f; am.ldu = 2 * c.f; am.T = c.T; am.C = c.f;
+  am.Xq = w.m_h; am.ldq = c.f; am.h = w.sm.h; am.z = w.sm.z; am.imax = w.sm.imax; am.imin = w.sm.imin;
+  am.abits = cfg.abits; am.eps = cfg.h_eps;
+  OMQ_TRY(act_fwd_launch(st, am));
+  OMQ_TRY(gemm_kk(st, c.T, c.d, c.f, w.m_h, c.f, w.Wd_h, c.f, y, nullptr, c.d, nullptr, w.h1, status));
+  return OMQ_OK;
+}
+
+omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, float* loss, const omq_block_params* g) {
+  cudaStream_t st = c.st;
+  BlockWS& w = c.ws;
+  const omq_qcfg& cfg = c.cfg;
+  const omq_block_params* th = c.th;
+  int32_t* status = cfg.dev_status;
+  const bf16* Wqkv = (const bf16*)c.w->wqkv;
+  const bf16* Wo = (const bf16*)c.w->wo;
+  const bf16* Wgu = (const bf16*)c.w->wgu;
+  const bf16* Wd = (const bf16*)c.w->wd;
+  const int acc = cfg.accumulate;
+
+  // ---- loss (Eq. 1) ------------------------------------------------------------------------------
+  OMQ_TRY(loss_launch(st, c.T * c.d, y, y_fp, loss, w.dy, w.dy_b, w.loss_part));
+
+  // ---- down_proj ----------------------------------------------------------------------------------
+  OMQ_TRY(gemm_dx(st, c.T, c.d, c.f, w.dy_b, w.Wd_h, w.dm, status));
+  OMQ_TRY(gemm_dw(st, c.T, c.d, c.f, w.dy_b, w.m_h, w.dW, status));
+  OMQ_TRY(lwc_bwd_full(st, Wd, c.d, c.f, cfg, nullptr, nullptr, th->gamma_d, th->beta_d, w.sq_d, w.dW, g->gamma_d,
+                       g->beta_d, nullptr, nullptr, nullptr, nullptr, 0, w.part));
+  ActBwdArgs bm{};
+  bm.producer = AP_SWIGLU; bm.X = w.Ygu; bm.ldx = 2 * c.f; bm.U = w.Ygu + c.f; bm.ldu = 2 * c.f; bm.T = c.T; bm.C = c.f;
+  bm.h = w.sm.h; bm.z = w.sm.z; bm.imax = w.sm.imax; bm.imin = w.sm.imin; bm.dXq = w.dm; bm.lddq = c.f;
+  bm.dX = w.dYgu; bm.lddx = 2 * c.f; bm.dXb = w.dYgu_b; bm.lddxb = 2 * c.f; bm.dU = w.dYgu + c.f; bm.dUb = w.dYgu_b + c.f;
+  bm.rows_per_cta = 4; bm.abits = cfg.abits; bm.eps = cfg.h_eps;
+  OMQ_TRY(act_bwd_launch(st, bm));
+
+  // ---- gate / up ----------------------------------------------------------------------------------
+  OMQ_TRY(gemm_dx(st, c.T, 2 * c.f, c.d, w.dYgu_b, w.Wgu_h, w.db, status));
+  OMQ_TRY(gemm_dw(st, c.T, 2 * c.f, c.d, w.dYgu_b, w.b_h, w.dW, status));
+  if (c.let) OMQ_TRY(colsum_rows(st, w.dYgu, c.T, 2 * c.f, 2 * c.f, w.part, w.dB_gu, 1.f, 0));
+  OMQ_TRY(lwc_bwd_full(st, Wgu, 2 * c.f, c.d, cfg, c.let ? th->s2 : nullptr, nullptr, th->gamma_gu, th->beta_gu,
+                       w.sq_gu, w.dW, g->gamma_gu, g->beta_gu, nullptr, c.let ? w.dB_gu : nullptr,
+                       c.let ? g->s2 : nullptr, c.let ? g->d2 : nullptr, acc, w.part));
+  ActBwdArgs bb{};
+  bb.producer = AP_RMS_LET; bb.X = w.h1; bb.ldx = c.d; bb.s = c.let ? th->s2 : nullptr; bb.delta = c.let ? th->d2 : nullptr;
+  bb.rstd = w.rstd2; bb.T = c.T; bb.C = c.d; bb.h = w.sb.h; bb.z = w.sb.z; bb.imax = w.sb.imax; bb.imin = w.sb.imin;
+  bb.dXq = w.db; bb.lddq = c.d; bb.dX = w.dh1; bb.lddx = c.d; bb.dXb = w.dh1_b; bb.lddxb = c.d; bb.resid = w.dy;
+  bb.part_s = c.let ? w.part : nullptr; bb.part_d = c.let ? w.part + ((c.T + 3) / 4) * c.d : nullptr;
+  bb.rows_per_cta = 4; bb.abits = cfg.abits; bb.eps = cfg.h_eps;
+  OMQ_TRY(act_bwd_launch(st, bb));
+  if (c.let) {
+    OMQ_TRY(omq_colsum_partials(st, bb.part_s, (c.T + 3) / 4, c.d, g->s2, 1.f, 1));
+    OMQ_TRY(omq_colsum_partials(st, bb.part_d, (c.T + 3) / 4, c.d, g->d2, 1.f, 1));
+  }
+
+  // ---- o_proj -------------------------------------------------------------------------------------
+  OMQ_TRY(gemm_dx(st, c.T, c.d, c.dq, w.dh1_b, w.Wo_h, w.dOh, status));
+  OMQ_TRY(gemm_dw(st, c.T, c.d, c.dq, w.dh1_b, w.O_h, w.dW, status));
+  if (c.let) OMQ_TRY(colsum_rows(st, w.dh1, c.T, c.d, c.d, w.part, w.dB_o, 1.f, 0));
+  OMQ_TRY(lwc_bwd_full(st, Wo, c.d, c.dq, cfg, c.let ? w.so_exp : nullptr, nullptr, th->gamma_o, th->beta_o, w.sq_o,
+                       w.dW, g->gamma_o, g->beta_o, nullptr, c.let ? w.dB_o : nullptr, c.let ? w.vtmp0 : nullptr,
+                       c.let ? w.vtmp1 : nullptr, 0, w.part));
+  ActBwdArgs bo{};
+  bo.producer = AP_PLAIN; bo.X = w.O; bo.ldx = c.dq; bo.T = c.T; bo.C = c.dq; bo.h = w.so.h; bo.z = w.so.z;
+  bo.imax = w.so.imax; bo.imin = w.so.imin; bo.dXq = w.dOh; bo.lddq = c.dq; bo.dX = nullptr; bo.lddx = c.dq;
+  bo.dXb = w.dO_b; bo.lddxb = c.dq; bo.rows_per_cta = 4; bo.abits = cfg.abits; bo.eps = cfg.h_eps;
+  OMQ_TRY(act_bwd_launch(st, bo));
+
+  // ---- attention (materialised causal scores) --------------------------------------------------------
+  const float scale = 1.0f / sqrtf((float)c.hd);
+  const int64_t TT = c.T * c.T;
+  float* dP = w.S;      // the scores are dead after the forward softmax
+  for (int64_t r = 0; r < c.rep; ++r) {
+    GemmOperand a{w.dO_b + r * c.hd, c.dq, c.rep * c.hd, 1}, b{w.Vh, c.dkv, c.hd, 1};
+    GemmEpilogue ep{dP + r * TT, nullptr, c.T, c.rep * TT, 1.f, nullptr, nullptr, 0, 0.f};
+    OMQ_TRY(gemm_launch(st, c.T, c.T, c.hd, c.Hkv, a, b, ep, 1, status));
+  }
+  OMQ_TRY(softmax_bwd_launch(st, (int)c.H, (int)c.T, w.P, dP, scale, w.dS));
+  for (int64_t r = 0; r < c.rep; ++r) {
+    const float beta = r > 0 ? 1.f : 0.f;
+    {   // dV = P^T dO  (keys x dims, summed over the query heads of the group)
+      GemmOperand a{w.P + r * TT, c.T, c.rep * TT, 0}, b{w.dO_b + r * c.hd, c.dq, c.rep * c.hd, 0};
+      GemmEpilogue ep{w.dQKV + c.dq + c.dkv, nullptr, c.nqkv, c.hd, 1.f, nullptr, nullptr, 0, beta};
+      OMQ_TRY(gemm_launch(st, c.T, c.hd, c.T, c.Hkv, a, b, ep, 3, status));
+    }
+    {   // dQ = dS K
+      GemmOperand a{w.dS + r * TT, c.T, c.rep * TT, 1}, b{w.Kh, c.dkv, c.hd, 0};
+      GemmEpilogue ep{w.dQKV + r * c.hd, nullptr, c.nqkv, c.rep * c.hd, 1.f, nullptr, nullptr, 0, 0.f};
+      OMQ_TRY(gemm_launch(st, c.T, c.hd, c.T, c.Hkv, a, b, ep, 2, status));
+    }
+    {   // dK = dS^T Q
+      GemmOperand a{w.dS + r * TT, c.T, c.rep * TT, 0}, b{w.Qh + r * c.hd, c.dq, c.rep * c.hd, 0};
+      GemmEpilogue ep{w.dQKV + c.dq, nullptr, c.nqkv, c.hd, 1.f, nullptr, nullptr, 0, beta};
+      OMQ_TRY(gemm_launch(st, c.T, c.hd, c.T, c.Hkv, a, b, ep, 3, status));
+    }
+  }
+  QkvArgs qa{};
+  qa.T = (int)c.T; qa.H = (int)c.H; qa.Hkv = (int)c.Hkv; qa.hd = (int)c.hd; qa.Y = w.Yqkv; qa.ldy = c.nqkv; qa.cs = w.cs;
+  qa.sa_exp = c.let ? w.sa_exp : nullptr; qa.sa = c.let ? th->sa : nullptr;
+  qa.h = w.sqkv.h; qa.z = w.sqkv.z; qa.imax = w.sqkv.imax; qa.imin = w.sqkv.imin; qa.abits = cfg.abits; qa.eps = cfg.h_eps;
+  qa.dQKV = w.dQKV; qa.ldd = c.nqkv; qa.dY = w.dYqkv; qa.dYb = w.dYqkv_b;
+  const int64_t nsq = qkv_bwd_nslab((int)c.T);
+  qa.part_q = c.let ? w.part : nullptr;
+  qa.part_k = c.let ? w.part + nsq * c.dq : nullptr;
+  OMQ_TRY(qkv_bwd_launch(st, qa, nullptr));
+  if (c.let) {
+    OMQ_TRY(omq_colsum_partials(st, qa.part_q, nsq, c.dq, w.vtmp2, 1.f, 0));
+    OMQ_TRY(omq_colsum_partials(st, qa.part_k, nsq, c.dkv, g->sa, 1.f, acc));
+    OMQ_TRY(gqa_fold(st, w.vtmp2, g->sa, (int)c.Hkv, (int)c.rep, (int)c.hd, 1));
+    // [v, out] pair: o_proj column-scale part (folded over the query heads), then v rows
+    OMQ_TRY(gqa_fold(st, w.vtmp0, g->so, (int)c.Hkv, (int)c.rep, (int)c.hd, acc));
+    OMQ_TRY(gqa_fold(st, w.vtmp1, g->do_, (int)c.Hkv, (int)c.rep, (int)c.hd, acc));
+  }
+
+  // ---- q / k / v projections ---------------------------------------------------------------------------
+  OMQ_TRY(gemm_dw(st, c.T, c.nqkv, c.d, w.dYqkv_b, w.a_h, w.dW, status));
+  if (c.let) OMQ_TRY(colsum_rows(st, w.dYqkv, c.T, c.nqkv, c.nqkv, w.part, w.dB_qkv, 1.f, 0));
+  OMQ_TRY(lwc_bwd_full(st, Wqkv, c.nqkv, c.d, cfg, c.let ? th->s1 : nullptr, c.let ? w.r_qkv : nullptr, th->gamma_qkv,
+                       th->beta_qkv, w.sq_qkv, w.dW, g->gamma_qkv, g->beta_qkv, c.let ? w.dr_qkv : nullptr,
+                       c.let ? w.dB_qkv : nullptr, c.let ? g->s1 : nullptr, c.let ? g->d1 : nullptr, acc, w.part));
+  if (c.let) {
+    const int64_t off = c.dq + c.dkv;
+    OMQ_TRY(let_vo_finalize(st, (int)c.dkv, th->so, w.dr_qkv + off, w.dB_qkv + off, w.B_qkv + off, g->so, g->do_, 1));
+    OMQ_TRY(gemm_dx(st, c.T, c.nqkv, c.d, w.dYqkv_b, w.Wqkv_h, w.da, status));
+    ActBwdArgs ba{};
+    ba.producer = AP_RMS_LET; ba.X = x; ba.ldx = c.d; ba.s = th->s1; ba.delta = th->d1; ba.rstd = w.rstd1; ba.T = c.T;
+    ba.C = c.d; ba.h = w.sa.h; ba.z = w.sa.z; ba.imax = w.sa.imax; ba.imin = w.sa.imin; ba.dXq = w.da; ba.lddq = c.d;
+    ba.dX = nullptr; ba.dXb = nullptr; ba.part_s = w.part; ba.part_d = w.part + ((c.T + 3) / 4) * c.d;
+    ba.rows_per_cta = 4; ba.abits = cfg.abits; ba.eps = cfg.h_eps;
+    OMQ_TRY(act_bwd_launch(st, ba));
+    OMQ_TRY(omq_colsum_partials(st, ba.part_s, (c.T + 3) / 4, c.d, g->s1, 1.f, 1));
+    OMQ_TRY(omq_colsum_partials(st, ba.part_d, (c.T + 3) / 4, c.d, g->d1, 1.f, 1));
+  }
+  return OMQ_OK;
+}
+
+omq_status make_ctx(Ctx& c, omq_stream_t stream, const omq_block_shape* shape, const omq_block_weights* w,
+                    const omq_block_params* theta, void* workspace, size_t ws_bytes, const omq_qcfg* cfg, bool bwd) {
+  OMQ_TRY(check_block(shape, cfg));
+  OMQ_REQUIRE(w && w->wqkv && w->wo && w->wgu && w->wd && theta, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(omq_aligned16(w->wqkv) && omq_aligned16(w->wo) && omq_aligned16(w->wgu) && omq_aligned16(w->wd),
+              OMQ_ERR_ALIGN);
+  if (cfg->wbits < 16)
+    OMQ_REQUIRE(theta->gamma_qkv && theta->beta_qkv && theta->gamma_o && theta->beta_o && theta->gamma_gu &&
+                    theta->beta_gu && theta->gamma_d && theta->beta_d,
+                OMQ_ERR_INVALID_ARG);
+  if (cfg->let)
+    OMQ_REQUIRE(theta->s1 && theta->d1 && theta->so && theta->do_ && theta->sa && theta->s2 && theta->d2,
+                OMQ_ERR_INVALID_ARG);
+  Carve dry{nullptr, 0};
+  BlockWS tmp;
+  carve_block(dry, *shape, *cfg, tmp, bwd);
+  OMQ_REQUIRE(workspace && ws_bytes >= dry.off, OMQ_ERR_WORKSPACE);
+  OMQ_REQUIRE(omq_aligned16(workspace), OMQ_ERR_ALIGN);
+  c.st = (cudaStream_t)stream;
+  c.s = *shape;
+  c.cfg = *cfg;
+  c.w = w;
+  c.th = theta;
+  Carve real{(uint8_t*)workspace, 0};
+  carve_block(real, *shape, *cfg, c.ws, bwd);
+  c.T = shape->T; c.d = shape->d; c.hd = shape->head_dim; c.H = shape->n_heads; c.Hkv = shape->n_kv;
+  c.rep = c.H / c.Hkv; c.f = shape->ffn; c.dq = c.H * c.hd; c.dkv = c.Hkv * c.hd; c.nqkv = c.dq + 2 * c.dkv;
+  c.let = cfg->let != 0; c.wq = cfg->wbits < 16; c.aq = cfg->abits < 16;
+  return OMQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t omq_block_workspace_size(const omq_block_shape* shape, const omq_qcfg* cfg) {
+  if (check_block(shape, cfg) != OMQ_OK) return 0;
+  Carve dry{nullptr, 0};
+  BlockWS tmp;
+  carve_block(dry, *shape, *cfg, tmp, true);
+  return dry.off + 256;
+}
+
+omq_status omq_block_forward(omq_stream_t stream, const omq_block_shape* shape, const omq_block_weights* w,
+                             const omq_block_params* theta, const float* x, float* y, void* workspace, size_t ws_bytes,
+                             const omq_qcfg* cfg) {
+  Ctx c;
+  OMQ_TRY(make_ctx(c, stream, shape, w, theta, workspace, ws_bytes, cfg, false));
+  OMQ_REQUIRE(x && y && omq_aligned16(x) && omq_aligned16(y), x && y ? OMQ_ERR_ALIGN : OMQ_ERR_INVALID_ARG);
+  return block_fwd(c, x, y);
+}
+
+omq_status omq_block_step(omq_stream_t stream, const omq_block_shape* shape, const omq_block_weights* w,
+                          const omq_block_params* theta, const float* x, const float* y_fp, float* y, float* loss,
+                          const omq_block_params* grads, void* workspace, size_t ws_bytes, const omq_qcfg* cfg) {
+  Ctx c;
+  OMQ_TRY(make_ctx(c, stream, shape, w, theta, workspace, ws_bytes, cfg, true));
+  OMQ_REQUIRE(x && y_fp && loss && grads, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(cfg->wbits < 16, OMQ_ERR_UNSUPPORTED);   // the step learns the clipping of Eq. 2
+  if (cfg->wbits < 16)
+    OMQ_REQUIRE(grads->gamma_qkv && grads->beta_qkv && grads->gamma_o && grads->beta_o && grads->gamma_gu &&
+                    grads->beta_gu && grads->gamma_d && grads->beta_d,
+                OMQ_ERR_INVALID_ARG);
+  if (cfg->let)
+    OMQ_REQUIRE(grads->s1 && grads->d1 && grads->so && grads->do_ && grads->sa && grads->s2 && grads->d2,
+                OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(omq_aligned16(x) && omq_aligned16(y_fp) && (!y || omq_aligned16(y)), OMQ_ERR_ALIGN);
+  float* yy = y ? y : c.ws.y;
+  OMQ_TRY(block_fwd(c, x, yy));
+  return block_bwd(c, x, yy, y_fp, loss, grads);
+}
+
+// ---------------------------------------------------------------------------------------------------
+// single quantized linear
+// ---------------------------------------------------------------------------------------------------
+__global__ void add_vec_kernel(float* y, const float* x, int64_t n) {
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) y[i] += x[i];
+}
+
+__global__ void f32_to_bf16_kernel(const float* x, __nv_bfloat16* y, int64_t n) {
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) y[i] = __float2bfloat16_rn(x[i]);
+}
+
+omq_status omq_qlinear_fwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t Cout, const float* X, const void* W,
+                           const float* B, const float* s, const float* delta, const float* gamma_logit,
+                           const float* beta_logit, float* Y, const omq_qlinear_saved* sv, const omq_qcfg* cfg) {
+  OMQ_TRY(omq_check_cfg(cfg));
+  OMQ_REQUIRE(T > 0 && Cin > 0 && Cout > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(X && W && Y && sv && sv->w_hat && sv->x_hat && sv->b_tilde, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(!cfg->let || (s && delta), OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(Cin % 8 == 0 && Cout % 8 == 0, OMQ_ERR_ALIGN);
+  cudaStream_t st = (cudaStream_t)stream;
+  const int g = cfg->group == 0 ? (int)Cin : cfg->group;
+  OMQ_REQUIRE(Cin % g == 0, OMQ_ERR_SHAPE);
+  QState4 qw{sv->h_w, sv->z_w, sv->imax_w, sv->imin_w};
+  const bool let = cfg->let != 0;
+  OMQ_TRY(lwc_fwd_launch(st, lwc_args((const bf16*)W, Cout, Cin, *cfg, let ? s : nullptr, nullptr, gamma_logit,
+                                      beta_logit, (bf16*)sv->w_hat, qw, let ? delta : nullptr, nullptr,
+                                      let ? sv->b_tilde : nullptr)));
+  const float* bias = nullptr;
+  if (let) {
+    if (B) { add_vec_kernel<<<(unsigned)((Cout + 255) / 256), 256, 0, st>>>(sv->b_tilde, B, Cout); OMQ_LAUNCH_CHECK(); }
+    bias = sv->b_tilde;
+  } else if (B) {
+    OMQ_TRY(vec_copy(st, sv->b_tilde, B, Cout));
+    bias = sv->b_tilde;
+  }
+  ActFwdArgs a{};
+  a.producer = let ? AP_LET : AP_PLAIN; a.X = X; a.ldx = Cin; a.s = let ? s : nullptr; a.delta = let ? delta : nullptr;
+  a.T = T; a.C = Cin; a.Xq = (bf16*)sv->x_hat; a.ldq = Cin; a.h = sv->h_a; a.z = sv->z_a; a.imax = sv->imax_a;
+  a.imin = sv->imin_a; a.abits = cfg->abits; a.eps = cfg->h_eps;
+  OMQ_TRY(act_fwd_launch(st, a));
+  return gemm_kk(st, T, Cout, Cin, (const bf16*)sv->x_hat, Cin, (const bf16*)sv->w_hat, Cin, Y, nullptr, Cout, bias,
+                 nullptr, cfg->dev_status);
+}
+
+size_t omq_qlinear_workspace_size(int64_t T, int64_t Cin, int64_t Cout, const omq_qcfg* cfg) {
+  (void)cfg;
+  Carve c{nullptr, 0};
+  c.take<bf16>(T * Cout);                       // dY in bf16
+  c.take<float>(Cout * Cin);                    // dW_hat
+  c.take<float>(T * Cin);                       // dX_hat
+  c.take<float>(Cout);                          // dB~
+  int64_t pe = imax64(2 * lwc_bwd_nslab(Cout) * Cin, 2 * ((T + 3) / 4) * Cin);
+  pe = imax64(pe, colsum_rows_parts(T) * Cout);
+  c.take<float>(pe);
+  return c.off + 256;
+}
+
+omq_status omq_qlinear_bwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t Cout, const float* X, const void* W,
+                           const float* s, const float* delta, const float* gamma_logit, const float* beta_logit,
+                           const omq_qlinear_saved* sv, const float* dY, float* dX, float* dgamma, float* dbeta,
+                           float* ds, float* ddelta, void* workspace, size_t ws_bytes, const omq_qcfg* cfg) {
+  OMQ_TRY(omq_check_cfg(cfg));
+  OMQ_REQUIRE(T > 0 && Cin > 0 && Cout > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(cfg->wbits < 16, OMQ_ERR_UNSUPPORTED);
+  OMQ_REQUIRE(X && W && sv && dY && dgamma && dbeta, OMQ_ERR_INVALID_ARG);
+  const bool let = cfg->let != 0;
+  OMQ_REQUIRE(!let || (s && delta && ds && ddelta), OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(workspace && ws_bytes >= omq_qlinear_workspace_size(T, Cin, Cout, cfg), OMQ_ERR_WORKSPACE);
+  OMQ_REQUIRE(omq_aligned16(workspace) && omq_aligned16(dY), OMQ_ERR_ALIGN);
+  cudaStream_t st = (cudaStream_t)stream;
+  Carve c{(uint8_t*)workspace, 0};
+  bf16* dYb = c.take<bf16>(T * Cout);
+  float* dWh = c.take<float>(Cout * Cin);
+  float* dXh = c.take<float>(T * Cin);
+  float* dB = c.take<float>(Cout);
+  int64_t pe = imax64(2 * lwc_bwd_nslab(Cout) * Cin, 2 * ((T + 3) / 4) * Cin);
+  pe = imax64(pe, colsum_rows_parts(T) * Cout);
+  float* part = c.take<float>(pe);
+  f32_to_bf16_kernel<<<(unsigned)((T * Cout + 255) / 256), 256, 0, st>>>(dY, dYb, T * Cout);
+  OMQ_LAUNCH_CHECK();
+  OMQ_TRY(gemm_dw(st, T, Cout, Cin, dYb, (const bf16*)sv->x_hat, dWh, cfg->dev_status));
+  if (let) OMQ_TRY(colsum_rows(st, dY, T, Cout, Cout, part, dB, 1.f, 0));
+  QState4 qw{sv->h_w, sv->z_w, sv->imax_w, sv->imin_w};
+  omq_qcfg cf = *cfg;
+  OMQ_TRY(lwc_bwd_full(st, (const bf16*)W, Cout, Cin, cf, let ? s : nullptr, nullptr, gamma_logit, beta_logit, qw, dWh,
+                       dgamma, dbeta, nullptr, let ? dB : nullptr, let ? ds : nullptr, let ? ddelta : nullptr,
+                       cfg->accumulate, part));
+  if (dX || let) {
+    OMQ_TRY(gemm_dx(st, T, Cout, Cin, dYb, (const bf16*)sv->w_hat, dXh, cfg->dev_status));
+    ActBwdArgs a{};
+    a.producer = let ? AP_LET : AP_PLAIN; a.X = X; a.ldx = Cin; a.s = let ? s : nullptr; a.delta = let ? delta : nullptr;
+    a.T = T; a.C = Cin; a.h = sv->h_a; a.z = sv->z_a; a.imax = sv->imax_a; a.imin = sv->imin_a; a.dXq = dXh; a.lddq = Cin;
+    a.dX = dX; a.lddx = Cin; a.rows_per_cta = 4; a.abits = cfg->abits; a.eps = cfg->h_eps;
+    a.part_s = let ? part : nullptr;
+    a.part_d = let ? part + ((T + 3) / 4) * Cin : nullptr;
+    OMQ_TRY(act_bwd_launch(st, a));
+    if (let) {
+      OMQ_TRY(omq_colsum_partials(st, a.part_s, (T + 3) / 4, Cin, ds, 1.f, 1));
+      OMQ_TRY(omq_colsum_partials(st, a.part_d, (T + 3) / 4, Cin, ddelta, 1.f, 1));
+    }
+  }
+  return OMQ_OK;
+}
+
+}  // extern "C"

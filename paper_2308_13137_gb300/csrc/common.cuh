@@ -1,0 +1,201 @@
+// Shared device/host helpers of libomq (sm_103a).
+#pragma once
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <math.h>
+
+#include "omq.h"
+
+#define OMQ_VERSION 1
+
+// ------------------------------------------------------------------------------------------------
+// host-side argument checks
+// ------------------------------------------------------------------------------------------------
+#define OMQ_REQUIRE(cond, code) do { if (!(cond)) return (code); } while (0)
+#define OMQ_LAUNCH_CHECK() do { if (cudaPeekAtLastError() != cudaSuccess) { cudaGetLastError(); return OMQ_ERR_CUDA; } } while (0)
+#define OMQ_TRY(expr) do { omq_status _s = (expr); if (_s != OMQ_OK) return _s; } while (0)
+
+static inline bool omq_aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+static inline bool omq_bits_ok(int b) { return (b >= 2 && b <= 8) || b == 16; }
+
+static inline omq_status omq_check_cfg(const omq_qcfg* cfg) {
+  if (!cfg) return OMQ_ERR_INVALID_ARG;
+  if (!omq_bits_ok(cfg->wbits) || !omq_bits_ok(cfg->abits)) return OMQ_ERR_UNSUPPORTED;
+  if (cfg->group < 0) return OMQ_ERR_SHAPE;
+  if (!(cfg->h_eps > 0.f)) return OMQ_ERR_INVALID_ARG;
+  return OMQ_OK;
+}
+
+static inline int omq_num_sms() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  }
+  return n;
+}
+
+// ------------------------------------------------------------------------------------------------
+// device status word and bounded waits
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ void omq_set_status(int32_t* st, int32_t code) {
+  if (st) atomicCAS(st, 0, code);
+}
+
+__device__ __forceinline__ uint64_t omq_globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Upper bound of any single device-side wait: one second.
+#define OMQ_WAIT_LIMIT_NS 1000000000ull
+
+// ------------------------------------------------------------------------------------------------
+// conversions
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ float bf16_to_f(__nv_bfloat16 v) { return __bfloat162float(v); }
+__device__ __forceinline__ __nv_bfloat16 f_to_bf16(float v) { return __float2bfloat16_rn(v); }
+
+__device__ __forceinline__ void unpack_bf16x8(const uint4& u, float* f) {
+  const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    float2 t = __bfloat1622float2(p[i]);
+    f[2 * i] = t.x;
+    f[2 * i + 1] = t.y;
+  }
+}
+
+__device__ __forceinline__ uint4 pack_bf16x8(const float* f) {
+  uint4 u;
+  __nv_bfloat162* p = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) p[i] = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
+  return u;
+}
+
+// ------------------------------------------------------------------------------------------------
+// Eq. 2 on one element, given the group's h and z (IEEE division, round half to even)
+// ------------------------------------------------------------------------------------------------
+struct QState {          // per-group quantizer state
+  float h;               // step, floored at eps
+  float z;               // zero point (integer valued)
+  float u;               // beta * min / h
+  float a, b;            // clipping strengths
+  float M, m;            // group max / min
+  int floored;
+};
+
+// gamma = sigmoid(gamma_hat), evaluated in double and rounded once to float, so that the
+// clipping strength is the correctly rounded value of the logit's sigmoid.
+__device__ __forceinline__ float omq_sigmoid(float t) { return (float)(1.0 / (1.0 + exp(-(double)t))); }
+
+__device__ __forceinline__ QState omq_qstate(float M, float m, float a, float b, float Q, float eps) {
+  QState s;
+  s.a = a; s.b = b; s.M = M; s.m = m;
+  float hr = __fdiv_rn(__fsub_rn(__fmul_rn(a, M), __fmul_rn(b, m)), Q);
+  s.floored = !(hr >= eps);
+  s.h = s.floored ? eps : hr;
+  s.u = __fdiv_rn(__fmul_rn(b, m), s.h);
+  s.z = -rintf(s.u);
+  return s;
+}
+
+// code c = round(w/h) + z before the clamp
+__device__ __forceinline__ float omq_code_raw(float w, const QState& s, float* x_out) {
+  float x = __fdiv_rn(w, s.h);
+  *x_out = x;
+  return rintf(x) + s.z;
+}
+
+__device__ __forceinline__ float omq_fakequant(float w, const QState& s, float Q, float* code) {
+  float x;
+  float c = omq_code_raw(w, s, &x);
+  float q = fminf(fmaxf(c, 0.f), Q);
+  if (code) *code = q;
+  return __fmul_rn(q - s.z, s.h);
+}
+
+// STE pieces of one element: returns dwhat/dh; *inr = 1 when 0 <= c <= Q
+__device__ __forceinline__ float omq_ste_dh(float w, const QState& s, float Q, int* inr) {
+  float x;
+  float c = omq_code_raw(w, s, &x);
+  if (c >= 0.f && c <= Q) { *inr = 1; return rintf(x) - x; }
+  *inr = 0;
+  float ru = rintf(s.u) - s.u;
+  return (c < 0.f) ? ru : (Q + ru);
+}
+
+// ------------------------------------------------------------------------------------------------
+// (value, index) reductions with first-index tie break
+// ------------------------------------------------------------------------------------------------
+struct MaxMin { float M; int iM; float m; int im; };
+
+__device__ __forceinline__ MaxMin mm_identity() { MaxMin r; r.M = -INFINITY; r.iM = 0x7fffffff; r.m = INFINITY; r.im = 0x7fffffff; return r; }
+
+__device__ __forceinline__ void mm_push(MaxMin& r, float v, int i) {
+  if (v > r.M || (v == r.M && i < r.iM)) { r.M = v; r.iM = i; }
+  if (v < r.m || (v == r.m && i < r.im)) { r.m = v; r.im = i; }
+}
+
+__device__ __forceinline__ void mm_merge(MaxMin& r, const MaxMin& o) {
+  if (o.M > r.M || (o.M == r.M && o.iM < r.iM)) { r.M = o.M; r.iM = o.iM; }
+  if (o.m < r.m || (o.m == r.m && o.im < r.im)) { r.m = o.m; r.im = o.im; }
+}
+
+// reduction across `width` consecutive lanes (width power of two, <= 32)
+__device__ __forceinline__ MaxMin mm_shfl_reduce(MaxMin r, int width) {
+  for (int off = width >> 1; off > 0; off >>= 1) {
+    MaxMin o;
+    o.M = __shfl_xor_sync(0xffffffffu, r.M, off);
+    o.iM = __shfl_xor_sync(0xffffffffu, r.iM, off);
+    o.m = __shfl_xor_sync(0xffffffffu, r.m, off);
+    o.im = __shfl_xor_sync(0xffffffffu, r.im, off);
+    mm_merge(r, o);
+  }
+  return r;
+}
+
+// block-wide reduction; result valid in every thread.  smem: >= 32 MaxMin.
+__device__ __forceinline__ MaxMin mm_block_reduce(MaxMin r, MaxMin* smem) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  r = mm_shfl_reduce(r, 32);
+  __syncthreads();
+  if (lane == 0) smem[wid] = r;
+  __syncthreads();
+  MaxMin t = mm_identity();
+  if (lane < nw) t = smem[lane];
+  t = mm_shfl_reduce(t, 32);
+  return t;
+}
+
+__device__ __forceinline__ float warp_sum(float v, int width = 32) {
+  for (int off = width >> 1; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return v;
+}
+
+// block-wide sum of up to 2 values; results valid in every thread.  smem: >= 64 floats.
+__device__ __forceinline__ float2 block_sum2(float a, float b, float* smem) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  a = warp_sum(a);
+  b = warp_sum(b);
+  __syncthreads();
+  if (lane == 0) { smem[wid] = a; smem[32 + wid] = b; }
+  __syncthreads();
+  float x = lane < nw ? smem[lane] : 0.f;
+  float y = lane < nw ? smem[32 + lane] : 0.f;
+  x = warp_sum(x);
+  y = warp_sum(y);
+  return make_float2(x, y);
+}
+
+// deterministic column reduction: out[c] (+)= sum_p part[p, c]
+__global__ void omq_colsum_partials_kernel(const float* __restrict__ part, int64_t P, int64_t C,
+                                           float* __restrict__ out, float scale, int accumulate);
+
+omq_status omq_colsum_partials(cudaStream_t st, const float* part, int64_t P, int64_t C, float* out,
+                               float scale, int accumulate);

@@ -1,0 +1,393 @@
+// Dense bf16 matrix product on the 5th-generation tensor cores (sm_103a):
+// TMA (cp.async.bulk.tensor, 128-byte swizzle) -> shared-memory ring of STAGES slots guarded by
+// mbarriers -> tcgen05.mma (M = 128, N = BN, K = 16, fp32 accumulator in tensor memory) ->
+// tcgen05.ld epilogue (alpha, bias, residual, accumulate) -> fp32 / bf16 global stores.
+//
+// Warp roles (192 threads): warp 0 issues TMA loads, warp 1 owns tensor memory and issues the
+// MMAs, warps 2..5 drain the accumulator (warp w reads TMEM lanes 32*(w%4) .. +31).
+// Every wait on an mbarrier is bounded (OMQ_WAIT_LIMIT_NS); on expiry the kernel writes
+// OMQ_ERR_TIMEOUT to the status word, stops issuing work, frees its tensor memory and exits.
+#include "gemm.cuh"
+#include <cuda.h>
+
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;          // one 128-byte swizzle row of bf16
+constexpr int UMMA_K = 16;
+constexpr int NUM_THREADS = 192;
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait on a phase parity; false when the time limit expired.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = omq_globaltimer();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 32; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
+    if (omq_globaltimer() - t0 > OMQ_WAIT_LIMIT_NS) return false;
+  }
+}
+
+__device__ __forceinline__ void tma_load_3d(const CUtensorMap* map, uint64_t* bar, void* dst, int c0, int c1, int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
+      ::"r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* holder, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(holder)), "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accum) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+      ::"r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum)
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor: 128-byte swizzle, descriptor version 1 (bits 46-47).
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, major-ness, N, M.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int a_mn, int b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)a_mn << 15) | ((uint32_t)b_mn << 16) |
+         ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+struct GemmParams {
+  int M, N, K, batch;
+  int a_mn, b_mn;            // 1 = MN-major operand
+  int causal;
+  GemmEpilogue ep;
+  int32_t* status;
+};
+
+template <int BN, int STAGES>
+struct SmemLayout {
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int BAR_OFF = STAGES * STAGE_BYTES;
+  static constexpr int TOTAL = BAR_OFF + 256 + 1024;  // + barriers + alignment slack
+};
+
+template <int BN, int STAGES>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                     const GemmParams p) {
+  using L = SmemLayout<BN, STAGES>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + L::BAR_OFF);
+  uint64_t* empty = full + STAGES;
+  uint64_t* accum = empty + STAGES;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(accum + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN, b = blockIdx.z;
+
+  // causal tile skip (scores / their gradient): keys beyond every query of the tile
+  if (p.causal == 1 && n0 > m0 + BM - 1) return;
+  int k_begin = 0, k_end = p.K;
+  if (p.causal == 2) k_end = min(p.K, m0 + BM);
+  if (p.causal == 3) k_begin = m0;
+  const int nkb = k_end > k_begin ? (k_end - k_begin + BK - 1) / BK : 0;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    mbar_init(accum, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, BN);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer ----------------
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int s = kb % STAGES;
+      if (kb >= STAGES) {
+        if (!mbar_wait(&empty[s], ((kb / STAGES) - 1) & 1)) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; break; }
+      }
+      if (*abort_flag) break;
+      uint8_t* sa = smem + s * L::STAGE_BYTES;
+      uint8_t* sb = sa + L::A_BYTES;
+      const int k0 = k_begin + kb * BK;
+      mbar_expect_tx(&full[s], L::STAGE_BYTES);
+      if (!p.a_mn) {
+        tma_load_3d(&tmA, &full[s], sa, k0, m0, b);
+      } else {
+        tma_load_3d(&tmA, &full[s], sa, m0, k0, b);
+        tma_load_3d(&tmA, &full[s], sa + 64 * BK * 2, m0 + 64, k0, b);
+      }
+      if (!p.b_mn) {
+        tma_load_3d(&tmB, &full[s], sb, k0, n0, b);
+      } else {
+#pragma unroll
+        for (int j = 0; j < BN / 64; ++j) tma_load_3d(&tmB, &full[s], sb + j * 64 * BK * 2, n0 + 64 * j, k0, b);
+      }
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer ----------------
+    constexpr uint32_t IDESC_KK = idesc_bf16(BM, BN, 0, 0);
+    const uint32_t idesc = IDESC_KK | ((uint32_t)p.a_mn << 15) | ((uint32_t)p.b_mn << 16);
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int s = kb % STAGES;
+      if (!mbar_wait(&full[s], (kb / STAGES) & 1)) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; break; }
+      tc_fence_after();
+      const uint32_t sa = smem_u32(smem + s * L::STAGE_BYTES);
+      const uint32_t sb = sa + L::A_BYTES;
+#pragma unroll
+      for (int k = 0; k < BK / UMMA_K; ++k) {
+        // K-major: advance 32 bytes inside the swizzle row; MN-major: advance 16 K-rows (2 KB)
+        const uint64_t ad = p.a_mn ? sdesc(sa + k * 2048, 64 * BK * 2, 1024) : sdesc(sa + k * 32, 16, 1024);
+        const uint64_t bd = p.b_mn ? sdesc(sb + k * 2048, 64 * BK * 2, 1024) : sdesc(sb + k * 32, 16, 1024);
+        umma_bf16(tmem, ad, bd, idesc, (kb | k) != 0);
+      }
+      umma_commit(&empty[s]);
+    }
+    umma_commit(accum);
+  } else if (warp >= 2) {
+    // ---------------- epilogue ----------------
+    const int q = warp & 3;                       // TMEM lane quadrant of this warp
+    const int row = m0 + q * 32 + lane;
+    bool ok = true;
+    if (nkb > 0) {
+      ok = mbar_wait(accum, 0);
+      if (!ok) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; }
+      tc_fence_after();
+    }
+    const GemmEpilogue& ep = p.ep;
+    const bool row_ok = row < p.M;
+    const int64_t crow = (int64_t)b * ep.c_bs + (int64_t)row * ep.ldc;
+#pragma unroll 1
+    for (int j0 = 0; j0 < BN; j0 += 32) {
+      float v[32];
+      if (nkb > 0 && ok) {
+        tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)j0, v);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = 0.f;
+      }
+      const int nb = n0 + j0;
+      if (!row_ok || nb >= p.N) continue;
+      const bool full_chunk = nb + 32 <= p.N;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        v[i] *= ep.alpha;
+      }
+      if (full_chunk) {
+        if (ep.bias) {
+#pragma unroll
+          for (int i = 0; i < 32; i += 4) {
+            float4 bb = __ldg(reinterpret_cast<const float4*>(ep.bias + nb + i));
+            v[i] += bb.x; v[i + 1] += bb.y; v[i + 2] += bb.z; v[i + 3] += bb.w;
+          }
+        }
+        if (ep.R) {
+          const float* rr = ep.R + (int64_t)b * ep.c_bs + (int64_t)row * ep.ldr + nb;
+#pragma unroll
+          for (int i = 0; i < 32; i += 4) {
+            float4 t = __ldg(reinterpret_cast<const float4*>(rr + i));
+            v[i] += t.x; v[i + 1] += t.y; v[i + 2] += t.z; v[i + 3] += t.w;
+          }
+        }
+        if (ep.Cf) {
+          float* cp = ep.Cf + crow + nb;
+          if (ep.beta_acc != 0.f) {
+#pragma unroll
+            for (int i = 0; i < 32; i += 4) {
+              float4 t = *reinterpret_cast<const float4*>(cp + i);
+              v[i] += ep.beta_acc * t.x; v[i + 1] += ep.beta_acc * t.y;
+              v[i + 2] += ep.beta_acc * t.z; v[i + 3] += ep.beta_acc * t.w;
+            }
+          }
+#pragma unroll
+          for (int i = 0; i < 32; i += 4) *reinterpret_cast<float4*>(cp + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+        }
+        if (ep.Cb) {
+          __nv_bfloat16* cp = ep.Cb + crow + nb;
+#pragma unroll
+          for (int i = 0; i < 32; i += 8) *reinterpret_cast<uint4*>(cp + i) = pack_bf16x8(v + i);
+        }
+      } else {
+        for (int i = 0; i < 32 && nb + i < p.N; ++i) {
+          const int n = nb + i;
+          float x = v[i];
+          if (ep.bias) x += ep.bias[n];
+          if (ep.R) x += ep.R[(int64_t)b * ep.c_bs + (int64_t)row * ep.ldr + n];
+          if (ep.Cf) {
+            if (ep.beta_acc != 0.f) x += ep.beta_acc * ep.Cf[crow + n];
+            ep.Cf[crow + n] = x;
+          }
+          if (ep.Cb) ep.Cb[crow + n] = f_to_bf16(x);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, BN);
+  }
+}
+
+// ---------------------------------------------------------------------------------------------
+// host side: tensor maps through the driver entry point (no link-time dependency on libcuda)
+// ---------------------------------------------------------------------------------------------
+typedef CUresult (*PFN_encodeTiled_t)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                      const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                      CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+PFN_encodeTiled_t get_encode() {
+  static PFN_encodeTiled_t fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_encodeTiled_t>(ptr);
+  }
+  return fn;
+}
+
+// 3-D bf16 map {inner, rows, batch} with a {64, box_rows, 1} box and 128-byte swizzle.
+bool make_map(CUtensorMap* map, const void* ptr, int64_t inner, int64_t rows, int64_t batch, int64_t ld, int64_t bs,
+              int box_rows) {
+  PFN_encodeTiled_t enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)inner, (cuuint64_t)rows, (cuuint64_t)batch};
+  cuuint64_t strides[2] = {(cuuint64_t)(ld * 2), (cuuint64_t)((batch > 1 ? bs : ld * rows) * 2)};
+  cuuint32_t box[3] = {64u, (cuuint32_t)box_rows, 1u};
+  cuuint32_t estr[3] = {1u, 1u, 1u};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+template <int BN, int STAGES>
+omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap& tb, const GemmParams& p) {
+  using L = SmemLayout<BN, STAGES>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    if (cudaFuncSetAttribute(gemm_bf16_kernel<BN, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::TOTAL) !=
+        cudaSuccess)
+      return OMQ_ERR_CUDA;
+    attr_set = true;
+  }
+  dim3 grid((unsigned)((p.M + BM - 1) / BM), (unsigned)((p.N + BN - 1) / BN), (unsigned)p.batch);
+  gemm_bf16_kernel<BN, STAGES><<<grid, NUM_THREADS, L::TOTAL, st>>>(ta, tb, p);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+}  // namespace
+
+omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t batch, const GemmOperand& A,
+                       const GemmOperand& B, const GemmEpilogue& ep, int causal, int32_t* status) {
+  OMQ_REQUIRE(M > 0 && N > 0 && K > 0 && batch > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(M < (1ll << 31) && N < (1ll << 31) && K < (1ll << 31) && batch < 65536, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(A.ptr && B.ptr && (ep.Cf || ep.Cb), OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(causal >= 0 && causal <= 3, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(omq_aligned16(A.ptr) && omq_aligned16(B.ptr), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(A.ld % 8 == 0 && B.ld % 8 == 0 && (batch == 1 || (A.bs % 8 == 0 && B.bs % 8 == 0)), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(ep.ldc % 8 == 0 && (batch == 1 || ep.c_bs % 8 == 0), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE((!ep.Cf || omq_aligned16(ep.Cf)) && (!ep.Cb || omq_aligned16(ep.Cb)), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(!ep.R || (omq_aligned16(ep.R) && ep.ldr % 4 == 0), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(!ep.bias || omq_aligned16(ep.bias), OMQ_ERR_ALIGN);
+  // the MN-major extents must cover whole 64-wide boxes inside the tensor (TMA zero-fills the rest)
+  const bool wide = (N % 256 == 0);
+  CUtensorMap ta, tb;
+  const int bn = wide ? 256 : 128;
+  bool ok = A.kmajor ? make_map(&ta, A.ptr, K, M, batch, A.ld, A.bs, BM) : make_map(&ta, A.ptr, M, K, batch, A.ld, A.bs, BK);
+  ok = ok && (B.kmajor ? make_map(&tb, B.ptr, K, N, batch, B.ld, B.bs, bn) : make_map(&tb, B.ptr, N, K, batch, B.ld, B.bs, BK));
+  if (!ok) return OMQ_ERR_UNSUPPORTED;
+  GemmParams p;
+  p.M = (int)M; p.N = (int)N; p.K = (int)K; p.batch = (int)batch;
+  p.a_mn = A.kmajor ? 0 : 1; p.b_mn = B.kmajor ? 0 : 1;
+  p.causal = causal; p.ep = ep; p.status = status;
+  if (wide) return launch_cfg<256, 4>(st, ta, tb, p);
+  return launch_cfg<128, 6>(st, ta, tb, p);
+}
+
+extern "C" omq_status omq_gemm_bf16(omq_stream_t stream, int64_t M, int64_t N, int64_t K, int64_t batch, const void* A,
+                                    int64_t a_ld, int64_t a_bs, int32_t a_kmajor, const void* B, int64_t b_ld,
+                                    int64_t b_bs, int32_t b_kmajor, float* Cf, void* Cb, int64_t ldc, int64_t c_bs,
+                                    float alpha, const float* bias, const float* R, int64_t ldr, float beta_acc,
+                                    int32_t causal, int32_t* dev_status) {
+  GemmOperand a{A, a_ld, a_bs, a_kmajor ? 1 : 0};
+  GemmOperand b{B, b_ld, b_bs, b_kmajor ? 1 : 0};
+  GemmEpilogue ep{Cf, (__nv_bfloat16*)Cb, ldc, c_bs, alpha, bias, R, ldr, beta_acc};
+  return gemm_launch((cudaStream_t)stream, M, N, K, batch, a, b, ep, causal, dev_status);
+}

@@ -1,0 +1,980 @@
+// HBM-bound kernels of the calibration step: LWC (Eq. 2) forward/backward on the LET-scaled
+// weight (Eq. 3), the per-token MinMax activation quantizer with fused producers (LET, RMSNorm,
+// SwiGLU) and its straight-through backward, the block loss (Eq. 1), column reductions and AdamW.
+#include "quant.cuh"
+
+#define LWC_MAXC 16        // 8-element chunks per thread held in registers (Cin <= 256*8*16)
+#define ACT_THREADS 256
+
+// ================================================================================================
+// LWC forward: one CTA per output row.
+// ================================================================================================
+__device__ __forceinline__ float lwc_wt(float w, const float* s, int64_t col, float rr) {
+  float sv = s ? s[col] : 1.f;
+  return __fmul_rn(__fmul_rn(w, sv), rr);
+}
+
+__global__ void __launch_bounds__(256) lwc_fwd_kernel(LwcFwdArgs a) {
+  __shared__ MaxMin red_mm[32];
+  __shared__ float red_f[64];
+  __shared__ MaxMin row_mm;
+  const int64_t o = blockIdx.x;
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int64_t nchunk = a.Cin / 8;
+  const int nit = (int)((nchunk + nt - 1) / nt);
+  const float Q = (float)((1 << a.wbits) - 1);
+  const int gsz = a.group;
+  const int lpg = gsz / 8;                       // lanes per group
+  const bool seg = (gsz < a.Cin) || (lpg <= 32 && (lpg & (lpg - 1)) == 0 && gsz == a.Cin && a.Cin <= 256);
+  const int64_t ngroups = a.Cin / gsz;
+  const float rr = a.r ? a.r[o] : 1.f;
+  const __nv_bfloat16* Wrow = a.W + o * a.Cin;
+
+  uint4 raw[LWC_MAXC];
+#pragma unroll
+  for (int i = 0; i < LWC_MAXC; ++i) {
+    raw[i] = make_uint4(0, 0, 0, 0);
+    if (i < nit) {
+      int64_t c = (int64_t)i * nt + tid;
+      if (c < nchunk) raw[i] = __ldg(reinterpret_cast<const uint4*>(Wrow) + c);
+    }
+  }
+  // LET bias B~_o = r_o (sum_i W_oi delta_i - shift_o)
+  if (a.Bt) {
+    float dot = 0.f;
+#pragma unroll
+    for (int i = 0; i < LWC_MAXC; ++i) {
+      if (i < nit) {
+        int64_t c = (int64_t)i * nt + tid;
+        if (c < nchunk) {
+          float w[8];
+          unpack_bf16x8(raw[i], w);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) dot = fmaf(w[e], a.bias_delta[c * 8 + e], dot);
+        }
+      }
+    }
+    float2 t = block_sum2(dot, 0.f, red_f);
+    if (tid == 0) a.Bt[o] = rr * (t.x - (a.bias_shift ? a.bias_shift[o] : 0.f));
+  }
+  if (a.wbits >= 16) {   // quantization off: W_hat = bf16(W~)
+#pragma unroll
+    for (int i = 0; i < LWC_MAXC; ++i) {
+      if (i < nit) {
+        int64_t c = (int64_t)i * nt + tid;
+        if (c < nchunk) {
+          float w[8];
+          unpack_bf16x8(raw[i], w);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w[e] = lwc_wt(w[e], a.s, c * 8 + e, rr);
+          if (a.Wq) reinterpret_cast<uint4*>(a.Wq + o * a.Cin)[c] = pack_bf16x8(w);
+        }
+      }
+    }
+    return;
+  }
+
+  if (!seg) {
+    // ---- one group per row: block-wide max/min, then quantize ----
+    MaxMin r = mm_identity();
+#pragma unroll
+    for (int i = 0; i < LWC_MAXC; ++i) {
+      if (i < nit) {
+        int64_t c = (int64_t)i * nt + tid;
+        if (c < nchunk) {
+          float w[8];
+          unpack_bf16x8(raw[i], w);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) mm_push(r, lwc_wt(w[e], a.s, c * 8 + e, rr), (int)(c * 8 + e));
+        }
+      }
+    }
+    r = mm_block_reduce(r, red_mm);
+    if (tid == 0) row_mm = r;
+    __syncthreads();
+    r = row_mm;
+    float ga = a.lwc ? omq_sigmoid(a.gl[o]) : 1.f;
+    float gb = a.lwc ? omq_sigmoid(a.bl[o]) : 1.f;
+    QState qs = omq_qstate(r.M, r.m, ga, gb, Q, a.eps);
+    if (tid == 0) {
+      a.h[o] = qs.h; a.z[o] = (int32_t)qs.z; a.imax[o] = r.iM; a.imin[o] = r.im;
+    }
+#pragma unroll
+    for (int i = 0; i < LWC_MAXC; ++i) {
+      if (i < nit) {
+        int64_t c = (int64_t)i * nt + tid;
+        if (c < nchunk) {
+          float w[8], cd[8];
+          unpack_bf16x8(raw[i], w);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w[e] = omq_fakequant(lwc_wt(w[e], a.s, c * 8 + e, rr), qs, Q, &cd[e]);
+          if (a.Wq) reinterpret_cast<uint4*>(a.Wq + o * a.Cin)[c] = pack_bf16x8(w);
+          if (a.codes) {
+            uint2 pk;
+            pk.x = (uint32_t)cd[0] | ((uint32_t)cd[1] << 8) | ((uint32_t)cd[2] << 16) | ((uint32_t)cd[3] << 24);
+            pk.y = (uint32_t)cd[4] | ((uint32_t)cd[5] << 8) | ((uint32_t)cd[6] << 16) | ((uint32_t)cd[7] << 24);
+            reinterpret_cast<uint2*>(a.codes + o * a.Cin)[c] = pk;
+          }
+        }
+      }
+    }
+    return;
+  }
+
+  // ---- groups of lpg consecutive lanes (lpg a power of two <= 32) ----
+  const int lane = tid & 31;
+#pragma unroll
+  for (int i = 0; i < LWC_MAXC; ++i) {
+    if (i < nit) {
+      int64_t c = (int64_t)i * nt + tid;
+      bool valid = c < nchunk;
+      float w[8];
+      unpack_bf16x8(raw[i], w);
+      MaxMin r = mm_identity();
+      if (valid) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) { w[e] = lwc_wt(w[e], a.s, c * 8 + e, rr); mm_push(r, w[e], (int)(c * 8 + e)); }
+      }
+      r = mm_shfl_reduce(r, lpg);
+      if (valid) {
+        int64_t gi = (c * 8) / gsz;
+        float ga = a.lwc ? omq_sigmoid(a.gl[o * ngroups + gi]) : 1.f;
+        float gb = a.lwc ? omq_sigmoid(a.bl[o * ngroups + gi]) : 1.f;
+        QState qs = omq_qstate(r.M, r.m, ga, gb, Q, a.eps);
+        if ((lane & (lpg - 1)) == 0) {
+          int64_t k = o * ngroups + gi;
+          a.h[k] = qs.h; a.z[k] = (int32_t)qs.z; a.imax[k] = r.iM; a.imin[k] = r.im;
+        }
+        float cd[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) w[e] = omq_fakequant(w[e], qs, Q, &cd[e]);
+        if (a.Wq) reinterpret_cast<uint4*>(a.Wq + o * a.Cin)[c] = pack_bf16x8(w);
+        if (a.codes) {
+          uint2 pk;
+          pk.x = (uint32_t)cd[0] | ((uint32_t)cd[1] << 8) | ((uint32_t)cd[2] << 16) | ((uint32_t)cd[3] << 24);
+          pk.y = (uint32_t)cd[4] | ((uint32_t)cd[5] << 8) | ((uint32_t)cd[6] << 16) | ((uint32_t)cd[7] << 24);
+          reinterpret_cast<uint2*>(a.codes + o * a.Cin)[c] = pk;
+        }
+      }
+    }
+  }
+}
+
+static bool lwc_group_ok(int64_t Cin, int g) {
+  if (g == Cin) return Cin % 8 == 0;
+  if (g < 8 || g > 256 || (g & (g - 1))) return false;
+  return Cin % g == 0;
+}
+
+static int lwc_threads(int64_t Cin) {
+  int64_t nchunk = Cin / 8;
+  int nt = 256;
+  if (nchunk < 256) nt = (int)((nchunk + 31) / 32 * 32);
+  return nt;
+}
+
+omq_status lwc_fwd_launch(cudaStream_t st, const LwcFwdArgs& a) {
+  OMQ_REQUIRE(lwc_group_ok(a.Cin, a.group), OMQ_ERR_UNSUPPORTED);
+  OMQ_REQUIRE(a.Cin / 8 <= (int64_t)256 * LWC_MAXC, OMQ_ERR_UNSUPPORTED);
+  lwc_fwd_kernel<<<(unsigned)a.Cout, lwc_threads(a.Cin), 0, st>>>(a);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+// ================================================================================================
+// LWC backward (straight-through, Eq. 2): one CTA per slab of rows; each thread owns fixed
+// columns and accumulates the LET column sums of its columns in shared memory.
+// ================================================================================================
+__global__ void __launch_bounds__(256) lwc_bwd_kernel(LwcBwdArgs a) {
+  extern __shared__ float acc[];                 // acc_s[Cin], acc_d[Cin]
+  __shared__ float red_f[64];
+  const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31;
+  const int64_t nchunk = a.Cin / 8;
+  const int nit = (int)((nchunk + nt - 1) / nt);
+  const float Q = (float)((1 << a.wbits) - 1);
+  const int gsz = a.group;
+  const int lpg = gsz / 8;
+  const bool seg = (gsz < a.Cin) || (lpg <= 32 && (lpg & (lpg - 1)) == 0 && gsz == a.Cin && a.Cin <= 256);
+  const int64_t ngroups = a.Cin / gsz;
+  const bool want_s = a.part_s != nullptr, want_d = a.part_d != nullptr && a.dBt != nullptr;
+  float* acc_s = acc;
+  float* acc_d = acc + a.Cin;
+  if (want_s || want_d)
+    for (int64_t c = tid; c < a.Cin; c += nt) { acc_s[c] = 0.f; acc_d[c] = 0.f; }
+  const int64_t o0 = (int64_t)blockIdx.x * a.rows_per_cta;
+  const int64_t o1 = min(a.Cout, o0 + a.rows_per_cta);
+
+  for (int64_t o = o0; o < o1; ++o) {
+    const float rr = a.r ? a.r[o] : 1.f;
+    const float dBo = (want_d) ? a.dBt[o] : 0.f;
+    const __nv_bfloat16* Wrow = a.W + o * a.Cin;
+    const float* grow = a.dWq + o * a.ld_dwq;
+    float dr_part = 0.f;
+
+    if (!seg) {
+      // per-row group: state from the saved indices
+      const int iM = a.imax[o], im = a.imin[o];
+      const float M = lwc_wt(bf16_to_f(Wrow[iM]), a.s, iM, rr);
+      const float m = lwc_wt(bf16_to_f(Wrow[im]), a.s, im, rr);
+      const float ga = a.lwc ? omq_sigmoid(a.gl[o]) : 1.f;
+      const float gb = a.lwc ? omq_sigmoid(a.bl[o]) : 1.f;
+      QState qs = omq_qstate(M, m, ga, gb, Q, a.eps);
+      qs.h = a.h[o]; qs.z = (float)a.z[o]; qs.u = __fdiv_rn(__fmul_rn(gb, m), qs.h);
+      float Gh = 0.f, Gbm = 0.f;
+      for (int i = 0; i < nit; ++i) {
+        int64_t c = (int64_t)i * nt + tid;
+        if (c < nchunk) {
+          float w[8];
+          unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(Wrow) + c), w);
+          float4 g0 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c);
+          float4 g1 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c + 1);
+          float g[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            int inr;
+            float dh = omq_ste_dh(lwc_wt(w[e], a.s, c * 8 + e, rr), qs, Q, &inr);
+            Gh = fmaf(g[e], dh, Gh);
+            if (!inr) Gbm += g[e];
+          }
+        }
+      }
+      float2 tot = block_sum2(Gh, Gbm, red_f);
+      Gh = qs.floored ? 0.f : tot.x;
+      Gbm = tot.y;
+      const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
+      if (tid == 0 && a.lwc) {
+        float dg = GaM * M * ga * (1.f - ga), db = Gbt * m * gb * (1.f - gb);
+        if (a.accumulate) { a.dgl[o] += dg; a.dbl[o] += db; } else { a.dgl[o] = dg; a.dbl[o] = db; }
+      }
+      for (int i = 0; i < nit; ++i) {
+        int64_t c = (int64_t)i * nt + tid;
+        if (c < nchunk) {
+          float w[8];
+          unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(Wrow) + c), w);
+          float4 g0 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c);
+          float4 g1 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c + 1);
+          float g[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+          float dwt[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            int64_t col = c * 8 + e;
+            int inr;
+            omq_ste_dh(lwc_wt(w[e], a.s, col, rr), qs, Q, &inr);
+            float d = inr ? g[e] : 0.f;
+            if (col == iM) d += GaM * ga;
+            if (col == im) d += Gbt * gb;
+            dwt[e] = d;
+            float sv = a.s ? a.s[col] : 1.f;
+            dr_part = fmaf(d * w[e], sv, dr_part);
+            if (want_s) acc_s[col] = fmaf(d * w[e], rr, acc_s[col]);
+            if (want_d) acc_d[col] = fmaf(dBo * rr, w[e], acc_d[col]);
+          }
+          if (a.dWt) {
+            float4* dst = reinterpret_cast<float4*>(a.dWt + o * a.Cin) + 2 * c;
+            dst[0] = make_float4(dwt[0], dwt[1], dwt[2], dwt[3]);
+            dst[1] = make_float4(dwt[4], dwt[5], dwt[6], dwt[7]);
+          }
+        }
+      }
+    } else {
+      for (int i = 0; i < nit; ++i) {
+        int64_t c = (int64_t)i * nt + tid;
+        bool valid = c < nchunk;
+        float w[8], g[8], wt[8];
+        int64_t gi = valid ? (c * 8) / gsz : 0;
+        int64_t k = o * ngroups + gi;
+        QState qs;
+        float ga = 1.f, gb = 1.f, M = 0.f, m = 0.f;
+        int iM = 0, im = 0;
+        float Gh = 0.f, Gbm = 0.f;
+        int inr_mask = 0;
+        if (valid) {
+          unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(Wrow) + c), w);
+          float4 g0 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c);
+          float4 g1 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c + 1);
+          g[0] = g0.x; g[1] = g0.y; g[2] = g0.z; g[3] = g0.w; g[4] = g1.x; g[5] = g1.y; g[6] = g1.z; g[7] = g1.w;
+          iM = a.imax[k]; im = a.imin[k];
+          M = lwc_wt(bf16_to_f(Wrow[iM]), a.s, iM, rr);
+          m = lwc_wt(bf16_to_f(Wrow[im]), a.s, im, rr);
+          ga = a.lwc ? omq_sigmoid(a.gl[k]) : 1.f;
+          gb = a.lwc ? omq_sigmoid(a.bl[k]) : 1.f;
+          qs = omq_qstate(M, m, ga, gb, Q, a.eps);
+          qs.h = a.h[k]; qs.z = (float)a.z[k]; qs.u = __fdiv_rn(__fmul_rn(gb, m), qs.h);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            wt[e] = lwc_wt(w[e], a.s, c * 8 + e, rr);
+            int inr;
+            float dh = omq_ste_dh(wt[e], qs, Q, &inr);
+            Gh = fmaf(g[e], dh, Gh);
+            if (!inr) Gbm += g[e];
+            inr_mask |= inr << e;
+          }
+        }
+        Gh = warp_sum(Gh, lpg);
+        Gbm = warp_sum(Gbm, lpg);
+        if (valid) {
+          if (qs.floored) Gh = 0.f;
+          const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
+          if ((lane & (lpg - 1)) == 0 && a.lwc) {
+            float dg = GaM * M * ga * (1.f - ga), db = Gbt * m * gb * (1.f - gb);
+            if (a.accumulate) { a.dgl[k] += dg; a.dbl[k] += db; } else { a.dgl[k] = dg; a.dbl[k] = db; }
+          }
+          float dwt[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            int64_t col = c * 8 + e;
+            float d = ((inr_mask >> e) & 1) ? g[e] : 0.f;
+            if (col == iM) d += GaM * ga;
+            if (col == im) d += Gbt * gb;
+            dwt[e] = d;
+            float sv = a.s ? a.s[col] : 1.f;
+            dr_part = fmaf(d * w[e], sv, dr_part);
+            if (want_s) acc_s[col] = fmaf(d * w[e], rr, acc_s[col]);
+            if (want_d) acc_d[col] = fmaf(dBo * rr, w[e], acc_d[col]);
+          }
+          if (a.dWt) {
+            float4* dst = reinterpret_cast<float4*>(a.dWt + o * a.Cin) + 2 * c;
+            dst[0] = make_float4(dwt[0], dwt[1], dwt[2], dwt[3]);
+            dst[1] = make_float4(dwt[4], dwt[5], dwt[6], dwt[7]);
+          }
+        }
+      }
+    }
+    if (a.dr) {
+      float2 t = block_sum2(dr_part, 0.f, red_f);
+      if (tid == 0) { if (a.accumulate_dr) a.dr[o] += t.x; else a.dr[o] = t.x; }
+    }
+  }
+  if (want_s || want_d) {
+    __syncthreads();
+    for (int64_t c = tid; c < a.Cin; c += nt) {
+      if (want_s) a.part_s[(int64_t)blockIdx.x * a.Cin + c] = acc_s[c];
+      if (want_d) a.part_d[(int64_t)blockIdx.x * a.Cin + c] = acc_d[c];
+    }
+  }
+}
+
+int64_t lwc_bwd_nslab(int64_t Cout) {
+  int64_t rows = 16;
+  return (Cout + rows - 1) / rows;
+}
+
+omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a0, int64_t* nslab_out) {
+  OMQ_REQUIRE(lwc_group_ok(a0.Cin, a0.group), OMQ_ERR_UNSUPPORTED);
+  LwcBwdArgs a = a0;
+  a.rows_per_cta = 16;
+  int64_t nslab = lwc_bwd_nslab(a.Cout);
+  size_t smem = (a.part_s || a.part_d) ? 2 * a.Cin * sizeof(float) : 0;
+  OMQ_REQUIRE(smem <= 200 * 1024, OMQ_ERR_UNSUPPORTED);
+  if (smem > 48 * 1024) cudaFuncSetAttribute(lwc_bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  lwc_bwd_kernel<<<(unsigned)nslab, lwc_threads(a.Cin), smem, st>>>(a);
+  OMQ_LAUNCH_CHECK();
+  if (nslab_out) *nslab_out = nslab;
+  return OMQ_OK;
+}
+
+// ================================================================================================
+// per-token activation quantizer: one CTA per token row, row staged in shared memory.
+// ================================================================================================
+__device__ __forceinline__ float silu_f(float g) { return g / (1.f + expf(-g)); }
+
+template <int P>
+__device__ __forceinline__ void act_produce_row(const ActFwdArgs& a, int64_t t, float* row, float* red_f,
+                                                float* rstd_out) {
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int64_t C = a.C;
+  const float* xr = a.X + t * a.ldx;
+  if (P == AP_RMS_LET) {
+    float ss = 0.f;
+    for (int64_t i = tid; i < C / 4; i += nt) {
+      float4 v = __ldg(reinterpret_cast<const float4*>(xr) + i);
+      reinterpret_cast<float4*>(row)[i] = v;
+      ss = fmaf(v.x, v.x, ss); ss = fmaf(v.y, v.y, ss); ss = fmaf(v.z, v.z, ss); ss = fmaf(v.w, v.w, ss);
+    }
+    float2 tot = block_sum2(ss, 0.f, red_f);
+    float rstd = 1.0f / sqrtf(tot.x / (float)C + a.rms_eps);
+    *rstd_out = rstd;
+    for (int64_t i = tid; i < C; i += nt) {
+      float v = row[i] * rstd;
+      if (a.delta) v = v - a.delta[i];
+      if (a.s) v = __fdiv_rn(v, a.s[i]);
+      row[i] = v;
+    }
+  } else if (P == AP_SWIGLU) {
+    const float* ur = a.U + t * a.ldu;
+    for (int64_t i = tid; i < C / 4; i += nt) {
+      float4 g = __ldg(reinterpret_cast<const float4*>(xr) + i);
+      float4 u = __ldg(reinterpret_cast<const float4*>(ur) + i);
+      reinterpret_cast<float4*>(row)[i] = make_float4(silu_f(g.x) * u.x, silu_f(g.y) * u.y, silu_f(g.z) * u.z, silu_f(g.w) * u.w);
+    }
+  } else {
+    for (int64_t i = tid; i < C / 4; i += nt) {
+      float4 v = __ldg(reinterpret_cast<const float4*>(xr) + i);
+      if (P == AP_LET) {
+        float vv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          int64_t c = 4 * i + e;
+          if (a.delta) vv[e] = vv[e] - a.delta[c];
+          if (a.s) vv[e] = __fdiv_rn(vv[e], a.s[c]);
+        }
+        v = make_float4(vv[0], vv[1], vv[2], vv[3]);
+      }
+      reinterpret_cast<float4*>(row)[i] = v;
+    }
+  }
+  __syncthreads();
+}
+
+template <int P>
+__global__ void __launch_bounds__(ACT_THREADS) act_fwd_kernel(ActFwdArgs a) {
+  extern __shared__ float row[];
+  __shared__ float red_f[64];
+  __shared__ MaxMin red_mm[32];
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int64_t t = blockIdx.x;
+  const int64_t C = a.C;
+  float rstd = 0.f;
+  act_produce_row<P>(a, t, row, red_f, &rstd);
+  if (P == AP_RMS_LET && tid == 0 && a.rstd) a.rstd[t] = rstd;
+  __nv_bfloat16* qr = a.Xq + t * a.ldq;
+  if (a.abits >= 16) {
+    for (int64_t i = tid; i < C / 2; i += nt) {
+      float2 v = reinterpret_cast<float2*>(row)[i];
+      reinterpret_cast<__nv_bfloat162*>(qr)[i] = __floats2bfloat162_rn(v.x, v.y);
+    }
+    return;
+  }
+  MaxMin r = mm_identity();
+  for (int64_t i = tid; i < C; i += nt) mm_push(r, row[i], (int)i);
+  r = mm_block_reduce(r, red_mm);
+  const float Q = (float)((1 << a.abits) - 1);
+  QState qs = omq_qstate(r.M, r.m, 1.f, 1.f, Q, a.eps);
+  if (tid == 0) { a.h[t] = qs.h; a.z[t] = (int32_t)qs.z; a.imax[t] = r.iM; a.imin[t] = r.im; }
+  for (int64_t i = tid; i < C / 2; i += nt) {
+    float2 v = reinterpret_cast<float2*>(row)[i];
+    float c0, c1;
+    float q0 = omq_fakequant(v.x, qs, Q, &c0);
+    float q1 = omq_fakequant(v.y, qs, Q, &c1);
+    reinterpret_cast<__nv_bfloat162*>(qr)[i] = __floats2bfloat162_rn(q0, q1);
+    if (a.codes) {
+      uint8_t* cr = a.codes + t * C;
+      cr[2 * i] = (uint8_t)c0; cr[2 * i + 1] = (uint8_t)c1;
+    }
+  }
+}
+
+omq_status act_fwd_launch(cudaStream_t st, const ActFwdArgs& a) {
+  OMQ_REQUIRE(a.C % 8 == 0 && a.T > 0, OMQ_ERR_SHAPE);
+  size_t smem = a.C * sizeof(float);
+  OMQ_REQUIRE(smem <= 200 * 1024, OMQ_ERR_UNSUPPORTED);
+  void (*k)(ActFwdArgs) = nullptr;
+  switch (a.producer) {
+    case AP_PLAIN: k = act_fwd_kernel<AP_PLAIN>; break;
+    case AP_LET: k = act_fwd_kernel<AP_LET>; break;
+    case AP_RMS_LET: k = act_fwd_kernel<AP_RMS_LET>; break;
+    case AP_SWIGLU: k = act_fwd_kernel<AP_SWIGLU>; break;
+    default: return OMQ_ERR_INVALID_ARG;
+  }
+  if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  k<<<(unsigned)a.T, ACT_THREADS, smem, st>>>(a);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+// ---- backward ----------------------------------------------------------------------------------
+template <int P>
+__global__ void __launch_bounds__(ACT_THREADS) act_bwd_kernel(ActBwdArgs a) {
+  extern __shared__ float smem[];
+  float* row = smem;                      // quantizer input X~ of the current token
+  float* dv = smem + a.C;                 // dL/dX~ of the current token
+  float* acc_s = smem + 2 * a.C;          // LET column partial sums of this CTA
+  float* acc_d = smem + 3 * a.C;
+  __shared__ float red_f[64];
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int64_t C = a.C;
+  const bool let_sums = a.part_s != nullptr;
+  if (let_sums)
+    for (int64_t i = tid; i < C; i += nt) { acc_s[i] = 0.f; acc_d[i] = 0.f; }
+  const int64_t t0 = (int64_t)blockIdx.x * a.rows_per_cta;
+  const int64_t t1 = min(a.T, t0 + a.rows_per_cta);
+  const float Q = (float)((1 << (a.abits >= 16 ? 1 : a.abits)) - 1);
+
+  ActFwdArgs f;
+  f.producer = P; f.X = a.X; f.ldx = a.ldx; f.U = a.U; f.ldu = a.ldu; f.s = a.s; f.delta = a.delta;
+  f.rms_eps = 0.f; f.C = a.C;
+
+  for (int64_t t = t0; t < t1; ++t) {
+    // recompute X~ exactly as the forward did (RMS uses the saved rstd)
+    const float* xr = a.X + t * a.ldx;
+    if (P == AP_RMS_LET) {
+      const float rstd = a.rstd[t];
+      for (int64_t i = tid; i < C; i += nt) {
+        float v = xr[i] * rstd;
+        if (a.delta) v = v - a.delta[i];
+        if (a.s) v = __fdiv_rn(v, a.s[i]);
+        row[i] = v;
+      }
+      __syncthreads();
+    } else {
+      float dummy;
+      act_produce_row<P>(f, t, row, red_f, &dummy);
+    }
+    const float* gr = a.dXq + t * a.lddq;
+    if (a.abits >= 16) {
+      for (int64_t i = tid; i < C; i += nt) dv[i] = gr[i];
+    } else {
+      QState qs;
+      const int iM = a.imax[t], im = a.imin[t];
+      const float M = row[iM], m = row[im];
+      qs = omq_qstate(M, m, 1.f, 1.f, Q, a.eps);
+      qs.h = a.h[t]; qs.z = (float)a.z[t]; qs.u = __fdiv_rn(m, qs.h);
+      float Gh = 0.f, Gbm = 0.f;
+      for (int64_t i = tid; i < C; i += nt) {
+        int inr;
+        float g = gr[i];
+        float dh = omq_ste_dh(row[i], qs, Q, &inr);
+        Gh = fmaf(g, dh, Gh);
+        if (!inr) Gbm += g;
+        dv[i] = inr ? g : 0.f;
+      }
+      float2 tot = block_sum2(Gh, Gbm, red_f);
+      Gh = qs.floored ? 0.f : tot.x;
+      Gbm = tot.y;
+      const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
+      if (tid == 0) { dv[iM] += GaM; dv[im] += Gbt; }
+    }
+    __syncthreads();
+    // producer backward
+    if (P == AP_PLAIN || P == AP_LET) {
+      for (int64_t i = tid; i < C; i += nt) {
+        float d = dv[i];
+        float sv = a.s ? a.s[i] : 1.f;
+        if (let_sums) { acc_s[i] -= d * row[i] / sv; acc_d[i] -= d / sv; }
+        float dx = a.s ? __fdiv_rn(d, sv) : d;
+        if (a.dX) a.dX[t * a.lddx + i] = dx;
+        if (a.dXb) a.dXb[t * a.lddxb + i] = f_to_bf16(dx);
+      }
+    } else if (P == AP_SWIGLU) {
+      const float* ur = a.U + t * a.ldu;
+      for (int64_t i = tid; i < C; i += nt) {
+        float d = dv[i];
+        float g = xr[i], u = ur[i];
+        float sg = 1.f / (1.f + expf(-g));
+        float dg = d * u * sg * (1.f + g * (1.f - sg));
+        float du = d * g * sg;
+        if (a.dX) { a.dX[t * a.lddx + i] = dg; a.dU[t * a.lddx + i] = du; }
+        if (a.dXb) { a.dXb[t * a.lddxb + i] = f_to_bf16(dg); a.dUb[t * a.lddxb + i] = f_to_bf16(du); }
+      }
+    } else {  // AP_RMS_LET: dX~ -> LET sums -> d(norm output) -> RMSNorm backward
+      const float rstd = a.rstd[t];
+      float dot = 0.f;
+      for (int64_t i = tid; i < C; i += nt) {
+        float d = dv[i];
+        float sv = a.s ? a.s[i] : 1.f;
+        if (let_sums) { acc_s[i] -= d * row[i] / sv; acc_d[i] -= d / sv; }
+        float dn = a.s ? __fdiv_rn(d, sv) : d;     // dL/d(RMSNorm output)
+        dv[i] = dn;
+        dot = fmaf(dn, xr[i] * rstd, dot);
+      }
+      float2 tot = block_sum2(dot, 0.f, red_f);
+      const float mean_dot = tot.x / (float)C;
+      if (a.dX || a.dXb) {
+        for (int64_t i = tid; i < C; i += nt) {
+          float an = xr[i] * rstd;
+          float dx = rstd * (dv[i] - an * mean_dot);
+          if (a.resid) dx += a.resid[t * a.lddx + i];
+          if (a.dX) a.dX[t * a.lddx + i] = dx;
+          if (a.dXb) a.dXb[t * a.lddxb + i] = f_to_bf16(dx);
+        }
+      }
+    }
+    __syncthreads();
+  }
+  if (let_sums) {
+    for (int64_t i = tid; i < C; i += nt) {
+      a.part_s[(int64_t)blockIdx.x * C + i] = acc_s[i];
+      a.part_d[(int64_t)blockIdx.x * C + i] = acc_d[i];
+    }
+  }
+}
+
+omq_status act_bwd_launch(cudaStream_t st, const ActBwdArgs& a0) {
+  ActBwdArgs a = a0;
+  OMQ_REQUIRE(a.C % 8 == 0 && a.T > 0, OMQ_ERR_SHAPE);
+  if (a.rows_per_cta <= 0) a.rows_per_cta = 4;
+  size_t smem = 4 * a.C * sizeof(float);
+  OMQ_REQUIRE(smem <= 200 * 1024, OMQ_ERR_UNSUPPORTED);
+  void (*k)(ActBwdArgs) = nullptr;
+  switch (a.producer) {
+    case AP_PLAIN: k = act_bwd_kernel<AP_PLAIN>; break;
+    case AP_LET: k = act_bwd_kernel<AP_LET>; break;
+    case AP_RMS_LET: k = act_bwd_kernel<AP_RMS_LET>; break;
+    case AP_SWIGLU: k = act_bwd_kernel<AP_SWIGLU>; break;
+    default: return OMQ_ERR_INVALID_ARG;
+  }
+  if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  unsigned grid = (unsigned)((a.T + a.rows_per_cta - 1) / a.rows_per_cta);
+  k<<<grid, ACT_THREADS, smem, st>>>(a);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+// ================================================================================================
+// reductions, loss, small vector kernels
+// ================================================================================================
+__global__ void omq_colsum_partials_kernel(const float* __restrict__ part, int64_t P, int64_t C,
+                                           float* __restrict__ out, float scale, int accumulate) {
+  int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= C) return;
+  float s = 0.f;
+  for (int64_t p = 0; p < P; ++p) s += part[p * C + c];
+  s *= scale;
+  out[c] = accumulate ? out[c] + s : s;
+}
+
+omq_status omq_colsum_partials(cudaStream_t st, const float* part, int64_t P, int64_t C, float* out,
+                               float scale, int accumulate) {
+  omq_colsum_partials_kernel<<<(unsigned)((C + 255) / 256), 256, 0, st>>>(part, P, C, out, scale, accumulate);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+// stage 1 of a column sum over rows: part[blockIdx.y, n] = sum of X[t, n] over 128 rows
+__global__ void colsum_rows_kernel(const float* __restrict__ X, int64_t T, int64_t N, int64_t ldx,
+                                   float* __restrict__ part) {
+  int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (n >= N) return;
+  int64_t t0 = (int64_t)blockIdx.y * 128, t1 = min(T, t0 + 128);
+  float s = 0.f;
+  for (int64_t t = t0; t < t1; ++t) s += X[t * ldx + n];
+  part[(int64_t)blockIdx.y * N + n] = s;
+}
+
+int64_t colsum_rows_parts(int64_t T) { return (T + 127) / 128; }
+
+omq_status colsum_rows(cudaStream_t st, const float* X, int64_t T, int64_t N, int64_t ldx, float* part,
+                       float* out, float scale, int accumulate) {
+  dim3 grid((unsigned)((N + 255) / 256), (unsigned)colsum_rows_parts(T));
+  colsum_rows_kernel<<<grid, 256, 0, st>>>(X, T, N, ldx, part);
+  OMQ_LAUNCH_CHECK();
+  return omq_colsum_partials(st, part, colsum_rows_parts(T), N, out, scale, accumulate);
+}
+
+__global__ void loss_partial_kernel(int64_t n, const float* __restrict__ Yq, const float* __restrict__ Yfp,
+                                    float* __restrict__ dY, __nv_bfloat16* __restrict__ dYb,
+                                    float* __restrict__ part) {
+  __shared__ float red_f[64];
+  float s = 0.f;
+  const float g = 2.0f / (float)n;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    float d = Yq[i] - Yfp[i];
+    s = fmaf(d, d, s);
+    float gd = g * d;
+    if (dY) dY[i] = gd;
+    if (dYb) dYb[i] = f_to_bf16(gd);
+  }
+  float2 t = block_sum2(s, 0.f, red_f);
+  if (threadIdx.x == 0) part[blockIdx.x] = t.x;
+}
+
+__global__ void loss_final_kernel(const float* __restrict__ part, int P, int64_t n, float* loss) {
+  __shared__ float red_f[64];
+  float s = 0.f;
+  for (int i = threadIdx.x; i < P; i += blockDim.x) s += part[i];
+  float2 t = block_sum2(s, 0.f, red_f);
+  if (threadIdx.x == 0) *loss = t.x / (float)n;
+}
+
+int64_t loss_parts(int64_t n) {
+  int64_t b = (n + 1023) / 1024;
+  return b < 1024 ? b : 1024;
+}
+
+omq_status loss_launch(cudaStream_t st, int64_t n, const float* Yq, const float* Yfp, float* loss,
+                       float* dY, __nv_bfloat16* dYb, float* part) {
+  int P = (int)loss_parts(n);
+  loss_partial_kernel<<<P, 256, 0, st>>>(n, Yq, Yfp, dY, dYb, part);
+  OMQ_LAUNCH_CHECK();
+  loss_final_kernel<<<1, 256, 0, st>>>(part, P, n, loss);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+__global__ void vec_fill_kernel(float* p, int64_t n, float v) {
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) p[i] = v;
+}
+omq_status vec_fill(cudaStream_t st, float* p, int64_t n, float v) {
+  vec_fill_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(p, n, v);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+__global__ void vec_copy_kernel(float* d, const float* s, int64_t n) {
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) d[i] = s[i];
+}
+omq_status vec_copy(cudaStream_t st, float* dst, const float* src, int64_t n) {
+  vec_copy_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(dst, src, n);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+__global__ void gqa_expand_kernel(const float* src, float* dst, int n_kv, int rep, int hd, int op) {
+  int i = blockIdx.x * blockDim.x + threadIdx.x;
+  int n = n_kv * rep * hd;
+  if (i >= n) return;
+  int h = i / hd, j = i % hd;
+  float v = src[(h / rep) * hd + j];
+  dst[i] = op == 1 ? 1.0f / v : v;
+}
+omq_status gqa_expand(cudaStream_t st, const float* src, float* dst, int n_kv, int rep, int hd, int op) {
+  int n = n_kv * rep * hd;
+  gqa_expand_kernel<<<(n + 255) / 256, 256, 0, st>>>(src, dst, n_kv, rep, hd, op);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+__global__ void gqa_fold_kernel(const float* src, float* dst, int n_kv, int rep, int hd, int accumulate) {
+  int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= n_kv * hd) return;
+  int kv = c / hd, j = c % hd;
+  float s = 0.f;
+  for (int r = 0; r < rep; ++r) s += src[(kv * rep + r) * hd + j];
+  dst[c] = accumulate ? dst[c] + s : s;
+}
+omq_status gqa_fold(cudaStream_t st, const float* src, float* dst, int n_kv, int rep, int hd, int accumulate) {
+  int n = n_kv * hd;
+  gqa_fold_kernel<<<(n + 255) / 256, 256, 0, st>>>(src, dst, n_kv, rep, hd, accumulate);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+// ================================================================================================
+// LET apply (Eq. 3) as a standalone operation
+// ================================================================================================
+__global__ void let_x_kernel(const float* X, int64_t T, int64_t C, const float* s, const float* d, float* Xt) {
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= T * C) return;
+  int64_t c = i % C;
+  Xt[i] = __fdiv_rn(X[i] - d[c], s[c]);
+}
+
+__global__ void let_w_kernel(const __nv_bfloat16* W, int64_t Cout, int64_t Cin, const float* s, float* Wt) {
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= Cout * Cin) return;
+  Wt[i] = __fmul_rn(bf16_to_f(W[i]), s[i % Cin]);
+}
+
+__global__ void let_b_kernel(const __nv_bfloat16* W, int64_t Cout, int64_t Cin, const float* B, const float* d, float* Bt) {
+  __shared__ float red_f[64];
+  int64_t o = blockIdx.x;
+  float acc = 0.f;
+  for (int64_t i = threadIdx.x; i < Cin; i += blockDim.x) acc = fmaf(bf16_to_f(W[o * Cin + i]), d[i], acc);
+  float2 t = block_sum2(acc, 0.f, red_f);
+  if (threadIdx.x == 0) Bt[o] = (B ? B[o] : 0.f) + t.x;
+}
+
+// ================================================================================================
+// AdamW (Sec. 4.1, weight decay 0 by default)
+// ================================================================================================
+__global__ void adamw_kernel(int64_t n, float* p, const float* g, float* m, float* v, float lr, float b1, float b2,
+                             float eps, float wd, float bc1, float bc2) {
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  float gi = g[i];
+  float mi = b1 * m[i] + (1.f - b1) * gi;
+  float vi = b2 * v[i] + (1.f - b2) * gi * gi;
+  m[i] = mi;
+  v[i] = vi;
+  float pi = p[i];
+  p[i] = pi - lr * (mi / bc1) / (sqrtf(vi / bc2) + eps) - lr * wd * pi;
+}
+
+// ================================================================================================
+// C ABI: kernel-level entry points
+// ================================================================================================
+extern "C" {
+
+omq_status omq_let_apply(omq_stream_t stream, int64_t T, int64_t Cin, int64_t Cout, const float* X,
+                         const void* W, const float* B, const float* s, const float* delta, float* Xt,
+                         float* Wt, float* Bt, const omq_qcfg* cfg) {
+  (void)cfg;
+  cudaStream_t st = (cudaStream_t)stream;
+  OMQ_REQUIRE(T > 0 && Cin > 0 && Cout > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(s && delta, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(Cin % 8 == 0, OMQ_ERR_ALIGN);
+  if (Xt) {
+    OMQ_REQUIRE(X, OMQ_ERR_INVALID_ARG);
+    let_x_kernel<<<(unsigned)((T * Cin + 255) / 256), 256, 0, st>>>(X, T, Cin, s, delta, Xt);
+    OMQ_LAUNCH_CHECK();
+  }
+  if (Wt) {
+    OMQ_REQUIRE(W, OMQ_ERR_INVALID_ARG);
+    let_w_kernel<<<(unsigned)((Cout * Cin + 255) / 256), 256, 0, st>>>((const __nv_bfloat16*)W, Cout, Cin, s, Wt);
+    OMQ_LAUNCH_CHECK();
+  }
+  if (Bt) {
+    OMQ_REQUIRE(W, OMQ_ERR_INVALID_ARG);
+    let_b_kernel<<<(unsigned)Cout, 256, 0, st>>>((const __nv_bfloat16*)W, Cout, Cin, B, delta, Bt);
+    OMQ_LAUNCH_CHECK();
+  }
+  return OMQ_OK;
+}
+
+omq_status omq_lwc_fakequant_fwd(omq_stream_t stream, int64_t Cout, int64_t Cin, const void* W, const float* s,
+                                 const float* r, const float* gamma_logit, const float* beta_logit, void* Wq,
+                                 uint8_t* codes, float* h, int32_t* z, int32_t* argmax, int32_t* argmin,
+                                 const float* bias_delta, const float* bias_shift, float* Bt, const omq_qcfg* cfg) {
+  OMQ_TRY(omq_check_cfg(cfg));
+  OMQ_REQUIRE(Cout > 0 && Cin > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(W, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(Cin % 8 == 0 && omq_aligned16(W) && (!Wq || omq_aligned16(Wq)), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(!codes || ((uintptr_t)codes & 7) == 0, OMQ_ERR_ALIGN);
+  const int g = cfg->group == 0 ? (int)Cin : cfg->group;
+  OMQ_REQUIRE(Cin % g == 0, OMQ_ERR_SHAPE);
+  if (cfg->wbits < 16) OMQ_REQUIRE(h && z && argmax && argmin && gamma_logit && beta_logit, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(!Bt || bias_delta, OMQ_ERR_INVALID_ARG);
+  LwcFwdArgs a{};
+  a.W = (const __nv_bfloat16*)W; a.Cout = Cout; a.Cin = Cin; a.group = g;
+  a.s = s; a.r = r; a.gl = gamma_logit; a.bl = beta_logit; a.lwc = 1;
+  a.Wq = (__nv_bfloat16*)Wq; a.codes = codes; a.h = h; a.z = z; a.imax = argmax; a.imin = argmin;
+  a.bias_delta = bias_delta; a.bias_shift = bias_shift; a.Bt = Bt;
+  a.wbits = cfg->wbits; a.eps = cfg->h_eps; a.status = cfg->dev_status;
+  return lwc_fwd_launch((cudaStream_t)stream, a);
+}
+
+size_t omq_lwc_bwd_workspace_size(int64_t Cout, int64_t Cin) {
+  return (size_t)(2 * lwc_bwd_nslab(Cout) * Cin) * sizeof(float) + 256;
+}
+
+omq_status omq_lwc_fakequant_bwd(omq_stream_t stream, int64_t Cout, int64_t Cin, const void* W, const float* s,
+                                 const float* r, const float* gamma_logit, const float* beta_logit, const float* h,
+                                 const int32_t* z, const int32_t* argmax, const int32_t* argmin, const float* dWq,
+                                 float* dgamma, float* dbeta, float* dWt, float* ds, float* dr, const float* dBt,
+                                 float* ddelta, void* workspace, size_t ws_bytes, const omq_qcfg* cfg) {
+  OMQ_TRY(omq_check_cfg(cfg));
+  OMQ_REQUIRE(Cout > 0 && Cin > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(cfg->wbits < 16, OMQ_ERR_UNSUPPORTED);
+  OMQ_REQUIRE(W && dWq && h && z && argmax && argmin && gamma_logit && beta_logit && dgamma && dbeta, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(Cin % 8 == 0 && omq_aligned16(W) && omq_aligned16(dWq) && (!dWt || omq_aligned16(dWt)), OMQ_ERR_ALIGN);
+  const int g = cfg->group == 0 ? (int)Cin : cfg->group;
+  OMQ_REQUIRE(Cin % g == 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(!ddelta || dBt, OMQ_ERR_INVALID_ARG);
+  const bool need_ws = ds || ddelta;
+  if (need_ws) {
+    OMQ_REQUIRE(workspace && ws_bytes >= omq_lwc_bwd_workspace_size(Cout, Cin), OMQ_ERR_WORKSPACE);
+    OMQ_REQUIRE(omq_aligned16(workspace), OMQ_ERR_ALIGN);
+  }
+  cudaStream_t st = (cudaStream_t)stream;
+  const int64_t nslab = lwc_bwd_nslab(Cout);
+  float* part_s = need_ws ? (float*)workspace : nullptr;
+  float* part_d = need_ws ? (float*)workspace + nslab * Cin : nullptr;
+  LwcBwdArgs a{};
+  a.W = (const __nv_bfloat16*)W; a.Cout = Cout; a.Cin = Cin; a.group = g; a.s = s; a.r = r;
+  a.gl = gamma_logit; a.bl = beta_logit; a.lwc = 1; a.h = h; a.z = z; a.imax = argmax; a.imin = argmin;
+  a.dWq = dWq; a.ld_dwq = Cin; a.dgl = dgamma; a.dbl = dbeta; a.dWt = dWt; a.dr = dr; a.dBt = dBt;
+  a.part_s = ds ? part_s : nullptr; a.part_d = ddelta ? part_d : nullptr;
+  a.wbits = cfg->wbits; a.eps = cfg->h_eps; a.accumulate = cfg->accumulate; a.accumulate_dr = cfg->accumulate;
+  int64_t ns = 0;
+  OMQ_TRY(lwc_bwd_launch(st, a, &ns));
+  if (ds) OMQ_TRY(omq_colsum_partials(st, part_s, ns, Cin, ds, 1.f, cfg->accumulate));
+  if (ddelta) OMQ_TRY(omq_colsum_partials(st, part_d, ns, Cin, ddelta, 1.f, cfg->accumulate));
+  return OMQ_OK;
+}
+
+omq_status omq_act_quant_per_token(omq_stream_t stream, int64_t T, int64_t C, const float* X, const float* s,
+                                   const float* delta, void* Xq, uint8_t* codes, float* h, int32_t* z,
+                                   int32_t* argmax, int32_t* argmin, const omq_qcfg* cfg) {
+  OMQ_TRY(omq_check_cfg(cfg));
+  OMQ_REQUIRE(T > 0 && C > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(X && Xq, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(C % 8 == 0 && omq_aligned16(X) && omq_aligned16(Xq), OMQ_ERR_ALIGN);
+  if (cfg->abits < 16) OMQ_REQUIRE(h && z && argmax && argmin, OMQ_ERR_INVALID_ARG);
+  ActFwdArgs a{};
+  a.producer = (s || delta) ? AP_LET : AP_PLAIN;
+  a.X = X; a.ldx = C; a.s = s; a.delta = delta; a.T = T; a.C = C;
+  a.Xq = (__nv_bfloat16*)Xq; a.ldq = C; a.codes = codes; a.h = h; a.z = z; a.imax = argmax; a.imin = argmin;
+  a.abits = cfg->abits; a.eps = cfg->h_eps;
+  return act_fwd_launch((cudaStream_t)stream, a);
+}
+
+size_t omq_act_bwd_workspace_size(int64_t T, int64_t C) {
+  return (size_t)(2 * ((T + 3) / 4) * C) * sizeof(float) + 256;
+}
+
+omq_status omq_act_quant_per_token_bwd(omq_stream_t stream, int64_t T, int64_t C, const float* X, const float* s,
+                                       const float* delta, const float* h, const int32_t* z, const int32_t* argmax,
+                                       const int32_t* argmin, const float* dXq, float* dX, float* ds, float* ddelta,
+                                       void* workspace, size_t ws_bytes, const omq_qcfg* cfg) {
+  OMQ_TRY(omq_check_cfg(cfg));
+  OMQ_REQUIRE(T > 0 && C > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(X && dXq, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(C % 8 == 0 && omq_aligned16(X) && omq_aligned16(dXq), OMQ_ERR_ALIGN);
+  if (cfg->abits < 16) OMQ_REQUIRE(h && z && argmax && argmin, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE((!ds && !ddelta) || (s && delta), OMQ_ERR_INVALID_ARG);
+  const bool need_ws = ds || ddelta;
+  const int64_t P = (T + 3) / 4;
+  if (need_ws) OMQ_REQUIRE(workspace && ws_bytes >= omq_act_bwd_workspace_size(T, C), OMQ_ERR_WORKSPACE);
+  cudaStream_t st = (cudaStream_t)stream;
+  ActBwdArgs a{};
+  a.producer = (s || delta) ? AP_LET : AP_PLAIN;
+  a.X = X; a.ldx = C; a.s = s; a.delta = delta; a.T = T; a.C = C;
+  a.h = h; a.z = z; a.imax = argmax; a.imin = argmin; a.dXq = dXq; a.lddq = C;
+  a.dX = dX; a.lddx = C; a.rows_per_cta = 4;
+  a.part_s = need_ws ? (float*)workspace : nullptr;
+  a.part_d = need_ws ? (float*)workspace + P * C : nullptr;
+  a.abits = cfg->abits; a.eps = cfg->h_eps;
+  OMQ_TRY(act_bwd_launch(st, a));
+  if (ds) OMQ_TRY(omq_colsum_partials(st, a.part_s, P, C, ds, 1.f, cfg->accumulate));
+  if (ddelta) OMQ_TRY(omq_colsum_partials(st, a.part_d, P, C, ddelta, 1.f, cfg->accumulate));
+  return OMQ_OK;
+}
+
+size_t omq_loss_workspace_size(int64_t n) { return (size_t)loss_parts(n) * sizeof(float) + 256; }
+
+omq_status omq_block_loss(omq_stream_t stream, int64_t n, const float* Yq, const float* Yfp, float* loss, float* dY,
+                          void* dY_bf16, void* workspace, size_t ws_bytes) {
+  OMQ_REQUIRE(n > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(Yq && Yfp && loss, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(workspace && ws_bytes >= omq_loss_workspace_size(n), OMQ_ERR_WORKSPACE);
+  return loss_launch((cudaStream_t)stream, n, Yq, Yfp, loss, dY, (__nv_bfloat16*)dY_bf16, (float*)workspace);
+}
+
+omq_status omq_adamw_update(omq_stream_t stream, int64_t n, float* p, const float* g, float* m, float* v, float lr,
+                            float beta1, float beta2, float eps, float weight_decay, int32_t step) {
+  OMQ_REQUIRE(n > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(p && g && m && v && step >= 1, OMQ_ERR_INVALID_ARG);
+  float bc1 = 1.f - powf(beta1, (float)step), bc2 = 1.f - powf(beta2, (float)step);
+  adamw_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(n, p, g, m, v, lr, beta1, beta2, eps,
+                                                                              weight_decay, bc1, bc2);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+omq_status omq_stream_status(omq_stream_t stream, const int32_t* dev_status, int32_t* host_out) {
+  OMQ_REQUIRE(dev_status && host_out, OMQ_ERR_INVALID_ARG);
+  if (cudaMemcpyAsync(host_out, dev_status, sizeof(int32_t), cudaMemcpyDeviceToHost, (cudaStream_t)stream) != cudaSuccess)
+    return OMQ_ERR_CUDA;
+  if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return OMQ_ERR_CUDA;
+  return OMQ_OK;
+}
+
+const char* omq_status_string(omq_status s) {
+  switch (s) {
+    case OMQ_OK: return "ok";
+    case OMQ_ERR_INVALID_ARG: return "invalid argument";
+    case OMQ_ERR_SHAPE: return "bad shape";
+    case OMQ_ERR_ALIGN: return "misaligned pointer or inner dimension";
+    case OMQ_ERR_UNSUPPORTED: return "unsupported configuration";
+    case OMQ_ERR_CUDA: return "CUDA launch failure";
+    case OMQ_ERR_TIMEOUT: return "device wait timed out";
+    case OMQ_ERR_WORKSPACE: return "workspace too small";
+  }
+  return "unknown status";
+}
+
+int32_t omq_version(void) { return OMQ_VERSION; }
+
+}  // extern "C"

@@ -1,0 +1,86 @@
+// Internal launchers of the HBM-bound kernels (quant.cu), shared with the block step (block.cu).
+#pragma once
+#include "common.cuh"
+
+// ---- LWC (Eq. 2) on W~ = r_o W_oi s_i --------------------------------------------------------
+struct LwcFwdArgs {
+  const __nv_bfloat16* W; int64_t Cout, Cin; int group;   // group = Cin for per-channel
+  const float* s; const float* r;
+  const float* gl; const float* bl;                        // logits [Cout, ngroups]
+  int lwc;                                                 // 0 = gamma = beta = 1 (plain MinMax)
+  __nv_bfloat16* Wq; uint8_t* codes;
+  float* h; int32_t* z; int32_t* imax; int32_t* imin;
+  const float* bias_delta; const float* bias_shift; float* Bt;
+  int wbits; float eps;
+  int32_t* status;
+};
+omq_status lwc_fwd_launch(cudaStream_t st, const LwcFwdArgs& a);
+
+struct LwcBwdArgs {
+  const __nv_bfloat16* W; int64_t Cout, Cin; int group;
+  const float* s; const float* r;
+  const float* gl; const float* bl; int lwc;
+  const float* h; const int32_t* z; const int32_t* imax; const int32_t* imin;
+  const float* dWq; int64_t ld_dwq;
+  float* dgl; float* dbl; float* dWt; float* dr;
+  const float* dBt;
+  float* part_s; float* part_d;          // [nslab, Cin] partial column sums (nullable)
+  int rows_per_cta;
+  int wbits; float eps; int accumulate; int accumulate_dr;
+};
+omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a, int64_t* nslab_out);
+int64_t lwc_bwd_nslab(int64_t Cout);
+
+// ---- per-token activation quantizer Q_a with a fused producer ------------------------------
+enum ActProducer { AP_PLAIN = 0, AP_LET = 1, AP_RMS_LET = 2, AP_SWIGLU = 3 };
+
+struct ActFwdArgs {
+  int producer;
+  const float* X; int64_t ldx;       // PLAIN / LET / RMS input; SWIGLU gate
+  const float* U; int64_t ldu;       // SWIGLU up
+  const float* s; const float* delta;
+  float rms_eps; float* rstd;        // RMS: rstd [T] written
+  int64_t T, C;
+  __nv_bfloat16* Xq; int64_t ldq;
+  uint8_t* codes;
+  float* h; int32_t* z; int32_t* imax; int32_t* imin;
+  int abits; float eps;
+};
+omq_status act_fwd_launch(cudaStream_t st, const ActFwdArgs& a);
+
+struct ActBwdArgs {
+  int producer;
+  const float* X; int64_t ldx;
+  const float* U; int64_t ldu;
+  const float* s; const float* delta;
+  const float* rstd;
+  int64_t T, C;
+  const float* h; const int32_t* z; const int32_t* imax; const int32_t* imin;
+  const float* dXq; int64_t lddq;
+  float* dX; int64_t lddx;           // PLAIN / LET: dL/dX; RMS: dL/d(norm input); SWIGLU: d gate
+  __nv_bfloat16* dXb; int64_t lddxb; // bf16 copy of dX (nullable)
+  float* dU; __nv_bfloat16* dUb;     // SWIGLU: d up (same ld as dX / dXb)
+  const float* resid;                // RMS: residual gradient added to dX (nullable)
+  float* part_s; float* part_d;      // [T / rows_per_cta, C] LET column partials (nullable)
+  int rows_per_cta;
+  int abits; float eps;
+};
+omq_status act_bwd_launch(cudaStream_t st, const ActBwdArgs& a);
+
+// ---- misc ------------------------------------------------------------------------------------
+// out[n] (+)= scale * sum_t X[t, n] (two-stage, deterministic); part: [ceil(T/128), N] scratch
+omq_status colsum_rows(cudaStream_t st, const float* X, int64_t T, int64_t N, int64_t ldx,
+                       float* part, float* out, float scale, int accumulate);
+int64_t colsum_rows_parts(int64_t T);
+
+omq_status loss_launch(cudaStream_t st, int64_t n, const float* Yq, const float* Yfp, float* loss,
+                       float* dY, __nv_bfloat16* dYb, float* part);
+int64_t loss_parts(int64_t n);
+
+// y[i] = f(x...) small vector kernels
+omq_status vec_fill(cudaStream_t st, float* p, int64_t n, float v);
+omq_status vec_copy(cudaStream_t st, float* dst, const float* src, int64_t n);
+// expand a per-KV-channel vector [n_kv*hd] to [n_heads*hd]; op 0: copy, 1: reciprocal
+omq_status gqa_expand(cudaStream_t st, const float* src, float* dst, int n_kv, int rep, int hd, int op);
+// dst[c] (+)= sum over the rep query heads of src[h*hd + j] for c = kv*hd + j
+omq_status gqa_fold(cudaStream_t st, const float* src, float* dst, int n_kv, int rep, int hd, int accumulate);

@@ -1,0 +1,57 @@
+"""Block-level parity: one calibration step through omq_block_step against the fp64 oracle
+(emulate mode: matmul operands rounded to bf16 as the kernels do).  Output and loss within 1e-2
+relative, every gradient within 3e-2 relative Frobenius error."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2308_13137_gb300 import inputs as I
+from paper_2308_13137_gb300.block import BlockState
+
+pytestmark = pytest.mark.gpu
+OUT_TOL, GRAD_TOL = 1e-2, 3e-2
+
+
+def _rel(a, b):
+    a, b = torch.as_tensor(a).double().cpu(), torch.as_tensor(b).double().cpu()
+    return float((a - b).norm() / b.norm().clamp_min(1e-300))
+
+
+def _run(shape, perturb=True, seed=0):
+    W = I.make_block_weights(shape, seed=seed + 1)
+    x = I.make_block_input(shape, sample=seed, weight_seed=seed + 1)
+    th = I.make_block_theta(shape, W, x, seed=seed + 2, perturb=perturb)
+    cfg = O.BlockCfg.from_shape(shape)
+    yfp = O.block_fp_forward(x, W, cfg).float()
+    ref = O.block_step(x, yfp, W, th, cfg)
+    st = BlockState(shape, W, th)
+    xd, yfd = torch.from_numpy(x).cuda(), yfp.cuda()
+    y = torch.empty_like(xd)
+    st.step(xd, yfd, y)
+    torch.cuda.synchronize()
+    assert int(st.status.item()) == 0
+    return ref, dict(y=y.cpu(), loss=float(st.loss.item()), **st.split_grads())
+
+
+SMALL = [
+    I.BlockShape("w4a4_let", T=256, d=256, n_heads=2, n_kv=2, ffn=512, wbits=4, abits=4, group=0, let=1),
+    I.BlockShape("w4a4_let_gqa", T=256, d=512, n_heads=4, n_kv=2, ffn=768, wbits=4, abits=4, group=0, let=1),
+    I.BlockShape("w3a16_g128", T=256, d=256, n_heads=2, n_kv=2, ffn=512, wbits=3, abits=16, group=128, let=0),
+    I.BlockShape("w2a16_g64", T=384, d=384, n_heads=3, n_kv=3, ffn=640, wbits=2, abits=16, group=64, let=0),
+    I.BlockShape("w4a8_let_ragged", T=200, d=256, n_heads=2, n_kv=1, ffn=520, wbits=4, abits=8, group=0, let=1),
+]
+
+
+@pytest.mark.parametrize("shape", SMALL, ids=[s.name for s in SMALL])
+def test_block_step_small(cuda_lib, shape):
+    ref, got = _run(shape)
+    assert _rel(got["y"], ref["y"]) < OUT_TOL
+    assert abs(got["loss"] - float(ref["loss"])) / float(ref["loss"]) < OUT_TOL
+    names = O.THETA_NAMES_LWC + (O.THETA_NAMES_LET if shape.let else [])
+    bad = {}
+    for n in names:
+        e = _rel(got["d" + n], ref["d" + n])
+        if not e < GRAD_TOL:
+            bad[n] = e
+    assert not bad, bad

@@ -433,3 +433,28 @@ def test_rope_rotation_direction():
     v = torch.tensor([[1.0, 0.0], [1.0, 0.0]], dtype=F64)
     r = O.rope(v, 1, 2, 10000.0)
     assert torch.allclose(r[1], torch.tensor([math.cos(1.0), math.sin(1.0)], dtype=F64), atol=1e-15)
+
+
+def test_fp32_decisions_match_independent_single_precision():
+    """decide="fp32" equals the same Eq. 2 arithmetic written with numpy float32 scalars, and
+    differs from float64 decisions only at elements within a few fp32 ulps of a .5 boundary."""
+    rng = np.random.default_rng(21)
+    w = (rng.standard_normal((40, 64)) * 0.03).astype(np.float32)
+    gl = rng.normal(1.0, 1.0, 40)
+    bl = rng.normal(1.0, 1.0, 40)
+    st = O.quant_fwd(torch.from_numpy(w).double(), O.sigmoid(torch.from_numpy(gl)), O.sigmoid(torch.from_numpy(bl)),
+                     3, decide="fp32")
+    for o in range(40):
+        a = np.float32(1.0 / (1.0 + math.exp(-gl[o])))
+        b = np.float32(1.0 / (1.0 + math.exp(-bl[o])))
+        M, m = np.float32(w[o].max()), np.float32(w[o].min())
+        h = np.float32(np.float32(np.float32(a * M) - np.float32(b * m)) / np.float32(7.0))
+        z = -np.rint(np.float32(np.float32(b * m) / h))
+        codes = np.clip(np.rint(np.float32(w[o] / h)) + z, 0, 7)
+        assert float(st["h"][o]) == float(h) and float(st["z"][o]) == float(z)
+        assert np.array_equal(st["q"][o].numpy(), codes)
+    st64 = O.quant_fwd(torch.from_numpy(w).double(), O.sigmoid(torch.from_numpy(gl)), O.sigmoid(torch.from_numpy(bl)),
+                       3, decide="fp64")
+    differ = (st["q"] != st64["q"])
+    frac = st64["x"] - torch.floor(st64["x"])
+    assert bool(((frac[differ] - 0.5).abs() < 1e-5).all())
