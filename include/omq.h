@@ -257,6 +257,17 @@ const char* omq_status_string(omq_status s);
 /* Library version, for the bindings' sanity check. */
 int32_t omq_version(void);
 
+/* Number of kernel launches the library has enqueued since it was loaded (host-side counter). */
+int64_t omq_launch_count(void);
+
+/* Tracing of the tensor-core matrix products.  After omq_profile_begin, every omq GEMM launch is
+ * bracketed by two CUDA events recorded on its own stream, and its algorithmic flop count (2 per
+ * multiply-add inside the causal domain) is accumulated.  omq_profile_end waits for those events
+ * and returns the summed device time in ms, the flops and the number of launches, then stops
+ * tracing.  Not for use during CUDA-graph capture (it creates events lazily). */
+void omq_profile_begin(void);
+omq_status omq_profile_end(double* gemm_ms, double* gemm_flops, int64_t* gemm_launches);
+
 #ifdef __cplusplus
 }
 #endif

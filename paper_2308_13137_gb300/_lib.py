@@ -79,6 +79,9 @@ _SIGS = {
     "omq_stream_status": (I32, [P, P, POINTER(c_int32)]),
     "omq_status_string": (c_char_p, [I32]),
     "omq_version": (I32, []),
+    "omq_launch_count": (I64, []),
+    "omq_profile_begin": (None, []),
+    "omq_profile_end": (I32, [POINTER(ctypes.c_double), POINTER(ctypes.c_double), POINTER(c_int64)]),
 }
 
 _LIB: Optional[ctypes.CDLL] = None
@@ -88,7 +91,8 @@ def header_functions():
     """Names of the functions include/omq.h declares."""
     with open(HEADER) as fh:
         text = fh.read()
-    return sorted(set(re.findall(r"^\s*(?:omq_status|size_t|int32_t|const char\*)\s+(omq_\w+)\s*\(", text, re.M)))
+    return sorted(set(re.findall(r"^\s*(?:omq_status|size_t|int32_t|int64_t|void|const char\*)\s+(omq_\w+)\s*\(",
+                                 text, re.M)))
 
 
 def lib() -> ctypes.CDLL:
@@ -255,3 +259,18 @@ def omq_status_string(code: int) -> str:
 
 def omq_version() -> int:
     return lib().omq_version()
+
+
+def omq_launch_count() -> int:
+    return lib().omq_launch_count()
+
+
+def omq_profile_begin():
+    lib().omq_profile_begin()
+
+
+def omq_profile_end():
+    """Returns (GEMM device ms, algorithmic GEMM flops, GEMM launches) traced since begin."""
+    ms, fl, n = ctypes.c_double(0), ctypes.c_double(0), c_int64(0)
+    check("omq_profile_end", lib().omq_profile_end(ctypes.byref(ms), ctypes.byref(fl), ctypes.byref(n)))
+    return ms.value, fl.value, n.value

@@ -44,18 +44,36 @@ class BlockState:
             o=dev_bf16(weights["wo"]),
             gu=dev_bf16(np.concatenate([weights["wg"], weights["wu"]], 0)),
             d=dev_bf16(weights["wd"]))
-        self.theta = {}
-        self.grads = {}
+        # learnable parameters live in two flat fp32 buffers (LWC logits | LET vectors) so that one
+        # optimizer launch per learning-rate group updates them; the names below are views
+        host = {}
         if self.wbits < 16:
             for key, parts in LWC_PARTS.items():
                 for gb in ("gamma", "beta"):
-                    v = np.concatenate([theta[f"{gb}_{p}"] for p in parts], 0)
-                    self.theta[f"{gb}_{key}"] = dev_f32(v)
-                    self.grads[f"{gb}_{key}"] = torch.zeros_like(self.theta[f"{gb}_{key}"])
+                    host[f"{gb}_{key}"] = np.concatenate([theta[f"{gb}_{p}"] for p in parts], 0)
+        n_lwc = sum(v.size for v in host.values())
         if self.let:
             for k in LET_NAMES:
-                self.theta[k] = dev_f32(theta[k])
-                self.grads[k] = torch.zeros_like(self.theta[k])
+                host[k] = np.asarray(theta[k])
+        self.theta_flat, self.grads_flat = {}, {}
+        self.theta, self.grads = {}, {}
+        groups = dict(lwc=[k for k in host if k not in LET_NAMES], let=[k for k in host if k in LET_NAMES])
+        for gname, keys in groups.items():
+            if not keys:
+                continue
+            # pad each view to a multiple of 4 floats so every view stays 16-byte aligned
+            sizes = [host[k].size for k in keys]
+            offs = np.cumsum([0] + [(n + 3) // 4 * 4 for n in sizes])
+            flat = torch.zeros(int(offs[-1]), dtype=torch.float32, device=device)
+            gflat = torch.zeros_like(flat)
+            for k, o, n in zip(keys, offs[:-1], sizes):
+                flat[o:o + n] = dev_f32(host[k].reshape(-1))
+                self.theta[k] = flat[o:o + n].view(host[k].shape)
+                self.grads[k] = gflat[o:o + n].view(host[k].shape)
+            self.theta_flat[gname], self.grads_flat[gname] = flat, gflat
+        self.n_lwc = n_lwc
+        self.adam = {g: (torch.zeros_like(f), torch.zeros_like(f)) for g, f in self.theta_flat.items()}
+        self.adam_step = 0
         self.c_shape = _lib.omq_block_shape(shape.T, shape.d, shape.n_heads, shape.n_kv, shape.head_dim, shape.ffn,
                                             shape.rms_eps, shape.rope_theta)
         self.c_w = _lib.omq_block_weights(*[self.W[k].data_ptr() for k in ("qkv", "o", "gu", "d")])
@@ -81,6 +99,14 @@ class BlockState:
         _lib.omq_block_step(self.c_shape, self.c_w, self.c_theta, x, y_fp, y, self.loss, self.c_grads,
                             self.workspace, self.cfg, stream)
         return self.loss
+
+    def adamw(self, lr_lwc: float = 5e-3, lr_let: float = 1e-2, stream=None):
+        """AdamW with zero weight decay on both parameter groups (Sec. 4.1 "Training")."""
+        self.adam_step += 1
+        for g, flat in self.theta_flat.items():
+            m, v = self.adam[g]
+            _lib.omq_adamw_update(flat.numel(), flat, self.grads_flat[g], m, v, lr_lwc if g == "lwc" else lr_let,
+                                  0.9, 0.999, 1e-8, 0.0, self.adam_step, stream)
 
     def forward(self, x, y, stream=None, cfg=None):
         _lib.omq_block_forward(self.c_shape, self.c_w, self.c_theta, x, y, self.workspace, cfg or self.cfg, stream)

@@ -13,7 +13,9 @@
 // host-side argument checks
 // ------------------------------------------------------------------------------------------------
 #define OMQ_REQUIRE(cond, code) do { if (!(cond)) return (code); } while (0)
-#define OMQ_LAUNCH_CHECK() do { if (cudaPeekAtLastError() != cudaSuccess) { cudaGetLastError(); return OMQ_ERR_CUDA; } } while (0)
+// every kernel launch of the library is followed by this check, which also counts it
+void omq_count_launch();
+#define OMQ_LAUNCH_CHECK() do { omq_count_launch(); if (cudaPeekAtLastError() != cudaSuccess) { cudaGetLastError(); return OMQ_ERR_CUDA; } } while (0)
 #define OMQ_TRY(expr) do { omq_status _s = (expr); if (_s != OMQ_OK) return _s; } while (0)
 
 static inline bool omq_aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }

@@ -9,6 +9,7 @@
 // OMQ_ERR_TIMEOUT to the status word, stops issuing work, frees its tensor memory and exits.
 #include "gemm.cuh"
 #include <cuda.h>
+#include <vector>
 
 namespace {
 
@@ -222,7 +223,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int row = m0 + q * 32 + lane;
     bool ok = true;
     if (nkb > 0) {
-      ok = mbar_wait(accum, 0);
+      ok = __all_sync(0xffffffffu, mbar_wait(accum, 0));   // tcgen05.ld below is warp-collective
       if (!ok) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; }
       tc_fence_after();
     }
@@ -352,6 +353,45 @@ omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap&
   return OMQ_OK;
 }
 
+// ---- optional per-launch timing (CUDA events recorded on the launching stream) ----
+struct GemmProfile {
+  bool on = false;
+  std::vector<cudaEvent_t> ev;     // pairs: start, stop
+  size_t used = 0;                 // events in use
+  double flops = 0.0;              // algorithmic flops of the recorded launches
+};
+GemmProfile g_prof;
+
+// multiply-adds of the launch counted once each, times two; causal modes count the triangle only
+double gemm_algorithmic_flops(int64_t M, int64_t N, int64_t K, int64_t batch, int causal) {
+  double mnk;
+  if (causal == 0) {
+    mnk = (double)M * N * K;
+  } else if (causal == 1) {         // keys n <= query m
+    double pairs = 0;
+    for (int64_t m = 0; m < M; ++m) pairs += (double)(m + 1 < N ? m + 1 : N);
+    mnk = pairs * K;
+  } else if (causal == 2) {         // k <= m
+    double s = 0;
+    for (int64_t m = 0; m < M; ++m) s += (double)(m + 1 < K ? m + 1 : K);
+    mnk = s * N;
+  } else {                          // k >= m
+    double s = 0;
+    for (int64_t m = 0; m < M; ++m) s += (double)(K - m > 0 ? K - m : 0);
+    mnk = s * N;
+  }
+  return 2.0 * mnk * batch;
+}
+
+cudaEvent_t prof_event() {
+  if (g_prof.used == g_prof.ev.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    g_prof.ev.push_back(e);
+  }
+  return g_prof.ev[g_prof.used++];
+}
+
 }  // namespace
 
 omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t batch, const GemmOperand& A,
@@ -377,8 +417,40 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
   p.M = (int)M; p.N = (int)N; p.K = (int)K; p.batch = (int)batch;
   p.a_mn = A.kmajor ? 0 : 1; p.b_mn = B.kmajor ? 0 : 1;
   p.causal = causal; p.ep = ep; p.status = status;
-  if (wide) return launch_cfg<256, 4>(st, ta, tb, p);
-  return launch_cfg<128, 6>(st, ta, tb, p);
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  if (g_prof.on) {
+    e0 = prof_event();
+    e1 = prof_event();
+    if (e0 && e1) {
+      cudaEventRecord(e0, st);
+      g_prof.flops += gemm_algorithmic_flops(M, N, K, batch, causal);
+    }
+  }
+  omq_status r = wide ? launch_cfg<256, 4>(st, ta, tb, p) : launch_cfg<128, 6>(st, ta, tb, p);
+  if (e0 && e1) cudaEventRecord(e1, st);
+  return r;
+}
+
+extern "C" void omq_profile_begin(void) {
+  g_prof.on = true;
+  g_prof.used = 0;
+  g_prof.flops = 0.0;
+}
+
+extern "C" omq_status omq_profile_end(double* gemm_ms, double* gemm_flops, int64_t* gemm_launches) {
+  g_prof.on = false;
+  double ms = 0.0;
+  for (size_t i = 0; i + 1 < g_prof.used; i += 2) {
+    if (cudaEventSynchronize(g_prof.ev[i + 1]) != cudaSuccess) return OMQ_ERR_CUDA;
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, g_prof.ev[i], g_prof.ev[i + 1]) != cudaSuccess) return OMQ_ERR_CUDA;
+    ms += t;
+  }
+  if (gemm_ms) *gemm_ms = ms;
+  if (gemm_flops) *gemm_flops = g_prof.flops;
+  if (gemm_launches) *gemm_launches = (int64_t)(g_prof.used / 2);
+  g_prof.used = 0;
+  return OMQ_OK;
 }
 
 extern "C" omq_status omq_gemm_bf16(omq_stream_t stream, int64_t M, int64_t N, int64_t K, int64_t batch, const void* A,

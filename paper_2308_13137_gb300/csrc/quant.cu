@@ -3,7 +3,12 @@
 // SwiGLU) and its straight-through backward, the block loss (Eq. 1), column reductions and AdamW.
 #include "quant.cuh"
 
+#include <atomic>
+
 #define LWC_MAXC 16        // 8-element chunks per thread held in registers (Cin <= 256*8*16)
+
+static std::atomic<long long> g_launches{0};
+void omq_count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 #define ACT_THREADS 256
 
 // ================================================================================================
@@ -976,5 +981,7 @@ const char* omq_status_string(omq_status s) {
 }
 
 int32_t omq_version(void) { return OMQ_VERSION; }
+
+int64_t omq_launch_count(void) { return (int64_t)g_launches.load(); }
 
 }  // extern "C"

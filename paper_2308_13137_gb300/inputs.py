@@ -112,10 +112,10 @@ def bf16_representable(a: np.ndarray) -> np.ndarray:
     Uses round-to-nearest-even on the float32 bit pattern; this is the storage
     format of the frozen weights, not part of the method."""
     a = np.ascontiguousarray(a, dtype=np.float32)
-    u = a.view(np.uint32).astype(np.uint64)
-    lsb = (u >> 16) & 1
-    u = (u + 0x7FFF + lsb) & 0xFFFF0000
-    return u.astype(np.uint32).view(np.float32)
+    u = a.view(np.uint32)
+    lsb = (u >> np.uint32(16)) & np.uint32(1)
+    u = (u + np.uint32(0x7FFF) + lsb) & np.uint32(0xFFFF0000)
+    return u.view(np.float32)
 
 
 def _rng(seed: int) -> np.random.Generator:
@@ -159,7 +159,9 @@ def make_block_weights(shape: BlockShape, seed: int = 1) -> Dict[str, np.ndarray
     d, dq, dkv, f = shape.d, shape.dq, shape.dkv, shape.ffn
 
     def w(cout, cin):
-        return bf16_representable((shape.w_std * rng.standard_normal((cout, cin))).astype(np.float32))
+        v = rng.standard_normal((cout, cin), dtype=np.float32)
+        v *= np.float32(shape.w_std)
+        return bf16_representable(v)
 
     return dict(wq=w(dq, d), wk=w(dkv, d), wv=w(dkv, d), wo=w(d, dq),
                 wg=w(f, d), wu=w(f, d), wd=w(d, f))
@@ -168,7 +170,7 @@ def make_block_weights(shape: BlockShape, seed: int = 1) -> Dict[str, np.ndarray
 def make_block_input(shape: BlockShape, sample: int = 0, weight_seed: int = 1) -> np.ndarray:
     """Block input x [T, d] fp32 for calibration sample `sample`."""
     rng = _rng(1000 + sample)
-    x = rng.standard_normal((shape.T, shape.d)).astype(np.float32)
+    x = rng.standard_normal((shape.T, shape.d), dtype=np.float32)
     ch = _outlier_channels(shape, weight_seed)
     x[:, ch] *= np.float32(shape.outlier_scale)
     return x
