@@ -3,18 +3,27 @@
 // scores, and the small finishers of the [v, out] LET pair gradients.
 #include "attn.cuh"
 
+// angle t * theta^(-2j/hd): the frequency and the product are formed in double, the angle is reduced
+// to [-pi, pi] in double, and sin/cos of the reduced angle are taken in float.
 __global__ void rope_table_kernel(int T, int hd, double theta, float* cs) {
+  __shared__ double inv[128];
   const int half = hd / 2;
-  int i = blockIdx.x * blockDim.x + threadIdx.x;
+  for (int j = threadIdx.x; j < half; j += blockDim.x) inv[j] = pow(theta, -2.0 * (double)j / (double)hd);
+  __syncthreads();
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= T * half) return;
-  int t = i / half, j = i % half;
-  double inv = pow(theta, -2.0 * (double)j / (double)hd);
-  double ang = (double)t * inv;
-  cs[2 * i] = (float)cos(ang);
-  cs[2 * i + 1] = (float)sin(ang);
+  const int t = i / half, j = i % half;
+  const double two_pi = 6.283185307179586476925286766559;
+  double ang = (double)t * inv[j];
+  ang -= two_pi * rint(ang / two_pi);
+  float sv, cv;
+  sincosf((float)ang, &sv, &cv);
+  cs[2 * i] = cv;
+  cs[2 * i + 1] = sv;
 }
 
 omq_status rope_table(cudaStream_t st, int T, int hd, float theta, float* cs) {
+  OMQ_REQUIRE(hd <= 256, OMQ_ERR_UNSUPPORTED);
   int n = T * (hd / 2);
   rope_table_kernel<<<(n + 255) / 256, 256, 0, st>>>(T, hd, (double)theta, cs);
   OMQ_LAUNCH_CHECK();
@@ -44,7 +53,7 @@ __device__ __forceinline__ QkvVal qkv_value(const QkvArgs& a, int seg, int t, in
   return r;
 }
 
-__global__ void __launch_bounds__(256) qkv_fwd_kernel(QkvArgs a) {
+__global__ void __launch_bounds__(512) qkv_fwd_kernel(QkvArgs a) {
   extern __shared__ float row[];
   __shared__ MaxMin red_mm[32];
   const int t = blockIdx.x, tid = threadIdx.x, nt = blockDim.x;
@@ -81,15 +90,15 @@ omq_status qkv_fwd_launch(cudaStream_t st, const QkvArgs& a) {
   const int dq = a.H * a.hd;
   size_t smem = (size_t)dq * sizeof(float);
   OMQ_REQUIRE(smem <= 200 * 1024, OMQ_ERR_UNSUPPORTED);
-  if (smem > 48 * 1024) cudaFuncSetAttribute(qkv_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  qkv_fwd_kernel<<<a.T, 256, smem, st>>>(a);
+  if (smem + 2048 > 48 * 1024) cudaFuncSetAttribute(qkv_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  qkv_fwd_kernel<<<a.T, 512, smem, st>>>(a);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 int64_t qkv_bwd_nslab(int T) { return (T + 3) / 4; }
 
-__global__ void __launch_bounds__(256) qkv_bwd_kernel(QkvArgs a) {
+__global__ void __launch_bounds__(512) qkv_bwd_kernel(QkvArgs a) {
   extern __shared__ float sm[];
   const int dq = a.H * a.hd, dkv = a.Hkv * a.hd;
   float* row = sm;            // X~ of the segment
@@ -178,10 +187,10 @@ omq_status qkv_bwd_launch(cudaStream_t st, const QkvArgs& a0, int64_t* nslab) {
   QkvArgs a = a0;
   a.rows_per_cta = 4;
   const int dq = a.H * a.hd, dkv = a.Hkv * a.hd;
-  size_t smem = (size_t)(3 * dq + dkv) * sizeof(float);
+  size_t smem = (size_t)(2 * dq + (a.part_q ? dq + dkv : 0)) * sizeof(float);
   OMQ_REQUIRE(smem <= 200 * 1024, OMQ_ERR_UNSUPPORTED);
-  if (smem > 48 * 1024) cudaFuncSetAttribute(qkv_bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  qkv_bwd_kernel<<<(unsigned)qkv_bwd_nslab(a.T), 256, smem, st>>>(a);
+  if (smem + 2048 > 48 * 1024) cudaFuncSetAttribute(qkv_bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  qkv_bwd_kernel<<<(unsigned)qkv_bwd_nslab(a.T), 512, smem, st>>>(a);
   OMQ_LAUNCH_CHECK();
   if (nslab) *nslab = qkv_bwd_nslab(a.T);
   return OMQ_OK;

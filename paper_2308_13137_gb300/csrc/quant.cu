@@ -5,163 +5,181 @@
 
 #include <atomic>
 
-#define LWC_MAXC 16        // 8-element chunks per thread held in registers (Cin <= 256*8*16)
+#define LWC_KEEP 16        // 8-element chunks per lane kept in registers between passes (Cin <= 4096)
 
 static std::atomic<long long> g_launches{0};
 void omq_count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 #define ACT_THREADS 256
 
 // ================================================================================================
-// LWC forward: one CTA per output row.
+// LWC forward: one warp per output row, eight rows per CTA; reductions by shuffles only.
 // ================================================================================================
 __device__ __forceinline__ float lwc_wt(float w, const float* s, int64_t col, float rr) {
   float sv = s ? s[col] : 1.f;
   return __fmul_rn(__fmul_rn(w, sv), rr);
 }
 
-__global__ void __launch_bounds__(256) lwc_fwd_kernel(LwcFwdArgs a) {
-  __shared__ MaxMin red_mm[32];
-  __shared__ float red_f[64];
-  __shared__ MaxMin row_mm;
-  const int64_t o = blockIdx.x;
-  const int tid = threadIdx.x, nt = blockDim.x;
-  const int64_t nchunk = a.Cin / 8;
-  const int nit = (int)((nchunk + nt - 1) / nt);
-  const float Q = (float)((1 << a.wbits) - 1);
-  const int gsz = a.group;
-  const int lpg = gsz / 8;                       // lanes per group
-  const bool seg = (gsz < a.Cin) || (lpg <= 32 && (lpg & (lpg - 1)) == 0 && gsz == a.Cin && a.Cin <= 256);
-  const int64_t ngroups = a.Cin / gsz;
-  const float rr = a.r ? a.r[o] : 1.f;
-  const __nv_bfloat16* Wrow = a.W + o * a.Cin;
-
-  uint4 raw[LWC_MAXC];
+// eight consecutive entries of an optional vector (1 when absent)
+__device__ __forceinline__ void load8(const float* v, int64_t c, float* out, float dflt) {
+  if (!v) {
 #pragma unroll
-  for (int i = 0; i < LWC_MAXC; ++i) {
-    raw[i] = make_uint4(0, 0, 0, 0);
-    if (i < nit) {
-      int64_t c = (int64_t)i * nt + tid;
-      if (c < nchunk) raw[i] = __ldg(reinterpret_cast<const uint4*>(Wrow) + c);
-    }
-  }
-  // LET bias B~_o = r_o (sum_i W_oi delta_i - shift_o)
-  if (a.Bt) {
-    float dot = 0.f;
-#pragma unroll
-    for (int i = 0; i < LWC_MAXC; ++i) {
-      if (i < nit) {
-        int64_t c = (int64_t)i * nt + tid;
-        if (c < nchunk) {
-          float w[8];
-          unpack_bf16x8(raw[i], w);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) dot = fmaf(w[e], a.bias_delta[c * 8 + e], dot);
-        }
-      }
-    }
-    float2 t = block_sum2(dot, 0.f, red_f);
-    if (tid == 0) a.Bt[o] = rr * (t.x - (a.bias_shift ? a.bias_shift[o] : 0.f));
-  }
-  if (a.wbits >= 16) {   // quantization off: W_hat = bf16(W~)
-#pragma unroll
-    for (int i = 0; i < LWC_MAXC; ++i) {
-      if (i < nit) {
-        int64_t c = (int64_t)i * nt + tid;
-        if (c < nchunk) {
-          float w[8];
-          unpack_bf16x8(raw[i], w);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) w[e] = lwc_wt(w[e], a.s, c * 8 + e, rr);
-          if (a.Wq) reinterpret_cast<uint4*>(a.Wq + o * a.Cin)[c] = pack_bf16x8(w);
-        }
-      }
-    }
+    for (int e = 0; e < 8; ++e) out[e] = dflt;
     return;
   }
+  float4 x = __ldg(reinterpret_cast<const float4*>(v) + 2 * c);
+  float4 y = __ldg(reinterpret_cast<const float4*>(v) + 2 * c + 1);
+  out[0] = x.x; out[1] = x.y; out[2] = x.z; out[3] = x.w; out[4] = y.x; out[5] = y.y; out[6] = y.z; out[7] = y.w;
+}
 
-  if (!seg) {
-    // ---- one group per row: block-wide max/min, then quantize ----
+// W~ = fl32(fl32(W * s) * r) for one 8-element chunk
+__device__ __forceinline__ void lwc_chunk(const uint4& raw, const float* s, int64_t c, float rr, float* wt) {
+  float sv[8];
+  unpack_bf16x8(raw, wt);
+  load8(s, c, sv, 1.f);
+#pragma unroll
+  for (int e = 0; e < 8; ++e) wt[e] = __fmul_rn(__fmul_rn(wt[e], sv[e]), rr);
+}
+
+__device__ __forceinline__ void lwc_store(const LwcFwdArgs& a, int64_t o, int64_t c, const float* wt, const QState& qs,
+                                          float Q) {
+  float w[8], cd[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) w[e] = omq_fakequant(wt[e], qs, Q, &cd[e]);
+  if (a.Wq) reinterpret_cast<uint4*>(a.Wq + o * a.Cin)[c] = pack_bf16x8(w);
+  if (a.codes) {
+    uint2 pk;
+    pk.x = (uint32_t)cd[0] | ((uint32_t)cd[1] << 8) | ((uint32_t)cd[2] << 16) | ((uint32_t)cd[3] << 24);
+    pk.y = (uint32_t)cd[4] | ((uint32_t)cd[5] << 8) | ((uint32_t)cd[6] << 16) | ((uint32_t)cd[7] << 24);
+    reinterpret_cast<uint2*>(a.codes + o * a.Cin)[c] = pk;
+  }
+}
+
+__device__ __forceinline__ float dot8(const uint4& raw, const float* d, int64_t c) {
+  float w[8], dv[8];
+  unpack_bf16x8(raw, w);
+  load8(d, c, dv, 0.f);
+  float acc = 0.f;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) acc = fmaf(w[e], dv[e], acc);
+  return acc;
+}
+
+__global__ void __launch_bounds__(256) lwc_fwd_kernel(LwcFwdArgs a) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t o = (int64_t)blockIdx.x * 8 + warp;
+  if (o >= a.Cout) return;                       // whole warp leaves; no block-level barrier below
+  const int64_t nchunk = a.Cin / 8;
+  const int iters = (int)((nchunk + 31) / 32);
+  const float Q = (float)((1 << (a.wbits >= 16 ? 1 : a.wbits)) - 1);
+  const float rr = a.r ? a.r[o] : 1.f;
+  const uint4* Wrow = reinterpret_cast<const uint4*>(a.W + o * a.Cin);
+  const int gsz = a.group;
+  const int64_t ngroups = a.Cin / gsz;
+  float dot = 0.f;
+
+  if (a.wbits >= 16) {                           // quantization off: W_hat = bf16(W~)
+    for (int it = 0; it < iters; ++it) {
+      const int64_t c = (int64_t)it * 32 + lane;
+      if (c < nchunk) {
+        uint4 raw = __ldg(Wrow + c);
+        float wt[8];
+        lwc_chunk(raw, a.s, c, rr, wt);
+        if (a.Wq) reinterpret_cast<uint4*>(a.Wq + o * a.Cin)[c] = pack_bf16x8(wt);
+        if (a.Bt) dot += dot8(raw, a.bias_delta, c);
+      }
+    }
+  } else if (gsz == a.Cin) {
+    // ---- one group per row: stats over the row (kept in registers up to LWC_KEEP chunks) ----
+    uint4 keep[LWC_KEEP];
     MaxMin r = mm_identity();
 #pragma unroll
-    for (int i = 0; i < LWC_MAXC; ++i) {
-      if (i < nit) {
-        int64_t c = (int64_t)i * nt + tid;
-        if (c < nchunk) {
-          float w[8];
-          unpack_bf16x8(raw[i], w);
+    for (int it = 0; it < LWC_KEEP; ++it) {
+      keep[it] = make_uint4(0, 0, 0, 0);
+      const int64_t c = (int64_t)it * 32 + lane;
+      if (it < iters && c < nchunk) {
+        keep[it] = __ldg(Wrow + c);
+        float wt[8];
+        lwc_chunk(keep[it], a.s, c, rr, wt);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) mm_push(r, lwc_wt(w[e], a.s, c * 8 + e, rr), (int)(c * 8 + e));
-        }
+        for (int e = 0; e < 8; ++e) mm_push(r, wt[e], (int)(c * 8 + e));
+        if (a.Bt) dot += dot8(keep[it], a.bias_delta, c);
       }
     }
-    r = mm_block_reduce(r, red_mm);
-    if (tid == 0) row_mm = r;
-    __syncthreads();
-    r = row_mm;
-    float ga = a.lwc ? omq_sigmoid(a.gl[o]) : 1.f;
-    float gb = a.lwc ? omq_sigmoid(a.bl[o]) : 1.f;
-    QState qs = omq_qstate(r.M, r.m, ga, gb, Q, a.eps);
-    if (tid == 0) {
-      a.h[o] = qs.h; a.z[o] = (int32_t)qs.z; a.imax[o] = r.iM; a.imin[o] = r.im;
-    }
+    for (int it = LWC_KEEP; it < iters; ++it) {
+      const int64_t c = (int64_t)it * 32 + lane;
+      if (c < nchunk) {
+        uint4 raw = __ldg(Wrow + c);
+        float wt[8];
+        lwc_chunk(raw, a.s, c, rr, wt);
 #pragma unroll
-    for (int i = 0; i < LWC_MAXC; ++i) {
-      if (i < nit) {
-        int64_t c = (int64_t)i * nt + tid;
-        if (c < nchunk) {
-          float w[8], cd[8];
-          unpack_bf16x8(raw[i], w);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) w[e] = omq_fakequant(lwc_wt(w[e], a.s, c * 8 + e, rr), qs, Q, &cd[e]);
-          if (a.Wq) reinterpret_cast<uint4*>(a.Wq + o * a.Cin)[c] = pack_bf16x8(w);
-          if (a.codes) {
-            uint2 pk;
-            pk.x = (uint32_t)cd[0] | ((uint32_t)cd[1] << 8) | ((uint32_t)cd[2] << 16) | ((uint32_t)cd[3] << 24);
-            pk.y = (uint32_t)cd[4] | ((uint32_t)cd[5] << 8) | ((uint32_t)cd[6] << 16) | ((uint32_t)cd[7] << 24);
-            reinterpret_cast<uint2*>(a.codes + o * a.Cin)[c] = pk;
-          }
-        }
+        for (int e = 0; e < 8; ++e) mm_push(r, wt[e], (int)(c * 8 + e));
+        if (a.Bt) dot += dot8(raw, a.bias_delta, c);
       }
     }
-    return;
-  }
-
-  // ---- groups of lpg consecutive lanes (lpg a power of two <= 32) ----
-  const int lane = tid & 31;
+    r = mm_shfl_reduce(r, 32);
+    float ga = 1.f, gb = 1.f;
+    if (a.lwc) {                                 // one sigmoid per group, broadcast
+      if (lane == 0) { ga = omq_sigmoid(a.gl[o]); gb = omq_sigmoid(a.bl[o]); }
+      ga = __shfl_sync(0xffffffffu, ga, 0);
+      gb = __shfl_sync(0xffffffffu, gb, 0);
+    }
+    const QState qs = omq_qstate(r.M, r.m, ga, gb, Q, a.eps);
+    if (lane == 0) { a.h[o] = qs.h; a.z[o] = (int32_t)qs.z; a.imax[o] = r.iM; a.imin[o] = r.im; }
 #pragma unroll
-  for (int i = 0; i < LWC_MAXC; ++i) {
-    if (i < nit) {
-      int64_t c = (int64_t)i * nt + tid;
-      bool valid = c < nchunk;
-      float w[8];
-      unpack_bf16x8(raw[i], w);
+    for (int it = 0; it < LWC_KEEP; ++it) {
+      const int64_t c = (int64_t)it * 32 + lane;
+      if (it < iters && c < nchunk) {
+        float wt[8];
+        lwc_chunk(keep[it], a.s, c, rr, wt);
+        lwc_store(a, o, c, wt, qs, Q);
+      }
+    }
+    for (int it = LWC_KEEP; it < iters; ++it) {
+      const int64_t c = (int64_t)it * 32 + lane;
+      if (c < nchunk) {
+        float wt[8];
+        lwc_chunk(__ldg(Wrow + c), a.s, c, rr, wt);
+        lwc_store(a, o, c, wt, qs, Q);
+      }
+    }
+  } else {
+    // ---- groups of lpg consecutive lanes (lpg a power of two <= 32) ----
+    const int lpg = gsz / 8;
+    const int leader = lane & ~(lpg - 1);
+    for (int it = 0; it < iters; ++it) {
+      const int64_t c = (int64_t)it * 32 + lane;
+      const bool valid = c < nchunk;
+      float wt[8];
       MaxMin r = mm_identity();
+      uint4 raw = make_uint4(0, 0, 0, 0);
       if (valid) {
+        raw = __ldg(Wrow + c);
+        lwc_chunk(raw, a.s, c, rr, wt);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) { w[e] = lwc_wt(w[e], a.s, c * 8 + e, rr); mm_push(r, w[e], (int)(c * 8 + e)); }
+        for (int e = 0; e < 8; ++e) mm_push(r, wt[e], (int)(c * 8 + e));
+        if (a.Bt) dot += dot8(raw, a.bias_delta, c);
       }
       r = mm_shfl_reduce(r, lpg);
+      const int64_t gi = valid ? (c * 8) / gsz : 0;
+      float ga = 1.f, gb = 1.f;
+      if (a.lwc) {
+        if (lane == leader && valid) { ga = omq_sigmoid(a.gl[o * ngroups + gi]); gb = omq_sigmoid(a.bl[o * ngroups + gi]); }
+        ga = __shfl_sync(0xffffffffu, ga, leader);
+        gb = __shfl_sync(0xffffffffu, gb, leader);
+      }
       if (valid) {
-        int64_t gi = (c * 8) / gsz;
-        float ga = a.lwc ? omq_sigmoid(a.gl[o * ngroups + gi]) : 1.f;
-        float gb = a.lwc ? omq_sigmoid(a.bl[o * ngroups + gi]) : 1.f;
-        QState qs = omq_qstate(r.M, r.m, ga, gb, Q, a.eps);
-        if ((lane & (lpg - 1)) == 0) {
-          int64_t k = o * ngroups + gi;
+        const QState qs = omq_qstate(r.M, r.m, ga, gb, Q, a.eps);
+        if (lane == leader) {
+          const int64_t k = o * ngroups + gi;
           a.h[k] = qs.h; a.z[k] = (int32_t)qs.z; a.imax[k] = r.iM; a.imin[k] = r.im;
         }
-        float cd[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) w[e] = omq_fakequant(w[e], qs, Q, &cd[e]);
-        if (a.Wq) reinterpret_cast<uint4*>(a.Wq + o * a.Cin)[c] = pack_bf16x8(w);
-        if (a.codes) {
-          uint2 pk;
-          pk.x = (uint32_t)cd[0] | ((uint32_t)cd[1] << 8) | ((uint32_t)cd[2] << 16) | ((uint32_t)cd[3] << 24);
-          pk.y = (uint32_t)cd[4] | ((uint32_t)cd[5] << 8) | ((uint32_t)cd[6] << 16) | ((uint32_t)cd[7] << 24);
-          reinterpret_cast<uint2*>(a.codes + o * a.Cin)[c] = pk;
-        }
+        lwc_store(a, o, c, wt, qs, Q);
       }
     }
+  }
+  if (a.Bt) {
+    dot = warp_sum(dot);
+    if (lane == 0) a.Bt[o] = rr * (dot - (a.bias_shift ? a.bias_shift[o] : 0.f));
   }
 }
 
@@ -180,8 +198,7 @@ static int lwc_threads(int64_t Cin) {
 
 omq_status lwc_fwd_launch(cudaStream_t st, const LwcFwdArgs& a) {
   OMQ_REQUIRE(lwc_group_ok(a.Cin, a.group), OMQ_ERR_UNSUPPORTED);
-  OMQ_REQUIRE(a.Cin / 8 <= (int64_t)256 * LWC_MAXC, OMQ_ERR_UNSUPPORTED);
-  lwc_fwd_kernel<<<(unsigned)a.Cout, lwc_threads(a.Cin), 0, st>>>(a);
+  lwc_fwd_kernel<<<(unsigned)((a.Cout + 7) / 8), 256, 0, st>>>(a);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -193,6 +210,7 @@ omq_status lwc_fwd_launch(cudaStream_t st, const LwcFwdArgs& a) {
 __global__ void __launch_bounds__(256) lwc_bwd_kernel(LwcBwdArgs a) {
   extern __shared__ float acc[];                 // acc_s[Cin], acc_d[Cin]
   __shared__ float red_f[64];
+  __shared__ float s_ab[2];
   const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31;
   const int64_t nchunk = a.Cin / 8;
   const int nit = (int)((nchunk + nt - 1) / nt);
@@ -221,8 +239,12 @@ __global__ void __launch_bounds__(256) lwc_bwd_kernel(LwcBwdArgs a) {
       const int iM = a.imax[o], im = a.imin[o];
       const float M = lwc_wt(bf16_to_f(Wrow[iM]), a.s, iM, rr);
       const float m = lwc_wt(bf16_to_f(Wrow[im]), a.s, im, rr);
-      const float ga = a.lwc ? omq_sigmoid(a.gl[o]) : 1.f;
-      const float gb = a.lwc ? omq_sigmoid(a.bl[o]) : 1.f;
+      if (tid == 0) {                          // one sigmoid per group, broadcast
+        s_ab[0] = a.lwc ? omq_sigmoid(a.gl[o]) : 1.f;
+        s_ab[1] = a.lwc ? omq_sigmoid(a.bl[o]) : 1.f;
+      }
+      __syncthreads();
+      const float ga = s_ab[0], gb = s_ab[1];
       QState qs = omq_qstate(M, m, ga, gb, Q, a.eps);
       qs.h = a.h[o]; qs.z = (float)a.z[o]; qs.u = __fdiv_rn(__fmul_rn(gb, m), qs.h);
       float Gh = 0.f, Gbm = 0.f;
@@ -293,6 +315,12 @@ __global__ void __launch_bounds__(256) lwc_bwd_kernel(LwcBwdArgs a) {
         int iM = 0, im = 0;
         float Gh = 0.f, Gbm = 0.f;
         int inr_mask = 0;
+        const int leader = lane & ~(lpg - 1);
+        if (a.lwc) {                             // one sigmoid per group, broadcast in the segment
+          if (lane == leader && valid) { ga = omq_sigmoid(a.gl[k]); gb = omq_sigmoid(a.bl[k]); }
+          ga = __shfl_sync(0xffffffffu, ga, leader);
+          gb = __shfl_sync(0xffffffffu, gb, leader);
+        }
         if (valid) {
           unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(Wrow) + c), w);
           float4 g0 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c);
@@ -301,8 +329,6 @@ __global__ void __launch_bounds__(256) lwc_bwd_kernel(LwcBwdArgs a) {
           iM = a.imax[k]; im = a.imin[k];
           M = lwc_wt(bf16_to_f(Wrow[iM]), a.s, iM, rr);
           m = lwc_wt(bf16_to_f(Wrow[im]), a.s, im, rr);
-          ga = a.lwc ? omq_sigmoid(a.gl[k]) : 1.f;
-          gb = a.lwc ? omq_sigmoid(a.bl[k]) : 1.f;
           qs = omq_qstate(M, m, ga, gb, Q, a.eps);
           qs.h = a.h[k]; qs.z = (float)a.z[k]; qs.u = __fdiv_rn(__fmul_rn(gb, m), qs.h);
 #pragma unroll
@@ -359,19 +385,25 @@ __global__ void __launch_bounds__(256) lwc_bwd_kernel(LwcBwdArgs a) {
   }
 }
 
+// rows per CTA so that at most 512 partial rows are written (independent of the device)
+static int64_t lwc_bwd_rows(int64_t Cout) {
+  int64_t rows = (Cout + 511) / 512;
+  return rows < 8 ? 8 : rows;
+}
+
 int64_t lwc_bwd_nslab(int64_t Cout) {
-  int64_t rows = 16;
+  const int64_t rows = lwc_bwd_rows(Cout);
   return (Cout + rows - 1) / rows;
 }
 
 omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a0, int64_t* nslab_out) {
   OMQ_REQUIRE(lwc_group_ok(a0.Cin, a0.group), OMQ_ERR_UNSUPPORTED);
   LwcBwdArgs a = a0;
-  a.rows_per_cta = 16;
+  a.rows_per_cta = (int)lwc_bwd_rows(a.Cout);
   int64_t nslab = lwc_bwd_nslab(a.Cout);
   size_t smem = (a.part_s || a.part_d) ? 2 * a.Cin * sizeof(float) : 0;
   OMQ_REQUIRE(smem <= 200 * 1024, OMQ_ERR_UNSUPPORTED);
-  if (smem > 48 * 1024) cudaFuncSetAttribute(lwc_bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (smem + 2048 > 48 * 1024) cudaFuncSetAttribute(lwc_bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   lwc_bwd_kernel<<<(unsigned)nslab, lwc_threads(a.Cin), smem, st>>>(a);
   OMQ_LAUNCH_CHECK();
   if (nslab_out) *nslab_out = nslab;
@@ -432,7 +464,7 @@ __device__ __forceinline__ void act_produce_row(const ActFwdArgs& a, int64_t t, 
 }
 
 template <int P>
-__global__ void __launch_bounds__(ACT_THREADS) act_fwd_kernel(ActFwdArgs a) {
+__global__ void __launch_bounds__(512) act_fwd_kernel(ActFwdArgs a) {
   extern __shared__ float row[];
   __shared__ float red_f[64];
   __shared__ MaxMin red_mm[32];
@@ -481,36 +513,39 @@ omq_status act_fwd_launch(cudaStream_t st, const ActFwdArgs& a) {
     case AP_SWIGLU: k = act_fwd_kernel<AP_SWIGLU>; break;
     default: return OMQ_ERR_INVALID_ARG;
   }
-  if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  k<<<(unsigned)a.T, ACT_THREADS, smem, st>>>(a);
+  if (smem + 2048 > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  k<<<(unsigned)a.T, a.C > 4096 ? 512 : ACT_THREADS, smem, st>>>(a);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 // ---- backward ----------------------------------------------------------------------------------
+// Shared memory: row[C] (quantizer input of the token) | dn[C] (RMS only) | acc_s[C], acc_d[C]
+// (LET column partials only).  The per-element STE gradient is recomputed where it is used.
 template <int P>
-__global__ void __launch_bounds__(ACT_THREADS) act_bwd_kernel(ActBwdArgs a) {
+__global__ void __launch_bounds__(512) act_bwd_kernel(ActBwdArgs a) {
   extern __shared__ float smem[];
-  float* row = smem;                      // quantizer input X~ of the current token
-  float* dv = smem + a.C;                 // dL/dX~ of the current token
-  float* acc_s = smem + 2 * a.C;          // LET column partial sums of this CTA
-  float* acc_d = smem + 3 * a.C;
-  __shared__ float red_f[64];
-  const int tid = threadIdx.x, nt = blockDim.x;
   const int64_t C = a.C;
   const bool let_sums = a.part_s != nullptr;
+  float* row = smem;
+  float* dn = smem + C;
+  float* acc_s = smem + (P == AP_RMS_LET ? 2 : 1) * C;
+  float* acc_d = acc_s + C;
+  __shared__ float red_f[64];
+  const int tid = threadIdx.x, nt = blockDim.x;
   if (let_sums)
     for (int64_t i = tid; i < C; i += nt) { acc_s[i] = 0.f; acc_d[i] = 0.f; }
   const int64_t t0 = (int64_t)blockIdx.x * a.rows_per_cta;
   const int64_t t1 = min(a.T, t0 + a.rows_per_cta);
-  const float Q = (float)((1 << (a.abits >= 16 ? 1 : a.abits)) - 1);
+  const bool quant = a.abits < 16;
+  const float Q = (float)((1 << (quant ? a.abits : 1)) - 1);
 
   ActFwdArgs f;
   f.producer = P; f.X = a.X; f.ldx = a.ldx; f.U = a.U; f.ldu = a.ldu; f.s = a.s; f.delta = a.delta;
   f.rms_eps = 0.f; f.C = a.C;
 
   for (int64_t t = t0; t < t1; ++t) {
-    // recompute X~ exactly as the forward did (RMS uses the saved rstd)
+    // X~ of the token exactly as the forward formed it (RMS uses the saved rstd)
     const float* xr = a.X + t * a.ldx;
     if (P == AP_RMS_LET) {
       const float rstd = a.rstd[t];
@@ -526,48 +561,54 @@ __global__ void __launch_bounds__(ACT_THREADS) act_bwd_kernel(ActBwdArgs a) {
       act_produce_row<P>(f, t, row, red_f, &dummy);
     }
     const float* gr = a.dXq + t * a.lddq;
-    if (a.abits >= 16) {
-      for (int64_t i = tid; i < C; i += nt) dv[i] = gr[i];
-    } else {
-      QState qs;
-      const int iM = a.imax[t], im = a.imin[t];
-      const float M = row[iM], m = row[im];
-      qs = omq_qstate(M, m, 1.f, 1.f, Q, a.eps);
-      qs.h = a.h[t]; qs.z = (float)a.z[t]; qs.u = __fdiv_rn(m, qs.h);
+    QState qs;
+    int iM = -1, im = -1;
+    float GaM = 0.f, Gbt = 0.f;
+    if (quant) {
+      iM = a.imax[t]; im = a.imin[t];
+      qs = omq_qstate(row[iM], row[im], 1.f, 1.f, Q, a.eps);
+      qs.h = a.h[t]; qs.z = (float)a.z[t]; qs.u = __fdiv_rn(row[im], qs.h);
       float Gh = 0.f, Gbm = 0.f;
       for (int64_t i = tid; i < C; i += nt) {
         int inr;
-        float g = gr[i];
-        float dh = omq_ste_dh(row[i], qs, Q, &inr);
+        const float g = gr[i];
+        const float dh = omq_ste_dh(row[i], qs, Q, &inr);
         Gh = fmaf(g, dh, Gh);
         if (!inr) Gbm += g;
-        dv[i] = inr ? g : 0.f;
       }
       float2 tot = block_sum2(Gh, Gbm, red_f);
-      Gh = qs.floored ? 0.f : tot.x;
-      Gbm = tot.y;
-      const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
-      if (tid == 0) { dv[iM] += GaM; dv[im] += Gbt; }
+      const float Gh_t = qs.floored ? 0.f : tot.x;
+      GaM = Gh_t / Q;
+      Gbt = tot.y - Gh_t / Q;
     }
-    __syncthreads();
-    // producer backward
+    // dL/dX~ of element i (straight-through, with the max/min routing)
+    auto dxt = [&](int64_t i) -> float {
+      const float g = gr[i];
+      if (!quant) return g;
+      int inr;
+      omq_ste_dh(row[i], qs, Q, &inr);
+      float d = inr ? g : 0.f;
+      if (i == iM) d += GaM;
+      if (i == im) d += Gbt;
+      return d;
+    };
     if (P == AP_PLAIN || P == AP_LET) {
       for (int64_t i = tid; i < C; i += nt) {
-        float d = dv[i];
-        float sv = a.s ? a.s[i] : 1.f;
+        const float d = dxt(i);
+        const float sv = a.s ? a.s[i] : 1.f;
         if (let_sums) { acc_s[i] -= d * row[i] / sv; acc_d[i] -= d / sv; }
-        float dx = a.s ? __fdiv_rn(d, sv) : d;
+        const float dx = a.s ? __fdiv_rn(d, sv) : d;
         if (a.dX) a.dX[t * a.lddx + i] = dx;
         if (a.dXb) a.dXb[t * a.lddxb + i] = f_to_bf16(dx);
       }
     } else if (P == AP_SWIGLU) {
       const float* ur = a.U + t * a.ldu;
       for (int64_t i = tid; i < C; i += nt) {
-        float d = dv[i];
-        float g = xr[i], u = ur[i];
-        float sg = 1.f / (1.f + expf(-g));
-        float dg = d * u * sg * (1.f + g * (1.f - sg));
-        float du = d * g * sg;
+        const float d = dxt(i);
+        const float g = xr[i], u = ur[i];
+        const float sg = 1.f / (1.f + expf(-g));
+        const float dg = d * u * sg * (1.f + g * (1.f - sg));
+        const float du = d * g * sg;
         if (a.dX) { a.dX[t * a.lddx + i] = dg; a.dU[t * a.lddx + i] = du; }
         if (a.dXb) { a.dXb[t * a.lddxb + i] = f_to_bf16(dg); a.dUb[t * a.lddxb + i] = f_to_bf16(du); }
       }
@@ -575,19 +616,19 @@ __global__ void __launch_bounds__(ACT_THREADS) act_bwd_kernel(ActBwdArgs a) {
       const float rstd = a.rstd[t];
       float dot = 0.f;
       for (int64_t i = tid; i < C; i += nt) {
-        float d = dv[i];
-        float sv = a.s ? a.s[i] : 1.f;
+        const float d = dxt(i);
+        const float sv = a.s ? a.s[i] : 1.f;
         if (let_sums) { acc_s[i] -= d * row[i] / sv; acc_d[i] -= d / sv; }
-        float dn = a.s ? __fdiv_rn(d, sv) : d;     // dL/d(RMSNorm output)
-        dv[i] = dn;
-        dot = fmaf(dn, xr[i] * rstd, dot);
+        const float v = a.s ? __fdiv_rn(d, sv) : d;
+        dn[i] = v;
+        dot = fmaf(v, xr[i] * rstd, dot);
       }
-      float2 tot = block_sum2(dot, 0.f, red_f);
-      const float mean_dot = tot.x / (float)C;
       if (a.dX || a.dXb) {
+        float2 tot = block_sum2(dot, 0.f, red_f);
+        const float mean_dot = tot.x / (float)C;
         for (int64_t i = tid; i < C; i += nt) {
-          float an = xr[i] * rstd;
-          float dx = rstd * (dv[i] - an * mean_dot);
+          const float an = xr[i] * rstd;
+          float dx = rstd * (dn[i] - an * mean_dot);
           if (a.resid) dx += a.resid[t * a.lddx + i];
           if (a.dX) a.dX[t * a.lddx + i] = dx;
           if (a.dXb) a.dXb[t * a.lddxb + i] = f_to_bf16(dx);
@@ -608,7 +649,8 @@ omq_status act_bwd_launch(cudaStream_t st, const ActBwdArgs& a0) {
   ActBwdArgs a = a0;
   OMQ_REQUIRE(a.C % 8 == 0 && a.T > 0, OMQ_ERR_SHAPE);
   if (a.rows_per_cta <= 0) a.rows_per_cta = 4;
-  size_t smem = 4 * a.C * sizeof(float);
+  const int mult = (a.producer == AP_RMS_LET ? 2 : 1) + (a.part_s ? 2 : 0);
+  size_t smem = (size_t)mult * a.C * sizeof(float);
   OMQ_REQUIRE(smem <= 200 * 1024, OMQ_ERR_UNSUPPORTED);
   void (*k)(ActBwdArgs) = nullptr;
   switch (a.producer) {
@@ -618,9 +660,9 @@ omq_status act_bwd_launch(cudaStream_t st, const ActBwdArgs& a0) {
     case AP_SWIGLU: k = act_bwd_kernel<AP_SWIGLU>; break;
     default: return OMQ_ERR_INVALID_ARG;
   }
-  if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  unsigned grid = (unsigned)((a.T + a.rows_per_cta - 1) / a.rows_per_cta);
-  k<<<grid, ACT_THREADS, smem, st>>>(a);
+  if (smem + 2048 > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  const unsigned grid = (unsigned)((a.T + a.rows_per_cta - 1) / a.rows_per_cta);
+  k<<<grid, a.C > 4096 ? 512 : 256, smem, st>>>(a);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -628,19 +670,29 @@ omq_status act_bwd_launch(cudaStream_t st, const ActBwdArgs& a0) {
 // ================================================================================================
 // reductions, loss, small vector kernels
 // ================================================================================================
+// 32 columns per CTA, eight row phases per column; fixed summation order (deterministic)
 __global__ void omq_colsum_partials_kernel(const float* __restrict__ part, int64_t P, int64_t C,
                                            float* __restrict__ out, float scale, int accumulate) {
-  int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= C) return;
+  __shared__ float red[8][33];
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const int64_t c = (int64_t)blockIdx.x * 32 + tx;
   float s = 0.f;
-  for (int64_t p = 0; p < P; ++p) s += part[p * C + c];
-  s *= scale;
-  out[c] = accumulate ? out[c] + s : s;
+  if (c < C)
+    for (int64_t p = ty; p < P; p += 8) s += part[p * C + c];
+  red[ty][tx] = s;
+  __syncthreads();
+  if (ty == 0 && c < C) {
+    float t = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) t += red[i][tx];
+    t *= scale;
+    out[c] = accumulate ? out[c] + t : t;
+  }
 }
 
 omq_status omq_colsum_partials(cudaStream_t st, const float* part, int64_t P, int64_t C, float* out,
                                float scale, int accumulate) {
-  omq_colsum_partials_kernel<<<(unsigned)((C + 255) / 256), 256, 0, st>>>(part, P, C, out, scale, accumulate);
+  omq_colsum_partials_kernel<<<(unsigned)((C + 31) / 32), 256, 0, st>>>(part, P, C, out, scale, accumulate);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
