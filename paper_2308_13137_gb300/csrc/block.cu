@@ -21,11 +21,13 @@ struct Carve {
 
 typedef __nv_bfloat16 bf16;
 
-struct QState4 { float* h; int32_t* z; int32_t* imax; int32_t* imin; };
+struct QState4 { float* h; int32_t* z; int32_t* imax; int32_t* imin; float* ga; float* gb; };
 
-QState4 take_qstate(Carve& c, size_t n) {
+QState4 take_qstate(Carve& c, size_t n, bool sig = false) {
   QState4 q;
   q.h = c.take<float>(n); q.z = c.take<int32_t>(n); q.imax = c.take<int32_t>(n); q.imin = c.take<int32_t>(n);
+  q.ga = sig ? c.take<float>(n) : nullptr;
+  q.gb = sig ? c.take<float>(n) : nullptr;
   return q;
 }
 
@@ -72,10 +74,10 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   w.Wo_h = c.take<bf16>(d * dq);
   w.Wgu_h = c.take<bf16>(2 * f * d);
   w.Wd_h = c.take<bf16>(d * f);
-  w.sq_qkv = take_qstate(c, nqkv * ng(d));
-  w.sq_o = take_qstate(c, d * ng(dq));
-  w.sq_gu = take_qstate(c, 2 * f * ng(d));
-  w.sq_d = take_qstate(c, d * ng(f));
+  w.sq_qkv = take_qstate(c, nqkv * ng(d), true);
+  w.sq_o = take_qstate(c, d * ng(dq), true);
+  w.sq_gu = take_qstate(c, 2 * f * ng(d), true);
+  w.sq_d = take_qstate(c, d * ng(f), true);
   w.B_qkv = c.take<float>(nqkv);
   w.B_o = c.take<float>(d);
   w.B_gu = c.take<float>(2 * f);
@@ -133,9 +135,10 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   w.vtmp1 = c.take<float>(vmax);
   w.vtmp2 = c.take<float>(vmax);
   int64_t pe = 0;
-  pe = imax64(pe, 2 * lwc_bwd_nslab(nqkv) * d);
-  pe = imax64(pe, 2 * lwc_bwd_nslab(d) * dq);
-  pe = imax64(pe, 2 * lwc_bwd_nslab(2 * f) * d);
+  pe = imax64(pe, (int64_t)lwc_bwd_scratch_bytes(nqkv, d) / 4 + 64);
+  pe = imax64(pe, (int64_t)lwc_bwd_scratch_bytes(d, dq) / 4 + 64);
+  pe = imax64(pe, (int64_t)lwc_bwd_scratch_bytes(2 * f, d) / 4 + 64);
+  pe = imax64(pe, (int64_t)lwc_bwd_scratch_bytes(d, f) / 4 + 64);
   pe = imax64(pe, 2 * ((T + 3) / 4) * imax64(d, dq));
   pe = imax64(pe, qkv_bwd_nslab((int)T) * (dq + dkv));
   pe = imax64(pe, colsum_rows_parts(T) * imax64(2 * f, nqkv));
@@ -189,6 +192,7 @@ LwcFwdArgs lwc_args(const bf16* W, int64_t Cout, int64_t Cin, const omq_qcfg& cf
   a.s = s; a.r = r; a.gl = gl; a.bl = bl; a.lwc = 1; a.Wq = Wq; a.codes = nullptr;
   a.h = q.h; a.z = q.z; a.imax = q.imax; a.imin = q.imin;
   a.bias_delta = bias_delta; a.bias_shift = bias_shift; a.Bt = Bt;
+  a.ga_out = q.ga; a.gb_out = q.gb;
   a.wbits = cfg.wbits; a.eps = cfg.h_eps; a.status = cfg.dev_status;
   return a;
 }
@@ -199,18 +203,14 @@ omq_status lwc_bwd_full(cudaStream_t st, const bf16* W, int64_t Cout, int64_t Ci
                         float* ddelta, int accumulate_sd, float* part) {
   LwcBwdArgs a{};
   a.W = W; a.Cout = Cout; a.Cin = Cin; a.group = cfg.group == 0 ? (int)Cin : cfg.group;
-  a.s = s; a.r = r; a.gl = gl; a.bl = bl; a.lwc = 1;
+  a.s = s; a.r = r; a.gl = gl; a.bl = bl; a.lwc = 1; a.ga = q.ga; a.gb = q.gb;
   a.h = q.h; a.z = q.z; a.imax = q.imax; a.imin = q.imin;
   a.dWq = dW; a.ld_dwq = Cin; a.dgl = dgl; a.dbl = dbl; a.dWt = nullptr; a.dr = dr; a.dBt = dBt;
-  const int64_t ns = lwc_bwd_nslab(Cout);
-  a.part_s = ds ? part : nullptr;
-  a.part_d = ddelta ? part + ns * Cin : nullptr;
-  a.wbits = cfg.wbits; a.eps = cfg.h_eps; a.accumulate = cfg.accumulate; a.accumulate_dr = 0;
-  int64_t n = 0;
-  OMQ_TRY(lwc_bwd_launch(st, a, &n));
-  if (ds) OMQ_TRY(omq_colsum_partials(st, a.part_s, n, Cin, ds, 1.f, accumulate_sd));
-  if (ddelta) OMQ_TRY(omq_colsum_partials(st, a.part_d, n, Cin, ddelta, 1.f, accumulate_sd));
-  return OMQ_OK;
+  a.ds = ds; a.ddelta = ddelta;
+  a.wbits = cfg.wbits; a.eps = cfg.h_eps;
+  // dgamma/dbeta follow cfg.accumulate; the LET sums follow the caller; dr is scratch
+  a.accumulate = cfg.accumulate; a.accumulate_sd = accumulate_sd; a.accumulate_dr = 0;
+  return lwc_bwd_launch(st, a, part);
 }
 
 struct Ctx {
@@ -526,7 +526,7 @@ omq_status omq_qlinear_fwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t 
   cudaStream_t st = (cudaStream_t)stream;
   const int g = cfg->group == 0 ? (int)Cin : cfg->group;
   OMQ_REQUIRE(Cin % g == 0, OMQ_ERR_SHAPE);
-  QState4 qw{sv->h_w, sv->z_w, sv->imax_w, sv->imin_w};
+  QState4 qw{sv->h_w, sv->z_w, sv->imax_w, sv->imin_w, nullptr, nullptr};
   const bool let = cfg->let != 0;
   OMQ_TRY(lwc_fwd_launch(st, lwc_args((const bf16*)W, Cout, Cin, *cfg, let ? s : nullptr, nullptr, gamma_logit,
                                       beta_logit, (bf16*)sv->w_hat, qw, let ? delta : nullptr, nullptr,
@@ -555,7 +555,7 @@ size_t omq_qlinear_workspace_size(int64_t T, int64_t Cin, int64_t Cout, const om
   c.take<float>(Cout * Cin);                    // dW_hat
   c.take<float>(T * Cin);                       // dX_hat
   c.take<float>(Cout);                          // dB~
-  int64_t pe = imax64(2 * lwc_bwd_nslab(Cout) * Cin, 2 * ((T + 3) / 4) * Cin);
+  int64_t pe = imax64((int64_t)lwc_bwd_scratch_bytes(Cout, Cin) / 4 + 64, 2 * ((T + 3) / 4) * Cin);
   pe = imax64(pe, colsum_rows_parts(T) * Cout);
   c.take<float>(pe);
   return c.off + 256;
@@ -579,14 +579,14 @@ omq_status omq_qlinear_bwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t 
   float* dWh = c.take<float>(Cout * Cin);
   float* dXh = c.take<float>(T * Cin);
   float* dB = c.take<float>(Cout);
-  int64_t pe = imax64(2 * lwc_bwd_nslab(Cout) * Cin, 2 * ((T + 3) / 4) * Cin);
+  int64_t pe = imax64((int64_t)lwc_bwd_scratch_bytes(Cout, Cin) / 4 + 64, 2 * ((T + 3) / 4) * Cin);
   pe = imax64(pe, colsum_rows_parts(T) * Cout);
   float* part = c.take<float>(pe);
   f32_to_bf16_kernel<<<(unsigned)((T * Cout + 255) / 256), 256, 0, st>>>(dY, dYb, T * Cout);
   OMQ_LAUNCH_CHECK();
   OMQ_TRY(gemm_dw(st, T, Cout, Cin, dYb, (const bf16*)sv->x_hat, dWh, cfg->dev_status));
   if (let) OMQ_TRY(colsum_rows(st, dY, T, Cout, Cout, part, dB, 1.f, 0));
-  QState4 qw{sv->h_w, sv->z_w, sv->imax_w, sv->imin_w};
+  QState4 qw{sv->h_w, sv->z_w, sv->imax_w, sv->imin_w, nullptr, nullptr};
   omq_qcfg cf = *cfg;
   OMQ_TRY(lwc_bwd_full(st, (const bf16*)W, Cout, Cin, cf, let ? s : nullptr, nullptr, gamma_logit, beta_logit, qw, dWh,
                        dgamma, dbeta, nullptr, let ? dB : nullptr, let ? ds : nullptr, let ? ddelta : nullptr,

@@ -124,7 +124,10 @@ __global__ void __launch_bounds__(256) lwc_fwd_kernel(LwcFwdArgs a) {
       gb = __shfl_sync(0xffffffffu, gb, 0);
     }
     const QState qs = omq_qstate(r.M, r.m, ga, gb, Q, a.eps);
-    if (lane == 0) { a.h[o] = qs.h; a.z[o] = (int32_t)qs.z; a.imax[o] = r.iM; a.imin[o] = r.im; }
+    if (lane == 0) {
+      a.h[o] = qs.h; a.z[o] = (int32_t)qs.z; a.imax[o] = r.iM; a.imin[o] = r.im;
+      if (a.ga_out) { a.ga_out[o] = ga; a.gb_out[o] = gb; }
+    }
 #pragma unroll
     for (int it = 0; it < LWC_KEEP; ++it) {
       const int64_t c = (int64_t)it * 32 + lane;
@@ -172,6 +175,7 @@ __global__ void __launch_bounds__(256) lwc_fwd_kernel(LwcFwdArgs a) {
         if (lane == leader) {
           const int64_t k = o * ngroups + gi;
           a.h[k] = qs.h; a.z[k] = (int32_t)qs.z; a.imax[k] = r.iM; a.imin[k] = r.im;
+          if (a.ga_out) { a.ga_out[k] = ga; a.gb_out[k] = gb; }
         }
         lwc_store(a, o, c, wt, qs, Q);
       }
@@ -189,12 +193,6 @@ static bool lwc_group_ok(int64_t Cin, int g) {
   return Cin % g == 0;
 }
 
-static int lwc_threads(int64_t Cin) {
-  int64_t nchunk = Cin / 8;
-  int nt = 256;
-  if (nchunk < 256) nt = (int)((nchunk + 31) / 32 * 32);
-  return nt;
-}
 
 omq_status lwc_fwd_launch(cudaStream_t st, const LwcFwdArgs& a) {
   OMQ_REQUIRE(lwc_group_ok(a.Cin, a.group), OMQ_ERR_UNSUPPORTED);
@@ -204,209 +202,273 @@ omq_status lwc_fwd_launch(cudaStream_t st, const LwcFwdArgs& a) {
 }
 
 // ================================================================================================
-// LWC backward (straight-through, Eq. 2): one CTA per slab of rows; each thread owns fixed
-// columns and accumulates the LET column sums of its columns in shared memory.
+// LWC backward (straight-through, Eq. 2), streaming over [row tile x column tile] blocks.
+// Each thread owns one 8-column chunk of a 2048-column tile and walks the rows of its row tile,
+// keeping the LET column sums of its columns in registers.  Per-row reductions are warp
+// shuffles: inside a group they complete in the warp (groups of <= 256 columns); for one group
+// per row every warp writes its 256-column partial and a per-row finalize combines them.
 // ================================================================================================
-__global__ void __launch_bounds__(256) lwc_bwd_kernel(LwcBwdArgs a) {
-  extern __shared__ float acc[];                 // acc_s[Cin], acc_d[Cin]
-  __shared__ float red_f[64];
-  __shared__ float s_ab[2];
-  const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31;
+#define LWC_BWD_THREADS 256
+#define LWC_BWD_TILE_COLS (LWC_BWD_THREADS * 8)
+
+struct LwcBwdScratch {
+  float* part_s;     // [nrt, Cin]
+  float* part_d;     // [nrt, Cin]
+  float* rowpart;    // [3, Cout, ncw]: G_h, G_bm, dr partials of every 256-column warp
+  float* sig;        // [2, Cout, ng]: clipping strengths when the caller has none saved
+  int64_t nrt, ncw, rows, ng;
+};
+
+static int64_t lwc_bwd_tile_rows(int64_t Cout, int64_t Cin) {
+  const int64_t ncol = (Cin / 8 + LWC_BWD_THREADS - 1) / LWC_BWD_THREADS;
+  int64_t rows = (Cout * ncol + 607) / 608;           // about four CTAs per SM of a 152-SM part
+  if (rows < 8) rows = 8;
+  if (rows > 64) rows = 64;
+  return rows;
+}
+
+static LwcBwdScratch lwc_bwd_carve(void* base, int64_t Cout, int64_t Cin, int64_t ng, size_t* bytes) {
+  LwcBwdScratch sc;
+  sc.ng = ng;
+  sc.rows = lwc_bwd_tile_rows(Cout, Cin);
+  sc.nrt = (Cout + sc.rows - 1) / sc.rows;
+  sc.ncw = (Cin / 8 + 31) / 32;
+  size_t off = 0;
+  auto take = [&](size_t n) { off = (off + 63) & ~size_t(63); float* p = base ? (float*)((char*)base + off * 4) : nullptr; off += n; return p; };
+  sc.part_s = take((size_t)sc.nrt * Cin);
+  sc.part_d = take((size_t)sc.nrt * Cin);
+  sc.rowpart = take((size_t)3 * Cout * sc.ncw);
+  sc.sig = take((size_t)2 * Cout * sc.ng);
+  if (bytes) *bytes = off * 4 + 256;
+  return sc;
+}
+
+size_t lwc_bwd_scratch_bytes(int64_t Cout, int64_t Cin) {
+  size_t b = 0;
+  lwc_bwd_carve(nullptr, Cout, Cin, Cin / 8, &b);      // groups of at least 8 columns
+  return b;
+}
+
+__global__ void sigmoid_pair_kernel(const float* gl, const float* bl, int64_t n, float* ga, float* gb) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) { ga[i] = omq_sigmoid(gl[i]); gb[i] = omq_sigmoid(bl[i]); }
+}
+
+__device__ __forceinline__ float lwc_sig(const float* saved, const float* logit, int64_t k, int lwc) {
+  if (!lwc) return 1.f;
+  return saved ? saved[k] : omq_sigmoid(logit[k]);
+}
+
+__global__ void __launch_bounds__(LWC_BWD_THREADS) lwc_bwd_tile_kernel(LwcBwdArgs a, LwcBwdScratch sc) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t nchunk = a.Cin / 8;
-  const int nit = (int)((nchunk + nt - 1) / nt);
+  const int64_t c = (int64_t)blockIdx.x * LWC_BWD_THREADS + tid;     // this thread's chunk
+  const bool valid = c < nchunk;
+  const int64_t wglob = (int64_t)blockIdx.x * (LWC_BWD_THREADS / 32) + warp;
   const float Q = (float)((1 << a.wbits) - 1);
   const int gsz = a.group;
-  const int lpg = gsz / 8;
-  const bool seg = (gsz < a.Cin) || (lpg <= 32 && (lpg & (lpg - 1)) == 0 && gsz == a.Cin && a.Cin <= 256);
+  const bool perch = gsz == a.Cin;
   const int64_t ngroups = a.Cin / gsz;
-  const bool want_s = a.part_s != nullptr, want_d = a.part_d != nullptr && a.dBt != nullptr;
-  float* acc_s = acc;
-  float* acc_d = acc + a.Cin;
-  if (want_s || want_d)
-    for (int64_t c = tid; c < a.Cin; c += nt) { acc_s[c] = 0.f; acc_d[c] = 0.f; }
-  const int64_t o0 = (int64_t)blockIdx.x * a.rows_per_cta;
-  const int64_t o1 = min(a.Cout, o0 + a.rows_per_cta);
+  const int lpg = perch ? 32 : gsz / 8;
+  const int leader = lane & ~(lpg - 1);
+  const bool want_s = a.ds != nullptr, want_d = a.ddelta != nullptr && a.dBt != nullptr;
+  float sv[8];
+  load8(a.s, valid ? c : 0, sv, 1.f);
+  float acc_s[8], acc_d[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) { acc_s[e] = 0.f; acc_d[e] = 0.f; }
+  const int64_t o0 = (int64_t)blockIdx.y * sc.rows;
+  const int64_t o1 = min(a.Cout, o0 + sc.rows);
+  const uint4 zero4 = make_uint4(0, 0, 0, 0);
 
   for (int64_t o = o0; o < o1; ++o) {
     const float rr = a.r ? a.r[o] : 1.f;
-    const float dBo = (want_d) ? a.dBt[o] : 0.f;
     const __nv_bfloat16* Wrow = a.W + o * a.Cin;
-    const float* grow = a.dWq + o * a.ld_dwq;
-    float dr_part = 0.f;
-
-    if (!seg) {
-      // per-row group: state from the saved indices
-      const int iM = a.imax[o], im = a.imin[o];
-      const float M = lwc_wt(bf16_to_f(Wrow[iM]), a.s, iM, rr);
-      const float m = lwc_wt(bf16_to_f(Wrow[im]), a.s, im, rr);
-      if (tid == 0) {                          // one sigmoid per group, broadcast
-        s_ab[0] = a.lwc ? omq_sigmoid(a.gl[o]) : 1.f;
-        s_ab[1] = a.lwc ? omq_sigmoid(a.bl[o]) : 1.f;
-      }
-      __syncthreads();
-      const float ga = s_ab[0], gb = s_ab[1];
-      QState qs = omq_qstate(M, m, ga, gb, Q, a.eps);
-      qs.h = a.h[o]; qs.z = (float)a.z[o]; qs.u = __fdiv_rn(__fmul_rn(gb, m), qs.h);
-      float Gh = 0.f, Gbm = 0.f;
-      for (int i = 0; i < nit; ++i) {
-        int64_t c = (int64_t)i * nt + tid;
-        if (c < nchunk) {
-          float w[8];
-          unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(Wrow) + c), w);
-          float4 g0 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c);
-          float4 g1 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c + 1);
-          float g[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+    const uint4 raw = valid ? __ldg(reinterpret_cast<const uint4*>(Wrow) + c) : zero4;
+    float g[8];
+    if (valid) {
+      const float4 g0 = __ldg(reinterpret_cast<const float4*>(a.dWq + o * a.ld_dwq) + 2 * c);
+      const float4 g1 = __ldg(reinterpret_cast<const float4*>(a.dWq + o * a.ld_dwq) + 2 * c + 1);
+      g[0] = g0.x; g[1] = g0.y; g[2] = g0.z; g[3] = g0.w; g[4] = g1.x; g[5] = g1.y; g[6] = g1.z; g[7] = g1.w;
+    } else {
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            int inr;
-            float dh = omq_ste_dh(lwc_wt(w[e], a.s, c * 8 + e, rr), qs, Q, &inr);
-            Gh = fmaf(g[e], dh, Gh);
-            if (!inr) Gbm += g[e];
-          }
+      for (int e = 0; e < 8; ++e) g[e] = 0.f;
+    }
+    float w[8];
+    unpack_bf16x8(raw, w);
+    // quantizer state of this lane's group
+    const int64_t k = perch ? o : o * ngroups + (valid ? (c * 8) / gsz : 0);
+    const int iM = a.imax[k], im = a.imin[k];
+    const float gb = lwc_sig(a.gb, a.bl, k, a.lwc);
+    const float m = lwc_wt(bf16_to_f(Wrow[im]), a.s, im, rr);
+    QState qs;
+    qs.h = a.h[k]; qs.z = (float)a.z[k]; qs.b = gb; qs.m = m;
+    qs.u = __fdiv_rn(__fmul_rn(gb, m), qs.h);
+    float Gh = 0.f, Gbm = 0.f, drm = 0.f;
+    int inr_mask = 0;
+    if (valid) {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const float wt = __fmul_rn(__fmul_rn(w[e], sv[e]), rr);
+        int inr;
+        const float dh = omq_ste_dh(wt, qs, Q, &inr);
+        Gh = fmaf(g[e], dh, Gh);
+        if (!inr) Gbm += g[e];
+        inr_mask |= inr << e;
+      }
+    }
+    if (perch) {
+      // warp partials of the row; routing to max/min is added by the per-row finalize
+      Gh = warp_sum(Gh);
+      Gbm = warp_sum(Gbm);
+      if (valid) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float d = ((inr_mask >> e) & 1) ? g[e] : 0.f;
+          drm = fmaf(d * w[e], sv[e], drm);
+          if (want_s) acc_s[e] = fmaf(d * w[e], rr, acc_s[e]);
+          if (a.dWt) g[e] = d;
+        }
+        if (a.dWt) {
+          float4* dst = reinterpret_cast<float4*>(a.dWt + o * a.Cin) + 2 * c;
+          dst[0] = make_float4(g[0], g[1], g[2], g[3]);
+          dst[1] = make_float4(g[4], g[5], g[6], g[7]);
         }
       }
-      float2 tot = block_sum2(Gh, Gbm, red_f);
-      Gh = qs.floored ? 0.f : tot.x;
-      Gbm = tot.y;
-      const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
-      if (tid == 0 && a.lwc) {
-        float dg = GaM * M * ga * (1.f - ga), db = Gbt * m * gb * (1.f - gb);
-        if (a.accumulate) { a.dgl[o] += dg; a.dbl[o] += db; } else { a.dgl[o] = dg; a.dbl[o] = db; }
-      }
-      for (int i = 0; i < nit; ++i) {
-        int64_t c = (int64_t)i * nt + tid;
-        if (c < nchunk) {
-          float w[8];
-          unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(Wrow) + c), w);
-          float4 g0 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c);
-          float4 g1 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c + 1);
-          float g[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
-          float dwt[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            int64_t col = c * 8 + e;
-            int inr;
-            omq_ste_dh(lwc_wt(w[e], a.s, col, rr), qs, Q, &inr);
-            float d = inr ? g[e] : 0.f;
-            if (col == iM) d += GaM * ga;
-            if (col == im) d += Gbt * gb;
-            dwt[e] = d;
-            float sv = a.s ? a.s[col] : 1.f;
-            dr_part = fmaf(d * w[e], sv, dr_part);
-            if (want_s) acc_s[col] = fmaf(d * w[e], rr, acc_s[col]);
-            if (want_d) acc_d[col] = fmaf(dBo * rr, w[e], acc_d[col]);
-          }
-          if (a.dWt) {
-            float4* dst = reinterpret_cast<float4*>(a.dWt + o * a.Cin) + 2 * c;
-            dst[0] = make_float4(dwt[0], dwt[1], dwt[2], dwt[3]);
-            dst[1] = make_float4(dwt[4], dwt[5], dwt[6], dwt[7]);
-          }
-        }
+      drm = warp_sum(drm);
+      if (lane == 0 && wglob < sc.ncw) {
+        sc.rowpart[(0 * a.Cout + o) * sc.ncw + wglob] = Gh;
+        sc.rowpart[(1 * a.Cout + o) * sc.ncw + wglob] = Gbm;
+        sc.rowpart[(2 * a.Cout + o) * sc.ncw + wglob] = drm;
       }
     } else {
-      for (int i = 0; i < nit; ++i) {
-        int64_t c = (int64_t)i * nt + tid;
-        bool valid = c < nchunk;
-        float w[8], g[8], wt[8];
-        int64_t gi = valid ? (c * 8) / gsz : 0;
-        int64_t k = o * ngroups + gi;
-        QState qs;
-        float ga = 1.f, gb = 1.f, M = 0.f, m = 0.f;
-        int iM = 0, im = 0;
-        float Gh = 0.f, Gbm = 0.f;
-        int inr_mask = 0;
-        const int leader = lane & ~(lpg - 1);
-        if (a.lwc) {                             // one sigmoid per group, broadcast in the segment
-          if (lane == leader && valid) { ga = omq_sigmoid(a.gl[k]); gb = omq_sigmoid(a.bl[k]); }
-          ga = __shfl_sync(0xffffffffu, ga, leader);
-          gb = __shfl_sync(0xffffffffu, gb, leader);
+      Gh = warp_sum(Gh, lpg);
+      Gbm = warp_sum(Gbm, lpg);
+      if (valid) {
+        const float ga = lwc_sig(a.ga, a.gl, k, a.lwc);
+        const float M = lwc_wt(bf16_to_f(Wrow[iM]), a.s, iM, rr);
+        const float hr = __fdiv_rn(__fsub_rn(__fmul_rn(ga, M), __fmul_rn(gb, m)), Q);
+        if (!(hr >= a.eps)) Gh = 0.f;                      // floored h: no gradient through h
+        const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
+        if (lane == leader && a.lwc) {
+          const float dg = GaM * M * ga * (1.f - ga), db = Gbt * m * gb * (1.f - gb);
+          if (a.accumulate) { a.dgl[k] += dg; a.dbl[k] += db; } else { a.dgl[k] = dg; a.dbl[k] = db; }
         }
-        if (valid) {
-          unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(Wrow) + c), w);
-          float4 g0 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c);
-          float4 g1 = __ldg(reinterpret_cast<const float4*>(grow) + 2 * c + 1);
-          g[0] = g0.x; g[1] = g0.y; g[2] = g0.z; g[3] = g0.w; g[4] = g1.x; g[5] = g1.y; g[6] = g1.z; g[7] = g1.w;
-          iM = a.imax[k]; im = a.imin[k];
-          M = lwc_wt(bf16_to_f(Wrow[iM]), a.s, iM, rr);
-          m = lwc_wt(bf16_to_f(Wrow[im]), a.s, im, rr);
-          qs = omq_qstate(M, m, ga, gb, Q, a.eps);
-          qs.h = a.h[k]; qs.z = (float)a.z[k]; qs.u = __fdiv_rn(__fmul_rn(gb, m), qs.h);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            wt[e] = lwc_wt(w[e], a.s, c * 8 + e, rr);
-            int inr;
-            float dh = omq_ste_dh(wt[e], qs, Q, &inr);
-            Gh = fmaf(g[e], dh, Gh);
-            if (!inr) Gbm += g[e];
-            inr_mask |= inr << e;
-          }
+        for (int e = 0; e < 8; ++e) {
+          const int64_t col = c * 8 + e;
+          float d = ((inr_mask >> e) & 1) ? g[e] : 0.f;
+          if (col == iM) d += GaM * ga;
+          if (col == im) d += Gbt * gb;
+          drm = fmaf(d * w[e], sv[e], drm);
+          if (want_s) acc_s[e] = fmaf(d * w[e], rr, acc_s[e]);
+          g[e] = d;
         }
-        Gh = warp_sum(Gh, lpg);
-        Gbm = warp_sum(Gbm, lpg);
-        if (valid) {
-          if (qs.floored) Gh = 0.f;
-          const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
-          if ((lane & (lpg - 1)) == 0 && a.lwc) {
-            float dg = GaM * M * ga * (1.f - ga), db = Gbt * m * gb * (1.f - gb);
-            if (a.accumulate) { a.dgl[k] += dg; a.dbl[k] += db; } else { a.dgl[k] = dg; a.dbl[k] = db; }
-          }
-          float dwt[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            int64_t col = c * 8 + e;
-            float d = ((inr_mask >> e) & 1) ? g[e] : 0.f;
-            if (col == iM) d += GaM * ga;
-            if (col == im) d += Gbt * gb;
-            dwt[e] = d;
-            float sv = a.s ? a.s[col] : 1.f;
-            dr_part = fmaf(d * w[e], sv, dr_part);
-            if (want_s) acc_s[col] = fmaf(d * w[e], rr, acc_s[col]);
-            if (want_d) acc_d[col] = fmaf(dBo * rr, w[e], acc_d[col]);
-          }
-          if (a.dWt) {
-            float4* dst = reinterpret_cast<float4*>(a.dWt + o * a.Cin) + 2 * c;
-            dst[0] = make_float4(dwt[0], dwt[1], dwt[2], dwt[3]);
-            dst[1] = make_float4(dwt[4], dwt[5], dwt[6], dwt[7]);
-          }
+        if (a.dWt) {
+          float4* dst = reinterpret_cast<float4*>(a.dWt + o * a.Cin) + 2 * c;
+          dst[0] = make_float4(g[0], g[1], g[2], g[3]);
+          dst[1] = make_float4(g[4], g[5], g[6], g[7]);
         }
       }
+      if (a.dr) {
+        drm = warp_sum(drm);
+        if (lane == 0 && wglob < sc.ncw) sc.rowpart[(2 * a.Cout + o) * sc.ncw + wglob] = drm;
+      }
     }
-    if (a.dr) {
-      float2 t = block_sum2(dr_part, 0.f, red_f);
-      if (tid == 0) { if (a.accumulate_dr) a.dr[o] += t.x; else a.dr[o] = t.x; }
-    }
-  }
-  if (want_s || want_d) {
-    __syncthreads();
-    for (int64_t c = tid; c < a.Cin; c += nt) {
-      if (want_s) a.part_s[(int64_t)blockIdx.x * a.Cin + c] = acc_s[c];
-      if (want_d) a.part_d[(int64_t)blockIdx.x * a.Cin + c] = acc_d[c];
+    if (want_d && valid) {
+      const float f = a.dBt[o] * rr;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc_d[e] = fmaf(f, w[e], acc_d[e]);
     }
   }
+  if (valid) {
+    if (want_s) {
+      float4* dst = reinterpret_cast<float4*>(sc.part_s + (int64_t)blockIdx.y * a.Cin) + 2 * c;
+      dst[0] = make_float4(acc_s[0], acc_s[1], acc_s[2], acc_s[3]);
+      dst[1] = make_float4(acc_s[4], acc_s[5], acc_s[6], acc_s[7]);
+    }
+    if (want_d) {
+      float4* dst = reinterpret_cast<float4*>(sc.part_d + (int64_t)blockIdx.y * a.Cin) + 2 * c;
+      dst[0] = make_float4(acc_d[0], acc_d[1], acc_d[2], acc_d[3]);
+      dst[1] = make_float4(acc_d[4], acc_d[5], acc_d[6], acc_d[7]);
+    }
+  }
 }
 
-// rows per CTA so that at most 512 partial rows are written (independent of the device)
-static int64_t lwc_bwd_rows(int64_t Cout) {
-  int64_t rows = (Cout + 511) / 512;
-  return rows < 8 ? 8 : rows;
+// per-row completion: one warp per row sums the warp partials; for one group per row it also
+// forms dgamma, dbeta, the max/min routing of dW~ and of the LET column sum ds.
+__global__ void __launch_bounds__(256) lwc_bwd_finalize_kernel(LwcBwdArgs a, LwcBwdScratch sc) {
+  const int lane = threadIdx.x & 31;
+  const int64_t o = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (o >= a.Cout) return;
+  const bool perch = a.group == a.Cin;
+  float Gh = 0.f, Gbm = 0.f, drm = 0.f;
+  for (int64_t w = lane; w < sc.ncw; w += 32) {
+    if (perch) {
+      Gh += sc.rowpart[(0 * a.Cout + o) * sc.ncw + w];
+      Gbm += sc.rowpart[(1 * a.Cout + o) * sc.ncw + w];
+    }
+    if (a.dr) drm += sc.rowpart[(2 * a.Cout + o) * sc.ncw + w];
+  }
+  Gh = warp_sum(Gh);
+  Gbm = warp_sum(Gbm);
+  drm = warp_sum(drm);
+  if (lane != 0) return;
+  const float rr = a.r ? a.r[o] : 1.f;
+  if (perch) {
+    const float Q = (float)((1 << a.wbits) - 1);
+    const __nv_bfloat16* Wrow = a.W + o * a.Cin;
+    const int iM = a.imax[o], im = a.imin[o];
+    const float ga = lwc_sig(a.ga, a.gl, o, a.lwc), gb = lwc_sig(a.gb, a.bl, o, a.lwc);
+    const float WM = bf16_to_f(Wrow[iM]), Wm = bf16_to_f(Wrow[im]);
+    const float sM = a.s ? a.s[iM] : 1.f, sm = a.s ? a.s[im] : 1.f;
+    const float M = __fmul_rn(__fmul_rn(WM, sM), rr), m = __fmul_rn(__fmul_rn(Wm, sm), rr);
+    const float hr = __fdiv_rn(__fsub_rn(__fmul_rn(ga, M), __fmul_rn(gb, m)), Q);
+    if (!(hr >= a.eps)) Gh = 0.f;
+    const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
+    if (a.lwc) {
+      const float dg = GaM * M * ga * (1.f - ga), db = Gbt * m * gb * (1.f - gb);
+      if (a.accumulate) { a.dgl[o] += dg; a.dbl[o] += db; } else { a.dgl[o] = dg; a.dbl[o] = db; }
+    }
+    const float rM = GaM * ga, rm = Gbt * gb;          // routing of dW~ to the max / min element
+    drm += rM * WM * sM + rm * Wm * sm;
+    if (a.ds) {
+      atomicAdd(a.ds + iM, rM * WM * rr);
+      atomicAdd(a.ds + im, rm * Wm * rr);
+    }
+    if (a.dWt) {
+      a.dWt[o * a.Cin + iM] += rM;
+      a.dWt[o * a.Cin + im] += rm;
+    }
+  }
+  if (a.dr) { if (a.accumulate_dr) a.dr[o] += drm; else a.dr[o] = drm; }
 }
 
-int64_t lwc_bwd_nslab(int64_t Cout) {
-  const int64_t rows = lwc_bwd_rows(Cout);
-  return (Cout + rows - 1) / rows;
-}
-
-omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a0, int64_t* nslab_out) {
+omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a0, void* scratch) {
   OMQ_REQUIRE(lwc_group_ok(a0.Cin, a0.group), OMQ_ERR_UNSUPPORTED);
+  OMQ_REQUIRE(scratch, OMQ_ERR_WORKSPACE);
   LwcBwdArgs a = a0;
-  a.rows_per_cta = (int)lwc_bwd_rows(a.Cout);
-  int64_t nslab = lwc_bwd_nslab(a.Cout);
-  size_t smem = (a.part_s || a.part_d) ? 2 * a.Cin * sizeof(float) : 0;
-  OMQ_REQUIRE(smem <= 200 * 1024, OMQ_ERR_UNSUPPORTED);
-  if (smem + 2048 > 48 * 1024) cudaFuncSetAttribute(lwc_bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  lwc_bwd_kernel<<<(unsigned)nslab, lwc_threads(a.Cin), smem, st>>>(a);
+  const bool perch = a.group == a.Cin;
+  const int64_t ng = a.Cin / a.group;
+  LwcBwdScratch sc = lwc_bwd_carve(scratch, a.Cout, a.Cin, ng, nullptr);
+  if (a.lwc && (!a.ga || !a.gb)) {           // one sigmoid per group, not one per element
+    const int64_t n = a.Cout * ng;
+    sigmoid_pair_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(a.gl, a.bl, n, sc.sig, sc.sig + n);
+    OMQ_LAUNCH_CHECK();
+    a.ga = sc.sig;
+    a.gb = sc.sig + n;
+  }
+  const int64_t ncol = (a.Cin / 8 + LWC_BWD_THREADS - 1) / LWC_BWD_THREADS;
+  dim3 grid((unsigned)ncol, (unsigned)sc.nrt);
+  lwc_bwd_tile_kernel<<<grid, LWC_BWD_THREADS, 0, st>>>(a, sc);
   OMQ_LAUNCH_CHECK();
-  if (nslab_out) *nslab_out = nslab;
+  // the LET column sums first, so that the finalize can add the max/min routing on top
+  if (a.ds) OMQ_TRY(omq_colsum_partials(st, sc.part_s, sc.nrt, a.Cin, a.ds, 1.f, a.accumulate_sd));
+  if (a.ddelta && a.dBt) OMQ_TRY(omq_colsum_partials(st, sc.part_d, sc.nrt, a.Cin, a.ddelta, 1.f, a.accumulate_sd));
+  if (perch || a.dr) {
+    lwc_bwd_finalize_kernel<<<(unsigned)((a.Cout + 7) / 8), 256, 0, st>>>(a, sc);
+    OMQ_LAUNCH_CHECK();
+  }
   return OMQ_OK;
 }
 
@@ -902,9 +964,7 @@ omq_status omq_lwc_fakequant_fwd(omq_stream_t stream, int64_t Cout, int64_t Cin,
   return lwc_fwd_launch((cudaStream_t)stream, a);
 }
 
-size_t omq_lwc_bwd_workspace_size(int64_t Cout, int64_t Cin) {
-  return (size_t)(2 * lwc_bwd_nslab(Cout) * Cin) * sizeof(float) + 256;
-}
+size_t omq_lwc_bwd_workspace_size(int64_t Cout, int64_t Cin) { return lwc_bwd_scratch_bytes(Cout, Cin); }
 
 omq_status omq_lwc_fakequant_bwd(omq_stream_t stream, int64_t Cout, int64_t Cin, const void* W, const float* s,
                                  const float* r, const float* gamma_logit, const float* beta_logit, const float* h,
@@ -916,29 +976,21 @@ omq_status omq_lwc_fakequant_bwd(omq_stream_t stream, int64_t Cout, int64_t Cin,
   OMQ_REQUIRE(cfg->wbits < 16, OMQ_ERR_UNSUPPORTED);
   OMQ_REQUIRE(W && dWq && h && z && argmax && argmin && gamma_logit && beta_logit && dgamma && dbeta, OMQ_ERR_INVALID_ARG);
   OMQ_REQUIRE(Cin % 8 == 0 && omq_aligned16(W) && omq_aligned16(dWq) && (!dWt || omq_aligned16(dWt)), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(!s || omq_aligned16(s), OMQ_ERR_ALIGN);
   const int g = cfg->group == 0 ? (int)Cin : cfg->group;
   OMQ_REQUIRE(Cin % g == 0, OMQ_ERR_SHAPE);
   OMQ_REQUIRE(!ddelta || dBt, OMQ_ERR_INVALID_ARG);
-  const bool need_ws = ds || ddelta;
-  if (need_ws) {
-    OMQ_REQUIRE(workspace && ws_bytes >= omq_lwc_bwd_workspace_size(Cout, Cin), OMQ_ERR_WORKSPACE);
-    OMQ_REQUIRE(omq_aligned16(workspace), OMQ_ERR_ALIGN);
-  }
-  cudaStream_t st = (cudaStream_t)stream;
-  const int64_t nslab = lwc_bwd_nslab(Cout);
-  float* part_s = need_ws ? (float*)workspace : nullptr;
-  float* part_d = need_ws ? (float*)workspace + nslab * Cin : nullptr;
+  OMQ_REQUIRE(workspace && ws_bytes >= omq_lwc_bwd_workspace_size(Cout, Cin), OMQ_ERR_WORKSPACE);
+  OMQ_REQUIRE(omq_aligned16(workspace), OMQ_ERR_ALIGN);
   LwcBwdArgs a{};
   a.W = (const __nv_bfloat16*)W; a.Cout = Cout; a.Cin = Cin; a.group = g; a.s = s; a.r = r;
-  a.gl = gamma_logit; a.bl = beta_logit; a.lwc = 1; a.h = h; a.z = z; a.imax = argmax; a.imin = argmin;
+  a.gl = gamma_logit; a.bl = beta_logit; a.lwc = 1; a.ga = nullptr; a.gb = nullptr;
+  a.h = h; a.z = z; a.imax = argmax; a.imin = argmin;
   a.dWq = dWq; a.ld_dwq = Cin; a.dgl = dgamma; a.dbl = dbeta; a.dWt = dWt; a.dr = dr; a.dBt = dBt;
-  a.part_s = ds ? part_s : nullptr; a.part_d = ddelta ? part_d : nullptr;
-  a.wbits = cfg->wbits; a.eps = cfg->h_eps; a.accumulate = cfg->accumulate; a.accumulate_dr = cfg->accumulate;
-  int64_t ns = 0;
-  OMQ_TRY(lwc_bwd_launch(st, a, &ns));
-  if (ds) OMQ_TRY(omq_colsum_partials(st, part_s, ns, Cin, ds, 1.f, cfg->accumulate));
-  if (ddelta) OMQ_TRY(omq_colsum_partials(st, part_d, ns, Cin, ddelta, 1.f, cfg->accumulate));
-  return OMQ_OK;
+  a.ds = ds; a.ddelta = ddelta;
+  a.wbits = cfg->wbits; a.eps = cfg->h_eps; a.accumulate = cfg->accumulate; a.accumulate_sd = cfg->accumulate;
+  a.accumulate_dr = cfg->accumulate;
+  return lwc_bwd_launch((cudaStream_t)stream, a, workspace);
 }
 
 omq_status omq_act_quant_per_token(omq_stream_t stream, int64_t T, int64_t C, const float* X, const float* s,

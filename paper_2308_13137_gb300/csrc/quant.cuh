@@ -11,25 +11,27 @@ struct LwcFwdArgs {
   __nv_bfloat16* Wq; uint8_t* codes;
   float* h; int32_t* z; int32_t* imax; int32_t* imin;
   const float* bias_delta; const float* bias_shift; float* Bt;
+  float* ga_out; float* gb_out;                            // clipping strengths per group (nullable)
   int wbits; float eps;
   int32_t* status;
 };
 omq_status lwc_fwd_launch(cudaStream_t st, const LwcFwdArgs& a);
 
 struct LwcBwdArgs {
-  const __nv_bfloat16* W; int64_t Cout, Cin; int group;
+  const __nv_bfloat16* W; int64_t Cout, Cin; int group;    // group = Cin for per-channel
   const float* s; const float* r;
   const float* gl; const float* bl; int lwc;
+  const float* ga; const float* gb;                        // saved sigmoids (nullable: recomputed)
   const float* h; const int32_t* z; const int32_t* imax; const int32_t* imin;
   const float* dWq; int64_t ld_dwq;
   float* dgl; float* dbl; float* dWt; float* dr;
   const float* dBt;
-  float* part_s; float* part_d;          // [nslab, Cin] partial column sums (nullable)
-  int rows_per_cta;
-  int wbits; float eps; int accumulate; int accumulate_dr;
+  float* ds; float* ddelta;                                // LET column sums (nullable)
+  int wbits; float eps; int accumulate; int accumulate_sd; int accumulate_dr;
 };
-omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a, int64_t* nslab_out);
-int64_t lwc_bwd_nslab(int64_t Cout);
+// scratch: partial column sums and per-row partials, carved from `scratch`
+size_t lwc_bwd_scratch_bytes(int64_t Cout, int64_t Cin);
+omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a, void* scratch);
 
 // ---- per-token activation quantizer Q_a with a fused producer ------------------------------
 enum ActProducer { AP_PLAIN = 0, AP_LET = 1, AP_RMS_LET = 2, AP_SWIGLU = 3 };
