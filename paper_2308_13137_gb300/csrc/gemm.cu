@@ -137,6 +137,32 @@ struct SmemLayout {
   static constexpr int TOTAL = BAR_OFF + 256 + 1024;  // + barriers + alignment slack
 };
 
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// Tile t of the launch (m fastest, then n, then batch) and its K range.
+struct TileInfo { int m0, n0, b, k_begin, nkb; bool skip; };
+
+__device__ __forceinline__ TileInfo tile_info(const GemmParams& p, int t, int bn) {
+  const int mt = (p.M + BM - 1) / BM, nt = (p.N + bn - 1) / bn;
+  TileInfo ti;
+  ti.m0 = (t % mt) * BM;
+  ti.n0 = ((t / mt) % nt) * bn;
+  ti.b = t / (mt * nt);
+  ti.skip = (p.causal == 1 && ti.n0 > ti.m0 + BM - 1);   // keys beyond every query of the tile
+  int k_end = p.K;
+  ti.k_begin = 0;
+  if (p.causal == 2) k_end = min(p.K, ti.m0 + BM);
+  if (p.causal == 3) ti.k_begin = ti.m0;
+  ti.nkb = k_end > ti.k_begin ? (k_end - ti.k_begin + BK - 1) / BK : 0;
+  return ti;
+}
+
+// Persistent kernel: one CTA per SM walks tiles blockIdx.x, blockIdx.x + gridDim.x, ...
+// The shared-memory ring runs continuously across tiles; the accumulator is double-buffered
+// in tensor memory (2 x BN columns) so that the epilogue of one tile overlaps the MMAs of
+// the next.
 template <int BN, int STAGES>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -146,27 +172,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L::BAR_OFF);
   uint64_t* empty = full + STAGES;
-  uint64_t* accum = empty + STAGES;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(accum + 1);
+  uint64_t* acc_full = empty + STAGES;     // [2]
+  uint64_t* acc_empty = acc_full + 2;      // [2]
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(acc_empty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN, b = blockIdx.z;
-
-  // causal tile skip (scores / their gradient): keys beyond every query of the tile
-  if (p.causal == 1 && n0 > m0 + BM - 1) return;
-  int k_begin = 0, k_end = p.K;
-  if (p.causal == 2) k_end = min(p.K, m0 + BM);
-  if (p.causal == 3) k_begin = m0;
-  const int nkb = k_end > k_begin ? (k_end - k_begin + BK - 1) / BK : 0;
+  const int mt = (p.M + BM - 1) / BM, nt = (p.N + BN - 1) / BN;
+  const int total = mt * nt * p.batch;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
-    mbar_init(accum, 1);
+    for (int b = 0; b < 2; ++b) { mbar_init(&acc_full[b], 1); mbar_init(&acc_empty[b], 4); }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 1) tmem_alloc(tmem_holder, BN);
+  if (warp == 1) tmem_alloc(tmem_holder, 2 * BN);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -174,132 +195,164 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer ----------------
-    for (int kb = 0; kb < nkb; ++kb) {
-      const int s = kb % STAGES;
-      if (kb >= STAGES) {
-        if (!mbar_wait(&empty[s], ((kb / STAGES) - 1) & 1)) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; break; }
-      }
-      if (*abort_flag) break;
-      uint8_t* sa = smem + s * L::STAGE_BYTES;
-      uint8_t* sb = sa + L::A_BYTES;
-      const int k0 = k_begin + kb * BK;
-      mbar_expect_tx(&full[s], L::STAGE_BYTES);
-      if (!p.a_mn) {
-        tma_load_3d(&tmA, &full[s], sa, k0, m0, b);
-      } else {
-        tma_load_3d(&tmA, &full[s], sa, m0, k0, b);
-        tma_load_3d(&tmA, &full[s], sa + 64 * BK * 2, m0 + 64, k0, b);
-      }
-      if (!p.b_mn) {
-        tma_load_3d(&tmB, &full[s], sb, k0, n0, b);
-      } else {
+    uint32_t it = 0;
+    for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
+      const TileInfo ti = tile_info(p, t, BN);
+      if (ti.skip) continue;
+      for (int kb = 0; kb < ti.nkb; ++kb, ++it) {
+        const int s = it % STAGES;
+        if (!mbar_wait(&empty[s], ((it / STAGES) & 1) ^ 1)) {
+          omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; break;
+        }
+        uint8_t* sa = smem + s * L::STAGE_BYTES;
+        uint8_t* sb = sa + L::A_BYTES;
+        const int k0 = ti.k_begin + kb * BK;
+        mbar_expect_tx(&full[s], L::STAGE_BYTES);
+        if (!p.a_mn) {
+          tma_load_3d(&tmA, &full[s], sa, k0, ti.m0, ti.b);
+        } else {
+          tma_load_3d(&tmA, &full[s], sa, ti.m0, k0, ti.b);
+          tma_load_3d(&tmA, &full[s], sa + 64 * BK * 2, ti.m0 + 64, k0, ti.b);
+        }
+        if (!p.b_mn) {
+          tma_load_3d(&tmB, &full[s], sb, k0, ti.n0, ti.b);
+        } else {
 #pragma unroll
-        for (int j = 0; j < BN / 64; ++j) tma_load_3d(&tmB, &full[s], sb + j * 64 * BK * 2, n0 + 64 * j, k0, b);
+          for (int j = 0; j < BN / 64; ++j) tma_load_3d(&tmB, &full[s], sb + j * 64 * BK * 2, ti.n0 + 64 * j, k0, ti.b);
+        }
       }
     }
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer ----------------
     constexpr uint32_t IDESC_KK = idesc_bf16(BM, BN, 0, 0);
     const uint32_t idesc = IDESC_KK | ((uint32_t)p.a_mn << 15) | ((uint32_t)p.b_mn << 16);
-    for (int kb = 0; kb < nkb; ++kb) {
-      const int s = kb % STAGES;
-      if (!mbar_wait(&full[s], (kb / STAGES) & 1)) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; break; }
-      tc_fence_after();
-      const uint32_t sa = smem_u32(smem + s * L::STAGE_BYTES);
-      const uint32_t sb = sa + L::A_BYTES;
-#pragma unroll
-      for (int k = 0; k < BK / UMMA_K; ++k) {
-        // K-major: advance 32 bytes inside the swizzle row; MN-major: advance 16 K-rows (2 KB)
-        const uint64_t ad = p.a_mn ? sdesc(sa + k * 2048, 64 * BK * 2, 1024) : sdesc(sa + k * 32, 16, 1024);
-        const uint64_t bd = p.b_mn ? sdesc(sb + k * 2048, 64 * BK * 2, 1024) : sdesc(sb + k * 32, 16, 1024);
-        umma_bf16(tmem, ad, bd, idesc, (kb | k) != 0);
+    uint32_t it = 0, acc_it = 0;
+    for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
+      const TileInfo ti = tile_info(p, t, BN);
+      if (ti.skip || ti.nkb == 0) continue;
+      const uint32_t buf = acc_it & 1;
+      if (!mbar_wait(&acc_empty[buf], ((acc_it >> 1) & 1) ^ 1)) {
+        omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; break;
       }
-      umma_commit(&empty[s]);
+      tc_fence_after();
+      const uint32_t d_tmem = tmem + buf * BN;
+      bool ok = true;
+      for (int kb = 0; kb < ti.nkb; ++kb, ++it) {
+        const int s = it % STAGES;
+        if (!mbar_wait(&full[s], (it / STAGES) & 1)) {
+          omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; ok = false; break;
+        }
+        tc_fence_after();
+        const uint32_t sa = smem_u32(smem + s * L::STAGE_BYTES);
+        const uint32_t sb = sa + L::A_BYTES;
+#pragma unroll
+        for (int k = 0; k < BK / UMMA_K; ++k) {
+          // K-major: advance 32 bytes inside the swizzle row; MN-major: advance 16 K-rows (2 KB)
+          const uint64_t ad = p.a_mn ? sdesc(sa + k * 2048, 64 * BK * 2, 1024) : sdesc(sa + k * 32, 16, 1024);
+          const uint64_t bd = p.b_mn ? sdesc(sb + k * 2048, 64 * BK * 2, 1024) : sdesc(sb + k * 32, 16, 1024);
+          umma_bf16(d_tmem, ad, bd, idesc, (kb | k) != 0);
+        }
+        umma_commit(&empty[s]);
+      }
+      umma_commit(&acc_full[buf]);
+      ++acc_it;
+      if (!ok) break;
     }
-    umma_commit(accum);
   } else if (warp >= 2) {
     // ---------------- epilogue ----------------
     const int q = warp & 3;                       // TMEM lane quadrant of this warp
-    const int row = m0 + q * 32 + lane;
-    bool ok = true;
-    if (nkb > 0) {
-      ok = __all_sync(0xffffffffu, mbar_wait(accum, 0));   // tcgen05.ld below is warp-collective
-      if (!ok) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; }
-      tc_fence_after();
-    }
     const GemmEpilogue& ep = p.ep;
-    const bool row_ok = row < p.M;
-    const int64_t crow = (int64_t)b * ep.c_bs + (int64_t)row * ep.ldc;
+    uint32_t acc_it = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+      const TileInfo ti = tile_info(p, t, BN);
+      if (ti.skip) continue;
+      const bool has_acc = ti.nkb > 0;
+      const uint32_t buf = acc_it & 1;
+      bool ok = true;
+      if (has_acc) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[buf], (acc_it >> 1) & 1));  // tcgen05.ld is warp-wide
+        if (!ok) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; }
+        tc_fence_after();
+      }
+      const int row = ti.m0 + q * 32 + lane;
+      const bool row_ok = row < p.M;
+      const int64_t crow = (int64_t)ti.b * ep.c_bs + (int64_t)row * ep.ldc;
 #pragma unroll 1
-    for (int j0 = 0; j0 < BN; j0 += 32) {
-      float v[32];
-      if (nkb > 0 && ok) {
-        tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)j0, v);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = 0.f;
-      }
-      const int nb = n0 + j0;
-      if (!row_ok || nb >= p.N) continue;
-      const bool full_chunk = nb + 32 <= p.N;
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        v[i] *= ep.alpha;
-      }
-      if (full_chunk) {
-        if (ep.bias) {
-#pragma unroll
-          for (int i = 0; i < 32; i += 4) {
-            float4 bb = __ldg(reinterpret_cast<const float4*>(ep.bias + nb + i));
-            v[i] += bb.x; v[i + 1] += bb.y; v[i + 2] += bb.z; v[i + 3] += bb.w;
+      for (int j0 = 0; j0 < BN; j0 += 32) {
+        float v[32];
+        if (has_acc && ok) {
+          tmem_ld32(tmem + buf * BN + ((uint32_t)(q * 32) << 16) + (uint32_t)j0, v);
+          if (j0 + 32 == BN) {                    // accumulator drained: hand the buffer back
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acc_empty[buf]);
           }
-        }
-        if (ep.R) {
-          const float* rr = ep.R + (int64_t)b * ep.c_bs + (int64_t)row * ep.ldr + nb;
+        } else {
 #pragma unroll
-          for (int i = 0; i < 32; i += 4) {
-            float4 t = __ldg(reinterpret_cast<const float4*>(rr + i));
-            v[i] += t.x; v[i + 1] += t.y; v[i + 2] += t.z; v[i + 3] += t.w;
-          }
+          for (int i = 0; i < 32; ++i) v[i] = 0.f;
         }
-        if (ep.Cf) {
-          float* cp = ep.Cf + crow + nb;
-          if (ep.beta_acc != 0.f) {
+        const int nb = ti.n0 + j0;
+        if (!row_ok || nb >= p.N) continue;
+        const bool full_chunk = nb + 32 <= p.N;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] *= ep.alpha;
+        if (full_chunk) {
+          if (ep.bias) {
 #pragma unroll
             for (int i = 0; i < 32; i += 4) {
-              float4 t = *reinterpret_cast<const float4*>(cp + i);
-              v[i] += ep.beta_acc * t.x; v[i + 1] += ep.beta_acc * t.y;
-              v[i + 2] += ep.beta_acc * t.z; v[i + 3] += ep.beta_acc * t.w;
+              float4 bb = __ldg(reinterpret_cast<const float4*>(ep.bias + nb + i));
+              v[i] += bb.x; v[i + 1] += bb.y; v[i + 2] += bb.z; v[i + 3] += bb.w;
             }
           }
+          if (ep.R) {
+            const float* rr = ep.R + (int64_t)ti.b * ep.c_bs + (int64_t)row * ep.ldr + nb;
 #pragma unroll
-          for (int i = 0; i < 32; i += 4) *reinterpret_cast<float4*>(cp + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
-        }
-        if (ep.Cb) {
-          __nv_bfloat16* cp = ep.Cb + crow + nb;
-#pragma unroll
-          for (int i = 0; i < 32; i += 8) *reinterpret_cast<uint4*>(cp + i) = pack_bf16x8(v + i);
-        }
-      } else {
-        for (int i = 0; i < 32 && nb + i < p.N; ++i) {
-          const int n = nb + i;
-          float x = v[i];
-          if (ep.bias) x += ep.bias[n];
-          if (ep.R) x += ep.R[(int64_t)b * ep.c_bs + (int64_t)row * ep.ldr + n];
-          if (ep.Cf) {
-            if (ep.beta_acc != 0.f) x += ep.beta_acc * ep.Cf[crow + n];
-            ep.Cf[crow + n] = x;
+            for (int i = 0; i < 32; i += 4) {
+              float4 tt = __ldg(reinterpret_cast<const float4*>(rr + i));
+              v[i] += tt.x; v[i + 1] += tt.y; v[i + 2] += tt.z; v[i + 3] += tt.w;
+            }
           }
-          if (ep.Cb) ep.Cb[crow + n] = f_to_bf16(x);
+          if (ep.Cf) {
+            float* cp = ep.Cf + crow + nb;
+            if (ep.beta_acc != 0.f) {
+#pragma unroll
+              for (int i = 0; i < 32; i += 4) {
+                float4 tt = *reinterpret_cast<const float4*>(cp + i);
+                v[i] += ep.beta_acc * tt.x; v[i + 1] += ep.beta_acc * tt.y;
+                v[i + 2] += ep.beta_acc * tt.z; v[i + 3] += ep.beta_acc * tt.w;
+              }
+            }
+#pragma unroll
+            for (int i = 0; i < 32; i += 4) *reinterpret_cast<float4*>(cp + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+          }
+          if (ep.Cb) {
+            __nv_bfloat16* cp = ep.Cb + crow + nb;
+#pragma unroll
+            for (int i = 0; i < 32; i += 8) *reinterpret_cast<uint4*>(cp + i) = pack_bf16x8(v + i);
+          }
+        } else {
+          for (int i = 0; i < 32 && nb + i < p.N; ++i) {
+            const int n = nb + i;
+            float x = v[i];
+            if (ep.bias) x += ep.bias[n];
+            if (ep.R) x += ep.R[(int64_t)ti.b * ep.c_bs + (int64_t)row * ep.ldr + n];
+            if (ep.Cf) {
+              if (ep.beta_acc != 0.f) x += ep.beta_acc * ep.Cf[crow + n];
+              ep.Cf[crow + n] = x;
+            }
+            if (ep.Cb) ep.Cb[crow + n] = f_to_bf16(x);
+          }
         }
       }
+      if (has_acc) ++acc_it;
+      if (!ok) break;
     }
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, BN);
+    tmem_dealloc(tmem, 2 * BN);
   }
 }
 
@@ -347,7 +400,9 @@ omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap&
       return OMQ_ERR_CUDA;
     attr_set = true;
   }
-  dim3 grid((unsigned)((p.M + BM - 1) / BM), (unsigned)((p.N + BN - 1) / BN), (unsigned)p.batch);
+  const int64_t tiles = (int64_t)((p.M + BM - 1) / BM) * ((p.N + BN - 1) / BN) * p.batch;
+  const int64_t sms = omq_num_sms();
+  const unsigned grid = (unsigned)(tiles < sms ? tiles : sms);
   gemm_bf16_kernel<BN, STAGES><<<grid, NUM_THREADS, L::TOTAL, st>>>(ta, tb, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
