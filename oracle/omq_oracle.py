@@ -51,8 +51,10 @@ notes of the repository):
  R15 where floating point decides an integer (a code, a zero point, a max/min
      index, the floor of h) the decision is taken in the precision of the
      kernels, IEEE single precision with one rounding per product, difference and
-     quotient, and the sigmoid rounded once from double; everything else stays
-     float64.  ("emulate" mode; "exact" mode decides in float64.)
+     quotient, the division by h formed as a product with the correctly rounded
+     reciprocal of h; the clipping strengths entering it are the single-precision sigmoid
+     of `sigmoid_fp32`.  Everything else stays float64.  ("emulate" mode; "exact"
+     mode decides in float64.)
 """
 from __future__ import annotations
 
@@ -68,7 +70,7 @@ __all__ = [
     "rne", "to_bf16", "sigmoid", "quant_fwd", "quant_bwd", "quant_ste", "codes_from_scale",
     "lwc_fakequant_fwd", "lwc_fakequant_bwd", "act_quant_per_token", "act_quant_per_token_bwd",
     "let_apply", "block_loss", "qlinear_step", "BlockCfg", "block_forward", "block_step",
-    "rmsnorm", "rope", "silu", "FrozenTape", "use_tape", "block_fp_forward",
+    "rmsnorm", "rope", "silu", "FrozenTape", "use_tape", "block_fp_forward", "sigmoid_fp32",
     "THETA_NAMES_LWC", "THETA_NAMES_LET",
 ]
 
@@ -95,6 +97,30 @@ def sigmoid(t: torch.Tensor) -> torch.Tensor:
     return 1.0 / (1.0 + torch.exp(-t))
 
 
+_LOG2E32 = 1.44269502162933349609375        # float32 nearest to log2(e)
+_LN2_HI = 0.693145751953125                 # 15-bit head of ln 2: n * head is exact
+_LN2_LO = 1.428606765330187e-06             # float32 tail, head + tail = ln 2 to 5e-14
+_EXP_TAYLOR = [1.98412701138295233249664e-04, 1.38888892251998186111450e-03, 8.33333376795053482055664e-03,
+               4.16666679084300994873047e-02, 1.66666671633720397949219e-01, 0.5, 1.0, 1.0]   # 1/7!, ..., 1/0!
+
+
+def sigmoid_fp32(t: torch.Tensor) -> torch.Tensor:
+    """sigmoid(t) as the kernels evaluate it in single precision (R15), one rounding per
+    operation: exp(-t) by Cody-Waite reduction -t = n ln2 + r, the degree-7 Taylor polynomial of
+    exp(r) in Horner form and an exact scaling by 2^n, then 1 / (1 + exp(-t)); |t| clamped to 80.
+    Returns float32."""
+    f32 = torch.float32
+    x = -torch.clamp(torch.as_tensor(t).to(f32), -80.0, 80.0)
+    n = torch.round(x * _LOG2E32)
+    r = (x - n * _LN2_HI) - n * _LN2_LO
+    p = torch.full_like(r, _EXP_TAYLOR[0])
+    for c in _EXP_TAYLOR[1:]:
+        p = p * r + c
+    two_n = ((n.to(torch.int32) + 127) << 23).view(f32)       # 2^n, exact
+    e = p * two_n
+    return 1.0 / (1.0 + e)
+
+
 def _first_argmax(w: torch.Tensor) -> torch.Tensor:
     """Index of the first maximum along the last axis (R7)."""
     M = w.max(dim=-1, keepdim=True).values
@@ -112,16 +138,17 @@ def _first_argmin(w: torch.Tensor) -> torch.Tensor:
 # Eq. 2, explicit forward and STE backward of one quantizer over groups on the last axis
 # ----------------------------------------------------------------------------------------------
 
-def _decide_fp32(w: torch.Tensor, a, b, Q: float, eps: float):
+def _decide_fp32(w: torch.Tensor, a, b, Q: float, eps: float, a32=None, b32=None):
     """The integer decisions of Eq. 2 taken in IEEE single precision (R15).
 
     Inputs are rounded to fp32 and every product, difference and quotient is rounded to fp32:
-    h = (a*M - b*m)/Q, u = (b*m)/h, x = w/h.  Returns the first argmax/argmin of the fp32
-    group, the floor flag and h, u, x as fp32 values."""
+    h = (a*M - b*m)/Q, r = 1/h, u = (b*m)*r, x = w*r; a32, b32 (default: a, b rounded) are the
+    single-precision clipping strengths.  Returns the first argmax/argmin of the fp32 group,
+    the floor flag and h, u, x as fp32 values."""
     f32 = torch.float32
     w32 = w.detach().to(f32)
-    a32 = torch.as_tensor(a).detach().to(f32)
-    b32 = torch.as_tensor(b).detach().to(f32)
+    a32 = torch.as_tensor(a).detach().to(f32) if a32 is None else torch.as_tensor(a32).to(f32)
+    b32 = torch.as_tensor(b).detach().to(f32) if b32 is None else torch.as_tensor(b32).to(f32)
     imax = _first_argmax(w32)
     imin = _first_argmin(w32)
     M32 = torch.gather(w32, -1, imax[..., None])[..., 0]
@@ -131,12 +158,14 @@ def _decide_fp32(w: torch.Tensor, a, b, Q: float, eps: float):
     hr = (aM - bm) / Q
     floored = hr < eps
     h32 = torch.where(floored, torch.full_like(hr, eps), hr)
-    u32 = bm / h32
-    x32 = w32 / h32[..., None]
+    rh32 = 1.0 / h32                       # correctly rounded reciprocal
+    u32 = bm * rh32
+    x32 = w32 * rh32[..., None]
     return imax, imin, floored, h32, u32, x32
 
 
-def quant_fwd(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5, decide: str = "fp64") -> Dict[str, torch.Tensor]:
+def quant_fwd(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5, decide: str = "fp64",
+              a32=None, b32=None) -> Dict[str, torch.Tensor]:
     """Eq. 2 over groups laid out on the last axis of `w` (shape [..., g]).
 
     a, b are the clipping strengths gamma, beta (tensors of shape [...] or floats; 1.0 gives
@@ -148,7 +177,7 @@ def quant_fwd(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5, decide: str 
     a = torch.as_tensor(a, dtype=F64)
     b = torch.as_tensor(b, dtype=F64)
     if decide == "fp32":
-        imax, imin, floored, h32, u32, x32 = _decide_fp32(w, a, b, Q, eps)
+        imax, imin, floored, h32, u32, x32 = _decide_fp32(w, a, b, Q, eps, a32, b32)
         M = torch.gather(w, -1, imax[..., None])[..., 0]
         m = torch.gather(w, -1, imin[..., None])[..., 0]
         h, u, x = h32.to(F64), u32.to(F64), x32.to(F64)
@@ -249,7 +278,7 @@ class use_tape:
 
 
 def quant_ste(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5, decide: str = "fp64",
-              w_dec: Optional[torch.Tensor] = None) -> torch.Tensor:
+              w_dec: Optional[torch.Tensor] = None, a32=None, b32=None) -> torch.Tensor:
     """Eq. 2 fake quantization as an autograd graph whose gradient is the STE of R7.
 
     Groups on the last axis; a, b broadcast against w[..., 0] (tensors that may require
@@ -273,7 +302,8 @@ def quant_ste(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5, decide: str 
     if decide == "fp32":
         assert tape is None, "the frozen-offset surrogate is defined for float64 decisions"
         with torch.no_grad():
-            imax, imin, floored, h32, u32, x32 = _decide_fp32(w if w_dec is None else w_dec, a, b, Q, eps)
+            imax, imin, floored, h32, u32, x32 = _decide_fp32(w if w_dec is None else w_dec, a, b, Q, eps,
+                                                              a32, b32)
         M = torch.gather(w, -1, imax[..., None])[..., 0]
         m = torch.gather(w, -1, imin[..., None])[..., 0]
         h_raw = (a * M - b * m) / Q
@@ -359,7 +389,9 @@ def lwc_fakequant_fwd(W, gamma_logit, beta_logit, nbits: int, group: int,
     G = _groups(Wt, group)
     a = sigmoid(gamma_logit.to(F64))
     b = sigmoid(beta_logit.to(F64))
-    st = quant_fwd(G, a, b, nbits, eps, decide)
+    a32 = sigmoid_fp32(gamma_logit) if decide == "fp32" else None
+    b32 = sigmoid_fp32(beta_logit) if decide == "fp32" else None
+    st = quant_fwd(G, a, b, nbits, eps, decide, a32, b32)
     gsz = G.shape[-1]
     base = torch.arange(G.shape[1], dtype=torch.int64)[None, :] * gsz
     return dict(st=st, Wt=Wt, h=st["h"], z=st["z"], argmax=st["imax"] + base, argmin=st["imin"] + base,
@@ -497,8 +529,10 @@ def qlinear_step(X, W, B, gamma_logit, beta_logit, Yfp, wbits: int, group: int, 
     cout, cin = W.shape
     gsz = cin if group == 0 else group
     wd = _dec32(W, sv).reshape(cout, cin // gsz, gsz)
+    a32 = sigmoid_fp32(gl.detach()) if decide == "fp32" else None
+    b32 = sigmoid_fp32(bl.detach()) if decide == "fp32" else None
     Wh = quant_ste(Wt.reshape(cout, cin // gsz, gsz), sigmoid(gl), sigmoid(bl), wbits, eps, decide,
-                   wd).reshape(cout, cin)
+                   wd, a32, b32).reshape(cout, cin)
     Y = _mm(Xh, Wh, mode) + Bt
     loss, _ = block_loss(Y, Yfp)
     grads = torch.autograd.grad(loss, leaves)
@@ -577,8 +611,11 @@ def _qw(Wt, gl, bl, cfg: BlockCfg, w_dec=None):
     cout, cin = Wt.shape
     gsz = cin if cfg.group == 0 else cfg.group
     dec = None if w_dec is None else w_dec.reshape(cout, cin // gsz, gsz)
+    fp32 = _decide(cfg) == "fp32"
+    a32 = sigmoid_fp32(gl.detach()) if fp32 else None
+    b32 = sigmoid_fp32(bl.detach()) if fp32 else None
     return quant_ste(Wt.reshape(cout, cin // gsz, gsz), sigmoid(gl), sigmoid(bl),
-                     cfg.wbits, cfg.h_eps, _decide(cfg), dec).reshape(cout, cin)
+                     cfg.wbits, cfg.h_eps, _decide(cfg), dec, a32, b32).reshape(cout, cin)
 
 
 def _qa(X, cfg: BlockCfg):

@@ -62,6 +62,7 @@ __global__ void __launch_bounds__(512) qkv_fwd_kernel(QkvArgs a) {
     const int W = seg == 0 ? dq : dkv;
     __nv_bfloat16* out = seg == 0 ? a.Qh + (int64_t)t * dq : (seg == 1 ? a.Kh + (int64_t)t * dkv : a.Vh + (int64_t)t * dkv);
     MaxMin r = mm_identity();
+    #pragma unroll 4
     for (int i = tid; i < W; i += nt) {
       float v = qkv_value(a, seg, t, i).xt;
       row[i] = v;
@@ -69,6 +70,7 @@ __global__ void __launch_bounds__(512) qkv_fwd_kernel(QkvArgs a) {
     }
     if (a.abits >= 16) {
       __syncthreads();
+      #pragma unroll 4
       for (int i = tid; i < W; i += nt) out[i] = f_to_bf16(row[i]);
       __syncthreads();
       continue;
@@ -78,6 +80,7 @@ __global__ void __launch_bounds__(512) qkv_fwd_kernel(QkvArgs a) {
     QState qs = omq_qstate(r.M, r.m, 1.f, 1.f, Q, a.eps);
     const int64_t k = (int64_t)seg * a.T + t;
     if (tid == 0) { a.h[k] = qs.h; a.z[k] = (int32_t)qs.z; a.imax[k] = r.iM; a.imin[k] = r.im; }
+    #pragma unroll 4
     for (int i = tid; i < W; i += nt) {
       float c;
       out[i] = f_to_bf16(omq_fakequant(row[i], qs, Q, &c));
@@ -109,7 +112,9 @@ __global__ void __launch_bounds__(512) qkv_bwd_kernel(QkvArgs a) {
   const int tid = threadIdx.x, nt = blockDim.x;
   const bool sums = a.part_q != nullptr;
   if (sums) {
+    #pragma unroll 4
     for (int i = tid; i < dq; i += nt) acc_q[i] = 0.f;
+    #pragma unroll 4
     for (int i = tid; i < dkv; i += nt) acc_k[i] = 0.f;
   }
   const int t0 = blockIdx.x * a.rows_per_cta, t1 = min(a.T, t0 + a.rows_per_cta);
@@ -119,17 +124,20 @@ __global__ void __launch_bounds__(512) qkv_bwd_kernel(QkvArgs a) {
       const int W = seg == 0 ? dq : dkv;
       const int off = seg == 0 ? 0 : (seg == 1 ? dq : dq + dkv);
       const float* g = a.dQKV + (int64_t)t * a.ldd + off;
+      #pragma unroll 4
       for (int i = tid; i < W; i += nt) row[i] = qkv_value(a, seg, t, i).xt;
       __syncthreads();
       if (a.abits >= 16) {
+        #pragma unroll 4
         for (int i = tid; i < W; i += nt) dv[i] = g[i];
       } else {
         const int64_t k = (int64_t)seg * a.T + t;
         const int iM = a.imax[k], im = a.imin[k];
         const float Q = (float)((1 << a.abits) - 1);
         QState qs = omq_qstate(row[iM], row[im], 1.f, 1.f, Q, a.eps);
-        qs.h = a.h[k]; qs.z = (float)a.z[k]; qs.u = __fdiv_rn(row[im], qs.h);
+        qs.h = a.h[k]; qs.z = (float)a.z[k]; qs.rh = __frcp_rn(qs.h); qs.u = __fmul_rn(row[im], qs.rh);
         float Gh = 0.f, Gbm = 0.f;
+        #pragma unroll 4
         for (int i = tid; i < W; i += nt) {
           int inr;
           float gi = g[i];
@@ -147,11 +155,13 @@ __global__ void __launch_bounds__(512) qkv_bwd_kernel(QkvArgs a) {
       float* dy = a.dY + (int64_t)t * a.ldy + off;
       __nv_bfloat16* dyb = a.dYb + (int64_t)t * a.ldy + off;
       if (seg == 2) {
+        #pragma unroll 4
         for (int i = tid; i < W; i += nt) { dy[i] = dv[i]; dyb[i] = f_to_bf16(dv[i]); }
         __syncthreads();
         continue;
       }
       // [Q, K] LET: gradient w.r.t. the rotated projection and the s_a partial sums
+      #pragma unroll 4
       for (int i = tid; i < W; i += nt) {
         float d = dv[i];
         if (a.sa_exp) {
@@ -167,6 +177,7 @@ __global__ void __launch_bounds__(512) qkv_bwd_kernel(QkvArgs a) {
       }
       __syncthreads();
       // RoPE backward: the transpose of the rotation
+      #pragma unroll 4
       for (int i = tid; i < W; i += nt) {
         const int j = i % a.hd, jj = j % half;
         const float c = a.cs[((int64_t)t * half + jj) * 2], s = a.cs[((int64_t)t * half + jj) * 2 + 1];
@@ -178,7 +189,9 @@ __global__ void __launch_bounds__(512) qkv_bwd_kernel(QkvArgs a) {
     }
   }
   if (sums) {
+    #pragma unroll 4
     for (int i = tid; i < dq; i += nt) a.part_q[(int64_t)blockIdx.x * dq + i] = acc_q[i];
+    #pragma unroll 4
     for (int i = tid; i < dkv; i += nt) a.part_k[(int64_t)blockIdx.x * dkv + i] = acc_k[i];
   }
 }

@@ -21,13 +21,15 @@ struct Carve {
 
 typedef __nv_bfloat16 bf16;
 
-struct QState4 { float* h; int32_t* z; int32_t* imax; int32_t* imin; float* ga; float* gb; };
+struct QState4 { float* h; int32_t* z; int32_t* imax; int32_t* imin; float* ga; float* gb; float* M; float* m; };
 
-QState4 take_qstate(Carve& c, size_t n, bool sig = false) {
+QState4 take_qstate(Carve& c, size_t n, bool saved = false) {
   QState4 q;
   q.h = c.take<float>(n); q.z = c.take<int32_t>(n); q.imax = c.take<int32_t>(n); q.imin = c.take<int32_t>(n);
-  q.ga = sig ? c.take<float>(n) : nullptr;
-  q.gb = sig ? c.take<float>(n) : nullptr;
+  q.ga = saved ? c.take<float>(n) : nullptr;
+  q.gb = saved ? c.take<float>(n) : nullptr;
+  q.M = saved ? c.take<float>(n) : nullptr;
+  q.m = saved ? c.take<float>(n) : nullptr;
   return q;
 }
 
@@ -192,7 +194,7 @@ LwcFwdArgs lwc_args(const bf16* W, int64_t Cout, int64_t Cin, const omq_qcfg& cf
   a.s = s; a.r = r; a.gl = gl; a.bl = bl; a.lwc = 1; a.Wq = Wq; a.codes = nullptr;
   a.h = q.h; a.z = q.z; a.imax = q.imax; a.imin = q.imin;
   a.bias_delta = bias_delta; a.bias_shift = bias_shift; a.Bt = Bt;
-  a.ga_out = q.ga; a.gb_out = q.gb;
+  a.ga_out = q.ga; a.gb_out = q.gb; a.M_out = q.M; a.m_out = q.m;
   a.wbits = cfg.wbits; a.eps = cfg.h_eps; a.status = cfg.dev_status;
   return a;
 }
@@ -203,7 +205,7 @@ omq_status lwc_bwd_full(cudaStream_t st, const bf16* W, int64_t Cout, int64_t Ci
                         float* ddelta, int accumulate_sd, float* part) {
   LwcBwdArgs a{};
   a.W = W; a.Cout = Cout; a.Cin = Cin; a.group = cfg.group == 0 ? (int)Cin : cfg.group;
-  a.s = s; a.r = r; a.gl = gl; a.bl = bl; a.lwc = 1; a.ga = q.ga; a.gb = q.gb;
+  a.s = s; a.r = r; a.gl = gl; a.bl = bl; a.lwc = 1; a.ga = q.ga; a.gb = q.gb; a.Mv = q.M; a.mv = q.m;
   a.h = q.h; a.z = q.z; a.imax = q.imax; a.imin = q.imin;
   a.dWq = dW; a.ld_dwq = Cin; a.dgl = dgl; a.dbl = dbl; a.dWt = nullptr; a.dr = dr; a.dBt = dBt;
   a.ds = ds; a.ddelta = ddelta;
@@ -526,7 +528,7 @@ omq_status omq_qlinear_fwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t 
   cudaStream_t st = (cudaStream_t)stream;
   const int g = cfg->group == 0 ? (int)Cin : cfg->group;
   OMQ_REQUIRE(Cin % g == 0, OMQ_ERR_SHAPE);
-  QState4 qw{sv->h_w, sv->z_w, sv->imax_w, sv->imin_w, nullptr, nullptr};
+  QState4 qw{sv->h_w, sv->z_w, sv->imax_w, sv->imin_w, nullptr, nullptr, nullptr, nullptr};
   const bool let = cfg->let != 0;
   OMQ_TRY(lwc_fwd_launch(st, lwc_args((const bf16*)W, Cout, Cin, *cfg, let ? s : nullptr, nullptr, gamma_logit,
                                       beta_logit, (bf16*)sv->w_hat, qw, let ? delta : nullptr, nullptr,
@@ -586,7 +588,7 @@ omq_status omq_qlinear_bwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t 
   OMQ_LAUNCH_CHECK();
   OMQ_TRY(gemm_dw(st, T, Cout, Cin, dYb, (const bf16*)sv->x_hat, dWh, cfg->dev_status));
   if (let) OMQ_TRY(colsum_rows(st, dY, T, Cout, Cout, part, dB, 1.f, 0));
-  QState4 qw{sv->h_w, sv->z_w, sv->imax_w, sv->imin_w, nullptr, nullptr};
+  QState4 qw{sv->h_w, sv->z_w, sv->imax_w, sv->imin_w, nullptr, nullptr, nullptr, nullptr};
   omq_qcfg cf = *cfg;
   OMQ_TRY(lwc_bwd_full(st, (const bf16*)W, Cout, Cin, cf, let ? s : nullptr, nullptr, gamma_logit, beta_logit, qw, dWh,
                        dgamma, dbeta, nullptr, let ? dB : nullptr, let ? ds : nullptr, let ? ddelta : nullptr,

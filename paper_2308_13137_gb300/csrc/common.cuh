@@ -85,6 +85,7 @@ __device__ __forceinline__ uint4 pack_bf16x8(const float* f) {
 // ------------------------------------------------------------------------------------------------
 struct QState {          // per-group quantizer state
   float h;               // step, floored at eps
+  float rh;              // 1/h, correctly rounded: w/h is formed as w * rh
   float z;               // zero point (integer valued)
   float u;               // beta * min / h
   float a, b;            // clipping strengths
@@ -92,24 +93,43 @@ struct QState {          // per-group quantizer state
   int floored;
 };
 
-// gamma = sigmoid(gamma_hat), evaluated in double and rounded once to float, so that the
-// clipping strength is the correctly rounded value of the logit's sigmoid.
-__device__ __forceinline__ float omq_sigmoid(float t) { return (float)(1.0 / (1.0 + exp(-(double)t))); }
+// gamma = sigmoid(gamma_hat) in single precision with every operation rounded once (no fused
+// multiply-add), so that the value is reproducible bit for bit on any IEEE machine:
+// exp(-t) by Cody-Waite reduction, -t = n ln2 + r with |r| <= ln2/2 (ln2 split into a 15-bit head,
+// whose product with n is exact, and a tail), a degree-7 Taylor polynomial for exp(r) in Horner
+// form, and an exact scaling by 2^n; then 1 / (1 + exp(-t)).  |t| is clamped to 80.
+__device__ __forceinline__ float omq_sigmoid(float t) {
+  const float x = -fminf(fmaxf(t, -80.f), 80.f);
+  const float n = rintf(__fmul_rn(x, 1.44269502162933349609375f));
+  const float r = __fsub_rn(__fsub_rn(x, __fmul_rn(n, 0.693145751953125f)), __fmul_rn(n, 1.428606765330187e-06f));
+  float p = 1.98412701138295233249664e-04f;
+  p = __fadd_rn(__fmul_rn(p, r), 1.38888892251998186111450e-03f);
+  p = __fadd_rn(__fmul_rn(p, r), 8.33333376795053482055664e-03f);
+  p = __fadd_rn(__fmul_rn(p, r), 4.16666679084300994873047e-02f);
+  p = __fadd_rn(__fmul_rn(p, r), 1.66666671633720397949219e-01f);
+  p = __fadd_rn(__fmul_rn(p, r), 0.5f);
+  p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+  p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+  const float e = __fmul_rn(p, __int_as_float((127 + (int)n) << 23));
+  return __fdiv_rn(1.0f, __fadd_rn(1.0f, e));
+}
 
+// h = (a*M - b*m)/Q floored at eps, its reciprocal, u = (b*m) * (1/h) and z = -round(u)
 __device__ __forceinline__ QState omq_qstate(float M, float m, float a, float b, float Q, float eps) {
   QState s;
   s.a = a; s.b = b; s.M = M; s.m = m;
   float hr = __fdiv_rn(__fsub_rn(__fmul_rn(a, M), __fmul_rn(b, m)), Q);
   s.floored = !(hr >= eps);
   s.h = s.floored ? eps : hr;
-  s.u = __fdiv_rn(__fmul_rn(b, m), s.h);
+  s.rh = __frcp_rn(s.h);
+  s.u = __fmul_rn(__fmul_rn(b, m), s.rh);
   s.z = -rintf(s.u);
   return s;
 }
 
-// code c = round(w/h) + z before the clamp
+// code c = round(w/h) + z before the clamp, with w/h formed as w * (1/h)
 __device__ __forceinline__ float omq_code_raw(float w, const QState& s, float* x_out) {
-  float x = __fdiv_rn(w, s.h);
+  float x = __fmul_rn(w, s.rh);
   *x_out = x;
   return rintf(x) + s.z;
 }

@@ -5,7 +5,6 @@
 
 #include <atomic>
 
-#define LWC_KEEP 16        // 8-element chunks per lane kept in registers between passes (Cin <= 4096)
 
 static std::atomic<long long> g_launches{0};
 void omq_count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
@@ -64,7 +63,9 @@ __device__ __forceinline__ float dot8(const uint4& raw, const float* d, int64_t 
   return acc;
 }
 
-__global__ void __launch_bounds__(256) lwc_fwd_kernel(LwcFwdArgs a) {
+// MODE 0: quantization off; 1: one group per row; 2: groups of <= 256 columns
+template <int MODE>
+__global__ void __launch_bounds__(256, 4) lwc_fwd_kernel(LwcFwdArgs a) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t o = (int64_t)blockIdx.x * 8 + warp;
   if (o >= a.Cout) return;                       // whole warp leaves; no block-level barrier below
@@ -75,109 +76,139 @@ __global__ void __launch_bounds__(256) lwc_fwd_kernel(LwcFwdArgs a) {
   const uint4* Wrow = reinterpret_cast<const uint4*>(a.W + o * a.Cin);
   const int gsz = a.group;
   const int64_t ngroups = a.Cin / gsz;
+  const uint4 zero4 = make_uint4(0, 0, 0, 0);
   float dot = 0.f;
 
-  if (a.wbits >= 16) {                           // quantization off: W_hat = bf16(W~)
-    for (int it = 0; it < iters; ++it) {
-      const int64_t c = (int64_t)it * 32 + lane;
-      if (c < nchunk) {
-        uint4 raw = __ldg(Wrow + c);
-        float wt[8];
-        lwc_chunk(raw, a.s, c, rr, wt);
-        if (a.Wq) reinterpret_cast<uint4*>(a.Wq + o * a.Cin)[c] = pack_bf16x8(wt);
-        if (a.Bt) dot += dot8(raw, a.bias_delta, c);
+  if (MODE == 0) {                               // quantization off: W_hat = bf16(W~)
+    for (int it0 = 0; it0 < iters; it0 += 4) {
+      uint4 raw[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int64_t c = (int64_t)(it0 + j) * 32 + lane;
+        raw[j] = (it0 + j < iters && c < nchunk) ? __ldg(Wrow + c) : zero4;
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int64_t c = (int64_t)(it0 + j) * 32 + lane;
+        if (it0 + j < iters && c < nchunk) {
+          float wt[8];
+          lwc_chunk(raw[j], a.s, c, rr, wt);
+          if (a.Wq) reinterpret_cast<uint4*>(a.Wq + o * a.Cin)[c] = pack_bf16x8(wt);
+          if (a.Bt) dot += dot8(raw[j], a.bias_delta, c);
+        }
       }
     }
-  } else if (gsz == a.Cin) {
-    // ---- one group per row: stats over the row (kept in registers up to LWC_KEEP chunks) ----
-    uint4 keep[LWC_KEEP];
-    MaxMin r = mm_identity();
+  } else if (MODE == 1) {
+    // ---- one group per row.  Pass 1: values of max / min (and the LET bias dot).  Pass 2
+    // (the row again, from L1/L2): quantize and store, and find the first index of max / min. ----
+    float M = -INFINITY, m = INFINITY;
+    for (int it0 = 0; it0 < iters; it0 += 4) {
+      uint4 raw[4];
 #pragma unroll
-    for (int it = 0; it < LWC_KEEP; ++it) {
-      keep[it] = make_uint4(0, 0, 0, 0);
-      const int64_t c = (int64_t)it * 32 + lane;
-      if (it < iters && c < nchunk) {
-        keep[it] = __ldg(Wrow + c);
-        float wt[8];
-        lwc_chunk(keep[it], a.s, c, rr, wt);
+      for (int j = 0; j < 4; ++j) {
+        const int64_t c = (int64_t)(it0 + j) * 32 + lane;
+        raw[j] = (it0 + j < iters && c < nchunk) ? __ldg(Wrow + c) : zero4;
+      }
 #pragma unroll
-        for (int e = 0; e < 8; ++e) mm_push(r, wt[e], (int)(c * 8 + e));
-        if (a.Bt) dot += dot8(keep[it], a.bias_delta, c);
+      for (int j = 0; j < 4; ++j) {
+        const int64_t c = (int64_t)(it0 + j) * 32 + lane;
+        if (it0 + j < iters && c < nchunk) {
+          float wt[8];
+          lwc_chunk(raw[j], a.s, c, rr, wt);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) { M = fmaxf(M, wt[e]); m = fminf(m, wt[e]); }
+          if (a.Bt) dot += dot8(raw[j], a.bias_delta, c);
+        }
       }
     }
-    for (int it = LWC_KEEP; it < iters; ++it) {
-      const int64_t c = (int64_t)it * 32 + lane;
-      if (c < nchunk) {
-        uint4 raw = __ldg(Wrow + c);
-        float wt[8];
-        lwc_chunk(raw, a.s, c, rr, wt);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) mm_push(r, wt[e], (int)(c * 8 + e));
-        if (a.Bt) dot += dot8(raw, a.bias_delta, c);
-      }
+    for (int off = 16; off > 0; off >>= 1) {
+      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+      m = fminf(m, __shfl_xor_sync(0xffffffffu, m, off));
     }
-    r = mm_shfl_reduce(r, 32);
     float ga = 1.f, gb = 1.f;
     if (a.lwc) {                                 // one sigmoid per group, broadcast
       if (lane == 0) { ga = omq_sigmoid(a.gl[o]); gb = omq_sigmoid(a.bl[o]); }
       ga = __shfl_sync(0xffffffffu, ga, 0);
       gb = __shfl_sync(0xffffffffu, gb, 0);
     }
-    const QState qs = omq_qstate(r.M, r.m, ga, gb, Q, a.eps);
-    if (lane == 0) {
-      a.h[o] = qs.h; a.z[o] = (int32_t)qs.z; a.imax[o] = r.iM; a.imin[o] = r.im;
-      if (a.ga_out) { a.ga_out[o] = ga; a.gb_out[o] = gb; }
+    const QState qs = omq_qstate(M, m, ga, gb, Q, a.eps);
+    int iM = 0x7fffffff, im = 0x7fffffff;        // first index of the max / min held by this lane
+    for (int it0 = 0; it0 < iters; it0 += 4) {
+      uint4 raw[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int64_t c = (int64_t)(it0 + j) * 32 + lane;
+        raw[j] = (it0 + j < iters && c < nchunk) ? __ldg(Wrow + c) : zero4;
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int64_t c = (int64_t)(it0 + j) * 32 + lane;
+        if (it0 + j < iters && c < nchunk) {
+          float wt[8];
+          lwc_chunk(raw[j], a.s, c, rr, wt);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int idx = (int)(c * 8 + e);
+            if (wt[e] == M && idx < iM) iM = idx;
+            if (wt[e] == m && idx < im) im = idx;
+          }
+          lwc_store(a, o, c, wt, qs, Q);
+        }
+      }
     }
 #pragma unroll
-    for (int it = 0; it < LWC_KEEP; ++it) {
-      const int64_t c = (int64_t)it * 32 + lane;
-      if (it < iters && c < nchunk) {
-        float wt[8];
-        lwc_chunk(keep[it], a.s, c, rr, wt);
-        lwc_store(a, o, c, wt, qs, Q);
-      }
+    for (int off = 16; off > 0; off >>= 1) {
+      iM = min(iM, __shfl_xor_sync(0xffffffffu, iM, off));
+      im = min(im, __shfl_xor_sync(0xffffffffu, im, off));
     }
-    for (int it = LWC_KEEP; it < iters; ++it) {
-      const int64_t c = (int64_t)it * 32 + lane;
-      if (c < nchunk) {
-        float wt[8];
-        lwc_chunk(__ldg(Wrow + c), a.s, c, rr, wt);
-        lwc_store(a, o, c, wt, qs, Q);
-      }
+    if (lane == 0) {
+      a.h[o] = qs.h; a.z[o] = (int32_t)qs.z; a.imax[o] = iM; a.imin[o] = im;
+      if (a.ga_out) { a.ga_out[o] = ga; a.gb_out[o] = gb; }
+      if (a.M_out) { a.M_out[o] = M; a.m_out[o] = m; }
     }
   } else {
-    // ---- groups of lpg consecutive lanes (lpg a power of two <= 32) ----
+    // ---- groups of lpg consecutive lanes (lpg a power of two <= 32), four chunks of loads ahead ----
     const int lpg = gsz / 8;
     const int leader = lane & ~(lpg - 1);
-    for (int it = 0; it < iters; ++it) {
-      const int64_t c = (int64_t)it * 32 + lane;
-      const bool valid = c < nchunk;
-      float wt[8];
-      MaxMin r = mm_identity();
-      uint4 raw = make_uint4(0, 0, 0, 0);
-      if (valid) {
-        raw = __ldg(Wrow + c);
-        lwc_chunk(raw, a.s, c, rr, wt);
+    for (int it0 = 0; it0 < iters; it0 += 4) {
+      uint4 raw[4];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) mm_push(r, wt[e], (int)(c * 8 + e));
-        if (a.Bt) dot += dot8(raw, a.bias_delta, c);
+      for (int j = 0; j < 4; ++j) {
+        const int64_t c = (int64_t)(it0 + j) * 32 + lane;
+        raw[j] = (it0 + j < iters && c < nchunk) ? __ldg(Wrow + c) : zero4;
       }
-      r = mm_shfl_reduce(r, lpg);
-      const int64_t gi = valid ? (c * 8) / gsz : 0;
-      float ga = 1.f, gb = 1.f;
-      if (a.lwc) {
-        if (lane == leader && valid) { ga = omq_sigmoid(a.gl[o * ngroups + gi]); gb = omq_sigmoid(a.bl[o * ngroups + gi]); }
-        ga = __shfl_sync(0xffffffffu, ga, leader);
-        gb = __shfl_sync(0xffffffffu, gb, leader);
-      }
-      if (valid) {
-        const QState qs = omq_qstate(r.M, r.m, ga, gb, Q, a.eps);
-        if (lane == leader) {
-          const int64_t k = o * ngroups + gi;
-          a.h[k] = qs.h; a.z[k] = (int32_t)qs.z; a.imax[k] = r.iM; a.imin[k] = r.im;
-          if (a.ga_out) { a.ga_out[k] = ga; a.gb_out[k] = gb; }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (it0 + j >= iters) break;                     // warp-uniform
+        const int64_t c = (int64_t)(it0 + j) * 32 + lane;
+        const bool valid = c < nchunk;
+        float wt[8];
+        MaxMin r = mm_identity();
+        if (valid) {
+          lwc_chunk(raw[j], a.s, c, rr, wt);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) mm_push(r, wt[e], (int)(c * 8 + e));
+          if (a.Bt) dot += dot8(raw[j], a.bias_delta, c);
         }
-        lwc_store(a, o, c, wt, qs, Q);
+        r = mm_shfl_reduce(r, lpg);
+        const int64_t gi = valid ? (c * 8) / gsz : 0;
+        float ga = 1.f, gb = 1.f;
+        if (a.lwc) {
+          if (lane == leader && valid) { ga = omq_sigmoid(a.gl[o * ngroups + gi]); gb = omq_sigmoid(a.bl[o * ngroups + gi]); }
+          ga = __shfl_sync(0xffffffffu, ga, leader);
+          gb = __shfl_sync(0xffffffffu, gb, leader);
+        }
+        if (valid) {
+          const QState qs = omq_qstate(r.M, r.m, ga, gb, Q, a.eps);
+          if (lane == leader) {
+            const int64_t k = o * ngroups + gi;
+            a.h[k] = qs.h; a.z[k] = (int32_t)qs.z; a.imax[k] = r.iM; a.imin[k] = r.im;
+            if (a.ga_out) { a.ga_out[k] = ga; a.gb_out[k] = gb; }
+            if (a.M_out) { a.M_out[k] = r.M; a.m_out[k] = r.m; }
+          }
+          lwc_store(a, o, c, wt, qs, Q);
+        }
       }
     }
   }
@@ -196,7 +227,10 @@ static bool lwc_group_ok(int64_t Cin, int g) {
 
 omq_status lwc_fwd_launch(cudaStream_t st, const LwcFwdArgs& a) {
   OMQ_REQUIRE(lwc_group_ok(a.Cin, a.group), OMQ_ERR_UNSUPPORTED);
-  lwc_fwd_kernel<<<(unsigned)((a.Cout + 7) / 8), 256, 0, st>>>(a);
+  const unsigned grid = (unsigned)((a.Cout + 7) / 8);
+  if (a.wbits >= 16) lwc_fwd_kernel<0><<<grid, 256, 0, st>>>(a);
+  else if (a.group == a.Cin) lwc_fwd_kernel<1><<<grid, 256, 0, st>>>(a);
+  else lwc_fwd_kernel<2><<<grid, 256, 0, st>>>(a);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -259,7 +293,9 @@ __device__ __forceinline__ float lwc_sig(const float* saved, const float* logit,
   return saved ? saved[k] : omq_sigmoid(logit[k]);
 }
 
-__global__ void __launch_bounds__(LWC_BWD_THREADS) lwc_bwd_tile_kernel(LwcBwdArgs a, LwcBwdScratch sc) {
+#define LWC_BWD_RB 1          // rows whose loads are issued together
+
+__global__ void __launch_bounds__(LWC_BWD_THREADS, 3) lwc_bwd_tile_kernel(LwcBwdArgs a, LwcBwdScratch sc) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t nchunk = a.Cin / 8;
   const int64_t c = (int64_t)blockIdx.x * LWC_BWD_THREADS + tid;     // this thread's chunk
@@ -271,6 +307,7 @@ __global__ void __launch_bounds__(LWC_BWD_THREADS) lwc_bwd_tile_kernel(LwcBwdArg
   const int64_t ngroups = a.Cin / gsz;
   const int lpg = perch ? 32 : gsz / 8;
   const int leader = lane & ~(lpg - 1);
+  const int64_t gi = valid ? (c * 8) / gsz : 0;
   const bool want_s = a.ds != nullptr, want_d = a.ddelta != nullptr && a.dBt != nullptr;
   float sv[8];
   load8(a.s, valid ? c : 0, sv, 1.f);
@@ -280,105 +317,120 @@ __global__ void __launch_bounds__(LWC_BWD_THREADS) lwc_bwd_tile_kernel(LwcBwdArg
   const int64_t o0 = (int64_t)blockIdx.y * sc.rows;
   const int64_t o1 = min(a.Cout, o0 + sc.rows);
   const uint4 zero4 = make_uint4(0, 0, 0, 0);
+  const float4 zf4 = make_float4(0.f, 0.f, 0.f, 0.f);
 
-  for (int64_t o = o0; o < o1; ++o) {
-    const float rr = a.r ? a.r[o] : 1.f;
-    const __nv_bfloat16* Wrow = a.W + o * a.Cin;
-    const uint4 raw = valid ? __ldg(reinterpret_cast<const uint4*>(Wrow) + c) : zero4;
-    float g[8];
-    if (valid) {
-      const float4 g0 = __ldg(reinterpret_cast<const float4*>(a.dWq + o * a.ld_dwq) + 2 * c);
-      const float4 g1 = __ldg(reinterpret_cast<const float4*>(a.dWq + o * a.ld_dwq) + 2 * c + 1);
-      g[0] = g0.x; g[1] = g0.y; g[2] = g0.z; g[3] = g0.w; g[4] = g1.x; g[5] = g1.y; g[6] = g1.z; g[7] = g1.w;
-    } else {
+  for (int64_t ob = o0; ob < o1; ob += LWC_BWD_RB) {
+    uint4 raw[LWC_BWD_RB];
+    float4 ga4[LWC_BWD_RB], gb4[LWC_BWD_RB];
+    float hv[LWC_BWD_RB], zv[LWC_BWD_RB], rv[LWC_BWD_RB], mv[LWC_BWD_RB], bv[LWC_BWD_RB], dbv[LWC_BWD_RB];
+    int imv[LWC_BWD_RB], iMv[LWC_BWD_RB];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) g[e] = 0.f;
+    for (int j = 0; j < LWC_BWD_RB; ++j) {      // every load of the batch first
+      const int64_t o = ob + j;
+      const bool rowok = o < o1;
+      const bool ld = rowok && valid;
+      const int64_t oo = rowok ? o : o0;
+      raw[j] = ld ? __ldg(reinterpret_cast<const uint4*>(a.W + oo * a.Cin) + c) : zero4;
+      ga4[j] = ld ? __ldg(reinterpret_cast<const float4*>(a.dWq + oo * a.ld_dwq) + 2 * c) : zf4;
+      gb4[j] = ld ? __ldg(reinterpret_cast<const float4*>(a.dWq + oo * a.ld_dwq) + 2 * c + 1) : zf4;
+      const int64_t k = perch ? oo : oo * ngroups + gi;
+      hv[j] = a.h[k]; zv[j] = (float)a.z[k]; imv[j] = a.imin[k]; iMv[j] = a.imax[k];
+      rv[j] = a.r ? a.r[oo] : 1.f;
+      bv[j] = lwc_sig(a.gb, a.bl, k, a.lwc);
+      mv[j] = a.mv ? a.mv[k] : lwc_wt(bf16_to_f(a.W[oo * a.Cin + imv[j]]), a.s, imv[j], rv[j]);
+      dbv[j] = want_d ? a.dBt[oo] : 0.f;
     }
-    float w[8];
-    unpack_bf16x8(raw, w);
-    // quantizer state of this lane's group
-    const int64_t k = perch ? o : o * ngroups + (valid ? (c * 8) / gsz : 0);
-    const int iM = a.imax[k], im = a.imin[k];
-    const float gb = lwc_sig(a.gb, a.bl, k, a.lwc);
-    const float m = lwc_wt(bf16_to_f(Wrow[im]), a.s, im, rr);
-    QState qs;
-    qs.h = a.h[k]; qs.z = (float)a.z[k]; qs.b = gb; qs.m = m;
-    qs.u = __fdiv_rn(__fmul_rn(gb, m), qs.h);
-    float Gh = 0.f, Gbm = 0.f, drm = 0.f;
-    int inr_mask = 0;
-    if (valid) {
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        const float wt = __fmul_rn(__fmul_rn(w[e], sv[e]), rr);
-        int inr;
-        const float dh = omq_ste_dh(wt, qs, Q, &inr);
-        Gh = fmaf(g[e], dh, Gh);
-        if (!inr) Gbm += g[e];
-        inr_mask |= inr << e;
-      }
-    }
-    if (perch) {
-      // warp partials of the row; routing to max/min is added by the per-row finalize
-      Gh = warp_sum(Gh);
-      Gbm = warp_sum(Gbm);
+    for (int j = 0; j < LWC_BWD_RB; ++j) {
+      const int64_t o = ob + j;
+      if (o >= o1) break;                          // uniform across the CTA
+      const float rr = rv[j];
+      const int64_t k = perch ? o : o * ngroups + gi;
+      float g[8] = {ga4[j].x, ga4[j].y, ga4[j].z, ga4[j].w, gb4[j].x, gb4[j].y, gb4[j].z, gb4[j].w};
+      float w[8];
+      unpack_bf16x8(raw[j], w);
+      QState qs;
+      qs.h = hv[j]; qs.z = zv[j]; qs.b = bv[j]; qs.m = mv[j];
+      qs.rh = __frcp_rn(qs.h);
+      qs.u = __fmul_rn(__fmul_rn(qs.b, qs.m), qs.rh);
+      float Gh = 0.f, Gbm = 0.f, drm = 0.f;
+      int inr_mask = 0;
       if (valid) {
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const float d = ((inr_mask >> e) & 1) ? g[e] : 0.f;
-          drm = fmaf(d * w[e], sv[e], drm);
-          if (want_s) acc_s[e] = fmaf(d * w[e], rr, acc_s[e]);
-          if (a.dWt) g[e] = d;
-        }
-        if (a.dWt) {
-          float4* dst = reinterpret_cast<float4*>(a.dWt + o * a.Cin) + 2 * c;
-          dst[0] = make_float4(g[0], g[1], g[2], g[3]);
-          dst[1] = make_float4(g[4], g[5], g[6], g[7]);
+          const float wt = __fmul_rn(__fmul_rn(w[e], sv[e]), rr);
+          int inr;
+          const float dh = omq_ste_dh(wt, qs, Q, &inr);
+          Gh = fmaf(g[e], dh, Gh);
+          if (!inr) Gbm += g[e];
+          inr_mask |= inr << e;
         }
       }
-      drm = warp_sum(drm);
-      if (lane == 0 && wglob < sc.ncw) {
-        sc.rowpart[(0 * a.Cout + o) * sc.ncw + wglob] = Gh;
-        sc.rowpart[(1 * a.Cout + o) * sc.ncw + wglob] = Gbm;
-        sc.rowpart[(2 * a.Cout + o) * sc.ncw + wglob] = drm;
-      }
-    } else {
-      Gh = warp_sum(Gh, lpg);
-      Gbm = warp_sum(Gbm, lpg);
-      if (valid) {
-        const float ga = lwc_sig(a.ga, a.gl, k, a.lwc);
-        const float M = lwc_wt(bf16_to_f(Wrow[iM]), a.s, iM, rr);
-        const float hr = __fdiv_rn(__fsub_rn(__fmul_rn(ga, M), __fmul_rn(gb, m)), Q);
-        if (!(hr >= a.eps)) Gh = 0.f;                      // floored h: no gradient through h
-        const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
-        if (lane == leader && a.lwc) {
-          const float dg = GaM * M * ga * (1.f - ga), db = Gbt * m * gb * (1.f - gb);
-          if (a.accumulate) { a.dgl[k] += dg; a.dbl[k] += db; } else { a.dgl[k] = dg; a.dbl[k] = db; }
-        }
+      if (perch) {
+        // warp partials of the row; routing to max/min is added by the per-row finalize
+        Gh = warp_sum(Gh);
+        Gbm = warp_sum(Gbm);
+        if (valid) {
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const int64_t col = c * 8 + e;
-          float d = ((inr_mask >> e) & 1) ? g[e] : 0.f;
-          if (col == iM) d += GaM * ga;
-          if (col == im) d += Gbt * gb;
-          drm = fmaf(d * w[e], sv[e], drm);
-          if (want_s) acc_s[e] = fmaf(d * w[e], rr, acc_s[e]);
-          g[e] = d;
+          for (int e = 0; e < 8; ++e) {
+            const float d = ((inr_mask >> e) & 1) ? g[e] : 0.f;
+            drm = fmaf(d * w[e], sv[e], drm);
+            if (want_s) acc_s[e] = fmaf(d * w[e], rr, acc_s[e]);
+            g[e] = d;
+          }
+          if (a.dWt) {
+            float4* dst = reinterpret_cast<float4*>(a.dWt + o * a.Cin) + 2 * c;
+            dst[0] = make_float4(g[0], g[1], g[2], g[3]);
+            dst[1] = make_float4(g[4], g[5], g[6], g[7]);
+          }
         }
-        if (a.dWt) {
-          float4* dst = reinterpret_cast<float4*>(a.dWt + o * a.Cin) + 2 * c;
-          dst[0] = make_float4(g[0], g[1], g[2], g[3]);
-          dst[1] = make_float4(g[4], g[5], g[6], g[7]);
-        }
-      }
-      if (a.dr) {
         drm = warp_sum(drm);
-        if (lane == 0 && wglob < sc.ncw) sc.rowpart[(2 * a.Cout + o) * sc.ncw + wglob] = drm;
-      }
-    }
-    if (want_d && valid) {
-      const float f = a.dBt[o] * rr;
+        if (lane == 0 && wglob < sc.ncw) {
+          sc.rowpart[(0 * a.Cout + o) * sc.ncw + wglob] = Gh;
+          sc.rowpart[(1 * a.Cout + o) * sc.ncw + wglob] = Gbm;
+          sc.rowpart[(2 * a.Cout + o) * sc.ncw + wglob] = drm;
+        }
+      } else {
+        Gh = warp_sum(Gh, lpg);
+        Gbm = warp_sum(Gbm, lpg);
+        if (valid) {
+          const int iM = iMv[j], im = imv[j];
+          const float ga = lwc_sig(a.ga, a.gl, k, a.lwc), gb = qs.b;
+          const float M = a.Mv ? a.Mv[k] : lwc_wt(bf16_to_f(a.W[o * a.Cin + iM]), a.s, iM, rr);
+          const float m = qs.m;
+          const float hr = __fdiv_rn(__fsub_rn(__fmul_rn(ga, M), __fmul_rn(gb, m)), Q);
+          if (!(hr >= a.eps)) Gh = 0.f;                      // floored h: no gradient through h
+          const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
+          if (lane == leader && a.lwc) {
+            const float dg = GaM * M * ga * (1.f - ga), db = Gbt * m * gb * (1.f - gb);
+            if (a.accumulate) { a.dgl[k] += dg; a.dbl[k] += db; } else { a.dgl[k] = dg; a.dbl[k] = db; }
+          }
 #pragma unroll
-      for (int e = 0; e < 8; ++e) acc_d[e] = fmaf(f, w[e], acc_d[e]);
+          for (int e = 0; e < 8; ++e) {
+            const int64_t col = c * 8 + e;
+            float d = ((inr_mask >> e) & 1) ? g[e] : 0.f;
+            if (col == iM) d += GaM * ga;
+            if (col == im) d += Gbt * gb;
+            drm = fmaf(d * w[e], sv[e], drm);
+            if (want_s) acc_s[e] = fmaf(d * w[e], rr, acc_s[e]);
+            g[e] = d;
+          }
+          if (a.dWt) {
+            float4* dst = reinterpret_cast<float4*>(a.dWt + o * a.Cin) + 2 * c;
+            dst[0] = make_float4(g[0], g[1], g[2], g[3]);
+            dst[1] = make_float4(g[4], g[5], g[6], g[7]);
+          }
+        }
+        if (a.dr) {
+          drm = warp_sum(drm);
+          if (lane == 0 && wglob < sc.ncw) sc.rowpart[(2 * a.Cout + o) * sc.ncw + wglob] = drm;
+        }
+      }
+      if (want_d && valid) {
+        const float f = dbv[j] * rr;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc_d[e] = fmaf(f, w[e], acc_d[e]);
+      }
     }
   }
   if (valid) {
@@ -422,7 +474,8 @@ __global__ void __launch_bounds__(256) lwc_bwd_finalize_kernel(LwcBwdArgs a, Lwc
     const float ga = lwc_sig(a.ga, a.gl, o, a.lwc), gb = lwc_sig(a.gb, a.bl, o, a.lwc);
     const float WM = bf16_to_f(Wrow[iM]), Wm = bf16_to_f(Wrow[im]);
     const float sM = a.s ? a.s[iM] : 1.f, sm = a.s ? a.s[im] : 1.f;
-    const float M = __fmul_rn(__fmul_rn(WM, sM), rr), m = __fmul_rn(__fmul_rn(Wm, sm), rr);
+    const float M = a.Mv ? a.Mv[o] : __fmul_rn(__fmul_rn(WM, sM), rr);
+    const float m = a.mv ? a.mv[o] : __fmul_rn(__fmul_rn(Wm, sm), rr);
     const float hr = __fdiv_rn(__fsub_rn(__fmul_rn(ga, M), __fmul_rn(gb, m)), Q);
     if (!(hr >= a.eps)) Gh = 0.f;
     const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
@@ -485,6 +538,7 @@ __device__ __forceinline__ void act_produce_row(const ActFwdArgs& a, int64_t t, 
   const float* xr = a.X + t * a.ldx;
   if (P == AP_RMS_LET) {
     float ss = 0.f;
+    #pragma unroll 4
     for (int64_t i = tid; i < C / 4; i += nt) {
       float4 v = __ldg(reinterpret_cast<const float4*>(xr) + i);
       reinterpret_cast<float4*>(row)[i] = v;
@@ -493,6 +547,7 @@ __device__ __forceinline__ void act_produce_row(const ActFwdArgs& a, int64_t t, 
     float2 tot = block_sum2(ss, 0.f, red_f);
     float rstd = 1.0f / sqrtf(tot.x / (float)C + a.rms_eps);
     *rstd_out = rstd;
+    #pragma unroll 4
     for (int64_t i = tid; i < C; i += nt) {
       float v = row[i] * rstd;
       if (a.delta) v = v - a.delta[i];
@@ -501,12 +556,14 @@ __device__ __forceinline__ void act_produce_row(const ActFwdArgs& a, int64_t t, 
     }
   } else if (P == AP_SWIGLU) {
     const float* ur = a.U + t * a.ldu;
+    #pragma unroll 4
     for (int64_t i = tid; i < C / 4; i += nt) {
       float4 g = __ldg(reinterpret_cast<const float4*>(xr) + i);
       float4 u = __ldg(reinterpret_cast<const float4*>(ur) + i);
       reinterpret_cast<float4*>(row)[i] = make_float4(silu_f(g.x) * u.x, silu_f(g.y) * u.y, silu_f(g.z) * u.z, silu_f(g.w) * u.w);
     }
   } else {
+    #pragma unroll 4
     for (int64_t i = tid; i < C / 4; i += nt) {
       float4 v = __ldg(reinterpret_cast<const float4*>(xr) + i);
       if (P == AP_LET) {
@@ -538,6 +595,7 @@ __global__ void __launch_bounds__(512) act_fwd_kernel(ActFwdArgs a) {
   if (P == AP_RMS_LET && tid == 0 && a.rstd) a.rstd[t] = rstd;
   __nv_bfloat16* qr = a.Xq + t * a.ldq;
   if (a.abits >= 16) {
+    #pragma unroll 4
     for (int64_t i = tid; i < C / 2; i += nt) {
       float2 v = reinterpret_cast<float2*>(row)[i];
       reinterpret_cast<__nv_bfloat162*>(qr)[i] = __floats2bfloat162_rn(v.x, v.y);
@@ -545,11 +603,13 @@ __global__ void __launch_bounds__(512) act_fwd_kernel(ActFwdArgs a) {
     return;
   }
   MaxMin r = mm_identity();
+  #pragma unroll 4
   for (int64_t i = tid; i < C; i += nt) mm_push(r, row[i], (int)i);
   r = mm_block_reduce(r, red_mm);
   const float Q = (float)((1 << a.abits) - 1);
   QState qs = omq_qstate(r.M, r.m, 1.f, 1.f, Q, a.eps);
   if (tid == 0) { a.h[t] = qs.h; a.z[t] = (int32_t)qs.z; a.imax[t] = r.iM; a.imin[t] = r.im; }
+  #pragma unroll 4
   for (int64_t i = tid; i < C / 2; i += nt) {
     float2 v = reinterpret_cast<float2*>(row)[i];
     float c0, c1;
@@ -596,6 +656,7 @@ __global__ void __launch_bounds__(512) act_bwd_kernel(ActBwdArgs a) {
   __shared__ float red_f[64];
   const int tid = threadIdx.x, nt = blockDim.x;
   if (let_sums)
+    #pragma unroll 4
     for (int64_t i = tid; i < C; i += nt) { acc_s[i] = 0.f; acc_d[i] = 0.f; }
   const int64_t t0 = (int64_t)blockIdx.x * a.rows_per_cta;
   const int64_t t1 = min(a.T, t0 + a.rows_per_cta);
@@ -611,6 +672,7 @@ __global__ void __launch_bounds__(512) act_bwd_kernel(ActBwdArgs a) {
     const float* xr = a.X + t * a.ldx;
     if (P == AP_RMS_LET) {
       const float rstd = a.rstd[t];
+      #pragma unroll 4
       for (int64_t i = tid; i < C; i += nt) {
         float v = xr[i] * rstd;
         if (a.delta) v = v - a.delta[i];
@@ -629,8 +691,9 @@ __global__ void __launch_bounds__(512) act_bwd_kernel(ActBwdArgs a) {
     if (quant) {
       iM = a.imax[t]; im = a.imin[t];
       qs = omq_qstate(row[iM], row[im], 1.f, 1.f, Q, a.eps);
-      qs.h = a.h[t]; qs.z = (float)a.z[t]; qs.u = __fdiv_rn(row[im], qs.h);
+      qs.h = a.h[t]; qs.z = (float)a.z[t]; qs.rh = __frcp_rn(qs.h); qs.u = __fmul_rn(row[im], qs.rh);
       float Gh = 0.f, Gbm = 0.f;
+      #pragma unroll 4
       for (int64_t i = tid; i < C; i += nt) {
         int inr;
         const float g = gr[i];
@@ -655,6 +718,7 @@ __global__ void __launch_bounds__(512) act_bwd_kernel(ActBwdArgs a) {
       return d;
     };
     if (P == AP_PLAIN || P == AP_LET) {
+      #pragma unroll 4
       for (int64_t i = tid; i < C; i += nt) {
         const float d = dxt(i);
         const float sv = a.s ? a.s[i] : 1.f;
@@ -665,6 +729,7 @@ __global__ void __launch_bounds__(512) act_bwd_kernel(ActBwdArgs a) {
       }
     } else if (P == AP_SWIGLU) {
       const float* ur = a.U + t * a.ldu;
+      #pragma unroll 4
       for (int64_t i = tid; i < C; i += nt) {
         const float d = dxt(i);
         const float g = xr[i], u = ur[i];
@@ -677,6 +742,7 @@ __global__ void __launch_bounds__(512) act_bwd_kernel(ActBwdArgs a) {
     } else {  // AP_RMS_LET: dX~ -> LET sums -> d(norm output) -> RMSNorm backward
       const float rstd = a.rstd[t];
       float dot = 0.f;
+      #pragma unroll 4
       for (int64_t i = tid; i < C; i += nt) {
         const float d = dxt(i);
         const float sv = a.s ? a.s[i] : 1.f;
@@ -688,6 +754,7 @@ __global__ void __launch_bounds__(512) act_bwd_kernel(ActBwdArgs a) {
       if (a.dX || a.dXb) {
         float2 tot = block_sum2(dot, 0.f, red_f);
         const float mean_dot = tot.x / (float)C;
+        #pragma unroll 4
         for (int64_t i = tid; i < C; i += nt) {
           const float an = xr[i] * rstd;
           float dx = rstd * (dn[i] - an * mean_dot);
@@ -700,6 +767,7 @@ __global__ void __launch_bounds__(512) act_bwd_kernel(ActBwdArgs a) {
     __syncthreads();
   }
   if (let_sums) {
+    #pragma unroll 4
     for (int64_t i = tid; i < C; i += nt) {
       a.part_s[(int64_t)blockIdx.x * C + i] = acc_s[i];
       a.part_d[(int64_t)blockIdx.x * C + i] = acc_d[i];

@@ -12,6 +12,7 @@ struct LwcFwdArgs {
   float* h; int32_t* z; int32_t* imax; int32_t* imin;
   const float* bias_delta; const float* bias_shift; float* Bt;
   float* ga_out; float* gb_out;                            // clipping strengths per group (nullable)
+  float* M_out; float* m_out;                              // group max / min of W~ (nullable)
   int wbits; float eps;
   int32_t* status;
 };
@@ -22,6 +23,7 @@ struct LwcBwdArgs {
   const float* s; const float* r;
   const float* gl; const float* bl; int lwc;
   const float* ga; const float* gb;                        // saved sigmoids (nullable: recomputed)
+  const float* Mv; const float* mv;                        // saved group max / min (nullable: re-read)
   const float* h; const int32_t* z; const int32_t* imax; const int32_t* imin;
   const float* dWq; int64_t ld_dwq;
   float* dgl; float* dbl; float* dWt; float* dr;
