@@ -137,6 +137,23 @@ omq_status omq_block_loss(omq_stream_t stream, int64_t n, const float* Yq, const
                           float* loss, float* dY, void* dY_bf16, void* workspace, size_t ws_bytes);
 size_t omq_loss_workspace_size(int64_t n);
 
+/* omq_block_loss for callers that cannot allocate device memory: code whose device memory belongs
+ * to another framework's fixed arena, interfaces that pass only inputs and outputs, and code that
+ * must not call cudaMalloc/cudaFree (which can synchronize the device) while work is in flight.
+ * The paper has no counterpart; it computes exactly what omq_block_loss computes.
+ *   Scratch: the partial sums live in a file-scope device array of 1024 floats (4 KB) that every
+ *   GPU which loads the library holds until the process exits.  No workspace argument, and no
+ *   cudaMalloc, cudaFree or allocating routine of any library is called.
+ *   Limit: 1 <= n <= OMQ_NOALLOC_LOSS_MAX_N; other sizes return OMQ_ERR_SHAPE before any launch.
+ *   Set-up: the first call on a device (with that device current) looks up the array's device
+ *   address with cudaGetSymbolAddress; make that first call before any stream capture.
+ *   Sharing: all calls on a device share the array and it keeps the last call's contents; each
+ *   call writes every partial it later reads, so nothing needs clearing.  Calls that overlap on
+ *   the GPU (different streams without ordering) race on the array: order them. */
+#define OMQ_NOALLOC_LOSS_MAX_N 2147483647LL
+omq_status omq_block_loss_noalloc(omq_stream_t stream, int64_t n, const float* Yq, const float* Yfp,
+                                  float* loss, float* dY, void* dY_bf16);
+
 /* Dense bf16 tensor-core matrix product used by every linear and attention product:
  *   C[b, m, n] = alpha * sum_k A[b, m, k] B[b, n, k] (+ bias[n]) (+ R[b, m, n]) (+ beta_acc * C)
  * A element (b, m, k) is at A + b*a_bs + (a_kmajor ? m*a_ld + k : k*a_ld + m); B likewise with n.

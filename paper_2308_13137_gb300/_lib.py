@@ -67,6 +67,7 @@ _SIGS = {
     "omq_act_bwd_workspace_size": (SZ, [I64, I64]),
     "omq_block_loss": (I32, [P, I64, P, P, P, P, P, P, SZ]),
     "omq_loss_workspace_size": (SZ, [I64]),
+    "omq_block_loss_noalloc": (I32, [P, I64, P, P, P, P, P]),
     "omq_gemm_bf16": (I32, [P, I64, I64, I64, I64, P, I64, I64, I32, P, I64, I64, I32, P, P, I64, I64, F32,
                             P, P, I64, F32, I32, P]),
     "omq_qlinear_fwd": (I32, [P, I64, I64, I64, P, P, P, P, P, P, P, P, P, P]),
@@ -196,6 +197,13 @@ def omq_block_loss(n, Yq, Yfp, loss, dY, dY_bf16, workspace, stream=None):
     ws_bytes = workspace.numel() * workspace.element_size()
     check("omq_block_loss", lib().omq_block_loss(stream_handle(stream), n, ptr(Yq), ptr(Yfp), ptr(loss), ptr(dY),
                                                  ptr(dY_bf16), ptr(workspace), ws_bytes))
+
+
+def omq_block_loss_noalloc(n, Yq, Yfp, loss, dY, dY_bf16, stream=None):
+    """omq_block_loss without a workspace: the scratch is a 4 KB device array inside the library.
+    For callers that cannot allocate device memory; calls that overlap on the GPU race."""
+    check("omq_block_loss_noalloc", lib().omq_block_loss_noalloc(stream_handle(stream), n, ptr(Yq), ptr(Yfp),
+                                                                 ptr(loss), ptr(dY), ptr(dY_bf16)))
 
 
 def omq_gemm_bf16(M, N, K, batch, A, a_ld, a_bs, a_kmajor, B, b_ld, b_bs, b_kmajor, Cf, Cb, ldc, c_bs, alpha=1.0,

@@ -1119,6 +1119,37 @@ omq_status omq_block_loss(omq_stream_t stream, int64_t n, const float* Yq, const
   return loss_launch((cudaStream_t)stream, n, Yq, Yfp, loss, dY, (__nv_bfloat16*)dY_bf16, (float*)workspace);
 }
 
+// ---- block loss without a caller workspace -------------------------------------------------------
+// Some callers cannot allocate device memory for a workspace: code whose device memory is owned by
+// another framework's fixed arena, plugin interfaces that pass only inputs and outputs, and code
+// that must not call cudaMalloc/cudaFree while other work is in flight (both can synchronize the
+// device).  This variant keeps the loss's partial sums in a file-scope device array instead.
+#define OMQ_NOALLOC_LOSS_PARTS 1024                   // partial sums: 4 KB per device
+#define OMQ_NOALLOC_MAX_DEVICES 64
+static __device__ __align__(256) float g_noalloc_loss_part[OMQ_NOALLOC_LOSS_PARTS];
+static std::atomic<float*> g_noalloc_loss_ptr[OMQ_NOALLOC_MAX_DEVICES];
+
+omq_status omq_block_loss_noalloc(omq_stream_t stream, int64_t n, const float* Yq, const float* Yfp, float* loss,
+                                  float* dY, void* dY_bf16) {
+  OMQ_REQUIRE(n > 0 && n <= OMQ_NOALLOC_LOSS_MAX_N, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(Yq && Yfp && loss, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(loss_parts(n) <= OMQ_NOALLOC_LOSS_PARTS, OMQ_ERR_SHAPE);
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return OMQ_ERR_CUDA;
+  OMQ_REQUIRE(dev >= 0 && dev < OMQ_NOALLOC_MAX_DEVICES, OMQ_ERR_UNSUPPORTED);
+  float* part = g_noalloc_loss_ptr[dev].load();
+  if (!part) {
+    // first call on this device: the host-side name of the array is not a device address, so
+    // ask the runtime for the array's address on the current device
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_loss_part) != cudaSuccess || !p) return OMQ_ERR_CUDA;
+    part = static_cast<float*>(p);
+    g_noalloc_loss_ptr[dev].store(part);
+  }
+  // every partial the final reduction reads is written by this call, so nothing needs clearing
+  return loss_launch((cudaStream_t)stream, n, Yq, Yfp, loss, dY, (__nv_bfloat16*)dY_bf16, part);
+}
+
 omq_status omq_adamw_update(omq_stream_t stream, int64_t n, float* p, const float* g, float* m, float* v, float lr,
                             float beta1, float beta2, float eps, float weight_decay, int32_t step) {
   OMQ_REQUIRE(n > 0, OMQ_ERR_SHAPE);
