@@ -203,6 +203,20 @@ def algorithmic_bytes(shape) -> float:
     return float(w_reads + 2 * acts + 2 * grads + streams)
 
 
+def _gemm_traffic():
+    """DRAM bytes per GEMM launch from the committed ncu capture, if it was taken of this exact
+    kernel source (else None)."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "gemm_traffic.json")) as fh:
+            d = json.load(fh)
+        with open(os.path.join(ROOT, d["source"]), "rb") as fh:
+            sha = hashlib.sha256(fh.read()).hexdigest()
+        return float(d["dram_bytes_per_launch"]) if sha == d["source_sha256"] else None
+    except Exception:
+        return None
+
+
 def run_ours(args, shape):
     import numpy as np
     import torch
@@ -312,7 +326,8 @@ def run_ours(args, shape):
                    "parallelism": "replicas" if ws > 1 else "single"},
         "roofline": {"bound": "tensor", "kernel": "gemm_bf16_kernel (tcgen05)",
                      "achieved": achieved, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
-                     "frac": achieved / peaks["bf16_sus"], "traffic": None,
+                     "frac": achieved / peaks["bf16_sus"], "traffic": _gemm_traffic(),
+                     "traffic_unit": "bytes per launch (ncu dram read+write, averaged over one step)",
                      "peak_kind": "%s bf16_tflops_sustained (timed inside the step)" % peaks["src"],
                      "gemm_share_of_step": gemm_ms_step / ms_step, "gemm_launches_per_step":
                          gemm_launches / args.steps},

@@ -123,6 +123,7 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int a_mn, int b_
 struct GemmParams {
   int M, N, K, batch;
   int a_mn, b_mn;            // 1 = MN-major operand
+  int n_fast;                // tile order: 1 = n fastest (A streamed once), 0 = m fastest (B streamed once)
   int causal;
   GemmEpilogue ep;
   int32_t* status;
@@ -147,8 +148,13 @@ struct TileInfo { int m0, n0, b, k_begin, nkb; bool skip; };
 __device__ __forceinline__ TileInfo tile_info(const GemmParams& p, int t, int bn) {
   const int mt = (p.M + BM - 1) / BM, nt = (p.N + bn - 1) / bn;
   TileInfo ti;
-  ti.m0 = (t % mt) * BM;
-  ti.n0 = ((t / mt) % nt) * bn;
+  if (p.n_fast) {
+    ti.n0 = (t % nt) * bn;
+    ti.m0 = ((t / nt) % mt) * BM;
+  } else {
+    ti.m0 = (t % mt) * BM;
+    ti.n0 = ((t / mt) % nt) * bn;
+  }
   ti.b = t / (mt * nt);
   ti.skip = (p.causal == 1 && ti.n0 > ti.m0 + BM - 1);   // keys beyond every query of the tile
   int k_end = p.K;
@@ -472,6 +478,9 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
   p.M = (int)M; p.N = (int)N; p.K = (int)K; p.batch = (int)batch;
   p.a_mn = A.kmajor ? 0 : 1; p.b_mn = B.kmajor ? 0 : 1;
   p.causal = causal; p.ep = ep; p.status = status;
+  // stream the larger operand once and keep the smaller one L2-resident: with m fastest, the
+  // CTAs working at one time share an N tile of B and sweep A; with n fastest, the reverse
+  p.n_fast = ((double)M > 1.5 * (double)N) ? 1 : 0;
   cudaEvent_t e0 = nullptr, e1 = nullptr;
   if (g_prof.on) {
     e0 = prof_event();
