@@ -526,278 +526,6 @@ omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a0, void* scratch) 
 }
 
 // ================================================================================================
-// per-token activation quantizer: one CTA per token row, row staged in shared memory.
-// ================================================================================================
-__device__ __forceinline__ float silu_f(float g) { return g / (1.f + expf(-g)); }
-
-template <int P>
-__device__ __forceinline__ void act_produce_row(const ActFwdArgs& a, int64_t t, float* row, float* red_f,
-                                                float* rstd_out) {
-  const int tid = threadIdx.x, nt = blockDim.x;
-  const int64_t C = a.C;
-  const float* xr = a.X + t * a.ldx;
-  if (P == AP_RMS_LET) {
-    float ss = 0.f;
-    #pragma unroll 4
-    for (int64_t i = tid; i < C / 4; i += nt) {
-      float4 v = __ldg(reinterpret_cast<const float4*>(xr) + i);
-      reinterpret_cast<float4*>(row)[i] = v;
-      ss = fmaf(v.x, v.x, ss); ss = fmaf(v.y, v.y, ss); ss = fmaf(v.z, v.z, ss); ss = fmaf(v.w, v.w, ss);
-    }
-    float2 tot = block_sum2(ss, 0.f, red_f);
-    float rstd = 1.0f / sqrtf(tot.x / (float)C + a.rms_eps);
-    *rstd_out = rstd;
-    #pragma unroll 4
-    for (int64_t i = tid; i < C; i += nt) {
-      float v = row[i] * rstd;
-      if (a.delta) v = v - a.delta[i];
-      if (a.s) v = __fdiv_rn(v, a.s[i]);
-      row[i] = v;
-    }
-  } else if (P == AP_SWIGLU) {
-    const float* ur = a.U + t * a.ldu;
-    #pragma unroll 4
-    for (int64_t i = tid; i < C / 4; i += nt) {
-      float4 g = __ldg(reinterpret_cast<const float4*>(xr) + i);
-      float4 u = __ldg(reinterpret_cast<const float4*>(ur) + i);
-      reinterpret_cast<float4*>(row)[i] = make_float4(silu_f(g.x) * u.x, silu_f(g.y) * u.y, silu_f(g.z) * u.z, silu_f(g.w) * u.w);
-    }
-  } else {
-    #pragma unroll 4
-    for (int64_t i = tid; i < C / 4; i += nt) {
-      float4 v = __ldg(reinterpret_cast<const float4*>(xr) + i);
-      if (P == AP_LET) {
-        float vv[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          int64_t c = 4 * i + e;
-          if (a.delta) vv[e] = vv[e] - a.delta[c];
-          if (a.s) vv[e] = __fdiv_rn(vv[e], a.s[c]);
-        }
-        v = make_float4(vv[0], vv[1], vv[2], vv[3]);
-      }
-      reinterpret_cast<float4*>(row)[i] = v;
-    }
-  }
-  __syncthreads();
-}
-
-template <int P>
-__global__ void __launch_bounds__(512) act_fwd_kernel(ActFwdArgs a) {
-  extern __shared__ float row[];
-  __shared__ float red_f[64];
-  __shared__ MaxMin red_mm[32];
-  const int tid = threadIdx.x, nt = blockDim.x;
-  const int64_t t = blockIdx.x;
-  const int64_t C = a.C;
-  float rstd = 0.f;
-  act_produce_row<P>(a, t, row, red_f, &rstd);
-  if (P == AP_RMS_LET && tid == 0 && a.rstd) a.rstd[t] = rstd;
-  __nv_bfloat16* qr = a.Xq + t * a.ldq;
-  if (a.abits >= 16) {
-    #pragma unroll 4
-    for (int64_t i = tid; i < C / 2; i += nt) {
-      float2 v = reinterpret_cast<float2*>(row)[i];
-      reinterpret_cast<__nv_bfloat162*>(qr)[i] = __floats2bfloat162_rn(v.x, v.y);
-    }
-    return;
-  }
-  MaxMin r = mm_identity();
-  #pragma unroll 4
-  for (int64_t i = tid; i < C; i += nt) mm_push(r, row[i], (int)i);
-  r = mm_block_reduce(r, red_mm);
-  const float Q = (float)((1 << a.abits) - 1);
-  QState qs = omq_qstate(r.M, r.m, 1.f, 1.f, Q, a.eps);
-  if (tid == 0) { a.h[t] = qs.h; a.z[t] = (int32_t)qs.z; a.imax[t] = r.iM; a.imin[t] = r.im; }
-  #pragma unroll 4
-  for (int64_t i = tid; i < C / 2; i += nt) {
-    float2 v = reinterpret_cast<float2*>(row)[i];
-    float c0, c1;
-    float q0 = omq_fakequant(v.x, qs, Q, &c0);
-    float q1 = omq_fakequant(v.y, qs, Q, &c1);
-    reinterpret_cast<__nv_bfloat162*>(qr)[i] = __floats2bfloat162_rn(q0, q1);
-    if (a.codes) {
-      uint8_t* cr = a.codes + t * C;
-      cr[2 * i] = (uint8_t)c0; cr[2 * i + 1] = (uint8_t)c1;
-    }
-  }
-}
-
-omq_status act_fwd_launch(cudaStream_t st, const ActFwdArgs& a) {
-  OMQ_REQUIRE(a.C % 8 == 0 && a.T > 0, OMQ_ERR_SHAPE);
-  size_t smem = a.C * sizeof(float);
-  OMQ_REQUIRE(smem <= 200 * 1024, OMQ_ERR_UNSUPPORTED);
-  void (*k)(ActFwdArgs) = nullptr;
-  switch (a.producer) {
-    case AP_PLAIN: k = act_fwd_kernel<AP_PLAIN>; break;
-    case AP_LET: k = act_fwd_kernel<AP_LET>; break;
-    case AP_RMS_LET: k = act_fwd_kernel<AP_RMS_LET>; break;
-    case AP_SWIGLU: k = act_fwd_kernel<AP_SWIGLU>; break;
-    default: return OMQ_ERR_INVALID_ARG;
-  }
-  if (smem + 2048 > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  k<<<(unsigned)a.T, a.C > 4096 ? 512 : ACT_THREADS, smem, st>>>(a);
-  OMQ_LAUNCH_CHECK();
-  return OMQ_OK;
-}
-
-// ---- backward ----------------------------------------------------------------------------------
-// Shared memory: row[C] (quantizer input of the token) | dn[C] (RMS only) | acc_s[C], acc_d[C]
-// (LET column partials only).  The per-element STE gradient is recomputed where it is used.
-template <int P>
-__global__ void __launch_bounds__(512) act_bwd_kernel(ActBwdArgs a) {
-  extern __shared__ float smem[];
-  const int64_t C = a.C;
-  const bool let_sums = a.part_s != nullptr;
-  float* row = smem;
-  float* dn = smem + C;
-  float* acc_s = smem + (P == AP_RMS_LET ? 2 : 1) * C;
-  float* acc_d = acc_s + C;
-  __shared__ float red_f[64];
-  const int tid = threadIdx.x, nt = blockDim.x;
-  if (let_sums)
-    #pragma unroll 4
-    for (int64_t i = tid; i < C; i += nt) { acc_s[i] = 0.f; acc_d[i] = 0.f; }
-  const int64_t t0 = (int64_t)blockIdx.x * a.rows_per_cta;
-  const int64_t t1 = min(a.T, t0 + a.rows_per_cta);
-  const bool quant = a.abits < 16;
-  const float Q = (float)((1 << (quant ? a.abits : 1)) - 1);
-
-  ActFwdArgs f;
-  f.producer = P; f.X = a.X; f.ldx = a.ldx; f.U = a.U; f.ldu = a.ldu; f.s = a.s; f.delta = a.delta;
-  f.rms_eps = 0.f; f.C = a.C;
-
-  for (int64_t t = t0; t < t1; ++t) {
-    // X~ of the token exactly as the forward formed it (RMS uses the saved rstd)
-    const float* xr = a.X + t * a.ldx;
-    if (P == AP_RMS_LET) {
-      const float rstd = a.rstd[t];
-      #pragma unroll 4
-      for (int64_t i = tid; i < C; i += nt) {
-        float v = xr[i] * rstd;
-        if (a.delta) v = v - a.delta[i];
-        if (a.s) v = __fdiv_rn(v, a.s[i]);
-        row[i] = v;
-      }
-      __syncthreads();
-    } else {
-      float dummy;
-      act_produce_row<P>(f, t, row, red_f, &dummy);
-    }
-    const float* gr = a.dXq + t * a.lddq;
-    QState qs;
-    int iM = -1, im = -1;
-    float GaM = 0.f, Gbt = 0.f;
-    if (quant) {
-      iM = a.imax[t]; im = a.imin[t];
-      qs = omq_qstate(row[iM], row[im], 1.f, 1.f, Q, a.eps);
-      qs.h = a.h[t]; qs.z = (float)a.z[t]; qs.rh = __frcp_rn(qs.h); qs.u = __fmul_rn(row[im], qs.rh);
-      float Gh = 0.f, Gbm = 0.f;
-      #pragma unroll 4
-      for (int64_t i = tid; i < C; i += nt) {
-        int inr;
-        const float g = gr[i];
-        const float dh = omq_ste_dh(row[i], qs, Q, &inr);
-        Gh = fmaf(g, dh, Gh);
-        if (!inr) Gbm += g;
-      }
-      float2 tot = block_sum2(Gh, Gbm, red_f);
-      const float Gh_t = qs.floored ? 0.f : tot.x;
-      GaM = Gh_t / Q;
-      Gbt = tot.y - Gh_t / Q;
-    }
-    // dL/dX~ of element i (straight-through, with the max/min routing)
-    auto dxt = [&](int64_t i) -> float {
-      const float g = gr[i];
-      if (!quant) return g;
-      int inr;
-      omq_ste_dh(row[i], qs, Q, &inr);
-      float d = inr ? g : 0.f;
-      if (i == iM) d += GaM;
-      if (i == im) d += Gbt;
-      return d;
-    };
-    if (P == AP_PLAIN || P == AP_LET) {
-      #pragma unroll 4
-      for (int64_t i = tid; i < C; i += nt) {
-        const float d = dxt(i);
-        const float sv = a.s ? a.s[i] : 1.f;
-        if (let_sums) { acc_s[i] -= d * row[i] / sv; acc_d[i] -= d / sv; }
-        const float dx = a.s ? __fdiv_rn(d, sv) : d;
-        if (a.dX) a.dX[t * a.lddx + i] = dx;
-        if (a.dXb) a.dXb[t * a.lddxb + i] = f_to_bf16(dx);
-      }
-    } else if (P == AP_SWIGLU) {
-      const float* ur = a.U + t * a.ldu;
-      #pragma unroll 4
-      for (int64_t i = tid; i < C; i += nt) {
-        const float d = dxt(i);
-        const float g = xr[i], u = ur[i];
-        const float sg = 1.f / (1.f + expf(-g));
-        const float dg = d * u * sg * (1.f + g * (1.f - sg));
-        const float du = d * g * sg;
-        if (a.dX) { a.dX[t * a.lddx + i] = dg; a.dU[t * a.lddx + i] = du; }
-        if (a.dXb) { a.dXb[t * a.lddxb + i] = f_to_bf16(dg); a.dUb[t * a.lddxb + i] = f_to_bf16(du); }
-      }
-    } else {  // AP_RMS_LET: dX~ -> LET sums -> d(norm output) -> RMSNorm backward
-      const float rstd = a.rstd[t];
-      float dot = 0.f;
-      #pragma unroll 4
-      for (int64_t i = tid; i < C; i += nt) {
-        const float d = dxt(i);
-        const float sv = a.s ? a.s[i] : 1.f;
-        if (let_sums) { acc_s[i] -= d * row[i] / sv; acc_d[i] -= d / sv; }
-        const float v = a.s ? __fdiv_rn(d, sv) : d;
-        dn[i] = v;
-        dot = fmaf(v, xr[i] * rstd, dot);
-      }
-      if (a.dX || a.dXb) {
-        float2 tot = block_sum2(dot, 0.f, red_f);
-        const float mean_dot = tot.x / (float)C;
-        #pragma unroll 4
-        for (int64_t i = tid; i < C; i += nt) {
-          const float an = xr[i] * rstd;
-          float dx = rstd * (dn[i] - an * mean_dot);
-          if (a.resid) dx += a.resid[t * a.lddx + i];
-          if (a.dX) a.dX[t * a.lddx + i] = dx;
-          if (a.dXb) a.dXb[t * a.lddxb + i] = f_to_bf16(dx);
-        }
-      }
-    }
-    __syncthreads();
-  }
-  if (let_sums) {
-    #pragma unroll 4
-    for (int64_t i = tid; i < C; i += nt) {
-      a.part_s[(int64_t)blockIdx.x * C + i] = acc_s[i];
-      a.part_d[(int64_t)blockIdx.x * C + i] = acc_d[i];
-    }
-  }
-}
-
-omq_status act_bwd_launch(cudaStream_t st, const ActBwdArgs& a0) {
-  ActBwdArgs a = a0;
-  OMQ_REQUIRE(a.C % 8 == 0 && a.T > 0, OMQ_ERR_SHAPE);
-  if (a.rows_per_cta <= 0) a.rows_per_cta = 4;
-  const int mult = (a.producer == AP_RMS_LET ? 2 : 1) + (a.part_s ? 2 : 0);
-  size_t smem = (size_t)mult * a.C * sizeof(float);
-  OMQ_REQUIRE(smem <= 200 * 1024, OMQ_ERR_UNSUPPORTED);
-  void (*k)(ActBwdArgs) = nullptr;
-  switch (a.producer) {
-    case AP_PLAIN: k = act_bwd_kernel<AP_PLAIN>; break;
-    case AP_LET: k = act_bwd_kernel<AP_LET>; break;
-    case AP_RMS_LET: k = act_bwd_kernel<AP_RMS_LET>; break;
-    case AP_SWIGLU: k = act_bwd_kernel<AP_SWIGLU>; break;
-    default: return OMQ_ERR_INVALID_ARG;
-  }
-  if (smem + 2048 > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  const unsigned grid = (unsigned)((a.T + a.rows_per_cta - 1) / a.rows_per_cta);
-  k<<<grid, a.C > 4096 ? 512 : 256, smem, st>>>(a);
-  OMQ_LAUNCH_CHECK();
-  return OMQ_OK;
-}
-
-// ================================================================================================
 // reductions, loss, small vector kernels
 // ================================================================================================
 // 32 columns per CTA, eight row phases per column; fixed summation order (deterministic)
