@@ -1,7 +1,8 @@
 // Dense bf16 matrix product on the 5th-generation tensor cores (sm_103a):
 // TMA (cp.async.bulk.tensor, 128-byte swizzle) -> shared-memory ring of STAGES slots guarded by
 // mbarriers -> tcgen05.mma (M = 128, N = BN, K = 16, fp32 accumulator in tensor memory) ->
-// tcgen05.ld epilogue (alpha, bias, residual, accumulate) -> fp32 / bf16 global stores.
+// tcgen05.ld epilogue (alpha, bias, residual, accumulate) -> fp32 output through TMA bulk tensor
+// stores from swizzled shared-memory staging blocks, bf16 output through direct global stores.
 //
 // Warp roles (192 threads): warp 0 issues TMA loads, warp 1 owns tensor memory and issues the
 // MMAs, warps 2..5 drain the accumulator (warp w reads TMEM lanes 32*(w%4) .. +31).
@@ -9,6 +10,7 @@
 // OMQ_ERR_TIMEOUT to the status word, stops issuing work, frees its tensor memory and exits.
 #include "gemm.cuh"
 #include <cuda.h>
+#include <cstring>
 #include <vector>
 
 namespace {
@@ -58,6 +60,20 @@ __device__ __forceinline__ void tma_load_3d(const CUtensorMap* map, uint64_t* ba
       ::"r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(bar))
       : "memory");
 }
+
+// fp32 block [32 rows x 32 cols] from shared memory to the C tensor; rows/columns outside the
+// tensor are clipped by the copy engine.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int c0, int c1, int c2) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.tile.bulk_group [%0, {%2, %3, %4}], [%1];"
+               ::"l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2)
+               : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// at most one committed store group may still be reading its shared-memory source
+__device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
@@ -129,13 +145,19 @@ struct GemmParams {
   int32_t* status;
 };
 
+constexpr int EPI_TILE_BYTES = 32 * 32 * 4;      // one 32 x 32 fp32 block, 128-byte rows
+
 template <int BN, int STAGES>
 struct SmemLayout {
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int BAR_OFF = STAGES * STAGE_BYTES;
+  static constexpr int EPI_OFF = STAGES * STAGE_BYTES;           // 1024-aligned (swizzle atom)
+  static constexpr int EPI_BYTES = 4 * 2 * EPI_TILE_BYTES;       // two staging blocks per epilogue warp
+  static constexpr int BAR_OFF = EPI_OFF + EPI_BYTES;
   static constexpr int TOTAL = BAR_OFF + 256 + 1024;  // + barriers + alignment slack
+  static_assert(EPI_OFF % 1024 == 0, "staging blocks must sit on the 1024-byte swizzle period");
+  static_assert(TOTAL <= 227 * 1024, "shared memory per CTA");
 };
 
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
@@ -172,7 +194,7 @@ __device__ __forceinline__ TileInfo tile_info(const GemmParams& p, int t, int bn
 template <int BN, int STAGES>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                     const GemmParams p) {
+                     const __grid_constant__ CUtensorMap tmC, const GemmParams p) {
   using L = SmemLayout<BN, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -266,8 +288,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else if (warp >= 2) {
     // ---------------- epilogue ----------------
+    // fp32 output leaves through TMA bulk stores: each warp stages its 32 x 32 block in one of two
+    // 128-byte-swizzled shared-memory slots (16-byte chunk c of row r at chunk c ^ (r & 7), so the
+    // eight rows of a quarter-warp hit distinct banks) and one lane issues the store.  bf16 output
+    // is written directly from registers.
     const int q = warp & 3;                       // TMEM lane quadrant of this warp
     const GemmEpilogue& ep = p.ep;
+    uint8_t* stage_base = smem + L::EPI_OFF + q * 2 * EPI_TILE_BYTES;
+    uint32_t n_stores = 0;
     uint32_t acc_it = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
       const TileInfo ti = tile_info(p, t, BN);
@@ -280,7 +308,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (!ok) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; }
         tc_fence_after();
       }
-      const int row = ti.m0 + q * 32 + lane;
+      const int row0 = ti.m0 + q * 32;
+      const int row = row0 + lane;
       const bool row_ok = row < p.M;
       const int64_t crow = (int64_t)ti.b * ep.c_bs + (int64_t)row * ep.ldc;
 #pragma unroll 1
@@ -298,11 +327,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           for (int i = 0; i < 32; ++i) v[i] = 0.f;
         }
         const int nb = ti.n0 + j0;
-        if (!row_ok || nb >= p.N) continue;
+        if (row0 >= p.M || nb >= p.N) continue;   // warp-uniform: block wholly outside C
         const bool full_chunk = nb + 32 <= p.N;
 #pragma unroll
         for (int i = 0; i < 32; ++i) v[i] *= ep.alpha;
-        if (full_chunk) {
+        if (row_ok && full_chunk) {
           if (ep.bias) {
 #pragma unroll
             for (int i = 0; i < 32; i += 4) {
@@ -318,41 +347,54 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               v[i] += tt.x; v[i + 1] += tt.y; v[i + 2] += tt.z; v[i + 3] += tt.w;
             }
           }
-          if (ep.Cf) {
-            float* cp = ep.Cf + crow + nb;
-            if (ep.beta_acc != 0.f) {
+          if (ep.Cf && ep.beta_acc != 0.f) {
+            const float* cp = ep.Cf + crow + nb;
 #pragma unroll
-              for (int i = 0; i < 32; i += 4) {
-                float4 tt = *reinterpret_cast<const float4*>(cp + i);
-                v[i] += ep.beta_acc * tt.x; v[i + 1] += ep.beta_acc * tt.y;
-                v[i + 2] += ep.beta_acc * tt.z; v[i + 3] += ep.beta_acc * tt.w;
-              }
+            for (int i = 0; i < 32; i += 4) {
+              float4 tt = *reinterpret_cast<const float4*>(cp + i);
+              v[i] += ep.beta_acc * tt.x; v[i + 1] += ep.beta_acc * tt.y;
+              v[i + 2] += ep.beta_acc * tt.z; v[i + 3] += ep.beta_acc * tt.w;
             }
-#pragma unroll
-            for (int i = 0; i < 32; i += 4) *reinterpret_cast<float4*>(cp + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
           }
           if (ep.Cb) {
             __nv_bfloat16* cp = ep.Cb + crow + nb;
 #pragma unroll
             for (int i = 0; i < 32; i += 8) *reinterpret_cast<uint4*>(cp + i) = pack_bf16x8(v + i);
           }
-        } else {
-          for (int i = 0; i < 32 && nb + i < p.N; ++i) {
+        } else if (row_ok) {                      // ragged last column block
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
             const int n = nb + i;
-            float x = v[i];
-            if (ep.bias) x += ep.bias[n];
-            if (ep.R) x += ep.R[(int64_t)ti.b * ep.c_bs + (int64_t)row * ep.ldr + n];
-            if (ep.Cf) {
-              if (ep.beta_acc != 0.f) x += ep.beta_acc * ep.Cf[crow + n];
-              ep.Cf[crow + n] = x;
+            if (n < p.N) {
+              if (ep.bias) v[i] += ep.bias[n];
+              if (ep.R) v[i] += ep.R[(int64_t)ti.b * ep.c_bs + (int64_t)row * ep.ldr + n];
+              if (ep.Cf && ep.beta_acc != 0.f) v[i] += ep.beta_acc * ep.Cf[crow + n];
+              if (ep.Cb) ep.Cb[crow + n] = f_to_bf16(v[i]);
             }
-            if (ep.Cb) ep.Cb[crow + n] = f_to_bf16(x);
           }
+        }
+        if (ep.Cf) {
+          uint8_t* stg = stage_base + (n_stores & 1) * EPI_TILE_BYTES;
+          if (lane == 0) bulk_wait_read1();       // the store that last used this slot has read it
+          __syncwarp();
+          uint8_t* my_row = stg + lane * 128;
+#pragma unroll
+          for (int c = 0; c < 8; ++c)
+            *reinterpret_cast<float4*>(my_row + ((c ^ (lane & 7)) << 4)) =
+                make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+          fence_async_smem();                     // generic-proxy writes -> visible to the copy engine
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_3d(&tmC, stg, nb, row0, ti.b);
+            bulk_commit();
+          }
+          ++n_stores;
         }
       }
       if (has_acc) ++acc_it;
       if (!ok) break;
     }
+    if (lane == 0) bulk_wait_all();
   }
   tc_fence_before();
   __syncthreads();
@@ -396,8 +438,23 @@ bool make_map(CUtensorMap* map, const void* ptr, int64_t inner, int64_t rows, in
   return r == CUDA_SUCCESS;
 }
 
+// 3-D fp32 map of the output {cols, rows, batch} with a {32, 32, 1} box and 128-byte swizzle
+// (the layout of the epilogue's staging blocks).
+bool make_map_c(CUtensorMap* map, float* ptr, int64_t N, int64_t M, int64_t batch, int64_t ldc, int64_t cbs) {
+  PFN_encodeTiled_t enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)N, (cuuint64_t)M, (cuuint64_t)batch};
+  cuuint64_t strides[2] = {(cuuint64_t)(ldc * 4), (cuuint64_t)((batch > 1 ? cbs : ldc * M) * 4)};
+  cuuint32_t box[3] = {32u, 32u, 1u};
+  cuuint32_t estr[3] = {1u, 1u, 1u};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, ptr, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 template <int BN, int STAGES>
-omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap& tb, const GemmParams& p) {
+omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
+                      const GemmParams& p) {
   using L = SmemLayout<BN, STAGES>;
   static bool attr_set = false;
   if (!attr_set) {
@@ -409,7 +466,7 @@ omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap&
   const int64_t tiles = (int64_t)((p.M + BM - 1) / BM) * ((p.N + BN - 1) / BN) * p.batch;
   const int64_t sms = omq_num_sms();
   const unsigned grid = (unsigned)(tiles < sms ? tiles : sms);
-  gemm_bf16_kernel<BN, STAGES><<<grid, NUM_THREADS, L::TOTAL, st>>>(ta, tb, p);
+  gemm_bf16_kernel<BN, STAGES><<<grid, NUM_THREADS, L::TOTAL, st>>>(ta, tb, tc, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -464,6 +521,7 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
   OMQ_REQUIRE(omq_aligned16(A.ptr) && omq_aligned16(B.ptr), OMQ_ERR_ALIGN);
   OMQ_REQUIRE(A.ld % 8 == 0 && B.ld % 8 == 0 && (batch == 1 || (A.bs % 8 == 0 && B.bs % 8 == 0)), OMQ_ERR_ALIGN);
   OMQ_REQUIRE(ep.ldc % 8 == 0 && (batch == 1 || ep.c_bs % 8 == 0), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(ep.ldc >= N, OMQ_ERR_SHAPE);
   OMQ_REQUIRE((!ep.Cf || omq_aligned16(ep.Cf)) && (!ep.Cb || omq_aligned16(ep.Cb)), OMQ_ERR_ALIGN);
   OMQ_REQUIRE(!ep.R || (omq_aligned16(ep.R) && ep.ldr % 4 == 0), OMQ_ERR_ALIGN);
   OMQ_REQUIRE(!ep.bias || omq_aligned16(ep.bias), OMQ_ERR_ALIGN);
@@ -473,6 +531,9 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
   const int bn = wide ? 256 : 128;
   bool ok = A.kmajor ? make_map(&ta, A.ptr, K, M, batch, A.ld, A.bs, BM) : make_map(&ta, A.ptr, M, K, batch, A.ld, A.bs, BK);
   ok = ok && (B.kmajor ? make_map(&tb, B.ptr, K, N, batch, B.ld, B.bs, bn) : make_map(&tb, B.ptr, N, K, batch, B.ld, B.bs, BK));
+  CUtensorMap tc;
+  memset(&tc, 0, sizeof(tc));
+  if (ep.Cf) ok = ok && make_map_c(&tc, ep.Cf, N, M, batch, ep.ldc, ep.c_bs);
   if (!ok) return OMQ_ERR_UNSUPPORTED;
   GemmParams p;
   p.M = (int)M; p.N = (int)N; p.K = (int)K; p.batch = (int)batch;
@@ -490,7 +551,7 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
       g_prof.flops += gemm_algorithmic_flops(M, N, K, batch, causal);
     }
   }
-  omq_status r = wide ? launch_cfg<256, 4>(st, ta, tb, p) : launch_cfg<128, 6>(st, ta, tb, p);
+  omq_status r = wide ? launch_cfg<256, 4>(st, ta, tb, tc, p) : launch_cfg<128, 6>(st, ta, tb, tc, p);
   if (e0 && e1) cudaEventRecord(e1, st);
   return r;
 }
