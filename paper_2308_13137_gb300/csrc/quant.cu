@@ -4,6 +4,9 @@
 #include "quant.cuh"
 
 #include <atomic>
+#include <cooperative_groups.h>
+
+namespace cg = cooperative_groups;
 
 
 static std::atomic<long long> g_launches{0};
@@ -528,7 +531,8 @@ omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a0, void* scratch) 
 // ================================================================================================
 // reductions, loss, small vector kernels
 // ================================================================================================
-// 32 columns per CTA, eight row phases per column; fixed summation order (deterministic)
+// 32 columns per CTA, eight row phases per column; fixed summation order (deterministic).
+// Used when the column count or a pointer does not allow 16-byte accesses.
 __global__ void omq_colsum_partials_kernel(const float* __restrict__ part, int64_t P, int64_t C,
                                            float* __restrict__ out, float scale, int accumulate) {
   __shared__ float red[8][33];
@@ -548,9 +552,65 @@ __global__ void omq_colsum_partials_kernel(const float* __restrict__ part, int64
   }
 }
 
+// 128 columns per cluster of eight CTAs: CTA k of the cluster sums the k-th contiguous eighth of
+// the P partial rows (its eight warps take every eighth row, four loads in flight per thread),
+// and CTA 0 adds the eight CTA sums in rank order through distributed shared memory.  The
+// summation order is fixed, so the result does not depend on scheduling.
+#define COLSUM_CLUSTER 8
+__device__ __forceinline__ void add4(float4& a, const float4 b) { a.x += b.x; a.y += b.y; a.z += b.z; a.w += b.w; }
+
+__global__ void __cluster_dims__(1, COLSUM_CLUSTER, 1) __launch_bounds__(256)
+    colsum_cluster_kernel(const float* __restrict__ part, int64_t P, int64_t C, float* __restrict__ out, float scale,
+                          int accumulate) {
+  __shared__ float4 red[8][32];
+  __shared__ float4 cta_sum[32];
+  cg::cluster_group cluster = cg::this_cluster();
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const unsigned rank = cluster.block_rank();
+  const int64_t nc4 = C / 4;
+  const int64_t c4 = (int64_t)blockIdx.x * 32 + lane;
+  const int64_t rows_per = (P + COLSUM_CLUSTER - 1) / COLSUM_CLUSTER;
+  const int64_t r0 = (int64_t)rank * rows_per, r1 = min(P, r0 + rows_per);
+  float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (c4 < nc4) {
+    const float4* base = reinterpret_cast<const float4*>(part) + c4;
+    int64_t r = r0 + w;
+    for (; r + 24 < r1; r += 32) {
+      const float4 v0 = __ldg(base + r * nc4), v1 = __ldg(base + (r + 8) * nc4);
+      const float4 v2 = __ldg(base + (r + 16) * nc4), v3 = __ldg(base + (r + 24) * nc4);
+      add4(s, v0); add4(s, v1); add4(s, v2); add4(s, v3);
+    }
+    for (; r < r1; r += 8) add4(s, __ldg(base + r * nc4));
+  }
+  red[w][lane] = s;
+  __syncthreads();
+  if (w == 0) {
+    float4 t = red[0][lane];
+#pragma unroll
+    for (int k = 1; k < 8; ++k) add4(t, red[k][lane]);
+    cta_sum[lane] = t;
+  }
+  cluster.sync();
+  if (rank == 0 && w == 0 && c4 < nc4) {
+    float4 t = cta_sum[lane];
+#pragma unroll
+    for (int k = 1; k < COLSUM_CLUSTER; ++k) add4(t, cluster.map_shared_rank(cta_sum, k)[lane]);
+    t.x *= scale; t.y *= scale; t.z *= scale; t.w *= scale;
+    float4* o = reinterpret_cast<float4*>(out) + c4;
+    if (accumulate) add4(t, *o);
+    *o = t;
+  }
+  cluster.sync();                  // keep every CTA's shared memory alive until CTA 0 has read it
+}
+
 omq_status omq_colsum_partials(cudaStream_t st, const float* part, int64_t P, int64_t C, float* out,
                                float scale, int accumulate) {
-  omq_colsum_partials_kernel<<<(unsigned)((C + 31) / 32), 256, 0, st>>>(part, P, C, out, scale, accumulate);
+  if (C % 4 == 0 && omq_aligned16(part) && omq_aligned16(out)) {
+    dim3 grid((unsigned)((C / 4 + 31) / 32), COLSUM_CLUSTER);
+    colsum_cluster_kernel<<<grid, 256, 0, st>>>(part, P, C, out, scale, accumulate);
+  } else {
+    omq_colsum_partials_kernel<<<(unsigned)((C + 31) / 32), 256, 0, st>>>(part, P, C, out, scale, accumulate);
+  }
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }

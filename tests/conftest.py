@@ -10,6 +10,7 @@ if ROOT not in sys.path:
 
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (sm_103a) and the built libomq")
+    config.addinivalue_line("markers", "full: runs the full workload sizes (minutes of oracle time on the host)")
 
 
 @pytest.fixture(scope="session")
