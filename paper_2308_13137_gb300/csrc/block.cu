@@ -23,6 +23,18 @@ typedef __nv_bfloat16 bf16;
 
 struct QState4 { float* h; int32_t* z; int32_t* imax; int32_t* imin; float* ga; float* gb; float* M; float* m; };
 
+// Scratch (floats) of the fused weight-gradient + LWC backward of one [Cout, Cin] weight
+int64_t lwc_fused_scratch_elems(int64_t Cout, int64_t Cin) {
+  const int64_t ntn = (Cin + gemm_n_tile(Cin) - 1) / gemm_n_tile(Cin);
+  return 2 * ((Cout + 31) / 32) * Cin + 3 * Cout * ntn + 64;
+}
+
+bool lwc_fused_ok(int64_t Cin, int group, bool let_terms) {
+  if (Cin % 32 != 0) return false;
+  if (group == Cin) return true;
+  return !let_terms && group % 32 == 0 && gemm_n_tile(Cin) % group == 0;
+}
+
 QState4 take_qstate(Carve& c, size_t n, bool saved = false) {
   QState4 q;
   q.h = c.take<float>(n); q.z = c.take<int32_t>(n); q.imax = c.take<int32_t>(n); q.imin = c.take<int32_t>(n);
@@ -141,6 +153,10 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   pe = imax64(pe, (int64_t)lwc_bwd_scratch_bytes(d, dq) / 4 + 64);
   pe = imax64(pe, (int64_t)lwc_bwd_scratch_bytes(2 * f, d) / 4 + 64);
   pe = imax64(pe, (int64_t)lwc_bwd_scratch_bytes(d, f) / 4 + 64);
+  pe = imax64(pe, lwc_fused_scratch_elems(nqkv, d));
+  pe = imax64(pe, lwc_fused_scratch_elems(d, dq));
+  pe = imax64(pe, lwc_fused_scratch_elems(2 * f, d));
+  pe = imax64(pe, lwc_fused_scratch_elems(d, f));
   pe = imax64(pe, 2 * ((T + 3) / 4) * imax64(d, dq));
   pe = imax64(pe, qkv_bwd_nslab((int)T) * (dq + dkv));
   pe = imax64(pe, colsum_rows_parts(T) * imax64(2 * f, nqkv));
@@ -213,6 +229,43 @@ omq_status lwc_bwd_full(cudaStream_t st, const bf16* W, int64_t Cout, int64_t Ci
   // dgamma/dbeta follow cfg.accumulate; the LET sums follow the caller; dr is scratch
   a.accumulate = cfg.accumulate; a.accumulate_sd = accumulate_sd; a.accumulate_dr = 0;
   return lwc_bwd_launch(st, a, part);
+}
+
+// dW_hat = dY^T X_hat and the straight-through LWC backward of W (Eq. 2, Eq. 3): the per-element
+// part runs in the GEMM epilogue (dW_hat stays in tensor memory), the reductions finish after it.
+// Falls back to the stored dW_hat + separate LWC backward for layouts the epilogue does not take.
+omq_status lwc_bwd_dw(cudaStream_t st, int64_t T, const bf16* dY, const bf16* Xh, const bf16* W, int64_t Cout,
+                      int64_t Cin, const omq_qcfg& cfg, const float* s, const float* r, const float* gl,
+                      const float* bl, const QState4& q, float* dgl, float* dbl, float* dr, const float* dBt, float* ds,
+                      float* ddelta, int accumulate_sd, float* part, float* dW_fallback, int32_t* status) {
+  const int group = cfg.group == 0 ? (int)Cin : cfg.group;
+  const bool let_terms = s || r || dBt || ds || ddelta || dr;
+  if (!lwc_fused_ok(Cin, group, let_terms)) {
+    OMQ_TRY(gemm_dw(st, T, Cout, Cin, dY, Xh, dW_fallback, status));
+    return lwc_bwd_full(st, W, Cout, Cin, cfg, s, r, gl, bl, q, dW_fallback, dgl, dbl, dr, dBt, ds, ddelta,
+                        accumulate_sd, part);
+  }
+  const int64_t P = (Cout + 31) / 32;
+  const int ntn = (int)((Cin + gemm_n_tile(Cin) - 1) / gemm_n_tile(Cin));
+  GemmLwcEpi lw{};
+  lw.W = W; lw.s = s; lw.r = r; lw.h = q.h; lw.z = q.z; lw.ga = q.ga; lw.gb = q.gb; lw.Mv = q.M; lw.mv = q.m;
+  lw.dBt = dBt;
+  lw.part_s = ds ? part : nullptr;
+  lw.part_d = (ddelta && dBt) ? part + P * Cin : nullptr;
+  lw.rowpart = part + 2 * P * Cin;
+  lw.dgl = dgl; lw.dbl = dbl;
+  lw.group = group; lw.accumulate = cfg.accumulate; lw.ntn = ntn;
+  lw.Q = (float)((1 << cfg.wbits) - 1); lw.eps = cfg.h_eps;
+  GemmOperand a{dY, Cout, 0, 0}, b{Xh, Cin, 0, 0};
+  OMQ_TRY(gemm_launch_lwc(st, Cout, Cin, T, a, b, lw, status));
+  LwcBwdArgs la{};
+  la.W = W; la.Cout = Cout; la.Cin = Cin; la.group = group;
+  la.s = s; la.r = r; la.gl = gl; la.bl = bl; la.lwc = 1; la.ga = q.ga; la.gb = q.gb; la.Mv = q.M; la.mv = q.m;
+  la.h = q.h; la.z = q.z; la.imax = q.imax; la.imin = q.imin;
+  la.dgl = dgl; la.dbl = dbl; la.dWt = nullptr; la.dr = dr; la.dBt = dBt; la.ds = ds; la.ddelta = ddelta;
+  la.wbits = cfg.wbits; la.eps = cfg.h_eps;
+  la.accumulate = cfg.accumulate; la.accumulate_sd = accumulate_sd; la.accumulate_dr = 0;
+  return lwc_bwd_fused_finish(st, la, lw.rowpart, ntn, lw.part_s, lw.part_d, P);
 }
 
 struct Ctx {
@@ -322,9 +375,8 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
 
   // ---- down_proj ----------------------------------------------------------------------------------
   OMQ_TRY(gemm_dx(st, c.T, c.d, c.f, w.dy_b, w.Wd_h, w.dm, status));
-  OMQ_TRY(gemm_dw(st, c.T, c.d, c.f, w.dy_b, w.m_h, w.dW, status));
-  OMQ_TRY(lwc_bwd_full(st, Wd, c.d, c.f, cfg, nullptr, nullptr, th->gamma_d, th->beta_d, w.sq_d, w.dW, g->gamma_d,
-                       g->beta_d, nullptr, nullptr, nullptr, nullptr, 0, w.part));
+  OMQ_TRY(lwc_bwd_dw(st, c.T, w.dy_b, w.m_h, Wd, c.d, c.f, cfg, nullptr, nullptr, th->gamma_d, th->beta_d, w.sq_d,
+                     g->gamma_d, g->beta_d, nullptr, nullptr, nullptr, nullptr, 0, w.part, w.dW, status));
   ActBwdArgs bm{};
   bm.producer = AP_SWIGLU; bm.X = w.Ygu; bm.ldx = 2 * c.f; bm.U = w.Ygu + c.f; bm.ldu = 2 * c.f; bm.T = c.T; bm.C = c.f;
   bm.h = w.sm.h; bm.z = w.sm.z; bm.imax = w.sm.imax; bm.imin = w.sm.imin; bm.dXq = w.dm; bm.lddq = c.f;
@@ -334,11 +386,11 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
 
   // ---- gate / up ----------------------------------------------------------------------------------
   OMQ_TRY(gemm_dx(st, c.T, 2 * c.f, c.d, w.dYgu_b, w.Wgu_h, w.db, status));
-  OMQ_TRY(gemm_dw(st, c.T, 2 * c.f, c.d, w.dYgu_b, w.b_h, w.dW, status));
   if (c.let) OMQ_TRY(colsum_rows(st, w.dYgu, c.T, 2 * c.f, 2 * c.f, w.part, w.dB_gu, 1.f, 0));
-  OMQ_TRY(lwc_bwd_full(st, Wgu, 2 * c.f, c.d, cfg, c.let ? th->s2 : nullptr, nullptr, th->gamma_gu, th->beta_gu,
-                       w.sq_gu, w.dW, g->gamma_gu, g->beta_gu, nullptr, c.let ? w.dB_gu : nullptr,
-                       c.let ? g->s2 : nullptr, c.let ? g->d2 : nullptr, acc, w.part));
+  OMQ_TRY(lwc_bwd_dw(st, c.T, w.dYgu_b, w.b_h, Wgu, 2 * c.f, c.d, cfg, c.let ? th->s2 : nullptr, nullptr,
+                     th->gamma_gu, th->beta_gu, w.sq_gu, g->gamma_gu, g->beta_gu, nullptr,
+                     c.let ? w.dB_gu : nullptr, c.let ? g->s2 : nullptr, c.let ? g->d2 : nullptr, acc, w.part, w.dW,
+                     status));
   ActBwdArgs bb{};
   bb.producer = AP_RMS_LET; bb.X = w.h1; bb.ldx = c.d; bb.s = c.let ? th->s2 : nullptr; bb.delta = c.let ? th->d2 : nullptr;
   bb.rstd = w.rstd2; bb.T = c.T; bb.C = c.d; bb.h = w.sb.h; bb.z = w.sb.z; bb.imax = w.sb.imax; bb.imin = w.sb.imin;
@@ -353,11 +405,10 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
 
   // ---- o_proj -------------------------------------------------------------------------------------
   OMQ_TRY(gemm_dx(st, c.T, c.d, c.dq, w.dh1_b, w.Wo_h, w.dOh, status));
-  OMQ_TRY(gemm_dw(st, c.T, c.d, c.dq, w.dh1_b, w.O_h, w.dW, status));
   if (c.let) OMQ_TRY(colsum_rows(st, w.dh1, c.T, c.d, c.d, w.part, w.dB_o, 1.f, 0));
-  OMQ_TRY(lwc_bwd_full(st, Wo, c.d, c.dq, cfg, c.let ? w.so_exp : nullptr, nullptr, th->gamma_o, th->beta_o, w.sq_o,
-                       w.dW, g->gamma_o, g->beta_o, nullptr, c.let ? w.dB_o : nullptr, c.let ? w.vtmp0 : nullptr,
-                       c.let ? w.vtmp1 : nullptr, 0, w.part));
+  OMQ_TRY(lwc_bwd_dw(st, c.T, w.dh1_b, w.O_h, Wo, c.d, c.dq, cfg, c.let ? w.so_exp : nullptr, nullptr, th->gamma_o,
+                     th->beta_o, w.sq_o, g->gamma_o, g->beta_o, nullptr, c.let ? w.dB_o : nullptr,
+                     c.let ? w.vtmp0 : nullptr, c.let ? w.vtmp1 : nullptr, 0, w.part, w.dW, status));
   ActBwdArgs bo{};
   bo.producer = AP_PLAIN; bo.X = w.O; bo.ldx = c.dq; bo.T = c.T; bo.C = c.dq; bo.h = w.so.h; bo.z = w.so.z;
   bo.imax = w.so.imax; bo.imin = w.so.imin; bo.dXq = w.dOh; bo.lddq = c.dq; bo.dX = nullptr; bo.lddx = c.dq;
@@ -411,11 +462,11 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   }
 
   // ---- q / k / v projections ---------------------------------------------------------------------------
-  OMQ_TRY(gemm_dw(st, c.T, c.nqkv, c.d, w.dYqkv_b, w.a_h, w.dW, status));
   if (c.let) OMQ_TRY(colsum_rows(st, w.dYqkv, c.T, c.nqkv, c.nqkv, w.part, w.dB_qkv, 1.f, 0));
-  OMQ_TRY(lwc_bwd_full(st, Wqkv, c.nqkv, c.d, cfg, c.let ? th->s1 : nullptr, c.let ? w.r_qkv : nullptr, th->gamma_qkv,
-                       th->beta_qkv, w.sq_qkv, w.dW, g->gamma_qkv, g->beta_qkv, c.let ? w.dr_qkv : nullptr,
-                       c.let ? w.dB_qkv : nullptr, c.let ? g->s1 : nullptr, c.let ? g->d1 : nullptr, acc, w.part));
+  OMQ_TRY(lwc_bwd_dw(st, c.T, w.dYqkv_b, w.a_h, Wqkv, c.nqkv, c.d, cfg, c.let ? th->s1 : nullptr,
+                     c.let ? w.r_qkv : nullptr, th->gamma_qkv, th->beta_qkv, w.sq_qkv, g->gamma_qkv, g->beta_qkv,
+                     c.let ? w.dr_qkv : nullptr, c.let ? w.dB_qkv : nullptr, c.let ? g->s1 : nullptr,
+                     c.let ? g->d1 : nullptr, acc, w.part, w.dW, status));
   if (c.let) {
     const int64_t off = c.dq + c.dkv;
     OMQ_TRY(let_vo_finalize(st, (int)c.dkv, th->so, w.dr_qkv + off, w.dB_qkv + off, w.B_qkv + off, g->so, g->do_, 1));

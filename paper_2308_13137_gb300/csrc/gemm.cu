@@ -142,6 +142,7 @@ struct GemmParams {
   int n_fast;                // tile order: 1 = n fastest (A streamed once), 0 = m fastest (B streamed once)
   int causal;
   GemmEpilogue ep;
+  GemmLwcEpi lw;             // used by the LWC-epilogue instantiation only
   int32_t* status;
 };
 
@@ -187,11 +188,162 @@ __device__ __forceinline__ TileInfo tile_info(const GemmParams& p, int t, int bn
   return ti;
 }
 
+// Column sums of a warp's 32 x 32 block: on entry lane L holds row L's 32 values, on exit v[0]
+// of lane L is the sum over the 32 rows of column L (five butterfly exchange stages, 31 shuffles).
+__device__ __forceinline__ float colsum_warp32(float (&v)[32], int lane) {
+#pragma unroll
+  for (int k = 16; k >= 1; k >>= 1) {
+    const bool up = (lane & k) != 0;
+#pragma unroll
+    for (int i = 0; i < k; ++i) {
+      const float send = up ? v[i] : v[i + k];
+      const float keep = up ? v[i + k] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, k);
+    }
+  }
+  return v[0];
+}
+
+__device__ __forceinline__ void ldw32(const __nv_bfloat16* p, bool ok, uint4 (&r)[4]) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) r[i] = ok ? __ldg(reinterpret_cast<const uint4*>(p) + i) : make_uint4(0, 0, 0, 0);
+}
+
+// Epilogue of the weight-gradient product with the straight-through LWC backward (Eq. 2) fused:
+// the accumulator dW_hat is consumed from tensor memory 32 columns at a time and never stored.
+// The weight row chunk of the next 32 columns is loaded while the current one is processed.
+template <int BN>
+__device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem, uint64_t* acc_full, uint64_t* acc_empty,
+                                             volatile int* abort_flag, int q, int lane, int total) {
+  const GemmLwcEpi& L = p.lw;
+  const int N = p.N;
+  const bool perch = L.group == N;
+  const int ngroups = N / L.group;
+  uint32_t acc_it = 0;
+  for (int t = blockIdx.x; t < total; t += gridDim.x) {
+    const TileInfo ti = tile_info(p, t, BN);
+    if (ti.skip) continue;
+    const bool has_acc = ti.nkb > 0;
+    const uint32_t buf = acc_it & 1;
+    bool ok = true;
+    if (has_acc) {
+      ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[buf], (acc_it >> 1) & 1));
+      if (!ok) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; }
+      tc_fence_after();
+    }
+    const int row0 = ti.m0 + q * 32;
+    const int row = row0 + lane;
+    const bool row_ok = row < p.M;
+    const bool quad_ok = row0 < p.M;
+    const float rr = (L.r && row_ok) ? L.r[row] : 1.f;
+    const float dbr = (L.dBt && row_ok) ? __fmul_rn(L.dBt[row], rr) : 0.f;
+    const __nv_bfloat16* wrow = L.W + (int64_t)(row_ok ? row : 0) * N;
+    QState qs;
+    qs.h = 1.f; qs.rh = 1.f; qs.z = 0.f; qs.u = 0.f; qs.b = 0.f; qs.m = 0.f; qs.a = 0.f; qs.M = 0.f; qs.floored = 0;
+    int64_t gk = 0;                                // (row, group) index of the current group
+    float Gh = 0.f, Gbm = 0.f, drm = 0.f;
+    uint4 wcur[4], wnext[4];
+    ldw32(wrow + ti.n0, row_ok && ti.n0 < N, wcur);
+#pragma unroll 1
+    for (int j0 = 0; j0 < BN; j0 += 32) {
+      float g[32];
+      if (has_acc && ok) {
+        tmem_ld32(tmem + buf * BN + ((uint32_t)(q * 32) << 16) + (uint32_t)j0, g);
+        if (j0 + 32 == BN) {                      // accumulator drained: hand the buffer back
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[buf]);
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) g[i] = 0.f;
+      }
+      const int nb = ti.n0 + j0;
+      if (j0 + 32 < BN) ldw32(wrow + nb + 32, row_ok && nb + 32 < N, wnext);
+      if (quad_ok && nb < N) {
+        if (nb % L.group == 0 && row_ok) {       // quantizer state of the group starting here
+          gk = perch ? (int64_t)row : (int64_t)row * ngroups + nb / L.group;
+          qs.h = L.h[gk];
+          qs.z = (float)L.z[gk];
+          qs.b = L.gb[gk];
+          qs.m = L.mv[gk];
+          qs.rh = __frcp_rn(qs.h);
+          qs.u = __fmul_rn(__fmul_rn(qs.b, qs.m), qs.rh);
+          if (!perch) { Gh = 0.f; Gbm = 0.f; }
+        } else if (perch && j0 == 0 && row_ok) {  // per-channel state, tile starting mid-row
+          gk = row;
+          qs.h = L.h[gk];
+          qs.z = (float)L.z[gk];
+          qs.b = L.gb[gk];
+          qs.m = L.mv[gk];
+          qs.rh = __frcp_rn(qs.h);
+          qs.u = __fmul_rn(__fmul_rn(qs.b, qs.m), qs.rh);
+        }
+        float cs[32], cd[32];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          float w8[8];
+          unpack_bf16x8(wcur[i], w8);
+          float s8[8];
+          if (L.s) {
+            const float4 a = __ldg(reinterpret_cast<const float4*>(L.s + nb) + 2 * i);
+            const float4 b = __ldg(reinterpret_cast<const float4*>(L.s + nb) + 2 * i + 1);
+            s8[0] = a.x; s8[1] = a.y; s8[2] = a.z; s8[3] = a.w; s8[4] = b.x; s8[5] = b.y; s8[6] = b.z; s8[7] = b.w;
+          } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) s8[e] = 1.f;
+          }
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int k = 8 * i + e;
+            const float wt = __fmul_rn(__fmul_rn(w8[e], s8[e]), rr);
+            int inr;
+            const float dh = omq_ste_dh(wt, qs, L.Q, &inr);
+            Gh = fmaf(g[k], dh, Gh);
+            if (!inr) Gbm += g[k];
+            const float d = inr ? g[k] : 0.f;
+            drm = fmaf(d * w8[e], s8[e], drm);
+            cs[k] = (d * w8[e]) * rr;
+            cd[k] = dbr * w8[e];
+          }
+        }
+        const int64_t prow = (int64_t)(row0 >> 5) * N + nb + lane;
+        if (L.part_s) {
+          const float v = colsum_warp32(cs, lane);
+          L.part_s[prow] = v;
+        }
+        if (L.part_d) {
+          const float v = colsum_warp32(cd, lane);
+          L.part_d[prow] = v;
+        }
+        if (!perch && (nb + 32) % L.group == 0 && row_ok) {   // group complete: dgamma, dbeta
+          const float ga = L.ga[gk], gb = qs.b, M = L.Mv[gk], m = qs.m;
+          const float hr = __fdiv_rn(__fsub_rn(__fmul_rn(ga, M), __fmul_rn(gb, m)), L.Q);
+          const float Ghe = (hr >= L.eps) ? Gh : 0.f;           // floored h: no gradient through h
+          const float GaM = Ghe / L.Q, Gbt = Gbm - Ghe / L.Q;
+          const float dg = GaM * M * ga * (1.f - ga), db = Gbt * m * gb * (1.f - gb);
+          if (L.accumulate) { L.dgl[gk] += dg; L.dbl[gk] += db; } else { L.dgl[gk] = dg; L.dbl[gk] = db; }
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) wcur[i] = wnext[i];
+    }
+    if (perch && quad_ok && row_ok) {
+      const int nt = ti.n0 / BN;
+      L.rowpart[((int64_t)0 * p.M + row) * L.ntn + nt] = Gh;
+      L.rowpart[((int64_t)1 * p.M + row) * L.ntn + nt] = Gbm;
+      L.rowpart[((int64_t)2 * p.M + row) * L.ntn + nt] = drm;
+    }
+    if (has_acc) ++acc_it;
+    if (!ok) break;
+  }
+}
+
 // Persistent kernel: one CTA per SM walks tiles blockIdx.x, blockIdx.x + gridDim.x, ...
 // The shared-memory ring runs continuously across tiles; the accumulator is double-buffered
 // in tensor memory (2 x BN columns) so that the epilogue of one tile overlaps the MMAs of
 // the next.
-template <int BN, int STAGES>
+template <int BN, int STAGES, bool LWC>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const __grid_constant__ CUtensorMap tmC, const GemmParams p) {
@@ -286,6 +438,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       ++acc_it;
       if (!ok) break;
     }
+  } else if (LWC && warp >= 2) {
+    lwc_epilogue<BN>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, lane, total);
   } else if (warp >= 2) {
     // ---------------- epilogue ----------------
     // fp32 output leaves through TMA bulk stores: each warp stages its 32 x 32 block in one of two
@@ -452,13 +606,13 @@ bool make_map_c(CUtensorMap* map, float* ptr, int64_t N, int64_t M, int64_t batc
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, bool LWC = false>
 omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
                       const GemmParams& p) {
   using L = SmemLayout<BN, STAGES>;
   static bool attr_set = false;
   if (!attr_set) {
-    if (cudaFuncSetAttribute(gemm_bf16_kernel<BN, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::TOTAL) !=
+    if (cudaFuncSetAttribute(gemm_bf16_kernel<BN, STAGES, LWC>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::TOTAL) !=
         cudaSuccess)
       return OMQ_ERR_CUDA;
     attr_set = true;
@@ -466,7 +620,7 @@ omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap&
   const int64_t tiles = (int64_t)((p.M + BM - 1) / BM) * ((p.N + BN - 1) / BN) * p.batch;
   const int64_t sms = omq_num_sms();
   const unsigned grid = (unsigned)(tiles < sms ? tiles : sms);
-  gemm_bf16_kernel<BN, STAGES><<<grid, NUM_THREADS, L::TOTAL, st>>>(ta, tb, tc, p);
+  gemm_bf16_kernel<BN, STAGES, LWC><<<grid, NUM_THREADS, L::TOTAL, st>>>(ta, tb, tc, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -526,7 +680,7 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
   OMQ_REQUIRE(!ep.R || (omq_aligned16(ep.R) && ep.ldr % 4 == 0), OMQ_ERR_ALIGN);
   OMQ_REQUIRE(!ep.bias || omq_aligned16(ep.bias), OMQ_ERR_ALIGN);
   // the MN-major extents must cover whole 64-wide boxes inside the tensor (TMA zero-fills the rest)
-  const bool wide = (N % 256 == 0);
+  const bool wide = gemm_n_tile(N) == 256;
   CUtensorMap ta, tb;
   const int bn = wide ? 256 : 128;
   bool ok = A.kmajor ? make_map(&ta, A.ptr, K, M, batch, A.ld, A.bs, BM) : make_map(&ta, A.ptr, M, K, batch, A.ld, A.bs, BK);
@@ -552,6 +706,50 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
     }
   }
   omq_status r = wide ? launch_cfg<256, 4>(st, ta, tb, tc, p) : launch_cfg<128, 6>(st, ta, tb, tc, p);
+  if (e0 && e1) cudaEventRecord(e1, st);
+  return r;
+}
+
+int gemm_n_tile(int64_t N) { return N % 256 == 0 ? 256 : 128; }
+
+omq_status gemm_launch_lwc(cudaStream_t st, int64_t M, int64_t N, int64_t K, const GemmOperand& A,
+                           const GemmOperand& B, const GemmLwcEpi& lw, int32_t* status) {
+  OMQ_REQUIRE(M > 0 && N > 0 && K > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(M < (1ll << 31) && N < (1ll << 31) && K < (1ll << 31), OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(A.ptr && B.ptr && lw.W && lw.h && lw.z && lw.gb && lw.mv, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(omq_aligned16(A.ptr) && omq_aligned16(B.ptr) && omq_aligned16(lw.W), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(A.ld % 8 == 0 && B.ld % 8 == 0 && N % 32 == 0, OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(!lw.s || omq_aligned16(lw.s), OMQ_ERR_ALIGN);
+  const int bn = gemm_n_tile(N);
+  const bool perch = lw.group == N;
+  // a group lies inside one 32-column chunk sequence of one tile; the grouped form carries no LET
+  OMQ_REQUIRE(lw.group > 0 && (perch || (lw.group % 32 == 0 && bn % lw.group == 0)), OMQ_ERR_UNSUPPORTED);
+  OMQ_REQUIRE(perch || (!lw.s && !lw.r && !lw.dBt && !lw.part_s && !lw.part_d), OMQ_ERR_UNSUPPORTED);
+  OMQ_REQUIRE(!perch || (lw.rowpart && lw.ntn == (int)((N + bn - 1) / bn)), OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(perch || (lw.dgl && lw.dbl && lw.ga && lw.Mv), OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(!lw.part_s || lw.s, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(!lw.part_d || lw.dBt, OMQ_ERR_INVALID_ARG);
+  CUtensorMap ta, tb, tc;
+  memset(&tc, 0, sizeof(tc));
+  bool ok = A.kmajor ? make_map(&ta, A.ptr, K, M, 1, A.ld, 0, BM) : make_map(&ta, A.ptr, M, K, 1, A.ld, 0, BK);
+  ok = ok && (B.kmajor ? make_map(&tb, B.ptr, K, N, 1, B.ld, 0, bn) : make_map(&tb, B.ptr, N, K, 1, B.ld, 0, BK));
+  if (!ok) return OMQ_ERR_UNSUPPORTED;
+  GemmParams p;
+  memset(&p, 0, sizeof(p));
+  p.M = (int)M; p.N = (int)N; p.K = (int)K; p.batch = 1;
+  p.a_mn = A.kmajor ? 0 : 1; p.b_mn = B.kmajor ? 0 : 1;
+  p.causal = 0; p.lw = lw; p.status = status;
+  p.n_fast = ((double)M > 1.5 * (double)N) ? 1 : 0;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  if (g_prof.on) {
+    e0 = prof_event();
+    e1 = prof_event();
+    if (e0 && e1) {
+      cudaEventRecord(e0, st);
+      g_prof.flops += gemm_algorithmic_flops(M, N, K, 1, 0);
+    }
+  }
+  omq_status r = bn == 256 ? launch_cfg<256, 4, true>(st, ta, tb, tc, p) : launch_cfg<128, 6, true>(st, ta, tb, tc, p);
   if (e0 && e1) cudaEventRecord(e1, st);
   return r;
 }

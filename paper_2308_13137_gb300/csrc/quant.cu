@@ -528,6 +528,32 @@ omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a0, void* scratch) 
   return OMQ_OK;
 }
 
+omq_status lwc_bwd_fused_finish(cudaStream_t st, const LwcBwdArgs& a0, float* rowpart, int64_t ntn,
+                                const float* part_s, const float* part_d, int64_t nparts) {
+  LwcBwdArgs a = a0;
+  const bool perch = a.group == a.Cin;
+  OMQ_REQUIRE(a.ga && a.gb, OMQ_ERR_INVALID_ARG);
+  // the LET column sums first, so that the finalize can add the max/min routing on top
+  if (a.ds) {
+    OMQ_REQUIRE(part_s, OMQ_ERR_INVALID_ARG);
+    OMQ_TRY(omq_colsum_partials(st, part_s, nparts, a.Cin, a.ds, 1.f, a.accumulate_sd));
+  }
+  if (a.ddelta && a.dBt) {
+    OMQ_REQUIRE(part_d, OMQ_ERR_INVALID_ARG);
+    OMQ_TRY(omq_colsum_partials(st, part_d, nparts, a.Cin, a.ddelta, 1.f, a.accumulate_sd));
+  }
+  if (perch || a.dr) {
+    OMQ_REQUIRE(rowpart, OMQ_ERR_INVALID_ARG);
+    LwcBwdScratch sc{};
+    sc.rowpart = rowpart;
+    sc.ncw = ntn;
+    sc.ng = a.Cin / a.group;
+    lwc_bwd_finalize_kernel<<<(unsigned)((a.Cout + 7) / 8), 256, 0, st>>>(a, sc);
+    OMQ_LAUNCH_CHECK();
+  }
+  return OMQ_OK;
+}
+
 // ================================================================================================
 // reductions, loss, small vector kernels
 // ================================================================================================

@@ -34,6 +34,11 @@ struct LwcBwdArgs {
 // scratch: partial column sums and per-row partials, carved from `scratch`
 size_t lwc_bwd_scratch_bytes(int64_t Cout, int64_t Cin);
 omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a, void* scratch);
+// Completion of the LWC backward whose per-element part ran inside the weight-gradient GEMM
+// epilogue: column partials [nparts, Cin] -> ds, ddelta; per-channel row partials [3, Cout, ntn]
+// -> dgamma, dbeta, max/min routing, dr (a.dWq and a.dWt unused).
+omq_status lwc_bwd_fused_finish(cudaStream_t st, const LwcBwdArgs& a, float* rowpart, int64_t ntn,
+                                const float* part_s, const float* part_d, int64_t nparts);
 
 // ---- per-token activation quantizer Q_a with a fused producer ------------------------------
 enum ActProducer { AP_PLAIN = 0, AP_LET = 1, AP_RMS_LET = 2, AP_SWIGLU = 3 };
