@@ -381,7 +381,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   bm.producer = AP_SWIGLU; bm.X = w.Ygu; bm.ldx = 2 * c.f; bm.U = w.Ygu + c.f; bm.ldu = 2 * c.f; bm.T = c.T; bm.C = c.f;
   bm.h = w.sm.h; bm.z = w.sm.z; bm.imax = w.sm.imax; bm.imin = w.sm.imin; bm.dXq = w.dm; bm.lddq = c.f;
   bm.dX = w.dYgu; bm.lddx = 2 * c.f; bm.dXb = w.dYgu_b; bm.lddxb = 2 * c.f; bm.dU = w.dYgu + c.f; bm.dUb = w.dYgu_b + c.f;
-  bm.rows_per_cta = 4; bm.abits = cfg.abits; bm.eps = cfg.h_eps;
+  bm.rows_per_cta = 1; bm.abits = cfg.abits; bm.eps = cfg.h_eps;
   OMQ_TRY(act_bwd_launch(st, bm));
 
   // ---- gate / up ----------------------------------------------------------------------------------

@@ -193,170 +193,248 @@ __global__ void __launch_bounds__(NT) act_fwd_rows(ActFwdArgs a) {
 }
 
 // ================================================================================================
-// activation quantizer backward: STE of Q_a, then the producer's backward
+// activation quantizer backward: STE of Q_a, then the producer's backward, streamed.
+// The STE gradient of a token is the in-range mask times the incoming gradient everywhere except
+// at the first max / min, which also receive the h-path routing (a row sum).  So one streaming
+// pass writes every output with the masked gradient and accumulates the row sums; after one block
+// reduction the owners of the two routed elements rewrite them.  Only RMSNorm, whose backward
+// needs the row dot product of the final gradient, streams the row a second time (from L2).
+// 256 threads, low register count: several CTAs (rows) per SM hide the load latency.  CTA p
+// handles rows [p * rows_per_cta, ...) and writes LET column partial p.
 // ================================================================================================
-template <int P, int NT, int VPT>
-__global__ void __launch_bounds__(NT) act_bwd_rows(ActBwdArgs a) {
-  constexpr int NE = 4 * VPT;
-  __shared__ float fsm[64];
-  const int tid = threadIdx.x;
-  const int64_t nv = a.C / 4;
-  const bool let_sums = (P != AP_SWIGLU) && a.part_s != nullptr;
-  const bool quant = a.abits < 16;
-  const float Q = (float)((1 << (quant ? a.abits : 1)) - 1);
-  float acc_s[NE], acc_d[NE];
-  int col[NE];
-#pragma unroll
-  for (int k = 0; k < NE; ++k) { acc_s[k] = 0.f; acc_d[k] = 0.f; }
-#pragma unroll
-  for (int j = 0; j < VPT; ++j) {
-    const int64_t vi = (int64_t)j * NT + tid;
-#pragma unroll
-    for (int e = 0; e < 4; ++e) col[4 * j + e] = vi < nv ? (int)(4 * vi + e) : -1;
-  }
-  // X~ of one element exactly as the forward formed it
-  auto xt_of = [&](int64_t t, int64_t i) -> float {
-    const float* xr = a.X + t * a.ldx;
+#define ACT_BWD_NT 256
+
+__device__ __forceinline__ float3 block_sum3(float a, float b, float c, float* smem) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  a = warp_sum(a); b = warp_sum(b); c = warp_sum(c);
+  __syncthreads();
+  if (lane == 0) { smem[wid] = a; smem[32 + wid] = b; smem[64 + wid] = c; }
+  __syncthreads();
+  float x = lane < nw ? smem[lane] : 0.f, y = lane < nw ? smem[32 + lane] : 0.f, z = lane < nw ? smem[64 + lane] : 0.f;
+  return make_float3(warp_sum(x), warp_sum(y), warp_sum(z));
+}
+
+template <int P>
+struct ActBwdRow {
+  const ActBwdArgs& a;
+  int64_t t;
+  float rstd;
+  // X~ of one element from the producer's inputs (exactly as the forward formed it)
+  __device__ __forceinline__ float xt(float x, float u, float dl, float sv) const {
     float v;
-    if (P == AP_SWIGLU) v = silu(xr[i]) * a.U[t * a.ldu + i];
-    else if (P == AP_RMS_LET) v = xr[i] * a.rstd[t];
-    else v = xr[i];
+    if (P == AP_SWIGLU) v = silu(x) * u;
+    else if (P == AP_RMS_LET) v = x * rstd;
+    else v = x;
     if (P == AP_LET || P == AP_RMS_LET) {
-      if (a.delta) v = v - a.delta[i];
-      if (a.s) v = __fdiv_rn(v, a.s[i]);
+      if (a.delta) v = v - dl;
+      if (a.s) v = __fdiv_rn(v, sv);
     }
     return v;
-  };
-  const int64_t t0 = (int64_t)blockIdx.x * a.rows_per_cta;
-  const int64_t t1 = min(a.T, t0 + a.rows_per_cta);
-  for (int64_t t = t0; t < t1; ++t) {
-    const float* xr = a.X + t * a.ldx;
-    const float* gr = a.dXq + t * a.lddq;
-    float val[NE], g[NE], xin[NE];
-    float4 raw[VPT], graw[VPT];
+  }
+  __device__ __forceinline__ float xt_at(int64_t i) const {
+    const float x = a.X[t * a.ldx + i];
+    const float u = (P == AP_SWIGLU) ? a.U[t * a.ldu + i] : 0.f;
+    const float dl = ((P == AP_LET || P == AP_RMS_LET) && a.delta) ? a.delta[i] : 0.f;
+    const float sv = ((P == AP_LET || P == AP_RMS_LET) && a.s) ? a.s[i] : 1.f;
+    return xt(x, u, dl, sv);
+  }
+};
+
+template <int P, int VPT, int JB, int MINB, bool SUMS>
+__global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a) {
+  constexpr int NT = ACT_BWD_NT;
+  constexpr bool LETP = (P == AP_LET || P == AP_RMS_LET);
+  static_assert(!(SUMS && P == AP_SWIGLU), "SwiGLU has no LET column sums");
+  constexpr int NE = SUMS ? 4 * VPT : 1;
+  __shared__ float fsm[96];
+  const int tid = threadIdx.x;
+  const int64_t nv = a.C / 4;
+  constexpr bool let_sums = SUMS;
+  const bool quant = a.abits < 16;
+  const float Q = (float)((1 << (quant ? a.abits : 1)) - 1);
+  const bool want_out = a.dX != nullptr || a.dXb != nullptr;
+  const int64_t nparts = (a.T + a.rows_per_cta - 1) / a.rows_per_cta;
+  const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f), o4 = make_float4(1.f, 1.f, 1.f, 1.f);
+  float acc_s[NE], acc_d[NE];
+  for (int64_t p = blockIdx.x; p < nparts; p += gridDim.x) {
 #pragma unroll
-    for (int j = 0; j < VPT; ++j) {                   // every load of the row first
-      const int64_t vi = (int64_t)j * NT + tid;
-      const bool ok = vi < nv;
-      raw[j] = ok ? ld4(xr + 4 * vi) : make_float4(0.f, 0.f, 0.f, 0.f);
-      graw[j] = ok ? ld4(gr + 4 * vi) : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-    const float rstd = (P == AP_RMS_LET) ? a.rstd[t] : 1.f;
-#pragma unroll
-    for (int j = 0; j < VPT; ++j) {
-      const int64_t vi = (int64_t)j * NT + tid;
-      float4 uu = make_float4(0.f, 0.f, 0.f, 0.f), dl = uu, sv = make_float4(1.f, 1.f, 1.f, 1.f);
-      if (vi < nv) {
-        if (P == AP_SWIGLU) uu = ld4(a.U + t * a.ldu + 4 * vi);
-        if ((P == AP_LET || P == AP_RMS_LET) && a.delta) dl = ld4(a.delta + 4 * vi);
-        if ((P == AP_LET || P == AP_RMS_LET) && a.s) sv = ld4(a.s + 4 * vi);
+    for (int k = 0; k < NE; ++k) { acc_s[k] = 0.f; acc_d[k] = 0.f; }
+    const int64_t t0 = p * a.rows_per_cta, t1 = min(a.T, t0 + a.rows_per_cta);
+    for (int64_t t = t0; t < t1; ++t) {
+      ActBwdRow<P> R{a, t, (P == AP_RMS_LET) ? a.rstd[t] : 1.f};
+      const float* xr = a.X + t * a.ldx;
+      const float* gr = a.dXq + t * a.lddq;
+      const float* ur = (P == AP_SWIGLU) ? a.U + t * a.ldu : nullptr;
+      QState qs;
+      int iM = -1, im = -1;
+      if (quant) {
+        iM = a.imax[t]; im = a.imin[t];
+        qs = omq_qstate(R.xt_at(iM), R.xt_at(im), 1.f, 1.f, Q, a.eps);
+        qs.h = a.h[t]; qs.z = (float)a.z[t]; qs.rh = __frcp_rn(qs.h); qs.u = __fmul_rn(qs.m, qs.rh);
       }
+      float Gh = 0.f, Gbm = 0.f, dot = 0.f;
+      // ---- pass 1: masked gradient through the producer, row sums ----
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int k = 4 * j + e;
-        const float x = f4get(raw[j], e);
-        xin[k] = x;
-        float v;
-        if (P == AP_SWIGLU) v = silu(x) * f4get(uu, e);
-        else if (P == AP_RMS_LET) v = x * rstd;
-        else v = x;
-        if (P == AP_LET || P == AP_RMS_LET) {
-          if (a.delta) v = v - f4get(dl, e);
-          if (a.s) v = __fdiv_rn(v, f4get(sv, e));
+      for (int jb = 0; jb < VPT; jb += JB) {
+        float4 x4[JB], g4[JB], u4[JB];
+#pragma unroll
+        for (int jj = 0; jj < JB; ++jj) {               // every load of the batch first
+          const int64_t vi = (int64_t)(jb + jj) * NT + tid;
+          const bool ok = jb + jj < VPT && vi < nv;
+          x4[jj] = ok ? ld4(xr + 4 * vi) : z4;
+          g4[jj] = ok ? ld4(gr + 4 * vi) : z4;
+          u4[jj] = (P == AP_SWIGLU && ok) ? ld4(ur + 4 * vi) : z4;
         }
-        val[k] = v;
-        g[k] = f4get(graw[j], e);
-      }
-    }
-    // STE of Q_a
-    float d[NE];
-    if (quant) {
-      const int iM = a.imax[t], im = a.imin[t];
-      const float M = xt_of(t, iM), m = xt_of(t, im);
-      QState qs = omq_qstate(M, m, 1.f, 1.f, Q, a.eps);
-      qs.h = a.h[t]; qs.z = (float)a.z[t]; qs.rh = __frcp_rn(qs.h); qs.u = __fmul_rn(m, qs.rh);
-      bool inr[NE];
-      float GaM, Gbt;
-      row_ste<NE>(val, col, g, qs, Q, inr, &GaM, &Gbt, fsm);
 #pragma unroll
-      for (int k = 0; k < NE; ++k) {
-        float dk = inr[k] ? g[k] : 0.f;
-        if (col[k] == iM) dk += GaM;
-        if (col[k] == im) dk += Gbt;
-        d[k] = dk;
-      }
-    } else {
+        for (int jj = 0; jj < JB; ++jj) {
+          const int j = jb + jj;
+          const int64_t vi = (int64_t)j * NT + tid;
+          if (j >= VPT || vi >= nv) continue;
+          float4 dl = z4, sv = o4;
+          if (LETP && a.delta) dl = ld4(a.delta + 4 * vi);
+          if (LETP && a.s) sv = ld4(a.s + 4 * vi);
+          float o1[4], o2[4];
 #pragma unroll
-      for (int k = 0; k < NE; ++k) d[k] = g[k];
-    }
-    // producer backward
-    float dn[NE];
-    float dot = 0.f;
-#pragma unroll
-    for (int j = 0; j < VPT; ++j) {
-      const int64_t vi = (int64_t)j * NT + tid;
-      if (vi >= nv) continue;
-      float sv[4] = {1.f, 1.f, 1.f, 1.f};
-      if ((P == AP_LET || P == AP_RMS_LET) && a.s) {
-        const float4 s4 = ld4(a.s + 4 * vi);
-        sv[0] = s4.x; sv[1] = s4.y; sv[2] = s4.z; sv[3] = s4.w;
-      }
-      float o1[4], o2[4];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int k = 4 * j + e;
-        if (P == AP_SWIGLU) {
-          const float gg = xin[k], uu = a.U[t * a.ldu + 4 * vi + e];
-          const float sg = 1.f / (1.f + expf(-gg));
-          o1[e] = d[k] * uu * sg * (1.f + gg * (1.f - sg));
-          o2[e] = d[k] * gg * sg;
-        } else {
-          if (let_sums) { acc_s[k] -= d[k] * val[k] / sv[e]; acc_d[k] -= d[k] / sv[e]; }
-          const float v = (a.s && (P == AP_LET || P == AP_RMS_LET)) ? __fdiv_rn(d[k], sv[e]) : d[k];
-          if (P == AP_RMS_LET) { dn[k] = v; dot = fmaf(v, xin[k] * rstd, dot); }
-          o1[e] = v;
+          for (int e = 0; e < 4; ++e) {
+            const float x = f4get(x4[jj], e), g = f4get(g4[jj], e), se = f4get(sv, e);
+            const float v = R.xt(x, f4get(u4[jj], e), f4get(dl, e), se);
+            float d = g;
+            if (quant) {
+              int in = 0;
+              const float dh = omq_ste_dh(v, qs, Q, &in);
+              Gh = fmaf(g, dh, Gh);
+              if (!in) { Gbm += g; d = 0.f; }
+            }
+            if (P == AP_SWIGLU) {
+              const float uu = f4get(u4[jj], e);
+              const float sg = 1.f / (1.f + expf(-x));
+              o1[e] = d * uu * sg * (1.f + x * (1.f - sg));
+              o2[e] = d * x * sg;
+            } else {
+              if (SUMS && let_sums) {
+                const int k = 4 * j + e;
+                acc_s[k] -= d * v / se;
+                acc_d[k] -= d / se;
+              }
+              const float dn = (LETP && a.s) ? __fdiv_rn(d, se) : d;
+              if (P == AP_RMS_LET) dot = fmaf(dn, x * R.rstd, dot);
+              o1[e] = dn;
+            }
+          }
+          if (P == AP_SWIGLU) {
+            if (a.dX) {
+              *reinterpret_cast<float4*>(a.dX + t * a.lddx + 4 * vi) = make_float4(o1[0], o1[1], o1[2], o1[3]);
+              *reinterpret_cast<float4*>(a.dU + t * a.lddx + 4 * vi) = make_float4(o2[0], o2[1], o2[2], o2[3]);
+            }
+            if (a.dXb) { st_bf16x4(a.dXb + t * a.lddxb + 4 * vi, o1); st_bf16x4(a.dUb + t * a.lddxb + 4 * vi, o2); }
+          } else if (P == AP_PLAIN || P == AP_LET) {
+            if (a.dX) *reinterpret_cast<float4*>(a.dX + t * a.lddx + 4 * vi) = make_float4(o1[0], o1[1], o1[2], o1[3]);
+            if (a.dXb) st_bf16x4(a.dXb + t * a.lddxb + 4 * vi, o1);
+          }
         }
       }
-      if (P == AP_SWIGLU) {
-        if (a.dX) {
-          *reinterpret_cast<float4*>(a.dX + t * a.lddx + 4 * vi) = make_float4(o1[0], o1[1], o1[2], o1[3]);
-          *reinterpret_cast<float4*>(a.dU + t * a.lddx + 4 * vi) = make_float4(o2[0], o2[1], o2[2], o2[3]);
+      if (!quant && !(P == AP_RMS_LET && want_out)) continue;
+      const float3 tot = block_sum3(Gh, Gbm, dot, fsm);
+      float GaM = 0.f, Gbt = 0.f;
+      if (quant) {
+        const float Gh_t = qs.floored ? 0.f : tot.x;
+        GaM = Gh_t / Q;
+        Gbt = tot.y - Gh_t / Q;
+      }
+      // ---- the routed elements: their owners rewrite them ----
+      float dot_t = tot.z;
+      if (quant) {
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const int64_t c = r == 0 ? iM : im;
+          if (r == 1 && im == iM) break;
+          const float route = (im == iM) ? GaM + Gbt : (r == 0 ? GaM : Gbt);
+          const float x = xr[c], g = gr[c];
+          const float se = (LETP && a.s) ? a.s[c] : 1.f;
+          const float v = R.xt_at(c);
+          int in = 0;
+          omq_ste_dh(v, qs, Q, &in);
+          const float d = (in ? g : 0.f) + route;
+          if (P == AP_RMS_LET) dot_t = fmaf((a.s ? __fdiv_rn(route, se) : route), x * R.rstd, dot_t);
+          if ((c >> 2) % NT != tid) continue;
+          if (P == AP_SWIGLU) {
+            const float uu = ur[c];
+            const float sg = 1.f / (1.f + expf(-x));
+            const float v1 = d * uu * sg * (1.f + x * (1.f - sg)), v2 = d * x * sg;
+            if (a.dX) { a.dX[t * a.lddx + c] = v1; a.dU[t * a.lddx + c] = v2; }
+            if (a.dXb) { a.dXb[t * a.lddxb + c] = f_to_bf16(v1); a.dUb[t * a.lddxb + c] = f_to_bf16(v2); }
+          } else {
+            if (let_sums) {
+#pragma unroll
+              for (int k = 0; k < NE; ++k)
+                if (4 * ((int64_t)(k >> 2) * NT + tid) + (k & 3) == c) {
+                  acc_s[k] -= route * v / se;
+                  acc_d[k] -= route / se;
+                }
+            }
+            if (P == AP_PLAIN || P == AP_LET) {
+              const float dn = (LETP && a.s) ? __fdiv_rn(d, se) : d;
+              if (a.dX) a.dX[t * a.lddx + c] = dn;
+              if (a.dXb) a.dXb[t * a.lddxb + c] = f_to_bf16(dn);
+            }
+          }
         }
-        if (a.dXb) { st_bf16x4(a.dXb + t * a.lddxb + 4 * vi, o1); st_bf16x4(a.dUb + t * a.lddxb + 4 * vi, o2); }
-      } else if (P == AP_PLAIN || P == AP_LET) {
-        if (a.dX) *reinterpret_cast<float4*>(a.dX + t * a.lddx + 4 * vi) = make_float4(o1[0], o1[1], o1[2], o1[3]);
-        if (a.dXb) st_bf16x4(a.dXb + t * a.lddxb + 4 * vi, o1);
+      }
+      // ---- RMSNorm backward: second stream of the row ----
+      if (P == AP_RMS_LET && want_out) {
+        const float mean_dot = dot_t / (float)a.C;
+#pragma unroll
+        for (int jb = 0; jb < VPT; jb += JB) {
+          float4 x4[JB], g4[JB], r4[JB];
+#pragma unroll
+          for (int jj = 0; jj < JB; ++jj) {
+            const int64_t vi = (int64_t)(jb + jj) * NT + tid;
+            const bool ok = jb + jj < VPT && vi < nv;
+            x4[jj] = ok ? ld4(xr + 4 * vi) : z4;
+            g4[jj] = ok ? ld4(gr + 4 * vi) : z4;
+            r4[jj] = (ok && a.resid) ? ld4(a.resid + t * a.lddx + 4 * vi) : z4;
+          }
+#pragma unroll
+          for (int jj = 0; jj < JB; ++jj) {
+            const int j = jb + jj;
+            const int64_t vi = (int64_t)j * NT + tid;
+            if (j >= VPT || vi >= nv) continue;
+            float4 dl = z4, sv = o4;
+            if (a.delta) dl = ld4(a.delta + 4 * vi);
+            if (a.s) sv = ld4(a.s + 4 * vi);
+            float o[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const int64_t c = 4 * vi + e;
+              const float x = f4get(x4[jj], e), g = f4get(g4[jj], e), se = f4get(sv, e);
+              float d = g;
+              if (quant) {
+                const float v = R.xt(x, 0.f, f4get(dl, e), se);
+                int in = 0;
+                omq_ste_dh(v, qs, Q, &in);
+                d = in ? g : 0.f;
+                if (c == iM) d += GaM;
+                if (c == im) d += Gbt;
+              }
+              const float dn = a.s ? __fdiv_rn(d, se) : d;
+              o[e] = R.rstd * (dn - x * R.rstd * mean_dot) + f4get(r4[jj], e);
+            }
+            if (a.dX) *reinterpret_cast<float4*>(a.dX + t * a.lddx + 4 * vi) = make_float4(o[0], o[1], o[2], o[3]);
+            if (a.dXb) st_bf16x4(a.dXb + t * a.lddxb + 4 * vi, o);
+          }
+        }
       }
     }
-    if (P == AP_RMS_LET && (a.dX || a.dXb)) {        // RMSNorm backward
-      const float2 tot = block_sum2(dot, 0.f, fsm);
-      const float mean_dot = tot.x / (float)a.C;
+    if (let_sums) {
 #pragma unroll
       for (int j = 0; j < VPT; ++j) {
         const int64_t vi = (int64_t)j * NT + tid;
-        if (vi >= nv) continue;
-        float4 rs = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (a.resid) rs = ld4(a.resid + t * a.lddx + 4 * vi);
-        float o[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int k = 4 * j + e;
-          o[e] = rstd * (dn[k] - xin[k] * rstd * mean_dot) + f4get(rs, e);
+        if (vi < nv) {
+          float* ps = a.part_s + p * a.C + 4 * vi;
+          float* pd = a.part_d + p * a.C + 4 * vi;
+          *reinterpret_cast<float4*>(ps) = make_float4(acc_s[4 * j], acc_s[4 * j + 1], acc_s[4 * j + 2], acc_s[4 * j + 3]);
+          *reinterpret_cast<float4*>(pd) = make_float4(acc_d[4 * j], acc_d[4 * j + 1], acc_d[4 * j + 2], acc_d[4 * j + 3]);
         }
-        if (a.dX) *reinterpret_cast<float4*>(a.dX + t * a.lddx + 4 * vi) = make_float4(o[0], o[1], o[2], o[3]);
-        if (a.dXb) st_bf16x4(a.dXb + t * a.lddxb + 4 * vi, o);
-      }
-    }
-  }
-  if (let_sums) {
-#pragma unroll
-    for (int j = 0; j < VPT; ++j) {
-      const int64_t vi = (int64_t)j * NT + tid;
-      if (vi < nv) {
-        float* ps = a.part_s + (int64_t)blockIdx.x * a.C + 4 * vi;
-        float* pd = a.part_d + (int64_t)blockIdx.x * a.C + 4 * vi;
-        *reinterpret_cast<float4*>(ps) = make_float4(acc_s[4 * j], acc_s[4 * j + 1], acc_s[4 * j + 2], acc_s[4 * j + 3]);
-        *reinterpret_cast<float4*>(pd) = make_float4(acc_d[4 * j], acc_d[4 * j + 1], acc_d[4 * j + 2], acc_d[4 * j + 3]);
       }
     }
   }
@@ -380,12 +458,34 @@ static omq_status act_fwd_dispatch(cudaStream_t st, const ActFwdArgs& a) {
   return OMQ_OK;
 }
 
-template <int PRODUCER>
-static omq_status act_bwd_dispatch(cudaStream_t st, const ActBwdArgs& a) {
-  const unsigned grid = (unsigned)((a.T + a.rows_per_cta - 1) / a.rows_per_cta);
-  ACT_DISPATCH(act_bwd_rows, a, grid, a.C);
+template <int PRODUCER, int VPT, int JB, int MINB, bool SUMS>
+static omq_status act_bwd_go(cudaStream_t st, const ActBwdArgs& a) {
+  const int64_t nparts = (a.T + a.rows_per_cta - 1) / a.rows_per_cta;
+  act_bwd_stream<PRODUCER, VPT, JB, MINB, SUMS><<<(unsigned)nparts, ACT_BWD_NT, 0, st>>>(a);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
+}
+
+// Row length -> vectors per thread.  Without LET column sums any length up to 28 K streams in
+// batches of four vectors; the column sums keep 8 VPT accumulators per thread in registers.
+template <int PRODUCER>
+static omq_status act_bwd_dispatch(cudaStream_t st, const ActBwdArgs& a) {
+  const int64_t vpt = (a.C / 4 + ACT_BWD_NT - 1) / ACT_BWD_NT;
+  const bool sums = PRODUCER != AP_SWIGLU && a.part_s != nullptr;
+  if (!sums) {
+    if (vpt <= 4) return act_bwd_go<PRODUCER, 4, 4, 4, false>(st, a);
+    if (vpt <= 8) return act_bwd_go<PRODUCER, 8, 4, 4, false>(st, a);
+    if (vpt <= 12) return act_bwd_go<PRODUCER, 12, 4, 4, false>(st, a);
+    if (vpt <= 16) return act_bwd_go<PRODUCER, 16, 4, 4, false>(st, a);
+    if (vpt <= 28) return act_bwd_go<PRODUCER, 28, 4, 4, false>(st, a);
+    return OMQ_ERR_UNSUPPORTED;
+  }
+  if constexpr (PRODUCER != AP_SWIGLU) {
+    if (vpt <= 4) return act_bwd_go<PRODUCER, 4, 1, 3, true>(st, a);
+    if (vpt <= 8) return act_bwd_go<PRODUCER, 8, 1, 2, true>(st, a);
+    if (vpt <= 16) return act_bwd_go<PRODUCER, 16, 1, 1, true>(st, a);
+  }
+  return OMQ_ERR_UNSUPPORTED;
 }
 
 omq_status act_fwd_launch(cudaStream_t st, const ActFwdArgs& a) {
