@@ -608,117 +608,180 @@ __global__ void __launch_bounds__(NT) qkv_fwd_rows(QkvArgs a) {
   }
 }
 
-template <int NT, int PPT>
-__global__ void __launch_bounds__(NT) qkv_bwd_rows(QkvArgs a) {
+// Backward of the q, k, v chain, streamed like the activation quantizer backward: one pass writes
+// the gradient with the in-range mask applied and accumulates the h-path row sums; after the
+// block reduction the owner of each routed pair (the first max / min and its RoPE partner)
+// recomputes that pair with the routing added and rewrites it.
+#define QKV_BWD_NT 256
+
+template <int PPT, int MINB>
+__global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
+  constexpr int NT = QKV_BWD_NT;
   constexpr int NE = 8 * PPT;
-  __shared__ float fsm[64];
+  __shared__ float fsm[96];
+  const int tid = threadIdx.x;
   const int dq = a.H * a.hd, dkv = a.Hkv * a.hd;
   const bool sums = a.part_q != nullptr;
+  const bool quant = a.abits < 16;
+  const float Q = (float)((1 << (quant ? a.abits : 1)) - 1);
+  const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
   float acc_q[NE], acc_k[NE];
 #pragma unroll
   for (int k = 0; k < NE; ++k) { acc_q[k] = 0.f; acc_k[k] = 0.f; }
-  int colq[NE], colk[NE];
   const int t0 = blockIdx.x * a.rows_per_cta, t1 = min(a.T, t0 + a.rows_per_cta);
   for (int t = t0; t < t1; ++t) {
     for (int seg = 0; seg < 3; ++seg) {
-      QkvRow<PPT> r;
-      qkv_load<NT, PPT>(a, seg, t, r);
+      const int Hs = seg == 0 ? a.H : a.Hkv;
+      const int np = Hs * 16;
       const int off = seg == 0 ? 0 : (seg == 1 ? dq : dq + dkv);
+      const float* base = a.Y + (int64_t)t * a.ldy + off;
       const float* gsrc = a.dQKV + (int64_t)t * a.ldd + off;
-      float g[NE], d[NE];
-#pragma unroll
-      for (int j = 0; j < PPT; ++j) {
-        const bool ok = r.col[8 * j] >= 0;
-        const float4 g1 = ok ? ld4(gsrc + r.col[8 * j]) : make_float4(0.f, 0.f, 0.f, 0.f);
-        const float4 g2 = ok ? ld4(gsrc + r.col[8 * j + 4]) : make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) { g[8 * j + e] = f4get(g1, e); g[8 * j + 4 + e] = f4get(g2, e); }
-      }
-      if (a.abits < 16) {
-        const int64_t k = (int64_t)seg * a.T + t;
-        const int iM = a.imax[k], im = a.imin[k];
-        const float Q = (float)((1 << a.abits) - 1);
-        // the saved max / min of X~: recompute those two elements exactly as the forward did
-        auto xt_at = [&](int i) -> float {
-          const float* base = a.Y + (int64_t)t * a.ldy + off;
-          if (seg == 2) return base[i];
-          const int jj = (i % 128) % 64, first = (i % 128) < 64;
-          const float cv = a.cs[((int64_t)t * 64 + jj) * 2], sv = a.cs[((int64_t)t * 64 + jj) * 2 + 1];
-          const float v = first ? base[i] * cv - base[i + 64] * sv : base[i] * cv + base[i - 64] * sv;
-          if (!a.sa_exp) return v;
-          return seg == 0 ? __fdiv_rn(v, a.sa_exp[i]) : __fmul_rn(v, a.sa[i]);
-        };
-        const float M = xt_at(iM), m = xt_at(im);
-        QState qs = omq_qstate(M, m, 1.f, 1.f, Q, a.eps);
-        qs.h = a.h[k]; qs.z = (float)a.z[k]; qs.rh = __frcp_rn(qs.h); qs.u = __fmul_rn(m, qs.rh);
-        bool inr[NE];
-        float GaM, Gbt;
-        row_ste<NE>(r.xt, r.col, g, qs, Q, inr, &GaM, &Gbt, fsm);
-#pragma unroll
-        for (int kk = 0; kk < NE; ++kk) {
-          float dk = inr[kk] ? g[kk] : 0.f;
-          if (r.col[kk] == iM) dk += GaM;
-          if (r.col[kk] == im) dk += Gbt;
-          d[kk] = dk;
-        }
-      } else {
-#pragma unroll
-        for (int kk = 0; kk < NE; ++kk) d[kk] = g[kk];
-      }
-      // [Q, K] LET backward and the s_a partial sums
-      if (seg < 2 && a.sa_exp) {
-#pragma unroll
-        for (int kk = 0; kk < NE; ++kk) {
-          if (r.col[kk] < 0) continue;
-          if (seg == 0) {
-            const float sa = a.sa_exp[r.col[kk]];
-            if (sums) acc_q[kk] -= d[kk] * r.xt[kk] / sa;
-            d[kk] = __fdiv_rn(d[kk], sa);
-          } else {
-            const float sa = a.sa[r.col[kk]];
-            if (sums) acc_k[kk] += d[kk] * r.rot[kk];
-            d[kk] = __fmul_rn(d[kk], sa);
-          }
-        }
-      }
-      if (seg == 0) {
-#pragma unroll
-        for (int kk = 0; kk < NE; ++kk) colq[kk] = r.col[kk];
-      } else if (seg == 1) {
-#pragma unroll
-        for (int kk = 0; kk < NE; ++kk) colk[kk] = r.col[kk];
-      }
-      // RoPE backward: the transpose of the rotation, pair-local
-      float o[NE];
-#pragma unroll
-      for (int j = 0; j < PPT; ++j)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int k1 = 8 * j + e, k2 = 8 * j + 4 + e;
-          if (seg == 2) { o[k1] = d[k1]; o[k2] = d[k2]; }
-          else {
-            o[k1] = d[k1] * r.c[k1] + d[k2] * r.sn[k1];
-            o[k2] = d[k2] * r.c[k1] - d[k1] * r.sn[k1];
-          }
-        }
       float* dy = a.dY + (int64_t)t * a.ldy + off;
       __nv_bfloat16* dyb = a.dYb + (int64_t)t * a.ldy + off;
+      const float* csr = a.cs + (int64_t)t * 128;
+      const bool rope = seg < 2, let = seg < 2 && a.sa_exp != nullptr;
+      // X~ of one element (the forward's exact operation order)
+      auto xt_of = [&](float v, int i) -> float {
+        if (!let) return v;
+        return seg == 0 ? __fdiv_rn(v, a.sa_exp[i]) : __fmul_rn(v, a.sa[i]);
+      };
+      QState qs;
+      int iM = -1, im = -1;
+      const int64_t kq = (int64_t)seg * a.T + t;
+      if (quant) {
+        iM = a.imax[kq]; im = a.imin[kq];
+        auto xt_at = [&](int i) -> float {
+          if (!rope) return base[i];
+          const int jj = (i % 128) % 64, first = (i % 128) < 64;
+          const float cv = csr[2 * jj], sv = csr[2 * jj + 1];
+          const float v = first ? base[i] * cv - base[i + 64] * sv : base[i] * cv + base[i - 64] * sv;
+          return xt_of(v, i);
+        };
+        const float m = xt_at(im);
+        qs = omq_qstate(xt_at(iM), m, 1.f, 1.f, Q, a.eps);
+        qs.h = a.h[kq]; qs.z = (float)a.z[kq]; qs.rh = __frcp_rn(qs.h); qs.u = __fmul_rn(m, qs.rh);
+      }
+      float Gh = 0.f, Gbm = 0.f;
+      // ---- pass 1 ----
 #pragma unroll
       for (int j = 0; j < PPT; ++j) {
-        if (r.col[8 * j] < 0) continue;
-        const int e1 = r.col[8 * j], e2 = r.col[8 * j + 4];
-        *reinterpret_cast<float4*>(dy + e1) = make_float4(o[8 * j], o[8 * j + 1], o[8 * j + 2], o[8 * j + 3]);
-        *reinterpret_cast<float4*>(dy + e2) = make_float4(o[8 * j + 4], o[8 * j + 5], o[8 * j + 6], o[8 * j + 7]);
-        st_bf16x4(dyb + e1, &o[8 * j]);
-        st_bf16x4(dyb + e2, &o[8 * j + 4]);
+        const int p = j * NT + tid;
+        if (p >= np) continue;
+        const int e1 = (p >> 4) * 128 + 4 * (p & 15);
+        float4 x1[1], x2[1], g1[1], g2[1], ca[1], cb[1];
+        x1[0] = ld4(base + e1);
+        x2[0] = ld4(base + e1 + 64);
+        g1[0] = ld4(gsrc + e1);
+        g2[0] = ld4(gsrc + e1 + 64);
+        ca[0] = rope ? ld4(csr + 8 * (p & 15)) : z4;
+        cb[0] = rope ? ld4(csr + 8 * (p & 15) + 4) : z4;
+        const float cv[4] = {ca[0].x, ca[0].z, cb[0].x, cb[0].z};
+        const float sv[4] = {ca[0].y, ca[0].w, cb[0].y, cb[0].w};
+        float o1[4], o2[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float a1 = f4get(x1[0], e), a2 = f4get(x2[0], e);
+          const float r1 = rope ? a1 * cv[e] - a2 * sv[e] : a1;
+          const float r2 = rope ? a2 * cv[e] + a1 * sv[e] : a2;
+          const float v1 = xt_of(r1, e1 + e), v2 = xt_of(r2, e1 + 64 + e);
+          float d1 = f4get(g1[0], e), d2 = f4get(g2[0], e);
+          if (quant) {
+            int in1 = 0, in2 = 0;
+            const float h1 = omq_ste_dh(v1, qs, Q, &in1), h2 = omq_ste_dh(v2, qs, Q, &in2);
+            Gh = fmaf(d1, h1, Gh);
+            Gh = fmaf(d2, h2, Gh);
+            if (!in1) { Gbm += d1; d1 = 0.f; }
+            if (!in2) { Gbm += d2; d2 = 0.f; }
+          }
+          if (let) {
+            const int k1 = 8 * j + e, k2 = 8 * j + 4 + e;
+            if (seg == 0) {
+              const float s1 = a.sa_exp[e1 + e], s2 = a.sa_exp[e1 + 64 + e];
+              if (sums) { acc_q[k1] -= d1 * v1 / s1; acc_q[k2] -= d2 * v2 / s2; }
+              d1 = __fdiv_rn(d1, s1); d2 = __fdiv_rn(d2, s2);
+            } else {
+              if (sums) { acc_k[k1] += d1 * r1; acc_k[k2] += d2 * r2; }
+              d1 = __fmul_rn(d1, a.sa[e1 + e]); d2 = __fmul_rn(d2, a.sa[e1 + 64 + e]);
+            }
+          }
+          o1[e] = rope ? d1 * cv[e] + d2 * sv[e] : d1;
+          o2[e] = rope ? d2 * cv[e] - d1 * sv[e] : d2;
+        }
+        *reinterpret_cast<float4*>(dy + e1) = make_float4(o1[0], o1[1], o1[2], o1[3]);
+        *reinterpret_cast<float4*>(dy + e1 + 64) = make_float4(o2[0], o2[1], o2[2], o2[3]);
+        st_bf16x4(dyb + e1, o1);
+        st_bf16x4(dyb + e1 + 64, o2);
+      }
+      if (!quant) continue;
+      const float3 tot = block_sum3(Gh, Gbm, 0.f, fsm);
+      const float Gh_t = qs.floored ? 0.f : tot.x;
+      const float GaM = Gh_t / Q, Gbt = tot.y - Gh_t / Q;
+      // ---- the routed pairs: recomputed with the routing by their owners ----
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        const int c = r == 0 ? iM : im;
+        const int first = (c & ~127) + (c & 63);           // element of the pair in the first half
+        if (r == 1 && ((iM & ~127) + (iM & 63)) == first) break;   // same pair: already done
+        const int pp = (first >> 7) * 16 + ((first & 63) >> 2);
+        if (pp % NT != tid) continue;
+        const int j = pp / NT;
+        const int e = first & 3;
+        const int jj = first & 63;
+        const float cv = rope ? csr[2 * jj] : 1.f, sv = rope ? csr[2 * jj + 1] : 0.f;
+        const float a1 = base[first], a2 = base[first + 64];
+        const float r1 = rope ? a1 * cv - a2 * sv : a1;
+        const float r2 = rope ? a2 * cv + a1 * sv : a2;
+        const float v1 = xt_of(r1, first), v2 = xt_of(r2, first + 64);
+        const float g1s = gsrc[first], g2s = gsrc[first + 64];
+        int in1 = 0, in2 = 0;
+        omq_ste_dh(v1, qs, Q, &in1);
+        omq_ste_dh(v2, qs, Q, &in2);
+        float ro1 = 0.f, ro2 = 0.f;                        // routing of each element of the pair
+        if (first == iM) ro1 += GaM;
+        if (first == im) ro1 += Gbt;
+        if (first + 64 == iM) ro2 += GaM;
+        if (first + 64 == im) ro2 += Gbt;
+        float d1 = (in1 ? g1s : 0.f) + ro1, d2 = (in2 ? g2s : 0.f) + ro2;
+        if (let) {
+#pragma unroll
+          for (int jx = 0; jx < PPT; ++jx)
+#pragma unroll
+            for (int ex = 0; ex < 4; ++ex) {
+              if (jx != j || ex != e) continue;
+              const int k1 = 8 * jx + ex, k2 = 8 * jx + 4 + ex;
+              if (seg == 0) {
+                const float s1 = a.sa_exp[first], s2 = a.sa_exp[first + 64];
+                if (sums) { acc_q[k1] -= ro1 * v1 / s1; acc_q[k2] -= ro2 * v2 / s2; }
+              } else {
+                if (sums) { acc_k[k1] += ro1 * r1; acc_k[k2] += ro2 * r2; }
+              }
+            }
+          if (seg == 0) { d1 = __fdiv_rn(d1, a.sa_exp[first]); d2 = __fdiv_rn(d2, a.sa_exp[first + 64]); }
+          else { d1 = __fmul_rn(d1, a.sa[first]); d2 = __fmul_rn(d2, a.sa[first + 64]); }
+        }
+        const float o1 = rope ? d1 * cv + d2 * sv : d1;
+        const float o2 = rope ? d2 * cv - d1 * sv : d2;
+        dy[first] = o1; dy[first + 64] = o2;
+        dyb[first] = f_to_bf16(o1); dyb[first + 64] = f_to_bf16(o2);
       }
     }
   }
   if (sums) {
 #pragma unroll
-    for (int kk = 0; kk < NE; ++kk) {
-      if (colq[kk] >= 0) a.part_q[(int64_t)blockIdx.x * dq + colq[kk]] = acc_q[kk];
-      if (colk[kk] >= 0) a.part_k[(int64_t)blockIdx.x * dkv + colk[kk]] = acc_k[kk];
+    for (int j = 0; j < PPT; ++j) {
+      const int p = j * NT + tid;
+      const int e1 = (p >> 4) * 128 + 4 * (p & 15);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if (p < a.H * 16) {
+          a.part_q[(int64_t)blockIdx.x * dq + e1 + e] = acc_q[8 * j + e];
+          a.part_q[(int64_t)blockIdx.x * dq + e1 + 64 + e] = acc_q[8 * j + 4 + e];
+        }
+        if (p < a.Hkv * 16) {
+          a.part_k[(int64_t)blockIdx.x * dkv + e1 + e] = acc_k[8 * j + e];
+          a.part_k[(int64_t)blockIdx.x * dkv + e1 + 64 + e] = acc_k[8 * j + 4 + e];
+        }
+      }
     }
   }
 }
@@ -742,9 +805,10 @@ omq_status qkv_bwd_launch(cudaStream_t st, const QkvArgs& a0, int64_t* nslab) {
   a.rows_per_cta = 4;
   const unsigned grid = (unsigned)qkv_bwd_nslab(a.T);
   const int np = a.H * 16;
-  if (np <= 512) qkv_bwd_rows<512, 1><<<grid, 512, 0, st>>>(a);
-  else if (np <= 1024) qkv_bwd_rows<512, 2><<<grid, 512, 0, st>>>(a);
-  else if (np <= 2048) qkv_bwd_rows<512, 4><<<grid, 512, 0, st>>>(a);
+  if (np <= 256) qkv_bwd_stream<1, 4><<<grid, QKV_BWD_NT, 0, st>>>(a);
+  else if (np <= 512) qkv_bwd_stream<2, 3><<<grid, QKV_BWD_NT, 0, st>>>(a);
+  else if (np <= 1024) qkv_bwd_stream<4, 2><<<grid, QKV_BWD_NT, 0, st>>>(a);
+  else if (np <= 2048) qkv_bwd_stream<8, 1><<<grid, QKV_BWD_NT, 0, st>>>(a);
   else return OMQ_ERR_UNSUPPORTED;
   OMQ_LAUNCH_CHECK();
   if (nslab) *nslab = qkv_bwd_nslab(a.T);
