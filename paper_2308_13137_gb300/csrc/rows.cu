@@ -311,10 +311,10 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
               o1[e] = d * uu * sg * (1.f + x * (1.f - sg));
               o2[e] = d * x * sg;
             } else {
-              if (SUMS && let_sums) {
+              if (SUMS && let_sums) {            // divided by s once, when the partial is written
                 const int k = 4 * j + e;
-                acc_s[k] -= d * v / se;
-                acc_d[k] -= d / se;
+                acc_s[k] = fmaf(d, v, acc_s[k]);
+                acc_d[k] += d;
               }
               const float dn = (LETP && a.s) ? __fdiv_rn(d, se) : d;
               if (P == AP_RMS_LET) dot = fmaf(dn, x * R.rstd, dot);
@@ -368,8 +368,8 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
 #pragma unroll
               for (int k = 0; k < NE; ++k)
                 if (4 * ((int64_t)(k >> 2) * NT + tid) + (k & 3) == c) {
-                  acc_s[k] -= route * v / se;
-                  acc_d[k] -= route / se;
+                  acc_s[k] = fmaf(route, v, acc_s[k]);
+                  acc_d[k] += route;
                 }
             }
             if (P == AP_PLAIN || P == AP_LET) {
@@ -425,15 +425,22 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
         }
       }
     }
-    if (let_sums) {
+    if (let_sums) {                              // ds partial -sum(d X~) / s, ddelta partial -sum(d) / s
 #pragma unroll
       for (int j = 0; j < VPT; ++j) {
         const int64_t vi = (int64_t)j * NT + tid;
         if (vi < nv) {
+          const float4 sv = (LETP && a.s) ? ld4(a.s + 4 * vi) : o4;
           float* ps = a.part_s + p * a.C + 4 * vi;
           float* pd = a.part_d + p * a.C + 4 * vi;
-          *reinterpret_cast<float4*>(ps) = make_float4(acc_s[4 * j], acc_s[4 * j + 1], acc_s[4 * j + 2], acc_s[4 * j + 3]);
-          *reinterpret_cast<float4*>(pd) = make_float4(acc_d[4 * j], acc_d[4 * j + 1], acc_d[4 * j + 2], acc_d[4 * j + 3]);
+          float os[4], od[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            os[e] = -acc_s[4 * j + e] / f4get(sv, e);
+            od[e] = -acc_d[4 * j + e] / f4get(sv, e);
+          }
+          *reinterpret_cast<float4*>(ps) = make_float4(os[0], os[1], os[2], os[3]);
+          *reinterpret_cast<float4*>(pd) = make_float4(od[0], od[1], od[2], od[3]);
         }
       }
     }
@@ -481,9 +488,9 @@ static omq_status act_bwd_dispatch(cudaStream_t st, const ActBwdArgs& a) {
     return OMQ_ERR_UNSUPPORTED;
   }
   if constexpr (PRODUCER != AP_SWIGLU) {
-    if (vpt <= 4) return act_bwd_go<PRODUCER, 4, 1, 3, true>(st, a);
-    if (vpt <= 8) return act_bwd_go<PRODUCER, 8, 1, 2, true>(st, a);
-    if (vpt <= 16) return act_bwd_go<PRODUCER, 16, 1, 1, true>(st, a);
+    if (vpt <= 4) return act_bwd_go<PRODUCER, 4, 4, 2, true>(st, a);
+    if (vpt <= 8) return act_bwd_go<PRODUCER, 8, 4, 1, true>(st, a);
+    if (vpt <= 16) return act_bwd_go<PRODUCER, 16, 4, 1, true>(st, a);
   }
   return OMQ_ERR_UNSUPPORTED;
 }
@@ -663,28 +670,34 @@ __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
       }
       float Gh = 0.f, Gbm = 0.f;
       // ---- pass 1 ----
+      float4 x1[PPT], x2[PPT], g1[PPT], g2[PPT], ca[PPT], cb[PPT];
+#pragma unroll
+      for (int j = 0; j < PPT; ++j) {                   // every load of the segment first
+        const int p = j * NT + tid;
+        const bool ok = p < np;
+        const int e1 = (p >> 4) * 128 + 4 * (p & 15);
+        x1[j] = ok ? ld4(base + e1) : z4;
+        x2[j] = ok ? ld4(base + e1 + 64) : z4;
+        g1[j] = ok ? ld4(gsrc + e1) : z4;
+        g2[j] = ok ? ld4(gsrc + e1 + 64) : z4;
+        ca[j] = (ok && rope) ? ld4(csr + 8 * (p & 15)) : z4;
+        cb[j] = (ok && rope) ? ld4(csr + 8 * (p & 15) + 4) : z4;
+      }
 #pragma unroll
       for (int j = 0; j < PPT; ++j) {
         const int p = j * NT + tid;
         if (p >= np) continue;
         const int e1 = (p >> 4) * 128 + 4 * (p & 15);
-        float4 x1[1], x2[1], g1[1], g2[1], ca[1], cb[1];
-        x1[0] = ld4(base + e1);
-        x2[0] = ld4(base + e1 + 64);
-        g1[0] = ld4(gsrc + e1);
-        g2[0] = ld4(gsrc + e1 + 64);
-        ca[0] = rope ? ld4(csr + 8 * (p & 15)) : z4;
-        cb[0] = rope ? ld4(csr + 8 * (p & 15) + 4) : z4;
-        const float cv[4] = {ca[0].x, ca[0].z, cb[0].x, cb[0].z};
-        const float sv[4] = {ca[0].y, ca[0].w, cb[0].y, cb[0].w};
+        const float cv[4] = {ca[j].x, ca[j].z, cb[j].x, cb[j].z};
+        const float sv[4] = {ca[j].y, ca[j].w, cb[j].y, cb[j].w};
         float o1[4], o2[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          const float a1 = f4get(x1[0], e), a2 = f4get(x2[0], e);
+          const float a1 = f4get(x1[j], e), a2 = f4get(x2[j], e);
           const float r1 = rope ? a1 * cv[e] - a2 * sv[e] : a1;
           const float r2 = rope ? a2 * cv[e] + a1 * sv[e] : a2;
           const float v1 = xt_of(r1, e1 + e), v2 = xt_of(r2, e1 + 64 + e);
-          float d1 = f4get(g1[0], e), d2 = f4get(g2[0], e);
+          float d1 = f4get(g1[j], e), d2 = f4get(g2[j], e);
           if (quant) {
             int in1 = 0, in2 = 0;
             const float h1 = omq_ste_dh(v1, qs, Q, &in1), h2 = omq_ste_dh(v2, qs, Q, &in2);
@@ -806,8 +819,8 @@ omq_status qkv_bwd_launch(cudaStream_t st, const QkvArgs& a0, int64_t* nslab) {
   const unsigned grid = (unsigned)qkv_bwd_nslab(a.T);
   const int np = a.H * 16;
   if (np <= 256) qkv_bwd_stream<1, 4><<<grid, QKV_BWD_NT, 0, st>>>(a);
-  else if (np <= 512) qkv_bwd_stream<2, 3><<<grid, QKV_BWD_NT, 0, st>>>(a);
-  else if (np <= 1024) qkv_bwd_stream<4, 2><<<grid, QKV_BWD_NT, 0, st>>>(a);
+  else if (np <= 512) qkv_bwd_stream<2, 2><<<grid, QKV_BWD_NT, 0, st>>>(a);
+  else if (np <= 1024) qkv_bwd_stream<4, 1><<<grid, QKV_BWD_NT, 0, st>>>(a);
   else if (np <= 2048) qkv_bwd_stream<8, 1><<<grid, QKV_BWD_NT, 0, st>>>(a);
   else return OMQ_ERR_UNSUPPORTED;
   OMQ_LAUNCH_CHECK();
