@@ -257,6 +257,29 @@ omq_status omq_block_step(omq_stream_t stream, const omq_block_shape* shape,
                           const omq_block_params* grads, void* workspace, size_t ws_bytes,
                           const omq_qcfg* cfg);
 
+/* Causal self-attention of the block (Sec. 3.3, Eq. 5 applies LET to Q and K before it; the
+ * softmax output is not quantized), computed without storing the [T, T] scores.
+ *   Q  [T, n_heads*128] bf16, row stride ldq; K, V [T, n_kv*128] bf16, row stride ldkv
+ *      (query head h attends with kv head h / (n_heads / n_kv));
+ *   O  [T, n_heads*128] fp32 out, row stride ldo: O = softmax(Q K^T / sqrt(128), causal) V;
+ *   lse [n_heads, T] fp32 out: per row, log2 of sum_j exp2(c s_j - m) plus m, where
+ *      c = log2(e)/sqrt(128) and s_j = q . k_j (the saved state the backward needs).
+ * Head dimension 128 only (OMQ_ERR_SHAPE otherwise).  Strides in elements, multiples of 8 (bf16)
+ * or 4 (fp32), base pointers 16-byte aligned (OMQ_ERR_ALIGN).  Device pointers, caller-owned;
+ * enqueued on `stream`; a stalled pipeline writes OMQ_ERR_TIMEOUT to *dev_status (nullable). */
+omq_status omq_attention_fwd(omq_stream_t stream, int32_t T, int32_t n_heads, int32_t n_kv, const void* Q,
+                             int64_t ldq, const void* K, const void* V, int64_t ldkv, float* O, int64_t ldo,
+                             float* lse, int32_t* dev_status);
+
+/* Backward of omq_attention_fwd given dO [T, n_heads*128] bf16 (row stride lddo), the forward's
+ * O and lse: dQ [T, n_heads*128] (row stride ldg), dK and dV [T, n_kv*128] (row stride ldgkv),
+ * fp32, overwritten.  D [n_heads, T] fp32 is caller scratch (rowsum of dO * O).  The scores and
+ * probabilities are recomputed from Q, K and lse. */
+omq_status omq_attention_bwd(omq_stream_t stream, int32_t T, int32_t n_heads, int32_t n_kv, const void* Q,
+                             int64_t ldq, const void* K, const void* V, int64_t ldkv, const float* O, int64_t ldo,
+                             const float* lse, const void* dO, int64_t lddo, float* D, float* dQ, int64_t ldg,
+                             float* dK, float* dV, int64_t ldgkv, int32_t* dev_status);
+
 /* AdamW update of one fp32 parameter vector (Sec. 4.1 "Training": AdamW, weight decay 0):
  * m = b1 m + (1-b1) g; v = b2 v + (1-b2) g^2; p -= lr * (m / (1-b1^t)) / (sqrt(v / (1-b2^t)) + eps)
  * - lr * wd * p.  step t >= 1. */

@@ -76,6 +76,9 @@ _SIGS = {
     "omq_block_workspace_size": (SZ, [P, P]),
     "omq_block_forward": (I32, [P, P, P, P, P, P, P, SZ, P]),
     "omq_block_step": (I32, [P, P, P, P, P, P, P, P, P, P, SZ, P]),
+    "omq_attention_fwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P]),
+    "omq_attention_bwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P, I64, P, P, I64, P, P, I64,
+                                P]),
     "omq_adamw_update": (I32, [P, I64, P, P, P, P, F32, F32, F32, F32, F32, I32]),
     "omq_stream_status": (I32, [P, P, POINTER(c_int32)]),
     "omq_status_string": (c_char_p, [I32]),
@@ -211,6 +214,19 @@ def omq_gemm_bf16(M, N, K, batch, A, a_ld, a_bs, a_kmajor, B, b_ld, b_bs, b_kmaj
     check("omq_gemm_bf16", lib().omq_gemm_bf16(
         stream_handle(stream), M, N, K, batch, ptr(A), a_ld, a_bs, a_kmajor, ptr(B), b_ld, b_bs, b_kmajor, ptr(Cf),
         ptr(Cb), ldc, c_bs, alpha, ptr(bias), ptr(R), ldr, beta_acc, causal, ptr(dev_status)))
+
+
+def omq_attention_fwd(T, n_heads, n_kv, Q, ldq, K, V, ldkv, O, ldo, lse, dev_status=None, stream=None):
+    check("omq_attention_fwd", lib().omq_attention_fwd(
+        stream_handle(stream), T, n_heads, n_kv, ptr(Q), ldq, ptr(K), ptr(V), ldkv, ptr(O), ldo, ptr(lse),
+        ptr(dev_status)))
+
+
+def omq_attention_bwd(T, n_heads, n_kv, Q, ldq, K, V, ldkv, O, ldo, lse, dO, lddo, D, dQ, ldg, dK, dV, ldgkv,
+                      dev_status=None, stream=None):
+    check("omq_attention_bwd", lib().omq_attention_bwd(
+        stream_handle(stream), T, n_heads, n_kv, ptr(Q), ldq, ptr(K), ptr(V), ldkv, ptr(O), ldo, ptr(lse), ptr(dO),
+        lddo, ptr(D), ptr(dQ), ldg, ptr(dK), ptr(dV), ldgkv, ptr(dev_status)))
 
 
 def omq_qlinear_fwd(T, Cin, Cout, X, W, B, s, delta, gamma_logit, beta_logit, Y, saved, cfg, stream=None):

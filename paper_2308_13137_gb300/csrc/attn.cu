@@ -1,6 +1,5 @@
-// Attention-side kernels: RoPE table, RoPE + [Q,K] LET (Eq. 5) + per-token Q_a of q, k, v and
-// the straight-through backward of that chain, causal softmax forward/backward on materialised
-// scores, and the small finishers of the [v, out] LET pair gradients.
+// Attention-side helpers: the RoPE table and the small finishers of the [v, out] LET pair
+// gradients (the q/k/v row kernels live in rows.cu, the attention itself in flash.cu).
 #include "attn.cuh"
 
 // angle t * theta^(-2j/hd): the frequency and the product are formed in double, the angle is reduced
@@ -26,58 +25,6 @@ omq_status rope_table(cudaStream_t st, int T, int hd, float theta, float* cs) {
   OMQ_REQUIRE(hd <= 256, OMQ_ERR_UNSUPPORTED);
   int n = T * (hd / 2);
   rope_table_kernel<<<(n + 255) / 256, 256, 0, st>>>(T, hd, (double)theta, cs);
-  OMQ_LAUNCH_CHECK();
-  return OMQ_OK;
-}
-
-// ------------------------------------------------------------------------------------------------
-// causal softmax on materialised scores: one warp per query row
-// ------------------------------------------------------------------------------------------------
-__global__ void softmax_fwd_kernel(int B, int T, const float* __restrict__ S, __nv_bfloat16* __restrict__ P) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp;
-  if (r >= (int64_t)B * T) return;
-  const int t = (int)(r % T);
-  const float* s = S + r * T;
-  __nv_bfloat16* p = P + r * T;
-  float mx = -INFINITY;
-  for (int j = lane; j <= t; j += 32) mx = fmaxf(mx, s[j]);
-  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-  float sum = 0.f;
-  for (int j = lane; j <= t; j += 32) sum += expf(s[j] - mx);
-  sum = warp_sum(sum);
-  const float inv = 1.0f / sum;
-  const int kend = min(T, (t / 128 + 1) * 128);
-  for (int j = lane; j < kend; j += 32) p[j] = f_to_bf16(j <= t ? expf(s[j] - mx) * inv : 0.f);
-}
-
-omq_status softmax_fwd_launch(cudaStream_t st, int B, int T, const float* S, __nv_bfloat16* P) {
-  int64_t rows = (int64_t)B * T;
-  softmax_fwd_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(B, T, S, P);
-  OMQ_LAUNCH_CHECK();
-  return OMQ_OK;
-}
-
-__global__ void softmax_bwd_kernel(int B, int T, const __nv_bfloat16* __restrict__ P, const float* __restrict__ dP,
-                                   float scale, __nv_bfloat16* __restrict__ dS) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp;
-  if (r >= (int64_t)B * T) return;
-  const int t = (int)(r % T);
-  const __nv_bfloat16* p = P + r * T;
-  const float* dp = dP + r * T;
-  __nv_bfloat16* ds = dS + r * T;
-  float D = 0.f;
-  for (int j = lane; j <= t; j += 32) D = fmaf(bf16_to_f(p[j]), dp[j], D);
-  D = warp_sum(D);
-  const int kend = min(T, (t / 128 + 1) * 128);
-  for (int j = lane; j < kend; j += 32) ds[j] = f_to_bf16(j <= t ? scale * bf16_to_f(p[j]) * (dp[j] - D) : 0.f);
-}
-
-omq_status softmax_bwd_launch(cudaStream_t st, int B, int T, const __nv_bfloat16* P, const float* dP, float scale,
-                              __nv_bfloat16* dS) {
-  int64_t rows = (int64_t)B * T;
-  softmax_bwd_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(B, T, P, dP, scale, dS);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }

@@ -24,12 +24,24 @@ omq_status qkv_fwd_launch(cudaStream_t st, const QkvArgs& a);
 omq_status qkv_bwd_launch(cudaStream_t st, const QkvArgs& a, int64_t* nslab);
 int64_t qkv_bwd_nslab(int T);
 
-// P = softmax(S) over keys j <= t (S already scaled); P bf16 [B, T, T], zero for t < j < the end of
-// t's 128-row block.
-omq_status softmax_fwd_launch(cudaStream_t st, int B, int T, const float* S, __nv_bfloat16* P);
-// dS = scale * P (dP - sum_j P dP), bf16, same zero convention
-omq_status softmax_bwd_launch(cudaStream_t st, int B, int T, const __nv_bfloat16* P, const float* dP, float scale,
-                              __nv_bfloat16* dS);
+// Causal attention without a materialised score matrix (flash.cu).  Q [T, H*128], K and V
+// [T, Hkv*128] bf16 (query head h reads kv head h / (H / Hkv)); O [T, H*128] fp32; lse [H, T] the
+// base-2 log-sum-exp of the scaled logits.  Backward: dO bf16 like O; D [H, T] scratch;
+// dQ [T, H*128], dK / dV [T, Hkv*128] fp32 (overwritten).
+struct FlashArgs {
+  int T, H, Hkv, hd;
+  const __nv_bfloat16* Q; const __nv_bfloat16* K; const __nv_bfloat16* V;
+  int64_t ldq, ldkv;
+  float* O; int64_t ldo;
+  float* lse;
+  const __nv_bfloat16* dO; int64_t lddo;
+  float* D;
+  float* dQ; int64_t ldg;
+  float* dK; float* dV; int64_t ldgkv;
+  int32_t* status;
+};
+omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a);
+omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a);
 
 // [v, out] LET pair vectors: r_qkv = [1 (q,k rows), 1/s_o (v rows)], shift_qkv = [0, delta_o]
 omq_status qkv_row_vectors(cudaStream_t st, int dq, int dkv, const float* so, const float* do_, float* r, float* shift);

@@ -55,7 +55,7 @@ struct BlockWS {
   // forward activations
   bf16* a_h; float* rstd1; QState4 sa;
   float* Yqkv; bf16 *Qh, *Kh, *Vh; QState4 sqkv;
-  float* S; bf16* P;
+  float* lse;                       // [H, T] base-2 log-sum-exp of the attention rows
   float* O; bf16* O_h; QState4 so;
   float* h1; bf16* b_h; float* rstd2; QState4 sb;
   float* Ygu; bf16* m_h; QState4 sm;
@@ -69,7 +69,7 @@ struct BlockWS {
   float* db;
   float* dh1; bf16* dh1_b;
   float* dOh; bf16* dO_b;
-  bf16* dS;
+  float* Drow;                      // [H, T] rowsum(dO * O)
   float* dQKV; float* dYqkv; bf16* dYqkv_b;
   float* da;
   float *dB_qkv, *dB_o, *dB_gu, *dr_qkv;
@@ -109,8 +109,7 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   w.Kh = c.take<bf16>(T * dkv);
   w.Vh = c.take<bf16>(T * dkv);
   w.sqkv = take_qstate(c, 3 * T);
-  w.S = c.take<float>(H * T * T);
-  w.P = c.take<bf16>(H * T * T);
+  w.lse = c.take<float>(H * T);
   w.O = c.take<float>(T * dq);
   w.O_h = c.take<bf16>(T * dq);
   w.so = take_qstate(c, T);
@@ -135,7 +134,7 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   w.dh1_b = c.take<bf16>(T * d);
   w.dOh = c.take<float>(T * dq);
   w.dO_b = c.take<bf16>(T * dq);
-  w.dS = c.take<bf16>(H * T * T);
+  w.Drow = c.take<float>(H * T);
   w.dQKV = c.take<float>(T * nqkv);
   w.dYqkv = c.take<float>(T * nqkv);
   w.dYqkv_b = c.take<bf16>(T * nqkv);
@@ -323,19 +322,11 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   qa.Qh = w.Qh; qa.Kh = w.Kh; qa.Vh = w.Vh;
   qa.h = w.sqkv.h; qa.z = w.sqkv.z; qa.imax = w.sqkv.imax; qa.imin = w.sqkv.imin; qa.abits = cfg.abits; qa.eps = cfg.h_eps;
   OMQ_TRY(qkv_fwd_launch(st, qa));
-  const float scale = 1.0f / sqrtf((float)c.hd);
-  const int64_t TT = c.T * c.T;
-  for (int64_t r = 0; r < c.rep; ++r) {     // query heads kv*rep + r share KV head kv
-    GemmOperand a{w.Qh + r * c.hd, c.dq, c.rep * c.hd, 1}, b{w.Kh, c.dkv, c.hd, 1};
-    GemmEpilogue ep{w.S + r * TT, nullptr, c.T, c.rep * TT, scale, nullptr, nullptr, 0, 0.f};
-    OMQ_TRY(gemm_launch(st, c.T, c.T, c.hd, c.Hkv, a, b, ep, 1, status));
-  }
-  OMQ_TRY(softmax_fwd_launch(st, (int)c.H, (int)c.T, w.S, w.P));
-  for (int64_t r = 0; r < c.rep; ++r) {
-    GemmOperand a{w.P + r * TT, c.T, c.rep * TT, 1}, b{w.Vh, c.dkv, c.hd, 0};
-    GemmEpilogue ep{w.O + r * c.hd, nullptr, c.dq, c.rep * c.hd, 1.f, nullptr, nullptr, 0, 0.f};
-    OMQ_TRY(gemm_launch(st, c.T, c.hd, c.T, c.Hkv, a, b, ep, 2, status));
-  }
+  FlashArgs fa{};
+  fa.T = (int)c.T; fa.H = (int)c.H; fa.Hkv = (int)c.Hkv; fa.hd = (int)c.hd;
+  fa.Q = w.Qh; fa.K = w.Kh; fa.V = w.Vh; fa.ldq = c.dq; fa.ldkv = c.dkv;
+  fa.O = w.O; fa.ldo = c.dq; fa.lse = w.lse; fa.status = status;
+  OMQ_TRY(flash_fwd_launch(st, fa));
   ActFwdArgs ao{};
   ao.producer = AP_PLAIN; ao.X = w.O; ao.ldx = c.dq; ao.T = c.T; ao.C = c.dq; ao.Xq = w.O_h; ao.ldq = c.dq;
   ao.h = w.so.h; ao.z = w.so.z; ao.imax = w.so.imax; ao.imin = w.so.imin; ao.abits = cfg.abits; ao.eps = cfg.h_eps;
@@ -415,34 +406,14 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   bo.dXb = w.dO_b; bo.lddxb = c.dq; bo.rows_per_cta = 4; bo.abits = cfg.abits; bo.eps = cfg.h_eps;
   OMQ_TRY(act_bwd_launch(st, bo));
 
-  // ---- attention (materialised causal scores) --------------------------------------------------------
-  const float scale = 1.0f / sqrtf((float)c.hd);
-  const int64_t TT = c.T * c.T;
-  float* dP = w.S;      // the scores are dead after the forward softmax
-  for (int64_t r = 0; r < c.rep; ++r) {
-    GemmOperand a{w.dO_b + r * c.hd, c.dq, c.rep * c.hd, 1}, b{w.Vh, c.dkv, c.hd, 1};
-    GemmEpilogue ep{dP + r * TT, nullptr, c.T, c.rep * TT, 1.f, nullptr, nullptr, 0, 0.f};
-    OMQ_TRY(gemm_launch(st, c.T, c.T, c.hd, c.Hkv, a, b, ep, 1, status));
-  }
-  OMQ_TRY(softmax_bwd_launch(st, (int)c.H, (int)c.T, w.P, dP, scale, w.dS));
-  for (int64_t r = 0; r < c.rep; ++r) {
-    const float beta = r > 0 ? 1.f : 0.f;
-    {   // dV = P^T dO  (keys x dims, summed over the query heads of the group)
-      GemmOperand a{w.P + r * TT, c.T, c.rep * TT, 0}, b{w.dO_b + r * c.hd, c.dq, c.rep * c.hd, 0};
-      GemmEpilogue ep{w.dQKV + c.dq + c.dkv, nullptr, c.nqkv, c.hd, 1.f, nullptr, nullptr, 0, beta};
-      OMQ_TRY(gemm_launch(st, c.T, c.hd, c.T, c.Hkv, a, b, ep, 3, status));
-    }
-    {   // dQ = dS K
-      GemmOperand a{w.dS + r * TT, c.T, c.rep * TT, 1}, b{w.Kh, c.dkv, c.hd, 0};
-      GemmEpilogue ep{w.dQKV + r * c.hd, nullptr, c.nqkv, c.rep * c.hd, 1.f, nullptr, nullptr, 0, 0.f};
-      OMQ_TRY(gemm_launch(st, c.T, c.hd, c.T, c.Hkv, a, b, ep, 2, status));
-    }
-    {   // dK = dS^T Q
-      GemmOperand a{w.dS + r * TT, c.T, c.rep * TT, 0}, b{w.Qh + r * c.hd, c.dq, c.rep * c.hd, 0};
-      GemmEpilogue ep{w.dQKV + c.dq, nullptr, c.nqkv, c.hd, 1.f, nullptr, nullptr, 0, beta};
-      OMQ_TRY(gemm_launch(st, c.T, c.hd, c.T, c.Hkv, a, b, ep, 3, status));
-    }
-  }
+  // ---- attention: dQ, dK, dV from the saved log-sum-exp (scores recomputed, never stored) --------
+  FlashArgs fa{};
+  fa.T = (int)c.T; fa.H = (int)c.H; fa.Hkv = (int)c.Hkv; fa.hd = (int)c.hd;
+  fa.Q = w.Qh; fa.K = w.Kh; fa.V = w.Vh; fa.ldq = c.dq; fa.ldkv = c.dkv;
+  fa.O = w.O; fa.ldo = c.dq; fa.lse = w.lse; fa.dO = w.dO_b; fa.lddo = c.dq; fa.D = w.Drow;
+  fa.dQ = w.dQKV; fa.ldg = c.nqkv; fa.dK = w.dQKV + c.dq; fa.dV = w.dQKV + c.dq + c.dkv; fa.ldgkv = c.nqkv;
+  fa.status = status;
+  OMQ_TRY(flash_bwd_launch(st, fa));
   QkvArgs qa{};
   qa.T = (int)c.T; qa.H = (int)c.H; qa.Hkv = (int)c.Hkv; qa.hd = (int)c.hd; qa.Y = w.Yqkv; qa.ldy = c.nqkv; qa.cs = w.cs;
   qa.sa_exp = c.let ? w.sa_exp : nullptr; qa.sa = c.let ? th->sa : nullptr;

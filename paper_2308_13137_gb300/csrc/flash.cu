@@ -1,0 +1,710 @@
+// Causal attention of the quantized block (Sec. 3.3 / Eq. 5: Q_a-quantized Q~, K~, V' in bf16,
+// softmax output kept unquantized) without materialising the score matrix.
+//
+// Forward: one CTA per (128-query block, query head), two passes over the key blocks.  TMA
+// streams 128-key blocks through a two-slot ring; tcgen05.mma forms S = Q K^T in one of two
+// tensor-memory buffers while the four compute warps (one query row per thread) work on the
+// previous one.  Pass 1 reduces S to the row maximum m and the row sum l of exp2(c S - m); pass 2
+// recomputes S and writes the normalised probabilities P = bf16(exp2(c S - m) / l) into shared
+// memory in the 128-byte-swizzled operand layout, and the MMA warp accumulates O += P V in tensor
+// memory.  Rounding the normalised P to bf16 (not a running, unnormalised one) keeps the product
+// identical to softmax-then-round; the extra S product costs one 128-dim contraction.  The row
+// log-sum-exp (base 2, scaled logits) is saved for the backward.
+//
+// Backward: dKV kernel per (128-key block, kv head) walks the 64-query blocks of every query head
+// of its group: S^T = K Q^T and dP^T = V dO^T (double-buffered in tensor memory), P^T and
+// dS^T = P^T (dP^T - D) scale formed by the compute warps (one key row per thread),
+// dV += P^T dO and dK += dS^T Q accumulated in tensor memory.  dQ kernel per (128-query block,
+// query head) recomputes S and dP for its keys and accumulates dQ += dS K.  D = rowsum(dO * O).
+//
+// Warp roles (192 threads): warp 0 TMA, warp 1 tensor memory + MMA issue, warps 2..5 compute.
+// Every mbarrier wait is bounded; on expiry the status word gets OMQ_ERR_TIMEOUT and the kernel
+// winds down (frees its tensor memory and returns).
+#include "attn.cuh"
+#include "tc.cuh"
+
+#include <cstring>
+
+namespace {
+
+using namespace tc;
+
+constexpr int FA_THREADS = 192;
+constexpr int HD = 128;                     // head dimension
+constexpr int ROW_BYTES = 128;              // one swizzle row: 64 bf16
+
+// K-major operand descriptor, k-step kk (16 columns), of a tile whose 64-column atoms are
+// atom_bytes apart (atom = rows x 128 bytes)
+__device__ __forceinline__ uint64_t desc_k(uint32_t tile, int kk, uint32_t atom_bytes) {
+  return sdesc(tile + (kk >> 2) * atom_bytes + (kk & 3) * 32, 16, 1024);
+}
+// MN-major view of the same tile (rows = K, 64-column atoms = N chunks), k-step kk (16 rows)
+__device__ __forceinline__ uint64_t desc_mn(uint32_t tile, int kk, uint32_t atom_bytes) {
+  return sdesc(tile + kk * 2048, atom_bytes, 1024);
+}
+
+// columns c0 .. c0+31 (c0 a multiple of 32) of row r of a K-major, 128-byte-swizzled bf16 tile
+__device__ __forceinline__ void st_row32(uint8_t* tile, uint32_t atom_bytes, int r, int c0, const float* v) {
+  uint8_t* row = tile + (c0 >> 6) * atom_bytes + r * ROW_BYTES;
+  const int ch0 = (c0 & 63) >> 3;
+#pragma unroll
+  for (int u = 0; u < 4; ++u) *reinterpret_cast<uint4*>(row + (((ch0 + u) ^ (r & 7)) << 4)) = pack_bf16x8(v + 8 * u);
+}
+
+
+// a [rows x 128] bf16 tile as two {64, rows} boxes (64-column atoms)
+__device__ __forceinline__ void load_tile(const CUtensorMap* m, uint64_t* bar, uint8_t* dst, int col0, int row0,
+                                          uint32_t atom_bytes) {
+  tma_load_3d(m, bar, dst, col0, row0, 0);
+  tma_load_3d(m, bar, dst + atom_bytes, col0 + 64, row0, 0);
+}
+
+struct Ctl {                 // barriers + tensor-memory holder + abort flag, after the tiles
+  uint64_t bar[16];
+  uint32_t tmem;
+  int abort;
+};
+
+__device__ __forceinline__ bool waitb(uint64_t* b, uint32_t parity, int32_t* status, volatile int* abort_flag) {
+  if (mbar_wait(b, parity)) return true;
+  omq_set_status(status, OMQ_ERR_TIMEOUT);
+  *abort_flag = 1;
+  return false;
+}
+
+// warp-uniform wait of the compute warps (tcgen05.ld / st are warp-collective)
+__device__ __forceinline__ bool waitw(uint64_t* b, uint32_t parity, int32_t* status, volatile int* abort_flag) {
+  const bool ok = __all_sync(0xffffffffu, mbar_wait(b, parity));
+  if (!ok) { omq_set_status(status, OMQ_ERR_TIMEOUT); *abort_flag = 1; }
+  return ok;
+}
+
+// ================================================================================================
+// forward
+// ================================================================================================
+struct FwdP {
+  int T, H, rep;
+  float c;                   // log2(e) / sqrt(head_dim)
+  float* O; int64_t ldo;     // [T, H*128] fp32
+  float* lse;                // [H, T]: m + log2(l) of the scaled base-2 logits
+  int32_t* status;
+};
+
+constexpr int F_TILE = 128 * ROW_BYTES * 2;           // 32 KB: [128 x 128] bf16
+constexpr int F_ATOM = 128 * ROW_BYTES;               // 16 KB
+constexpr int F_Q = 0, F_K = F_TILE, F_V = 3 * F_TILE, F_P = 5 * F_TILE, F_CTL = 6 * F_TILE;
+constexpr int F_SMEM = F_CTL + 1024 + 1024;
+
+__global__ void __launch_bounds__(FA_THREADS, 1)
+    flash_fwd_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                     const __grid_constant__ CUtensorMap tmV, const FwdP p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  Ctl* ctl = reinterpret_cast<Ctl*>(smem + F_CTL);
+  uint64_t* q_full = &ctl->bar[0];
+  uint64_t* kv_full = &ctl->bar[1];       // [2]
+  uint64_t* kv_empty = &ctl->bar[3];      // [2]
+  uint64_t* s_full = &ctl->bar[5];        // [2]
+  uint64_t* p_full = &ctl->bar[7];
+  uint64_t* o_done = &ctl->bar[8];
+  volatile int* abort_flag = &ctl->abort;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nqb = (p.T + 127) / 128;
+  const int qb = nqb - 1 - (int)blockIdx.x;          // longest rows first
+  const int h = blockIdx.y, g = h / p.rep;
+  const int nkb = qb + 1;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < 2; ++s) { mbar_init(&kv_full[s], 1); mbar_init(&kv_empty[s], 1); mbar_init(&s_full[s], 1); }
+    mbar_init(p_full, 4);
+    mbar_init(o_done, 1);
+    ctl->abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(&ctl->tmem, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = ctl->tmem;           // S buffers at columns 0 / 128, O at 256
+
+  // iterations 0 .. nkb-1: statistics pass (S only: row max m, row sum l of exp2(c S - m));
+  // iterations nkb .. 2 nkb-1: output pass (S again, P = bf16(exp2(c S - m) / l), O += P V)
+  const int nit = 2 * nkb;
+  if (warp == 0 && lane == 0) {
+    mbar_expect_tx(q_full, F_TILE);
+    load_tile(&tmQ, q_full, smem + F_Q, h * HD, qb * 128, F_ATOM);
+    for (int it = 0; it < nit && !*abort_flag; ++it) {
+      const int s = it & 1, j = it < nkb ? it : it - nkb;
+      if (!waitb(&kv_empty[s], ((it >> 1) & 1) ^ 1, p.status, abort_flag)) break;
+      mbar_expect_tx(&kv_full[s], it < nkb ? F_TILE : 2 * F_TILE);
+      load_tile(&tmK, &kv_full[s], smem + F_K + s * F_TILE, g * HD, j * 128, F_ATOM);
+      if (it >= nkb) load_tile(&tmV, &kv_full[s], smem + F_V + s * F_TILE, g * HD, j * 128, F_ATOM);
+    }
+  } else if (warp == 1 && lane == 0) {
+    constexpr uint32_t ID_S = idesc_bf16(128, 128, 0, 0), ID_O = idesc_bf16(128, 128, 0, 1);
+    const uint32_t sq = smem_u32(smem + F_Q), sk = smem_u32(smem + F_K), sv = smem_u32(smem + F_V);
+    const uint32_t sp = smem_u32(smem + F_P);
+    bool ok = waitb(q_full, 0, p.status, abort_flag);
+    auto issue_s = [&](int it) -> bool {
+      const int s = it & 1;
+      if (!waitb(&kv_full[s], (it >> 1) & 1, p.status, abort_flag)) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk)
+        umma_bf16(tmem + 128 * s, desc_k(sq, kk, F_ATOM), desc_k(sk + s * F_TILE, kk, F_ATOM), ID_S, kk > 0);
+      umma_commit(&s_full[s]);
+      return true;
+    };
+    if (ok) ok = issue_s(0);
+    for (int it = 0; ok && it < nit; ++it) {
+      // S buffer (it+1)&1 was last read at it-1, whose p_full was waited for below
+      if (it + 1 < nit && !issue_s(it + 1)) break;
+      if (!waitb(p_full, it & 1, p.status, abort_flag)) break;
+      tc_fence_after();
+      if (it >= nkb) {
+        const int j = it - nkb;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          umma_bf16(tmem + 256, desc_k(sp, kk, F_ATOM), desc_mn(sv + (it & 1) * F_TILE, kk, F_ATOM), ID_O,
+                    (j | kk) != 0);
+        umma_commit(o_done);
+      }
+      umma_commit(&kv_empty[it & 1]);
+    }
+  } else if (warp >= 2) {
+    const int q = warp & 3;
+    const int r = q * 32 + lane;                      // row of the block = TMEM lane
+    const int row = qb * 128 + r;
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    uint8_t* ptile = smem + F_P;
+    float m = -INFINITY, l = 0.f, inv_l = 0.f;
+    bool ok = true;
+    for (int it = 0; it < nit; ++it) {
+      const int j = it < nkb ? it : it - nkb;
+      if (!(ok = waitw(&s_full[it & 1], (it >> 1) & 1, p.status, abort_flag))) break;
+      tc_fence_after();
+      const uint32_t sb = tmem + 128 * (it & 1) + lane_off;
+      const bool diag = (j == qb);                    // keys beyond the row exist only here
+      if (it < nkb) {                                 // statistics: running max, rescaled sum
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld32(sb + 32 * c, v);
+          if (diag) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) if (32 * c + i > r) v[i] = -INFINITY;
+          }
+          float t[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) t[i] = fmaxf(v[i], v[i + 16]);
+#pragma unroll
+          for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+            for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
+          const float m_new = fmaxf(m, t[0] * p.c);
+          float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int i = 0; i < 32; ++i) s4[i & 3] += ex2(fmaf(v[i], p.c, -m_new));
+          l = l * ex2(m - m_new) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
+          m = m_new;
+        }
+        if (it == nkb - 1) inv_l = 1.f / l;
+      } else {                                        // probabilities of this key block
+        if (j > 0) {                                  // the previous P V product has read P
+          if (!(ok = waitw(o_done, (j - 1) & 1, p.status, abort_flag))) break;
+          tc_fence_after();
+        }
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld32(sb + 32 * c, v);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = ex2(fmaf(v[i], p.c, -m)) * inv_l;
+          if (diag) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) if (32 * c + i > r) v[i] = 0.f;
+          }
+          st_row32(ptile, F_ATOM, r, 32 * c, v);
+        }
+        fence_async_smem();                           // P visible to the tensor core
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+    }
+    if (ok && waitw(o_done, (nkb - 1) & 1, p.status, abort_flag)) {
+      tc_fence_after();
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        float o[32];
+        tmem_ld32(tmem + 256 + lane_off + 32 * c, o);
+        if (row < p.T) {
+          float4* dst = reinterpret_cast<float4*>(p.O + (int64_t)row * p.ldo + h * HD + 32 * c);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) dst[i] = make_float4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+        }
+      }
+      if (row < p.T) p.lse[(int64_t)h * p.T + row] = m + log2f(l);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ================================================================================================
+// backward: D = rowsum(dO * O) per (token, head)
+// ================================================================================================
+__global__ void attn_rowdot_kernel(int T, int H, const __nv_bfloat16* __restrict__ dO, int64_t lddo,
+                                   const float* __restrict__ O, int64_t ldo, float* __restrict__ D) {
+  const int64_t w = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (w >= (int64_t)T * H) return;
+  const int t = (int)(w / H), h = (int)(w % H);
+  const float4 o = *reinterpret_cast<const float4*>(O + (int64_t)t * ldo + h * HD + 4 * lane);
+  const uint2 u = *reinterpret_cast<const uint2*>(dO + (int64_t)t * lddo + h * HD + 4 * lane);
+  const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&u);
+  const float2 d01 = __bfloat1622float2(b[0]), d23 = __bfloat1622float2(b[1]);
+  const float s = warp_sum(o.x * d01.x + o.y * d01.y + o.z * d23.x + o.w * d23.y);
+  if (lane == 0) D[(int64_t)h * T + t] = s;
+}
+
+// ================================================================================================
+// backward, dK and dV: one CTA per (128-key block, kv head)
+// ================================================================================================
+struct BwdP {
+  int T, H, rep;
+  float c;                   // log2(e) / sqrt(head_dim)
+  float scale;               // 1 / sqrt(head_dim)
+  const float* lse; const float* D;      // [H, T]
+  float* dQ; int64_t ldq;    // [T, H*128]
+  float* dK; float* dV; int64_t ldkv;    // [T, Hkv*128]
+  int32_t* status;
+};
+
+constexpr int B_QATOM = 64 * ROW_BYTES;               // 8 KB: 64-row atom
+constexpr int B_QTILE = 2 * B_QATOM;                  // [64 x 128] bf16
+constexpr int B_K = 0, B_V = F_TILE, B_Q = 2 * F_TILE, B_DO = B_Q + 2 * B_QTILE;
+constexpr int B_PT = B_DO + 2 * B_QTILE;              // P^T [128 keys x 64 queries]: one 16 KB atom
+constexpr int B_DST = B_PT + F_ATOM;                  // dS^T, same shape
+constexpr int B_LD = B_DST + F_ATOM;                  // [2 stages][lse 64 | D 64] fp32
+constexpr int B_CTL = B_LD + 1024;
+constexpr int B_SMEM = B_CTL + 1024 + 1024;
+
+__global__ void __launch_bounds__(FA_THREADS, 1)
+    flash_bwd_dkv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                         const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
+                         const BwdP p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  Ctl* ctl = reinterpret_cast<Ctl*>(smem + B_CTL);
+  uint64_t* kv_full = &ctl->bar[0];
+  uint64_t* qd_full = &ctl->bar[1];      // [2]
+  uint64_t* qd_empty = &ctl->bar[3];     // [2]
+  uint64_t* s_full = &ctl->bar[5];       // [2]: S^T and dP^T of a query block ready
+  uint64_t* p_full = &ctl->bar[7];       // P^T, dS^T written
+  uint64_t* g_done = &ctl->bar[8];       // dV / dK products of a query block done (P^T, dS^T free)
+  volatile int* abort_flag = &ctl->abort;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int kb = blockIdx.x, g = blockIdx.y;
+  const int nq64 = (p.T + 63) / 64;
+  const int i0 = 2 * kb;                              // first 64-query block with a visible key
+  const int niq = nq64 > i0 ? nq64 - i0 : 0;
+  const int nit = niq * p.rep;                        // (head, query block) iterations
+
+  if (threadIdx.x == 0) {
+    mbar_init(kv_full, 1);
+    for (int s = 0; s < 2; ++s) { mbar_init(&qd_full[s], 1); mbar_init(&qd_empty[s], 1); mbar_init(&s_full[s], 1); }
+    mbar_init(p_full, 4);
+    mbar_init(g_done, 1);
+    ctl->abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(&ctl->tmem, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  // tensor memory: S^T at 0 / 64, dP^T at 128 / 192 (per buffer), dV at 256, dK at 384
+  const uint32_t tmem = ctl->tmem;
+
+  if (warp == 0 && lane == 0) {
+    mbar_expect_tx(kv_full, 2 * F_TILE);
+    load_tile(&tmK, kv_full, smem + B_K, g * HD, kb * 128, F_ATOM);
+    load_tile(&tmV, kv_full, smem + B_V, g * HD, kb * 128, F_ATOM);
+    for (int it = 0; it < nit && !*abort_flag; ++it) {
+      const int s = it & 1;
+      const int h = g * p.rep + it / niq, qi = i0 + it % niq;
+      if (!waitb(&qd_empty[s], ((it >> 1) & 1) ^ 1, p.status, abort_flag)) break;
+      const uint32_t nb = (uint32_t)min(64, p.T - qi * 64) * 4;     // lse / D bytes inside [0, T)
+      mbar_expect_tx(&qd_full[s], 2 * B_QTILE + 2 * nb);
+      load_tile(&tmQ, &qd_full[s], smem + B_Q + s * B_QTILE, h * HD, qi * 64, B_QATOM);
+      load_tile(&tmdO, &qd_full[s], smem + B_DO + s * B_QTILE, h * HD, qi * 64, B_QATOM);
+      float* ld = reinterpret_cast<float*>(smem + B_LD + s * 512);
+      bulk_g2s(ld, p.lse + (int64_t)h * p.T + qi * 64, nb, &qd_full[s]);
+      bulk_g2s(ld + 64, p.D + (int64_t)h * p.T + qi * 64, nb, &qd_full[s]);
+    }
+  } else if (warp == 1 && lane == 0) {
+    constexpr uint32_t ID_S = idesc_bf16(128, 64, 0, 0), ID_G = idesc_bf16(128, 128, 0, 1);
+    const uint32_t sk = smem_u32(smem + B_K), sv = smem_u32(smem + B_V);
+    const uint32_t sq = smem_u32(smem + B_Q), sd = smem_u32(smem + B_DO);
+    const uint32_t spt = smem_u32(smem + B_PT), sdst = smem_u32(smem + B_DST);
+    bool ok = waitb(kv_full, 0, p.status, abort_flag);
+    auto issue_s = [&](int it) -> bool {
+      const int s = it & 1;
+      if (!waitb(&qd_full[s], (it >> 1) & 1, p.status, abort_flag)) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        umma_bf16(tmem + 64 * s, desc_k(sk, kk, F_ATOM), desc_k(sq + s * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
+        umma_bf16(tmem + 128 + 64 * s, desc_k(sv, kk, F_ATOM), desc_k(sd + s * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
+      }
+      umma_commit(&s_full[s]);
+      return true;
+    };
+    if (ok && nit > 0) ok = issue_s(0);
+    for (int it = 0; ok && it < nit; ++it) {
+      const int s = it & 1;
+      if (it + 1 < nit && !issue_s(it + 1)) break;
+      if (!waitb(p_full, it & 1, p.status, abort_flag)) break;
+      tc_fence_after();
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {               // K = 64 queries
+        umma_bf16(tmem + 256, desc_k(spt, kk, F_ATOM), desc_mn(sd + s * B_QTILE, kk, B_QATOM), ID_G, (it | kk) != 0);
+        umma_bf16(tmem + 384, desc_k(sdst, kk, F_ATOM), desc_mn(sq + s * B_QTILE, kk, B_QATOM), ID_G, (it | kk) != 0);
+      }
+      umma_commit(g_done);
+      umma_commit(&qd_empty[s]);
+    }
+  } else if (warp >= 2) {
+    const int q = warp & 3;
+    const int r = q * 32 + lane;                      // key row of the block = TMEM lane
+    const int key = kb * 128 + r;
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    uint8_t* pt = smem + B_PT;
+    uint8_t* dst = smem + B_DST;
+    bool ok = true;
+    for (int it = 0; it < nit; ++it) {
+      const int s = it & 1;
+      const int qi = i0 + it % niq;
+      const float* L = reinterpret_cast<const float*>(smem + B_LD + s * 512);
+      const float* Dq = L + 64;
+      // queries below the key block's last key, or past T, need the mask; the rest see every key
+      const bool need_mask = qi * 64 < kb * 128 + 127 || qi * 64 + 64 > p.T;
+      if (!(ok = waitw(&s_full[s], (it >> 1) & 1, p.status, abort_flag))) break;
+      tc_fence_after();
+      if (it > 0) {                                   // previous dV / dK products done: P^T, dS^T free
+        if (!(ok = waitw(g_done, (it - 1) & 1, p.status, abort_flag))) break;
+        tc_fence_after();
+      }
+#pragma unroll 1
+      for (int c = 0; c < 2; ++c) {
+        float sv[32], dp[32];
+        tmem_ld32(tmem + 64 * s + lane_off + 32 * c, sv);
+        tmem_ld32(tmem + 128 + 64 * s + lane_off + 32 * c, dp);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float pv = ex2(fmaf(sv[i], p.c, -L[32 * c + i]));
+          sv[i] = pv;
+          dp[i] = pv * (dp[i] - Dq[32 * c + i]) * p.scale;
+        }
+        if (need_mask) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int qrow = qi * 64 + 32 * c + i;
+            if (key > qrow || qrow >= p.T) { sv[i] = 0.f; dp[i] = 0.f; }
+          }
+        }
+        st_row32(pt, F_ATOM, r, 32 * c, sv);
+        st_row32(dst, F_ATOM, r, 32 * c, dp);
+      }
+      fence_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+    }
+    if (ok && nit > 0 && waitw(g_done, (nit - 1) & 1, p.status, abort_flag)) {
+      tc_fence_after();
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        float dv[32], dk[32];
+        tmem_ld32(tmem + 256 + lane_off + 32 * c, dv);
+        tmem_ld32(tmem + 384 + lane_off + 32 * c, dk);
+        if (key < p.T) {
+          float4* a = reinterpret_cast<float4*>(p.dV + (int64_t)key * p.ldkv + g * HD + 32 * c);
+          float4* b = reinterpret_cast<float4*>(p.dK + (int64_t)key * p.ldkv + g * HD + 32 * c);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            a[i] = make_float4(dv[4 * i], dv[4 * i + 1], dv[4 * i + 2], dv[4 * i + 3]);
+            b[i] = make_float4(dk[4 * i], dk[4 * i + 1], dk[4 * i + 2], dk[4 * i + 3]);
+          }
+        }
+      }
+    } else if (ok && nit == 0 && key < p.T) {        // keys no query sees (cannot happen for T > 0)
+      for (int c = 0; c < HD; ++c) {
+        p.dV[(int64_t)key * p.ldkv + g * HD + c] = 0.f;
+        p.dK[(int64_t)key * p.ldkv + g * HD + c] = 0.f;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ================================================================================================
+// backward, dQ: one CTA per (128-query block, query head), 64-key blocks, S / dP / dS double-buffered
+// ================================================================================================
+constexpr int Q_Q = 0, Q_DO = F_TILE, Q_K = 2 * F_TILE, Q_V = Q_K + 2 * B_QTILE, Q_DS = Q_V + 2 * B_QTILE;
+constexpr int Q_CTL = Q_DS + 2 * F_ATOM;
+constexpr int Q_SMEM = Q_CTL + 1024 + 1024;
+
+__global__ void __launch_bounds__(FA_THREADS, 1)
+    flash_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                        const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
+                        const BwdP p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  Ctl* ctl = reinterpret_cast<Ctl*>(smem + Q_CTL);
+  uint64_t* q_full = &ctl->bar[0];
+  uint64_t* kv_full = &ctl->bar[1];      // [2]
+  uint64_t* kv_empty = &ctl->bar[3];     // [2]
+  uint64_t* s_full = &ctl->bar[5];       // [2]: S and dP of a key block ready
+  uint64_t* p_full = &ctl->bar[7];       // dS written
+  uint64_t* g_done = &ctl->bar[8];       // dQ product of a key block done
+  volatile int* abort_flag = &ctl->abort;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nqb = (p.T + 127) / 128;
+  const int qb = nqb - 1 - (int)blockIdx.x;
+  const int h = blockIdx.y, g = h / p.rep;
+  const int nkb = 2 * qb + 2;                         // 64-key blocks up to the block's last query
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&kv_full[s], 1); mbar_init(&kv_empty[s], 1); mbar_init(&s_full[s], 1);
+    }
+    mbar_init(p_full, 4);
+    mbar_init(g_done, 1);
+    ctl->abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(&ctl->tmem, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = ctl->tmem;       // S at 0 / 64, dP at 128 / 192, dQ at 256
+
+  if (warp == 0 && lane == 0) {
+    mbar_expect_tx(q_full, 2 * F_TILE);
+    load_tile(&tmQ, q_full, smem + Q_Q, h * HD, qb * 128, F_ATOM);
+    load_tile(&tmdO, q_full, smem + Q_DO, h * HD, qb * 128, F_ATOM);
+    for (int j = 0; j < nkb && !*abort_flag; ++j) {
+      const int s = j & 1;
+      if (!waitb(&kv_empty[s], ((j >> 1) & 1) ^ 1, p.status, abort_flag)) break;
+      mbar_expect_tx(&kv_full[s], 2 * B_QTILE);
+      load_tile(&tmK, &kv_full[s], smem + Q_K + s * B_QTILE, g * HD, j * 64, B_QATOM);
+      load_tile(&tmV, &kv_full[s], smem + Q_V + s * B_QTILE, g * HD, j * 64, B_QATOM);
+    }
+  } else if (warp == 1 && lane == 0) {
+    constexpr uint32_t ID_S = idesc_bf16(128, 64, 0, 0), ID_G = idesc_bf16(128, 128, 0, 1);
+    const uint32_t sq = smem_u32(smem + Q_Q), sd = smem_u32(smem + Q_DO);
+    const uint32_t sk = smem_u32(smem + Q_K), sv = smem_u32(smem + Q_V), sds = smem_u32(smem + Q_DS);
+    bool ok = waitb(q_full, 0, p.status, abort_flag);
+    auto issue_s = [&](int j) -> bool {
+      const int s = j & 1;
+      if (!waitb(&kv_full[s], (j >> 1) & 1, p.status, abort_flag)) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        umma_bf16(tmem + 64 * s, desc_k(sq, kk, F_ATOM), desc_k(sk + s * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
+        umma_bf16(tmem + 128 + 64 * s, desc_k(sd, kk, F_ATOM), desc_k(sv + s * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
+      }
+      umma_commit(&s_full[s]);
+      return true;
+    };
+    if (ok) ok = issue_s(0);
+    for (int j = 0; ok && j < nkb; ++j) {
+      const int s = j & 1;
+      // S / dP buffer (j+1)&1 was last read at j-1, whose p_full was waited for below
+      if (j + 1 < nkb && !issue_s(j + 1)) break;
+      if (!waitb(p_full, j & 1, p.status, abort_flag)) break;
+      tc_fence_after();
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)               // K = 64 keys
+        umma_bf16(tmem + 256, desc_k(sds + s * F_ATOM, kk, F_ATOM), desc_mn(sk + s * B_QTILE, kk, B_QATOM), ID_G,
+                  (j | kk) != 0);
+      umma_commit(g_done);
+      umma_commit(&kv_empty[s]);
+    }
+  } else if (warp >= 2) {
+    const int q = warp & 3;
+    const int r = q * 32 + lane;
+    const int row = qb * 128 + r;
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    const bool row_ok = row < p.T;
+    const float Lr = row_ok ? p.lse[(int64_t)h * p.T + row] : 0.f;
+    const float Dr = row_ok ? p.D[(int64_t)h * p.T + row] : 0.f;
+    bool ok = true;
+    int waited = 0;                                   // g_done phases waited for so far
+    for (int j = 0; j < nkb; ++j) {
+      const int s = j & 1;
+      if (!(ok = waitw(&s_full[s], (j >> 1) & 1, p.status, abort_flag))) break;
+      tc_fence_after();
+      for (; waited <= j - 2; ++waited) {             // dQ product j-2 has read dS buffer s
+        if (!(ok = waitw(g_done, waited & 1, p.status, abort_flag))) break;
+      }
+      if (!ok) break;
+      tc_fence_after();
+      const bool need_mask = j * 64 + 63 > qb * 128 || !row_ok;
+      uint8_t* dst = smem + Q_DS + s * F_ATOM;
+#pragma unroll 1
+      for (int c = 0; c < 2; ++c) {
+        float sv[32], dp[32];
+        tmem_ld32(tmem + 64 * s + lane_off + 32 * c, sv);
+        tmem_ld32(tmem + 128 + 64 * s + lane_off + 32 * c, dp);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) dp[i] = ex2(fmaf(sv[i], p.c, -Lr)) * (dp[i] - Dr) * p.scale;
+        if (need_mask) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (j * 64 + 32 * c + i > row || !row_ok) dp[i] = 0.f;
+        }
+        st_row32(dst, F_ATOM, r, 32 * c, dp);
+      }
+      fence_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+    }
+    for (; ok && waited < nkb; ++waited) ok = waitw(g_done, waited & 1, p.status, abort_flag);
+    if (ok) {
+      tc_fence_after();
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        float o[32];
+        tmem_ld32(tmem + 256 + lane_off + 32 * c, o);
+        if (row_ok) {
+          float4* a = reinterpret_cast<float4*>(p.dQ + (int64_t)row * p.ldq + h * HD + 32 * c);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) a[i] = make_float4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+bool set_smem(const void* fn, int bytes) {
+  return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) == cudaSuccess;
+}
+
+}  // namespace
+
+omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
+  OMQ_REQUIRE(a.T > 0 && a.H > 0 && a.Hkv > 0 && a.H % a.Hkv == 0 && a.hd == HD, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(a.Q && a.K && a.V && a.O && a.lse, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(a.ldq % 8 == 0 && a.ldkv % 8 == 0 && a.ldo % 4 == 0, OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(omq_aligned16(a.Q) && omq_aligned16(a.K) && omq_aligned16(a.V) && omq_aligned16(a.O), OMQ_ERR_ALIGN);
+  CUtensorMap tq, tk, tv;
+  bool ok = omq_make_map_bf16(&tq, a.Q, (int64_t)a.H * HD, a.T, 1, a.ldq, 0, 64, 128);
+  ok = ok && omq_make_map_bf16(&tk, a.K, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 128);
+  ok = ok && omq_make_map_bf16(&tv, a.V, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 128);
+  CUtensorMap tk64, tv64;
+  ok = ok && omq_make_map_bf16(&tk64, a.K, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
+  ok = ok && omq_make_map_bf16(&tv64, a.V, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
+  if (!ok) return OMQ_ERR_UNSUPPORTED;
+  static bool attr = false;
+  if (!attr) { if (!set_smem((const void*)flash_fwd_kernel, F_SMEM)) return OMQ_ERR_CUDA; attr = true; }
+  FwdP p;
+  p.T = a.T; p.H = a.H; p.rep = a.H / a.Hkv;
+  p.c = (float)(1.4426950408889634 / sqrt((double)HD));
+  p.O = a.O; p.ldo = a.ldo; p.lse = a.lse; p.status = a.status;
+  dim3 grid((unsigned)((a.T + 127) / 128), (unsigned)a.H);
+  flash_fwd_kernel<<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, p);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
+  OMQ_REQUIRE(a.T > 0 && a.H > 0 && a.Hkv > 0 && a.H % a.Hkv == 0 && a.hd == HD, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(a.Q && a.K && a.V && a.O && a.lse && a.dO && a.D && a.dQ && a.dK && a.dV, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(a.ldq % 8 == 0 && a.ldkv % 8 == 0 && a.ldo % 4 == 0 && a.lddo % 8 == 0 && a.ldg % 4 == 0 &&
+                  a.ldgkv % 4 == 0,
+              OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(omq_aligned16(a.dO) && omq_aligned16(a.dQ) && omq_aligned16(a.dK) && omq_aligned16(a.dV), OMQ_ERR_ALIGN);
+  // lse and D rows are fetched by 16-byte bulk copies
+  OMQ_REQUIRE(a.T % 4 == 0 && omq_aligned16(a.lse) && omq_aligned16(a.D), OMQ_ERR_ALIGN);
+  CUtensorMap tq64, tdo64, tk, tv, tq, tdo;
+  bool ok = omq_make_map_bf16(&tq64, a.Q, (int64_t)a.H * HD, a.T, 1, a.ldq, 0, 64, 64);
+  ok = ok && omq_make_map_bf16(&tdo64, a.dO, (int64_t)a.H * HD, a.T, 1, a.lddo, 0, 64, 64);
+  ok = ok && omq_make_map_bf16(&tq, a.Q, (int64_t)a.H * HD, a.T, 1, a.ldq, 0, 64, 128);
+  ok = ok && omq_make_map_bf16(&tdo, a.dO, (int64_t)a.H * HD, a.T, 1, a.lddo, 0, 64, 128);
+  ok = ok && omq_make_map_bf16(&tk, a.K, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 128);
+  ok = ok && omq_make_map_bf16(&tv, a.V, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 128);
+  CUtensorMap tk64, tv64;
+  ok = ok && omq_make_map_bf16(&tk64, a.K, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
+  ok = ok && omq_make_map_bf16(&tv64, a.V, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
+  if (!ok) return OMQ_ERR_UNSUPPORTED;
+  static bool attr = false;
+  if (!attr) {
+    if (!set_smem((const void*)flash_bwd_dkv_kernel, B_SMEM) || !set_smem((const void*)flash_bwd_dq_kernel, Q_SMEM))
+      return OMQ_ERR_CUDA;
+    attr = true;
+  }
+  const int64_t rows = (int64_t)a.T * a.H;
+  attn_rowdot_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(a.T, a.H, a.dO, a.lddo, a.O, a.ldo, a.D);
+  OMQ_LAUNCH_CHECK();
+  BwdP p;
+  p.T = a.T; p.H = a.H; p.rep = a.H / a.Hkv;
+  p.c = (float)(1.4426950408889634 / sqrt((double)HD));
+  p.scale = (float)(1.0 / sqrt((double)HD));
+  p.lse = a.lse; p.D = a.D;
+  p.dQ = a.dQ; p.ldq = a.ldg; p.dK = a.dK; p.dV = a.dV; p.ldkv = a.ldgkv;
+  p.status = a.status;
+  dim3 g1((unsigned)((a.T + 127) / 128), (unsigned)a.Hkv);
+  flash_bwd_dkv_kernel<<<g1, FA_THREADS, B_SMEM, st>>>(tq64, tk, tv, tdo64, p);
+  OMQ_LAUNCH_CHECK();
+  dim3 g2((unsigned)((a.T + 127) / 128), (unsigned)a.H);
+  flash_bwd_dq_kernel<<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, p);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+extern "C" omq_status omq_attention_fwd(omq_stream_t stream, int32_t T, int32_t n_heads, int32_t n_kv, const void* Q,
+                                        int64_t ldq, const void* K, const void* V, int64_t ldkv, float* O,
+                                        int64_t ldo, float* lse, int32_t* dev_status) {
+  FlashArgs a{};
+  a.T = T; a.H = n_heads; a.Hkv = n_kv; a.hd = HD;
+  a.Q = (const __nv_bfloat16*)Q; a.K = (const __nv_bfloat16*)K; a.V = (const __nv_bfloat16*)V;
+  a.ldq = ldq; a.ldkv = ldkv; a.O = O; a.ldo = ldo; a.lse = lse; a.status = dev_status;
+  return flash_fwd_launch((cudaStream_t)stream, a);
+}
+
+extern "C" omq_status omq_attention_bwd(omq_stream_t stream, int32_t T, int32_t n_heads, int32_t n_kv, const void* Q,
+                                        int64_t ldq, const void* K, const void* V, int64_t ldkv, const float* O,
+                                        int64_t ldo, const float* lse, const void* dO, int64_t lddo, float* D,
+                                        float* dQ, int64_t ldg, float* dK, float* dV, int64_t ldgkv,
+                                        int32_t* dev_status) {
+  FlashArgs a{};
+  a.T = T; a.H = n_heads; a.Hkv = n_kv; a.hd = HD;
+  a.Q = (const __nv_bfloat16*)Q; a.K = (const __nv_bfloat16*)K; a.V = (const __nv_bfloat16*)V;
+  a.ldq = ldq; a.ldkv = ldkv; a.O = const_cast<float*>(O); a.ldo = ldo; a.lse = const_cast<float*>(lse);
+  a.dO = (const __nv_bfloat16*)dO; a.lddo = lddo; a.D = D;
+  a.dQ = dQ; a.ldg = ldg; a.dK = dK; a.dV = dV; a.ldgkv = ldgkv; a.status = dev_status;
+  return flash_bwd_launch((cudaStream_t)stream, a);
+}
