@@ -5,6 +5,8 @@
 #include "gemm.cuh"
 #include "quant.cuh"
 
+#include <mutex>
+
 namespace {
 
 struct Carve {
@@ -75,6 +77,7 @@ struct BlockWS {
   float *dB_qkv, *dB_o, *dB_gu, *dr_qkv;
   float *vtmp0, *vtmp1, *vtmp2;     // [max(d, dq)] scratch vectors
   float* part;                      // shared partial-sum scratch
+  float* part_aux;                  // scratch of the weight-gradient launches on the auxiliary stream
   size_t part_elems;
 };
 
@@ -161,6 +164,11 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   pe = imax64(pe, colsum_rows_parts(T) * imax64(2 * f, nqkv));
   w.part_elems = (size_t)pe;
   w.part = c.take<float>(pe);
+  int64_t pa = 0;
+  const int64_t lin[4][2] = {{nqkv, d}, {d, dq}, {2 * f, d}, {d, f}};
+  for (const auto& l : lin)
+    pa = imax64(pa, imax64(lwc_fused_scratch_elems(l[0], l[1]), (int64_t)lwc_bwd_scratch_bytes(l[0], l[1]) / 4 + 64));
+  w.part_aux = c.take<float>(pa);
 }
 
 omq_status check_block(const omq_block_shape* s, const omq_qcfg* cfg) {
@@ -267,8 +275,42 @@ omq_status lwc_bwd_dw(cudaStream_t st, int64_t T, const bf16* dY, const bf16* Xh
   return lwc_bwd_fused_finish(st, la, lw.rowpart, ntn, lw.part_s, lw.part_d, P);
 }
 
+// Auxiliary stream of a device: work off the step's critical chain (the LWC forward of the later
+// weights, the weight-gradient products with their LWC backward) runs there, concurrently with
+// the caller's stream, and joins it through events.  One per device, created on first use; block
+// calls of one device that overlap on the GPU share it and must not be issued concurrently.
+struct Aux {
+  cudaStream_t s = nullptr;
+  cudaEvent_t ev[12] = {};
+  bool ready = false;
+};
+std::mutex g_aux_mu;
+Aux g_aux[64];
+
+omq_status aux_get(Aux** out) {
+  int dev = 0;
+  OMQ_REQUIRE(cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64, OMQ_ERR_CUDA);
+  std::lock_guard<std::mutex> lk(g_aux_mu);
+  Aux& a = g_aux[dev];
+  if (!a.ready) {
+    OMQ_REQUIRE(cudaStreamCreateWithFlags(&a.s, cudaStreamNonBlocking) == cudaSuccess, OMQ_ERR_CUDA);
+    for (auto& e : a.ev) OMQ_REQUIRE(cudaEventCreateWithFlags(&e, cudaEventDisableTiming) == cudaSuccess, OMQ_ERR_CUDA);
+    a.ready = true;
+  }
+  *out = &a;
+  return OMQ_OK;
+}
+
+// `to` waits for everything enqueued on `from` so far
+omq_status join(cudaStream_t from, cudaStream_t to, cudaEvent_t e) {
+  OMQ_REQUIRE(cudaEventRecord(e, from) == cudaSuccess, OMQ_ERR_CUDA);
+  OMQ_REQUIRE(cudaStreamWaitEvent(to, e, 0) == cudaSuccess, OMQ_ERR_CUDA);
+  return OMQ_OK;
+}
+
 struct Ctx {
   cudaStream_t st;
+  Aux* aux;
   omq_block_shape s;
   omq_qcfg cfg;
   const omq_block_weights* w;
@@ -296,17 +338,24 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
     OMQ_TRY(gqa_expand(st, th->do_, w.do_exp, (int)c.Hkv, (int)c.rep, (int)c.hd, 0));
     OMQ_TRY(gqa_expand(st, th->sa, w.sa_exp, (int)c.Hkv, (int)c.rep, (int)c.hd, 0));
   }
-  // ---- LET (Eq. 3) + LWC (Eq. 2) on every weight ------------------------------------------------
+  // ---- LET (Eq. 3) + LWC (Eq. 2) on every weight: q|k|v here, the others on the auxiliary stream
+  // while the attention half runs -------------------------------------------------------------------
+  cudaStream_t ax = c.aux->s;
+  cudaEvent_t* ev = c.aux->ev;
+  OMQ_TRY(join(st, ax, ev[0]));
   OMQ_TRY(lwc_fwd_launch(st, lwc_args(Wqkv, c.nqkv, c.d, cfg, c.let ? th->s1 : nullptr, c.let ? w.r_qkv : nullptr,
                                       th->gamma_qkv, th->beta_qkv, w.Wqkv_h, w.sq_qkv, c.let ? th->d1 : nullptr,
                                       c.let ? w.shift_qkv : nullptr, c.let ? w.B_qkv : nullptr)));
-  OMQ_TRY(lwc_fwd_launch(st, lwc_args(Wo, c.d, c.dq, cfg, c.let ? w.so_exp : nullptr, nullptr, th->gamma_o, th->beta_o,
+  OMQ_TRY(lwc_fwd_launch(ax, lwc_args(Wo, c.d, c.dq, cfg, c.let ? w.so_exp : nullptr, nullptr, th->gamma_o, th->beta_o,
                                       w.Wo_h, w.sq_o, c.let ? w.do_exp : nullptr, nullptr, c.let ? w.B_o : nullptr)));
-  OMQ_TRY(lwc_fwd_launch(st, lwc_args(Wgu, 2 * c.f, c.d, cfg, c.let ? th->s2 : nullptr, nullptr, th->gamma_gu,
+  OMQ_REQUIRE(cudaEventRecord(ev[1], ax) == cudaSuccess, OMQ_ERR_CUDA);
+  OMQ_TRY(lwc_fwd_launch(ax, lwc_args(Wgu, 2 * c.f, c.d, cfg, c.let ? th->s2 : nullptr, nullptr, th->gamma_gu,
                                       th->beta_gu, w.Wgu_h, w.sq_gu, c.let ? th->d2 : nullptr, nullptr,
                                       c.let ? w.B_gu : nullptr)));
-  OMQ_TRY(lwc_fwd_launch(st, lwc_args(Wd, c.d, c.f, cfg, nullptr, nullptr, th->gamma_d, th->beta_d, w.Wd_h, w.sq_d,
+  OMQ_REQUIRE(cudaEventRecord(ev[2], ax) == cudaSuccess, OMQ_ERR_CUDA);
+  OMQ_TRY(lwc_fwd_launch(ax, lwc_args(Wd, c.d, c.f, cfg, nullptr, nullptr, th->gamma_d, th->beta_d, w.Wd_h, w.sq_d,
                                       nullptr, nullptr, nullptr)));
+  OMQ_REQUIRE(cudaEventRecord(ev[3], ax) == cudaSuccess, OMQ_ERR_CUDA);
 
   // ---- attention half ---------------------------------------------------------------------------
   ActFwdArgs af{};
@@ -331,6 +380,7 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   ao.producer = AP_PLAIN; ao.X = w.O; ao.ldx = c.dq; ao.T = c.T; ao.C = c.dq; ao.Xq = w.O_h; ao.ldq = c.dq;
   ao.h = w.so.h; ao.z = w.so.z; ao.imax = w.so.imax; ao.imin = w.so.imin; ao.abits = cfg.abits; ao.eps = cfg.h_eps;
   OMQ_TRY(act_fwd_launch(st, ao));
+  OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[1], 0) == cudaSuccess, OMQ_ERR_CUDA);      // W_hat of o_proj
   OMQ_TRY(gemm_kk(st, c.T, c.d, c.dq, w.O_h, c.dq, w.Wo_h, c.dq, w.h1, nullptr, c.d, c.let ? w.B_o : nullptr, x, status));
 
   // ---- FFN half ---------------------------------------------------------------------------------
@@ -338,6 +388,7 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   ab.X = w.h1; ab.s = c.let ? th->s2 : nullptr; ab.delta = c.let ? th->d2 : nullptr; ab.rstd = w.rstd2; ab.Xq = w.b_h;
   ab.h = w.sb.h; ab.z = w.sb.z; ab.imax = w.sb.imax; ab.imin = w.sb.imin;
   OMQ_TRY(act_fwd_launch(st, ab));
+  OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[2], 0) == cudaSuccess, OMQ_ERR_CUDA);      // W_hat of gate|up
   OMQ_TRY(gemm_kk(st, c.T, 2 * c.f, c.d, w.b_h, c.d, w.Wgu_h, c.d, w.Ygu, nullptr, 2 * c.f, c.let ? w.B_gu : nullptr,
                   nullptr, status));
   ActFwdArgs am{};
@@ -345,6 +396,7 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   am.Xq = w.m_h; am.ldq = c.f; am.h = w.sm.h; am.z = w.sm.z; am.imax = w.sm.imax; am.imin = w.sm.imin;
   am.abits = cfg.abits; am.eps = cfg.h_eps;
   OMQ_TRY(act_fwd_launch(st, am));
+  OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[3], 0) == cudaSuccess, OMQ_ERR_CUDA);      // W_hat of down (joins)
   OMQ_TRY(gemm_kk(st, c.T, c.d, c.f, w.m_h, c.f, w.Wd_h, c.f, y, nullptr, c.d, nullptr, w.h1, status));
   return OMQ_OK;
 }
@@ -361,13 +413,20 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   const bf16* Wd = (const bf16*)c.w->wd;
   const int acc = cfg.accumulate;
 
+  // The weight-gradient products with their LWC backward run on the auxiliary stream (scratch
+  // part_aux, fallback dW), each started once its inputs exist; the caller's stream waits for
+  // them only where their outputs are accumulated further, and for all of them at the end.
+  cudaStream_t ax = c.aux->s;
+  cudaEvent_t* ev = c.aux->ev;
+
   // ---- loss (Eq. 1) ------------------------------------------------------------------------------
   OMQ_TRY(loss_launch(st, c.T * c.d, y, y_fp, loss, w.dy, w.dy_b, w.loss_part));
 
   // ---- down_proj ----------------------------------------------------------------------------------
+  OMQ_TRY(join(st, ax, ev[4]));
+  OMQ_TRY(lwc_bwd_dw(ax, c.T, w.dy_b, w.m_h, Wd, c.d, c.f, cfg, nullptr, nullptr, th->gamma_d, th->beta_d, w.sq_d,
+                     g->gamma_d, g->beta_d, nullptr, nullptr, nullptr, nullptr, 0, w.part_aux, w.dW, status));
   OMQ_TRY(gemm_dx(st, c.T, c.d, c.f, w.dy_b, w.Wd_h, w.dm, status));
-  OMQ_TRY(lwc_bwd_dw(st, c.T, w.dy_b, w.m_h, Wd, c.d, c.f, cfg, nullptr, nullptr, th->gamma_d, th->beta_d, w.sq_d,
-                     g->gamma_d, g->beta_d, nullptr, nullptr, nullptr, nullptr, 0, w.part, w.dW, status));
   ActBwdArgs bm{};
   bm.producer = AP_SWIGLU; bm.X = w.Ygu; bm.ldx = 2 * c.f; bm.U = w.Ygu + c.f; bm.ldu = 2 * c.f; bm.T = c.T; bm.C = c.f;
   bm.h = w.sm.h; bm.z = w.sm.z; bm.imax = w.sm.imax; bm.imin = w.sm.imin; bm.dXq = w.dm; bm.lddq = c.f;
@@ -376,12 +435,14 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   OMQ_TRY(act_bwd_launch(st, bm));
 
   // ---- gate / up ----------------------------------------------------------------------------------
-  OMQ_TRY(gemm_dx(st, c.T, 2 * c.f, c.d, w.dYgu_b, w.Wgu_h, w.db, status));
   if (c.let) OMQ_TRY(colsum_rows(st, w.dYgu, c.T, 2 * c.f, 2 * c.f, w.part, w.dB_gu, 1.f, 0));
-  OMQ_TRY(lwc_bwd_dw(st, c.T, w.dYgu_b, w.b_h, Wgu, 2 * c.f, c.d, cfg, c.let ? th->s2 : nullptr, nullptr,
+  OMQ_TRY(join(st, ax, ev[5]));
+  OMQ_TRY(lwc_bwd_dw(ax, c.T, w.dYgu_b, w.b_h, Wgu, 2 * c.f, c.d, cfg, c.let ? th->s2 : nullptr, nullptr,
                      th->gamma_gu, th->beta_gu, w.sq_gu, g->gamma_gu, g->beta_gu, nullptr,
-                     c.let ? w.dB_gu : nullptr, c.let ? g->s2 : nullptr, c.let ? g->d2 : nullptr, acc, w.part, w.dW,
-                     status));
+                     c.let ? w.dB_gu : nullptr, c.let ? g->s2 : nullptr, c.let ? g->d2 : nullptr, acc, w.part_aux,
+                     w.dW, status));
+  OMQ_REQUIRE(cudaEventRecord(ev[6], ax) == cudaSuccess, OMQ_ERR_CUDA);
+  OMQ_TRY(gemm_dx(st, c.T, 2 * c.f, c.d, w.dYgu_b, w.Wgu_h, w.db, status));
   ActBwdArgs bb{};
   bb.producer = AP_RMS_LET; bb.X = w.h1; bb.ldx = c.d; bb.s = c.let ? th->s2 : nullptr; bb.delta = c.let ? th->d2 : nullptr;
   bb.rstd = w.rstd2; bb.T = c.T; bb.C = c.d; bb.h = w.sb.h; bb.z = w.sb.z; bb.imax = w.sb.imax; bb.imin = w.sb.imin;
@@ -390,16 +451,19 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   bb.rows_per_cta = 4; bb.abits = cfg.abits; bb.eps = cfg.h_eps;
   OMQ_TRY(act_bwd_launch(st, bb));
   if (c.let) {
+    OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[6], 0) == cudaSuccess, OMQ_ERR_CUDA);   // LWC part of ds2, dd2
     OMQ_TRY(omq_colsum_partials(st, bb.part_s, (c.T + 3) / 4, c.d, g->s2, 1.f, 1));
     OMQ_TRY(omq_colsum_partials(st, bb.part_d, (c.T + 3) / 4, c.d, g->d2, 1.f, 1));
   }
 
   // ---- o_proj -------------------------------------------------------------------------------------
-  OMQ_TRY(gemm_dx(st, c.T, c.d, c.dq, w.dh1_b, w.Wo_h, w.dOh, status));
   if (c.let) OMQ_TRY(colsum_rows(st, w.dh1, c.T, c.d, c.d, w.part, w.dB_o, 1.f, 0));
-  OMQ_TRY(lwc_bwd_dw(st, c.T, w.dh1_b, w.O_h, Wo, c.d, c.dq, cfg, c.let ? w.so_exp : nullptr, nullptr, th->gamma_o,
+  OMQ_TRY(join(st, ax, ev[7]));
+  OMQ_TRY(lwc_bwd_dw(ax, c.T, w.dh1_b, w.O_h, Wo, c.d, c.dq, cfg, c.let ? w.so_exp : nullptr, nullptr, th->gamma_o,
                      th->beta_o, w.sq_o, g->gamma_o, g->beta_o, nullptr, c.let ? w.dB_o : nullptr,
-                     c.let ? w.vtmp0 : nullptr, c.let ? w.vtmp1 : nullptr, 0, w.part, w.dW, status));
+                     c.let ? w.vtmp0 : nullptr, c.let ? w.vtmp1 : nullptr, 0, w.part_aux, w.dW, status));
+  OMQ_REQUIRE(cudaEventRecord(ev[8], ax) == cudaSuccess, OMQ_ERR_CUDA);
+  OMQ_TRY(gemm_dx(st, c.T, c.d, c.dq, w.dh1_b, w.Wo_h, w.dOh, status));
   ActBwdArgs bo{};
   bo.producer = AP_PLAIN; bo.X = w.O; bo.ldx = c.dq; bo.T = c.T; bo.C = c.dq; bo.h = w.so.h; bo.z = w.so.z;
   bo.imax = w.so.imax; bo.imin = w.so.imin; bo.dXq = w.dOh; bo.lddq = c.dq; bo.dX = nullptr; bo.lddx = c.dq;
@@ -428,20 +492,24 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
     OMQ_TRY(omq_colsum_partials(st, qa.part_k, nsq, c.dkv, g->sa, 1.f, acc));
     OMQ_TRY(gqa_fold(st, w.vtmp2, g->sa, (int)c.Hkv, (int)c.rep, (int)c.hd, 1));
     // [v, out] pair: o_proj column-scale part (folded over the query heads), then v rows
+    OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[8], 0) == cudaSuccess, OMQ_ERR_CUDA);   // o_proj LWC backward
     OMQ_TRY(gqa_fold(st, w.vtmp0, g->so, (int)c.Hkv, (int)c.rep, (int)c.hd, acc));
     OMQ_TRY(gqa_fold(st, w.vtmp1, g->do_, (int)c.Hkv, (int)c.rep, (int)c.hd, acc));
   }
 
   // ---- q / k / v projections ---------------------------------------------------------------------------
   if (c.let) OMQ_TRY(colsum_rows(st, w.dYqkv, c.T, c.nqkv, c.nqkv, w.part, w.dB_qkv, 1.f, 0));
-  OMQ_TRY(lwc_bwd_dw(st, c.T, w.dYqkv_b, w.a_h, Wqkv, c.nqkv, c.d, cfg, c.let ? th->s1 : nullptr,
+  OMQ_TRY(join(st, ax, ev[9]));
+  OMQ_TRY(lwc_bwd_dw(ax, c.T, w.dYqkv_b, w.a_h, Wqkv, c.nqkv, c.d, cfg, c.let ? th->s1 : nullptr,
                      c.let ? w.r_qkv : nullptr, th->gamma_qkv, th->beta_qkv, w.sq_qkv, g->gamma_qkv, g->beta_qkv,
                      c.let ? w.dr_qkv : nullptr, c.let ? w.dB_qkv : nullptr, c.let ? g->s1 : nullptr,
-                     c.let ? g->d1 : nullptr, acc, w.part, w.dW, status));
+                     c.let ? g->d1 : nullptr, acc, w.part_aux, w.dW, status));
+  OMQ_REQUIRE(cudaEventRecord(ev[10], ax) == cudaSuccess, OMQ_ERR_CUDA);
   if (c.let) {
     const int64_t off = c.dq + c.dkv;
-    OMQ_TRY(let_vo_finalize(st, (int)c.dkv, th->so, w.dr_qkv + off, w.dB_qkv + off, w.B_qkv + off, g->so, g->do_, 1));
     OMQ_TRY(gemm_dx(st, c.T, c.nqkv, c.d, w.dYqkv_b, w.Wqkv_h, w.da, status));
+    OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[10], 0) == cudaSuccess, OMQ_ERR_CUDA);  // dr of the v rows, ds1, dd1
+    OMQ_TRY(let_vo_finalize(st, (int)c.dkv, th->so, w.dr_qkv + off, w.dB_qkv + off, w.B_qkv + off, g->so, g->do_, 1));
     ActBwdArgs ba{};
     ba.producer = AP_RMS_LET; ba.X = x; ba.ldx = c.d; ba.s = th->s1; ba.delta = th->d1; ba.rstd = w.rstd1; ba.T = c.T;
     ba.C = c.d; ba.h = w.sa.h; ba.z = w.sa.z; ba.imax = w.sa.imax; ba.imin = w.sa.imin; ba.dXq = w.da; ba.lddq = c.d;
@@ -451,6 +519,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
     OMQ_TRY(omq_colsum_partials(st, ba.part_s, (c.T + 3) / 4, c.d, g->s1, 1.f, 1));
     OMQ_TRY(omq_colsum_partials(st, ba.part_d, (c.T + 3) / 4, c.d, g->d1, 1.f, 1));
   }
+  OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[10], 0) == cudaSuccess, OMQ_ERR_CUDA);    // every auxiliary launch
   return OMQ_OK;
 }
 
@@ -473,6 +542,7 @@ omq_status make_ctx(Ctx& c, omq_stream_t stream, const omq_block_shape* shape, c
   OMQ_REQUIRE(workspace && ws_bytes >= dry.off, OMQ_ERR_WORKSPACE);
   OMQ_REQUIRE(omq_aligned16(workspace), OMQ_ERR_ALIGN);
   c.st = (cudaStream_t)stream;
+  OMQ_TRY(aux_get(&c.aux));
   c.s = *shape;
   c.cfg = *cfg;
   c.w = w;
