@@ -17,7 +17,8 @@
 // dV += P^T dO and dK += dS^T Q accumulated in tensor memory.  dQ kernel per (128-query block,
 // query head) recomputes S and dP for its keys and accumulates dQ += dS K.  D = rowsum(dO * O).
 //
-// Warp roles (192 threads): warp 0 TMA, warp 1 tensor memory + MMA issue, warps 2..5 compute.
+// Warp roles (320 threads): warp 0 TMA, warp 1 tensor memory + MMA issue, warps 2..9 compute
+// (two warps per tensor-memory lane quadrant, each taking half of a block's columns).
 // Every mbarrier wait is bounded; on expiry the status word gets OMQ_ERR_TIMEOUT and the kernel
 // winds down (frees its tensor memory and returns).
 #include "attn.cuh"
@@ -29,7 +30,7 @@ namespace {
 
 using namespace tc;
 
-constexpr int FA_THREADS = 192;
+constexpr int FA_THREADS = 320;            // warp 0 TMA, warp 1 MMA, warps 2..9 compute
 constexpr int HD = 128;                     // head dimension
 constexpr int ROW_BYTES = 128;              // one swizzle row: 64 bf16
 
@@ -92,7 +93,7 @@ struct FwdP {
 
 constexpr int F_TILE = 128 * ROW_BYTES * 2;           // 32 KB: [128 x 128] bf16
 constexpr int F_ATOM = 128 * ROW_BYTES;               // 16 KB
-constexpr int F_Q = 0, F_K = F_TILE, F_V = 3 * F_TILE, F_P = 5 * F_TILE, F_CTL = 6 * F_TILE;
+constexpr int F_Q = 0, F_K = F_TILE, F_V = 3 * F_TILE, F_P = 5 * F_TILE, F_ST = 6 * F_TILE, F_CTL = F_ST + 2048;
 constexpr int F_SMEM = F_CTL + 1024 + 1024;
 
 __global__ void __launch_bounds__(FA_THREADS, 1)
@@ -111,14 +112,15 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nqb = (p.T + 127) / 128;
-  const int qb = nqb - 1 - (int)blockIdx.x;          // longest rows first
-  const int h = blockIdx.y, g = h / p.rep;
+  // blocks launch in x-fastest order: every head's longest query block first
+  const int qb = nqb - 1 - (int)blockIdx.y;
+  const int h = blockIdx.x, g = h / p.rep;
   const int nkb = qb + 1;
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     for (int s = 0; s < 2; ++s) { mbar_init(&kv_full[s], 1); mbar_init(&kv_empty[s], 1); mbar_init(&s_full[s], 1); }
-    mbar_init(p_full, 4);
+    mbar_init(p_full, 8);
     mbar_init(o_done, 1);
     ctl->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -155,6 +157,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       for (int kk = 0; kk < 8; ++kk)
         umma_bf16(tmem + 128 * s, desc_k(sq, kk, F_ATOM), desc_k(sk + s * F_TILE, kk, F_ATOM), ID_S, kk > 0);
       umma_commit(&s_full[s]);
+      if (it < nkb) umma_commit(&kv_empty[s]);      // statistics pass: K is free once S is formed
       return true;
     };
     if (ok) ok = issue_s(0);
@@ -170,66 +173,86 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
           umma_bf16(tmem + 256, desc_k(sp, kk, F_ATOM), desc_mn(sv + (it & 1) * F_TILE, kk, F_ATOM), ID_O,
                     (j | kk) != 0);
         umma_commit(o_done);
+        umma_commit(&kv_empty[it & 1]);
       }
-      umma_commit(&kv_empty[it & 1]);
     }
   } else if (warp >= 2) {
-    const int q = warp & 3;
+    // eight compute warps: warps w and w+4 share TMEM lane quadrant w % 4 (rows), half 0 takes
+    // columns 0..63 of each block, half 1 columns 64..127
+    const int q = warp & 3, half = (warp - 2) >> 2;
     const int r = q * 32 + lane;                      // row of the block = TMEM lane
     const int row = qb * 128 + r;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     uint8_t* ptile = smem + F_P;
-    float m = -INFINITY, l = 0.f, inv_l = 0.f;
+    float* stat = reinterpret_cast<float*>(smem + F_ST);   // [2 halves][m | l][128 rows]
+    float m = -INFINITY, l = 0.f;
     bool ok = true;
-    for (int it = 0; it < nit; ++it) {
-      const int j = it < nkb ? it : it - nkb;
-      if (!(ok = waitw(&s_full[it & 1], (it >> 1) & 1, p.status, abort_flag))) break;
+    for (int j = 0; j < nkb; ++j) {                   // pass 1: running max and rescaled sum
+      if (!(ok = waitw(&s_full[j & 1], (j >> 1) & 1, p.status, abort_flag))) break;
       tc_fence_after();
-      const uint32_t sb = tmem + 128 * (it & 1) + lane_off;
+      const uint32_t sb = tmem + 128 * (j & 1) + lane_off;
       const bool diag = (j == qb);                    // keys beyond the row exist only here
-      if (it < nkb) {                                 // statistics: running max, rescaled sum
 #pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(sb + 32 * c, v);
-          if (diag) {
+      for (int c = 2 * half; c < 2 * half + 2; ++c) {
+        float v[32];
+        tmem_ld32(sb + 32 * c, v);
+        if (diag) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) if (32 * c + i > r) v[i] = -INFINITY;
-          }
-          float t[16];
+          for (int i = 0; i < 32; ++i) if (32 * c + i > r) v[i] = -INFINITY;
+        }
+        float t[16];
 #pragma unroll
-          for (int i = 0; i < 16; ++i) t[i] = fmaxf(v[i], v[i + 16]);
+        for (int i = 0; i < 16; ++i) t[i] = fmaxf(v[i], v[i + 16]);
 #pragma unroll
-          for (int w = 8; w >= 1; w >>= 1)
+        for (int w = 8; w >= 1; w >>= 1)
 #pragma unroll
-            for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
-          const float m_new = fmaxf(m, t[0] * p.c);
+          for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
+        const float m_new = fmaxf(m, t[0] * p.c);
+        if (m_new != -INFINITY) {                     // a chunk wholly above the diagonal adds nothing
           float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int i = 0; i < 32; ++i) s4[i & 3] += ex2(fmaf(v[i], p.c, -m_new));
           l = l * ex2(m - m_new) + ((s4[0] + s4[1]) + (s4[2] + s4[3]));
           m = m_new;
         }
-        if (it == nkb - 1) inv_l = 1.f / l;
-      } else {                                        // probabilities of this key block
-        if (j > 0) {                                  // the previous P V product has read P
-          if (!(ok = waitw(o_done, (j - 1) & 1, p.status, abort_flag))) break;
-          tc_fence_after();
-        }
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(sb + 32 * c, v);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = ex2(fmaf(v[i], p.c, -m)) * inv_l;
-          if (diag) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) if (32 * c + i > r) v[i] = 0.f;
-          }
-          st_row32(ptile, F_ATOM, r, 32 * c, v);
-        }
-        fence_async_smem();                           // P visible to the tensor core
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+    }
+    // combine the two halves of every row (each compute thread reaches this barrier exactly once)
+    stat[(half * 2 + 0) * 128 + r] = m;
+    stat[(half * 2 + 1) * 128 + r] = l;
+    asm volatile("bar.sync 1, 256;" ::: "memory");
+    const float mo = stat[((1 - half) * 2 + 0) * 128 + r], lo = stat[((1 - half) * 2 + 1) * 128 + r];
+    const float mt = fmaxf(m, mo);
+    const float lt = (m == -INFINITY ? 0.f : l * ex2(m - mt)) + (mo == -INFINITY ? 0.f : lo * ex2(mo - mt));
+    const float inv_l = 1.f / lt;
+    for (int j = 0; ok && j < nkb; ++j) {             // pass 2: probabilities, O += P V
+      const int it = nkb + j;
+      if (!(ok = waitw(&s_full[it & 1], (it >> 1) & 1, p.status, abort_flag))) break;
+      tc_fence_after();
+      const uint32_t sb = tmem + 128 * (it & 1) + lane_off;
+      const bool diag = (j == qb);
+      float v[2][32];
+#pragma unroll
+      for (int cc = 0; cc < 2; ++cc) {
+        const int c = 2 * half + cc;
+        tmem_ld32(sb + 32 * c, v[cc]);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[cc][i] = ex2(fmaf(v[cc][i], p.c, -mt)) * inv_l;
+        if (diag) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) if (32 * c + i > r) v[cc][i] = 0.f;
+        }
+      }
+      if (j > 0) {                                    // the previous P V product has read P
+        if (!(ok = waitw(o_done, (j - 1) & 1, p.status, abort_flag))) break;
+        tc_fence_after();
+      }
+#pragma unroll
+      for (int cc = 0; cc < 2; ++cc) st_row32(ptile, F_ATOM, r, 32 * (2 * half + cc), v[cc]);
+      fence_async_smem();                             // P visible to the tensor core
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(p_full);
@@ -237,7 +260,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     if (ok && waitw(o_done, (nkb - 1) & 1, p.status, abort_flag)) {
       tc_fence_after();
 #pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
+      for (int c = 2 * half; c < 2 * half + 2; ++c) {
         float o[32];
         tmem_ld32(tmem + 256 + lane_off + 32 * c, o);
         if (row < p.T) {
@@ -246,7 +269,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
           for (int i = 0; i < 8; ++i) dst[i] = make_float4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
         }
       }
-      if (row < p.T) p.lse[(int64_t)h * p.T + row] = m + log2f(l);
+      if (row < p.T && half == 0) p.lse[(int64_t)h * p.T + row] = mt + log2f(lt);
     }
   }
   tc_fence_before();
@@ -290,9 +313,9 @@ struct BwdP {
 constexpr int B_QATOM = 64 * ROW_BYTES;               // 8 KB: 64-row atom
 constexpr int B_QTILE = 2 * B_QATOM;                  // [64 x 128] bf16
 constexpr int B_K = 0, B_V = F_TILE, B_Q = 2 * F_TILE, B_DO = B_Q + 2 * B_QTILE;
-constexpr int B_PT = B_DO + 2 * B_QTILE;              // P^T [128 keys x 64 queries]: one 16 KB atom
-constexpr int B_DST = B_PT + F_ATOM;                  // dS^T, same shape
-constexpr int B_LD = B_DST + F_ATOM;                  // [2 stages][lse 64 | D 64] fp32
+constexpr int B_PT = B_DO + 2 * B_QTILE;              // P^T [128 keys x 64 queries]: 16 KB, two buffers
+constexpr int B_DST = B_PT + 2 * F_ATOM;              // dS^T, same shape, two buffers
+constexpr int B_LD = B_DST + 2 * F_ATOM;              // [2 stages][lse 64 | D 64] fp32
 constexpr int B_CTL = B_LD + 1024;
 constexpr int B_SMEM = B_CTL + 1024 + 1024;
 
@@ -308,11 +331,11 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
   uint64_t* qd_empty = &ctl->bar[3];     // [2]
   uint64_t* s_full = &ctl->bar[5];       // [2]: S^T and dP^T of a query block ready
   uint64_t* p_full = &ctl->bar[7];       // P^T, dS^T written
-  uint64_t* g_done = &ctl->bar[8];       // dV / dK products of a query block done (P^T, dS^T free)
+  uint64_t* g_done = &ctl->bar[8];       // [2]: dV / dK products that read P^T / dS^T buffer b done
   volatile int* abort_flag = &ctl->abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int kb = blockIdx.x, g = blockIdx.y;
+  const int kb = blockIdx.y, g = blockIdx.x;           // key block 0 (most queries) of every head first
   const int nq64 = (p.T + 63) / 64;
   const int i0 = 2 * kb;                              // first 64-query block with a visible key
   const int niq = nq64 > i0 ? nq64 - i0 : 0;
@@ -321,8 +344,9 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
   if (threadIdx.x == 0) {
     mbar_init(kv_full, 1);
     for (int s = 0; s < 2; ++s) { mbar_init(&qd_full[s], 1); mbar_init(&qd_empty[s], 1); mbar_init(&s_full[s], 1); }
-    mbar_init(p_full, 4);
-    mbar_init(g_done, 1);
+    mbar_init(p_full, 8);
+    mbar_init(&g_done[0], 1);
+    mbar_init(&g_done[1], 1);
     ctl->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -375,14 +399,16 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       tc_fence_after();
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk) {               // K = 64 queries
-        umma_bf16(tmem + 256, desc_k(spt, kk, F_ATOM), desc_mn(sd + s * B_QTILE, kk, B_QATOM), ID_G, (it | kk) != 0);
-        umma_bf16(tmem + 384, desc_k(sdst, kk, F_ATOM), desc_mn(sq + s * B_QTILE, kk, B_QATOM), ID_G, (it | kk) != 0);
+        umma_bf16(tmem + 256, desc_k(spt + s * F_ATOM, kk, F_ATOM), desc_mn(sd + s * B_QTILE, kk, B_QATOM), ID_G,
+                  (it | kk) != 0);
+        umma_bf16(tmem + 384, desc_k(sdst + s * F_ATOM, kk, F_ATOM), desc_mn(sq + s * B_QTILE, kk, B_QATOM), ID_G,
+                  (it | kk) != 0);
       }
-      umma_commit(g_done);
+      umma_commit(&g_done[s]);
       umma_commit(&qd_empty[s]);
     }
   } else if (warp >= 2) {
-    const int q = warp & 3;
+    const int q = warp & 3, half = (warp - 2) >> 2;   // half: which 32 of the 64 query columns
     const int r = q * 32 + lane;                      // key row of the block = TMEM lane
     const int key = kb * 128 + r;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
@@ -398,12 +424,8 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       const bool need_mask = qi * 64 < kb * 128 + 127 || qi * 64 + 64 > p.T;
       if (!(ok = waitw(&s_full[s], (it >> 1) & 1, p.status, abort_flag))) break;
       tc_fence_after();
-      if (it > 0) {                                   // previous dV / dK products done: P^T, dS^T free
-        if (!(ok = waitw(g_done, (it - 1) & 1, p.status, abort_flag))) break;
-        tc_fence_after();
-      }
-#pragma unroll 1
-      for (int c = 0; c < 2; ++c) {
+      {
+        const int c = half;
         float sv[32], dp[32];
         tmem_ld32(tmem + 64 * s + lane_off + 32 * c, sv);
         tmem_ld32(tmem + 128 + 64 * s + lane_off + 32 * c, dp);
@@ -420,18 +442,26 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
             if (key > qrow || qrow >= p.T) { sv[i] = 0.f; dp[i] = 0.f; }
           }
         }
-        st_row32(pt, F_ATOM, r, 32 * c, sv);
-        st_row32(dst, F_ATOM, r, 32 * c, dp);
+        // buffer s was last read by the dV / dK products of it-2: phase (it >> 1) - 1 of g_done[s]
+        // (each buffer's barrier is waited phase by phase, never more than one phase behind)
+        if (it >= 2 && !(ok = waitw(&g_done[s], ((it >> 1) - 1) & 1, p.status, abort_flag))) break;
+        tc_fence_after();
+        st_row32(pt + s * F_ATOM, F_ATOM, r, 32 * c, sv);
+        st_row32(dst + s * F_ATOM, F_ATOM, r, 32 * c, dp);
       }
       fence_async_smem();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(p_full);
     }
-    if (ok && nit > 0 && waitw(g_done, (nit - 1) & 1, p.status, abort_flag)) {
+    for (int b = 0; ok && b < 2 && b < nit; ++b) {  // the last use of each buffer
+      const int last = ((nit - 1 - b) & ~1) + b;
+      ok = waitw(&g_done[b], (last >> 1) & 1, p.status, abort_flag);
+    }
+    if (ok && nit > 0) {
       tc_fence_after();
 #pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
+      for (int c = 2 * half; c < 2 * half + 2; ++c) {
         float dv[32], dk[32];
         tmem_ld32(tmem + 256 + lane_off + 32 * c, dv);
         tmem_ld32(tmem + 384 + lane_off + 32 * c, dk);
@@ -446,7 +476,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
         }
       }
     } else if (ok && nit == 0 && key < p.T) {        // keys no query sees (cannot happen for T > 0)
-      for (int c = 0; c < HD; ++c) {
+      for (int c = 64 * half; c < 64 * half + 64; ++c) {
         p.dV[(int64_t)key * p.ldkv + g * HD + c] = 0.f;
         p.dK[(int64_t)key * p.ldkv + g * HD + c] = 0.f;
       }
@@ -479,13 +509,13 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
   uint64_t* kv_empty = &ctl->bar[3];     // [2]
   uint64_t* s_full = &ctl->bar[5];       // [2]: S and dP of a key block ready
   uint64_t* p_full = &ctl->bar[7];       // dS written
-  uint64_t* g_done = &ctl->bar[8];       // dQ product of a key block done
+  uint64_t* g_done = &ctl->bar[8];       // [2]: dQ product that read dS buffer b done
   volatile int* abort_flag = &ctl->abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nqb = (p.T + 127) / 128;
-  const int qb = nqb - 1 - (int)blockIdx.x;
-  const int h = blockIdx.y, g = h / p.rep;
+  const int qb = nqb - 1 - (int)blockIdx.y;           // longest query blocks of every head first
+  const int h = blockIdx.x, g = h / p.rep;
   const int nkb = 2 * qb + 2;                         // 64-key blocks up to the block's last query
 
   if (threadIdx.x == 0) {
@@ -493,8 +523,9 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     for (int s = 0; s < 2; ++s) {
       mbar_init(&kv_full[s], 1); mbar_init(&kv_empty[s], 1); mbar_init(&s_full[s], 1);
     }
-    mbar_init(p_full, 4);
-    mbar_init(g_done, 1);
+    mbar_init(p_full, 8);
+    mbar_init(&g_done[0], 1);
+    mbar_init(&g_done[1], 1);
     ctl->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -543,11 +574,11 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       for (int kk = 0; kk < 4; ++kk)               // K = 64 keys
         umma_bf16(tmem + 256, desc_k(sds + s * F_ATOM, kk, F_ATOM), desc_mn(sk + s * B_QTILE, kk, B_QATOM), ID_G,
                   (j | kk) != 0);
-      umma_commit(g_done);
+      umma_commit(&g_done[s]);
       umma_commit(&kv_empty[s]);
     }
   } else if (warp >= 2) {
-    const int q = warp & 3;
+    const int q = warp & 3, half = (warp - 2) >> 2;   // half: which 32 of the 64 key columns
     const int r = q * 32 + lane;
     const int row = qb * 128 + r;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
@@ -555,20 +586,17 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     const float Lr = row_ok ? p.lse[(int64_t)h * p.T + row] : 0.f;
     const float Dr = row_ok ? p.D[(int64_t)h * p.T + row] : 0.f;
     bool ok = true;
-    int waited = 0;                                   // g_done phases waited for so far
     for (int j = 0; j < nkb; ++j) {
       const int s = j & 1;
       if (!(ok = waitw(&s_full[s], (j >> 1) & 1, p.status, abort_flag))) break;
       tc_fence_after();
-      for (; waited <= j - 2; ++waited) {             // dQ product j-2 has read dS buffer s
-        if (!(ok = waitw(g_done, waited & 1, p.status, abort_flag))) break;
-      }
-      if (!ok) break;
+      // dS buffer s was last read by the dQ product of j-2: phase (j >> 1) - 1 of g_done[s]
+      if (j >= 2 && !(ok = waitw(&g_done[s], ((j >> 1) - 1) & 1, p.status, abort_flag))) break;
       tc_fence_after();
       const bool need_mask = j * 64 + 63 > qb * 128 || !row_ok;
       uint8_t* dst = smem + Q_DS + s * F_ATOM;
-#pragma unroll 1
-      for (int c = 0; c < 2; ++c) {
+      {
+        const int c = half;
         float sv[32], dp[32];
         tmem_ld32(tmem + 64 * s + lane_off + 32 * c, sv);
         tmem_ld32(tmem + 128 + 64 * s + lane_off + 32 * c, dp);
@@ -586,11 +614,14 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(p_full);
     }
-    for (; ok && waited < nkb; ++waited) ok = waitw(g_done, waited & 1, p.status, abort_flag);
+    for (int b = 0; ok && b < 2 && b < nkb; ++b) {  // the last use of each buffer
+      const int last = ((nkb - 1 - b) & ~1) + b;
+      ok = waitw(&g_done[b], (last >> 1) & 1, p.status, abort_flag);
+    }
     if (ok) {
       tc_fence_after();
 #pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
+      for (int c = 2 * half; c < 2 * half + 2; ++c) {
         float o[32];
         tmem_ld32(tmem + 256 + lane_off + 32 * c, o);
         if (row_ok) {
@@ -634,7 +665,7 @@ omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
   p.T = a.T; p.H = a.H; p.rep = a.H / a.Hkv;
   p.c = (float)(1.4426950408889634 / sqrt((double)HD));
   p.O = a.O; p.ldo = a.ldo; p.lse = a.lse; p.status = a.status;
-  dim3 grid((unsigned)((a.T + 127) / 128), (unsigned)a.H);
+  dim3 grid((unsigned)a.H, (unsigned)((a.T + 127) / 128));
   flash_fwd_kernel<<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
@@ -676,10 +707,10 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
   p.lse = a.lse; p.D = a.D;
   p.dQ = a.dQ; p.ldq = a.ldg; p.dK = a.dK; p.dV = a.dV; p.ldkv = a.ldgkv;
   p.status = a.status;
-  dim3 g1((unsigned)((a.T + 127) / 128), (unsigned)a.Hkv);
+  dim3 g1((unsigned)a.Hkv, (unsigned)((a.T + 127) / 128));
   flash_bwd_dkv_kernel<<<g1, FA_THREADS, B_SMEM, st>>>(tq64, tk, tv, tdo64, p);
   OMQ_LAUNCH_CHECK();
-  dim3 g2((unsigned)((a.T + 127) / 128), (unsigned)a.H);
+  dim3 g2((unsigned)a.H, (unsigned)((a.T + 127) / 128));
   flash_bwd_dq_kernel<<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
