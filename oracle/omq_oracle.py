@@ -48,6 +48,14 @@ notes of the repository):
      its transform into v_proj: W_v' = diag(1/s_o) W_v diag(s1),
      b_v' = (W_v delta1 - delta_o) / s_o, and the out_proj input is P V'
      (Sec. 3.3, last paragraph).
+ R16 LET initialisation (Sec. 4.1 "Training": scaling as in SmoothQuant, shifting as in
+     Outlier Suppression+), statistics of the full-precision block over the calibration
+     tokens: s = max(max|X|^alpha / max|W|^(1-alpha), 1e-5) per input channel (alpha 0.5,
+     max|W| over every output row of the weights sharing the input), delta = the channel mean
+     of X; [ln1, (q,k,v)] on the ln1 output, [ln2, (gate,up)] on the ln2 output; the [v, out]
+     pair the same recipe on the attention output O and W_o, per value channel (maxima and
+     mean taken over the query heads of its group); [Q, K]: s_a = sqrt(max|Q| / max|K|) per
+     channel after RoPE (max over the group's query heads), no shift.
  R15 where floating point decides an integer (a code, a zero point, a max/min
      index, the floor of h) the decision is taken in the precision of the
      kernels, IEEE single precision with one rounding per product, difference and
@@ -71,7 +79,7 @@ __all__ = [
     "lwc_fakequant_fwd", "lwc_fakequant_bwd", "act_quant_per_token", "act_quant_per_token_bwd",
     "let_apply", "block_loss", "qlinear_step", "BlockCfg", "block_forward", "block_step",
     "rmsnorm", "rope", "silu", "FrozenTape", "use_tape", "block_fp_forward", "sigmoid_fp32",
-    "THETA_NAMES_LWC", "THETA_NAMES_LET",
+    "THETA_NAMES_LWC", "THETA_NAMES_LET", "let_init",
 ]
 
 
@@ -748,3 +756,49 @@ def block_fp_forward(x, weights: Dict[str, object], cfg: BlockCfg) -> torch.Tens
     t = lambda v: torch.as_tensor(v).to(F64)
     with torch.no_grad():
         return block_forward(t(x), {k: t(v) for k, v in weights.items()}, {}, fp)
+
+
+# ----------------------------------------------------------------------------------------------
+# LET initialisation (R16)
+# ----------------------------------------------------------------------------------------------
+
+def let_init(xs, weights: Dict[str, object], cfg: BlockCfg, alpha: float = 0.5, floor: float = 1e-5):
+    """Initial LET parameters s1, d1, so, do, sa, s2, d2 from the calibration inputs `xs` (a list
+    of [T, d] block inputs) through the full-precision block (reading R16)."""
+    fp = dataclasses.replace(cfg, wbits=16, abits=16, let=False, mode="exact")
+    t = lambda v: torch.as_tensor(v).to(F64)
+    Wd = {k: t(v) for k, v in weights.items()}
+    H, Hkv, hd = cfg.n_heads, cfg.n_kv, cfg.head_dim
+    rep = H // Hkv
+    amax = {}
+    sums = {}
+    n = 0
+    with torch.no_grad():
+        for x in xs:
+            keep: Dict[str, torch.Tensor] = {}
+            block_forward(t(x), Wd, {}, fp, keep)
+            stats = dict(a=keep["a"], q=keep["q"], k=keep["k"], O=keep["O"], b=rmsnorm(keep["h1"], cfg.rms_eps))
+            for key, v in stats.items():
+                m = v.abs().max(0).values
+                amax[key] = m if key not in amax else torch.maximum(amax[key], m)
+                sm = v.sum(0)
+                sums[key] = sm if key not in sums else sums[key] + sm
+            n += x.shape[0]
+
+    def smooth(xmax, wmax):
+        return torch.clamp(xmax ** alpha / wmax ** (1.0 - alpha), min=floor)
+
+    def per_kv(v, op):                    # [H*hd] -> [Hkv*hd] over the query heads of each group
+        g = v.reshape(Hkv, rep, hd)
+        return (g.max(1).values if op == "max" else g.mean(1)).reshape(Hkv * hd)
+
+    wmax_qkv = torch.cat([Wd["wq"], Wd["wk"], Wd["wv"]]).abs().max(0).values
+    wmax_gu = torch.cat([Wd["wg"], Wd["wu"]]).abs().max(0).values
+    wmax_o = per_kv(Wd["wo"].abs().max(0).values, "max")
+    out = dict(
+        s1=smooth(amax["a"], wmax_qkv), d1=sums["a"] / n,
+        s2=smooth(amax["b"], wmax_gu), d2=sums["b"] / n,
+        so=smooth(per_kv(amax["O"], "max"), wmax_o), do=per_kv(sums["O"] / n, "mean"),
+        sa=torch.clamp(torch.sqrt(per_kv(amax["q"], "max") / amax["k"]), min=floor),
+    )
+    return out

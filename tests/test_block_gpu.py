@@ -40,6 +40,11 @@ SMALL = [
     I.BlockShape("w3a16_g128", T=256, d=256, n_heads=2, n_kv=2, ffn=512, wbits=3, abits=16, group=128, let=0),
     I.BlockShape("w2a16_g64", T=384, d=384, n_heads=3, n_kv=3, ffn=640, wbits=2, abits=16, group=64, let=0),
     I.BlockShape("w4a8_let_ragged", T=200, d=256, n_heads=2, n_kv=1, ffn=520, wbits=4, abits=8, group=0, let=1),
+    # the other weight-activation settings the paper reports: W6A6 (its main weight-activation results) and the asymmetric
+    # W4A6, W8A4 of its asymmetric-bits table (W4A8 above)
+    I.BlockShape("w4a6_let", T=256, d=256, n_heads=2, n_kv=2, ffn=512, wbits=4, abits=6, group=0, let=1),
+    I.BlockShape("w6a6_let", T=256, d=256, n_heads=2, n_kv=2, ffn=512, wbits=6, abits=6, group=0, let=1),
+    I.BlockShape("w8a4_let", T=256, d=256, n_heads=2, n_kv=2, ffn=512, wbits=8, abits=4, group=0, let=1),
 ]
 
 

@@ -486,3 +486,54 @@ def test_sigmoid_fp32_bitwise_and_error_bound():
     exact = 1.0 / (1.0 + np.exp(-np.clip(t.astype(np.float32).astype(np.float64), -80, 80)))
     ulp = np.spacing(exact.astype(np.float32)).astype(np.float64)
     assert np.max(np.abs(v.astype(np.float64) - exact) / ulp) <= 4.0
+
+
+@pytest.mark.parametrize("n_kv", [4, 2])
+def test_let_init_balances_ranges_and_centres(n_kv):
+    """LET initialisation (Sec. 4.1: scaling as SmoothQuant, shifting as OS+; reading R16),
+    checked through the properties that define it rather than its formula: with alpha = 0.5
+    every unclamped channel of X / s and of W * s has the same maximum magnitude (the difficulty
+    is split evenly between activation and weight), the shift makes the channel mean of X - delta
+    zero over the calibration tokens, and s_a equalises max|Q / s_a| and max|K * s_a| per channel
+    (maxima over the query heads of a kv group).  Statistics are recomputed here in numpy from
+    the full-precision block's intermediates."""
+    shape, W, _, _, cfg = _tiny_block(n_kv=n_kv)
+    xs = [I.make_block_input(shape, sample=i, weight_seed=1) for i in range(3)]
+    th = O.let_init(xs, W, cfg)
+    H, Hkv, hd = shape.n_heads, shape.n_kv, shape.head_dim
+    rep = H // Hkv
+    keeps = []
+    for x in xs:
+        k = {}
+        O.block_forward(torch.as_tensor(x, dtype=F64), _t(W), {},
+                        O.BlockCfg.from_shape(shape, wbits=16, abits=16, let=False, mode="exact"), k)
+        keeps.append({n: v.numpy() for n, v in k.items()})
+    rms = lambda v: v / np.sqrt((v * v).mean(1, keepdims=True) + shape.rms_eps)
+    A = np.concatenate([rms(np.asarray(x, np.float64)) for x in xs])
+    B = np.concatenate([rms(k["h1"]) for k in keeps])
+    Q = np.concatenate([k["q"] for k in keeps]).reshape(-1, Hkv, rep, hd)
+    K = np.concatenate([k["k"] for k in keeps]).reshape(-1, Hkv, hd)
+    Ob = np.concatenate([k["O"] for k in keeps]).reshape(-1, Hkv, rep, hd)
+    g = {n: v.numpy() for n, v in th.items()}
+
+    def balanced(Xa, Wa, s):
+        lhs = np.abs(Xa / s).max(0)
+        rhs = np.abs(Wa * s).max(0)
+        free = s > 1e-5 * (1 + 1e-9)
+        assert free.any()
+        assert np.allclose(lhs[free], rhs[free], rtol=1e-12, atol=0)
+
+    balanced(A, np.concatenate([W["wq"], W["wk"], W["wv"]]).astype(np.float64), g["s1"])
+    balanced(B, np.concatenate([W["wg"], W["wu"]]).astype(np.float64), g["s2"])
+    assert np.abs((A - g["d1"]).mean(0)).max() < 1e-12
+    assert np.abs((B - g["d2"]).mean(0)).max() < 1e-12
+    # [v, out]: per value channel, maxima over the group's heads of O / s_o and W_o * s_o columns
+    Wo = np.asarray(W["wo"], np.float64).reshape(-1, Hkv, rep, hd)
+    lhs = np.abs(Ob / g["so"].reshape(1, Hkv, 1, hd)).max(axis=(0, 2))
+    rhs = np.abs(Wo * g["so"].reshape(1, Hkv, 1, hd)).max(axis=(0, 2))
+    assert np.allclose(lhs, rhs, rtol=1e-12, atol=0)
+    assert np.abs((Ob - g["do"].reshape(1, Hkv, 1, hd)).mean(axis=(0, 2))).max() < 1e-12
+    # [Q, K]
+    qs = np.abs(Q / g["sa"].reshape(1, Hkv, 1, hd)).max(axis=(0, 2))
+    ks = np.abs(K * g["sa"].reshape(1, Hkv, hd)).max(0)
+    assert np.allclose(qs, ks, rtol=1e-12, atol=0)
