@@ -280,6 +280,39 @@ omq_status omq_attention_bwd(omq_stream_t stream, int32_t T, int32_t n_heads, in
                              const float* lse, const void* dO, int64_t lddo, float* D, float* dQ, int64_t ldg,
                              float* dK, float* dV, int64_t ldgkv, int32_t* dev_status);
 
+/* LET initialisation (Sec. 4.1 "Training": the channel-wise scaling is initialised as in
+ * SmoothQuant, the channel-wise shifting as in Outlier Suppression+).  Column statistics of the
+ * full-precision block over the calibration tokens, device fp32 vectors:
+ *   a_*  [d]            ln1 output (the [ln1, (q,k,v)] pair's X)
+ *   q_absmax [n_heads*hd], k_absmax [n_kv*hd]   Q and K after RoPE
+ *   o_*  [n_heads*hd]   attention output (the [v, out] pair's X)
+ *   b_*  [d]            ln2 output (the [ln2, (gate,up)] pair's X) */
+typedef struct omq_let_stats {
+  float* a_absmax; float* a_sum;
+  float* q_absmax; float* k_absmax;
+  float* o_absmax; float* o_sum;
+  float* b_absmax; float* b_sum;
+} omq_let_stats;
+
+/* Runs the full-precision block (no quantization, no LET) on one calibration input x [T, d] fp32
+ * and folds its column statistics into `stats` (first != 0 overwrites, else max / add).  The
+ * workspace is the one omq_block_workspace_size gives for `shape` with wbits = abits = 16. */
+omq_status omq_let_stats_accumulate(omq_stream_t stream, const omq_block_shape* shape,
+                                    const omq_block_weights* w, const float* x, const omq_let_stats* stats,
+                                    int32_t first, void* workspace, size_t ws_bytes, int32_t* dev_status);
+
+size_t omq_let_init_workspace_size(const omq_block_shape* shape);
+
+/* Initial LET parameters from the statistics of ntok calibration tokens, into theta's s1, d1,
+ * so, do_, sa, s2, d2:  s = max(max|X|^alpha / max|W|^(1-alpha), 1e-5) per input channel with
+ * max|W| over all output rows of the weights that share the input, delta = channel mean of X;
+ * the [v, out] pair per value channel with maxima / means over the query heads of its group;
+ * s_a = max(sqrt(max|Q| / max|K|), 1e-5), no Q/K shift.  alpha = 0.5 reproduces SmoothQuant's
+ * default migration strength. */
+omq_status omq_let_init(omq_stream_t stream, const omq_block_shape* shape, const omq_block_weights* w,
+                        const omq_let_stats* stats, int64_t ntok, float alpha, const omq_block_params* theta,
+                        void* workspace, size_t ws_bytes);
+
 /* AdamW update of one fp32 parameter vector (Sec. 4.1 "Training": AdamW, weight decay 0):
  * m = b1 m + (1-b1) g; v = b2 v + (1-b2) g^2; p -= lr * (m / (1-b1^t)) / (sqrt(v / (1-b2^t)) + eps)
  * - lr * wd * p.  step t >= 1. */

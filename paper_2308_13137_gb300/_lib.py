@@ -56,6 +56,13 @@ class omq_block_params(Structure):
     _fields_ = [(n, c_void_p) for n in PARAM_FIELDS]
 
 
+LET_STATS_FIELDS = ["a_absmax", "a_sum", "q_absmax", "k_absmax", "o_absmax", "o_sum", "b_absmax", "b_sum"]
+
+
+class omq_let_stats(Structure):
+    _fields_ = [(n, c_void_p) for n in LET_STATS_FIELDS]
+
+
 P, I64, I32, F32, SZ = c_void_p, c_int64, c_int32, c_float, c_size_t
 _SIGS = {
     "omq_let_apply": (I32, [P, I64, I64, I64, P, P, P, P, P, P, P, P, P]),
@@ -79,6 +86,9 @@ _SIGS = {
     "omq_attention_fwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P]),
     "omq_attention_bwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P, I64, P, P, I64, P, P, I64,
                                 P]),
+    "omq_let_stats_accumulate": (I32, [P, P, P, P, P, I32, P, SZ, P]),
+    "omq_let_init_workspace_size": (SZ, [P]),
+    "omq_let_init": (I32, [P, P, P, P, I64, F32, P, P, SZ]),
     "omq_adamw_update": (I32, [P, I64, P, P, P, P, F32, F32, F32, F32, F32, I32]),
     "omq_stream_status": (I32, [P, P, POINTER(c_int32)]),
     "omq_status_string": (c_char_p, [I32]),
@@ -227,6 +237,24 @@ def omq_attention_bwd(T, n_heads, n_kv, Q, ldq, K, V, ldkv, O, ldo, lse, dO, ldd
     check("omq_attention_bwd", lib().omq_attention_bwd(
         stream_handle(stream), T, n_heads, n_kv, ptr(Q), ldq, ptr(K), ptr(V), ldkv, ptr(O), ldo, ptr(lse), ptr(dO),
         lddo, ptr(D), ptr(dQ), ldg, ptr(dK), ptr(dV), ldgkv, ptr(dev_status)))
+
+
+def omq_let_stats_accumulate(shape, weights, x, stats, first, workspace, dev_status=None, stream=None):
+    ws_bytes = workspace.numel() * workspace.element_size()
+    check("omq_let_stats_accumulate", lib().omq_let_stats_accumulate(
+        stream_handle(stream), ctypes.byref(shape), ctypes.byref(weights), ptr(x), ctypes.byref(stats), int(first),
+        ptr(workspace), ws_bytes, ptr(dev_status)))
+
+
+def omq_let_init_workspace_size(shape) -> int:
+    return lib().omq_let_init_workspace_size(ctypes.byref(shape))
+
+
+def omq_let_init(shape, weights, stats, ntok, alpha, theta, workspace, stream=None):
+    ws_bytes = workspace.numel() * workspace.element_size()
+    check("omq_let_init", lib().omq_let_init(
+        stream_handle(stream), ctypes.byref(shape), ctypes.byref(weights), ctypes.byref(stats), ntok, alpha,
+        ctypes.byref(theta), ptr(workspace), ws_bytes))
 
 
 def omq_qlinear_fwd(T, Cin, Cout, X, W, B, s, delta, gamma_logit, beta_logit, Y, saved, cfg, stream=None):

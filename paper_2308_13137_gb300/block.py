@@ -117,6 +117,27 @@ class BlockState:
         cfg = _lib.make_cfg(16, 16, 0, 0, 1e-5, 0, self.status)
         return self.forward(x, y, stream, cfg)
 
+    def let_init(self, xs, alpha: float = 0.5, stream=None):
+        """Initial LET parameters (Sec. 4.1 "Training": SmoothQuant scaling, OS+ shifting) from
+        the calibration inputs xs (device [T, d] fp32 tensors), written into the LET views of the
+        parameter buffer; returns them as a dict of device tensors."""
+        torch = self.torch
+        if not self.let:
+            raise ValueError("LET is off for this block")
+        sh = self.shape
+        f32 = dict(dtype=torch.float32, device=self.device)
+        st = {n: torch.empty(sz, **f32) for n, sz in
+              dict(a_absmax=sh.d, a_sum=sh.d, q_absmax=sh.dq, k_absmax=sh.dkv, o_absmax=sh.dq, o_sum=sh.dq,
+                   b_absmax=sh.d, b_sum=sh.d).items()}
+        c_st = _lib.omq_let_stats(*[st[n].data_ptr() for n in _lib.LET_STATS_FIELDS])
+        for i, x in enumerate(xs):
+            _lib.omq_let_stats_accumulate(self.c_shape, self.c_w, x, c_st, i == 0, self.workspace, self.status,
+                                          stream)
+        ws = torch.empty(_lib.omq_let_init_workspace_size(self.c_shape), dtype=torch.uint8, device=self.device)
+        _lib.omq_let_init(self.c_shape, self.c_w, c_st, sum(int(x.shape[0]) for x in xs), alpha, self.c_theta, ws,
+                          stream)
+        return {k: self.theta[k] for k in LET_NAMES}
+
     def split_grads(self) -> Dict[str, np.ndarray]:
         """Gradients on the host, named like the oracle's parameters."""
         out = {}

@@ -703,3 +703,67 @@ omq_status omq_qlinear_bwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t 
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------------------------
+// LET initialisation: statistics of the full-precision block, then the initial parameters
+// ---------------------------------------------------------------------------------------------
+extern "C" omq_status omq_let_stats_accumulate(omq_stream_t stream, const omq_block_shape* shape,
+                                               const omq_block_weights* w, const float* x,
+                                               const omq_let_stats* stats, int32_t first, void* workspace,
+                                               size_t ws_bytes, int32_t* dev_status) {
+  OMQ_REQUIRE(x && stats && stats->a_absmax && stats->a_sum && stats->q_absmax && stats->k_absmax &&
+                  stats->o_absmax && stats->o_sum && stats->b_absmax && stats->b_sum,
+              OMQ_ERR_INVALID_ARG);
+  omq_qcfg fp{};
+  fp.wbits = 16; fp.abits = 16; fp.group = 0; fp.let = 0; fp.h_eps = 1e-5f; fp.accumulate = 0;
+  fp.dev_status = dev_status;
+  omq_block_params none{};
+  Ctx c;
+  OMQ_TRY(make_ctx(c, stream, shape, w, &none, workspace, ws_bytes, &fp, false));
+  BlockWS& ws = c.ws;
+  OMQ_TRY(block_fwd(c, x, ws.y));
+  const int f = first ? 1 : 0;
+  OMQ_TRY(let_colstats(c.st, x, c.T, c.d, c.d, ws.rstd1, stats->a_absmax, stats->a_sum, f));
+  OMQ_TRY(let_colstats_bf16(c.st, ws.Qh, c.T, c.dq, c.dq, stats->q_absmax, f));
+  OMQ_TRY(let_colstats_bf16(c.st, ws.Kh, c.T, c.dkv, c.dkv, stats->k_absmax, f));
+  OMQ_TRY(let_colstats(c.st, ws.O, c.T, c.dq, c.dq, nullptr, stats->o_absmax, stats->o_sum, f));
+  OMQ_TRY(let_colstats(c.st, ws.h1, c.T, c.d, c.d, ws.rstd2, stats->b_absmax, stats->b_sum, f));
+  return OMQ_OK;
+}
+
+extern "C" size_t omq_let_init_workspace_size(const omq_block_shape* shape) {
+  if (!shape) return 0;
+  const int64_t d = shape->d, dq = (int64_t)shape->n_heads * shape->head_dim;
+  return (size_t)(2 * d + dq) * sizeof(float) + 1024;
+}
+
+extern "C" omq_status omq_let_init(omq_stream_t stream, const omq_block_shape* shape, const omq_block_weights* w,
+                                   const omq_let_stats* stats, int64_t ntok, float alpha,
+                                   const omq_block_params* theta, void* workspace, size_t ws_bytes) {
+  OMQ_REQUIRE(shape && w && stats && theta && ntok > 0, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(alpha >= 0.f && alpha <= 1.f, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(theta->s1 && theta->d1 && theta->so && theta->do_ && theta->sa && theta->s2 && theta->d2,
+              OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(w->wqkv && w->wo && w->wgu, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(shape->n_heads > 0 && shape->n_kv > 0 && shape->n_heads % shape->n_kv == 0 && shape->head_dim > 0,
+              OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(workspace && ws_bytes >= omq_let_init_workspace_size(shape), OMQ_ERR_WORKSPACE);
+  cudaStream_t st = (cudaStream_t)stream;
+  const int64_t d = shape->d, hd = shape->head_dim, dq = shape->n_heads * hd, dkv = shape->n_kv * hd;
+  const int64_t f = shape->ffn, nqkv = dq + 2 * dkv;
+  float* wm_qkv = (float*)workspace;
+  float* wm_gu = wm_qkv + d;
+  float* wm_o = wm_gu + d;
+  const float floor = 1e-5f;
+  OMQ_TRY(let_weight_colmax(st, (const __nv_bfloat16*)w->wqkv, nqkv, d, wm_qkv, 1));
+  OMQ_TRY(let_weight_colmax(st, (const __nv_bfloat16*)w->wgu, 2 * f, d, wm_gu, 1));
+  OMQ_TRY(let_weight_colmax(st, (const __nv_bfloat16*)w->wo, d, dq, wm_o, 1));
+  OMQ_TRY(let_smooth_pair(st, d, stats->a_absmax, stats->a_sum, wm_qkv, (double)ntok, alpha, floor, theta->s1,
+                          theta->d1));
+  OMQ_TRY(let_smooth_pair(st, d, stats->b_absmax, stats->b_sum, wm_gu, (double)ntok, alpha, floor, theta->s2,
+                          theta->d2));
+  OMQ_TRY(let_kv_pairs(st, shape->n_kv, shape->n_heads / shape->n_kv, (int)hd, stats->o_absmax, stats->o_sum, wm_o,
+                       stats->q_absmax, stats->k_absmax, (double)ntok, alpha, floor, theta->so, theta->do_, theta->sa));
+  (void)dkv;
+  return OMQ_OK;
+}

@@ -93,3 +93,19 @@ omq_status vec_copy(cudaStream_t st, float* dst, const float* src, int64_t n);
 omq_status gqa_expand(cudaStream_t st, const float* src, float* dst, int n_kv, int rep, int hd, int op);
 // dst[c] (+)= sum over the rep query heads of src[h*hd + j] for c = kv*hd + j
 omq_status gqa_fold(cudaStream_t st, const float* src, float* dst, int n_kv, int rep, int hd, int accumulate);
+
+// ---- LET initialisation (letinit.cu) -------------------------------------------------------------
+// column max|X| and sum of X over n rows (X optionally scaled per row by rstd); first: overwrite
+omq_status let_colstats(cudaStream_t st, const float* X, int64_t n, int64_t C, int64_t ldx, const float* rstd,
+                        float* absmax, float* sum, int first);
+omq_status let_colstats_bf16(cudaStream_t st, const __nv_bfloat16* X, int64_t n, int64_t C, int64_t ldx,
+                             float* absmax, int first);
+// max over output rows of |W[:, c]|
+omq_status let_weight_colmax(cudaStream_t st, const __nv_bfloat16* W, int64_t Cout, int64_t Cin, float* out, int first);
+// s = max(xmax^alpha / wmax^(1-alpha), floor), delta = xsum / ntok
+omq_status let_smooth_pair(cudaStream_t st, int64_t C, const float* xmax, const float* xsum, const float* wmax,
+                           double ntok, float alpha, float floor, float* s, float* delta);
+// [v, out] and [Q, K] pairs per value channel (query-head maxima / means over each kv group)
+omq_status let_kv_pairs(cudaStream_t st, int Hkv, int rep, int hd, const float* omax, const float* osum,
+                        const float* womax, const float* qmax, const float* kmax, double ntok, float alpha, float floor,
+                        float* so, float* do_, float* sa);
