@@ -56,6 +56,14 @@ notes of the repository):
      pair the same recipe on the attention output O and W_o, per value channel (maxima and
      mean taken over the query heads of its group); [Q, K]: s_a = sqrt(max|Q| / max|K|) per
      channel after RoPE (max over the group's query heads), no shift.
+ R17 fold & pack (Algorithm 1, after training: transform with the learned parameters, then
+     quantize): the scales and shifts of the [ln, linears] pairs are absorbed into the
+     RMSNorm as a gain 1/s and a bias -delta/s (the block's RMSNorm has unit gain and no bias
+     of its own), the linear biases B~ of Eq. 3 and the [v, out] pair's row scale stay in the
+     quantized weights and biases (R14), s_a stays a per-channel scale of the Q / K cache
+     (it sits after RoPE, R9, so it cannot be folded into the projection weights).  Weight
+     codes are packed per output row as a little-endian bit stream: code i occupies bits
+     [N i, N i + N) of the row.
  R15 where floating point decides an integer (a code, a zero point, a max/min
      index, the floor of h) the decision is taken in the precision of the
      kernels, IEEE single precision with one rounding per product, difference and
@@ -79,7 +87,8 @@ __all__ = [
     "lwc_fakequant_fwd", "lwc_fakequant_bwd", "act_quant_per_token", "act_quant_per_token_bwd",
     "let_apply", "block_loss", "qlinear_step", "BlockCfg", "block_forward", "block_step",
     "rmsnorm", "rope", "silu", "FrozenTape", "use_tape", "block_fp_forward", "sigmoid_fp32",
-    "THETA_NAMES_LWC", "THETA_NAMES_LET", "let_init",
+    "THETA_NAMES_LWC", "THETA_NAMES_LET", "let_init", "pack_codes", "unpack_codes", "block_fold_pack",
+    "folded_forward",
 ]
 
 
@@ -802,3 +811,118 @@ def let_init(xs, weights: Dict[str, object], cfg: BlockCfg, alpha: float = 0.5, 
         sa=torch.clamp(torch.sqrt(per_kv(amax["q"], "max") / amax["k"]), min=floor),
     )
     return out
+
+
+# ----------------------------------------------------------------------------------------------
+# fold & pack (R17)
+# ----------------------------------------------------------------------------------------------
+
+def pack_codes(codes: torch.Tensor, nbits: int) -> torch.Tensor:
+    """Integer codes [Cout, Cin] (0 <= c < 2^nbits) -> uint8 [Cout, Cin * nbits / 8]: code i of a
+    row at bits [nbits i, nbits i + nbits) of the row's little-endian bit stream."""
+    cout, cin = codes.shape
+    assert (cin * nbits) % 8 == 0
+    bits = ((codes.to(torch.int64)[..., None] >> torch.arange(nbits)) & 1).reshape(cout, cin * nbits)
+    bytes_ = bits.reshape(cout, -1, 8)
+    return (bytes_ << torch.arange(8)).sum(-1).to(torch.uint8)
+
+
+def unpack_codes(packed: torch.Tensor, nbits: int, cin: int) -> torch.Tensor:
+    cout = packed.shape[0]
+    bits = ((packed.to(torch.int64)[..., None] >> torch.arange(8)) & 1).reshape(cout, -1)[:, :cin * nbits]
+    return (bits.reshape(cout, cin, nbits) << torch.arange(nbits)).sum(-1)
+
+
+def block_fold_pack(weights: Dict[str, object], theta: Dict[str, object], cfg: BlockCfg) -> Dict[str, torch.Tensor]:
+    """The block after calibration, with its learned parameters folded in and its weights
+    quantized (Algorithm 1, last steps; reading R17): per linear (q|k|v stacked, o, gate|up,
+    down) packed codes, h and z per group; biases of q|k|v, o, gate|up; the two RMSNorm gains
+    and biases; s_a."""
+    t = lambda v: torch.as_tensor(v).to(F64)
+    Wd = {k: t(v) for k, v in weights.items()}
+    th = {k: t(v) for k, v in theta.items()}
+    H, Hkv, hd = cfg.n_heads, cfg.n_kv, cfg.head_dim
+    decide = _decide(cfg)
+    out: Dict[str, torch.Tensor] = {}
+    let = cfg.let
+    with torch.no_grad():
+        if let:
+            s1, d1, so, do_, s2, d2 = th["s1"], th["d1"], th["so"], th["do"], th["s2"], th["d2"]
+            r_o = (1.0 / so.to(torch.float32)).to(F64)
+            rows = torch.cat([torch.ones(H * hd + Hkv * hd, dtype=F64), r_o])
+            so_e, do_e = _expand_kv(so, cfg), _expand_kv(do_, cfg)
+        lin = dict(
+            qkv=(torch.cat([Wd["wq"], Wd["wk"], Wd["wv"]]), ("q", "k", "v"), s1 if let else None, rows if let else None),
+            o=(Wd["wo"], ("o",), so_e if let else None, None),
+            gu=(torch.cat([Wd["wg"], Wd["wu"]]), ("g", "u"), s2 if let else None, None),
+            d=(Wd["wd"], ("d",), None, None))
+        for name, (Wl, parts, s, r) in lin.items():
+            gl = torch.cat([th["gamma_" + p_] for p_ in parts])
+            bl = torch.cat([th["beta_" + p_] for p_ in parts])
+            f = lwc_fakequant_fwd(Wl, gl, bl, cfg.wbits, cfg.group, s=s, eps=cfg.h_eps, row_scale=r, decide=decide)
+            out["codes_" + name] = pack_codes(f["codes"], cfg.wbits)
+            out["h_" + name] = f["h"]
+            out["z_" + name] = f["z"]
+        if let:
+            wv_b = (Wd["wv"] @ d1 - do_) / so
+            out["b_qkv"] = torch.cat([Wd["wq"] @ d1, Wd["wk"] @ d1, wv_b])
+            out["b_o"] = Wd["wo"] @ do_e
+            out["b_gu"] = torch.cat([Wd["wg"], Wd["wu"]]) @ d2
+            out["ln1_gain"], out["ln1_bias"] = 1.0 / s1, -d1 / s1
+            out["ln2_gain"], out["ln2_bias"] = 1.0 / s2, -d2 / s2
+            out["sa"] = th["sa"]
+    return out
+
+
+def folded_forward(folded: Dict[str, torch.Tensor], x, cfg: BlockCfg) -> torch.Tensor:
+    """The deployed block built only from block_fold_pack's output: dequantized weights
+    (code - z) h, folded RMSNorm gains and biases, biases, s_a on Q / K; activations quantized
+    per token as in the calibrated block."""
+    H, Hkv, hd = cfg.n_heads, cfg.n_kv, cfg.head_dim
+    mode = cfg.mode
+    T = x.shape[0]
+    let = cfg.let
+
+    def deq(name, cout, cin):
+        c = unpack_codes(folded["codes_" + name], cfg.wbits, cin).to(F64)
+        g = cin if cfg.group == 0 else cfg.group
+        h = folded["h_" + name].to(F64).repeat_interleave(g, 1)
+        z = folded["z_" + name].to(F64).repeat_interleave(g, 1)
+        return (c - z) * h
+
+    d, f = cfg.d, cfg.ffn
+    dq, dkv = H * hd, Hkv * hd
+    x = torch.as_tensor(x).to(F64)
+    with torch.no_grad():
+        a = rmsnorm(x, cfg.rms_eps)
+        if let:
+            a = a * folded["ln1_gain"] + folded["ln1_bias"]
+        y = _mm(_qa(a, cfg), deq("qkv", dq + 2 * dkv, d), mode)
+        if let:
+            y = y + folded["b_qkv"]
+        q, k, v = y[:, :dq], y[:, dq:dq + dkv], y[:, dq + dkv:]
+        q = rope(q, H, hd, cfg.rope_theta)
+        k = rope(k, Hkv, hd, cfg.rope_theta)
+        if let:
+            q = q / _expand_kv(folded["sa"], cfg)
+            k = k * folded["sa"]
+        qh, kh, vh = _qa(q, cfg), _qa(k, cfg), _qa(v, cfg)
+        rep = H // Hkv
+        Qh = qh.reshape(T, H, hd).transpose(0, 1)
+        Kh = kh.reshape(T, Hkv, hd).transpose(0, 1).repeat_interleave(rep, 0)
+        Vh = vh.reshape(T, Hkv, hd).transpose(0, 1).repeat_interleave(rep, 0)
+        S = _mm(Qh, Kh, mode) / math.sqrt(hd)
+        S = S.masked_fill(~torch.ones(T, T, dtype=torch.bool).tril(), float("-inf"))
+        O = _mm(torch.softmax(S, dim=-1), Vh.transpose(-1, -2), mode).transpose(0, 1).reshape(T, dq)
+        o = _mm(_qa(O, cfg), deq("o", d, dq), mode)
+        if let:
+            o = o + folded["b_o"]
+        h1 = x + o
+        b = rmsnorm(h1, cfg.rms_eps)
+        if let:
+            b = b * folded["ln2_gain"] + folded["ln2_bias"]
+        gu = _mm(_qa(b, cfg), deq("gu", 2 * f, d), mode)
+        if let:
+            gu = gu + folded["b_gu"]
+        m = silu(gu[:, :f]) * gu[:, f:]
+        return h1 + _mm(_qa(m, cfg), deq("d", d, f), mode)

@@ -537,3 +537,40 @@ def test_let_init_balances_ranges_and_centres(n_kv):
     qs = np.abs(Q / g["sa"].reshape(1, Hkv, 1, hd)).max(axis=(0, 2))
     ks = np.abs(K * g["sa"].reshape(1, Hkv, hd)).max(0)
     assert np.allclose(qs, ks, rtol=1e-12, atol=0)
+
+
+def test_pack_codes_bit_layout_by_hand():
+    """Packed codes (reading R17): code i of a row occupies bits [N i, N i + N) of the row's
+    little-endian bit stream.  Hand-packed bytes for N = 4, 2 and 3."""
+    c4 = torch.tensor([[1, 2, 3, 4, 15, 0, 7, 8]])
+    assert O.pack_codes(c4, 4).tolist() == [[0x21, 0x43, 0x0F, 0x87]]
+    c2 = torch.tensor([[1, 2, 3, 0, 3, 3, 0, 1]])
+    assert O.pack_codes(c2, 2).tolist() == [[0b00111001, 0b01001111]]
+    # N = 3: stream 001 010 011 100 101 110 111 000 (LSB first) -> bytes 0xD1, 0x58, 0x1F
+    c3 = torch.tensor([[1, 2, 3, 4, 5, 6, 7, 0]])
+    bits = [(v >> b) & 1 for v in [1, 2, 3, 4, 5, 6, 7, 0] for b in range(3)]
+    hand = [sum(bits[8 * k + j] << j for j in range(8)) for k in range(3)]
+    assert hand == [0xD1, 0x58, 0x1F]
+    assert O.pack_codes(c3, 3).tolist() == [hand]
+    g = torch.Generator().manual_seed(5)
+    for n in (2, 3, 4, 8):
+        c = torch.randint(0, 2 ** n, (6, 64), generator=g)
+        assert torch.equal(O.unpack_codes(O.pack_codes(c, n), n, 64), c)
+
+
+@pytest.mark.parametrize("let,abits,wbits,group,n_kv", [(True, 4, 4, 0, 4), (True, 4, 4, 0, 2),
+                                                         (False, 16, 3, 8, 4)])
+def test_folded_block_equals_calibrated_block(let, abits, wbits, group, n_kv):
+    """Fold & pack (Algorithm 1's transform-then-quantize; reading R17): the deployed block built
+    only from the packed codes, h, z, biases, folded RMSNorm gains / biases and s_a computes the
+    same output as the calibrated block with its LET and LWC parameters (fp64, decisions in fp64)."""
+    shape, W, x, th, cfg = _tiny_block(let=let, abits=abits, wbits=wbits, group=group, n_kv=n_kv)
+    c = O.BlockCfg.from_shape(shape, mode="exact")
+    folded = O.block_fold_pack(W, th, c)
+    y_fold = O.folded_forward(folded, x, c)
+    y_ref = O.block_forward(torch.as_tensor(x, dtype=F64), _t(W), _t(th), c)
+    # the packed v_proj rows are divided by s_o through the single-precision reciprocal the
+    # kernels use (R14, R15), the calibrated block divides exactly: ~1e-8 relative on h of those rows
+    assert _rel(y_fold, y_ref) < (1e-8 if let else 1e-12)
+    assert folded["codes_qkv"].dtype == torch.uint8
+    assert folded["codes_qkv"].shape[1] * 8 == shape.d * wbits
