@@ -313,6 +313,29 @@ omq_status omq_let_init(omq_stream_t stream, const omq_block_shape* shape, const
                         const omq_let_stats* stats, int64_t ntok, float alpha, const omq_block_params* theta,
                         void* workspace, size_t ws_bytes);
 
+/* Fold & pack (Algorithm 1's last steps: transform the block with its learned parameters, then
+ * quantize).  Per linear (q|k|v stacked, o, gate|up stacked, down): the integer codes of Eq. 2,
+ * packed per output row as a little-endian bit stream (code i at bits [N i, N i + N), N = wbits,
+ * Cin * N / 8 bytes per row), and h, z per group [Cout, Cin / group] (group 0: one per row).
+ * With LET on, the LET parameters are absorbed: the linear biases B~ of Eq. 3 (the [v, out]
+ * pair's shift and row scale inside q|k|v's v rows and o), the two RMSNorm layers as a gain 1/s and
+ * a bias -delta/s (the block's RMSNorm has unit gain, no bias), and s_a, which scales Q and K after
+ * RoPE and stays a runtime per-channel factor.  Device pointers, caller-owned; LET-only outputs
+ * may be NULL when LET is off. */
+typedef struct omq_block_packed {
+  uint8_t* codes_qkv; uint8_t* codes_o; uint8_t* codes_gu; uint8_t* codes_d;
+  float* h_qkv; int32_t* z_qkv; float* h_o; int32_t* z_o;
+  float* h_gu; int32_t* z_gu; float* h_d; int32_t* z_d;
+  float* b_qkv; float* b_o; float* b_gu;          /* [dq+2dkv], [d], [2 ffn] */
+  float* ln1_gain; float* ln1_bias; float* ln2_gain; float* ln2_bias;   /* [d] */
+  float* sa;                                      /* [n_kv*hd] */
+} omq_block_packed;
+
+size_t omq_block_pack_workspace_size(const omq_block_shape* shape, const omq_qcfg* cfg);
+omq_status omq_block_fold_pack(omq_stream_t stream, const omq_block_shape* shape, const omq_block_weights* w,
+                               const omq_block_params* theta, const omq_qcfg* cfg, const omq_block_packed* out,
+                               void* workspace, size_t ws_bytes);
+
 /* AdamW update of one fp32 parameter vector (Sec. 4.1 "Training": AdamW, weight decay 0):
  * m = b1 m + (1-b1) g; v = b2 v + (1-b2) g^2; p -= lr * (m / (1-b1^t)) / (sqrt(v / (1-b2^t)) + eps)
  * - lr * wd * p.  step t >= 1. */

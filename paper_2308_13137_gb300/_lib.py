@@ -56,6 +56,14 @@ class omq_block_params(Structure):
     _fields_ = [(n, c_void_p) for n in PARAM_FIELDS]
 
 
+PACKED_FIELDS = ["codes_qkv", "codes_o", "codes_gu", "codes_d", "h_qkv", "z_qkv", "h_o", "z_o", "h_gu", "z_gu",
+                 "h_d", "z_d", "b_qkv", "b_o", "b_gu", "ln1_gain", "ln1_bias", "ln2_gain", "ln2_bias", "sa"]
+
+
+class omq_block_packed(Structure):
+    _fields_ = [(n, c_void_p) for n in PACKED_FIELDS]
+
+
 LET_STATS_FIELDS = ["a_absmax", "a_sum", "q_absmax", "k_absmax", "o_absmax", "o_sum", "b_absmax", "b_sum"]
 
 
@@ -86,6 +94,8 @@ _SIGS = {
     "omq_attention_fwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P]),
     "omq_attention_bwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P, I64, P, P, I64, P, P, I64,
                                 P]),
+    "omq_block_pack_workspace_size": (SZ, [P, P]),
+    "omq_block_fold_pack": (I32, [P, P, P, P, P, P, P, SZ]),
     "omq_let_stats_accumulate": (I32, [P, P, P, P, P, I32, P, SZ, P]),
     "omq_let_init_workspace_size": (SZ, [P]),
     "omq_let_init": (I32, [P, P, P, P, I64, F32, P, P, SZ]),
@@ -237,6 +247,17 @@ def omq_attention_bwd(T, n_heads, n_kv, Q, ldq, K, V, ldkv, O, ldo, lse, dO, ldd
     check("omq_attention_bwd", lib().omq_attention_bwd(
         stream_handle(stream), T, n_heads, n_kv, ptr(Q), ldq, ptr(K), ptr(V), ldkv, ptr(O), ldo, ptr(lse), ptr(dO),
         lddo, ptr(D), ptr(dQ), ldg, ptr(dK), ptr(dV), ldgkv, ptr(dev_status)))
+
+
+def omq_block_pack_workspace_size(shape, cfg) -> int:
+    return lib().omq_block_pack_workspace_size(ctypes.byref(shape), ctypes.byref(cfg))
+
+
+def omq_block_fold_pack(shape, weights, theta, cfg, out, workspace, stream=None):
+    ws_bytes = workspace.numel() * workspace.element_size()
+    check("omq_block_fold_pack", lib().omq_block_fold_pack(
+        stream_handle(stream), ctypes.byref(shape), ctypes.byref(weights), ctypes.byref(theta), ctypes.byref(cfg),
+        ctypes.byref(out), ptr(workspace), ws_bytes))
 
 
 def omq_let_stats_accumulate(shape, weights, x, stats, first, workspace, dev_status=None, stream=None):

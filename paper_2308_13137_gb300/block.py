@@ -138,6 +138,31 @@ class BlockState:
                           stream)
         return {k: self.theta[k] for k in LET_NAMES}
 
+    def fold_pack(self, stream=None):
+        """The calibrated block with its LET parameters folded in and its weights quantized and
+        packed (Algorithm 1, after training): device tensors named as in omq_block_packed."""
+        torch = self.torch
+        sh = self.shape
+        dev = self.device
+        nq = sh.dq + 2 * sh.dkv
+        ng = lambda cin: cin // (self.group if self.group else cin)
+        lins = dict(qkv=(nq, sh.d), o=(sh.d, sh.dq), gu=(2 * sh.ffn, sh.d), d=(sh.d, sh.ffn))
+        out = {}
+        for k, (co, ci) in lins.items():
+            out["codes_" + k] = torch.empty(co, ci * self.wbits // 8, dtype=torch.uint8, device=dev)
+            out["h_" + k] = torch.empty(co, ng(ci), dtype=torch.float32, device=dev)
+            out["z_" + k] = torch.empty(co, ng(ci), dtype=torch.int32, device=dev)
+        if self.let:
+            f32 = dict(dtype=torch.float32, device=dev)
+            out.update(b_qkv=torch.empty(nq, **f32), b_o=torch.empty(sh.d, **f32), b_gu=torch.empty(2 * sh.ffn, **f32),
+                       ln1_gain=torch.empty(sh.d, **f32), ln1_bias=torch.empty(sh.d, **f32),
+                       ln2_gain=torch.empty(sh.d, **f32), ln2_bias=torch.empty(sh.d, **f32),
+                       sa=torch.empty(sh.dkv, **f32))
+        c_out = _lib.omq_block_packed(*[(out[n].data_ptr() if n in out else None) for n in _lib.PACKED_FIELDS])
+        ws = torch.empty(_lib.omq_block_pack_workspace_size(self.c_shape, self.cfg), dtype=torch.uint8, device=dev)
+        _lib.omq_block_fold_pack(self.c_shape, self.c_w, self.c_theta, self.cfg, c_out, ws, stream)
+        return out
+
     def split_grads(self) -> Dict[str, np.ndarray]:
         """Gradients on the host, named like the oracle's parameters."""
         out = {}

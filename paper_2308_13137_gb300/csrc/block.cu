@@ -767,3 +767,97 @@ extern "C" omq_status omq_let_init(omq_stream_t stream, const omq_block_shape* s
   (void)dkv;
   return OMQ_OK;
 }
+
+// ---------------------------------------------------------------------------------------------
+// fold & pack
+// ---------------------------------------------------------------------------------------------
+namespace {
+struct PackWS {
+  uint8_t* codes; float* r_qkv; float* shift_qkv; float* so_exp; float* do_exp; int32_t* imax; int32_t* imin;
+};
+PackWS carve_pack(Carve& c, const omq_block_shape& s) {
+  const int64_t d = s.d, hd = s.head_dim, dq = (int64_t)s.n_heads * hd, dkv = (int64_t)s.n_kv * hd, f = s.ffn;
+  const int64_t nqkv = dq + 2 * dkv;
+  const int64_t big = imax64(imax64(nqkv * d, d * dq), imax64(2 * f * d, d * f));
+  PackWS p;
+  p.codes = c.take<uint8_t>(big);
+  p.r_qkv = c.take<float>(nqkv);
+  p.shift_qkv = c.take<float>(nqkv);
+  p.so_exp = c.take<float>(dq);
+  p.do_exp = c.take<float>(dq);
+  p.imax = c.take<int32_t>(big / 8 + 64);          // one entry per group, groups of >= 8 columns
+  p.imin = c.take<int32_t>(big / 8 + 64);
+  return p;
+}
+}  // namespace
+
+extern "C" size_t omq_block_pack_workspace_size(const omq_block_shape* shape, const omq_qcfg* cfg) {
+  if (check_block(shape, cfg) != OMQ_OK) return 0;
+  Carve dry{nullptr, 0};
+  carve_pack(dry, *shape);
+  return dry.off + 256;
+}
+
+extern "C" omq_status omq_block_fold_pack(omq_stream_t stream, const omq_block_shape* shape, const omq_block_weights* w,
+                                          const omq_block_params* theta, const omq_qcfg* cfg,
+                                          const omq_block_packed* out, void* workspace, size_t ws_bytes) {
+  OMQ_TRY(check_block(shape, cfg));
+  OMQ_REQUIRE(cfg->wbits < 16 && cfg->wbits >= 2 && cfg->wbits <= 8, OMQ_ERR_UNSUPPORTED);
+  OMQ_REQUIRE(w && theta && out && w->wqkv && w->wo && w->wgu && w->wd, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(theta->gamma_qkv && theta->beta_qkv && theta->gamma_o && theta->beta_o && theta->gamma_gu &&
+                  theta->beta_gu && theta->gamma_d && theta->beta_d,
+              OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(out->codes_qkv && out->codes_o && out->codes_gu && out->codes_d && out->h_qkv && out->z_qkv &&
+                  out->h_o && out->z_o && out->h_gu && out->z_gu && out->h_d && out->z_d,
+              OMQ_ERR_INVALID_ARG);
+  const bool let = cfg->let != 0;
+  if (let)
+    OMQ_REQUIRE(theta->s1 && theta->d1 && theta->so && theta->do_ && theta->sa && theta->s2 && theta->d2 &&
+                    out->b_qkv && out->b_o && out->b_gu && out->ln1_gain && out->ln1_bias && out->ln2_gain &&
+                    out->ln2_bias && out->sa,
+                OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(workspace && ws_bytes >= omq_block_pack_workspace_size(shape, cfg) && omq_aligned16(workspace),
+              OMQ_ERR_WORKSPACE);
+  cudaStream_t st = (cudaStream_t)stream;
+  Carve cv{(uint8_t*)workspace, 0};
+  PackWS p = carve_pack(cv, *shape);
+  const int64_t d = shape->d, hd = shape->head_dim, H = shape->n_heads, Hkv = shape->n_kv;
+  const int64_t dq = H * hd, dkv = Hkv * hd, f = shape->ffn, nqkv = dq + 2 * dkv, rep = H / Hkv;
+  if (let) {
+    OMQ_TRY(qkv_row_vectors(st, (int)dq, (int)dkv, theta->so, theta->do_, p.r_qkv, p.shift_qkv));
+    OMQ_TRY(gqa_expand(st, theta->so, p.so_exp, (int)Hkv, (int)rep, (int)hd, 0));
+    OMQ_TRY(gqa_expand(st, theta->do_, p.do_exp, (int)Hkv, (int)rep, (int)hd, 0));
+  }
+  struct One {
+    const void* W; int64_t Cout, Cin; const float *s, *r, *gl, *bl, *delta, *shift; float* Bt;
+    uint8_t* codes; float* h; int32_t* z;
+  } lin[4] = {
+      {w->wqkv, nqkv, d, let ? theta->s1 : nullptr, let ? p.r_qkv : nullptr, theta->gamma_qkv, theta->beta_qkv,
+       let ? theta->d1 : nullptr, let ? p.shift_qkv : nullptr, let ? out->b_qkv : nullptr, out->codes_qkv,
+       out->h_qkv, out->z_qkv},
+      {w->wo, d, dq, let ? p.so_exp : nullptr, nullptr, theta->gamma_o, theta->beta_o, let ? p.do_exp : nullptr,
+       nullptr, let ? out->b_o : nullptr, out->codes_o, out->h_o, out->z_o},
+      {w->wgu, 2 * f, d, let ? theta->s2 : nullptr, nullptr, theta->gamma_gu, theta->beta_gu,
+       let ? theta->d2 : nullptr, nullptr, let ? out->b_gu : nullptr, out->codes_gu, out->h_gu, out->z_gu},
+      {w->wd, d, f, nullptr, nullptr, theta->gamma_d, theta->beta_d, nullptr, nullptr, nullptr, out->codes_d,
+       out->h_d, out->z_d},
+  };
+  for (const One& l : lin) {
+    LwcFwdArgs a{};
+    a.W = (const bf16*)l.W; a.Cout = l.Cout; a.Cin = l.Cin; a.group = cfg->group == 0 ? (int)l.Cin : cfg->group;
+    a.s = l.s; a.r = l.r; a.gl = l.gl; a.bl = l.bl; a.lwc = 1; a.Wq = nullptr; a.codes = p.codes;
+    a.h = l.h; a.z = l.z; a.imax = p.imax; a.imin = p.imin;
+    a.bias_delta = l.delta; a.bias_shift = l.shift; a.Bt = l.Bt;
+    a.wbits = cfg->wbits; a.eps = cfg->h_eps; a.status = cfg->dev_status;
+    OMQ_TRY(lwc_fwd_launch(st, a));
+    OMQ_TRY(pack_codes_launch(st, p.codes, l.Cout, l.Cin, cfg->wbits, l.codes));
+  }
+  if (let) {
+    OMQ_TRY(norm_fold_launch(st, d, theta->s1, theta->d1, out->ln1_gain, out->ln1_bias));
+    OMQ_TRY(norm_fold_launch(st, d, theta->s2, theta->d2, out->ln2_gain, out->ln2_bias));
+    OMQ_REQUIRE(cudaMemcpyAsync(out->sa, theta->sa, (size_t)dkv * sizeof(float), cudaMemcpyDeviceToDevice, st) ==
+                    cudaSuccess,
+                OMQ_ERR_CUDA);
+  }
+  return OMQ_OK;
+}

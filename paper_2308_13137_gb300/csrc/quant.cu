@@ -555,6 +555,45 @@ omq_status lwc_bwd_fused_finish(cudaStream_t st, const LwcBwdArgs& a0, float* ro
 }
 
 // ================================================================================================
+// packing of integer codes: code i of a row at bits [N i, N i + N) of its little-endian stream
+// ================================================================================================
+__global__ void pack_codes_kernel(const uint8_t* __restrict__ codes, int64_t Cout, int64_t Cin, int nbits,
+                                  uint8_t* __restrict__ out) {
+  const int64_t nchunk = Cin / 8;
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;     // one 8-code chunk
+  if (i >= Cout * nchunk) return;
+  const int64_t o = i / nchunk, c = i % nchunk;
+  const uint2 raw = *reinterpret_cast<const uint2*>(codes + o * Cin + 8 * c);
+  const uint32_t w[2] = {raw.x, raw.y};
+  uint64_t acc = 0;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) acc |= (uint64_t)((w[e >> 2] >> (8 * (e & 3))) & 0xffu) << (nbits * e);
+  uint8_t* dst = out + o * (Cin * nbits / 8) + c * nbits;
+  for (int b = 0; b < nbits; ++b) dst[b] = (uint8_t)(acc >> (8 * b));
+}
+
+omq_status pack_codes_launch(cudaStream_t st, const uint8_t* codes, int64_t Cout, int64_t Cin, int nbits, uint8_t* out) {
+  OMQ_REQUIRE(Cin % 8 == 0 && nbits >= 1 && nbits <= 8, OMQ_ERR_SHAPE);
+  const int64_t n = Cout * (Cin / 8);
+  pack_codes_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(codes, Cout, Cin, nbits, out);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+__global__ void norm_fold_kernel(int64_t n, const float* s, const float* d, float* gain, float* bias) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  gain[i] = 1.0f / s[i];
+  bias[i] = -d[i] / s[i];
+}
+
+omq_status norm_fold_launch(cudaStream_t st, int64_t n, const float* s, const float* d, float* gain, float* bias) {
+  norm_fold_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(n, s, d, gain, bias);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+// ================================================================================================
 // reductions, loss, small vector kernels
 // ================================================================================================
 // 32 columns per CTA, eight row phases per column; fixed summation order (deterministic).

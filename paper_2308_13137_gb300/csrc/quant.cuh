@@ -109,3 +109,8 @@ omq_status let_smooth_pair(cudaStream_t st, int64_t C, const float* xmax, const 
 omq_status let_kv_pairs(cudaStream_t st, int Hkv, int rep, int hd, const float* omax, const float* osum,
                         const float* womax, const float* qmax, const float* kmax, double ntok, float alpha, float floor,
                         float* so, float* do_, float* sa);
+
+// ---- fold & pack --------------------------------------------------------------------------------
+omq_status pack_codes_launch(cudaStream_t st, const uint8_t* codes, int64_t Cout, int64_t Cin, int nbits, uint8_t* out);
+// gain = 1 / s, bias = -delta / s
+omq_status norm_fold_launch(cudaStream_t st, int64_t n, const float* s, const float* d, float* gain, float* bias);
