@@ -64,6 +64,10 @@ notes of the repository):
      (it sits after RoPE, R9, so it cannot be folded into the projection weights).  Weight
      codes are packed per output row as a little-endian bit stream: code i occupies bits
      [N i, N i + N) of the row.
+ R18 optimizer (Sec. 4.1 "Training": AdamW, zero weight decay, lr 5e-3 for the LWC logits and
+     1e-2 for the LET vectors): betas 0.9 / 0.999, eps 1e-8, bias-corrected moments, decoupled
+     weight decay; one update after every calibration sample (batch size 1).  Algorithm 1's
+     LET statistics (R16) are taken on the fp inputs of each block before they are advanced.
  R15 where floating point decides an integer (a code, a zero point, a max/min
      index, the floor of h) the decision is taken in the precision of the
      kernels, IEEE single precision with one rounding per product, difference and
@@ -88,7 +92,7 @@ __all__ = [
     "let_apply", "block_loss", "qlinear_step", "BlockCfg", "block_forward", "block_step",
     "rmsnorm", "rope", "silu", "FrozenTape", "use_tape", "block_fp_forward", "sigmoid_fp32",
     "THETA_NAMES_LWC", "THETA_NAMES_LET", "let_init", "pack_codes", "unpack_codes", "block_fold_pack",
-    "folded_forward",
+    "folded_forward", "adamw_step", "calibrate_blocks",
 ]
 
 
@@ -926,3 +930,50 @@ def folded_forward(folded: Dict[str, torch.Tensor], x, cfg: BlockCfg) -> torch.T
             gu = gu + folded["b_gu"]
         m = silu(gu[:, :f]) * gu[:, f:]
         return h1 + _mm(_qa(m, cfg), deq("d", d, f), mode)
+
+
+# ----------------------------------------------------------------------------------------------
+# Algorithm 1: block-wise calibration (R18)
+# ----------------------------------------------------------------------------------------------
+
+def adamw_step(p, g, m, v, lr: float, t: int, b1: float = 0.9, b2: float = 0.999, eps: float = 1e-8,
+               wd: float = 0.0):
+    """One AdamW update (in place) of parameter p with gradient g and moments m, v; t >= 1."""
+    m.mul_(b1).add_((1 - b1) * g)
+    v.mul_(b2).add_((1 - b2) * g * g)
+    mh = m / (1 - b1 ** t)
+    vh = v / (1 - b2 ** t)
+    p.sub_(lr * mh / (torch.sqrt(vh) + eps) + lr * wd * p)
+
+
+def calibrate_blocks(blocks, xs, cfg: BlockCfg, theta0, epochs: int = 1, lr_lwc: float = 5e-3,
+                     lr_let: float = 1e-2, let_init_alpha: Optional[float] = 0.5):
+    """Algorithm 1 over a stack of blocks: X_fp = X_q = X; per block: X_fp <- B(X_fp), initialise
+    Theta1 (theta0's LWC logits) and Theta2 (let_init on the block's fp inputs, R16), train on the
+    (x_q, x_fp) pairs for `epochs` epochs with AdamW (R18), then X_q <- the quantized block(X_q).
+    Returns the per-block parameters and the final X_fp, X_q."""
+    t = lambda v: torch.as_tensor(v).to(F64)
+    x_fp = [t(x) for x in xs]
+    x_q = [t(x) for x in xs]
+    names = (THETA_NAMES_LWC if cfg.wbits < 16 else []) + (THETA_NAMES_LET if cfg.let else [])
+    out = []
+    for W in blocks:
+        th = {k: t(theta0[k]).clone() for k in names}
+        if cfg.let and let_init_alpha is not None:
+            th.update(let_init(x_fp, W, cfg, alpha=let_init_alpha))
+        y_fp = [block_fp_forward(x, W, cfg) for x in x_fp]
+        mom = {k: (torch.zeros_like(v), torch.zeros_like(v)) for k, v in th.items()}
+        step = 0
+        for _ in range(epochs):
+            for xq, yf in zip(x_q, y_fp):
+                r = block_step(xq, yf, W, th, cfg)
+                step += 1
+                for k in names:
+                    lr = lr_let if k in THETA_NAMES_LET else lr_lwc
+                    adamw_step(th[k], r["d" + k], mom[k][0], mom[k][1], lr, step)
+        with torch.no_grad():
+            Wd = {k: t(v) for k, v in W.items()}
+            x_q = [block_forward(xq, Wd, th, cfg) for xq in x_q]
+        x_fp = y_fp
+        out.append({k: v.clone() for k, v in th.items()})
+    return out, x_fp, x_q

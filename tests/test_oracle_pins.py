@@ -574,3 +574,42 @@ def test_folded_block_equals_calibrated_block(let, abits, wbits, group, n_kv):
     assert _rel(y_fold, y_ref) < (1e-8 if let else 1e-12)
     assert folded["codes_qkv"].dtype == torch.uint8
     assert folded["codes_qkv"].shape[1] * 8 == shape.d * wbits
+
+
+def test_adamw_step_matches_library_adamw():
+    """The oracle's AdamW update (Sec. 4.1 "Training"; reading R18) equals torch.optim.AdamW over
+    several steps, with and without decoupled weight decay."""
+    g = torch.Generator().manual_seed(3)
+    for wd in (0.0, 0.1):
+        p0 = torch.randn(7, generator=g, dtype=F64)
+        p_ref = p0.clone().requires_grad_(True)
+        opt = torch.optim.AdamW([p_ref], lr=1e-2, betas=(0.9, 0.999), eps=1e-8, weight_decay=wd)
+        p, m, v = p0.clone(), torch.zeros(7, dtype=F64), torch.zeros(7, dtype=F64)
+        for step in range(1, 6):
+            grad = torch.randn(7, generator=g, dtype=F64)
+            p_ref.grad = grad.clone()
+            opt.step()
+            O.adamw_step(p, grad, m, v, 1e-2, step, wd=wd)
+        assert torch.allclose(p, p_ref.detach(), rtol=1e-12, atol=1e-14)
+
+
+def test_calibration_driver_data_flow():
+    """Algorithm 1's data flow: with zero epochs, after each block X_fp is the full-precision block
+    of the previous X_fp and X_q the quantized block (initial parameters) of the previous X_q, and
+    the LET parameters of each block are let_init of that block's fp inputs."""
+    shape, W0, x, th, cfg = _tiny_block(let=True, abits=4, wbits=4, n_kv=2)
+    W1 = {k: v[::-1].copy() for k, v in W0.items()}
+    xs = [x, I.make_block_input(shape, sample=1, weight_seed=1)]
+    params, x_fp, x_q = O.calibrate_blocks([W0, W1], xs, cfg, th, epochs=0)
+    f0 = [O.block_fp_forward(xx, W0, cfg) for xx in xs]
+    f1 = [O.block_fp_forward(xx, W1, cfg) for xx in f0]
+    for a, b in zip(x_fp, f1):
+        assert torch.equal(a, b)
+    p0 = dict(_t(th), **O.let_init(xs, W0, cfg))
+    q0 = [O.block_forward(torch.as_tensor(xx, dtype=F64), _t(W0), p0, cfg) for xx in xs]
+    p1 = dict(_t(th), **O.let_init(f0, W1, cfg))
+    q1 = [O.block_forward(xx, _t(W1), p1, cfg) for xx in q0]
+    for a, b in zip(x_q, q1):
+        assert torch.equal(a, b)
+    for k in O.THETA_NAMES_LET:
+        assert torch.equal(params[1][k], p1[k])
