@@ -163,22 +163,29 @@ class BlockState:
         _lib.omq_block_fold_pack(self.c_shape, self.c_w, self.c_theta, self.cfg, c_out, ws, stream)
         return out
 
-    def split_grads(self) -> Dict[str, np.ndarray]:
-        """Gradients on the host, named like the oracle's parameters."""
+    def _split(self, src, prefix: str) -> Dict[str, np.ndarray]:
         out = {}
         sh = self.shape
         sizes = dict(qkv=[sh.dq, sh.dkv, sh.dkv], o=[sh.d], gu=[sh.ffn, sh.ffn], d=[sh.d])
         for key, parts in LWC_PARTS.items():
             for gb in ("gamma", "beta"):
                 name = f"{gb}_{key}"
-                if name not in self.grads:
+                if name not in src:
                     continue
-                g = self.grads[name].float().cpu().numpy()
+                g = src[name].float().cpu().numpy()
                 off = 0
                 for p, n in zip(parts, sizes[key]):
-                    out[f"d{gb}_{p}"] = g[off:off + n]
+                    out[f"{prefix}{gb}_{p}"] = g[off:off + n]
                     off += n
         for k in LET_NAMES:
-            if k in self.grads:
-                out["d" + k] = self.grads[k].float().cpu().numpy()
+            if k in src:
+                out[prefix + k] = src[k].float().cpu().numpy()
         return out
+
+    def split_grads(self) -> Dict[str, np.ndarray]:
+        """Gradients on the host, named like the oracle's parameters (d<name>)."""
+        return self._split(self.grads, "d")
+
+    def split_theta(self) -> Dict[str, np.ndarray]:
+        """Parameters on the host, named like the oracle's parameters."""
+        return self._split(self.theta, "")
