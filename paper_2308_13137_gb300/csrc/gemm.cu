@@ -31,14 +31,15 @@ struct GemmParams {
   GemmEpilogue ep;
   GemmLwcEpi lw;             // used by the LWC-epilogue instantiation only
   int32_t* status;
+  int pair;                  // 1: CTA pairs, one 256-row tile per pair (cta_group::2)
 };
 
 constexpr int EPI_TILE_BYTES = 32 * 32 * 4;      // one 32 x 32 fp32 block, 128-byte rows
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, bool PAIR = false>
 struct SmemLayout {
   static constexpr int A_BYTES = BM * BK * 2;
-  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int B_BYTES = (PAIR ? BN / 2 : BN) * BK * 2;   // a pair splits B's columns
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int EPI_OFF = STAGES * STAGE_BYTES;           // 1024-aligned (swizzle atom)
   static constexpr int EPI_BYTES = 4 * 2 * EPI_TILE_BYTES;       // two staging blocks per epilogue warp
@@ -52,16 +53,19 @@ struct SmemLayout {
 // Tile t of the launch (m fastest, then n, then batch) and its K range.
 struct TileInfo { int m0, n0, b, k_begin, nkb; bool skip; };
 
-__device__ __forceinline__ TileInfo tile_info(const GemmParams& p, int t, int bn) {
-  const int mt = (p.M + BM - 1) / BM, nt = (p.N + bn - 1) / bn;
+// With CTA pairs a tile is 2 BM rows; CTA `rank` of the pair owns rows m0 .. m0 + BM - 1.
+__device__ __forceinline__ TileInfo tile_info(const GemmParams& p, int t, int bn, int rank = 0) {
+  const int bm = p.pair ? 2 * BM : BM;
+  const int mt = (p.M + bm - 1) / bm, nt = (p.N + bn - 1) / bn;
   TileInfo ti;
   if (p.n_fast) {
     ti.n0 = (t % nt) * bn;
-    ti.m0 = ((t / nt) % mt) * BM;
+    ti.m0 = ((t / nt) % mt) * bm;
   } else {
-    ti.m0 = (t % mt) * BM;
+    ti.m0 = (t % mt) * bm;
     ti.n0 = ((t / mt) % nt) * bn;
   }
+  ti.m0 += rank * BM;
   ti.b = t / (mt * nt);
   ti.skip = (p.causal == 1 && ti.n0 > ti.m0 + BM - 1);   // keys beyond every query of the tile
   int k_end = p.K;
@@ -96,16 +100,29 @@ __device__ __forceinline__ void ldw32(const __nv_bfloat16* p, bool ok, uint4 (&r
 // Epilogue of the weight-gradient product with the straight-through LWC backward (Eq. 2) fused:
 // the accumulator dW_hat is consumed from tensor memory 32 columns at a time and never stored.
 // The weight row chunk of the next 32 columns is loaded while the current one is processed.
-template <int BN>
+// hands accumulator buffer `buf` back to the MMA issuer (with CTA pairs: the leader CTA's barrier)
+template <bool PAIR>
+__device__ __forceinline__ void release_acc(uint64_t* acc_empty, uint32_t buf, int lane) {
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) {
+    if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&acc_empty[buf]), 0));
+    else mbar_arrive(&acc_empty[buf]);
+  }
+}
+
+template <int BN, bool PAIR>
 __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem, uint64_t* acc_full, uint64_t* acc_empty,
-                                             volatile int* abort_flag, int q, int lane, int total) {
+                                             volatile int* abort_flag, int q, int lane, int total, int rank) {
   const GemmLwcEpi& L = p.lw;
   const int N = p.N;
   const bool perch = L.group == N;
   const int ngroups = N / L.group;
   uint32_t acc_it = 0;
-  for (int t = blockIdx.x; t < total; t += gridDim.x) {
-    const TileInfo ti = tile_info(p, t, BN);
+  const int t_first = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int t_step = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+  for (int t = t_first; t < total; t += t_step) {
+    const TileInfo ti = tile_info(p, t, BN, rank);
     if (ti.skip) continue;
     const bool has_acc = ti.nkb > 0;
     const uint32_t buf = acc_it & 1;
@@ -133,11 +150,7 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
       float g[32];
       if (has_acc && ok) {
         tmem_ld32(tmem + buf * BN + ((uint32_t)(q * 32) << 16) + (uint32_t)j0, g);
-        if (j0 + 32 == BN) {                      // accumulator drained: hand the buffer back
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&acc_empty[buf]);
-        }
+        if (j0 + 32 == BN) release_acc<PAIR>(acc_empty, buf, lane);   // accumulator drained
       } else {
 #pragma unroll
         for (int i = 0; i < 32; ++i) g[i] = 0.f;
@@ -227,11 +240,17 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
 // The shared-memory ring runs continuously across tiles; the accumulator is double-buffered
 // in tensor memory (2 x BN columns) so that the epilogue of one tile overlaps the MMAs of
 // the next.
-template <int BN, int STAGES, bool LWC>
+//
+// PAIR: the grid is made of 2-CTA clusters; the pair computes one 2 BM x BN tile with one
+// tcgen05.mma of cta_group::2 (M = 256): each CTA stages its BM rows of A and BN / 2 columns of B
+// (both TMA loads complete on the leader CTA's mbarrier), the leader issues the MMAs, commits
+// reach both CTAs' barriers, and each CTA drains its own BM rows of the accumulator.  Per CTA
+// the shared-memory bytes per MMA flop halve for B, so six stages fit where four did.
+template <int BN, int STAGES, bool LWC, bool PAIR>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const __grid_constant__ CUtensorMap tmC, const GemmParams p) {
-  using L = SmemLayout<BN, STAGES>;
+  using L = SmemLayout<BN, STAGES, PAIR>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L::BAR_OFF);
@@ -242,27 +261,38 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int mt = (p.M + BM - 1) / BM, nt = (p.N + BN - 1) / BN;
+  const int bm_tile = PAIR ? 2 * BM : BM;
+  const int mt = (p.M + bm_tile - 1) / bm_tile, nt = (p.N + BN - 1) / BN;
   const int total = mt * nt * p.batch;
+  const int rank = PAIR ? (int)cluster_ctarank() : 0;
+  const bool leader = rank == 0;
+  const int t_first = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int t_step = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
-    for (int b = 0; b < 2; ++b) { mbar_init(&acc_full[b], 1); mbar_init(&acc_empty[b], 4); }
+    for (int b = 0; b < 2; ++b) { mbar_init(&acc_full[b], 1); mbar_init(&acc_empty[b], PAIR ? 8 : 4); }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 1) tmem_alloc(tmem_holder, 2 * BN);
+  if (warp == 1) {
+    if (PAIR) tmem_alloc_pair(tmem_holder, 2 * BN);
+    else tmem_alloc(tmem_holder, 2 * BN);
+  }
   tc_fence_before();
   __syncthreads();
+  if (PAIR) cluster_sync();                 // both CTAs' barriers initialised before any remote use
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
 
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer ----------------
     uint32_t it = 0;
-    for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
-      const TileInfo ti = tile_info(p, t, BN);
+    constexpr int BNH = PAIR ? BN / 2 : BN;      // B columns staged by this CTA
+    for (int t = t_first; t < total && !*abort_flag; t += t_step) {
+      const TileInfo ti = tile_info(p, t, BN, rank);
       if (ti.skip) continue;
+      const int nb0 = ti.n0 + rank * BNH;
       for (int kb = 0; kb < ti.nkb; ++kb, ++it) {
         const int s = it % STAGES;
         if (!mbar_wait(&empty[s], ((it / STAGES) & 1) ^ 1)) {
@@ -271,28 +301,46 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         uint8_t* sa = smem + s * L::STAGE_BYTES;
         uint8_t* sb = sa + L::A_BYTES;
         const int k0 = ti.k_begin + kb * BK;
-        mbar_expect_tx(&full[s], L::STAGE_BYTES);
-        if (!p.a_mn) {
-          tma_load_3d(&tmA, &full[s], sa, k0, ti.m0, ti.b);
-        } else {
-          tma_load_3d(&tmA, &full[s], sa, ti.m0, k0, ti.b);
-          tma_load_3d(&tmA, &full[s], sa + 64 * BK * 2, ti.m0 + 64, k0, ti.b);
-        }
-        if (!p.b_mn) {
-          tma_load_3d(&tmB, &full[s], sb, k0, ti.n0, ti.b);
-        } else {
+        if (PAIR) {
+          // both CTAs' loads complete on the leader's barrier, which expects the pair's bytes
+          const uint32_t fb = mapa_shared(smem_u32(&full[s]), 0);
+          if (leader) mbar_expect_tx(&full[s], 2 * L::STAGE_BYTES);
+          if (!p.a_mn) {
+            tma_load_3d_pair(&tmA, fb, sa, k0, ti.m0, ti.b);
+          } else {
+            tma_load_3d_pair(&tmA, fb, sa, ti.m0, k0, ti.b);
+            tma_load_3d_pair(&tmA, fb, sa + 64 * BK * 2, ti.m0 + 64, k0, ti.b);
+          }
+          if (!p.b_mn) {
+            tma_load_3d_pair(&tmB, fb, sb, k0, nb0, ti.b);
+          } else {
 #pragma unroll
-          for (int j = 0; j < BN / 64; ++j) tma_load_3d(&tmB, &full[s], sb + j * 64 * BK * 2, ti.n0 + 64 * j, k0, ti.b);
+            for (int j = 0; j < BNH / 64; ++j) tma_load_3d_pair(&tmB, fb, sb + j * 64 * BK * 2, nb0 + 64 * j, k0, ti.b);
+          }
+        } else {
+          mbar_expect_tx(&full[s], L::STAGE_BYTES);
+          if (!p.a_mn) {
+            tma_load_3d(&tmA, &full[s], sa, k0, ti.m0, ti.b);
+          } else {
+            tma_load_3d(&tmA, &full[s], sa, ti.m0, k0, ti.b);
+            tma_load_3d(&tmA, &full[s], sa + 64 * BK * 2, ti.m0 + 64, k0, ti.b);
+          }
+          if (!p.b_mn) {
+            tma_load_3d(&tmB, &full[s], sb, k0, ti.n0, ti.b);
+          } else {
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j) tma_load_3d(&tmB, &full[s], sb + j * 64 * BK * 2, ti.n0 + 64 * j, k0, ti.b);
+          }
         }
       }
     }
-  } else if (warp == 1 && lane == 0) {
-    // ---------------- MMA issuer ----------------
-    constexpr uint32_t IDESC_KK = idesc_bf16(BM, BN, 0, 0);
+  } else if (warp == 1 && lane == 0 && leader) {
+    // ---------------- MMA issuer (with CTA pairs: the leader CTA only) ----------------
+    constexpr uint32_t IDESC_KK = idesc_bf16(PAIR ? 2 * BM : BM, BN, 0, 0);
     const uint32_t idesc = IDESC_KK | ((uint32_t)p.a_mn << 15) | ((uint32_t)p.b_mn << 16);
     uint32_t it = 0, acc_it = 0;
-    for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
-      const TileInfo ti = tile_info(p, t, BN);
+    for (int t = t_first; t < total && !*abort_flag; t += t_step) {
+      const TileInfo ti = tile_info(p, t, BN, rank);
       if (ti.skip || ti.nkb == 0) continue;
       const uint32_t buf = acc_it & 1;
       if (!mbar_wait(&acc_empty[buf], ((acc_it >> 1) & 1) ^ 1)) {
@@ -314,16 +362,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           // K-major: advance 32 bytes inside the swizzle row; MN-major: advance 16 K-rows (2 KB)
           const uint64_t ad = p.a_mn ? sdesc(sa + k * 2048, 64 * BK * 2, 1024) : sdesc(sa + k * 32, 16, 1024);
           const uint64_t bd = p.b_mn ? sdesc(sb + k * 2048, 64 * BK * 2, 1024) : sdesc(sb + k * 32, 16, 1024);
-          umma_bf16(d_tmem, ad, bd, idesc, (kb | k) != 0);
+          if (PAIR) umma_bf16_pair(d_tmem, ad, bd, idesc, (kb | k) != 0);
+          else umma_bf16(d_tmem, ad, bd, idesc, (kb | k) != 0);
         }
-        umma_commit(&empty[s]);
+        if (PAIR) umma_commit_pair(&empty[s], 0x3);
+        else umma_commit(&empty[s]);
       }
-      umma_commit(&acc_full[buf]);
+      if (PAIR) umma_commit_pair(&acc_full[buf], 0x3);
+      else umma_commit(&acc_full[buf]);
       ++acc_it;
       if (!ok) break;
     }
   } else if (LWC && warp >= 2) {
-    lwc_epilogue<BN>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, lane, total);
+    lwc_epilogue<BN, PAIR>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, lane, total, rank);
   } else if (warp >= 2) {
     // ---------------- epilogue ----------------
     // fp32 output leaves through TMA bulk stores: each warp stages its 32 x 32 block in one of two
@@ -335,8 +386,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     uint8_t* stage_base = smem + L::EPI_OFF + q * 2 * EPI_TILE_BYTES;
     uint32_t n_stores = 0;
     uint32_t acc_it = 0;
-    for (int t = blockIdx.x; t < total; t += gridDim.x) {
-      const TileInfo ti = tile_info(p, t, BN);
+    for (int t = t_first; t < total; t += t_step) {
+      const TileInfo ti = tile_info(p, t, BN, rank);
       if (ti.skip) continue;
       const bool has_acc = ti.nkb > 0;
       const uint32_t buf = acc_it & 1;
@@ -355,11 +406,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         float v[32];
         if (has_acc && ok) {
           tmem_ld32(tmem + buf * BN + ((uint32_t)(q * 32) << 16) + (uint32_t)j0, v);
-          if (j0 + 32 == BN) {                    // accumulator drained: hand the buffer back
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&acc_empty[buf]);
-          }
+          if (j0 + 32 == BN) release_acc<PAIR>(acc_empty, buf, lane);   // accumulator drained
         } else {
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = 0.f;
@@ -436,9 +483,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
   tc_fence_before();
   __syncthreads();
+  if (PAIR) cluster_sync();                 // no CTA leaves while its peer may still signal it
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, 2 * BN);
+    if (PAIR) tmem_dealloc_pair(tmem, 2 * BN);
+    else tmem_dealloc(tmem, 2 * BN);
   }
 }
 
@@ -490,21 +539,40 @@ bool make_map_c(CUtensorMap* map, float* ptr, int64_t N, int64_t M, int64_t batc
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES, bool LWC = false>
+template <int BN, int STAGES, bool LWC = false, bool PAIR = false>
 omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
                       const GemmParams& p) {
-  using L = SmemLayout<BN, STAGES>;
+  using L = SmemLayout<BN, STAGES, PAIR>;
+  auto kern = gemm_bf16_kernel<BN, STAGES, LWC, PAIR>;
   static bool attr_set = false;
   if (!attr_set) {
-    if (cudaFuncSetAttribute(gemm_bf16_kernel<BN, STAGES, LWC>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::TOTAL) !=
-        cudaSuccess)
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::TOTAL) != cudaSuccess)
       return OMQ_ERR_CUDA;
     attr_set = true;
   }
-  const int64_t tiles = (int64_t)((p.M + BM - 1) / BM) * ((p.N + BN - 1) / BN) * p.batch;
+  const int bm_tile = PAIR ? 2 * BM : BM;
+  const int64_t tiles = (int64_t)((p.M + bm_tile - 1) / bm_tile) * ((p.N + BN - 1) / BN) * p.batch;
   const int64_t sms = omq_num_sms();
-  const unsigned grid = (unsigned)(tiles < sms ? tiles : sms);
-  gemm_bf16_kernel<BN, STAGES, LWC><<<grid, NUM_THREADS, L::TOTAL, st>>>(ta, tb, tc, p);
+  if (!PAIR) {
+    const unsigned grid = (unsigned)(tiles < sms ? tiles : sms);
+    kern<<<grid, NUM_THREADS, L::TOTAL, st>>>(ta, tb, tc, p);
+  } else {
+    const int64_t pairs = sms / 2;
+    const unsigned grid = (unsigned)(2 * (tiles < pairs ? tiles : pairs));
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid, 1, 1);
+    cfg.blockDim = dim3(NUM_THREADS, 1, 1);
+    cfg.dynamicSmemBytes = L::TOTAL;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, p) != cudaSuccess) return OMQ_ERR_CUDA;
+  }
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -565,10 +633,13 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
   OMQ_REQUIRE(!ep.bias || omq_aligned16(ep.bias), OMQ_ERR_ALIGN);
   // the MN-major extents must cover whole 64-wide boxes inside the tensor (TMA zero-fills the rest)
   const bool wide = gemm_n_tile(N) == 256;
+  // CTA pairs (one 256 x 256 tile per pair) for plain single products
+  const bool pair = wide && batch == 1 && causal == 0 && M > BM;
   CUtensorMap ta, tb;
   const int bn = wide ? 256 : 128;
   bool ok = A.kmajor ? make_map(&ta, A.ptr, K, M, batch, A.ld, A.bs, BM) : make_map(&ta, A.ptr, M, K, batch, A.ld, A.bs, BK);
-  ok = ok && (B.kmajor ? make_map(&tb, B.ptr, K, N, batch, B.ld, B.bs, bn) : make_map(&tb, B.ptr, N, K, batch, B.ld, B.bs, BK));
+  ok = ok && (B.kmajor ? make_map(&tb, B.ptr, K, N, batch, B.ld, B.bs, pair ? bn / 2 : bn)
+                       : make_map(&tb, B.ptr, N, K, batch, B.ld, B.bs, BK));
   CUtensorMap tc;
   memset(&tc, 0, sizeof(tc));
   if (ep.Cf) ok = ok && make_map_c(&tc, ep.Cf, N, M, batch, ep.ldc, ep.c_bs);
@@ -576,7 +647,7 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
   GemmParams p;
   p.M = (int)M; p.N = (int)N; p.K = (int)K; p.batch = (int)batch;
   p.a_mn = A.kmajor ? 0 : 1; p.b_mn = B.kmajor ? 0 : 1;
-  p.causal = causal; p.ep = ep; p.status = status;
+  p.causal = causal; p.ep = ep; p.status = status; p.pair = pair ? 1 : 0;
   // stream the larger operand once and keep the smaller one L2-resident: with m fastest, the
   // CTAs working at one time share an N tile of B and sweep A; with n fastest, the reverse
   p.n_fast = ((double)M > 1.5 * (double)N) ? 1 : 0;
@@ -589,7 +660,8 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
       g_prof.flops += gemm_algorithmic_flops(M, N, K, batch, causal);
     }
   }
-  omq_status r = wide ? launch_cfg<256, 4>(st, ta, tb, tc, p) : launch_cfg<128, 6>(st, ta, tb, tc, p);
+  omq_status r = pair ? launch_cfg<256, 6, false, true>(st, ta, tb, tc, p)
+                      : (wide ? launch_cfg<256, 4>(st, ta, tb, tc, p) : launch_cfg<128, 6>(st, ta, tb, tc, p));
   if (e0 && e1) cudaEventRecord(e1, st);
   return r;
 }
@@ -627,16 +699,18 @@ omq_status gemm_launch_lwc(cudaStream_t st, int64_t M, int64_t N, int64_t K, con
   OMQ_REQUIRE(perch || (lw.dgl && lw.dbl && lw.ga && lw.Mv), OMQ_ERR_INVALID_ARG);
   OMQ_REQUIRE(!lw.part_s || lw.s, OMQ_ERR_INVALID_ARG);
   OMQ_REQUIRE(!lw.part_d || lw.dBt, OMQ_ERR_INVALID_ARG);
+  const bool pair = bn == 256 && M > BM;           // CTA pairs, one 256 x 256 tile per pair
   CUtensorMap ta, tb, tc;
   memset(&tc, 0, sizeof(tc));
   bool ok = A.kmajor ? make_map(&ta, A.ptr, K, M, 1, A.ld, 0, BM) : make_map(&ta, A.ptr, M, K, 1, A.ld, 0, BK);
-  ok = ok && (B.kmajor ? make_map(&tb, B.ptr, K, N, 1, B.ld, 0, bn) : make_map(&tb, B.ptr, N, K, 1, B.ld, 0, BK));
+  ok = ok && (B.kmajor ? make_map(&tb, B.ptr, K, N, 1, B.ld, 0, pair ? bn / 2 : bn)
+                       : make_map(&tb, B.ptr, N, K, 1, B.ld, 0, BK));
   if (!ok) return OMQ_ERR_UNSUPPORTED;
   GemmParams p;
   memset(&p, 0, sizeof(p));
   p.M = (int)M; p.N = (int)N; p.K = (int)K; p.batch = 1;
   p.a_mn = A.kmajor ? 0 : 1; p.b_mn = B.kmajor ? 0 : 1;
-  p.causal = 0; p.lw = lw; p.status = status;
+  p.causal = 0; p.lw = lw; p.status = status; p.pair = pair ? 1 : 0;
   p.n_fast = ((double)M > 1.5 * (double)N) ? 1 : 0;
   cudaEvent_t e0 = nullptr, e1 = nullptr;
   if (g_prof.on) {
@@ -647,7 +721,8 @@ omq_status gemm_launch_lwc(cudaStream_t st, int64_t M, int64_t N, int64_t K, con
       g_prof.flops += gemm_algorithmic_flops(M, N, K, 1, 0);
     }
   }
-  omq_status r = bn == 256 ? launch_cfg<256, 4, true>(st, ta, tb, tc, p) : launch_cfg<128, 6, true>(st, ta, tb, tc, p);
+  omq_status r = pair ? launch_cfg<256, 6, true, true>(st, ta, tb, tc, p)
+                      : (bn == 256 ? launch_cfg<256, 4, true>(st, ta, tb, tc, p) : launch_cfg<128, 6, true>(st, ta, tb, tc, p));
   if (e0 && e1) cudaEventRecord(e1, st);
   return r;
 }
