@@ -27,14 +27,14 @@ struct QState4 { float* h; int32_t* z; int32_t* imax; int32_t* imin; float* ga; 
 
 // Scratch (floats) of the fused weight-gradient + LWC backward of one [Cout, Cin] weight
 int64_t lwc_fused_scratch_elems(int64_t Cout, int64_t Cin) {
-  const int64_t ntn = (Cin + gemm_n_tile(Cin) - 1) / gemm_n_tile(Cin);
+  const int64_t ntn = 2 * ((Cin + gemm_n_tile(Cin) - 1) / gemm_n_tile(Cin));   // row partials per row
   return 2 * ((Cout + 31) / 32) * Cin + 3 * Cout * ntn + 64;
 }
 
 bool lwc_fused_ok(int64_t Cin, int group, bool let_terms) {
   if (Cin % 32 != 0) return false;
   if (group == Cin) return true;
-  return !let_terms && group % 32 == 0 && gemm_n_tile(Cin) % group == 0;
+  return !let_terms && group % 32 == 0 && (gemm_n_tile(Cin) / 2) % group == 0;
 }
 
 QState4 take_qstate(Carve& c, size_t n, bool saved = false) {
@@ -253,7 +253,7 @@ omq_status lwc_bwd_dw(cudaStream_t st, int64_t T, const bf16* dY, const bf16* Xh
                         accumulate_sd, part);
   }
   const int64_t P = (Cout + 31) / 32;
-  const int ntn = (int)((Cin + gemm_n_tile(Cin) - 1) / gemm_n_tile(Cin));
+  const int ntn = 2 * (int)((Cin + gemm_n_tile(Cin) - 1) / gemm_n_tile(Cin));
   GemmLwcEpi lw{};
   lw.W = W; lw.s = s; lw.r = r; lw.h = q.h; lw.z = q.z; lw.ga = q.ga; lw.gb = q.gb; lw.Mv = q.M; lw.mv = q.m;
   lw.dBt = dBt;

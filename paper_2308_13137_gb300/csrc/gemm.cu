@@ -21,7 +21,8 @@ using namespace tc;
 constexpr int BM = 128;
 constexpr int BK = 64;          // one 128-byte swizzle row of bf16
 constexpr int UMMA_K = 16;
-constexpr int NUM_THREADS = 192;
+constexpr int NUM_THREADS = 192;          // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
+constexpr int NUM_THREADS_LWC = 320;      // LWC epilogue: warps 2..9, two per TMEM lane quadrant
 
 struct GemmParams {
   int M, N, K, batch;
@@ -111,9 +112,12 @@ __device__ __forceinline__ void release_acc(uint64_t* acc_empty, uint32_t buf, i
   }
 }
 
+// Eight epilogue warps: warps w and w+4 drain the same 32 accumulator rows (lane quadrant w % 4),
+// `half` 0 the first BN / 2 columns of the tile, 1 the others; each keeps its own row partials.
 template <int BN, bool PAIR>
 __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem, uint64_t* acc_full, uint64_t* acc_empty,
-                                             volatile int* abort_flag, int q, int lane, int total, int rank) {
+                                             volatile int* abort_flag, int q, int half, int lane, int total, int rank) {
+  constexpr int HB = BN / 2;                      // columns of a half
   const GemmLwcEpi& L = p.lw;
   const int N = p.N;
   const bool perch = L.group == N;
@@ -143,38 +147,40 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
     qs.h = 1.f; qs.rh = 1.f; qs.z = 0.f; qs.u = 0.f; qs.b = 0.f; qs.m = 0.f; qs.a = 0.f; qs.M = 0.f; qs.floored = 0;
     int64_t gk = 0;                                // (row, group) index of the current group
     float Gh = 0.f, Gbm = 0.f, drm = 0.f;
+    const int jb = half * HB;
     uint4 wcur[4], wnext[4];
-    ldw32(wrow + ti.n0, row_ok && ti.n0 < N, wcur);
+    ldw32(wrow + ti.n0 + jb, row_ok && ti.n0 + jb < N, wcur);
+    if (perch && row_ok) {                        // one quantizer state for the whole row
+      gk = row;
+      qs.h = L.h[gk];
+      qs.z = (float)L.z[gk];
+      qs.b = L.gb[gk];
+      qs.m = L.mv[gk];
+      qs.rh = __frcp_rn(qs.h);
+      qs.u = __fmul_rn(__fmul_rn(qs.b, qs.m), qs.rh);
+    }
 #pragma unroll 1
-    for (int j0 = 0; j0 < BN; j0 += 32) {
+    for (int j0 = jb; j0 < jb + HB; j0 += 32) {
       float g[32];
       if (has_acc && ok) {
         tmem_ld32(tmem + buf * BN + ((uint32_t)(q * 32) << 16) + (uint32_t)j0, g);
-        if (j0 + 32 == BN) release_acc<PAIR>(acc_empty, buf, lane);   // accumulator drained
+        if (j0 + 32 == jb + HB) release_acc<PAIR>(acc_empty, buf, lane);   // this warp's part drained
       } else {
 #pragma unroll
         for (int i = 0; i < 32; ++i) g[i] = 0.f;
       }
       const int nb = ti.n0 + j0;
-      if (j0 + 32 < BN) ldw32(wrow + nb + 32, row_ok && nb + 32 < N, wnext);
+      if (j0 + 32 < jb + HB) ldw32(wrow + nb + 32, row_ok && nb + 32 < N, wnext);
       if (quad_ok && nb < N) {
-        if (nb % L.group == 0 && row_ok) {       // quantizer state of the group starting here
-          gk = perch ? (int64_t)row : (int64_t)row * ngroups + nb / L.group;
+        if (!perch && nb % L.group == 0 && row_ok) {   // quantizer state of the group starting here
+          gk = (int64_t)row * ngroups + nb / L.group;
           qs.h = L.h[gk];
           qs.z = (float)L.z[gk];
           qs.b = L.gb[gk];
           qs.m = L.mv[gk];
           qs.rh = __frcp_rn(qs.h);
           qs.u = __fmul_rn(__fmul_rn(qs.b, qs.m), qs.rh);
-          if (!perch) { Gh = 0.f; Gbm = 0.f; }
-        } else if (perch && j0 == 0 && row_ok) {  // per-channel state, tile starting mid-row
-          gk = row;
-          qs.h = L.h[gk];
-          qs.z = (float)L.z[gk];
-          qs.b = L.gb[gk];
-          qs.m = L.mv[gk];
-          qs.rh = __frcp_rn(qs.h);
-          qs.u = __fmul_rn(__fmul_rn(qs.b, qs.m), qs.rh);
+          Gh = 0.f; Gbm = 0.f;
         }
         float cs[32], cd[32];
 #pragma unroll
@@ -226,7 +232,7 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
       for (int i = 0; i < 4; ++i) wcur[i] = wnext[i];
     }
     if (perch && quad_ok && row_ok) {
-      const int nt = ti.n0 / BN;
+      const int nt = 2 * (ti.n0 / BN) + half;     // one partial per (N tile, half)
       L.rowpart[((int64_t)0 * p.M + row) * L.ntn + nt] = Gh;
       L.rowpart[((int64_t)1 * p.M + row) * L.ntn + nt] = Gbm;
       L.rowpart[((int64_t)2 * p.M + row) * L.ntn + nt] = drm;
@@ -247,7 +253,7 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
 // reach both CTAs' barriers, and each CTA drains its own BM rows of the accumulator.  Per CTA
 // the shared-memory bytes per MMA flop halve for B, so six stages fit where four did.
 template <int BN, int STAGES, bool LWC, bool PAIR>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+__global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
     gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const __grid_constant__ CUtensorMap tmC, const GemmParams p) {
   using L = SmemLayout<BN, STAGES, PAIR>;
@@ -271,7 +277,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
-    for (int b = 0; b < 2; ++b) { mbar_init(&acc_full[b], 1); mbar_init(&acc_empty[b], PAIR ? 8 : 4); }
+    constexpr int EPI_WARPS = LWC ? 8 : 4;
+    for (int b = 0; b < 2; ++b) { mbar_init(&acc_full[b], 1); mbar_init(&acc_empty[b], (PAIR ? 2 : 1) * EPI_WARPS); }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -374,7 +381,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (!ok) break;
     }
   } else if (LWC && warp >= 2) {
-    lwc_epilogue<BN, PAIR>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, lane, total, rank);
+    lwc_epilogue<BN, PAIR>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, (warp - 2) >> 2, lane, total, rank);
   } else if (warp >= 2) {
     // ---------------- epilogue ----------------
     // fp32 output leaves through TMA bulk stores: each warp stages its 32 x 32 block in one of two
@@ -555,13 +562,13 @@ omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap&
   const int64_t sms = omq_num_sms();
   if (!PAIR) {
     const unsigned grid = (unsigned)(tiles < sms ? tiles : sms);
-    kern<<<grid, NUM_THREADS, L::TOTAL, st>>>(ta, tb, tc, p);
+    kern<<<grid, LWC ? NUM_THREADS_LWC : NUM_THREADS, L::TOTAL, st>>>(ta, tb, tc, p);
   } else {
     const int64_t pairs = sms / 2;
     const unsigned grid = (unsigned)(2 * (tiles < pairs ? tiles : pairs));
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid, 1, 1);
-    cfg.blockDim = dim3(NUM_THREADS, 1, 1);
+    cfg.blockDim = dim3(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1, 1);
     cfg.dynamicSmemBytes = L::TOTAL;
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
@@ -693,9 +700,10 @@ omq_status gemm_launch_lwc(cudaStream_t st, int64_t M, int64_t N, int64_t K, con
   const int bn = gemm_n_tile(N);
   const bool perch = lw.group == N;
   // a group lies inside one 32-column chunk sequence of one tile; the grouped form carries no LET
-  OMQ_REQUIRE(lw.group > 0 && (perch || (lw.group % 32 == 0 && bn % lw.group == 0)), OMQ_ERR_UNSUPPORTED);
+  // a group lies inside one half of a tile (the part one epilogue warp drains)
+  OMQ_REQUIRE(lw.group > 0 && (perch || (lw.group % 32 == 0 && (bn / 2) % lw.group == 0)), OMQ_ERR_UNSUPPORTED);
   OMQ_REQUIRE(perch || (!lw.s && !lw.r && !lw.dBt && !lw.part_s && !lw.part_d), OMQ_ERR_UNSUPPORTED);
-  OMQ_REQUIRE(!perch || (lw.rowpart && lw.ntn == (int)((N + bn - 1) / bn)), OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(!perch || (lw.rowpart && lw.ntn == 2 * (int)((N + bn - 1) / bn)), OMQ_ERR_INVALID_ARG);
   OMQ_REQUIRE(perch || (lw.dgl && lw.dbl && lw.ga && lw.Mv), OMQ_ERR_INVALID_ARG);
   OMQ_REQUIRE(!lw.part_s || lw.s, OMQ_ERR_INVALID_ARG);
   OMQ_REQUIRE(!lw.part_d || lw.dBt, OMQ_ERR_INVALID_ARG);

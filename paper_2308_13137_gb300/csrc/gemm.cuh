@@ -23,8 +23,9 @@ struct GemmEpilogue {
 // thread owns one output row o of the tile and, per element, forms W~ = fl(fl(W s) r), its
 // code decision, the STE gradient d = [0 <= code <= Q] dW_hat and the h-path term.  Outputs:
 //  * per-channel (group == N): row partials of G_h = sum dW_hat dWhat/dh, G_bm = sum of dW_hat over
-//    clamped elements and dr = sum d W s, one per N tile ([3, M, ntn]); a finalize completes them;
-//  * grouped (group | N tile, no LET): dgamma_hat, dbeta_hat of every group directly;
+//    clamped elements and dr = sum d W s, one per half N tile ([3, M, ntn], ntn = 2 ceil(N / 256));
+//    a finalize completes them;
+//  * grouped (group | half N tile, no LET): dgamma_hat, dbeta_hat of every group directly;
 //  * LET column partials per 32-row quadrant ([ceil(M/32), N]): sum_o d W r (for ds) and
 //    sum_o dB~_o r_o W (for ddelta).
 struct GemmLwcEpi {
