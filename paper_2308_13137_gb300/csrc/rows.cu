@@ -256,6 +256,19 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
   const int64_t nparts = (a.T + a.rows_per_cta - 1) / a.rows_per_cta;
   const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f), o4 = make_float4(1.f, 1.f, 1.f, 1.f);
   float acc_s[NE], acc_d[NE];
+  // with column sums and rows of at most 8 K: 1/s of the thread's columns in shared memory (each
+  // thread reads back only its own slots), computed once; the RMSNorm backward also keeps x * rstd
+  // and the masked gradient of its elements in registers for pass 2
+  constexpr bool RS = SUMS && VPT <= 8;
+  constexpr bool KEEP = RS && P == AP_RMS_LET;
+  __shared__ float4 rs_sm[RS ? VPT * NT : 1];
+  float xk[KEEP ? NE : 1], dk[KEEP ? NE : 1];
+#pragma unroll
+  for (int j = 0; j < (RS ? VPT : 0); ++j) {
+    const int64_t vi = (int64_t)j * NT + tid;
+    const float4 sv = (LETP && a.s && vi < nv) ? ld4(a.s + 4 * vi) : o4;
+    rs_sm[j * NT + tid] = make_float4(__frcp_rn(sv.x), __frcp_rn(sv.y), __frcp_rn(sv.z), __frcp_rn(sv.w));
+  }
   for (int64_t p = blockIdx.x; p < nparts; p += gridDim.x) {
 #pragma unroll
     for (int k = 0; k < NE; ++k) { acc_s[k] = 0.f; acc_d[k] = 0.f; }
@@ -293,6 +306,7 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
           float4 dl = z4, sv = o4;
           if (LETP && a.delta) dl = ld4(a.delta + 4 * vi);
           if (LETP && a.s) sv = ld4(a.s + 4 * vi);
+          const float4 rs4 = RS ? rs_sm[j * NT + tid] : o4;
           float o1[4], o2[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
@@ -316,8 +330,11 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
                 acc_s[k] = fmaf(d, v, acc_s[k]);
                 acc_d[k] += d;
               }
-              const float dn = (LETP && a.s) ? __fdiv_rn(d, se) : d;
+              const int k = (4 * j + e) % NE;
+              const float rcp = RS ? f4get(rs4, e) : __frcp_rn(se);
+              const float dn = (LETP && a.s) ? d * rcp : d;
               if (P == AP_RMS_LET) dot = fmaf(dn, x * R.rstd, dot);
+              if (KEEP) { xk[k] = x * R.rstd; dk[k] = dn; }
               o1[e] = dn;
             }
           }
@@ -381,7 +398,39 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
         }
       }
       // ---- RMSNorm backward: second stream of the row ----
-      if (P == AP_RMS_LET && want_out) {
+      if (KEEP && want_out) {                    // x * rstd and dn kept from pass 1: only resid is read
+        const float mean_dot = dot_t / (float)a.C;
+#pragma unroll
+        for (int jb = 0; jb < VPT; jb += JB) {
+          float4 r4[JB];
+#pragma unroll
+          for (int jj = 0; jj < JB; ++jj) {
+            const int64_t vi = (int64_t)(jb + jj) * NT + tid;
+            r4[jj] = (jb + jj < VPT && vi < nv && a.resid) ? ld4(a.resid + t * a.lddx + 4 * vi) : z4;
+          }
+#pragma unroll
+          for (int jj = 0; jj < JB; ++jj) {
+            const int j = jb + jj;
+            const int64_t vi = (int64_t)j * NT + tid;
+            if (j >= VPT || vi >= nv) continue;
+            float o[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const int k = (4 * j + e) % NE;
+              const int64_t c = 4 * vi + e;
+              float dn = dk[k];
+              if (c == iM || c == im) {
+                const float rc = f4get(rs_sm[j * NT + tid], e);
+                if (c == iM) dn = fmaf(GaM, rc, dn);
+                if (c == im) dn = fmaf(Gbt, rc, dn);
+              }
+              o[e] = R.rstd * (dn - xk[k] * mean_dot) + f4get(r4[jj], e);
+            }
+            if (a.dX) *reinterpret_cast<float4*>(a.dX + t * a.lddx + 4 * vi) = make_float4(o[0], o[1], o[2], o[3]);
+            if (a.dXb) st_bf16x4(a.dXb + t * a.lddxb + 4 * vi, o);
+          }
+        }
+      } else if (P == AP_RMS_LET && want_out) {
         const float mean_dot = dot_t / (float)a.C;
 #pragma unroll
         for (int jb = 0; jb < VPT; jb += JB) {
@@ -632,7 +681,20 @@ __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
   const bool quant = a.abits < 16;
   const float Q = (float)((1 << (quant ? a.abits : 1)) - 1);
   const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
-  float acc_q[NE], acc_k[NE];
+  float acc_q[NE], acc_k[NE], rq[NE];      // rq: 1/s_a of the thread's query columns, computed once
+#pragma unroll
+  for (int j = 0; j < PPT; ++j) {
+    const int p = j * NT + tid;
+    const int e1 = (p >> 4) * 128 + 4 * (p & 15);
+    const bool ok = a.sa_exp != nullptr && p < a.H * 16;
+    const float4 s1 = ok ? ld4(a.sa_exp + e1) : make_float4(1.f, 1.f, 1.f, 1.f);
+    const float4 s2 = ok ? ld4(a.sa_exp + e1 + 64) : make_float4(1.f, 1.f, 1.f, 1.f);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      rq[8 * j + e] = __frcp_rn(f4get(s1, e));
+      rq[8 * j + 4 + e] = __frcp_rn(f4get(s2, e));
+    }
+  }
 #pragma unroll
   for (int k = 0; k < NE; ++k) { acc_q[k] = 0.f; acc_k[k] = 0.f; }
   const int t0 = blockIdx.x * a.rows_per_cta, t1 = min(a.T, t0 + a.rows_per_cta);
@@ -708,10 +770,9 @@ __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
           }
           if (let) {
             const int k1 = 8 * j + e, k2 = 8 * j + 4 + e;
-            if (seg == 0) {
-              const float s1 = a.sa_exp[e1 + e], s2 = a.sa_exp[e1 + 64 + e];
-              if (sums) { acc_q[k1] -= d1 * v1 / s1; acc_q[k2] -= d2 * v2 / s2; }
-              d1 = __fdiv_rn(d1, s1); d2 = __fdiv_rn(d2, s2);
+            if (seg == 0) {                      // the 1/s_a of the ds_a terms is applied once, at the end
+              if (sums) { acc_q[k1] = fmaf(-d1, v1, acc_q[k1]); acc_q[k2] = fmaf(-d2, v2, acc_q[k2]); }
+              d1 *= rq[k1]; d2 *= rq[k2];
             } else {
               if (sums) { acc_k[k1] += d1 * r1; acc_k[k2] += d2 * r2; }
               d1 = __fmul_rn(d1, a.sa[e1 + e]); d2 = __fmul_rn(d2, a.sa[e1 + 64 + e]);
@@ -763,8 +824,7 @@ __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
               if (jx != j || ex != e) continue;
               const int k1 = 8 * jx + ex, k2 = 8 * jx + 4 + ex;
               if (seg == 0) {
-                const float s1 = a.sa_exp[first], s2 = a.sa_exp[first + 64];
-                if (sums) { acc_q[k1] -= ro1 * v1 / s1; acc_q[k2] -= ro2 * v2 / s2; }
+                if (sums) { acc_q[k1] = fmaf(-ro1, v1, acc_q[k1]); acc_q[k2] = fmaf(-ro2, v2, acc_q[k2]); }
               } else {
                 if (sums) { acc_k[k1] += ro1 * r1; acc_k[k2] += ro2 * r2; }
               }
@@ -787,8 +847,8 @@ __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         if (p < a.H * 16) {
-          a.part_q[(int64_t)blockIdx.x * dq + e1 + e] = acc_q[8 * j + e];
-          a.part_q[(int64_t)blockIdx.x * dq + e1 + 64 + e] = acc_q[8 * j + 4 + e];
+          a.part_q[(int64_t)blockIdx.x * dq + e1 + e] = acc_q[8 * j + e] * rq[8 * j + e];
+          a.part_q[(int64_t)blockIdx.x * dq + e1 + 64 + e] = acc_q[8 * j + 4 + e] * rq[8 * j + 4 + e];
         }
         if (p < a.Hkv * 16) {
           a.part_k[(int64_t)blockIdx.x * dkv + e1 + e] = acc_k[8 * j + e];
