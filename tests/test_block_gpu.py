@@ -45,6 +45,11 @@ SMALL = [
     I.BlockShape("w4a6_let", T=256, d=256, n_heads=2, n_kv=2, ffn=512, wbits=4, abits=6, group=0, let=1),
     I.BlockShape("w6a6_let", T=256, d=256, n_heads=2, n_kv=2, ffn=512, wbits=6, abits=6, group=0, let=1),
     I.BlockShape("w8a4_let", T=256, d=256, n_heads=2, n_kv=2, ffn=512, wbits=8, abits=4, group=0, let=1),
+    # mid-size blocks (T = d = 1024): every product spans tens of 256 x 256 tiles and at least 16 k-blocks,
+    # including the weight-gradient products with the LWC backward fused in their epilogue (per channel with LET,
+    # and grouped)
+    I.BlockShape("w4a4_let_mid", T=1024, d=1024, n_heads=8, n_kv=8, ffn=2816, wbits=4, abits=4, group=0, let=1),
+    I.BlockShape("w3a16_g128_mid", T=1024, d=1024, n_heads=8, n_kv=4, ffn=2816, wbits=3, abits=16, group=128, let=0),
 ]
 
 

@@ -112,3 +112,36 @@ def test_gemm_large_weight_shape(cuda_lib):
     rows = torch.randint(0, M, (64,), generator=g)
     ref = A[rows].double() @ B.double().T
     assert _rel(C.cpu()[rows], ref) < 2e-5
+
+
+# Shapes whose tiles do not fill whole waves of the 76 CTA pairs (or 152 CTAs): fewer tiles than
+# CTAs, a partial last wave, ragged rows, short K; with bias and residual in the epilogue.
+SPLIT_CASES = [  # M, N, K, a_kmajor, b_kmajor
+    (1024, 2816, 4096, 1, 1),   # 44 pair tiles: fewer tiles than workers, each tile cut over 2-3 pairs
+    (2048, 5376, 1024, 1, 0),   # 168 pair tiles: one wave of whole tiles, then a cut tail
+    (1000, 1152, 2048, 0, 1),   # one CTA per 128 x 128 tile (N not a multiple of 256), ragged M, 72 tiles
+    (4096, 2304, 512, 0, 0),    # 144 pair tiles of 8 k-blocks
+]
+
+
+@pytest.mark.parametrize("M,N,K,ak,bk", SPLIT_CASES)
+def test_gemm_split_tail(cuda_lib, M, N, K, ak, bk):
+    g = torch.Generator().manual_seed(M + N + K + 3 * ak + bk)
+    A = _bf16((M, K) if ak else (K, M), g)
+    B = _bf16((N, K) if bk else (K, N), g, 0.05)
+    bias = torch.randn(N, generator=g)
+    R = torch.randn(M, N, generator=g)
+    ref = 0.5 * (_logical(A, ak, M, K).double() @ _logical(B, bk, N, K).double().T) + bias.double() + R.double()
+    Ad, Bd, bd, Rd = A.cuda(), B.cuda(), bias.cuda(), R.cuda()
+    outs = []
+    for _ in range(3):   # repeated launches give identical results
+        C = torch.full((M, N), float("nan"), device="cuda")
+        Cb = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+        _lib.omq_gemm_bf16(M, N, K, 1, Ad, K if ak else M, 0, ak, Bd, K if bk else N, 0, bk, C, Cb, N, 0, alpha=0.5,
+                           bias=bd, R=Rd, ldr=N)
+        outs.append((C.cpu(), Cb.cpu()))
+    torch.cuda.synchronize()
+    for C, Cb in outs:
+        assert _rel(C, ref) < 2e-5
+        assert torch.equal(Cb, C.to(torch.bfloat16))
+        assert torch.equal(C, outs[0][0])
