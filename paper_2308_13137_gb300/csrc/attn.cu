@@ -2,29 +2,34 @@
 // gradients (the q/k/v row kernels live in rows.cu, the attention itself in flash.cu).
 #include "attn.cuh"
 
-// angle t * theta^(-2j/hd): the frequency and the product are formed in double, the angle is reduced
-// to [-pi, pi] in double, and sin/cos of the reduced angle are taken in float.
-__global__ void rope_table_kernel(int T, int hd, double theta, float* cs) {
-  __shared__ double inv[128];
-  const int half = hd / 2;
-  for (int j = threadIdx.x; j < half; j += blockDim.x) inv[j] = pow(theta, -2.0 * (double)j / (double)hd);
-  __syncthreads();
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= T * half) return;
-  const int t = i / half, j = i % half;
+#include <cmath>
+
+// angle t * theta^(-2j/hd): the frequencies are formed on the host in double, the product and the
+// reduction of the angle to [-pi, pi] in double on the device, and sin/cos of the reduced angle in
+// float.  One thread per (position, frequency).
+struct RopeFreq { double inv[128]; };
+
+__global__ void rope_table_kernel(int T, int half, RopeFreq f, float* cs) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (int64_t)T * half) return;
+  const int t = (int)(i / half), j = (int)(i % half);
   const double two_pi = 6.283185307179586476925286766559;
-  double ang = (double)t * inv[j];
-  ang -= two_pi * rint(ang / two_pi);
+  const double inv_two_pi = 0.15915494309189533576888376337251;
+  double ang = (double)t * f.inv[j];
+  ang = fma(-two_pi, rint(ang * inv_two_pi), ang);
   float sv, cv;
   sincosf((float)ang, &sv, &cv);
-  cs[2 * i] = cv;
-  cs[2 * i + 1] = sv;
+  reinterpret_cast<float2*>(cs)[i] = make_float2(cv, sv);
 }
 
 omq_status rope_table(cudaStream_t st, int T, int hd, float theta, float* cs) {
-  OMQ_REQUIRE(hd <= 256, OMQ_ERR_UNSUPPORTED);
-  int n = T * (hd / 2);
-  rope_table_kernel<<<(n + 255) / 256, 256, 0, st>>>(T, hd, (double)theta, cs);
+  OMQ_REQUIRE(hd <= 256 && hd % 2 == 0, OMQ_ERR_UNSUPPORTED);
+  OMQ_REQUIRE(omq_aligned16(cs), OMQ_ERR_ALIGN);
+  RopeFreq f;
+  const int half = hd / 2;
+  for (int j = 0; j < half; ++j) f.inv[j] = std::pow((double)theta, -2.0 * (double)j / (double)hd);
+  const int64_t n = (int64_t)T * half;
+  rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(T, half, f, cs);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }

@@ -325,6 +325,10 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   BlockWS& w = c.ws;
   const omq_qcfg& cfg = c.cfg;
   const omq_block_params* th = c.th;
+  // s_o, delta_o, s_a per query channel (broadcast over the query heads of a kv head)
+  const float* so_e = c.rep > 1 ? c.ws.so_exp : th->so;
+  const float* do_e = c.rep > 1 ? c.ws.do_exp : th->do_;
+  const float* sa_e = c.rep > 1 ? c.ws.sa_exp : th->sa;
   int32_t* status = cfg.dev_status;
   const bf16* Wqkv = (const bf16*)c.w->wqkv;
   const bf16* Wo = (const bf16*)c.w->wo;
@@ -334,9 +338,11 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   OMQ_TRY(rope_table(st, (int)c.T, (int)c.hd, c.s.rope_theta, w.cs));
   if (c.let) {
     OMQ_TRY(qkv_row_vectors(st, (int)c.dq, (int)c.dkv, th->so, th->do_, w.r_qkv, w.shift_qkv));
-    OMQ_TRY(gqa_expand(st, th->so, w.so_exp, (int)c.Hkv, (int)c.rep, (int)c.hd, 0));
-    OMQ_TRY(gqa_expand(st, th->do_, w.do_exp, (int)c.Hkv, (int)c.rep, (int)c.hd, 0));
-    OMQ_TRY(gqa_expand(st, th->sa, w.sa_exp, (int)c.Hkv, (int)c.rep, (int)c.hd, 0));
+    if (c.rep > 1) {                            // one kv head per query head: the vectors serve as they are
+      OMQ_TRY(gqa_expand(st, th->so, w.so_exp, (int)c.Hkv, (int)c.rep, (int)c.hd, 0));
+      OMQ_TRY(gqa_expand(st, th->do_, w.do_exp, (int)c.Hkv, (int)c.rep, (int)c.hd, 0));
+      OMQ_TRY(gqa_expand(st, th->sa, w.sa_exp, (int)c.Hkv, (int)c.rep, (int)c.hd, 0));
+    }
   }
   // ---- LET (Eq. 3) + LWC (Eq. 2) on every weight: q|k|v here, the others on the auxiliary stream
   // while the attention half runs -------------------------------------------------------------------
@@ -346,8 +352,8 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   OMQ_TRY(lwc_fwd_launch(st, lwc_args(Wqkv, c.nqkv, c.d, cfg, c.let ? th->s1 : nullptr, c.let ? w.r_qkv : nullptr,
                                       th->gamma_qkv, th->beta_qkv, w.Wqkv_h, w.sq_qkv, c.let ? th->d1 : nullptr,
                                       c.let ? w.shift_qkv : nullptr, c.let ? w.B_qkv : nullptr)));
-  OMQ_TRY(lwc_fwd_launch(ax, lwc_args(Wo, c.d, c.dq, cfg, c.let ? w.so_exp : nullptr, nullptr, th->gamma_o, th->beta_o,
-                                      w.Wo_h, w.sq_o, c.let ? w.do_exp : nullptr, nullptr, c.let ? w.B_o : nullptr)));
+  OMQ_TRY(lwc_fwd_launch(ax, lwc_args(Wo, c.d, c.dq, cfg, c.let ? so_e : nullptr, nullptr, th->gamma_o, th->beta_o,
+                                      w.Wo_h, w.sq_o, c.let ? do_e : nullptr, nullptr, c.let ? w.B_o : nullptr)));
   OMQ_REQUIRE(cudaEventRecord(ev[1], ax) == cudaSuccess, OMQ_ERR_CUDA);
   OMQ_TRY(lwc_fwd_launch(ax, lwc_args(Wgu, 2 * c.f, c.d, cfg, c.let ? th->s2 : nullptr, nullptr, th->gamma_gu,
                                       th->beta_gu, w.Wgu_h, w.sq_gu, c.let ? th->d2 : nullptr, nullptr,
@@ -367,7 +373,7 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
                   nullptr, status));
   QkvArgs qa{};
   qa.T = (int)c.T; qa.H = (int)c.H; qa.Hkv = (int)c.Hkv; qa.hd = (int)c.hd; qa.Y = w.Yqkv; qa.ldy = c.nqkv; qa.cs = w.cs;
-  qa.sa_exp = c.let ? w.sa_exp : nullptr; qa.sa = c.let ? th->sa : nullptr;
+  qa.sa_exp = c.let ? sa_e : nullptr; qa.sa = c.let ? th->sa : nullptr;
   qa.Qh = w.Qh; qa.Kh = w.Kh; qa.Vh = w.Vh;
   qa.h = w.sqkv.h; qa.z = w.sqkv.z; qa.imax = w.sqkv.imax; qa.imin = w.sqkv.imin; qa.abits = cfg.abits; qa.eps = cfg.h_eps;
   OMQ_TRY(qkv_fwd_launch(st, qa));
@@ -406,6 +412,9 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   BlockWS& w = c.ws;
   const omq_qcfg& cfg = c.cfg;
   const omq_block_params* th = c.th;
+  // s_o, delta_o, s_a per query channel (broadcast over the query heads of a kv head)
+  const float* so_e = c.rep > 1 ? c.ws.so_exp : th->so;
+  const float* sa_e = c.rep > 1 ? c.ws.sa_exp : th->sa;
   int32_t* status = cfg.dev_status;
   const bf16* Wqkv = (const bf16*)c.w->wqkv;
   const bf16* Wo = (const bf16*)c.w->wo;
@@ -452,16 +461,19 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   OMQ_TRY(act_bwd_launch(st, bb));
   if (c.let) {
     OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[6], 0) == cudaSuccess, OMQ_ERR_CUDA);   // LWC part of ds2, dd2
-    OMQ_TRY(omq_colsum_partials(st, bb.part_s, (c.T + 3) / 4, c.d, g->s2, 1.f, 1));
-    OMQ_TRY(omq_colsum_partials(st, bb.part_d, (c.T + 3) / 4, c.d, g->d2, 1.f, 1));
+    OMQ_TRY(omq_colsum_partials2(st, ColsumJob{bb.part_s, (c.T + 3) / 4, c.d, g->s2, 1.f, 1},
+                                 ColsumJob{bb.part_d, (c.T + 3) / 4, c.d, g->d2, 1.f, 1}));
   }
 
   // ---- o_proj -------------------------------------------------------------------------------------
   if (c.let) OMQ_TRY(colsum_rows(st, w.dh1, c.T, c.d, c.d, w.part, w.dB_o, 1.f, 0));
   OMQ_TRY(join(st, ax, ev[7]));
-  OMQ_TRY(lwc_bwd_dw(ax, c.T, w.dh1_b, w.O_h, Wo, c.d, c.dq, cfg, c.let ? w.so_exp : nullptr, nullptr, th->gamma_o,
+  // ds_o, ddelta_o per query channel; with one query head per kv head straight into the gradients
+  const bool fold_o = c.rep > 1;
+  OMQ_TRY(lwc_bwd_dw(ax, c.T, w.dh1_b, w.O_h, Wo, c.d, c.dq, cfg, c.let ? so_e : nullptr, nullptr, th->gamma_o,
                      th->beta_o, w.sq_o, g->gamma_o, g->beta_o, nullptr, c.let ? w.dB_o : nullptr,
-                     c.let ? w.vtmp0 : nullptr, c.let ? w.vtmp1 : nullptr, 0, w.part_aux, w.dW, status));
+                     c.let ? (fold_o ? w.vtmp0 : g->so) : nullptr, c.let ? (fold_o ? w.vtmp1 : g->do_) : nullptr,
+                     fold_o ? 0 : acc, w.part_aux, w.dW, status));
   OMQ_REQUIRE(cudaEventRecord(ev[8], ax) == cudaSuccess, OMQ_ERR_CUDA);
   OMQ_TRY(gemm_dx(st, c.T, c.d, c.dq, w.dh1_b, w.Wo_h, w.dOh, status));
   ActBwdArgs bo{};
@@ -480,7 +492,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   OMQ_TRY(flash_bwd_launch(st, fa));
   QkvArgs qa{};
   qa.T = (int)c.T; qa.H = (int)c.H; qa.Hkv = (int)c.Hkv; qa.hd = (int)c.hd; qa.Y = w.Yqkv; qa.ldy = c.nqkv; qa.cs = w.cs;
-  qa.sa_exp = c.let ? w.sa_exp : nullptr; qa.sa = c.let ? th->sa : nullptr;
+  qa.sa_exp = c.let ? sa_e : nullptr; qa.sa = c.let ? th->sa : nullptr;
   qa.h = w.sqkv.h; qa.z = w.sqkv.z; qa.imax = w.sqkv.imax; qa.imin = w.sqkv.imin; qa.abits = cfg.abits; qa.eps = cfg.h_eps;
   qa.dQKV = w.dQKV; qa.ldd = c.nqkv; qa.dY = w.dYqkv; qa.dYb = w.dYqkv_b;
   const int64_t nsq = qkv_bwd_nslab((int)c.T);
@@ -488,13 +500,19 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   qa.part_k = c.let ? w.part + nsq * c.dq : nullptr;
   OMQ_TRY(qkv_bwd_launch(st, qa, nullptr));
   if (c.let) {
-    OMQ_TRY(omq_colsum_partials(st, qa.part_q, nsq, c.dq, w.vtmp2, 1.f, 0));
-    OMQ_TRY(omq_colsum_partials(st, qa.part_k, nsq, c.dkv, g->sa, 1.f, acc));
-    OMQ_TRY(gqa_fold(st, w.vtmp2, g->sa, (int)c.Hkv, (int)c.rep, (int)c.hd, 1));
+    if (c.rep == 1) {       // q and k partials are one contiguous [2 nslab, d_kv] array over the same channels
+      OMQ_TRY(omq_colsum_partials(st, qa.part_q, 2 * nsq, c.dq, g->sa, 1.f, acc));
+    } else {
+      OMQ_TRY(omq_colsum_partials2(st, ColsumJob{qa.part_q, nsq, c.dq, w.vtmp2, 1.f, 0},
+                                   ColsumJob{qa.part_k, nsq, c.dkv, g->sa, 1.f, acc}));
+      OMQ_TRY(gqa_fold(st, w.vtmp2, g->sa, (int)c.Hkv, (int)c.rep, (int)c.hd, 1));
+    }
     // [v, out] pair: o_proj column-scale part (folded over the query heads), then v rows
     OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[8], 0) == cudaSuccess, OMQ_ERR_CUDA);   // o_proj LWC backward
-    OMQ_TRY(gqa_fold(st, w.vtmp0, g->so, (int)c.Hkv, (int)c.rep, (int)c.hd, acc));
-    OMQ_TRY(gqa_fold(st, w.vtmp1, g->do_, (int)c.Hkv, (int)c.rep, (int)c.hd, acc));
+    if (fold_o) {
+      OMQ_TRY(gqa_fold(st, w.vtmp0, g->so, (int)c.Hkv, (int)c.rep, (int)c.hd, acc));
+      OMQ_TRY(gqa_fold(st, w.vtmp1, g->do_, (int)c.Hkv, (int)c.rep, (int)c.hd, acc));
+    }
   }
 
   // ---- q / k / v projections ---------------------------------------------------------------------------
@@ -516,8 +534,8 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
     ba.dX = nullptr; ba.dXb = nullptr; ba.part_s = w.part; ba.part_d = w.part + ((c.T + 3) / 4) * c.d;
     ba.rows_per_cta = 4; ba.abits = cfg.abits; ba.eps = cfg.h_eps;
     OMQ_TRY(act_bwd_launch(st, ba));
-    OMQ_TRY(omq_colsum_partials(st, ba.part_s, (c.T + 3) / 4, c.d, g->s1, 1.f, 1));
-    OMQ_TRY(omq_colsum_partials(st, ba.part_d, (c.T + 3) / 4, c.d, g->d1, 1.f, 1));
+    OMQ_TRY(omq_colsum_partials2(st, ColsumJob{ba.part_s, (c.T + 3) / 4, c.d, g->s1, 1.f, 1},
+                                 ColsumJob{ba.part_d, (c.T + 3) / 4, c.d, g->d1, 1.f, 1}));
   }
   OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[10], 0) == cudaSuccess, OMQ_ERR_CUDA);    // every auxiliary launch
   return OMQ_OK;
@@ -695,8 +713,8 @@ omq_status omq_qlinear_bwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t 
     a.part_d = let ? part + ((T + 3) / 4) * Cin : nullptr;
     OMQ_TRY(act_bwd_launch(st, a));
     if (let) {
-      OMQ_TRY(omq_colsum_partials(st, a.part_s, (T + 3) / 4, Cin, ds, 1.f, 1));
-      OMQ_TRY(omq_colsum_partials(st, a.part_d, (T + 3) / 4, Cin, ddelta, 1.f, 1));
+      OMQ_TRY(omq_colsum_partials2(st, ColsumJob{a.part_s, (T + 3) / 4, Cin, ds, 1.f, 1},
+                                   ColsumJob{a.part_d, (T + 3) / 4, Cin, ddelta, 1.f, 1}));
     }
   }
   return OMQ_OK;

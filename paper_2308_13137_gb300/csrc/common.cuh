@@ -219,5 +219,11 @@ __device__ __forceinline__ float2 block_sum2(float a, float b, float* smem) {
 __global__ void omq_colsum_partials_kernel(const float* __restrict__ part, int64_t P, int64_t C,
                                            float* __restrict__ out, float scale, int accumulate);
 
+// one column reduction out[c] (+)= scale * sum_p part[p, c] of a [P, C] row-major array
+struct ColsumJob {
+  const float* part; int64_t P, C; float* out; float scale; int accumulate;
+};
+// two independent column reductions in one launch
+omq_status omq_colsum_partials2(cudaStream_t st, const ColsumJob& a, const ColsumJob& b);
 omq_status omq_colsum_partials(cudaStream_t st, const float* part, int64_t P, int64_t C, float* out,
                                float scale, int accumulate);

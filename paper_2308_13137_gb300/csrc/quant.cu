@@ -221,6 +221,108 @@ __global__ void __launch_bounds__(256, 4) lwc_fwd_kernel(LwcFwdArgs a) {
   }
 }
 
+// One group per row, one CTA per row: the row lives in registers (CPT 8-column chunks per thread)
+// between the block reduction of max / min (and the LET bias dot) and the quantize pass, so every
+// weight is read from HBM once.  The weights are streamed with evict-first loads so that W_hat,
+// which the next product reads, stays in L2.  The first index of the max / min is searched only by
+// the threads whose own extreme equals the row's.  Every value matches lwc_fwd_kernel<1> bit for
+// bit except the LET bias dot, whose summation order differs.
+template <int NT, int CPT>
+__global__ void __launch_bounds__(NT) lwc_fwd_row_kernel(LwcFwdArgs a) {
+  constexpr int NW = NT / 32;
+  __shared__ float red[3][NW];
+  __shared__ int sidx[2];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t o = blockIdx.x;
+  const int64_t nchunk = a.Cin / 8;
+  const float Q = (float)((1 << a.wbits) - 1);
+  const float rr = a.r ? a.r[o] : 1.f;
+  const uint4* Wrow = reinterpret_cast<const uint4*>(a.W + o * a.Cin);
+  uint4 raw[CPT];
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) {
+    const int64_t c = (int64_t)j * NT + tid;
+    raw[j] = c < nchunk ? __ldcs(Wrow + c) : make_uint4(0, 0, 0, 0);
+  }
+  if (tid == 0) { sidx[0] = 0x7fffffff; sidx[1] = 0x7fffffff; }
+  float wt[CPT][8];
+  float M = -INFINITY, m = INFINITY, dot = 0.f;
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) {
+    const int64_t c = (int64_t)j * NT + tid;
+    if (c < nchunk) {
+      float w8[8], sv[8];
+      unpack_bf16x8(raw[j], w8);
+      load8(a.s, c, sv, 1.f);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        wt[j][e] = __fmul_rn(__fmul_rn(w8[e], sv[e]), rr);
+        M = fmaxf(M, wt[j][e]); m = fminf(m, wt[j][e]);
+      }
+      if (a.Bt) {
+        float dv[8];
+        load8(a.bias_delta, c, dv, 0.f);
+        float acc = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc = fmaf(w8[e], dv[e], acc);
+        dot += acc;
+      }
+    }
+  }
+  float bM = M, bm = m, bd = dot;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    bM = fmaxf(bM, __shfl_xor_sync(0xffffffffu, bM, off));
+    bm = fminf(bm, __shfl_xor_sync(0xffffffffu, bm, off));
+    bd += __shfl_xor_sync(0xffffffffu, bd, off);
+  }
+  if (lane == 0) { red[0][warp] = bM; red[1][warp] = bm; red[2][warp] = bd; }
+  __syncthreads();
+  bM = red[0][0]; bm = red[1][0]; bd = red[2][0];
+#pragma unroll
+  for (int w = 1; w < NW; ++w) { bM = fmaxf(bM, red[0][w]); bm = fminf(bm, red[1][w]); bd += red[2][w]; }
+  float ga = 1.f, gb = 1.f;
+  if (a.lwc) { ga = omq_sigmoid(a.gl[o]); gb = omq_sigmoid(a.bl[o]); }
+  const QState qs = omq_qstate(bM, bm, ga, gb, Q, a.eps);
+  if (M == bM || m == bm) {
+    int iM = 0x7fffffff, im = 0x7fffffff;
+#pragma unroll
+    for (int j = CPT - 1; j >= 0; --j) {
+      const int64_t c = (int64_t)j * NT + tid;
+      if (c < nchunk) {
+#pragma unroll
+        for (int e = 7; e >= 0; --e) {
+          if (wt[j][e] == bM) iM = (int)(c * 8 + e);
+          if (wt[j][e] == bm) im = (int)(c * 8 + e);
+        }
+      }
+    }
+    if (iM != 0x7fffffff) atomicMin(&sidx[0], iM);
+    if (im != 0x7fffffff) atomicMin(&sidx[1], im);
+  }
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) {
+    const int64_t c = (int64_t)j * NT + tid;
+    if (c < nchunk) lwc_store(a, o, c, wt[j], qs, Q);
+  }
+  __syncthreads();
+  if (tid == 0) {
+    a.h[o] = qs.h; a.z[o] = (int32_t)qs.z; a.imax[o] = sidx[0]; a.imin[o] = sidx[1];
+    if (a.ga_out) { a.ga_out[o] = ga; a.gb_out[o] = gb; }
+    if (a.M_out) { a.M_out[o] = bM; a.m_out[o] = bm; }
+    if (a.Bt) a.Bt[o] = rr * (bd - (a.bias_shift ? a.bias_shift[o] : 0.f));
+  }
+}
+
+template <int NT>
+static void lwc_fwd_row_go(cudaStream_t st, const LwcFwdArgs& a, int64_t cpt) {
+  const unsigned grid = (unsigned)a.Cout;
+  if (cpt <= 2) lwc_fwd_row_kernel<NT, 2><<<grid, NT, 0, st>>>(a);
+  else if (cpt <= 4) lwc_fwd_row_kernel<NT, 4><<<grid, NT, 0, st>>>(a);
+  else if (cpt <= 6) lwc_fwd_row_kernel<NT, 6><<<grid, NT, 0, st>>>(a);
+  else lwc_fwd_row_kernel<NT, 8><<<grid, NT, 0, st>>>(a);
+}
+
 static bool lwc_group_ok(int64_t Cin, int g) {
   if (g == Cin) return Cin % 8 == 0;
   if (g < 8 || g > 256 || (g & (g - 1))) return false;
@@ -231,7 +333,11 @@ static bool lwc_group_ok(int64_t Cin, int g) {
 omq_status lwc_fwd_launch(cudaStream_t st, const LwcFwdArgs& a) {
   OMQ_REQUIRE(lwc_group_ok(a.Cin, a.group), OMQ_ERR_UNSUPPORTED);
   const unsigned grid = (unsigned)((a.Cout + 7) / 8);
+  const int64_t nchunk = a.Cin / 8;
   if (a.wbits >= 16) lwc_fwd_kernel<0><<<grid, 256, 0, st>>>(a);
+  else if (a.group == a.Cin && nchunk <= 128 * 8) lwc_fwd_row_go<128>(st, a, (nchunk + 127) / 128);
+  else if (a.group == a.Cin && nchunk <= 256 * 8) lwc_fwd_row_go<256>(st, a, (nchunk + 255) / 256);
+  else if (a.group == a.Cin && nchunk <= 512 * 8) lwc_fwd_row_go<512>(st, a, (nchunk + 511) / 512);
   else if (a.group == a.Cin) lwc_fwd_kernel<1><<<grid, 256, 0, st>>>(a);
   else lwc_fwd_kernel<2><<<grid, 256, 0, st>>>(a);
   OMQ_LAUNCH_CHECK();
@@ -534,12 +640,14 @@ omq_status lwc_bwd_fused_finish(cudaStream_t st, const LwcBwdArgs& a0, float* ro
   const bool perch = a.group == a.Cin;
   OMQ_REQUIRE(a.ga && a.gb, OMQ_ERR_INVALID_ARG);
   // the LET column sums first, so that the finalize can add the max/min routing on top
-  if (a.ds) {
-    OMQ_REQUIRE(part_s, OMQ_ERR_INVALID_ARG);
+  const bool want_s = a.ds != nullptr, want_d = a.ddelta && a.dBt;
+  OMQ_REQUIRE((!want_s || part_s) && (!want_d || part_d), OMQ_ERR_INVALID_ARG);
+  if (want_s && want_d) {
+    OMQ_TRY(omq_colsum_partials2(st, ColsumJob{part_s, nparts, a.Cin, a.ds, 1.f, a.accumulate_sd},
+                                 ColsumJob{part_d, nparts, a.Cin, a.ddelta, 1.f, a.accumulate_sd}));
+  } else if (want_s) {
     OMQ_TRY(omq_colsum_partials(st, part_s, nparts, a.Cin, a.ds, 1.f, a.accumulate_sd));
-  }
-  if (a.ddelta && a.dBt) {
-    OMQ_REQUIRE(part_d, OMQ_ERR_INVALID_ARG);
+  } else if (want_d) {
     OMQ_TRY(omq_colsum_partials(st, part_d, nparts, a.Cin, a.ddelta, 1.f, a.accumulate_sd));
   }
   if (perch || a.dr) {
@@ -624,9 +732,16 @@ __global__ void omq_colsum_partials_kernel(const float* __restrict__ part, int64
 #define COLSUM_CLUSTER 8
 __device__ __forceinline__ void add4(float4& a, const float4 b) { a.x += b.x; a.y += b.y; a.z += b.z; a.w += b.w; }
 
+// blockIdx.z selects one of two independent reductions of one launch
 __global__ void __cluster_dims__(1, COLSUM_CLUSTER, 1) __launch_bounds__(256)
-    colsum_cluster_kernel(const float* __restrict__ part, int64_t P, int64_t C, float* __restrict__ out, float scale,
-                          int accumulate) {
+    colsum_cluster_kernel(ColsumJob j0, ColsumJob j1) {
+  const ColsumJob& J = blockIdx.z == 0 ? j0 : j1;
+  const float* __restrict__ part = J.part;
+  const int64_t P = J.P, C = J.C;
+  float* __restrict__ out = J.out;
+  const float scale = J.scale;
+  const int accumulate = J.accumulate;
+  if ((int64_t)blockIdx.x * 128 >= C) return;     // the narrower job of a pair: whole cluster leaves
   __shared__ float4 red[8][32];
   __shared__ float4 cta_sum[32];
   cg::cluster_group cluster = cg::this_cluster();
@@ -668,11 +783,28 @@ __global__ void __cluster_dims__(1, COLSUM_CLUSTER, 1) __launch_bounds__(256)
   cluster.sync();                  // keep every CTA's shared memory alive until CTA 0 has read it
 }
 
+static bool colsum_vec_ok(const ColsumJob& j) {
+  return j.C % 4 == 0 && omq_aligned16(j.part) && omq_aligned16(j.out);
+}
+
+omq_status omq_colsum_partials2(cudaStream_t st, const ColsumJob& a, const ColsumJob& b) {
+  if (!colsum_vec_ok(a) || !colsum_vec_ok(b)) {
+    OMQ_TRY(omq_colsum_partials(st, a.part, a.P, a.C, a.out, a.scale, a.accumulate));
+    return omq_colsum_partials(st, b.part, b.P, b.C, b.out, b.scale, b.accumulate);
+  }
+  const int64_t C = a.C > b.C ? a.C : b.C;
+  dim3 grid((unsigned)((C / 4 + 31) / 32), COLSUM_CLUSTER, 2);
+  colsum_cluster_kernel<<<grid, 256, 0, st>>>(a, b);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
 omq_status omq_colsum_partials(cudaStream_t st, const float* part, int64_t P, int64_t C, float* out,
                                float scale, int accumulate) {
-  if (C % 4 == 0 && omq_aligned16(part) && omq_aligned16(out)) {
+  ColsumJob j{part, P, C, out, scale, accumulate};
+  if (colsum_vec_ok(j)) {
     dim3 grid((unsigned)((C / 4 + 31) / 32), COLSUM_CLUSTER);
-    colsum_cluster_kernel<<<grid, 256, 0, st>>>(part, P, C, out, scale, accumulate);
+    colsum_cluster_kernel<<<grid, 256, 0, st>>>(j, j);
   } else {
     omq_colsum_partials_kernel<<<(unsigned)((C + 31) / 32), 256, 0, st>>>(part, P, C, out, scale, accumulate);
   }
@@ -691,12 +823,48 @@ __global__ void colsum_rows_kernel(const float* __restrict__ X, int64_t T, int64
   part[(int64_t)blockIdx.y * N + n] = s;
 }
 
+// the same with 16-byte loads: a CTA covers 128 columns x 128 rows, lane l of warp w reads
+// columns 4l .. 4l+3 of rows w, w + 8, ... (four loads in flight), and the eight warp sums are added
+// in warp order
+__global__ void __launch_bounds__(256) colsum_rows_vec_kernel(const float* __restrict__ X, int64_t T, int64_t N,
+                                                              int64_t ldx, float* __restrict__ part) {
+  __shared__ float4 red[8][32];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t c = (int64_t)blockIdx.x * 128 + 4 * lane;
+  const int64_t t0 = (int64_t)blockIdx.y * 128, t1 = min(T, t0 + 128);
+  float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (c < N) {
+    int64_t t = t0 + w;
+    for (; t + 24 < t1; t += 32) {
+      const float4 v0 = __ldg(reinterpret_cast<const float4*>(X + t * ldx + c));
+      const float4 v1 = __ldg(reinterpret_cast<const float4*>(X + (t + 8) * ldx + c));
+      const float4 v2 = __ldg(reinterpret_cast<const float4*>(X + (t + 16) * ldx + c));
+      const float4 v3 = __ldg(reinterpret_cast<const float4*>(X + (t + 24) * ldx + c));
+      add4(s, v0); add4(s, v1); add4(s, v2); add4(s, v3);
+    }
+    for (; t < t1; t += 8) add4(s, __ldg(reinterpret_cast<const float4*>(X + t * ldx + c)));
+  }
+  red[w][lane] = s;
+  __syncthreads();
+  if (w == 0 && c < N) {
+    float4 r = red[0][lane];
+#pragma unroll
+    for (int k = 1; k < 8; ++k) add4(r, red[k][lane]);
+    *reinterpret_cast<float4*>(part + (int64_t)blockIdx.y * N + c) = r;
+  }
+}
+
 int64_t colsum_rows_parts(int64_t T) { return (T + 127) / 128; }
 
 omq_status colsum_rows(cudaStream_t st, const float* X, int64_t T, int64_t N, int64_t ldx, float* part,
                        float* out, float scale, int accumulate) {
-  dim3 grid((unsigned)((N + 255) / 256), (unsigned)colsum_rows_parts(T));
-  colsum_rows_kernel<<<grid, 256, 0, st>>>(X, T, N, ldx, part);
+  if (N % 4 == 0 && ldx % 4 == 0 && omq_aligned16(X) && omq_aligned16(part)) {
+    dim3 grid((unsigned)((N + 127) / 128), (unsigned)colsum_rows_parts(T));
+    colsum_rows_vec_kernel<<<grid, 256, 0, st>>>(X, T, N, ldx, part);
+  } else {
+    dim3 grid((unsigned)((N + 255) / 256), (unsigned)colsum_rows_parts(T));
+    colsum_rows_kernel<<<grid, 256, 0, st>>>(X, T, N, ldx, part);
+  }
   OMQ_LAUNCH_CHECK();
   return omq_colsum_partials(st, part, colsum_rows_parts(T), N, out, scale, accumulate);
 }
