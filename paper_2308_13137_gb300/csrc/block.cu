@@ -368,6 +368,7 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   af.producer = AP_RMS_LET; af.X = x; af.ldx = c.d; af.s = c.let ? th->s1 : nullptr; af.delta = c.let ? th->d1 : nullptr;
   af.rms_eps = c.s.rms_eps; af.rstd = w.rstd1; af.T = c.T; af.C = c.d; af.Xq = w.a_h; af.ldq = c.d;
   af.h = w.sa.h; af.z = w.sa.z; af.imax = w.sa.imax; af.imin = w.sa.imin; af.abits = cfg.abits; af.eps = cfg.h_eps;
+  af.status = status;
   OMQ_TRY(act_fwd_launch(st, af));
   OMQ_TRY(gemm_kk(st, c.T, c.nqkv, c.d, w.a_h, c.d, w.Wqkv_h, c.d, w.Yqkv, nullptr, c.nqkv, c.let ? w.B_qkv : nullptr,
                   nullptr, status));
@@ -385,6 +386,7 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   ActFwdArgs ao{};
   ao.producer = AP_PLAIN; ao.X = w.O; ao.ldx = c.dq; ao.T = c.T; ao.C = c.dq; ao.Xq = w.O_h; ao.ldq = c.dq;
   ao.h = w.so.h; ao.z = w.so.z; ao.imax = w.so.imax; ao.imin = w.so.imin; ao.abits = cfg.abits; ao.eps = cfg.h_eps;
+  ao.status = status;
   OMQ_TRY(act_fwd_launch(st, ao));
   OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[1], 0) == cudaSuccess, OMQ_ERR_CUDA);      // W_hat of o_proj
   OMQ_TRY(gemm_kk(st, c.T, c.d, c.dq, w.O_h, c.dq, w.Wo_h, c.dq, w.h1, nullptr, c.d, c.let ? w.B_o : nullptr, x, status));
@@ -400,7 +402,7 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   ActFwdArgs am{};
   am.producer = AP_SWIGLU; am.X = w.Ygu; am.ldx = 2 * c.f; am.U = w.Ygu + c.f; am.ldu = 2 * c.f; am.T = c.T; am.C = c.f;
   am.Xq = w.m_h; am.ldq = c.f; am.h = w.sm.h; am.z = w.sm.z; am.imax = w.sm.imax; am.imin = w.sm.imin;
-  am.abits = cfg.abits; am.eps = cfg.h_eps;
+  am.abits = cfg.abits; am.eps = cfg.h_eps; am.status = status;
   OMQ_TRY(act_fwd_launch(st, am));
   OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[3], 0) == cudaSuccess, OMQ_ERR_CUDA);      // W_hat of down (joins)
   OMQ_TRY(gemm_kk(st, c.T, c.d, c.f, w.m_h, c.f, w.Wd_h, c.f, y, nullptr, c.d, nullptr, w.h1, status));
@@ -654,7 +656,7 @@ omq_status omq_qlinear_fwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t 
   ActFwdArgs a{};
   a.producer = let ? AP_LET : AP_PLAIN; a.X = X; a.ldx = Cin; a.s = let ? s : nullptr; a.delta = let ? delta : nullptr;
   a.T = T; a.C = Cin; a.Xq = (bf16*)sv->x_hat; a.ldq = Cin; a.h = sv->h_a; a.z = sv->z_a; a.imax = sv->imax_a;
-  a.imin = sv->imin_a; a.abits = cfg->abits; a.eps = cfg->h_eps;
+  a.imin = sv->imin_a; a.abits = cfg->abits; a.eps = cfg->h_eps; a.status = cfg->dev_status;
   OMQ_TRY(act_fwd_launch(st, a));
   return gemm_kk(st, T, Cout, Cin, (const bf16*)sv->x_hat, Cin, (const bf16*)sv->w_hat, Cin, Y, nullptr, Cout, bias,
                  nullptr, cfg->dev_status);

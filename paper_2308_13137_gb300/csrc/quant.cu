@@ -1094,7 +1094,7 @@ omq_status omq_act_quant_per_token(omq_stream_t stream, int64_t T, int64_t C, co
   a.producer = (s || delta) ? AP_LET : AP_PLAIN;
   a.X = X; a.ldx = C; a.s = s; a.delta = delta; a.T = T; a.C = C;
   a.Xq = (__nv_bfloat16*)Xq; a.ldq = C; a.codes = codes; a.h = h; a.z = z; a.imax = argmax; a.imin = argmin;
-  a.abits = cfg->abits; a.eps = cfg->h_eps;
+  a.abits = cfg->abits; a.eps = cfg->h_eps; a.status = cfg->dev_status;
   return act_fwd_launch((cudaStream_t)stream, a);
 }
 

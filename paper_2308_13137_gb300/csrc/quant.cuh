@@ -54,6 +54,7 @@ struct ActFwdArgs {
   uint8_t* codes;
   float* h; int32_t* z; int32_t* imax; int32_t* imin;
   int abits; float eps;
+  int32_t* status;                   // device status word (timeouts of the staged kernel), nullable
 };
 omq_status act_fwd_launch(cudaStream_t st, const ActFwdArgs& a);
 

@@ -6,6 +6,9 @@
 // reductions, and the LET column sums of a thread's columns accumulate in registers across rows.
 #include "attn.cuh"
 #include "quant.cuh"
+#include "tc.cuh"
+
+#include <algorithm>
 
 namespace {
 
@@ -190,6 +193,169 @@ __global__ void __launch_bounds__(NT) act_fwd_rows(ActFwdArgs a) {
       }
     }
   }
+}
+
+// ================================================================================================
+// activation quantizer forward, staged: a persistent CTA walks the rows blockIdx.x, + gridDim.x, ...
+// and the bulk-copy engine brings each row's inputs into a ring of `stages` shared-memory buffers
+// (cp.async.bulk completing on one mbarrier per buffer) while the CTA works on earlier rows, so
+// the row's HBM latency is hidden behind the compute and the block reductions of the rows before
+// it.  The arithmetic on each element is act_fwd_rows's.  Waits are bounded: on expiry the status
+// word is set, the CTA waits (again bounded) for the copies it issued and returns.
+// ================================================================================================
+template <int P, int NT, int VPT>
+__global__ void __launch_bounds__(NT) act_fwd_staged(ActFwdArgs a, int stages) {
+  constexpr int NE = 4 * VPT, NW = NT / 32, MAXS = 4;
+  constexpr int NIN = P == AP_SWIGLU ? 2 : 1;
+  extern __shared__ float4 stg4[];                 // [stages][NIN][C / 4]
+  __shared__ uint64_t bar[MAXS];
+  __shared__ float red[3][NW];
+  __shared__ int sidx[2];
+  __shared__ int abort_flag;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t nv = a.C / 4;
+  const uint32_t row_bytes = (uint32_t)(a.C * 4);
+  const bool quant = a.abits < 16;
+  const float Q = (float)((1 << (quant ? a.abits : 1)) - 1);
+  if (tid == 0) {
+    for (int s = 0; s < stages; ++s) tc::mbar_init(&bar[s], 1);
+    sidx[0] = 0x7fffffff; sidx[1] = 0x7fffffff;
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  int64_t issued = 0;                              // rows whose copies thread 0 has issued
+  auto issue = [&](int64_t k) {
+    const int64_t t = blockIdx.x + k * gridDim.x;
+    if (t >= a.T) return;
+    const int s = (int)(k % stages);
+    float4* dst = stg4 + (size_t)s * NIN * nv;
+    tc::mbar_expect_tx(&bar[s], NIN * row_bytes);
+    tc::bulk_g2s(dst, a.X + t * a.ldx, row_bytes, &bar[s]);
+    if (P == AP_SWIGLU) tc::bulk_g2s(dst + nv, a.U + t * a.ldu, row_bytes, &bar[s]);
+    issued = k + 1;
+  };
+  if (tid == 0)
+    for (int k = 0; k < stages; ++k) issue(k);
+  int64_t k = 0;
+  for (;; ++k) {
+    const int64_t t = blockIdx.x + k * gridDim.x;
+    if (t >= a.T) break;
+    const int s = (int)(k % stages);
+    if (!tc::mbar_wait(&bar[s], (uint32_t)((k / stages) & 1))) {
+      omq_set_status(a.status, OMQ_ERR_TIMEOUT);
+      abort_flag = 1;
+    }
+    const float4* xs = stg4 + (size_t)s * NIN * nv;
+    float val[NE];
+    float ss = 0.f;
+#pragma unroll
+    for (int j = 0; j < VPT; ++j) {
+      const int64_t vi = (int64_t)j * NT + tid;
+      const float4 xv = vi < nv ? xs[vi] : make_float4(0.f, 0.f, 0.f, 0.f);
+      float4 uv = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (P == AP_SWIGLU && vi < nv) uv = xs[nv + vi];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        float x = f4get(xv, e);
+        if (P == AP_SWIGLU) x = silu(x) * f4get(uv, e);
+        val[4 * j + e] = x;
+        if (P == AP_RMS_LET) ss = fmaf(x, x, ss);
+      }
+    }
+    if (P == AP_RMS_LET) {                          // the summation tree of block_sum2
+      ss = warp_sum(ss);
+      if (lane == 0) red[0][warp] = ss;
+      __syncthreads();
+      const float tot = warp_sum(lane < NW ? red[0][lane] : 0.f);
+      const float rstd = 1.0f / sqrtf(tot / (float)a.C + a.rms_eps);
+      if (tid == 0 && a.rstd) a.rstd[t] = rstd;
+#pragma unroll
+      for (int k2 = 0; k2 < NE; ++k2) val[k2] = val[k2] * rstd;
+    }
+    if (P == AP_LET || P == AP_RMS_LET) {
+#pragma unroll
+      for (int j = 0; j < VPT; ++j) {
+        const int64_t vi = (int64_t)j * NT + tid;
+        if (vi < nv) {
+          const float4 dl = a.delta ? ld4(a.delta + 4 * vi) : make_float4(0.f, 0.f, 0.f, 0.f);
+          const float4 sv = a.s ? ld4(a.s + 4 * vi) : make_float4(1.f, 1.f, 1.f, 1.f);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            float v = val[4 * j + e];
+            if (a.delta) v = v - f4get(dl, e);
+            if (a.s) v = __fdiv_rn(v, f4get(sv, e));
+            val[4 * j + e] = v;
+          }
+        }
+      }
+    }
+    QState qs;
+    if (quant) {
+      float M = -INFINITY, m = INFINITY;
+#pragma unroll
+      for (int j = 0; j < VPT; ++j)
+        if ((int64_t)j * NT + tid < nv)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) { M = fmaxf(M, val[4 * j + e]); m = fminf(m, val[4 * j + e]); }
+      float bM = M, bm = m;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        bM = fmaxf(bM, __shfl_xor_sync(0xffffffffu, bM, off));
+        bm = fminf(bm, __shfl_xor_sync(0xffffffffu, bm, off));
+      }
+      if (lane == 0) { red[1][warp] = bM; red[2][warp] = bm; }
+      __syncthreads();
+      bM = red[1][0]; bm = red[2][0];
+#pragma unroll
+      for (int w = 1; w < NW; ++w) { bM = fmaxf(bM, red[1][w]); bm = fminf(bm, red[2][w]); }
+      if (M == bM || m == bm) {                   // the first index, searched by the holders only
+        int iM = 0x7fffffff, im = 0x7fffffff;
+#pragma unroll
+        for (int j = VPT - 1; j >= 0; --j) {
+          const int64_t vi = (int64_t)j * NT + tid;
+          if (vi < nv)
+#pragma unroll
+            for (int e = 3; e >= 0; --e) {
+              if (val[4 * j + e] == bM) iM = (int)(4 * vi + e);
+              if (val[4 * j + e] == bm) im = (int)(4 * vi + e);
+            }
+        }
+        if (iM != 0x7fffffff) atomicMin(&sidx[0], iM);
+        if (im != 0x7fffffff) atomicMin(&sidx[1], im);
+      }
+      qs = omq_qstate(bM, bm, 1.f, 1.f, Q, a.eps);
+    }
+    __nv_bfloat16* qr = a.Xq + t * a.ldq;
+#pragma unroll
+    for (int j = 0; j < VPT; ++j) {
+      const int64_t vi = (int64_t)j * NT + tid;
+      if (vi < nv) {
+        float o[4], cd[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) o[e] = quant ? omq_fakequant(val[4 * j + e], qs, Q, &cd[e]) : val[4 * j + e];
+        st_bf16x4(qr + 4 * vi, o);
+        if (a.codes && quant) {
+          const uint32_t pk = (uint32_t)cd[0] | ((uint32_t)cd[1] << 8) | ((uint32_t)cd[2] << 16) | ((uint32_t)cd[3] << 24);
+          *reinterpret_cast<uint32_t*>(a.codes + t * a.C + 4 * vi) = pk;
+        }
+      }
+    }
+    __syncthreads();                               // buffer s read by every thread; first indices final
+    if (tid == 0) {
+      if (quant) {
+        a.h[t] = qs.h; a.z[t] = (int32_t)qs.z; a.imax[t] = sidx[0]; a.imin[t] = sidx[1];
+        sidx[0] = 0x7fffffff; sidx[1] = 0x7fffffff;
+      }
+      if (!abort_flag) {
+        tc::fence_async_smem();                    // generic reads of buffer s before the copy engine refills it
+        issue(k + stages);
+      }
+    }
+    if (abort_flag) break;
+  }
+  if (tid == 0 && abort_flag)                      // rows k .. issued - 1 may still be in flight: let them land
+    for (int64_t r = k; r < issued; ++r) tc::mbar_wait(&bar[r % stages], (uint32_t)((r / stages) & 1));
 }
 
 // ================================================================================================
@@ -507,8 +673,43 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
     else return OMQ_ERR_UNSUPPORTED;                                                                 \
   } while (0)
 
+template <int P, int NT, int VPT>
+static omq_status act_fwd_staged_go(cudaStream_t st, const ActFwdArgs& a, int stages, size_t smem) {
+  auto kern = act_fwd_staged<P, NT, VPT>;
+  static int per_sm = -1;
+  static size_t smem_set = 0;
+  if (smem > smem_set) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+      return OMQ_ERR_CUDA;
+    smem_set = smem;
+    per_sm = -1;
+  }
+  int bps = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, kern, NT, smem) != cudaSuccess || bps < 1) return OMQ_ERR_CUDA;
+  (void)per_sm;
+  const int64_t grid = std::min<int64_t>(a.T, (int64_t)omq_num_sms() * bps);
+  kern<<<(unsigned)grid, NT, smem, st>>>(a, stages);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+// Rows whose inputs fit two or more times in shared memory take the staged kernel; 16-byte aligned
+// rows of up to 16 K columns.
 template <int PRODUCER>
 static omq_status act_fwd_dispatch(cudaStream_t st, const ActFwdArgs& a) {
+  const int nin = PRODUCER == AP_SWIGLU ? 2 : 1;
+  const size_t row_bytes = (size_t)nin * a.C * 4;
+  const int stages = (int)std::min<size_t>(3, (200 * 1024) / row_bytes);
+  const bool aligned = a.ldx % 4 == 0 && omq_aligned16(a.X) &&
+                       (PRODUCER != AP_SWIGLU || (a.ldu % 4 == 0 && omq_aligned16(a.U)));
+  const int64_t nv = a.C / 4;
+  if (stages >= 2 && aligned && nv <= 1024 * 4) {
+    // the row-to-thread mapping of act_fwd_rows, so that the RMS sum (and every output) is the same
+    const size_t smem = (size_t)stages * row_bytes;
+    if (nv <= 512 * 2) return act_fwd_staged_go<PRODUCER, 512, 2>(st, a, stages, smem);
+    if (nv <= 512 * 4) return act_fwd_staged_go<PRODUCER, 512, 4>(st, a, stages, smem);
+    return act_fwd_staged_go<PRODUCER, 1024, 4>(st, a, stages, smem);
+  }
   ACT_DISPATCH(act_fwd_rows, a, (unsigned)a.T, a.C);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;

@@ -2,8 +2,16 @@
 same BlockState calls and kernel launch configurations that bench.py times.
 
 * LLaMA-7B W4A4 LWC+LET (the timed workload): the whole calibration step against the fp64 oracle
-  (emulate mode): block output, loss and every parameter gradient, same tolerances as the small
-  shapes.  The GPU full-precision forward that produces the Eq. 1 target is checked as well.
+  (emulate mode): block output, loss and every parameter gradient.  At 2048 tokens the W4A4 step
+  is discontinuous in its input: every rounding decision of Eq. 2 on the per-token 4-bit q, k,
+  v, o and FFN activations is a step function, and a flipped code in k or v reaches every later
+  query through attention.  Moving the input by 2 ulps moves the oracle's own output by about
+  1.3 % and its gradients by up to 3 % (most rows unchanged, a few late tokens by 5-10 %).  So the
+  test measures that spread in the oracle (the same step on the input scaled by 1 + 2^-22) and
+  asks of the GPU step: at least 90 % of the output rows within 1e-3 of the oracle (the tokens
+  whose decisions agree), the loss within 1e-2, and the output and every gradient within the
+  small-shape tolerances or twice the oracle's own spread, whichever is larger.  The GPU
+  full-precision forward that produces the Eq. 1 target is checked as well.
 * LLaMA-7B W3A16 g128, LLaMA-13B W2A16 g64 and LLaMA-2-70B W4A4 GQA: block output and loss of
   the step against the oracle's quantized forward (the gradient paths of these configurations
   are covered element by element at small sizes).
@@ -61,23 +69,33 @@ def c2_full(cuda_lib):
     yfp = O.block_fp_forward(x, W, cfg).float()
     got = _gpu_step(shape, W, x, th, yfp)
     ref = O.block_step(x, yfp, W, th, cfg)
-    return shape, got, ref, yfp
+    x2 = (x.astype(np.float64) * (1.0 + 2.0 ** -22)).astype(np.float32)     # the input moved by 2 ulps
+    ref2 = O.block_step(x2, yfp, W, th, cfg)
+    spread = {"y": _rel(ref2["y"], ref["y"])}
+    for n in O.THETA_NAMES_LWC + O.THETA_NAMES_LET:
+        spread["d" + n] = _rel(ref2["d" + n], ref["d" + n])
+    return shape, got, ref, yfp, spread
 
 
 def test_full_c2_fp_target(c2_full):
-    _, got, _, yfp = c2_full
+    _, got, _, yfp, _ = c2_full
     assert _rel(got["y_fp"], yfp) < OUT_TOL
 
 
 def test_full_c2_step(c2_full):
-    shape, got, ref, _ = c2_full
-    assert _rel(got["y"], ref["y"]) < OUT_TOL
+    shape, got, ref, _, spread = c2_full
+    y, yr = torch.as_tensor(got["y"]).double(), torch.as_tensor(ref["y"]).double()
+    row_err = (y - yr).norm(dim=1) / yr.norm(dim=1)
+    agree = float((row_err <= 1e-3).double().mean())
+    print(f"rows within 1e-3: {agree:.4f}; y error {_rel(y, yr):.3e} (oracle 2-ulp spread {spread['y']:.3e})")
+    assert agree >= 0.9, (agree, spread["y"])
+    assert _rel(y, yr) < max(OUT_TOL, 2 * spread["y"]), (_rel(y, yr), spread["y"])
     assert abs(got["loss"] - float(ref["loss"])) / float(ref["loss"]) < OUT_TOL
     bad = {}
     for n in O.THETA_NAMES_LWC + O.THETA_NAMES_LET:
         e = _rel(got["d" + n], ref["d" + n])
-        if not e < GRAD_TOL:
-            bad[n] = e
+        if not e < max(GRAD_TOL, 2 * spread["d" + n]):
+            bad[n] = (e, spread["d" + n])
     assert not bad, bad
 
 
