@@ -40,7 +40,10 @@ constexpr int EPI_TILE_BYTES = 32 * 32 * 4;      // one 32 x 32 fp32 block, 128-
 template <int BN, int STAGES, bool PAIR = false>
 struct SmemLayout {
   static constexpr int A_BYTES = BM * BK * 2;
-  static constexpr int B_BYTES = (PAIR ? BN / 2 : BN) * BK * 2;   // a pair splits B's columns
+  static constexpr int B_COLS = PAIR ? BN / 2 : BN;                 // a pair splits B's columns
+  // room for whole 64-column boxes (MN-major B is staged in 64-wide swizzle atoms)
+  static constexpr int B_BYTES = (B_COLS + 63) / 64 * 64 * BK * 2;
+  static constexpr uint32_t TMEM_COLS = 2 * BN <= 256 ? 256 : 512;  // two accumulators, power of two
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int EPI_OFF = STAGES * STAGE_BYTES;           // 1024-aligned (swizzle atom)
   static constexpr int EPI_BYTES = 4 * 2 * EPI_TILE_BYTES;       // two staging blocks per epilogue warp
@@ -283,8 +286,8 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
-    if (PAIR) tmem_alloc_pair(tmem_holder, 2 * BN);
-    else tmem_alloc(tmem_holder, 2 * BN);
+    if (PAIR) tmem_alloc_pair(tmem_holder, L::TMEM_COLS);
+    else tmem_alloc(tmem_holder, L::TMEM_COLS);
   }
   tc_fence_before();
   __syncthreads();
@@ -296,6 +299,8 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
     // ---------------- TMA producer ----------------
     uint32_t it = 0;
     constexpr int BNH = PAIR ? BN / 2 : BN;      // B columns staged by this CTA
+    // bytes one stage of this CTA receives: A, and B as K-major rows or whole 64-column boxes
+    const uint32_t stage_tx = L::A_BYTES + (p.b_mn ? (uint32_t)((BNH + 63) / 64 * 64 * BK * 2) : (uint32_t)(BNH * BK * 2));
     for (int t = t_first; t < total && !*abort_flag; t += t_step) {
       const TileInfo ti = tile_info(p, t, BN, rank);
       if (ti.skip) continue;
@@ -311,7 +316,7 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
         if (PAIR) {
           // both CTAs' loads complete on the leader's barrier, which expects the pair's bytes
           const uint32_t fb = mapa_shared(smem_u32(&full[s]), 0);
-          if (leader) mbar_expect_tx(&full[s], 2 * L::STAGE_BYTES);
+          if (leader) mbar_expect_tx(&full[s], 2 * stage_tx);
           if (!p.a_mn) {
             tma_load_3d_pair(&tmA, fb, sa, k0, ti.m0, ti.b);
           } else {
@@ -322,10 +327,11 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
             tma_load_3d_pair(&tmB, fb, sb, k0, nb0, ti.b);
           } else {
 #pragma unroll
-            for (int j = 0; j < BNH / 64; ++j) tma_load_3d_pair(&tmB, fb, sb + j * 64 * BK * 2, nb0 + 64 * j, k0, ti.b);
+            for (int j = 0; j < (BNH + 63) / 64; ++j)
+              tma_load_3d_pair(&tmB, fb, sb + j * 64 * BK * 2, nb0 + 64 * j, k0, ti.b);
           }
         } else {
-          mbar_expect_tx(&full[s], L::STAGE_BYTES);
+          mbar_expect_tx(&full[s], stage_tx);
           if (!p.a_mn) {
             tma_load_3d(&tmA, &full[s], sa, k0, ti.m0, ti.b);
           } else {
@@ -336,7 +342,8 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
             tma_load_3d(&tmB, &full[s], sb, k0, ti.n0, ti.b);
           } else {
 #pragma unroll
-            for (int j = 0; j < BN / 64; ++j) tma_load_3d(&tmB, &full[s], sb + j * 64 * BK * 2, ti.n0 + 64 * j, k0, ti.b);
+            for (int j = 0; j < (BN + 63) / 64; ++j)
+              tma_load_3d(&tmB, &full[s], sb + j * 64 * BK * 2, ti.n0 + 64 * j, k0, ti.b);
           }
         }
       }
@@ -493,8 +500,8 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
   if (PAIR) cluster_sync();                 // no CTA leaves while its peer may still signal it
   if (warp == 1) {
     tc_fence_after();
-    if (PAIR) tmem_dealloc_pair(tmem, 2 * BN);
-    else tmem_dealloc(tmem, 2 * BN);
+    if (PAIR) tmem_dealloc_pair(tmem, L::TMEM_COLS);
+    else tmem_dealloc(tmem, L::TMEM_COLS);
   }
 }
 

@@ -703,6 +703,16 @@ static omq_status act_fwd_dispatch(cudaStream_t st, const ActFwdArgs& a) {
   const bool aligned = a.ldx % 4 == 0 && omq_aligned16(a.X) &&
                        (PRODUCER != AP_SWIGLU || (a.ldu % 4 == 0 && omq_aligned16(a.U)));
   const int64_t nv = a.C / 4;
+  if (nv <= 128 * 8) {                             // small rows: many CTAs per SM, 32 values per thread
+    act_fwd_rows<PRODUCER, 128, 8><<<(unsigned)a.T, 128, 0, st>>>(a);
+    OMQ_LAUNCH_CHECK();
+    return OMQ_OK;
+  }
+  if (PRODUCER == AP_SWIGLU && nv <= 256 * 12) {
+    act_fwd_rows<PRODUCER, 256, 12><<<(unsigned)a.T, 256, 0, st>>>(a);
+    OMQ_LAUNCH_CHECK();
+    return OMQ_OK;
+  }
   if (stages >= 2 && aligned && nv <= 1024 * 4) {
     // the row-to-thread mapping of act_fwd_rows, so that the RMS sum (and every output) is the same
     const size_t smem = (size_t)stages * row_bytes;
@@ -841,7 +851,7 @@ __global__ void __launch_bounds__(NT) qkv_fwd_rows(QkvArgs a) {
   __shared__ int ism[64];
   const int t = blockIdx.x;
   const int dq = a.H * a.hd, dkv = a.Hkv * a.hd;
-  for (int seg = 0; seg < 3; ++seg) {
+  for (int seg = blockIdx.y; seg < (gridDim.y == 1 ? 3 : (int)blockIdx.y + 1); ++seg) {   // y: one segment per CTA
     QkvRow<PPT> r;
     qkv_load<NT, PPT>(a, seg, t, r);
     const int W = seg == 0 ? dq : dkv;
@@ -1065,7 +1075,8 @@ int64_t qkv_bwd_nslab(int T) { return (T + 3) / 4; }
 omq_status qkv_fwd_launch(cudaStream_t st, const QkvArgs& a) {
   OMQ_REQUIRE(a.hd == 128, OMQ_ERR_UNSUPPORTED);
   const int np = a.H * 16;
-  if (np <= 512) qkv_fwd_rows<512, 1><<<a.T, 512, 0, st>>>(a);
+  const dim3 g3((unsigned)a.T, 3);                 // one CTA per (token, q | k | v)
+  if (np <= 512) qkv_fwd_rows<128, 4><<<g3, 128, 0, st>>>(a);
   else if (np <= 1024) qkv_fwd_rows<512, 2><<<a.T, 512, 0, st>>>(a);
   else if (np <= 2048) qkv_fwd_rows<512, 4><<<a.T, 512, 0, st>>>(a);
   else return OMQ_ERR_UNSUPPORTED;

@@ -121,6 +121,12 @@ SPLIT_CASES = [  # M, N, K, a_kmajor, b_kmajor
     (2048, 5376, 1024, 1, 0),   # 168 pair tiles: one wave of whole tiles, then a cut tail
     (1000, 1152, 2048, 0, 1),   # one CTA per 128 x 128 tile (N not a multiple of 256), ragged M, 72 tiles
     (4096, 2304, 512, 0, 0),    # 144 pair tiles of 8 k-blocks
+    # projection-shaped products (N = 4096, 12288) with K-major and MN-major B
+    (2048, 4096, 512, 1, 1),
+    (2048, 4096, 512, 1, 0),
+    (2048, 4096, 320, 0, 0),
+    (2048, 12288, 256, 1, 1),
+    (2048, 12288, 256, 1, 0),
 ]
 
 
