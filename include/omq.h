@@ -343,6 +343,16 @@ omq_status omq_adamw_update(omq_stream_t stream, int64_t n, float* p, const floa
                             float* v, float lr, float beta1, float beta2, float eps,
                             float weight_decay, int32_t step);
 
+/* The same update with the step count t read from device memory at *step_dev (int32, >= 1), so that
+ * a captured CUDA graph replays correctly across steps.  Bias corrections 1 - b^t are formed on
+ * the device in single precision. */
+omq_status omq_adamw_update_dev(omq_stream_t stream, int64_t n, float* p, const float* g, float* m,
+                                float* v, float lr, float beta1, float beta2, float eps,
+                                float weight_decay, const int32_t* step_dev);
+
+/* *step_dev += 1 on `stream` (one thread). */
+omq_status omq_step_advance(omq_stream_t stream, int32_t* step_dev);
+
 /* Reads the device status word written by kernels (synchronises `stream`).  *host_out receives
  * the word (0 = ok); the return value is OMQ_OK or OMQ_ERR_CUDA if the copy failed. */
 omq_status omq_stream_status(omq_stream_t stream, const int32_t* dev_status, int32_t* host_out);

@@ -100,6 +100,8 @@ _SIGS = {
     "omq_let_init_workspace_size": (SZ, [P]),
     "omq_let_init": (I32, [P, P, P, P, I64, F32, P, P, SZ]),
     "omq_adamw_update": (I32, [P, I64, P, P, P, P, F32, F32, F32, F32, F32, I32]),
+    "omq_adamw_update_dev": (I32, [P, I64, P, P, P, P, F32, F32, F32, F32, F32, P]),
+    "omq_step_advance": (I32, [P, P]),
     "omq_stream_status": (I32, [P, P, POINTER(c_int32)]),
     "omq_status_string": (c_char_p, [I32]),
     "omq_version": (I32, []),
@@ -318,6 +320,15 @@ def omq_block_step(shape, weights, theta, x, y_fp, y, loss, grads, workspace, cf
 def omq_adamw_update(n, p, g, m, v, lr, beta1, beta2, eps, weight_decay, step, stream=None):
     check("omq_adamw_update", lib().omq_adamw_update(stream_handle(stream), n, ptr(p), ptr(g), ptr(m), ptr(v), lr,
                                                      beta1, beta2, eps, weight_decay, step))
+
+
+def omq_adamw_update_dev(n, p, g, m, v, lr, beta1, beta2, eps, weight_decay, step_dev, stream=None):
+    check("omq_adamw_update_dev", lib().omq_adamw_update_dev(stream_handle(stream), n, ptr(p), ptr(g), ptr(m), ptr(v),
+                                                             lr, beta1, beta2, eps, weight_decay, ptr(step_dev)))
+
+
+def omq_step_advance(step_dev, stream=None):
+    check("omq_step_advance", lib().omq_step_advance(stream_handle(stream), ptr(step_dev)))
 
 
 def omq_stream_status(dev_status, stream=None) -> int:

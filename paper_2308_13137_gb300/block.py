@@ -74,6 +74,9 @@ class BlockState:
         self.n_lwc = n_lwc
         self.adam = {g: (torch.zeros_like(f), torch.zeros_like(f)) for g, f in self.theta_flat.items()}
         self.adam_step = 0
+        # the AdamW step count also lives on the device, so that captured graphs replay correctly
+        self.adam_step_dev = torch.zeros(1, dtype=torch.int32, device=device)
+        self._graphs = {}
         self.c_shape = _lib.omq_block_shape(shape.T, shape.d, shape.n_heads, shape.n_kv, shape.head_dim, shape.ffn,
                                             shape.rms_eps, shape.rope_theta)
         self.c_w = _lib.omq_block_weights(*[self.W[k].data_ptr() for k in ("qkv", "o", "gu", "d")])
@@ -101,12 +104,40 @@ class BlockState:
         return self.loss
 
     def adamw(self, lr_lwc: float = 5e-3, lr_let: float = 1e-2, stream=None):
-        """AdamW with zero weight decay on both parameter groups (Sec. 4.1 "Training")."""
+        """AdamW with zero weight decay on both parameter groups (Sec. 4.1 "Training"); the step
+        count advances on the device."""
         self.adam_step += 1
+        _lib.omq_step_advance(self.adam_step_dev, stream)
         for g, flat in self.theta_flat.items():
             m, v = self.adam[g]
-            _lib.omq_adamw_update(flat.numel(), flat, self.grads_flat[g], m, v, lr_lwc if g == "lwc" else lr_let,
-                                  0.9, 0.999, 1e-8, 0.0, self.adam_step, stream)
+            _lib.omq_adamw_update_dev(flat.numel(), flat, self.grads_flat[g], m, v, lr_lwc if g == "lwc" else lr_let,
+                                      0.9, 0.999, 1e-8, 0.0, self.adam_step_dev, stream)
+
+    def step_adamw_graph(self, x, y_fp, lr_lwc: float = 5e-3, lr_let: float = 1e-2):
+        """One calibration step and its AdamW update, replayed from a CUDA graph of the same launches
+        (one graph per input pair (x, y_fp) and learning rates, captured on first use after one
+        ordinary step has set up the library's state).  The result equals step() + adamw()."""
+        torch = self.torch
+        key = (x.data_ptr(), y_fp.data_ptr(), lr_lwc, lr_let)
+        g = self._graphs.get(key)
+        if g is not None:
+            self.adam_step += 1
+            g.replay()
+            return self.loss
+        self.step(x, y_fp)                  # one ordinary step: lazy set-up inside libomq happens here
+        self.adamw(lr_lwc, lr_let)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.step(x, y_fp)
+            _lib.omq_step_advance(self.adam_step_dev)
+            for name, flat in self.theta_flat.items():
+                m, v = self.adam[name]
+                _lib.omq_adamw_update_dev(flat.numel(), flat, self.grads_flat[name], m, v,
+                                          lr_lwc if name == "lwc" else lr_let, 0.9, 0.999, 1e-8, 0.0,
+                                          self.adam_step_dev)
+        self._graphs[key] = g
+        return self.loss
 
     def forward(self, x, y, stream=None, cfg=None):
         _lib.omq_block_forward(self.c_shape, self.c_w, self.c_theta, x, y, self.workspace, cfg or self.cfg, stream)

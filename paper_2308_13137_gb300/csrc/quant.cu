@@ -1000,6 +1000,29 @@ __global__ void adamw_kernel(int64_t n, float* p, const float* g, float* m, floa
   p[i] = pi - lr * (mi / bc1) / (sqrtf(vi / bc2) + eps) - lr * wd * pi;
 }
 
+// the same, t read from device memory; bias corrections formed once per CTA
+__global__ void adamw_dev_kernel(int64_t n, float* p, const float* g, float* m, float* v, float lr, float b1, float b2,
+                                 float eps, float wd, const int32_t* step) {
+  __shared__ float bc[2];
+  if (threadIdx.x == 0) {
+    const float t = (float)*step;
+    bc[0] = 1.f - powf(b1, t);
+    bc[1] = 1.f - powf(b2, t);
+  }
+  __syncthreads();
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const float gi = g[i];
+  const float mi = b1 * m[i] + (1.f - b1) * gi;
+  const float vi = b2 * v[i] + (1.f - b2) * gi * gi;
+  m[i] = mi;
+  v[i] = vi;
+  const float pi = p[i];
+  p[i] = pi - lr * (mi / bc[0]) / (sqrtf(vi / bc[1]) + eps) - lr * wd * pi;
+}
+
+__global__ void step_advance_kernel(int32_t* step) { *step += 1; }
+
 // ================================================================================================
 // C ABI: kernel-level entry points
 // ================================================================================================
@@ -1178,6 +1201,24 @@ omq_status omq_adamw_update(omq_stream_t stream, int64_t n, float* p, const floa
   float bc1 = 1.f - powf(beta1, (float)step), bc2 = 1.f - powf(beta2, (float)step);
   adamw_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(n, p, g, m, v, lr, beta1, beta2, eps,
                                                                               weight_decay, bc1, bc2);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+omq_status omq_adamw_update_dev(omq_stream_t stream, int64_t n, float* p, const float* g, float* m, float* v,
+                                float lr, float beta1, float beta2, float eps, float weight_decay,
+                                const int32_t* step_dev) {
+  OMQ_REQUIRE(n > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(p && g && m && v && step_dev, OMQ_ERR_INVALID_ARG);
+  adamw_dev_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(n, p, g, m, v, lr, beta1, beta2,
+                                                                                  eps, weight_decay, step_dev);
+  OMQ_LAUNCH_CHECK();
+  return OMQ_OK;
+}
+
+omq_status omq_step_advance(omq_stream_t stream, int32_t* step_dev) {
+  OMQ_REQUIRE(step_dev, OMQ_ERR_INVALID_ARG);
+  step_advance_kernel<<<1, 1, 0, (cudaStream_t)stream>>>(step_dev);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }

@@ -315,3 +315,22 @@ def test_adamw(cuda_lib):
     v2 = 0.999 * v.double() + 0.001 * gr.double() ** 2
     p2 = p.double() - 5e-3 * (m2 / (1 - 0.9 ** 3)) / ((v2 / (1 - 0.999 ** 3)).sqrt() + 1e-8)
     assert _rel(pd.cpu(), p2) < 1e-6 and _rel(md.cpu(), m2) < 1e-6 and _rel(vd.cpu(), v2) < 1e-6
+
+
+def test_adamw_device_step(cuda_lib):
+    """The device-counter form: three advances then one update equals the update at step 3."""
+    g = torch.Generator().manual_seed(3)
+    n = 1000
+    p, gr = torch.randn(n, generator=g), torch.randn(n, generator=g)
+    m, v = torch.randn(n, generator=g) * 0.1, torch.rand(n, generator=g) * 0.1
+    pd, md, vd = p.cuda(), m.cuda(), v.cuda()
+    t = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for _ in range(3):
+        _lib.omq_step_advance(t)
+    _lib.omq_adamw_update_dev(n, pd, gr.cuda(), md, vd, 5e-3, 0.9, 0.999, 1e-8, 0.0, t)
+    torch.cuda.synchronize()
+    assert int(t.item()) == 3
+    m2 = 0.9 * m.double() + 0.1 * gr.double()
+    v2 = 0.999 * v.double() + 0.001 * gr.double() ** 2
+    p2 = p.double() - 5e-3 * (m2 / (1 - 0.9 ** 3)) / ((v2 / (1 - 0.999 ** 3)).sqrt() + 1e-8)
+    assert _rel(pd.cpu(), p2) < 1e-6 and _rel(md.cpu(), m2) < 1e-6 and _rel(vd.cpu(), v2) < 1e-6
