@@ -312,12 +312,14 @@ struct BwdP {
 
 constexpr int B_QATOM = 64 * ROW_BYTES;               // 8 KB: 64-row atom
 constexpr int B_QTILE = 2 * B_QATOM;                  // [64 x 128] bf16
-constexpr int B_K = 0, B_V = F_TILE, B_Q = 2 * F_TILE, B_DO = B_Q + 2 * B_QTILE;
-constexpr int B_PT = B_DO + 2 * B_QTILE;              // P^T [128 keys x 64 queries]: 16 KB, two buffers
+constexpr int B_NQD = 3;                              // slots of the Q / dO / lse / D ring
+constexpr int B_K = 0, B_V = F_TILE, B_Q = 2 * F_TILE, B_DO = B_Q + B_NQD * B_QTILE;
+constexpr int B_PT = B_DO + B_NQD * B_QTILE;          // P^T [128 keys x 64 queries]: 16 KB, two buffers
 constexpr int B_DST = B_PT + 2 * F_ATOM;              // dS^T, same shape, two buffers
-constexpr int B_LD = B_DST + 2 * F_ATOM;              // [2 stages][lse 64 | D 64] fp32
-constexpr int B_CTL = B_LD + 1024;
-constexpr int B_SMEM = B_CTL + 1024 + 1024;
+constexpr int B_LD = B_DST + 2 * F_ATOM;              // [slot][lse 64 | D 64] fp32
+constexpr int B_CTL = B_LD + B_NQD * 512;
+constexpr int B_SMEM = B_CTL + 256 + 1024;            // + barriers + alignment slack
+static_assert(sizeof(Ctl) <= 256 && B_SMEM <= 227 * 1024, "dKV shared memory");
 
 __global__ void __launch_bounds__(FA_THREADS, 1)
     flash_bwd_dkv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -327,11 +329,11 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   Ctl* ctl = reinterpret_cast<Ctl*>(smem + B_CTL);
   uint64_t* kv_full = &ctl->bar[0];
-  uint64_t* qd_full = &ctl->bar[1];      // [2]
-  uint64_t* qd_empty = &ctl->bar[3];     // [2]
-  uint64_t* s_full = &ctl->bar[5];       // [2]: S^T and dP^T of a query block ready
-  uint64_t* p_full = &ctl->bar[7];       // P^T, dS^T written
-  uint64_t* g_done = &ctl->bar[8];       // [2]: dV / dK products that read P^T / dS^T buffer b done
+  uint64_t* qd_full = &ctl->bar[1];      // [B_NQD]
+  uint64_t* qd_empty = &ctl->bar[1 + B_NQD];   // [B_NQD]
+  uint64_t* s_full = &ctl->bar[1 + 2 * B_NQD];   // [2]: S^T and dP^T of a query block ready
+  uint64_t* p_full = &ctl->bar[3 + 2 * B_NQD];   // P^T, dS^T written
+  uint64_t* g_done = &ctl->bar[4 + 2 * B_NQD];   // [2]: dV / dK products that read P^T / dS^T buffer b done
   volatile int* abort_flag = &ctl->abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -343,7 +345,8 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(kv_full, 1);
-    for (int s = 0; s < 2; ++s) { mbar_init(&qd_full[s], 1); mbar_init(&qd_empty[s], 1); mbar_init(&s_full[s], 1); }
+    for (int s = 0; s < B_NQD; ++s) { mbar_init(&qd_full[s], 1); mbar_init(&qd_empty[s], 1); }
+    for (int s = 0; s < 2; ++s) mbar_init(&s_full[s], 1);
     mbar_init(p_full, 8);
     mbar_init(&g_done[0], 1);
     mbar_init(&g_done[1], 1);
@@ -362,14 +365,14 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     load_tile(&tmK, kv_full, smem + B_K, g * HD, kb * 128, F_ATOM);
     load_tile(&tmV, kv_full, smem + B_V, g * HD, kb * 128, F_ATOM);
     for (int it = 0; it < nit && !*abort_flag; ++it) {
-      const int s = it & 1;
+      const int s = it % B_NQD;
       const int h = g * p.rep + it / niq, qi = i0 + it % niq;
-      if (!waitb(&qd_empty[s], ((it >> 1) & 1) ^ 1, p.status, abort_flag)) break;
+      if (!waitb(&qd_empty[s], ((it / B_NQD) & 1) ^ 1, p.status, abort_flag)) break;
       const uint32_t nb = (uint32_t)min(64, p.T - qi * 64) * 4;     // lse / D bytes inside [0, T)
       mbar_expect_tx(&qd_full[s], 2 * B_QTILE + 2 * nb);
       load_tile(&tmQ, &qd_full[s], smem + B_Q + s * B_QTILE, h * HD, qi * 64, B_QATOM);
       load_tile(&tmdO, &qd_full[s], smem + B_DO + s * B_QTILE, h * HD, qi * 64, B_QATOM);
-      float* ld = reinterpret_cast<float*>(smem + B_LD + s * 512);
+      float* ld = reinterpret_cast<float*>(smem + B_LD + s * 512);    // s: the ring slot
       bulk_g2s(ld, p.lse + (int64_t)h * p.T + qi * 64, nb, &qd_full[s]);
       bulk_g2s(ld + 64, p.D + (int64_t)h * p.T + qi * 64, nb, &qd_full[s]);
     }
@@ -379,33 +382,35 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     const uint32_t sq = smem_u32(smem + B_Q), sd = smem_u32(smem + B_DO);
     const uint32_t spt = smem_u32(smem + B_PT), sdst = smem_u32(smem + B_DST);
     bool ok = waitb(kv_full, 0, p.status, abort_flag);
+    // ring slot r = it % B_NQD holds Q, dO of iteration it; S^T / dP^T (tensor memory) and P^T /
+    // dS^T (shared memory) are double-buffered by b = it & 1
     auto issue_s = [&](int it) -> bool {
-      const int s = it & 1;
-      if (!waitb(&qd_full[s], (it >> 1) & 1, p.status, abort_flag)) return false;
+      const int r = it % B_NQD, b = it & 1;
+      if (!waitb(&qd_full[r], (it / B_NQD) & 1, p.status, abort_flag)) return false;
       tc_fence_after();
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
-        umma_bf16(tmem + 64 * s, desc_k(sk, kk, F_ATOM), desc_k(sq + s * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
-        umma_bf16(tmem + 128 + 64 * s, desc_k(sv, kk, F_ATOM), desc_k(sd + s * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
+        umma_bf16(tmem + 64 * b, desc_k(sk, kk, F_ATOM), desc_k(sq + r * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
+        umma_bf16(tmem + 128 + 64 * b, desc_k(sv, kk, F_ATOM), desc_k(sd + r * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
       }
-      umma_commit(&s_full[s]);
+      umma_commit(&s_full[b]);
       return true;
     };
     if (ok && nit > 0) ok = issue_s(0);
     for (int it = 0; ok && it < nit; ++it) {
-      const int s = it & 1;
+      const int r = it % B_NQD, b = it & 1;
       if (it + 1 < nit && !issue_s(it + 1)) break;
       if (!waitb(p_full, it & 1, p.status, abort_flag)) break;
       tc_fence_after();
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk) {               // K = 64 queries
-        umma_bf16(tmem + 256, desc_k(spt + s * F_ATOM, kk, F_ATOM), desc_mn(sd + s * B_QTILE, kk, B_QATOM), ID_G,
+        umma_bf16(tmem + 256, desc_k(spt + b * F_ATOM, kk, F_ATOM), desc_mn(sd + r * B_QTILE, kk, B_QATOM), ID_G,
                   (it | kk) != 0);
-        umma_bf16(tmem + 384, desc_k(sdst + s * F_ATOM, kk, F_ATOM), desc_mn(sq + s * B_QTILE, kk, B_QATOM), ID_G,
+        umma_bf16(tmem + 384, desc_k(sdst + b * F_ATOM, kk, F_ATOM), desc_mn(sq + r * B_QTILE, kk, B_QATOM), ID_G,
                   (it | kk) != 0);
       }
-      umma_commit(&g_done[s]);
-      umma_commit(&qd_empty[s]);
+      umma_commit(&g_done[b]);
+      umma_commit(&qd_empty[r]);
     }
   } else if (warp >= 2) {
     const int q = warp & 3, half = (warp - 2) >> 2;   // half: which 32 of the 64 query columns
@@ -418,7 +423,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     for (int it = 0; it < nit; ++it) {
       const int s = it & 1;
       const int qi = i0 + it % niq;
-      const float* L = reinterpret_cast<const float*>(smem + B_LD + s * 512);
+      const float* L = reinterpret_cast<const float*>(smem + B_LD + (it % B_NQD) * 512);
       const float* Dq = L + 64;
       // queries below the key block's last key, or past T, need the mask; the rest see every key
       const bool need_mask = qi * 64 < kb * 128 + 127 || qi * 64 + 64 > p.T;
@@ -493,9 +498,11 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
 // ================================================================================================
 // backward, dQ: one CTA per (128-query block, query head), 64-key blocks, S / dP / dS double-buffered
 // ================================================================================================
-constexpr int Q_Q = 0, Q_DO = F_TILE, Q_K = 2 * F_TILE, Q_V = Q_K + 2 * B_QTILE, Q_DS = Q_V + 2 * B_QTILE;
+constexpr int Q_NKV = 4;                              // slots of the K / V ring
+constexpr int Q_Q = 0, Q_DO = F_TILE, Q_K = 2 * F_TILE, Q_V = Q_K + Q_NKV * B_QTILE, Q_DS = Q_V + Q_NKV * B_QTILE;
 constexpr int Q_CTL = Q_DS + 2 * F_ATOM;
-constexpr int Q_SMEM = Q_CTL + 1024 + 1024;
+constexpr int Q_SMEM = Q_CTL + 256 + 1024;            // + barriers + alignment slack
+static_assert(Q_SMEM <= 227 * 1024, "dQ shared memory");
 
 __global__ void __launch_bounds__(FA_THREADS, 1)
     flash_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -505,11 +512,11 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   Ctl* ctl = reinterpret_cast<Ctl*>(smem + Q_CTL);
   uint64_t* q_full = &ctl->bar[0];
-  uint64_t* kv_full = &ctl->bar[1];      // [2]
-  uint64_t* kv_empty = &ctl->bar[3];     // [2]
-  uint64_t* s_full = &ctl->bar[5];       // [2]: S and dP of a key block ready
-  uint64_t* p_full = &ctl->bar[7];       // dS written
-  uint64_t* g_done = &ctl->bar[8];       // [2]: dQ product that read dS buffer b done
+  uint64_t* kv_full = &ctl->bar[1];      // [Q_NKV]
+  uint64_t* kv_empty = &ctl->bar[1 + Q_NKV];     // [Q_NKV]
+  uint64_t* s_full = &ctl->bar[1 + 2 * Q_NKV];   // [2]: S and dP of a key block ready
+  uint64_t* p_full = &ctl->bar[3 + 2 * Q_NKV];   // dS written
+  uint64_t* g_done = &ctl->bar[4 + 2 * Q_NKV];   // [2]: dQ product that read dS buffer b done
   volatile int* abort_flag = &ctl->abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -520,9 +527,8 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(&kv_full[s], 1); mbar_init(&kv_empty[s], 1); mbar_init(&s_full[s], 1);
-    }
+    for (int s = 0; s < Q_NKV; ++s) { mbar_init(&kv_full[s], 1); mbar_init(&kv_empty[s], 1); }
+    for (int s = 0; s < 2; ++s) mbar_init(&s_full[s], 1);
     mbar_init(p_full, 8);
     mbar_init(&g_done[0], 1);
     mbar_init(&g_done[1], 1);
@@ -540,8 +546,8 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     load_tile(&tmQ, q_full, smem + Q_Q, h * HD, qb * 128, F_ATOM);
     load_tile(&tmdO, q_full, smem + Q_DO, h * HD, qb * 128, F_ATOM);
     for (int j = 0; j < nkb && !*abort_flag; ++j) {
-      const int s = j & 1;
-      if (!waitb(&kv_empty[s], ((j >> 1) & 1) ^ 1, p.status, abort_flag)) break;
+      const int s = j % Q_NKV;
+      if (!waitb(&kv_empty[s], ((j / Q_NKV) & 1) ^ 1, p.status, abort_flag)) break;
       mbar_expect_tx(&kv_full[s], 2 * B_QTILE);
       load_tile(&tmK, &kv_full[s], smem + Q_K + s * B_QTILE, g * HD, j * 64, B_QATOM);
       load_tile(&tmV, &kv_full[s], smem + Q_V + s * B_QTILE, g * HD, j * 64, B_QATOM);
@@ -551,31 +557,33 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     const uint32_t sq = smem_u32(smem + Q_Q), sd = smem_u32(smem + Q_DO);
     const uint32_t sk = smem_u32(smem + Q_K), sv = smem_u32(smem + Q_V), sds = smem_u32(smem + Q_DS);
     bool ok = waitb(q_full, 0, p.status, abort_flag);
+    // ring slot r = j % Q_NKV holds K, V of key block j; S / dP (tensor memory) and dS (shared
+    // memory) are double-buffered by b = j & 1
     auto issue_s = [&](int j) -> bool {
-      const int s = j & 1;
-      if (!waitb(&kv_full[s], (j >> 1) & 1, p.status, abort_flag)) return false;
+      const int r = j % Q_NKV, b = j & 1;
+      if (!waitb(&kv_full[r], (j / Q_NKV) & 1, p.status, abort_flag)) return false;
       tc_fence_after();
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
-        umma_bf16(tmem + 64 * s, desc_k(sq, kk, F_ATOM), desc_k(sk + s * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
-        umma_bf16(tmem + 128 + 64 * s, desc_k(sd, kk, F_ATOM), desc_k(sv + s * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
+        umma_bf16(tmem + 64 * b, desc_k(sq, kk, F_ATOM), desc_k(sk + r * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
+        umma_bf16(tmem + 128 + 64 * b, desc_k(sd, kk, F_ATOM), desc_k(sv + r * B_QTILE, kk, B_QATOM), ID_S, kk > 0);
       }
-      umma_commit(&s_full[s]);
+      umma_commit(&s_full[b]);
       return true;
     };
     if (ok) ok = issue_s(0);
     for (int j = 0; ok && j < nkb; ++j) {
-      const int s = j & 1;
+      const int r = j % Q_NKV, b = j & 1;
       // S / dP buffer (j+1)&1 was last read at j-1, whose p_full was waited for below
       if (j + 1 < nkb && !issue_s(j + 1)) break;
       if (!waitb(p_full, j & 1, p.status, abort_flag)) break;
       tc_fence_after();
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk)               // K = 64 keys
-        umma_bf16(tmem + 256, desc_k(sds + s * F_ATOM, kk, F_ATOM), desc_mn(sk + s * B_QTILE, kk, B_QATOM), ID_G,
+        umma_bf16(tmem + 256, desc_k(sds + b * F_ATOM, kk, F_ATOM), desc_mn(sk + r * B_QTILE, kk, B_QATOM), ID_G,
                   (j | kk) != 0);
-      umma_commit(&g_done[s]);
-      umma_commit(&kv_empty[s]);
+      umma_commit(&g_done[b]);
+      umma_commit(&kv_empty[r]);
     }
   } else if (warp >= 2) {
     const int q = warp & 3, half = (warp - 2) >> 2;   // half: which 32 of the 64 key columns
