@@ -93,8 +93,13 @@ struct FwdP {
 
 constexpr int F_TILE = 128 * ROW_BYTES * 2;           // 32 KB: [128 x 128] bf16
 constexpr int F_ATOM = 128 * ROW_BYTES;               // 16 KB
-constexpr int F_Q = 0, F_K = F_TILE, F_V = 3 * F_TILE, F_P = 5 * F_TILE, F_ST = 6 * F_TILE, F_CTL = F_ST + 2048;
-constexpr int F_SMEM = F_CTL + 1024 + 1024;
+// K and V in separate rings: K (three slots) is free once S is formed, V (two slots) once P V is
+constexpr int F_NK = 3, F_NV = 2;
+constexpr int F_Q = 0, F_K = F_TILE, F_V = F_K + F_NK * F_TILE, F_P = F_V + F_NV * F_TILE;
+constexpr int F_ST = F_P;                             // row statistics: in the P tile before P is written
+constexpr int F_CTL = F_P + F_TILE;
+constexpr int F_SMEM = F_CTL + 256 + 1024;            // + barriers + alignment slack
+static_assert(F_SMEM <= 227 * 1024, "forward shared memory");
 
 __global__ void __launch_bounds__(FA_THREADS, 1)
     flash_fwd_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -103,11 +108,13 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   Ctl* ctl = reinterpret_cast<Ctl*>(smem + F_CTL);
   uint64_t* q_full = &ctl->bar[0];
-  uint64_t* kv_full = &ctl->bar[1];       // [2]
-  uint64_t* kv_empty = &ctl->bar[3];      // [2]
-  uint64_t* s_full = &ctl->bar[5];        // [2]
-  uint64_t* p_full = &ctl->bar[7];
-  uint64_t* o_done = &ctl->bar[8];
+  uint64_t* k_full = &ctl->bar[1];        // [F_NK]
+  uint64_t* k_empty = &ctl->bar[4];       // [F_NK]
+  uint64_t* v_full = &ctl->bar[7];        // [F_NV]
+  uint64_t* v_empty = &ctl->bar[9];       // [F_NV]
+  uint64_t* s_full = &ctl->bar[11];       // [2]
+  uint64_t* p_full = &ctl->bar[13];
+  uint64_t* o_done = &ctl->bar[14];
   volatile int* abort_flag = &ctl->abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -119,7 +126,9 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < 2; ++s) { mbar_init(&kv_full[s], 1); mbar_init(&kv_empty[s], 1); mbar_init(&s_full[s], 1); }
+    for (int s = 0; s < F_NK; ++s) { mbar_init(&k_full[s], 1); mbar_init(&k_empty[s], 1); }
+    for (int s = 0; s < F_NV; ++s) { mbar_init(&v_full[s], 1); mbar_init(&v_empty[s], 1); }
+    for (int s = 0; s < 2; ++s) mbar_init(&s_full[s], 1);
     mbar_init(p_full, 8);
     mbar_init(o_done, 1);
     ctl->abort = 0;
@@ -138,11 +147,17 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     mbar_expect_tx(q_full, F_TILE);
     load_tile(&tmQ, q_full, smem + F_Q, h * HD, qb * 128, F_ATOM);
     for (int it = 0; it < nit && !*abort_flag; ++it) {
-      const int s = it & 1, j = it < nkb ? it : it - nkb;
-      if (!waitb(&kv_empty[s], ((it >> 1) & 1) ^ 1, p.status, abort_flag)) break;
-      mbar_expect_tx(&kv_full[s], it < nkb ? F_TILE : 2 * F_TILE);
-      load_tile(&tmK, &kv_full[s], smem + F_K + s * F_TILE, g * HD, j * 128, F_ATOM);
-      if (it >= nkb) load_tile(&tmV, &kv_full[s], smem + F_V + s * F_TILE, g * HD, j * 128, F_ATOM);
+      const int j = it < nkb ? it : it - nkb;
+      const int sk = it % F_NK;
+      if (!waitb(&k_empty[sk], ((it / F_NK) & 1) ^ 1, p.status, abort_flag)) break;
+      mbar_expect_tx(&k_full[sk], F_TILE);
+      load_tile(&tmK, &k_full[sk], smem + F_K + sk * F_TILE, g * HD, j * 128, F_ATOM);
+      if (it >= nkb) {
+        const int sv = j % F_NV;
+        if (!waitb(&v_empty[sv], ((j / F_NV) & 1) ^ 1, p.status, abort_flag)) break;
+        mbar_expect_tx(&v_full[sv], F_TILE);
+        load_tile(&tmV, &v_full[sv], smem + F_V + sv * F_TILE, g * HD, j * 128, F_ATOM);
+      }
     }
   } else if (warp == 1 && lane == 0) {
     constexpr uint32_t ID_S = idesc_bf16(128, 128, 0, 0), ID_O = idesc_bf16(128, 128, 0, 1);
@@ -150,14 +165,14 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     const uint32_t sp = smem_u32(smem + F_P);
     bool ok = waitb(q_full, 0, p.status, abort_flag);
     auto issue_s = [&](int it) -> bool {
-      const int s = it & 1;
-      if (!waitb(&kv_full[s], (it >> 1) & 1, p.status, abort_flag)) return false;
+      const int s = it & 1, r = it % F_NK;
+      if (!waitb(&k_full[r], (it / F_NK) & 1, p.status, abort_flag)) return false;
       tc_fence_after();
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk)
-        umma_bf16(tmem + 128 * s, desc_k(sq, kk, F_ATOM), desc_k(sk + s * F_TILE, kk, F_ATOM), ID_S, kk > 0);
+        umma_bf16(tmem + 128 * s, desc_k(sq, kk, F_ATOM), desc_k(sk + r * F_TILE, kk, F_ATOM), ID_S, kk > 0);
       umma_commit(&s_full[s]);
-      if (it < nkb) umma_commit(&kv_empty[s]);      // statistics pass: K is free once S is formed
+      umma_commit(&k_empty[r]);                       // K is free once S is formed
       return true;
     };
     if (ok) ok = issue_s(0);
@@ -167,13 +182,14 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       if (!waitb(p_full, it & 1, p.status, abort_flag)) break;
       tc_fence_after();
       if (it >= nkb) {
-        const int j = it - nkb;
+        const int j = it - nkb, r = j % F_NV;
+        if (!waitb(&v_full[r], (j / F_NV) & 1, p.status, abort_flag)) break;
+        tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          umma_bf16(tmem + 256, desc_k(sp, kk, F_ATOM), desc_mn(sv + (it & 1) * F_TILE, kk, F_ATOM), ID_O,
-                    (j | kk) != 0);
+          umma_bf16(tmem + 256, desc_k(sp, kk, F_ATOM), desc_mn(sv + r * F_TILE, kk, F_ATOM), ID_O, (j | kk) != 0);
         umma_commit(o_done);
-        umma_commit(&kv_empty[it & 1]);
+        umma_commit(&v_empty[r]);
       }
     }
   } else if (warp >= 2) {
@@ -225,6 +241,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     stat[(half * 2 + 1) * 128 + r] = l;
     asm volatile("bar.sync 1, 256;" ::: "memory");
     const float mo = stat[((1 - half) * 2 + 0) * 128 + r], lo = stat[((1 - half) * 2 + 1) * 128 + r];
+    asm volatile("bar.sync 1, 256;" ::: "memory");   // statistics read before P overwrites them
     const float mt = fmaxf(m, mo);
     const float lt = (m == -INFINITY ? 0.f : l * ex2(m - mt)) + (mo == -INFINITY ? 0.f : lo * ex2(mo - mt));
     const float inv_l = 1.f / lt;
