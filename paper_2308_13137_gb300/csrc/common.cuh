@@ -134,19 +134,21 @@ __device__ __forceinline__ float omq_code_raw(float w, const QState& s, float* x
   return rintf(x) + s.z;
 }
 
+// clamp(rint(w/h) + z, 0, Q) - z formed as clamp(rint(w/h), -z, Q - z): every term is an integer
+// below 2^24 after the clamp, so both forms give the same value
 __device__ __forceinline__ float omq_fakequant(float w, const QState& s, float Q, float* code) {
-  float x;
-  float c = omq_code_raw(w, s, &x);
-  float q = fminf(fmaxf(c, 0.f), Q);
-  if (code) *code = q;
-  return __fmul_rn(q - s.z, s.h);
+  const float r = rintf(__fmul_rn(w, s.rh));
+  const float qz = fminf(fmaxf(r, -s.z), Q - s.z);
+  if (code) *code = qz + s.z;
+  return __fmul_rn(qz, s.h);
 }
 
 // STE pieces of one element: returns dwhat/dh; *inr = 1 when 0 <= c <= Q
 __device__ __forceinline__ float omq_ste_dh(float w, const QState& s, float Q, int* inr) {
-  float x;
-  float c = omq_code_raw(w, s, &x);
-  if (c >= 0.f && c <= Q) { *inr = 1; return rintf(x) - x; }
+  const float x = __fmul_rn(w, s.rh);
+  const float r = rintf(x);
+  const float c = r + s.z;
+  if (c >= 0.f && c <= Q) { *inr = 1; return r - x; }
   *inr = 0;
   float ru = rintf(s.u) - s.u;
   return (c < 0.f) ? ru : (Q + ru);

@@ -253,12 +253,21 @@ __global__ void __launch_bounds__(NT) lwc_fwd_row_kernel(LwcFwdArgs a) {
     if (c < nchunk) {
       float w8[8], sv[8];
       unpack_bf16x8(raw[j], w8);
-      load8(a.s, c, sv, 1.f);
+      // W~ = fl(fl(W s) r); a factor that is absent is 1 and its product is skipped (exact)
+      if (a.s) {
+        load8(a.s, c, sv, 1.f);
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        wt[j][e] = __fmul_rn(__fmul_rn(w8[e], sv[e]), rr);
-        M = fmaxf(M, wt[j][e]); m = fminf(m, wt[j][e]);
+        for (int e = 0; e < 8; ++e) wt[j][e] = __fmul_rn(w8[e], sv[e]);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) wt[j][e] = w8[e];
       }
+      if (a.r) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) wt[j][e] = __fmul_rn(wt[j][e], rr);
+      }
+#pragma unroll
+      for (int e = 0; e < 8; ++e) { M = fmaxf(M, wt[j][e]); m = fminf(m, wt[j][e]); }
       if (a.Bt) {
         float dv[8];
         load8(a.bias_delta, c, dv, 0.f);
