@@ -260,6 +260,7 @@ omq_status lwc_bwd_dw(cudaStream_t st, int64_t T, const bf16* dY, const bf16* Xh
   lw.part_s = ds ? part : nullptr;
   lw.part_d = (ddelta && dBt) ? part + P * Cin : nullptr;
   lw.rowpart = part + 2 * P * Cin;
+  lw.want_dr = dr != nullptr;
   lw.dgl = dgl; lw.dbl = dbl;
   lw.group = group; lw.accumulate = cfg.accumulate; lw.ntn = ntn;
   lw.Q = (float)((1 << cfg.wbits) - 1); lw.eps = cfg.h_eps;

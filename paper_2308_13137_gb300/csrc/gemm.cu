@@ -101,6 +101,42 @@ __device__ __forceinline__ void ldw32(const __nv_bfloat16* p, bool ok, uint4 (&r
   for (int i = 0; i < 4; ++i) r[i] = ok ? __ldg(reinterpret_cast<const uint4*>(p) + i) : make_uint4(0, 0, 0, 0);
 }
 
+// The per-element part of the LWC backward for one 32-column chunk of a row: W~ = fl(fl(W s) r),
+// the code decision, the STE mask and h-path sums, and the LET column terms.  HS / HR: the column
+// scale s / row scale r are present (an absent one is 1, its product skipped, exactly); DR: the row
+// sum for dr is wanted; LET: the column terms for ds (cs) and ddelta (cd).
+template <bool HS, bool HR, bool DR, bool LET>
+__device__ __forceinline__ void lwc_elems(const uint4 (&wc)[4], const float* s_nb, float rr, float dbr, const QState& qs,
+                                          float Q, const float (&g)[32], float& Gh, float& Gbm, float& drm,
+                                          float (&cs)[32], float (&cd)[32]) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    float w8[8], s8[8];
+    unpack_bf16x8(wc[i], w8);
+    if (HS) {
+      const float4 a = __ldg(reinterpret_cast<const float4*>(s_nb) + 2 * i);
+      const float4 b = __ldg(reinterpret_cast<const float4*>(s_nb) + 2 * i + 1);
+      s8[0] = a.x; s8[1] = a.y; s8[2] = a.z; s8[3] = a.w; s8[4] = b.x; s8[5] = b.y; s8[6] = b.z; s8[7] = b.w;
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const int k = 8 * i + e;
+      float wt = HS ? __fmul_rn(w8[e], s8[e]) : w8[e];
+      if (HR) wt = __fmul_rn(wt, rr);
+      int inr;
+      const float dh = omq_ste_dh(wt, qs, Q, &inr);
+      Gh = fmaf(g[k], dh, Gh);
+      if (!inr) Gbm += g[k];
+      const float d = inr ? g[k] : 0.f;
+      if (DR) drm = fmaf(d * w8[e], HS ? s8[e] : 1.f, drm);
+      if (LET) {
+        cs[k] = HR ? (d * w8[e]) * rr : d * w8[e];
+        cd[k] = dbr * w8[e];
+      }
+    }
+  }
+}
+
 // Epilogue of the weight-gradient product with the straight-through LWC backward (Eq. 2) fused:
 // the accumulator dW_hat is consumed from tensor memory 32 columns at a time and never stored.
 // The weight row chunk of the next 32 columns is loaded while the current one is processed.
@@ -117,7 +153,7 @@ __device__ __forceinline__ void release_acc(uint64_t* acc_empty, uint32_t buf, i
 
 // Eight epilogue warps: warps w and w+4 drain the same 32 accumulator rows (lane quadrant w % 4),
 // `half` 0 the first BN / 2 columns of the tile, 1 the others; each keeps its own row partials.
-template <int BN, bool PAIR>
+template <int BN, bool PAIR, int FORM>
 __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem, uint64_t* acc_full, uint64_t* acc_empty,
                                              volatile int* abort_flag, int q, int half, int lane, int total, int rank) {
   constexpr int HB = BN / 2;                      // columns of a half
@@ -186,33 +222,12 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
           Gh = 0.f; Gbm = 0.f;
         }
         float cs[32], cd[32];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          float w8[8];
-          unpack_bf16x8(wcur[i], w8);
-          float s8[8];
-          if (L.s) {
-            const float4 a = __ldg(reinterpret_cast<const float4*>(L.s + nb) + 2 * i);
-            const float4 b = __ldg(reinterpret_cast<const float4*>(L.s + nb) + 2 * i + 1);
-            s8[0] = a.x; s8[1] = a.y; s8[2] = a.z; s8[3] = a.w; s8[4] = b.x; s8[5] = b.y; s8[6] = b.z; s8[7] = b.w;
-          } else {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) s8[e] = 1.f;
-          }
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const int k = 8 * i + e;
-            const float wt = __fmul_rn(__fmul_rn(w8[e], s8[e]), rr);
-            int inr;
-            const float dh = omq_ste_dh(wt, qs, L.Q, &inr);
-            Gh = fmaf(g[k], dh, Gh);
-            if (!inr) Gbm += g[k];
-            const float d = inr ? g[k] : 0.f;
-            drm = fmaf(d * w8[e], s8[e], drm);
-            cs[k] = (d * w8[e]) * rr;
-            cd[k] = dbr * w8[e];
-          }
-        }
+        // without LET only the STE part; with it every term (an absent s or r is 1: products by it
+        // are exact)
+        if (FORM == 2) lwc_elems<false, false, false, false>(wcur, nullptr, rr, dbr, qs, L.Q, g, Gh, Gbm, drm, cs, cd);
+        else if (FORM == 3) lwc_elems<true, false, false, true>(wcur, L.s + nb, rr, dbr, qs, L.Q, g, Gh, Gbm, drm, cs, cd);
+        else if (L.s) lwc_elems<true, true, true, true>(wcur, L.s + nb, rr, dbr, qs, L.Q, g, Gh, Gbm, drm, cs, cd);
+        else lwc_elems<false, true, true, true>(wcur, nullptr, rr, dbr, qs, L.Q, g, Gh, Gbm, drm, cs, cd);
         const int64_t prow = (int64_t)(row0 >> 5) * N + nb + lane;
         if (L.part_s) {
           const float v = colsum_warp32(cs, lane);
@@ -255,7 +270,9 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
 // (both TMA loads complete on the leader CTA's mbarrier), the leader issues the MMAs, commits
 // reach both CTAs' barriers, and each CTA drains its own BM rows of the accumulator.  Per CTA
 // the shared-memory bytes per MMA flop halve for B, so six stages fit where four did.
-template <int BN, int STAGES, bool LWC, bool PAIR>
+// LWC: 0 plain product; LWC epilogue 1 general, 2 without LET terms, 3 with the LET column scale but
+// neither row scale nor dr
+template <int BN, int STAGES, int LWC, bool PAIR>
 __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
     gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const __grid_constant__ CUtensorMap tmC, const GemmParams p) {
@@ -388,7 +405,7 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
       if (!ok) break;
     }
   } else if (LWC && warp >= 2) {
-    lwc_epilogue<BN, PAIR>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, (warp - 2) >> 2, lane, total, rank);
+    lwc_epilogue<BN, PAIR, LWC>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, (warp - 2) >> 2, lane, total, rank);
   } else if (warp >= 2) {
     // ---------------- epilogue ----------------
     // fp32 output leaves through TMA bulk stores: each warp stages its 32 x 32 block in one of two
@@ -553,7 +570,7 @@ bool make_map_c(CUtensorMap* map, float* ptr, int64_t N, int64_t M, int64_t batc
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES, bool LWC = false, bool PAIR = false>
+template <int BN, int STAGES, int LWC = 0, bool PAIR = false>
 omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
                       const GemmParams& p) {
   using L = SmemLayout<BN, STAGES, PAIR>;
@@ -674,7 +691,7 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
       g_prof.flops += gemm_algorithmic_flops(M, N, K, batch, causal);
     }
   }
-  omq_status r = pair ? launch_cfg<256, 6, false, true>(st, ta, tb, tc, p)
+  omq_status r = pair ? launch_cfg<256, 6, 0, true>(st, ta, tb, tc, p)
                       : (wide ? launch_cfg<256, 4>(st, ta, tb, tc, p) : launch_cfg<128, 6>(st, ta, tb, tc, p));
   if (e0 && e1) cudaEventRecord(e1, st);
   return r;
@@ -736,8 +753,12 @@ omq_status gemm_launch_lwc(cudaStream_t st, int64_t M, int64_t N, int64_t K, con
       g_prof.flops += gemm_algorithmic_flops(M, N, K, 1, 0);
     }
   }
-  omq_status r = pair ? launch_cfg<256, 6, true, true>(st, ta, tb, tc, p)
-                      : (bn == 256 ? launch_cfg<256, 4, true>(st, ta, tb, tc, p) : launch_cfg<128, 6, true>(st, ta, tb, tc, p));
+  const bool nolet = !lw.s && !lw.r && !lw.want_dr && !lw.part_s && !lw.part_d;
+  const bool scale_only = lw.s && !lw.r && !lw.want_dr;
+  omq_status r = pair ? (nolet        ? launch_cfg<256, 6, 2, true>(st, ta, tb, tc, p)
+                         : scale_only ? launch_cfg<256, 6, 3, true>(st, ta, tb, tc, p)
+                                      : launch_cfg<256, 6, 1, true>(st, ta, tb, tc, p))
+                      : (bn == 256 ? launch_cfg<256, 4, 1>(st, ta, tb, tc, p) : launch_cfg<128, 6, 1>(st, ta, tb, tc, p));
   if (e0 && e1) cudaEventRecord(e1, st);
   return r;
 }

@@ -39,6 +39,7 @@ struct GemmLwcEpi {
   float* dgl; float* dbl;         // grouped: [M, N/group]
   int group, accumulate, ntn;
   float Q, eps;
+  int want_dr;                    // the row sums for dr (rowpart[2]) are needed
 };
 
 // N-tile width the GEMM uses for a product with N columns
