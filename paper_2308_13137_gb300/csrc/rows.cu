@@ -881,11 +881,13 @@ __global__ void __launch_bounds__(NT) qkv_fwd_rows(QkvArgs a) {
 // recomputes that pair with the routing added and rewrites it.
 #define QKV_BWD_NT 256
 
-template <int PPT, int MINB>
-__global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
+// SEG < 0: the three segments of every row in turn; SEG = 0, 1, 2: the q, k or v segment only (a
+// CTA of each segment per row slab, so that the three run side by side).
+template <int PPT, int SEG>
+__device__ __forceinline__ void qkv_bwd_body(const QkvArgs& a, float* fsm) {
   constexpr int NT = QKV_BWD_NT;
   constexpr int NE = 8 * PPT;
-  __shared__ float fsm[96];
+  constexpr bool HAS_Q = SEG < 0 || SEG == 0, HAS_K = SEG < 0 || SEG == 1;
   const int tid = threadIdx.x;
   const int dq = a.H * a.hd, dkv = a.Hkv * a.hd;
   const bool sums = a.part_q != nullptr;
@@ -894,7 +896,7 @@ __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
   const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
   float acc_q[NE], acc_k[NE], rq[NE];      // rq: 1/s_a of the thread's query columns, computed once
 #pragma unroll
-  for (int j = 0; j < PPT; ++j) {
+  for (int j = 0; j < (HAS_Q ? PPT : 0); ++j) {
     const int p = j * NT + tid;
     const int e1 = (p >> 4) * 128 + 4 * (p & 15);
     const bool ok = a.sa_exp != nullptr && p < a.H * 16;
@@ -910,7 +912,7 @@ __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
   for (int k = 0; k < NE; ++k) { acc_q[k] = 0.f; acc_k[k] = 0.f; }
   const int t0 = blockIdx.x * a.rows_per_cta, t1 = min(a.T, t0 + a.rows_per_cta);
   for (int t = t0; t < t1; ++t) {
-    for (int seg = 0; seg < 3; ++seg) {
+    for (int seg = (SEG < 0 ? 0 : SEG); seg < (SEG < 0 ? 3 : SEG + 1); ++seg) {
       const int Hs = seg == 0 ? a.H : a.Hkv;
       const int np = Hs * 16;
       const int off = seg == 0 ? 0 : (seg == 1 ? dq : dq + dkv);
@@ -1057,17 +1059,32 @@ __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
       const int e1 = (p >> 4) * 128 + 4 * (p & 15);
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        if (p < a.H * 16) {
+        if (HAS_Q && p < a.H * 16) {
           a.part_q[(int64_t)blockIdx.x * dq + e1 + e] = acc_q[8 * j + e] * rq[8 * j + e];
           a.part_q[(int64_t)blockIdx.x * dq + e1 + 64 + e] = acc_q[8 * j + 4 + e] * rq[8 * j + 4 + e];
         }
-        if (p < a.Hkv * 16) {
+        if (HAS_K && p < a.Hkv * 16) {
           a.part_k[(int64_t)blockIdx.x * dkv + e1 + e] = acc_k[8 * j + e];
           a.part_k[(int64_t)blockIdx.x * dkv + e1 + 64 + e] = acc_k[8 * j + 4 + e];
         }
       }
     }
   }
+}
+
+template <int PPT, int MINB>
+__global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
+  __shared__ float fsm[96];
+  qkv_bwd_body<PPT, -1>(a, fsm);
+}
+
+// one CTA per (row slab, segment): blockIdx.y picks q, k or v
+template <int PPT, int MINB>
+__global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_seg(QkvArgs a) {
+  __shared__ float fsm[96];
+  if (blockIdx.y == 0) qkv_bwd_body<PPT, 0>(a, fsm);
+  else if (blockIdx.y == 1) qkv_bwd_body<PPT, 1>(a, fsm);
+  else qkv_bwd_body<PPT, 2>(a, fsm);
 }
 
 int64_t qkv_bwd_nslab(int T) { return (T + 3) / 4; }
@@ -1091,7 +1108,7 @@ omq_status qkv_bwd_launch(cudaStream_t st, const QkvArgs& a0, int64_t* nslab) {
   const unsigned grid = (unsigned)qkv_bwd_nslab(a.T);
   const int np = a.H * 16;
   if (np <= 256) qkv_bwd_stream<1, 4><<<grid, QKV_BWD_NT, 0, st>>>(a);
-  else if (np <= 512) qkv_bwd_stream<2, 2><<<grid, QKV_BWD_NT, 0, st>>>(a);
+  else if (np <= 512) qkv_bwd_seg<2, 2><<<dim3(grid, 3), QKV_BWD_NT, 0, st>>>(a);
   else if (np <= 1024) qkv_bwd_stream<4, 1><<<grid, QKV_BWD_NT, 0, st>>>(a);
   else if (np <= 2048) qkv_bwd_stream<8, 1><<<grid, QKV_BWD_NT, 0, st>>>(a);
   else return OMQ_ERR_UNSUPPORTED;
