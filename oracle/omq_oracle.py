@@ -75,6 +75,10 @@ notes of the repository):
      reciprocal of h; the clipping strengths entering it are the single-precision sigmoid
      of `sigmoid_fp32`.  Everything else stays float64.  ("emulate" mode; "exact"
      mode decides in float64.)
+ R20 softmax-output quantization (the ablation of Table A7, off by default): the causal softmax
+     output is quantized per query row with the MinMax Q_a (gamma = beta = 1, the floor of h
+     included) over the visible keys j <= t only; the masked entries stay 0.  Its decisions are
+     taken on P in single precision (R15) and its backward is the STE of R7.
 """
 from __future__ import annotations
 
@@ -92,7 +96,7 @@ __all__ = [
     "let_apply", "block_loss", "qlinear_step", "BlockCfg", "block_forward", "block_step",
     "rmsnorm", "rope", "silu", "FrozenTape", "use_tape", "block_fp_forward", "sigmoid_fp32",
     "THETA_NAMES_LWC", "THETA_NAMES_LET", "let_init", "pack_codes", "unpack_codes", "block_fold_pack",
-    "folded_forward", "adamw_step", "calibrate_blocks",
+    "folded_forward", "adamw_step", "calibrate_blocks", "softmax_quant",
 ]
 
 
@@ -582,6 +586,7 @@ class BlockCfg:
     rope_theta: float = 10000.0
     h_eps: float = 1e-5
     mode: str = "emulate"
+    pbits: int = 16       # softmax-output bits (R20); 16 = kept at full precision (the default)
 
     @staticmethod
     def from_shape(shape, **kw) -> "BlockCfg":
@@ -645,6 +650,27 @@ def _qa(X, cfg: BlockCfg):
     return quant_ste(X, 1.0, 1.0, cfg.abits, cfg.h_eps, _decide(cfg))
 
 
+def softmax_quant(P, nbits: int, eps: float = 1e-5, decide: str = "fp64"):
+    """Q_p (R20): the causal softmax output P [..., T, T] quantized per query row with the
+    MinMax quantizer of Eq. 2 (gamma = beta = 1) over the row's visible keys j <= t, as an
+    autograd graph with the STE of R7 (h not detached; max / min pass their gradient to the first
+    index).  The masked entries stay exactly 0 and take no part in the row's range.  nbits >= 16
+    returns P."""
+    if nbits >= 16:
+        return P
+    T = P.shape[-1]
+    causal = torch.ones(T, T, dtype=torch.bool).tril()
+    # the masked entries are filled with the row's diagonal probability: a value inside the row's
+    # range at an index after every visible key, so max, min and their first indices are unchanged
+    diag = torch.diagonal(P, dim1=-2, dim2=-1)[..., :, None]
+    Pf = torch.where(causal, P, diag.detach().expand_as(P))
+    return quant_ste(Pf, 1.0, 1.0, nbits, eps, decide).masked_fill(~causal, 0.0)
+
+
+def _qp(P, cfg: BlockCfg):
+    return softmax_quant(P, cfg.pbits, cfg.h_eps, _decide(cfg))
+
+
 def _dec32(W, s=None, r=None):
     """fp32 quantizer input of a scaled weight, formed as the kernels form it (R15)."""
     with torch.no_grad():
@@ -702,7 +728,7 @@ def block_forward(x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], c
     S = _mm(Qh, Kh, mode) / math.sqrt(hd)                                # R10
     causal = torch.ones(T, T, dtype=torch.bool).tril()
     S = S.masked_fill(~causal, float("-inf"))
-    P = torch.softmax(S, dim=-1)                                         # not quantized (R12)
+    P = _qp(torch.softmax(S, dim=-1), cfg)                              # unquantized by default (R12, R20)
     O = _mm(P, Vh.transpose(-1, -2), mode)                               # P V, [H, T, hd]
     O = O.transpose(0, 1).reshape(T, H * hd)
     oh = _qa(O, cfg)
@@ -917,7 +943,7 @@ def folded_forward(folded: Dict[str, torch.Tensor], x, cfg: BlockCfg) -> torch.T
         Vh = vh.reshape(T, Hkv, hd).transpose(0, 1).repeat_interleave(rep, 0)
         S = _mm(Qh, Kh, mode) / math.sqrt(hd)
         S = S.masked_fill(~torch.ones(T, T, dtype=torch.bool).tril(), float("-inf"))
-        O = _mm(torch.softmax(S, dim=-1), Vh.transpose(-1, -2), mode).transpose(0, 1).reshape(T, dq)
+        O = _mm(_qp(torch.softmax(S, dim=-1), cfg), Vh.transpose(-1, -2), mode).transpose(0, 1).reshape(T, dq)
         o = _mm(_qa(O, cfg), deq("o", d, dq), mode)
         if let:
             o = o + folded["b_o"]

@@ -399,6 +399,58 @@ def test_attention_matches_naive_loops():
     assert _rel(Ok, out) < 1e-13
 
 
+def _causal_probs(H, T, seed, spread=2.0):
+    g = torch.Generator().manual_seed(seed)
+    S = torch.randn(H, T, T, generator=g, dtype=F64) * spread
+    S = S.masked_fill(~torch.ones(T, T, dtype=torch.bool).tril(), float("-inf"))
+    return torch.softmax(S, -1)
+
+
+def test_softmax_quant_hand_example():
+    """R20 on a 3-key causal matrix, 2 bits (Q = 3).  Row 2, P = (0.6, 0.3, 0.1): h = 0.5/3 = 1/6,
+    z = -round(0.1 * 6) = -1, codes 3, 1, 0, values (code - z) h = 4/6, 2/6, 1/6.  Row 0 has one
+    key: range 0, h floored at eps, z = -round(1/eps), value (0 - z) eps = 1.  Row 1,
+    P = (0.7, 0.3): h = 0.4/3 = 2/15, z = -round(2.25) = -2, codes round(5.25) - 2 = 3 and
+    round(2.25) - 2 = 0, values 5 h = 2/3 and 2 h = 4/15."""
+    P = torch.tensor([[[1.0, 0.0, 0.0], [0.7, 0.3, 0.0], [0.6, 0.3, 0.1]]], dtype=F64)
+    got = O.softmax_quant(P, 2)
+    want = torch.tensor([[[1.0, 0.0, 0.0], [2 / 3, 4 / 15, 0.0], [4 / 6, 2 / 6, 1 / 6]]], dtype=F64)
+    assert torch.allclose(got, want, rtol=0, atol=1e-12)
+    assert float(got[0, 0, 1]) == 0.0 and float(got[0, 1, 2]) == 0.0
+
+
+@pytest.mark.parametrize("nbits,decide", [(8, "fp64"), (6, "fp32"), (4, "fp32"), (3, "fp64")])
+def test_softmax_quant_is_rowwise_minmax_over_visible_keys(nbits, decide):
+    """Each query row equals Eq. 2's MinMax quantizer applied to the row's visible slice
+    P[t, :t+1] alone (a per-row loop, no filling of the masked part); masked entries are 0."""
+    H, T = 2, 9
+    P = _causal_probs(H, T, 30 + nbits)
+    got = O.softmax_quant(P, nbits, decide=decide)
+    for hh in range(H):
+        for t in range(T):
+            st = O.quant_fwd(P[hh, t, :t + 1][None], 1.0, 1.0, nbits, decide=decide)
+            assert torch.allclose(got[hh, t, :t + 1], st["what"][0], rtol=0, atol=1e-15)
+            assert bool((got[hh, t, t + 1:] == 0).all())
+
+
+@pytest.mark.parametrize("nbits", [8, 4])
+def test_softmax_quant_ste_gradient_is_per_row_quant_bwd(nbits):
+    """Autograd through Q_p equals the explicit STE backward of Eq. 2 (pinned above against finite
+    differences) applied to each row's visible slice; masked entries get no gradient."""
+    H, T = 2, 8
+    P = _causal_probs(H, T, 40 + nbits, spread=1.0).requires_grad_(True)
+    g = torch.Generator().manual_seed(41)
+    gq = torch.randn(H, T, T, generator=g, dtype=F64)
+    (dP,) = torch.autograd.grad(O.softmax_quant(P, nbits), [P], gq)
+    Pd = P.detach()
+    for hh in range(H):
+        for t in range(T):
+            st = O.quant_fwd(Pd[hh, t, :t + 1][None], 1.0, 1.0, nbits)
+            ex = O.quant_bwd(st, gq[hh, t, :t + 1][None])
+            assert torch.allclose(dP[hh, t, :t + 1], ex["dw"][0], rtol=1e-12, atol=1e-14)
+            assert bool((dP[hh, t, t + 1:] == 0).all())
+
+
 def test_rope_properties():
     g = torch.Generator().manual_seed(13)
     T, H, hd = 9, 2, 8
