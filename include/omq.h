@@ -62,6 +62,8 @@ typedef struct {
   float   h_eps;       /* floor of the quantizer step h (1e-5); a floored h has zero gradient    */
   int32_t accumulate;  /* 1 = add into gradient outputs instead of overwriting them              */
   int32_t* dev_status; /* optional device int32: 0 = ok, else an omq_status set by a kernel      */
+  int32_t pbits;       /* softmax-output bits (the ablation beside Table A7): 2..8, or 0 / 16 = the
+                          softmax output is not quantized (the method's default)                  */
 } omq_qcfg;
 
 /* ------------------------------------------------------------------------------------------
@@ -279,6 +281,28 @@ omq_status omq_attention_bwd(omq_stream_t stream, int32_t T, int32_t n_heads, in
                              int64_t ldq, const void* K, const void* V, int64_t ldkv, const float* O, int64_t ldo,
                              const float* lse, const void* dO, int64_t lddo, float* D, float* dQ, int64_t ldg,
                              float* dK, float* dV, int64_t ldgkv, int32_t* dev_status);
+
+/* Softmax-output quantization variant of the attention (the ablation beside Table A7; off in the
+ * method's default configuration).  As omq_attention_fwd, except that the probabilities of every
+ * query row are fake-quantized with the MinMax quantizer of Eq. 2 (gamma = beta = 1, step floored at
+ * h_eps) over the row's visible keys j <= t before the P V product; masked entries stay 0.
+ *   pbits   2..8 (OMQ_ERR_UNSUPPORTED otherwise);
+ *   pq_rows [n_heads, T, 8] fp32 out, 16-byte aligned: per query row h, 1/h, z, min/h, floored
+ *           (0/1), the first key of the row's max and of its min (as exact floats), unused. */
+omq_status omq_attention_pq_fwd(omq_stream_t stream, int32_t T, int32_t n_heads, int32_t n_kv, const void* Q,
+                                int64_t ldq, const void* K, const void* V, int64_t ldkv, float* O, int64_t ldo,
+                                float* lse, int32_t pbits, float h_eps, float* pq_rows, int32_t* dev_status);
+
+/* Backward of omq_attention_pq_fwd: straight-through estimator of the quantizer (R7 of the oracle:
+ * the gradient passes inside the clamp range; h is not detached, the max and the min pass theirs to
+ * their first key), then the softmax backward.  pq_rows is the forward's; pq_stats [n_heads, T, 4]
+ * fp32 caller scratch, 16-byte aligned (per row sum_j P_j dP_j and the totals reaching the max and
+ * the min).  Other arguments as omq_attention_bwd, without D. */
+omq_status omq_attention_pq_bwd(omq_stream_t stream, int32_t T, int32_t n_heads, int32_t n_kv, const void* Q,
+                                int64_t ldq, const void* K, const void* V, int64_t ldkv, const float* lse,
+                                const void* dO, int64_t lddo, float* dQ, int64_t ldg, float* dK, float* dV,
+                                int64_t ldgkv, int32_t pbits, const float* pq_rows, float* pq_stats,
+                                int32_t* dev_status);
 
 /* LET initialisation (Sec. 4.1 "Training": the channel-wise scaling is initialised as in
  * SmoothQuant, the channel-wise shifting as in Outlier Suppression+).  Column statistics of the

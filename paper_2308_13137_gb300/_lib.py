@@ -30,7 +30,7 @@ class OmqError(RuntimeError):
 
 class omq_qcfg(Structure):
     _fields_ = [("wbits", c_int32), ("abits", c_int32), ("group", c_int32), ("let", c_int32),
-                ("h_eps", c_float), ("accumulate", c_int32), ("dev_status", c_void_p)]
+                ("h_eps", c_float), ("accumulate", c_int32), ("dev_status", c_void_p), ("pbits", c_int32)]
 
 
 class omq_qlinear_saved(Structure):
@@ -94,6 +94,9 @@ _SIGS = {
     "omq_attention_fwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P]),
     "omq_attention_bwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P, I64, P, P, I64, P, P, I64,
                                 P]),
+    "omq_attention_pq_fwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, I32, F32, P, P]),
+    "omq_attention_pq_bwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, P, I64, P, I64, P, P, I64, I32, P, P,
+                                   P]),
     "omq_block_pack_workspace_size": (SZ, [P, P]),
     "omq_block_fold_pack": (I32, [P, P, P, P, P, P, P, SZ]),
     "omq_let_stats_accumulate": (I32, [P, P, P, P, P, I32, P, SZ, P]),
@@ -162,8 +165,8 @@ def check(name: str, code: int):
         raise OmqError(name, code)
 
 
-def make_cfg(wbits=4, abits=16, group=0, let=0, h_eps=1e-5, accumulate=0, dev_status=None) -> omq_qcfg:
-    return omq_qcfg(wbits, abits, group, int(let), h_eps, accumulate, ptr(dev_status))
+def make_cfg(wbits=4, abits=16, group=0, let=0, h_eps=1e-5, accumulate=0, dev_status=None, pbits=16) -> omq_qcfg:
+    return omq_qcfg(wbits, abits, group, int(let), h_eps, accumulate, ptr(dev_status), pbits)
 
 
 # ------------------------------------------------------------------------------------------------
@@ -249,6 +252,20 @@ def omq_attention_bwd(T, n_heads, n_kv, Q, ldq, K, V, ldkv, O, ldo, lse, dO, ldd
     check("omq_attention_bwd", lib().omq_attention_bwd(
         stream_handle(stream), T, n_heads, n_kv, ptr(Q), ldq, ptr(K), ptr(V), ldkv, ptr(O), ldo, ptr(lse), ptr(dO),
         lddo, ptr(D), ptr(dQ), ldg, ptr(dK), ptr(dV), ldgkv, ptr(dev_status)))
+
+
+def omq_attention_pq_fwd(T, n_heads, n_kv, Q, ldq, K, V, ldkv, O, ldo, lse, pbits, h_eps, pq_rows,
+                         dev_status=None, stream=None):
+    check("omq_attention_pq_fwd", lib().omq_attention_pq_fwd(
+        stream_handle(stream), T, n_heads, n_kv, ptr(Q), ldq, ptr(K), ptr(V), ldkv, ptr(O), ldo, ptr(lse), pbits,
+        h_eps, ptr(pq_rows), ptr(dev_status)))
+
+
+def omq_attention_pq_bwd(T, n_heads, n_kv, Q, ldq, K, V, ldkv, lse, dO, lddo, dQ, ldg, dK, dV, ldgkv, pbits,
+                         pq_rows, pq_stats, dev_status=None, stream=None):
+    check("omq_attention_pq_bwd", lib().omq_attention_pq_bwd(
+        stream_handle(stream), T, n_heads, n_kv, ptr(Q), ldq, ptr(K), ptr(V), ldkv, ptr(lse), ptr(dO), lddo,
+        ptr(dQ), ldg, ptr(dK), ptr(dV), ldgkv, pbits, ptr(pq_rows), ptr(pq_stats), ptr(dev_status)))
 
 
 def omq_block_pack_workspace_size(shape, cfg) -> int:

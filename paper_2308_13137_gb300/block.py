@@ -22,7 +22,7 @@ class BlockState:
 
     def __init__(self, shape, weights: Dict[str, np.ndarray], theta: Dict[str, np.ndarray], device: str = "cuda",
                  wbits: Optional[int] = None, abits: Optional[int] = None, group: Optional[int] = None,
-                 let: Optional[int] = None):
+                 let: Optional[int] = None, pbits: int = 16):
         import torch
         self.torch = torch
         self.shape = shape
@@ -31,6 +31,7 @@ class BlockState:
         self.abits = shape.abits if abits is None else abits
         self.group = shape.group if group is None else group
         self.let = shape.let if let is None else let
+        self.pbits = pbits                 # softmax-output bits; 16 = not quantized (the default)
         bf = torch.bfloat16
 
         def dev_bf16(a):
@@ -83,7 +84,7 @@ class BlockState:
         self.c_theta = self._params(self.theta)
         self.c_grads = self._params(self.grads)
         self.status = torch.zeros(1, dtype=torch.int32, device=device)
-        self.cfg = _lib.make_cfg(self.wbits, self.abits, self.group, self.let, 1e-5, 0, self.status)
+        self.cfg = _lib.make_cfg(self.wbits, self.abits, self.group, self.let, 1e-5, 0, self.status, self.pbits)
         ws = _lib.omq_block_workspace_size(self.c_shape, self.cfg)
         if ws == 0:
             raise ValueError("block shape or configuration rejected by libomq")

@@ -39,7 +39,13 @@ struct FlashArgs {
   float* dQ; int64_t ldg;
   float* dK; float* dV; int64_t ldgkv;
   int32_t* status;
+  // softmax-output quantization (pbits 2..8; 0 or 16 = off): per query row, MinMax over the
+  // visible keys.  pqr [H, T, 8] quantizer state written by the forward, pqb [H, T, 4] backward
+  // row statistics (scratch); both 16-byte aligned.
+  int pbits; float eps;
+  float* pqr; float* pqb;
 };
+static inline bool flash_pq_on(int pbits) { return pbits >= 2 && pbits <= 8; }
 omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a);
 omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a);
 

@@ -58,6 +58,7 @@ struct BlockWS {
   bf16* a_h; float* rstd1; QState4 sa;
   float* Yqkv; bf16 *Qh, *Kh, *Vh; QState4 sqkv;
   float* lse;                       // [H, T] base-2 log-sum-exp of the attention rows
+  float* pqr;                       // [H, T, 8] softmax-output quantizer rows (pbits on only)
   float* O; bf16* O_h; QState4 so;
   float* h1; bf16* b_h; float* rstd2; QState4 sb;
   float* Ygu; bf16* m_h; QState4 sm;
@@ -72,6 +73,7 @@ struct BlockWS {
   float* dh1; bf16* dh1_b;
   float* dOh; bf16* dO_b;
   float* Drow;                      // [H, T] rowsum(dO * O)
+  float* pqb;                       // [H, T, 4] softmax-output quantizer backward rows (pbits on only)
   float* dQKV; float* dYqkv; bf16* dYqkv_b;
   float* da;
   float *dB_qkv, *dB_o, *dB_gu, *dr_qkv;
@@ -113,6 +115,7 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   w.Vh = c.take<bf16>(T * dkv);
   w.sqkv = take_qstate(c, 3 * T);
   w.lse = c.take<float>(H * T);
+  w.pqr = flash_pq_on(cfg.pbits) ? c.take<float>(H * T * 8) : nullptr;
   w.O = c.take<float>(T * dq);
   w.O_h = c.take<bf16>(T * dq);
   w.so = take_qstate(c, T);
@@ -138,6 +141,7 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   w.dOh = c.take<float>(T * dq);
   w.dO_b = c.take<bf16>(T * dq);
   w.Drow = c.take<float>(H * T);
+  w.pqb = flash_pq_on(cfg.pbits) ? c.take<float>(H * T * 4) : nullptr;
   w.dQKV = c.take<float>(T * nqkv);
   w.dYqkv = c.take<float>(T * nqkv);
   w.dYqkv_b = c.take<bf16>(T * nqkv);
@@ -383,6 +387,7 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   fa.T = (int)c.T; fa.H = (int)c.H; fa.Hkv = (int)c.Hkv; fa.hd = (int)c.hd;
   fa.Q = w.Qh; fa.K = w.Kh; fa.V = w.Vh; fa.ldq = c.dq; fa.ldkv = c.dkv;
   fa.O = w.O; fa.ldo = c.dq; fa.lse = w.lse; fa.status = status;
+  fa.pbits = cfg.pbits; fa.eps = cfg.h_eps; fa.pqr = w.pqr;
   OMQ_TRY(flash_fwd_launch(st, fa));
   ActFwdArgs ao{};
   ao.producer = AP_PLAIN; ao.X = w.O; ao.ldx = c.dq; ao.T = c.T; ao.C = c.dq; ao.Xq = w.O_h; ao.ldq = c.dq;
@@ -492,6 +497,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   fa.O = w.O; fa.ldo = c.dq; fa.lse = w.lse; fa.dO = w.dO_b; fa.lddo = c.dq; fa.D = w.Drow;
   fa.dQ = w.dQKV; fa.ldg = c.nqkv; fa.dK = w.dQKV + c.dq; fa.dV = w.dQKV + c.dq + c.dkv; fa.ldgkv = c.nqkv;
   fa.status = status;
+  fa.pbits = cfg.pbits; fa.eps = cfg.h_eps; fa.pqr = w.pqr; fa.pqb = w.pqb;
   OMQ_TRY(flash_bwd_launch(st, fa));
   QkvArgs qa{};
   qa.T = (int)c.T; qa.H = (int)c.H; qa.Hkv = (int)c.Hkv; qa.hd = (int)c.hd; qa.Y = w.Yqkv; qa.ldy = c.nqkv; qa.cs = w.cs;

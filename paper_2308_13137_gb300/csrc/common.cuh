@@ -26,6 +26,7 @@ static inline omq_status omq_check_cfg(const omq_qcfg* cfg) {
   if (!omq_bits_ok(cfg->wbits) || !omq_bits_ok(cfg->abits)) return OMQ_ERR_UNSUPPORTED;
   if (cfg->group < 0) return OMQ_ERR_SHAPE;
   if (!(cfg->h_eps > 0.f)) return OMQ_ERR_INVALID_ARG;
+  if (cfg->pbits != 0 && cfg->pbits != 16 && !(cfg->pbits >= 2 && cfg->pbits <= 8)) return OMQ_ERR_UNSUPPORTED;
   return OMQ_OK;
 }
 

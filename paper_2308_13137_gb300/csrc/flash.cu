@@ -89,7 +89,17 @@ struct FwdP {
   float* O; int64_t ldo;     // [T, H*128] fp32
   float* lse;                // [H, T]: m + log2(l) of the scaled base-2 logits
   int32_t* status;
+  float Q, eps;              // softmax-output quantizer: 2^bits - 1, floor of h
+  float* pqr;                // [H, T, 8] quantizer state per query row (PQ only)
 };
+
+// Quantizer state of one query row of the softmax output (MinMax over the visible keys, Eq. 2
+// with gamma = beta = 1): h, 1/h, z, u = m/h, floored (0/1), first index of the max and of the
+// min (as exact floats), unused.
+enum { PQ_H = 0, PQ_RH, PQ_Z, PQ_U, PQ_FL, PQ_IMAX, PQ_IMIN, PQ_N = 8 };
+// Backward statistics of one query row (PQ): D = sum_j P_j dP_j with dP the gradient reaching P
+// through the quantizer, and the totals that reach the row's max and min (R7).
+enum { PG_D = 0, PG_DM, PG_DMIN, PG_N = 4 };
 
 constexpr int F_TILE = 128 * ROW_BYTES * 2;           // 32 KB: [128 x 128] bf16
 constexpr int F_ATOM = 128 * ROW_BYTES;               // 16 KB
@@ -101,6 +111,9 @@ constexpr int F_CTL = F_P + F_TILE;
 constexpr int F_SMEM = F_CTL + 256 + 1024;            // + barriers + alignment slack
 static_assert(F_SMEM <= 227 * 1024, "forward shared memory");
 
+// PQ: the probabilities are quantized per query row before the P V product (softmax-output
+// quantization); the statistics pass also finds the row's max and min score with first indices.
+template <bool PQ>
 __global__ void __launch_bounds__(FA_THREADS, 1)
     flash_fwd_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                      const __grid_constant__ CUtensorMap tmV, const FwdP p) {
@@ -200,8 +213,10 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     const int row = qb * 128 + r;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     uint8_t* ptile = smem + F_P;
-    float* stat = reinterpret_cast<float*>(smem + F_ST);   // [2 halves][m | l][128 rows]
+    float* stat = reinterpret_cast<float*>(smem + F_ST);   // [2 halves][m | l (| PQ extremes)][128 rows]
     float m = -INFINITY, l = 0.f;
+    float smax = -INFINITY, smin = INFINITY;        // PQ: raw extreme scores and their first keys
+    int imx = 0x7fffffff, imn = 0x7fffffff;
     bool ok = true;
     for (int j = 0; j < nkb; ++j) {                   // pass 1: running max and rescaled sum
       if (!(ok = waitw(&s_full[j & 1], (j >> 1) & 1, p.status, abort_flag))) break;
@@ -212,6 +227,15 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       for (int c = 2 * half; c < 2 * half + 2; ++c) {
         float v[32];
         tmem_ld32(sb + 32 * c, v);
+        if constexpr (PQ) {                           // this thread's keys arrive in increasing order
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            if (diag && 32 * c + i > r) continue;
+            const int key = j * 128 + 32 * c + i;
+            if (v[i] > smax) { smax = v[i]; imx = key; }
+            if (v[i] < smin) { smin = v[i]; imn = key; }
+          }
+        }
         if (diag) {
 #pragma unroll
           for (int i = 0; i < 32; ++i) if (32 * c + i > r) v[i] = -INFINITY;
@@ -237,14 +261,35 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       if (lane == 0) mbar_arrive(p_full);
     }
     // combine the two halves of every row (each compute thread reaches this barrier exactly once)
-    stat[(half * 2 + 0) * 128 + r] = m;
-    stat[(half * 2 + 1) * 128 + r] = l;
+    constexpr int NS = PQ ? 6 : 2;                  // statistics per row and half
+    stat[(half * NS + 0) * 128 + r] = m;
+    stat[(half * NS + 1) * 128 + r] = l;
+    if constexpr (PQ) {
+      stat[(half * NS + 2) * 128 + r] = smax;
+      stat[(half * NS + 3) * 128 + r] = smin;
+      stat[(half * NS + 4) * 128 + r] = __int_as_float(imx);
+      stat[(half * NS + 5) * 128 + r] = __int_as_float(imn);
+    }
     asm volatile("bar.sync 1, 256;" ::: "memory");
-    const float mo = stat[((1 - half) * 2 + 0) * 128 + r], lo = stat[((1 - half) * 2 + 1) * 128 + r];
+    const int oh = 1 - half;
+    const float mo = stat[(oh * NS + 0) * 128 + r], lo = stat[(oh * NS + 1) * 128 + r];
+    if constexpr (PQ) {                               // extremes of both halves, first index on ties
+      const float xo = stat[(oh * NS + 2) * 128 + r], no = stat[(oh * NS + 3) * 128 + r];
+      const int ixo = __float_as_int(stat[(oh * NS + 4) * 128 + r]), ino = __float_as_int(stat[(oh * NS + 5) * 128 + r]);
+      if (xo > smax || (xo == smax && ixo < imx)) { smax = xo; imx = ixo; }
+      if (no < smin || (no == smin && ino < imn)) { smin = no; imn = ino; }
+    }
     asm volatile("bar.sync 1, 256;" ::: "memory");   // statistics read before P overwrites them
     const float mt = fmaxf(m, mo);
     const float lt = (m == -INFINITY ? 0.f : l * ex2(m - mt)) + (mo == -INFINITY ? 0.f : lo * ex2(mo - mt));
     const float inv_l = 1.f / lt;
+    // PQ: the row's quantizer from the probabilities of its max and min score (the map from a score
+    // to its probability below is the one pass 2 applies to every key)
+    QState qs{};
+    if constexpr (PQ) {
+      const float Mp = ex2(fmaf(smax, p.c, -mt)) * inv_l, mp = ex2(fmaf(smin, p.c, -mt)) * inv_l;
+      qs = omq_qstate(Mp, mp, 1.f, 1.f, p.Q, p.eps);
+    }
     for (int j = 0; ok && j < nkb; ++j) {             // pass 2: probabilities, O += P V
       const int it = nkb + j;
       if (!(ok = waitw(&s_full[it & 1], (it >> 1) & 1, p.status, abort_flag))) break;
@@ -258,6 +303,10 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
         tmem_ld32(sb + 32 * c, v[cc]);
 #pragma unroll
         for (int i = 0; i < 32; ++i) v[cc][i] = ex2(fmaf(v[cc][i], p.c, -mt)) * inv_l;
+        if constexpr (PQ) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[cc][i] = omq_fakequant(v[cc][i], qs, p.Q, nullptr);
+        }
         if (diag) {
 #pragma unroll
           for (int i = 0; i < 32; ++i) if (32 * c + i > r) v[cc][i] = 0.f;
@@ -287,6 +336,13 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
         }
       }
       if (row < p.T && half == 0) p.lse[(int64_t)h * p.T + row] = mt + log2f(lt);
+      if constexpr (PQ) {
+        if (row < p.T && half == 0) {
+          float4* d = reinterpret_cast<float4*>(p.pqr + ((int64_t)h * p.T + row) * PQ_N);
+          d[0] = make_float4(qs.h, qs.rh, qs.z, qs.u);
+          d[1] = make_float4(qs.floored ? 1.f : 0.f, (float)imx, (float)imn, 0.f);
+        }
+      }
     }
   }
   tc_fence_before();
@@ -325,26 +381,41 @@ struct BwdP {
   float* dQ; int64_t ldq;    // [T, H*128]
   float* dK; float* dV; int64_t ldkv;    // [T, Hkv*128]
   int32_t* status;
+  float Q;                   // PQ: 2^bits - 1 of the softmax-output quantizer
+  const float* pqr;          // PQ: [H, T, PQ_N] forward quantizer state
+  float* pqb;                // PQ: [H, T, PG_N] backward row statistics
 };
 
 constexpr int B_QATOM = 64 * ROW_BYTES;               // 8 KB: 64-row atom
 constexpr int B_QTILE = 2 * B_QATOM;                  // [64 x 128] bf16
-constexpr int B_NQD = 3;                              // slots of the Q / dO / lse / D ring
-constexpr int B_K = 0, B_V = F_TILE, B_Q = 2 * F_TILE, B_DO = B_Q + B_NQD * B_QTILE;
-constexpr int B_PT = B_DO + B_NQD * B_QTILE;          // P^T [128 keys x 64 queries]: 16 KB, two buffers
-constexpr int B_DST = B_PT + 2 * F_ATOM;              // dS^T, same shape, two buffers
-constexpr int B_LD = B_DST + 2 * F_ATOM;              // [slot][lse 64 | D 64] fp32
-constexpr int B_CTL = B_LD + B_NQD * 512;
-constexpr int B_SMEM = B_CTL + 256 + 1024;            // + barriers + alignment slack
-static_assert(sizeof(Ctl) <= 256 && B_SMEM <= 227 * 1024, "dKV shared memory");
 
+// dKV shared-memory layout.  Ring slots hold Q, dO and the row data of a 64-query block: lse and
+// D (plain), or lse, the quantizer state and the backward row statistics (PQ, two slots).
+template <bool PQ>
+struct BL {
+  static constexpr int NQD = PQ ? 2 : 3;              // slots of the Q / dO / row-data ring
+  static constexpr int RD = PQ ? 64 * 4 * (1 + PQ_N + PG_N) : 512;   // row-data bytes per slot
+  static constexpr int K = 0, V = F_TILE, Qo = 2 * F_TILE, DO = Qo + NQD * B_QTILE;
+  static constexpr int PT = DO + NQD * B_QTILE;       // P^T [128 keys x 64 queries]: 16 KB, two buffers
+  static constexpr int DST = PT + 2 * F_ATOM;         // dS^T, same shape, two buffers
+  static constexpr int LD = DST + 2 * F_ATOM;         // [slot][row data]
+  static constexpr int CTL = LD + NQD * RD;
+  static constexpr int SMEM = CTL + 256 + 1024;       // + barriers + alignment slack
+};
+static_assert(sizeof(Ctl) <= 256 && BL<false>::SMEM <= 227 * 1024 && BL<true>::SMEM <= 227 * 1024,
+              "dKV shared memory");
+
+template <bool PQ>
 __global__ void __launch_bounds__(FA_THREADS, 1)
     flash_bwd_dkv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                          const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
                          const BwdP p) {
+  using L = BL<PQ>;
+  constexpr int B_NQD = L::NQD;
+  constexpr int B_K = L::K, B_V = L::V, B_Q = L::Qo, B_DO = L::DO, B_PT = L::PT, B_DST = L::DST, B_LD = L::LD;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  Ctl* ctl = reinterpret_cast<Ctl*>(smem + B_CTL);
+  Ctl* ctl = reinterpret_cast<Ctl*>(smem + L::CTL);
   uint64_t* kv_full = &ctl->bar[0];
   uint64_t* qd_full = &ctl->bar[1];      // [B_NQD]
   uint64_t* qd_empty = &ctl->bar[1 + B_NQD];   // [B_NQD]
@@ -386,12 +457,20 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       const int h = g * p.rep + it / niq, qi = i0 + it % niq;
       if (!waitb(&qd_empty[s], ((it / B_NQD) & 1) ^ 1, p.status, abort_flag)) break;
       const uint32_t nb = (uint32_t)min(64, p.T - qi * 64) * 4;     // lse / D bytes inside [0, T)
-      mbar_expect_tx(&qd_full[s], 2 * B_QTILE + 2 * nb);
+      const int64_t r0 = (int64_t)h * p.T + qi * 64;
+      float* ld = reinterpret_cast<float*>(smem + B_LD + s * L::RD);  // s: the ring slot
+      if constexpr (PQ) {
+        mbar_expect_tx(&qd_full[s], 2 * B_QTILE + (1 + PQ_N + PG_N) * nb);
+        bulk_g2s(ld, p.lse + r0, nb, &qd_full[s]);
+        bulk_g2s(ld + 64, p.pqr + r0 * PQ_N, PQ_N * nb, &qd_full[s]);
+        bulk_g2s(ld + 64 * (1 + PQ_N), p.pqb + r0 * PG_N, PG_N * nb, &qd_full[s]);
+      } else {
+        mbar_expect_tx(&qd_full[s], 2 * B_QTILE + 2 * nb);
+        bulk_g2s(ld, p.lse + r0, nb, &qd_full[s]);
+        bulk_g2s(ld + 64, p.D + r0, nb, &qd_full[s]);
+      }
       load_tile(&tmQ, &qd_full[s], smem + B_Q + s * B_QTILE, h * HD, qi * 64, B_QATOM);
       load_tile(&tmdO, &qd_full[s], smem + B_DO + s * B_QTILE, h * HD, qi * 64, B_QATOM);
-      float* ld = reinterpret_cast<float*>(smem + B_LD + s * 512);    // s: the ring slot
-      bulk_g2s(ld, p.lse + (int64_t)h * p.T + qi * 64, nb, &qd_full[s]);
-      bulk_g2s(ld + 64, p.D + (int64_t)h * p.T + qi * 64, nb, &qd_full[s]);
     }
   } else if (warp == 1 && lane == 0) {
     constexpr uint32_t ID_S = idesc_bf16(128, 64, 0, 0), ID_G = idesc_bf16(128, 128, 0, 1);
@@ -440,8 +519,10 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     for (int it = 0; it < nit; ++it) {
       const int s = it & 1;
       const int qi = i0 + it % niq;
-      const float* L = reinterpret_cast<const float*>(smem + B_LD + (it % B_NQD) * 512);
-      const float* Dq = L + 64;
+      const float* Lr = reinterpret_cast<const float*>(smem + B_LD + (it % B_NQD) * L::RD);
+      const float* Dq = Lr + 64;
+      const float* R8 = Lr + 64;                      // PQ: quantizer state, then row statistics
+      const float* G4 = Lr + 64 * (1 + PQ_N);
       // queries below the key block's last key, or past T, need the mask; the rest see every key
       const bool need_mask = qi * 64 < kb * 128 + 127 || qi * 64 + 64 > p.T;
       if (!(ok = waitw(&s_full[s], (it >> 1) & 1, p.status, abort_flag))) break;
@@ -451,11 +532,33 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
         float sv[32], dp[32];
         tmem_ld32(tmem + 64 * s + lane_off + 32 * c, sv);
         tmem_ld32(tmem + 128 + 64 * s + lane_off + 32 * c, dp);
+        if constexpr (PQ) {
+          // dV takes the quantized probabilities; dS = P (dP - D) with dP the gradient that reaches P
+          // through the quantizer: straight through inside the clamp range, plus the totals of the
+          // row's max and min at their first keys
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float pv = ex2(fmaf(sv[i], p.c, -L[32 * c + i]));
-          sv[i] = pv;
-          dp[i] = pv * (dp[i] - Dq[32 * c + i]) * p.scale;
+          for (int i = 0; i < 32; ++i) {
+            const int qc = 32 * c + i;
+            const float* st = R8 + qc * PQ_N;
+            const float* gs = G4 + qc * PG_N;
+            const float pv = ex2(fmaf(sv[i], p.c, -Lr[qc]));
+            const float rr = rintf(__fmul_rn(pv, st[PQ_RH]));
+            const float z = st[PQ_Z];
+            const float cd = rr + z;
+            const bool inr = cd >= 0.f && cd <= p.Q;
+            float g = inr ? dp[i] : 0.f;
+            if ((float)key == st[PQ_IMAX]) g += gs[PG_DM];
+            if ((float)key == st[PQ_IMIN]) g += gs[PG_DMIN];
+            sv[i] = __fmul_rn(fminf(fmaxf(rr, -z), p.Q - z), st[PQ_H]);
+            dp[i] = pv * (g - gs[PG_D]) * p.scale;
+          }
+        } else {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float pv = ex2(fmaf(sv[i], p.c, -Lr[32 * c + i]));
+            sv[i] = pv;
+            dp[i] = pv * (dp[i] - Dq[32 * c + i]) * p.scale;
+          }
         }
         if (need_mask) {
 #pragma unroll
@@ -521,6 +624,10 @@ constexpr int Q_CTL = Q_DS + 2 * F_ATOM;
 constexpr int Q_SMEM = Q_CTL + 256 + 1024;            // + barriers + alignment slack
 static_assert(Q_SMEM <= 227 * 1024, "dQ shared memory");
 
+// MODE 0: dQ.  PQ (softmax-output quantization): MODE 1 is a statistics pass over the same products
+// (no dQ) that writes each query row's backward statistics (PG_*); MODE 2 is dQ with dS formed as
+// in the PQ dKV kernel.
+template <int MODE>
 __global__ void __launch_bounds__(FA_THREADS, 1)
     flash_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
@@ -595,10 +702,12 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       if (j + 1 < nkb && !issue_s(j + 1)) break;
       if (!waitb(p_full, j & 1, p.status, abort_flag)) break;
       tc_fence_after();
+      if constexpr (MODE != 1) {
 #pragma unroll
-      for (int kk = 0; kk < 4; ++kk)               // K = 64 keys
-        umma_bf16(tmem + 256, desc_k(sds + b * F_ATOM, kk, F_ATOM), desc_mn(sk + r * B_QTILE, kk, B_QATOM), ID_G,
-                  (j | kk) != 0);
+        for (int kk = 0; kk < 4; ++kk)             // K = 64 keys
+          umma_bf16(tmem + 256, desc_k(sds + b * F_ATOM, kk, F_ATOM), desc_mn(sk + r * B_QTILE, kk, B_QATOM), ID_G,
+                    (j | kk) != 0);
+      }
       umma_commit(&g_done[b]);
       umma_commit(&kv_empty[r]);
     }
@@ -609,7 +718,23 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     const bool row_ok = row < p.T;
     const float Lr = row_ok ? p.lse[(int64_t)h * p.T + row] : 0.f;
-    const float Dr = row_ok ? p.D[(int64_t)h * p.T + row] : 0.f;
+    float Dr = (MODE == 0 && row_ok) ? p.D[(int64_t)h * p.T + row] : 0.f;
+    // PQ: the row's quantizer state (and, for MODE 2, its backward statistics)
+    float q_h = 0.f, q_rh = 0.f, q_z = 0.f, q_ru = 0.f, q_fl = 1.f, q_imax = -1.f, q_imin = -1.f;
+    float g_dM = 0.f, g_dm = 0.f;
+    if (MODE != 0 && row_ok) {
+      const float4* st = reinterpret_cast<const float4*>(p.pqr + ((int64_t)h * p.T + row) * PQ_N);
+      const float4 a0 = st[0], a1 = st[1];
+      q_h = a0.x; q_rh = a0.y; q_z = a0.z; q_ru = rintf(a0.w) - a0.w; q_fl = a1.x; q_imax = a1.y; q_imin = a1.z;
+      if (MODE == 2) {
+        const float4 gs = *reinterpret_cast<const float4*>(p.pqb + ((int64_t)h * p.T + row) * PG_N);
+        Dr = gs.x; g_dM = gs.y; g_dm = gs.z;
+      }
+    }
+    (void)q_h;
+    // MODE 1 sums over the row's keys: sum of P dP inside the clamp range, the h-path total G_h,
+    // the clamped total, and P at the row's max / min keys
+    float a_E = 0.f, a_Gh = 0.f, a_Gc = 0.f, a_PM = 0.f, a_Pm = 0.f;
     bool ok = true;
     for (int j = 0; j < nkb; ++j) {
       const int s = j & 1;
@@ -625,14 +750,43 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
         float sv[32], dp[32];
         tmem_ld32(tmem + 64 * s + lane_off + 32 * c, sv);
         tmem_ld32(tmem + 128 + 64 * s + lane_off + 32 * c, dp);
+        if constexpr (MODE == 0) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) dp[i] = ex2(fmaf(sv[i], p.c, -Lr)) * (dp[i] - Dr) * p.scale;
-        if (need_mask) {
+          for (int i = 0; i < 32; ++i) dp[i] = ex2(fmaf(sv[i], p.c, -Lr)) * (dp[i] - Dr) * p.scale;
+        } else {
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (j * 64 + 32 * c + i > row || !row_ok) dp[i] = 0.f;
+          for (int i = 0; i < 32; ++i) {
+            const int key = j * 64 + 32 * c + i;
+            const bool vis = !need_mask || (key <= row && row_ok);
+            const float pv = ex2(fmaf(sv[i], p.c, -Lr));
+            const float x = __fmul_rn(pv, q_rh);
+            const float rr = rintf(x);
+            const float cd = rr + q_z;
+            const bool inr = cd >= 0.f && cd <= p.Q;
+            if constexpr (MODE == 1) {
+              if (vis) {
+                const float dh = inr ? rr - x : (cd < 0.f ? q_ru : p.Q + q_ru);
+                if (inr) a_E = fmaf(pv, dp[i], a_E); else a_Gc += dp[i];
+                a_Gh = fmaf(dp[i], dh, a_Gh);
+                if ((float)key == q_imax) a_PM = pv;
+                if ((float)key == q_imin) a_Pm = pv;
+              }
+            } else {
+              float g = inr ? dp[i] : 0.f;
+              if ((float)key == q_imax) g += g_dM;
+              if ((float)key == q_imin) g += g_dm;
+              dp[i] = pv * (g - Dr) * p.scale;
+            }
+          }
         }
-        st_row32(dst, F_ATOM, r, 32 * c, dp);
+        if constexpr (MODE != 1) {
+          if (need_mask) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (j * 64 + 32 * c + i > row || !row_ok) dp[i] = 0.f;
+          }
+          st_row32(dst, F_ATOM, r, 32 * c, dp);
+        }
       }
       fence_async_smem();
       tc_fence_before();
@@ -643,7 +797,26 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       const int last = ((nkb - 1 - b) & ~1) + b;
       ok = waitw(&g_done[b], (last >> 1) & 1, p.status, abort_flag);
     }
-    if (ok) {
+    if constexpr (MODE == 1) {
+      // combine the two halves of every row through the (unused) dS buffers; every compute thread
+      // reaches this barrier exactly once
+      float* x5 = reinterpret_cast<float*>(smem + Q_DS);              // [half][5][128]
+      x5[(half * 5 + 0) * 128 + r] = a_E;
+      x5[(half * 5 + 1) * 128 + r] = a_Gh;
+      x5[(half * 5 + 2) * 128 + r] = a_Gc;
+      x5[(half * 5 + 3) * 128 + r] = a_PM;
+      x5[(half * 5 + 4) * 128 + r] = a_Pm;
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+      if (ok && half == 0 && row_ok) {
+        float t[5];
+#pragma unroll
+        for (int k = 0; k < 5; ++k) t[k] = x5[k * 128 + r] + x5[(5 + k) * 128 + r];   // one half holds each P
+        const float Gh = q_fl != 0.f ? 0.f : t[1];    // a floored step has no gradient
+        const float dM = Gh / p.Q, dm = t[2] - Gh / p.Q;
+        *reinterpret_cast<float4*>(p.pqb + ((int64_t)h * p.T + row) * PG_N) =
+            make_float4(t[0] + t[3] * dM + t[4] * dm, dM, dm, 0.f);
+      }
+    } else if (ok) {
       tc_fence_after();
 #pragma unroll 1
       for (int c = 2 * half; c < 2 * half + 2; ++c) {
@@ -684,27 +857,36 @@ omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
   ok = ok && omq_make_map_bf16(&tk64, a.K, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
   ok = ok && omq_make_map_bf16(&tv64, a.V, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
   if (!ok) return OMQ_ERR_UNSUPPORTED;
+  const bool pq = flash_pq_on(a.pbits);
+  OMQ_REQUIRE(!pq || (a.pqr && omq_aligned16(a.pqr)), OMQ_ERR_INVALID_ARG);
   static bool attr = false;
-  if (!attr) { if (!set_smem((const void*)flash_fwd_kernel, F_SMEM)) return OMQ_ERR_CUDA; attr = true; }
+  if (!attr) {
+    if (!set_smem((const void*)flash_fwd_kernel<false>, F_SMEM) || !set_smem((const void*)flash_fwd_kernel<true>, F_SMEM))
+      return OMQ_ERR_CUDA;
+    attr = true;
+  }
   FwdP p;
   p.T = a.T; p.H = a.H; p.rep = a.H / a.Hkv;
   p.c = (float)(1.4426950408889634 / sqrt((double)HD));
   p.O = a.O; p.ldo = a.ldo; p.lse = a.lse; p.status = a.status;
+  p.Q = pq ? (float)((1 << a.pbits) - 1) : 0.f; p.eps = a.eps; p.pqr = a.pqr;
   dim3 grid((unsigned)a.H, (unsigned)((a.T + 127) / 128));
-  flash_fwd_kernel<<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, p);
+  if (pq) flash_fwd_kernel<true><<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, p);
+  else flash_fwd_kernel<false><<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
   OMQ_REQUIRE(a.T > 0 && a.H > 0 && a.Hkv > 0 && a.H % a.Hkv == 0 && a.hd == HD, OMQ_ERR_SHAPE);
-  OMQ_REQUIRE(a.Q && a.K && a.V && a.O && a.lse && a.dO && a.D && a.dQ && a.dK && a.dV, OMQ_ERR_INVALID_ARG);
-  OMQ_REQUIRE(a.ldq % 8 == 0 && a.ldkv % 8 == 0 && a.ldo % 4 == 0 && a.lddo % 8 == 0 && a.ldg % 4 == 0 &&
+  const bool pq = flash_pq_on(a.pbits);             // O and D are not used then
+  OMQ_REQUIRE(a.Q && a.K && a.V && a.lse && a.dO && a.dQ && a.dK && a.dV && (pq || (a.O && a.D)), OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(a.ldq % 8 == 0 && a.ldkv % 8 == 0 && (pq || a.ldo % 4 == 0) && a.lddo % 8 == 0 && a.ldg % 4 == 0 &&
                   a.ldgkv % 4 == 0,
               OMQ_ERR_ALIGN);
   OMQ_REQUIRE(omq_aligned16(a.dO) && omq_aligned16(a.dQ) && omq_aligned16(a.dK) && omq_aligned16(a.dV), OMQ_ERR_ALIGN);
-  // lse and D rows are fetched by 16-byte bulk copies
-  OMQ_REQUIRE(a.T % 4 == 0 && omq_aligned16(a.lse) && omq_aligned16(a.D), OMQ_ERR_ALIGN);
+  // lse, D and the PQ row data are fetched by 16-byte bulk copies
+  OMQ_REQUIRE(a.T % 4 == 0 && omq_aligned16(a.lse) && (pq || omq_aligned16(a.D)), OMQ_ERR_ALIGN);
   CUtensorMap tq64, tdo64, tk, tv, tq, tdo;
   bool ok = omq_make_map_bf16(&tq64, a.Q, (int64_t)a.H * HD, a.T, 1, a.ldq, 0, 64, 64);
   ok = ok && omq_make_map_bf16(&tdo64, a.dO, (int64_t)a.H * HD, a.T, 1, a.lddo, 0, 64, 64);
@@ -716,15 +898,16 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
   ok = ok && omq_make_map_bf16(&tk64, a.K, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
   ok = ok && omq_make_map_bf16(&tv64, a.V, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
   if (!ok) return OMQ_ERR_UNSUPPORTED;
+  OMQ_REQUIRE(!pq || (a.pqr && a.pqb && omq_aligned16(a.pqr) && omq_aligned16(a.pqb)), OMQ_ERR_INVALID_ARG);
   static bool attr = false;
   if (!attr) {
-    if (!set_smem((const void*)flash_bwd_dkv_kernel, B_SMEM) || !set_smem((const void*)flash_bwd_dq_kernel, Q_SMEM))
+    if (!set_smem((const void*)flash_bwd_dkv_kernel<false>, BL<false>::SMEM) ||
+        !set_smem((const void*)flash_bwd_dkv_kernel<true>, BL<true>::SMEM) ||
+        !set_smem((const void*)flash_bwd_dq_kernel<0>, Q_SMEM) || !set_smem((const void*)flash_bwd_dq_kernel<1>, Q_SMEM) ||
+        !set_smem((const void*)flash_bwd_dq_kernel<2>, Q_SMEM))
       return OMQ_ERR_CUDA;
     attr = true;
   }
-  const int64_t rows = (int64_t)a.T * a.H;
-  attn_rowdot_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(a.T, a.H, a.dO, a.lddo, a.O, a.ldo, a.D);
-  OMQ_LAUNCH_CHECK();
   BwdP p;
   p.T = a.T; p.H = a.H; p.rep = a.H / a.Hkv;
   p.c = (float)(1.4426950408889634 / sqrt((double)HD));
@@ -732,11 +915,25 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
   p.lse = a.lse; p.D = a.D;
   p.dQ = a.dQ; p.ldq = a.ldg; p.dK = a.dK; p.dV = a.dV; p.ldkv = a.ldgkv;
   p.status = a.status;
+  p.Q = pq ? (float)((1 << a.pbits) - 1) : 0.f; p.pqr = a.pqr; p.pqb = a.pqb;
   dim3 g1((unsigned)a.Hkv, (unsigned)((a.T + 127) / 128));
-  flash_bwd_dkv_kernel<<<g1, FA_THREADS, B_SMEM, st>>>(tq64, tk, tv, tdo64, p);
-  OMQ_LAUNCH_CHECK();
   dim3 g2((unsigned)a.H, (unsigned)((a.T + 127) / 128));
-  flash_bwd_dq_kernel<<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, p);
+  if (pq) {
+    // row statistics first (they replace D = rowsum(dO * O), which no longer is sum_j P_j dP_j)
+    flash_bwd_dq_kernel<1><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, p);
+    OMQ_LAUNCH_CHECK();
+    flash_bwd_dkv_kernel<true><<<g1, FA_THREADS, BL<true>::SMEM, st>>>(tq64, tk, tv, tdo64, p);
+    OMQ_LAUNCH_CHECK();
+    flash_bwd_dq_kernel<2><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, p);
+    OMQ_LAUNCH_CHECK();
+    return OMQ_OK;
+  }
+  const int64_t rows = (int64_t)a.T * a.H;
+  attn_rowdot_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(a.T, a.H, a.dO, a.lddo, a.O, a.ldo, a.D);
+  OMQ_LAUNCH_CHECK();
+  flash_bwd_dkv_kernel<false><<<g1, FA_THREADS, BL<false>::SMEM, st>>>(tq64, tk, tv, tdo64, p);
+  OMQ_LAUNCH_CHECK();
+  flash_bwd_dq_kernel<0><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -762,5 +959,35 @@ extern "C" omq_status omq_attention_bwd(omq_stream_t stream, int32_t T, int32_t 
   a.ldq = ldq; a.ldkv = ldkv; a.O = const_cast<float*>(O); a.ldo = ldo; a.lse = const_cast<float*>(lse);
   a.dO = (const __nv_bfloat16*)dO; a.lddo = lddo; a.D = D;
   a.dQ = dQ; a.ldg = ldg; a.dK = dK; a.dV = dV; a.ldgkv = ldgkv; a.status = dev_status;
+  return flash_bwd_launch((cudaStream_t)stream, a);
+}
+
+extern "C" omq_status omq_attention_pq_fwd(omq_stream_t stream, int32_t T, int32_t n_heads, int32_t n_kv,
+                                           const void* Q, int64_t ldq, const void* K, const void* V, int64_t ldkv,
+                                           float* O, int64_t ldo, float* lse, int32_t pbits, float h_eps,
+                                           float* pq_rows, int32_t* dev_status) {
+  OMQ_REQUIRE(flash_pq_on(pbits), OMQ_ERR_UNSUPPORTED);
+  OMQ_REQUIRE(h_eps > 0.f, OMQ_ERR_INVALID_ARG);
+  FlashArgs a{};
+  a.T = T; a.H = n_heads; a.Hkv = n_kv; a.hd = HD;
+  a.Q = (const __nv_bfloat16*)Q; a.K = (const __nv_bfloat16*)K; a.V = (const __nv_bfloat16*)V;
+  a.ldq = ldq; a.ldkv = ldkv; a.O = O; a.ldo = ldo; a.lse = lse; a.status = dev_status;
+  a.pbits = pbits; a.eps = h_eps; a.pqr = pq_rows;
+  return flash_fwd_launch((cudaStream_t)stream, a);
+}
+
+extern "C" omq_status omq_attention_pq_bwd(omq_stream_t stream, int32_t T, int32_t n_heads, int32_t n_kv,
+                                           const void* Q, int64_t ldq, const void* K, const void* V, int64_t ldkv,
+                                           const float* lse, const void* dO, int64_t lddo, float* dQ, int64_t ldg,
+                                           float* dK, float* dV, int64_t ldgkv, int32_t pbits, const float* pq_rows,
+                                           float* pq_stats, int32_t* dev_status) {
+  OMQ_REQUIRE(flash_pq_on(pbits), OMQ_ERR_UNSUPPORTED);
+  FlashArgs a{};
+  a.T = T; a.H = n_heads; a.Hkv = n_kv; a.hd = HD;
+  a.Q = (const __nv_bfloat16*)Q; a.K = (const __nv_bfloat16*)K; a.V = (const __nv_bfloat16*)V;
+  a.ldq = ldq; a.ldkv = ldkv; a.lse = const_cast<float*>(lse);
+  a.dO = (const __nv_bfloat16*)dO; a.lddo = lddo;
+  a.dQ = dQ; a.ldg = ldg; a.dK = dK; a.dV = dV; a.ldgkv = ldgkv; a.status = dev_status;
+  a.pbits = pbits; a.pqr = const_cast<float*>(pq_rows); a.pqb = pq_stats;
   return flash_bwd_launch((cudaStream_t)stream, a);
 }

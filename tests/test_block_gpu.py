@@ -18,14 +18,16 @@ def _rel(a, b):
     return float((a - b).norm() / b.norm().clamp_min(1e-300))
 
 
-def _run(shape, perturb=True, seed=0):
+def _run(shape, perturb=True, seed=0, pbits=16, run_cuda=True):
     W = I.make_block_weights(shape, seed=seed + 1)
     x = I.make_block_input(shape, sample=seed, weight_seed=seed + 1)
     th = I.make_block_theta(shape, W, x, seed=seed + 2, perturb=perturb)
-    cfg = O.BlockCfg.from_shape(shape)
-    yfp = O.block_fp_forward(x, W, cfg).float()
+    cfg = O.BlockCfg.from_shape(shape, pbits=pbits)
+    yfp = O.block_fp_forward(x, W, O.BlockCfg.from_shape(shape)).float()
     ref = O.block_step(x, yfp, W, th, cfg)
-    st = BlockState(shape, W, th)
+    if not run_cuda:
+        return ref, None
+    st = BlockState(shape, W, th, pbits=pbits)
     xd, yfd = torch.from_numpy(x).cuda(), yfp.cuda()
     y = torch.empty_like(xd)
     st.step(xd, yfd, y)
@@ -65,3 +67,32 @@ def test_block_step_small(cuda_lib, shape):
         if not e < GRAD_TOL:
             bad[n] = e
     assert not bad, bad
+
+
+# softmax-output quantization (the ablation beside Table A7: W4A4 with the softmax output at 8, 6
+# and 4 bits), per query row over the visible keys
+PQ_CASES = [
+    (I.BlockShape("w4a4_let_p8", T=256, d=256, n_heads=2, n_kv=2, ffn=512, wbits=4, abits=4, group=0, let=1), 8),
+    (I.BlockShape("w4a4_let_gqa_p6", T=256, d=512, n_heads=4, n_kv=2, ffn=768, wbits=4, abits=4, group=0, let=1), 6),
+    (I.BlockShape("w4a4_let_ragged_p4", T=200, d=256, n_heads=2, n_kv=1, ffn=520, wbits=4, abits=4, group=0, let=1), 4),
+    (I.BlockShape("w4a4_let_p2", T=256, d=256, n_heads=2, n_kv=2, ffn=512, wbits=4, abits=4, group=0, let=1), 2),
+]
+
+
+@pytest.mark.parametrize("shape,pbits", PQ_CASES, ids=[s.name for s, _ in PQ_CASES])
+def test_block_step_softmax_quant(cuda_lib, shape, pbits):
+    ref, got = _run(shape, pbits=pbits)
+    assert _rel(got["y"], ref["y"]) < OUT_TOL
+    assert abs(got["loss"] - float(ref["loss"])) / float(ref["loss"]) < OUT_TOL
+    names = O.THETA_NAMES_LWC + O.THETA_NAMES_LET
+    bad = {}
+    for n in names:
+        e = _rel(got["d" + n], ref["d" + n])
+        if not e < GRAD_TOL:
+            bad[n] = e
+    assert not bad, bad
+    if pbits == 2:
+        # the quantizer is really in the path: at 2 bits the s_a gradient moves by ~15% between the
+        # quantized and the unquantized softmax; the kernels must sit much closer to the former
+        ref0, _ = _run(shape, pbits=16, run_cuda=False)
+        assert _rel(got["dsa"], ref["dsa"]) < 0.25 * _rel(ref0["dsa"], ref["dsa"])
