@@ -250,7 +250,7 @@ def run_ours(args, shape):
     n_samples = 4
     xs = [I.make_block_input(shape, sample=i, weight_seed=1 + rank) for i in range(n_samples)]
     th = I.make_block_theta(shape, W, xs[0], seed=2 + rank)
-    st = BlockState(shape, W, th)
+    st = BlockState(shape, W, th, pbits=args.pbits)
     xd = [torch.from_numpy(x).cuda() for x in xs]
     yfp = [torch.empty_like(v) for v in xd]
     for v, y in zip(xd, yfp):          # Eq. 1 targets: the full-precision block (not timed)
@@ -369,9 +369,10 @@ def run_ours(args, shape):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": shape.name, "tokens_per_step": shape.T, "hidden": shape.d,
+        "config": {"workload": shape.name + ("" if args.pbits == 16 else "_softmax%d" % args.pbits),
+                   "tokens_per_step": shape.T, "hidden": shape.d,
                    "heads": shape.n_heads, "kv_heads": shape.n_kv, "ffn": shape.ffn, "wbits": shape.wbits,
-                   "abits": shape.abits, "group": shape.group, "let": shape.let,
+                   "abits": shape.abits, "group": shape.group, "let": shape.let, "softmax_bits": args.pbits,
                    "step": "LET+LWC fake-quant, block fwd, MSE loss, STE bwd, AdamW",
                    "launch": "each step replays a CUDA graph of its launches (one graph per input sample)",
                    "l2": "inputs larger than L2 (bf16 weights %.0f MB per block)" % (
@@ -422,6 +423,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-samples", type=int, default=14)
+    ap.add_argument("--pbits", type=int, default=16,
+                    help="softmax-output bits (2..8: the quantized-softmax ablation; 16: not quantized, the default)")
     args = ap.parse_args()
     from paper_2308_13137_gb300 import inputs as I
     shape = I.block_shape(args.config)

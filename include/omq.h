@@ -287,8 +287,9 @@ omq_status omq_attention_bwd(omq_stream_t stream, int32_t T, int32_t n_heads, in
  * query row are fake-quantized with the MinMax quantizer of Eq. 2 (gamma = beta = 1, step floored at
  * h_eps) over the row's visible keys j <= t before the P V product; masked entries stay 0.
  *   pbits   2..8 (OMQ_ERR_UNSUPPORTED otherwise);
- *   pq_rows [n_heads, T, 8] fp32 out, 16-byte aligned: per query row h, 1/h, z, min/h, floored
- *           (0/1), the first key of the row's max and of its min (as exact floats), unused. */
+ *   pq_rows [n_heads, T, 8] fp32 out, 16-byte aligned: per query row h, 1/h, z, the row's max and
+ *           min probability, floored (0/1), the first key of the max and of the min (as exact
+ *           floats). */
 omq_status omq_attention_pq_fwd(omq_stream_t stream, int32_t T, int32_t n_heads, int32_t n_kv, const void* Q,
                                 int64_t ldq, const void* K, const void* V, int64_t ldkv, float* O, int64_t ldo,
                                 float* lse, int32_t pbits, float h_eps, float* pq_rows, int32_t* dev_status);

@@ -94,9 +94,9 @@ struct FwdP {
 };
 
 // Quantizer state of one query row of the softmax output (MinMax over the visible keys, Eq. 2
-// with gamma = beta = 1): h, 1/h, z, u = m/h, floored (0/1), first index of the max and of the
-// min (as exact floats), unused.
-enum { PQ_H = 0, PQ_RH, PQ_Z, PQ_U, PQ_FL, PQ_IMAX, PQ_IMIN, PQ_N = 8 };
+// with gamma = beta = 1): h, 1/h, z, the row's max and min probability M and m (u = m/h is
+// m * (1/h)), floored (0/1), first index of the max and of the min (as exact floats).
+enum { PQ_H = 0, PQ_RH, PQ_Z, PQ_PMAX, PQ_PMIN, PQ_FL, PQ_IMAX, PQ_IMIN, PQ_N = 8 };
 // Backward statistics of one query row (PQ): D = sum_j P_j dP_j with dP the gradient reaching P
 // through the quantizer, and the totals that reach the row's max and min (R7).
 enum { PG_D = 0, PG_DM, PG_DMIN, PG_N = 4 };
@@ -227,13 +227,25 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       for (int c = 2 * half; c < 2 * half + 2; ++c) {
         float v[32];
         tmem_ld32(sb + 32 * c, v);
-        if constexpr (PQ) {                           // this thread's keys arrive in increasing order
+        if constexpr (PQ) {                           // row minimum of the visible keys
+          float u[16];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            if (diag && 32 * c + i > r) continue;
-            const int key = j * 128 + 32 * c + i;
-            if (v[i] > smax) { smax = v[i]; imx = key; }
-            if (v[i] < smin) { smin = v[i]; imn = key; }
+          for (int i = 0; i < 16; ++i) {
+            const float a = (diag && 32 * c + i > r) ? INFINITY : v[i];
+            const float b = (diag && 32 * c + i + 16 > r) ? INFINITY : v[i + 16];
+            u[i] = fminf(a, b);
+          }
+#pragma unroll
+          for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+            for (int i = 0; i < w; ++i) u[i] = fminf(u[i], u[i + w]);
+          if (u[0] < smin) {                          // this thread's keys arrive in increasing order:
+            smin = u[0];                              // a strict improvement keeps the first index
+            int f = 0;
+#pragma unroll
+            for (int i = 31; i >= 0; --i)
+              if (v[i] == smin && !(diag && 32 * c + i > r)) f = i;
+            imn = j * 128 + 32 * c + f;
           }
         }
         if (diag) {
@@ -247,6 +259,16 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
         for (int w = 8; w >= 1; w >>= 1)
 #pragma unroll
           for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
+        if constexpr (PQ) {
+          if (t[0] > smax) {
+            smax = t[0];
+            int f = 0;
+#pragma unroll
+            for (int i = 31; i >= 0; --i)
+              if (v[i] == smax) f = i;
+            imx = j * 128 + 32 * c + f;
+          }
+        }
         const float m_new = fmaxf(m, t[0] * p.c);
         if (m_new != -INFINITY) {                     // a chunk wholly above the diagonal adds nothing
           float s4[4] = {0.f, 0.f, 0.f, 0.f};
@@ -286,8 +308,10 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     // PQ: the row's quantizer from the probabilities of its max and min score (the map from a score
     // to its probability below is the one pass 2 applies to every key)
     QState qs{};
+    float Mp = 0.f, mp = 0.f;
     if constexpr (PQ) {
-      const float Mp = ex2(fmaf(smax, p.c, -mt)) * inv_l, mp = ex2(fmaf(smin, p.c, -mt)) * inv_l;
+      Mp = ex2(fmaf(smax, p.c, -mt)) * inv_l;
+      mp = ex2(fmaf(smin, p.c, -mt)) * inv_l;
       qs = omq_qstate(Mp, mp, 1.f, 1.f, p.Q, p.eps);
     }
     for (int j = 0; ok && j < nkb; ++j) {             // pass 2: probabilities, O += P V
@@ -339,8 +363,8 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       if constexpr (PQ) {
         if (row < p.T && half == 0) {
           float4* d = reinterpret_cast<float4*>(p.pqr + ((int64_t)h * p.T + row) * PQ_N);
-          d[0] = make_float4(qs.h, qs.rh, qs.z, qs.u);
-          d[1] = make_float4(qs.floored ? 1.f : 0.f, (float)imx, (float)imn, 0.f);
+          d[0] = make_float4(qs.h, qs.rh, qs.z, Mp);
+          d[1] = make_float4(mp, qs.floored ? 1.f : 0.f, (float)imx, (float)imn);
         }
       }
     }
@@ -512,6 +536,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     const int q = warp & 3, half = (warp - 2) >> 2;   // half: which 32 of the 64 query columns
     const int r = q * 32 + lane;                      // key row of the block = TMEM lane
     const int key = kb * 128 + r;
+    const float fkey = (float)key;                    // PQ: compared with the rows' extreme indices
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     uint8_t* pt = smem + B_PT;
     uint8_t* dst = smem + B_DST;
@@ -539,18 +564,18 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             const int qc = 32 * c + i;
-            const float* st = R8 + qc * PQ_N;
-            const float* gs = G4 + qc * PG_N;
+            const float4 s0 = reinterpret_cast<const float4*>(R8 + qc * PQ_N)[0];   // h, 1/h, z, M
+            const float4 s1 = reinterpret_cast<const float4*>(R8 + qc * PQ_N)[1];   // m, fl, imax, imin
+            const float4 gs = *reinterpret_cast<const float4*>(G4 + qc * PG_N);     // D, dM, dm
             const float pv = ex2(fmaf(sv[i], p.c, -Lr[qc]));
-            const float rr = rintf(__fmul_rn(pv, st[PQ_RH]));
-            const float z = st[PQ_Z];
-            const float cd = rr + z;
+            const float rr = rintf(__fmul_rn(pv, s0.y));
+            const float cd = rr + s0.z;
             const bool inr = cd >= 0.f && cd <= p.Q;
             float g = inr ? dp[i] : 0.f;
-            if ((float)key == st[PQ_IMAX]) g += gs[PG_DM];
-            if ((float)key == st[PQ_IMIN]) g += gs[PG_DMIN];
-            sv[i] = __fmul_rn(fminf(fmaxf(rr, -z), p.Q - z), st[PQ_H]);
-            dp[i] = pv * (g - gs[PG_D]) * p.scale;
+            if (fkey == s1.z) g += gs.y;
+            if (fkey == s1.w) g += gs.z;
+            sv[i] = __fmul_rn(fminf(fmaxf(rr, -s0.z), p.Q - s0.z), s0.x);
+            dp[i] = pv * (g - gs.x) * p.scale;
           }
         } else {
 #pragma unroll
@@ -720,21 +745,23 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     const float Lr = row_ok ? p.lse[(int64_t)h * p.T + row] : 0.f;
     float Dr = (MODE == 0 && row_ok) ? p.D[(int64_t)h * p.T + row] : 0.f;
     // PQ: the row's quantizer state (and, for MODE 2, its backward statistics)
-    float q_h = 0.f, q_rh = 0.f, q_z = 0.f, q_ru = 0.f, q_fl = 1.f, q_imax = -1.f, q_imin = -1.f;
+    float q_rh = 0.f, q_z = 0.f, q_ru = 0.f, q_fl = 1.f, q_M = 0.f, q_m = 0.f;
+    int q_imax = -1, q_imin = -1;
     float g_dM = 0.f, g_dm = 0.f;
     if (MODE != 0 && row_ok) {
       const float4* st = reinterpret_cast<const float4*>(p.pqr + ((int64_t)h * p.T + row) * PQ_N);
       const float4 a0 = st[0], a1 = st[1];
-      q_h = a0.x; q_rh = a0.y; q_z = a0.z; q_ru = rintf(a0.w) - a0.w; q_fl = a1.x; q_imax = a1.y; q_imin = a1.z;
+      const float u = __fmul_rn(a1.x, a0.y);        // m / h as the forward formed it
+      q_rh = a0.y; q_z = a0.z; q_M = a0.w; q_m = a1.x; q_ru = rintf(u) - u; q_fl = a1.y;
+      q_imax = (int)a1.z; q_imin = (int)a1.w;
       if (MODE == 2) {
         const float4 gs = *reinterpret_cast<const float4*>(p.pqb + ((int64_t)h * p.T + row) * PG_N);
         Dr = gs.x; g_dM = gs.y; g_dm = gs.z;
       }
     }
-    (void)q_h;
-    // MODE 1 sums over the row's keys: sum of P dP inside the clamp range, the h-path total G_h,
-    // the clamped total, and P at the row's max / min keys
-    float a_E = 0.f, a_Gh = 0.f, a_Gc = 0.f, a_PM = 0.f, a_Pm = 0.f;
+    // MODE 1 sums over the row's keys: sum of P dP inside the clamp range, the h-path total G_h and
+    // the clamped total
+    float a_E = 0.f, a_Gh = 0.f, a_Gc = 0.f;
     bool ok = true;
     for (int j = 0; j < nkb; ++j) {
       const int s = j & 1;
@@ -768,13 +795,11 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
                 const float dh = inr ? rr - x : (cd < 0.f ? q_ru : p.Q + q_ru);
                 if (inr) a_E = fmaf(pv, dp[i], a_E); else a_Gc += dp[i];
                 a_Gh = fmaf(dp[i], dh, a_Gh);
-                if ((float)key == q_imax) a_PM = pv;
-                if ((float)key == q_imin) a_Pm = pv;
               }
             } else {
               float g = inr ? dp[i] : 0.f;
-              if ((float)key == q_imax) g += g_dM;
-              if ((float)key == q_imin) g += g_dm;
+              if (key == q_imax) g += g_dM;
+              if (key == q_imin) g += g_dm;
               dp[i] = pv * (g - Dr) * p.scale;
             }
           }
@@ -800,21 +825,20 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     if constexpr (MODE == 1) {
       // combine the two halves of every row through the (unused) dS buffers; every compute thread
       // reaches this barrier exactly once
-      float* x5 = reinterpret_cast<float*>(smem + Q_DS);              // [half][5][128]
-      x5[(half * 5 + 0) * 128 + r] = a_E;
-      x5[(half * 5 + 1) * 128 + r] = a_Gh;
-      x5[(half * 5 + 2) * 128 + r] = a_Gc;
-      x5[(half * 5 + 3) * 128 + r] = a_PM;
-      x5[(half * 5 + 4) * 128 + r] = a_Pm;
+      float* x3 = reinterpret_cast<float*>(smem + Q_DS);              // [half][3][128]
+      x3[(half * 3 + 0) * 128 + r] = a_E;
+      x3[(half * 3 + 1) * 128 + r] = a_Gh;
+      x3[(half * 3 + 2) * 128 + r] = a_Gc;
       asm volatile("bar.sync 1, 256;" ::: "memory");
       if (ok && half == 0 && row_ok) {
-        float t[5];
+        float t[3];
 #pragma unroll
-        for (int k = 0; k < 5; ++k) t[k] = x5[k * 128 + r] + x5[(5 + k) * 128 + r];   // one half holds each P
+        for (int k = 0; k < 3; ++k) t[k] = x3[k * 128 + r] + x3[(3 + k) * 128 + r];
         const float Gh = q_fl != 0.f ? 0.f : t[1];    // a floored step has no gradient
         const float dM = Gh / p.Q, dm = t[2] - Gh / p.Q;
+        // sum_j P_j dP_j, dP including the totals that reach the max and the min (R7)
         *reinterpret_cast<float4*>(p.pqb + ((int64_t)h * p.T + row) * PG_N) =
-            make_float4(t[0] + t[3] * dM + t[4] * dm, dM, dm, 0.f);
+            make_float4(t[0] + q_M * dM + q_m * dm, dM, dm, 0.f);
       }
     } else if (ok) {
       tc_fence_after();

@@ -78,8 +78,8 @@ def test_attention_pq_fwd_bwd(cuda_lib, T, H, Hkv, bits):
     Pv = P.masked_fill(~causal, float("nan"))
     want_imax = torch.nan_to_num(Pv, nan=-1.0).argmax(-1)
     want_imin = torch.nan_to_num(Pv, nan=2.0).argmin(-1)
-    assert torch.equal(pr[..., 5].long(), want_imax)
-    assert torch.equal(pr[..., 6].long(), want_imin)
+    assert torch.equal(pr[..., 6].long(), want_imax)
+    assert torch.equal(pr[..., 7].long(), want_imin)
     Mx = P.gather(-1, want_imax[..., None])[..., 0]
     mn = P.gather(-1, want_imin[..., None])[..., 0]
     h_ref = torch.clamp((Mx - mn) / (2 ** bits - 1), min=EPS)
