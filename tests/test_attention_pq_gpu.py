@@ -95,3 +95,42 @@ def test_attention_pq_fwd_bwd(cuda_lib, T, H, Hkv, bits):
         # the h path matters at low bit widths: a backward without it would be far off
         _, wdQ, wdK, _, _ = _ref(Q.float(), K.float(), V.float(), dO.float(), H, Hkv, bits, plain_ste=True)
         assert errs["dQ"] < 0.2 * _rel(wdQ, rdQ) and errs["dK"] < 0.2 * _rel(wdK, rdK)
+
+
+@pytest.mark.full
+@pytest.mark.parametrize("bits", [8, 4])
+def test_attention_pq_full_size(cuda_lib, bits):
+    """The LLaMA-7B attention of the step (2048 tokens, 32 heads of 128) with the softmax output
+    quantized: the kernels run the whole grid; heads 0 and 31 are checked against the oracle
+    composition in full (every row, every key)."""
+    T, H, Hkv = 2048, 32, 32
+    g = torch.Generator().manual_seed(2048 + bits)
+    Q = (torch.randn(T, H * 128, generator=g) * 1.5).to(torch.bfloat16)
+    K = (torch.randn(T, Hkv * 128, generator=g) * 1.5).to(torch.bfloat16)
+    V = torch.randn(T, Hkv * 128, generator=g).to(torch.bfloat16)
+    dO = torch.randn(T, H * 128, generator=g).to(torch.bfloat16)
+    d = lambda t: t.cuda().contiguous()
+    Od = torch.empty(T, H * 128, device="cuda")
+    lse = torch.empty(H, T, device="cuda")
+    pqr = torch.empty(H, T, 8, device="cuda")
+    pqb = torch.empty(H, T, 4, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    dQ = torch.empty(T, H * 128, device="cuda")
+    dK = torch.empty(T, Hkv * 128, device="cuda")
+    dV = torch.empty(T, Hkv * 128, device="cuda")
+    Qd, Kd, Vd, dOd = d(Q), d(K), d(V), d(dO)
+    _lib.omq_attention_pq_fwd(T, H, Hkv, Qd, H * 128, Kd, Vd, Hkv * 128, Od, H * 128, lse, bits, EPS, pqr, st)
+    _lib.omq_attention_pq_bwd(T, H, Hkv, Qd, H * 128, Kd, Vd, Hkv * 128, lse, dOd, H * 128, dQ, H * 128, dK, dV,
+                              Hkv * 128, bits, pqr, pqb, st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    for hh in (0, H - 1):
+        cols = slice(hh * 128, (hh + 1) * 128)
+        rO, rdQ, rdK, rdV, _ = _ref(Q[:, cols].float(), K[:, cols].float(), V[:, cols].float(),
+                                    dO[:, cols].float(), 1, 1, bits)
+        errs = dict(O=_rel(Od[:, cols], rO), dQ=_rel(dQ[:, cols], rdQ), dK=_rel(dK[:, cols], rdK),
+                    dV=_rel(dV[:, cols], rdV))
+        print(hh, bits, errs)
+        assert errs["O"] < 1e-2
+        for n in ("dQ", "dK", "dV"):
+            assert errs[n] < 2e-2, (n, errs)
