@@ -75,6 +75,9 @@ notes of the repository):
      reciprocal of h; the clipping strengths entering it are the single-precision sigmoid
      of `sigmoid_fp32`.  Everything else stays float64.  ("emulate" mode; "exact"
      mode decides in float64.)
+ R19 ("emulate" mode) the unquantized softmax enters the P V product unnormalised: bf16 of
+     2^(S log2(e) - M) with M an integer not below the row maximum of S log2(e) (the rounding is the
+     same for every such M), the product divided by the unrounded row sum afterwards.
  R20 softmax-output quantization (the ablation of Table A7, off by default): the causal softmax
      output is quantized per query row with the MinMax Q_a (gamma = beta = 1, the floor of h
      included) over the visible keys j <= t only; the masked entries stay 0.  Its decisions are
@@ -96,7 +99,7 @@ __all__ = [
     "let_apply", "block_loss", "qlinear_step", "BlockCfg", "block_forward", "block_step",
     "rmsnorm", "rope", "silu", "FrozenTape", "use_tape", "block_fp_forward", "sigmoid_fp32",
     "THETA_NAMES_LWC", "THETA_NAMES_LET", "let_init", "pack_codes", "unpack_codes", "block_fold_pack",
-    "folded_forward", "adamw_step", "calibrate_blocks", "softmax_quant",
+    "folded_forward", "adamw_step", "calibrate_blocks", "softmax_quant", "softmax_pv",
 ]
 
 
@@ -671,6 +674,35 @@ def _qp(P, cfg: BlockCfg):
     return softmax_quant(P, cfg.pbits, cfg.h_eps, _decide(cfg))
 
 
+LOG2E = 1.0 / math.log(2.0)
+
+
+def softmax_pv(S, Vh, mode: str):
+    """softmax(S) V per head, S [..., T, T] with -inf at masked keys, Vh [..., T, hd] (Sec. 3.3; the
+    softmax output is not quantized, R12).  "emulate" (R19): the value is
+    (bf16(2^(S log2(e) - M)) bf16(V)) / l, with M the row maximum of S log2(e) rounded up to an
+    integer and l the unrounded row sum of 2^(S log2(e) - M): the probabilities enter the product
+    unnormalised and the row sum divides it afterwards.  Rounding to bf16 commutes with scaling by
+    a power of two, so any integer M gives the same value.  The gradient is that of softmax(S) V
+    under R13."""
+    O = _mm(torch.softmax(S, dim=-1), Vh.transpose(-1, -2), mode)
+    if mode != "emulate":
+        return O
+    with torch.no_grad():
+        t = S * LOG2E
+        E = torch.exp2(t - torch.ceil(t.amax(dim=-1, keepdim=True)))
+        On = (to_bf16(E) @ to_bf16(Vh)) / E.sum(dim=-1, keepdim=True)
+    return O + (On - O).detach()
+
+
+def _attn_pv(S, Vh, cfg: BlockCfg):
+    """The attention output from the masked scores: softmax(S) V (R19), or with the softmax
+    output quantized (R20) the quantized probabilities, rounded to bf16 (R13), times V."""
+    if cfg.pbits >= 16:
+        return softmax_pv(S, Vh, cfg.mode)
+    return _mm(_qp(torch.softmax(S, dim=-1), cfg), Vh.transpose(-1, -2), cfg.mode)
+
+
 def _dec32(W, s=None, r=None):
     """fp32 quantizer input of a scaled weight, formed as the kernels form it (R15)."""
     with torch.no_grad():
@@ -728,8 +760,7 @@ def block_forward(x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], c
     S = _mm(Qh, Kh, mode) / math.sqrt(hd)                                # R10
     causal = torch.ones(T, T, dtype=torch.bool).tril()
     S = S.masked_fill(~causal, float("-inf"))
-    P = _qp(torch.softmax(S, dim=-1), cfg)                              # unquantized by default (R12, R20)
-    O = _mm(P, Vh.transpose(-1, -2), mode)                               # P V, [H, T, hd]
+    O = _attn_pv(S, Vh, cfg)                                             # P V, [H, T, hd] (R12, R19, R20)
     O = O.transpose(0, 1).reshape(T, H * hd)
     oh = _qa(O, cfg)
     if let:
@@ -761,7 +792,7 @@ def block_forward(x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], c
     mh = _qa(m, cfg)                                      # down_proj input: no LET (Sec. 3.3)
     y = h1 + _mm(mh, _qw(wdn, th.get("gamma_d"), th.get("beta_d"), cfg), mode)
     if keep is not None:
-        keep.update(dict(a=a, q=q, k=k, v=v, O=O, h1=h1, gate=gt, up=up, m=m, P=P))
+        keep.update(dict(a=a, q=q, k=k, v=v, O=O, h1=h1, gate=gt, up=up, m=m))
     return y
 
 
@@ -943,7 +974,7 @@ def folded_forward(folded: Dict[str, torch.Tensor], x, cfg: BlockCfg) -> torch.T
         Vh = vh.reshape(T, Hkv, hd).transpose(0, 1).repeat_interleave(rep, 0)
         S = _mm(Qh, Kh, mode) / math.sqrt(hd)
         S = S.masked_fill(~torch.ones(T, T, dtype=torch.bool).tril(), float("-inf"))
-        O = _mm(_qp(torch.softmax(S, dim=-1), cfg), Vh.transpose(-1, -2), mode).transpose(0, 1).reshape(T, dq)
+        O = _attn_pv(S, Vh, cfg).transpose(0, 1).reshape(T, dq)
         o = _mm(_qa(O, cfg), deq("o", d, dq), mode)
         if let:
             o = o + folded["b_o"]

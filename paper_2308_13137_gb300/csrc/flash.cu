@@ -1,15 +1,16 @@
-// Causal attention of the quantized block (Sec. 3.3 / Eq. 5: Q_a-quantized Q~, K~, V' in bf16,
-// softmax output kept unquantized) without materialising the score matrix.
+// Causal attention of the quantized block (Sec. 3.3 / Eq. 5: Q_a-quantized Q~, K~, V' in bf16)
+// without materialising the score matrix.
 //
-// Forward: one CTA per (128-query block, query head), two passes over the key blocks.  TMA
-// streams 128-key blocks through a two-slot ring; tcgen05.mma forms S = Q K^T in one of two
-// tensor-memory buffers while the four compute warps (one query row per thread) work on the
-// previous one.  Pass 1 reduces S to the row maximum m and the row sum l of exp2(c S - m); pass 2
-// recomputes S and writes the normalised probabilities P = bf16(exp2(c S - m) / l) into shared
-// memory in the 128-byte-swizzled operand layout, and the MMA warp accumulates O += P V in tensor
-// memory.  Rounding the normalised P to bf16 (not a running, unnormalised one) keeps the product
-// identical to softmax-then-round; the extra S product costs one 128-dim contraction.  The row
-// log-sum-exp (base 2, scaled logits) is saved for the backward.
+// Forward (softmax output not quantized): one CTA per (128-query block, query head), one pass over
+// the key blocks.  TMA streams 128-key blocks of K (three slots) and V (two slots); tcgen05.mma
+// forms S = Q K^T in one of two tensor-memory buffers while the compute warps work on the previous
+// one; each 64-key half of a row turns its scores into unnormalised probabilities 2^(c S - M)
+// against its own integer reference M (moved up by whole powers of two, see flash_fwd1_kernel),
+// writes them as bf16 into shared memory in the 128-byte-swizzled operand layout, and the MMA warp
+// accumulates the half's O += P V in tensor memory; the halves are combined and divided by the
+// row sum at the end.  The row log-sum-exp (base 2, scaled logits) is saved for the backward.
+// With the softmax output quantized (flash_fwd_kernel<true>), the forward takes two passes: row
+// max, sum and extremes first, then the normalised probabilities, quantized per row.
 //
 // Backward: dKV kernel per (128-key block, kv head) walks the 64-query blocks of every query head
 // of its group: S^T = K Q^T and dP^T = V dO^T (double-buffered in tensor memory), P^T and
@@ -367,6 +368,212 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
           d[1] = make_float4(mp, qs.floored ? 1.f : 0.f, (float)imx, (float)imn);
         }
       }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// 2^k for an integer-valued k <= 0 (0 below the normal range), exact
+__device__ __forceinline__ float pow2_int(float k) {
+  return k < -126.f ? 0.f : __int_as_float((127 + (int)k) << 23);
+}
+
+// Single-pass forward (softmax output not quantized).  Each 64-key half of a row (one compute warp
+// of the pair sharing the row's lane quadrant) keeps its own integer reference M of the scaled
+// logits, its own row sum l and its own output accumulator in tensor memory (O_0, O_1): the
+// probabilities 2^(c S - M) enter the P V product unnormalised, and when a block lifts the half's
+// maximum more than F_TAU above M, M moves up to the ceiling of the new maximum and l and the
+// half's accumulator rows are scaled by the exact power of two 2^(M_old - M_new).  Rounding to
+// bf16 commutes with powers of two, so the product is exactly that of one common reference; the
+// halves are combined and divided by l once, at the end.
+constexpr float F_TAU = 8.f;                          // unnormalised probabilities stay below 2^8
+
+__global__ void __launch_bounds__(FA_THREADS, 1)
+    flash_fwd1_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                      const __grid_constant__ CUtensorMap tmV, const FwdP p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  Ctl* ctl = reinterpret_cast<Ctl*>(smem + F_CTL);
+  uint64_t* q_full = &ctl->bar[0];
+  uint64_t* k_full = &ctl->bar[1];        // [F_NK]
+  uint64_t* k_empty = &ctl->bar[4];       // [F_NK]
+  uint64_t* v_full = &ctl->bar[7];        // [F_NV]
+  uint64_t* v_empty = &ctl->bar[9];       // [F_NV]
+  uint64_t* s_full = &ctl->bar[11];       // [2]
+  uint64_t* p_full = &ctl->bar[13];
+  uint64_t* o_done = &ctl->bar[14];
+  volatile int* abort_flag = &ctl->abort;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nqb = (p.T + 127) / 128;
+  const int qb = nqb - 1 - (int)blockIdx.y;           // every head's longest query block first
+  const int h = blockIdx.x, g = h / p.rep;
+  const int nkb = qb + 1;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < F_NK; ++s) { mbar_init(&k_full[s], 1); mbar_init(&k_empty[s], 1); }
+    for (int s = 0; s < F_NV; ++s) { mbar_init(&v_full[s], 1); mbar_init(&v_empty[s], 1); }
+    for (int s = 0; s < 2; ++s) mbar_init(&s_full[s], 1);
+    mbar_init(p_full, 8);
+    mbar_init(o_done, 1);
+    ctl->abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(&ctl->tmem, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = ctl->tmem;           // S buffers at columns 0 / 128, O_0 at 256, O_1 at 384
+
+  if (warp == 0 && lane == 0) {
+    mbar_expect_tx(q_full, F_TILE);
+    load_tile(&tmQ, q_full, smem + F_Q, h * HD, qb * 128, F_ATOM);
+    for (int j = 0; j < nkb && !*abort_flag; ++j) {
+      const int sk = j % F_NK, sv = j % F_NV;
+      if (!waitb(&k_empty[sk], ((j / F_NK) & 1) ^ 1, p.status, abort_flag)) break;
+      mbar_expect_tx(&k_full[sk], F_TILE);
+      load_tile(&tmK, &k_full[sk], smem + F_K + sk * F_TILE, g * HD, j * 128, F_ATOM);
+      if (!waitb(&v_empty[sv], ((j / F_NV) & 1) ^ 1, p.status, abort_flag)) break;
+      mbar_expect_tx(&v_full[sv], F_TILE);
+      load_tile(&tmV, &v_full[sv], smem + F_V + sv * F_TILE, g * HD, j * 128, F_ATOM);
+    }
+  } else if (warp == 1 && lane == 0) {
+    constexpr uint32_t ID_S = idesc_bf16(128, 128, 0, 0), ID_O = idesc_bf16(128, 128, 0, 1);
+    const uint32_t sq = smem_u32(smem + F_Q), sk = smem_u32(smem + F_K), sv = smem_u32(smem + F_V);
+    const uint32_t sp = smem_u32(smem + F_P);
+    bool ok = waitb(q_full, 0, p.status, abort_flag);
+    auto issue_s = [&](int j) -> bool {
+      const int s = j & 1, r = j % F_NK;
+      if (!waitb(&k_full[r], (j / F_NK) & 1, p.status, abort_flag)) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk)
+        umma_bf16(tmem + 128 * s, desc_k(sq, kk, F_ATOM), desc_k(sk + r * F_TILE, kk, F_ATOM), ID_S, kk > 0);
+      umma_commit(&s_full[s]);
+      umma_commit(&k_empty[r]);                       // K is free once S is formed
+      return true;
+    };
+    if (ok) ok = issue_s(0);
+    for (int j = 0; ok && j < nkb; ++j) {
+      // S buffer (j+1)&1 was last read at j-1, whose p_full was waited for below
+      if (j + 1 < nkb && !issue_s(j + 1)) break;
+      if (!waitb(p_full, j & 1, p.status, abort_flag)) break;
+      const int r = j % F_NV;
+      if (!waitb(&v_full[r], (j / F_NV) & 1, p.status, abort_flag)) break;
+      tc_fence_after();
+      // keys 0..63 of the block (P atom 0, V rows 0..63) into O_0, keys 64..127 into O_1
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk)
+        umma_bf16(tmem + 256 + 128 * (kk >> 2), desc_k(sp, kk, F_ATOM), desc_mn(sv + r * F_TILE, kk, F_ATOM), ID_O,
+                  (j | (kk & 3)) != 0);
+      umma_commit(o_done);
+      umma_commit(&v_empty[r]);
+    }
+  } else if (warp >= 2) {
+    // eight compute warps: warps w and w+4 share TMEM lane quadrant w % 4 (rows); half 0 takes
+    // keys 0..63 of each block, half 1 keys 64..127, each with its own reference and accumulator
+    const int q = warp & 3, half = (warp - 2) >> 2;
+    const int r = q * 32 + lane;                      // row of the block = TMEM lane
+    const int row = qb * 128 + r;
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    const uint32_t o_acc = tmem + 256 + 128 * half + lane_off;
+    uint8_t* ptile = smem + F_P;
+    float M = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nkb; ++j) {
+      if (!(ok = waitw(&s_full[j & 1], (j >> 1) & 1, p.status, abort_flag))) break;
+      tc_fence_after();
+      const uint32_t sb = tmem + 128 * (j & 1) + lane_off;
+      const bool diag = (j == qb);                    // keys beyond the row exist only here
+      float v[2][32];
+#pragma unroll
+      for (int cc = 0; cc < 2; ++cc) {
+        const int c = 2 * half + cc;
+        tmem_ld32(sb + 32 * c, v[cc]);
+        if (diag) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) if (32 * c + i > r) v[cc][i] = -INFINITY;
+        }
+      }
+      float t[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) t[i] = fmaxf(fmaxf(v[0][i], v[0][i + 16]), fmaxf(v[1][i], v[1][i + 16]));
+#pragma unroll
+      for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
+      const float mb = t[0] * p.c;                    // c > 0: max of c S = c max S
+      const bool lift = mb > M + F_TAU;               // false while the half has seen no key (mb = -inf)
+      const float Mn = lift ? ceilf(mb) : M;
+      const float fac = lift ? (M == -INFINITY ? 0.f : pow2_int(M - Mn)) : 1.f;
+      float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int cc = 0; cc < 2; ++cc) {
+        const int c = 2 * half + cc;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float e = (Mn == -INFINITY || (diag && 32 * c + i > r)) ? 0.f : ex2(fmaf(v[cc][i], p.c, -Mn));
+          v[cc][i] = e;
+          ls[i & 3] += e;
+        }
+      }
+      l = l * fac + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
+      M = Mn;
+      if (j > 0) {                                    // the previous P V product has read P, written O
+        if (!(ok = waitw(o_done, (j - 1) & 1, p.status, abort_flag))) break;
+        tc_fence_after();
+        if (__any_sync(0xffffffffu, fac != 1.f)) {    // rows whose reference moved: rescale their O rows
+#pragma unroll 1
+          for (int c = 0; c < 4; ++c) {
+            float o[32];
+            tmem_ld32(o_acc + 32 * c, o);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] *= fac;
+            tmem_st32(o_acc + 32 * c, o);
+          }
+        }
+      }
+#pragma unroll
+      for (int cc = 0; cc < 2; ++cc) st_row32(ptile, F_ATOM, r, 32 * (2 * half + cc), v[cc]);
+      fence_async_smem();                             // P visible to the tensor core
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+    }
+    // the last P V product has read P: its tile holds the halves' references and sums now
+    if (ok) ok = waitw(o_done, (nkb - 1) & 1, p.status, abort_flag);
+    float* stat = reinterpret_cast<float*>(smem + F_ST);   // [2 halves][M | l][128 rows]
+    stat[(half * 2 + 0) * 128 + r] = M;
+    stat[(half * 2 + 1) * 128 + r] = l;
+    asm volatile("bar.sync 1, 256;" ::: "memory");   // every compute thread arrives exactly once
+    const float M0 = stat[r], l0 = stat[128 + r], M1 = stat[256 + r], l1 = stat[384 + r];
+    const float Mt = fmaxf(M0, M1);
+    const float f0 = M0 == -INFINITY ? 0.f : pow2_int(M0 - Mt), f1 = M1 == -INFINITY ? 0.f : pow2_int(M1 - Mt);
+    const float lt = l0 * f0 + l1 * f1;
+    const float a0 = f0 / lt, a1 = f1 / lt;
+    if (ok) {
+      tc_fence_after();
+#pragma unroll 1
+      for (int c = 2 * half; c < 2 * half + 2; ++c) {
+        float o0[32], o1[32];
+        tmem_ld32(tmem + 256 + lane_off + 32 * c, o0);
+        tmem_ld32(tmem + 384 + lane_off + 32 * c, o1);
+        if (row < p.T) {
+          float4* dst = reinterpret_cast<float4*>(p.O + (int64_t)row * p.ldo + h * HD + 32 * c);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            dst[i] = make_float4(fmaf(o0[4 * i], a0, o1[4 * i] * a1), fmaf(o0[4 * i + 1], a0, o1[4 * i + 1] * a1),
+                                 fmaf(o0[4 * i + 2], a0, o1[4 * i + 2] * a1),
+                                 fmaf(o0[4 * i + 3], a0, o1[4 * i + 3] * a1));
+        }
+      }
+      if (row < p.T && half == 0) p.lse[(int64_t)h * p.T + row] = Mt + log2f(lt);
     }
   }
   tc_fence_before();
@@ -885,7 +1092,7 @@ omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
   OMQ_REQUIRE(!pq || (a.pqr && omq_aligned16(a.pqr)), OMQ_ERR_INVALID_ARG);
   static bool attr = false;
   if (!attr) {
-    if (!set_smem((const void*)flash_fwd_kernel<false>, F_SMEM) || !set_smem((const void*)flash_fwd_kernel<true>, F_SMEM))
+    if (!set_smem((const void*)flash_fwd1_kernel, F_SMEM) || !set_smem((const void*)flash_fwd_kernel<true>, F_SMEM))
       return OMQ_ERR_CUDA;
     attr = true;
   }
@@ -896,7 +1103,7 @@ omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
   p.Q = pq ? (float)((1 << a.pbits) - 1) : 0.f; p.eps = a.eps; p.pqr = a.pqr;
   dim3 grid((unsigned)a.H, (unsigned)((a.T + 127) / 128));
   if (pq) flash_fwd_kernel<true><<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, p);
-  else flash_fwd_kernel<false><<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, p);
+  else flash_fwd1_kernel<<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }

@@ -451,6 +451,39 @@ def test_softmax_quant_ste_gradient_is_per_row_quant_bwd(nbits):
             assert bool((dP[hh, t, t + 1:] == 0).all())
 
 
+def test_emulated_softmax_pv():
+    """R19: the emulated P V product rounds the unnormalised probabilities 2^(S log2 e - M) (M an
+    integer) to bf16 and divides by their unrounded sum.  Equal scores make every probability
+    exactly 1: the causal prefix mean of the bf16 values.  Shifting a row's scores by an integer
+    multiple of ln 2 changes nothing (bf16 rounding commutes with powers of two).  Every output is
+    a convex combination with each weight perturbed by at most 2^-9 relative, so it stays within
+    2^-8 max|V| of the exact softmax(S) V on the same bf16 V.  The gradient is that of
+    softmax(S) V with bf16 operands (R13)."""
+    g = torch.Generator().manual_seed(19)
+    H, T, hd = 2, 7, 4
+    V = torch.randn(H, T, hd, generator=g, dtype=F64)
+    Vb = O.to_bf16(V)
+    causal = torch.ones(T, T, dtype=torch.bool).tril()
+    S0 = torch.zeros(H, T, T, dtype=F64).masked_fill(~causal, float("-inf"))
+    got = O.softmax_pv(S0, V, "emulate")
+    want = torch.cumsum(Vb, 1) / torch.arange(1, T + 1, dtype=F64)[None, :, None]
+    assert torch.allclose(got, want, rtol=0, atol=1e-14)
+    S = (torch.randn(H, T, T, generator=g, dtype=F64) * 3).masked_fill(~causal, float("-inf"))
+    got = O.softmax_pv(S, V, "emulate")
+    shift = torch.randint(-5, 6, (H, T, 1), generator=g).to(F64) * math.log(2.0)
+    assert torch.allclose(O.softmax_pv(S + shift, V, "emulate"), got, rtol=0, atol=1e-13)
+    exact = torch.softmax(S, -1) @ Vb
+    err = float((got - exact).abs().max())
+    assert 0 < err <= 2.0 ** -8 * float(Vb.abs().max())
+    Sg = S.clone().requires_grad_(True)
+    gO = torch.randn(H, T, hd, generator=g, dtype=F64)
+    (gS,) = torch.autograd.grad(O.softmax_pv(Sg, V, "emulate"), [Sg], gO)
+    P = torch.softmax(S, -1)
+    dP = O.to_bf16(gO) @ Vb.transpose(-1, -2)
+    ref = P * (dP - (dP * P).sum(-1, keepdim=True))
+    assert torch.allclose(gS, ref, rtol=1e-12, atol=1e-14)
+
+
 def test_rope_properties():
     g = torch.Generator().manual_seed(13)
     T, H, hd = 9, 2, 8
