@@ -286,7 +286,8 @@ omq_status omq_attention_bwd(omq_stream_t stream, int32_t T, int32_t n_heads, in
  * method's default configuration).  As omq_attention_fwd, except that the probabilities of every
  * query row are fake-quantized with the MinMax quantizer of Eq. 2 (gamma = beta = 1, step floored at
  * h_eps) over the row's visible keys j <= t before the P V product; masked entries stay 0.
- *   pbits   2..8 (OMQ_ERR_UNSUPPORTED otherwise);
+ *   pbits   2..8 (OMQ_ERR_UNSUPPORTED otherwise); h_eps > 0 (OMQ_ERR_INVALID_ARG otherwise);
+ *   (a null pq_rows is OMQ_ERR_INVALID_ARG, a misaligned one OMQ_ERR_ALIGN)
  *   pq_rows [n_heads, T, 8] fp32 out, 16-byte aligned: per query row h, 1/h, z, the row's max and
  *           min probability, floored (0/1), the first key of the max and of the min (as exact
  *           floats). */

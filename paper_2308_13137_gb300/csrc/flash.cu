@@ -1080,6 +1080,9 @@ omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
   OMQ_REQUIRE(a.Q && a.K && a.V && a.O && a.lse, OMQ_ERR_INVALID_ARG);
   OMQ_REQUIRE(a.ldq % 8 == 0 && a.ldkv % 8 == 0 && a.ldo % 4 == 0, OMQ_ERR_ALIGN);
   OMQ_REQUIRE(omq_aligned16(a.Q) && omq_aligned16(a.K) && omq_aligned16(a.V) && omq_aligned16(a.O), OMQ_ERR_ALIGN);
+  const bool pq = flash_pq_on(a.pbits);
+  OMQ_REQUIRE(!pq || a.pqr, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(!pq || omq_aligned16(a.pqr), OMQ_ERR_ALIGN);
   CUtensorMap tq, tk, tv;
   bool ok = omq_make_map_bf16(&tq, a.Q, (int64_t)a.H * HD, a.T, 1, a.ldq, 0, 64, 128);
   ok = ok && omq_make_map_bf16(&tk, a.K, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 128);
@@ -1088,8 +1091,6 @@ omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
   ok = ok && omq_make_map_bf16(&tk64, a.K, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
   ok = ok && omq_make_map_bf16(&tv64, a.V, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
   if (!ok) return OMQ_ERR_UNSUPPORTED;
-  const bool pq = flash_pq_on(a.pbits);
-  OMQ_REQUIRE(!pq || (a.pqr && omq_aligned16(a.pqr)), OMQ_ERR_INVALID_ARG);
   static bool attr = false;
   if (!attr) {
     if (!set_smem((const void*)flash_fwd1_kernel, F_SMEM) || !set_smem((const void*)flash_fwd_kernel<true>, F_SMEM))
@@ -1118,6 +1119,8 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
   OMQ_REQUIRE(omq_aligned16(a.dO) && omq_aligned16(a.dQ) && omq_aligned16(a.dK) && omq_aligned16(a.dV), OMQ_ERR_ALIGN);
   // lse, D and the PQ row data are fetched by 16-byte bulk copies
   OMQ_REQUIRE(a.T % 4 == 0 && omq_aligned16(a.lse) && (pq || omq_aligned16(a.D)), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(!pq || (a.pqr && a.pqb), OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(!pq || (omq_aligned16(a.pqr) && omq_aligned16(a.pqb)), OMQ_ERR_ALIGN);
   CUtensorMap tq64, tdo64, tk, tv, tq, tdo;
   bool ok = omq_make_map_bf16(&tq64, a.Q, (int64_t)a.H * HD, a.T, 1, a.ldq, 0, 64, 64);
   ok = ok && omq_make_map_bf16(&tdo64, a.dO, (int64_t)a.H * HD, a.T, 1, a.lddo, 0, 64, 64);
@@ -1129,7 +1132,6 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
   ok = ok && omq_make_map_bf16(&tk64, a.K, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
   ok = ok && omq_make_map_bf16(&tv64, a.V, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
   if (!ok) return OMQ_ERR_UNSUPPORTED;
-  OMQ_REQUIRE(!pq || (a.pqr && a.pqb && omq_aligned16(a.pqr) && omq_aligned16(a.pqb)), OMQ_ERR_INVALID_ARG);
   static bool attr = false;
   if (!attr) {
     if (!set_smem((const void*)flash_bwd_dkv_kernel<false>, BL<false>::SMEM) ||

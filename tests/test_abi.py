@@ -22,10 +22,10 @@ def test_exports_every_declared_function():
 
 
 def _cfg(**kw):
-    base = dict(wbits=4, abits=16, group=128, let=0, h_eps=1e-5, accumulate=0, dev_status=None)
+    base = dict(wbits=4, abits=16, group=128, let=0, h_eps=1e-5, accumulate=0, dev_status=None, pbits=0)
     base.update(kw)
     return _lib.omq_qcfg(base["wbits"], base["abits"], base["group"], base["let"], base["h_eps"],
-                         base["accumulate"], base["dev_status"])
+                         base["accumulate"], base["dev_status"], base["pbits"])
 
 
 FAKE = 0x10000     # 16-byte aligned dummy address: every call below returns before touching it
@@ -56,6 +56,22 @@ def test_argument_errors_before_launch():
                            None, None, 0, 0.0, 7, None) == 1
 
 
+def test_softmax_quant_argument_errors():
+    """The softmax-output quantizer's bit width and step floor are checked before any launch."""
+    L = _lib.lib()
+    assert _lwc_fwd(64, 512, _cfg(pbits=9)) == 4               # pbits outside 2..8 (0 / 16 = off)
+    assert _lwc_fwd(64, 512, _cfg(pbits=1)) == 4
+    for bits in (1, 9, 16, 0):
+        assert L.omq_attention_pq_fwd(None, 256, 2, 2, FAKE, 256, FAKE, FAKE, 256, FAKE, 256, FAKE, bits, 1e-5,
+                                      FAKE, None) == 4
+        assert L.omq_attention_pq_bwd(None, 256, 2, 2, FAKE, 256, FAKE, FAKE, 256, FAKE, FAKE, 256, FAKE, 256, FAKE,
+                                      FAKE, 256, bits, FAKE, FAKE, None) == 4
+    assert L.omq_attention_pq_fwd(None, 256, 2, 2, FAKE, 256, FAKE, FAKE, 256, FAKE, 256, FAKE, 8, 0.0,
+                                  FAKE, None) == 1             # h_eps must be positive
+    assert L.omq_attention_pq_fwd(None, 256, 2, 2, FAKE, 256, FAKE, FAKE, 256, FAKE, 256, FAKE, 8, 1e-5,
+                                  None, None) == 1             # the row records are required
+
+
 def test_block_workspace_sizes():
     sh = I.SHAPES["llama7b_w4a4"]
     s = _lib.omq_block_shape(sh.T, sh.d, sh.n_heads, sh.n_kv, sh.head_dim, sh.ffn, sh.rms_eps, sh.rope_theta)
@@ -66,3 +82,7 @@ def test_block_workspace_sizes():
     hd64 = _lib.omq_block_shape(sh.T, sh.d, 64, 64, 64, sh.ffn, 1e-6, 1e4)   # head_dim must be 128
     assert _lib.omq_block_workspace_size(hd64, _cfg()) == 0
     assert _lib.omq_qlinear_workspace_size(256, 512, 512, _cfg()) > 512 * 512 * 4
+    # the softmax-quantized step carries two small per-row arrays more
+    ws8 = _lib.omq_block_workspace_size(s, _cfg(wbits=4, abits=4, group=0, let=1, pbits=8))
+    assert ws < ws8 < ws + 16 * sh.n_heads * sh.T * 4
+    assert _lib.omq_block_workspace_size(s, _cfg(wbits=4, abits=4, group=0, let=1, pbits=12)) == 0
