@@ -28,7 +28,7 @@ struct QState4 { float* h; int32_t* z; int32_t* imax; int32_t* imin; float* ga; 
 // Scratch (floats) of the fused weight-gradient + LWC backward of one [Cout, Cin] weight
 int64_t lwc_fused_scratch_elems(int64_t Cout, int64_t Cin) {
   const int64_t ntn = 2 * ((Cin + gemm_n_tile(Cin) - 1) / gemm_n_tile(Cin));   // row partials per row
-  return 2 * ((Cout + 31) / 32) * Cin + 3 * Cout * ntn + 64;
+  return 2 * ((Cout + 31) / 32) * Cin + 3 * Cout * ntn + 4 * Cout + 64;
 }
 
 bool lwc_fused_ok(int64_t Cin, int group, bool let_terms) {
@@ -277,7 +277,8 @@ omq_status lwc_bwd_dw(cudaStream_t st, int64_t T, const bf16* dY, const bf16* Xh
   la.dgl = dgl; la.dbl = dbl; la.dWt = nullptr; la.dr = dr; la.dBt = dBt; la.ds = ds; la.ddelta = ddelta;
   la.wbits = cfg.wbits; la.eps = cfg.h_eps;
   la.accumulate = cfg.accumulate; la.accumulate_sd = accumulate_sd; la.accumulate_dr = 0;
-  return lwc_bwd_fused_finish(st, la, lw.rowpart, ntn, lw.part_s, lw.part_d, P);
+  float* route = lw.rowpart + ((3 * Cout * ntn + 3) & ~int64_t(3));   // [Cout, 4], 16-byte aligned
+  return lwc_bwd_fused_finish(st, la, lw.rowpart, ntn, lw.part_s, lw.part_d, P, route);
 }
 
 // Auxiliary stream of a device: work off the step's critical chain (the LWC forward of the later

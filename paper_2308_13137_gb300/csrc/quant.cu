@@ -368,6 +368,7 @@ struct LwcBwdScratch {
   float* part_d;     // [nrt, Cin]
   float* rowpart;    // [3, Cout, ncw]: G_h, G_bm, dr partials of every 256-column warp
   float* sig;        // [2, Cout, ng]: clipping strengths when the caller has none saved
+  float* route;      // [Cout, 4]: max column, its ds term, min column, its ds term
   int64_t nrt, ncw, rows, ng;
 };
 
@@ -391,6 +392,7 @@ static LwcBwdScratch lwc_bwd_carve(void* base, int64_t Cout, int64_t Cin, int64_
   sc.part_d = take((size_t)sc.nrt * Cin);
   sc.rowpart = take((size_t)3 * Cout * sc.ncw);
   sc.sig = take((size_t)2 * Cout * sc.ng);
+  sc.route = take((size_t)4 * Cout);
   if (bytes) *bytes = off * 4 + 256;
   return sc;
 }
@@ -565,93 +567,87 @@ __global__ void __launch_bounds__(LWC_BWD_THREADS, 3) lwc_bwd_tile_kernel(LwcBwd
   }
 }
 
+// Per-row completion of the LWC backward, one warp per weight row: the warp sums the row's warp
+// partials (G_h, G_bm, dr); lane 0 forms dgamma, dbeta, dr and, for one group per row, the routing
+// of dW~ to the row's max / min element.  The routing's share of ds is written to route[o] =
+// (max column, value, min column, value) and added to the column partials by lwc_route_kernel.
+__global__ void __launch_bounds__(256) lwc_bwd_finalize_kernel(LwcBwdArgs a, LwcBwdScratch sc, float4* route) {
+  const int lane = threadIdx.x & 31;
+  const int64_t o = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (o >= a.Cout) return;
+  const bool perch = a.group == a.Cin;
+  float Gh = 0.f, Gbm = 0.f, drm = 0.f;
+  for (int64_t w = lane; w < sc.ncw; w += 32) {
+    if (perch) {
+      Gh += sc.rowpart[(0 * a.Cout + o) * sc.ncw + w];
+      Gbm += sc.rowpart[(1 * a.Cout + o) * sc.ncw + w];
+    }
+    if (a.dr) drm += sc.rowpart[(2 * a.Cout + o) * sc.ncw + w];
+  }
+  Gh = warp_sum(Gh);
+  Gbm = warp_sum(Gbm);
+  drm = warp_sum(drm);
+  if (lane != 0) return;
+  const float rr = a.r ? a.r[o] : 1.f;
+  if (perch) {
+    const float Q = (float)((1 << a.wbits) - 1);
+    const __nv_bfloat16* Wrow = a.W + o * a.Cin;
+    const int iM = a.imax[o], im = a.imin[o];
+    const float ga = lwc_sig(a.ga, a.gl, o, a.lwc), gb = lwc_sig(a.gb, a.bl, o, a.lwc);
+    const float WM = bf16_to_f(Wrow[iM]), Wm = bf16_to_f(Wrow[im]);
+    const float sM = a.s ? a.s[iM] : 1.f, sm = a.s ? a.s[im] : 1.f;
+    const float M = a.Mv ? a.Mv[o] : __fmul_rn(__fmul_rn(WM, sM), rr);
+    const float m = a.mv ? a.mv[o] : __fmul_rn(__fmul_rn(Wm, sm), rr);
+    const float hr = __fdiv_rn(__fsub_rn(__fmul_rn(ga, M), __fmul_rn(gb, m)), Q);
+    if (!(hr >= a.eps)) Gh = 0.f;
+    const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
+    if (a.lwc) {
+      const float dg = GaM * M * ga * (1.f - ga), db = Gbt * m * gb * (1.f - gb);
+      if (a.accumulate) { a.dgl[o] += dg; a.dbl[o] += db; } else { a.dgl[o] = dg; a.dbl[o] = db; }
+    }
+    const float rM = GaM * ga, rm = Gbt * gb;          // routing of dW~ to the max / min element
+    drm += rM * WM * sM + rm * Wm * sm;
+    if (a.ds) route[o] = make_float4((float)iM, rM * WM * rr, (float)im, rm * Wm * rr);
+    if (a.dWt) {
+      a.dWt[o * a.Cin + iM] += rM;
+      a.dWt[o * a.Cin + im] += rm;
+    }
+  }
+  if (a.dr) { if (a.accumulate_dr) a.dr[o] += drm; else a.dr[o] = drm; }
+}
+
 // Adds v to prow[col] for every lane's (col, v), col < 0 meaning none.  The lanes that share a
 // column are summed in lane order and the first of them adds the sum: a fixed order, no atomics.
 __device__ __forceinline__ void route_add(float* prow, int col, float v, int lane) {
-  float sum = 0.f;
-  int first = -1;
-#pragma unroll 1
-  for (int l = 0; l < 32; ++l) {
-    const int cl = __shfl_sync(0xffffffffu, col, l);
+  const unsigned m = __match_any_sync(0xffffffffu, col);           // lanes with this lane's column
+  const unsigned dup = __ballot_sync(0xffffffffu, __popc(m) > 1);  // lanes in groups of two or more
+  float sum = __popc(m) == 1 ? v : 0.f;
+  for (unsigned u = dup; u; u &= u - 1) {                         // warp-uniform, increasing lanes
+    const int l = __ffs(u) - 1;
     const float vl = __shfl_sync(0xffffffffu, v, l);
-    if (cl == col) {
-      sum += vl;
-      if (first < 0) first = l;
-    }
+    if ((m >> l) & 1u) sum += vl;
   }
-  if (col >= 0 && first == lane) prow[col] += sum;
+  if (col >= 0 && __ffs(m) - 1 == lane) prow[col] += sum;
 }
 
-// Per-row completion of the LWC backward, one warp per partial row p of the LET column sums
-// (weight rows [p R, p R + R)): the warp sums each row's warp partials (G_h, G_bm, dr), then lane i
-// completes row p R + 32 c + i of chunk c: dgamma, dbeta, dr and, for one group per row, the
-// routing of dW~ to the row's max / min element.  Its share of ds is added into partial row p
-// (chunk by chunk, maxima before minima, lanes in order) before the partial rows are reduced, so
-// ds does not depend on the order in which warps run.
-__global__ void __launch_bounds__(256) lwc_bwd_finalize_kernel(LwcBwdArgs a, LwcBwdScratch sc, float* part_s,
-                                                               int64_t R) {
+// The max / min routing of ds (Eq. 2's max / min path) added into the LET column partials: one warp
+// per partial row p (weight rows [p R, p R + R)), rows in chunks of 32 lanes, maxima before minima,
+// so that ds does not depend on the order in which warps run.
+__global__ void __launch_bounds__(256) lwc_route_kernel(const float4* __restrict__ route, int64_t Cout, int64_t R,
+                                                        float* __restrict__ part_s, int64_t Cin) {
   const int lane = threadIdx.x & 31;
   const int64_t pidx = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
-  const int64_t r_end = min((pidx + 1) * R, a.Cout);
-  if (pidx * R >= a.Cout) return;                     // whole warp
-  const bool perch = a.group == a.Cin;
-  const float Q = (float)((1 << a.wbits) - 1);
+  if (pidx * R >= Cout) return;                       // whole warp
+  const int64_t r_end = min((pidx + 1) * R, Cout);
+  float* prow = part_s + pidx * Cin;
   for (int64_t c0 = pidx * R; c0 < r_end; c0 += 32) {
-    float Gh = 0.f, Gbm = 0.f, drm = 0.f;             // of row c0 + lane
-#pragma unroll 1
-    for (int i = 0; i < 32 && c0 + i < r_end; ++i) {
-      const int64_t o = c0 + i;
-      float h0 = 0.f, h1 = 0.f, h2 = 0.f;
-      for (int64_t w = lane; w < sc.ncw; w += 32) {
-        if (perch) {
-          h0 += sc.rowpart[(0 * a.Cout + o) * sc.ncw + w];
-          h1 += sc.rowpart[(1 * a.Cout + o) * sc.ncw + w];
-        }
-        if (a.dr) h2 += sc.rowpart[(2 * a.Cout + o) * sc.ncw + w];
-      }
-      h0 = warp_sum(h0);
-      h1 = warp_sum(h1);
-      h2 = warp_sum(h2);
-      if (lane == i) { Gh = h0; Gbm = h1; drm = h2; }
-    }
     const int64_t o = c0 + lane;
-    const bool act = o < r_end;
-    int colM = -1, colm = -1;
-    float vM = 0.f, vm = 0.f;
-    if (act) {
-      const float rr = a.r ? a.r[o] : 1.f;
-      if (perch) {
-        const __nv_bfloat16* Wrow = a.W + o * a.Cin;
-        const int iM = a.imax[o], im = a.imin[o];
-        const float ga = lwc_sig(a.ga, a.gl, o, a.lwc), gb = lwc_sig(a.gb, a.bl, o, a.lwc);
-        const float WM = bf16_to_f(Wrow[iM]), Wm = bf16_to_f(Wrow[im]);
-        const float sM = a.s ? a.s[iM] : 1.f, sm = a.s ? a.s[im] : 1.f;
-        const float M = a.Mv ? a.Mv[o] : __fmul_rn(__fmul_rn(WM, sM), rr);
-        const float m = a.mv ? a.mv[o] : __fmul_rn(__fmul_rn(Wm, sm), rr);
-        const float hr = __fdiv_rn(__fsub_rn(__fmul_rn(ga, M), __fmul_rn(gb, m)), Q);
-        if (!(hr >= a.eps)) Gh = 0.f;
-        const float GaM = Gh / Q, Gbt = Gbm - Gh / Q;
-        if (a.lwc) {
-          const float dg = GaM * M * ga * (1.f - ga), db = Gbt * m * gb * (1.f - gb);
-          if (a.accumulate) { a.dgl[o] += dg; a.dbl[o] += db; } else { a.dgl[o] = dg; a.dbl[o] = db; }
-        }
-        const float rM = GaM * ga, rm = Gbt * gb;      // routing of dW~ to the max / min element
-        drm += rM * WM * sM + rm * Wm * sm;
-        if (a.ds) { colM = iM; colm = im; vM = rM * WM * rr; vm = rm * Wm * rr; }
-        if (a.dWt) {
-          a.dWt[o * a.Cin + iM] += rM;
-          a.dWt[o * a.Cin + im] += rm;
-        }
-      }
-      if (a.dr) { if (a.accumulate_dr) a.dr[o] += drm; else a.dr[o] = drm; }
-    }
-    if (perch && a.ds) {                               // warp-uniform
-      float* prow = part_s + pidx * a.Cin;
-      route_add(prow, colM, vM, lane);
-      __syncwarp();
-      route_add(prow, colm, vm, lane);
-      __syncwarp();
-    }
+    float4 e = make_float4(-1.f, 0.f, -1.f, 0.f);
+    if (o < r_end) e = route[o];
+    route_add(prow, (int)e.x, e.y, lane);
+    __syncwarp();
+    route_add(prow, (int)e.z, e.w, lane);
+    __syncwarp();
   }
 }
 
@@ -673,9 +669,14 @@ omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a0, void* scratch) 
   dim3 grid((unsigned)ncol, (unsigned)sc.nrt);
   lwc_bwd_tile_kernel<<<grid, LWC_BWD_THREADS, 0, st>>>(a, sc);
   OMQ_LAUNCH_CHECK();
-  // the finalize adds the max/min routing of ds into the partial rows, then they are reduced
+  // the finalize and the routing of ds into the partial rows, then the partial rows are reduced
   if (perch || a.dr) {
-    lwc_bwd_finalize_kernel<<<(unsigned)((sc.nrt + 7) / 8), 256, 0, st>>>(a, sc, sc.part_s, sc.rows);
+    lwc_bwd_finalize_kernel<<<(unsigned)((a.Cout + 7) / 8), 256, 0, st>>>(a, sc, reinterpret_cast<float4*>(sc.route));
+    OMQ_LAUNCH_CHECK();
+  }
+  if (perch && a.ds) {
+    lwc_route_kernel<<<(unsigned)((sc.nrt + 7) / 8), 256, 0, st>>>(reinterpret_cast<const float4*>(sc.route), a.Cout,
+                                                                    sc.rows, sc.part_s, a.Cin);
     OMQ_LAUNCH_CHECK();
   }
   if (a.ds) OMQ_TRY(omq_colsum_partials(st, sc.part_s, sc.nrt, a.Cin, a.ds, 1.f, a.accumulate_sd));
@@ -684,22 +685,28 @@ omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a0, void* scratch) 
 }
 
 omq_status lwc_bwd_fused_finish(cudaStream_t st, const LwcBwdArgs& a0, float* rowpart, int64_t ntn,
-                                float* part_s, const float* part_d, int64_t nparts) {
+                                float* part_s, const float* part_d, int64_t nparts, float* route) {
   LwcBwdArgs a = a0;
   const bool perch = a.group == a.Cin;
   OMQ_REQUIRE(a.ga && a.gb, OMQ_ERR_INVALID_ARG);
   const bool want_s = a.ds != nullptr, want_d = a.ddelta && a.dBt;
   OMQ_REQUIRE((!want_s || part_s) && (!want_d || part_d), OMQ_ERR_INVALID_ARG);
-  // the finalize adds the max/min routing of ds into the 32-row partials, then they are reduced
+  // the finalize and the routing of ds into the 32-row partials, then the partials are reduced
   if (perch || a.dr) {
     OMQ_REQUIRE(rowpart, OMQ_ERR_INVALID_ARG);
-    OMQ_REQUIRE(nparts == (a.Cout + 31) / 32, OMQ_ERR_INVALID_ARG);
+    OMQ_REQUIRE(!(perch && want_s) || (route && omq_aligned16(route) && nparts == (a.Cout + 31) / 32),
+                OMQ_ERR_INVALID_ARG);
     LwcBwdScratch sc{};
     sc.rowpart = rowpart;
     sc.ncw = ntn;
     sc.ng = a.Cin / a.group;
-    lwc_bwd_finalize_kernel<<<(unsigned)((nparts + 7) / 8), 256, 0, st>>>(a, sc, part_s, 32);
+    lwc_bwd_finalize_kernel<<<(unsigned)((a.Cout + 7) / 8), 256, 0, st>>>(a, sc, reinterpret_cast<float4*>(route));
     OMQ_LAUNCH_CHECK();
+    if (perch && want_s) {
+      lwc_route_kernel<<<(unsigned)((nparts + 7) / 8), 256, 0, st>>>(reinterpret_cast<const float4*>(route), a.Cout,
+                                                                      32, part_s, a.Cin);
+      OMQ_LAUNCH_CHECK();
+    }
   }
   if (want_s && want_d) {
     OMQ_TRY(omq_colsum_partials2(st, ColsumJob{part_s, nparts, a.Cin, a.ds, 1.f, a.accumulate_sd},

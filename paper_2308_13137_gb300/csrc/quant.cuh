@@ -36,10 +36,11 @@ size_t lwc_bwd_scratch_bytes(int64_t Cout, int64_t Cin);
 omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a, void* scratch);
 // Completion of the LWC backward whose per-element part ran inside the weight-gradient GEMM
 // epilogue: per-channel row partials [3, Cout, ntn] -> dgamma, dbeta, max/min routing, dr (a.dWq and
-// a.dWt unused); the routing's share of ds is added into the 32-row column partials part_s
-// [nparts = ceil(Cout / 32), Cin], which are then reduced to ds (and part_d to ddelta).
+// a.dWt unused); the routing's share of ds (staged in route [Cout, 4], 16-byte aligned) is added
+// into the 32-row column partials part_s [nparts = ceil(Cout / 32), Cin] in a fixed order, which
+// are then reduced to ds (and part_d to ddelta).
 omq_status lwc_bwd_fused_finish(cudaStream_t st, const LwcBwdArgs& a, float* rowpart, int64_t ntn,
-                                float* part_s, const float* part_d, int64_t nparts);
+                                float* part_s, const float* part_d, int64_t nparts, float* route);
 
 // ---- per-token activation quantizer Q_a with a fused producer ------------------------------
 enum ActProducer { AP_PLAIN = 0, AP_LET = 1, AP_RMS_LET = 2, AP_SWIGLU = 3 };
