@@ -484,6 +484,21 @@ def test_emulated_softmax_pv():
     assert torch.allclose(gS, ref, rtol=1e-12, atol=1e-14)
 
 
+def test_emulated_softmax_pv_integer_reference():
+    """R19's rounding point on a hand-evaluated row: scores with S log2(e) = (0.5, -0.5) and
+    V = (1, 0).  The integer reference is M = 1, so the bf16 operands are bf16(2^-0.5) =
+    0.70703125 and bf16(2^-1.5) = 0.353515625, and the value is 0.70703125 / (2^-0.5 + 2^-1.5)
+    = 0.666595...; subtracting the non-integer maximum 0.5 instead would give exactly 2/3."""
+    ln2 = math.log(2.0)
+    S = torch.tensor([[[0.0, float("-inf")], [0.5 * ln2, -0.5 * ln2]]], dtype=F64)
+    V = torch.tensor([[[1.0], [0.0]]], dtype=F64)
+    got = O.softmax_pv(S, V, "emulate")
+    want = 0.70703125 / (2 ** -0.5 + 2 ** -1.5)
+    assert abs(float(got[0, 1, 0]) - want) < 1e-12
+    assert abs(float(got[0, 1, 0]) - 2 / 3) > 5e-5
+    assert float(got[0, 0, 0]) == 1.0
+
+
 def test_rope_properties():
     g = torch.Generator().manual_seed(13)
     T, H, hd = 9, 2, 8
