@@ -200,6 +200,12 @@ omq_status omq_qlinear_bwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t 
                            float* dgamma, float* dbeta, float* ds, float* ddelta,
                            void* workspace, size_t ws_bytes, const omq_qcfg* cfg);
 size_t omq_qlinear_workspace_size(int64_t T, int64_t Cin, int64_t Cout, const omq_qcfg* cfg);
+/* Element counts of the omq_qlinear_saved arrays, in the struct's field order (w_hat, h_w, z_w,
+ * imax_w, imin_w, x_hat, h_a, z_a, imax_a, imin_a, b_tilde), written to sizes[0..10] (host array
+ * owned by the caller); the caller allocates each array with its field's element type (bf16, fp32
+ * or int32).  Pure host function.  OMQ_ERR_SHAPE for non-positive sizes or a group that does not
+ * divide Cin; the configuration checks of omq_check_cfg otherwise. */
+omq_status omq_qlinear_saved_sizes(int64_t T, int64_t Cin, int64_t Cout, const omq_qcfg* cfg, int64_t* sizes);
 
 /* ------------------------------------------------------------------------------------------
  * One LLaMA decoder block (RMSNorm -> RoPE causal attention -> RMSNorm -> SwiGLU FFN), the

@@ -94,6 +94,7 @@ _SIGS = {
     "omq_attention_fwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P]),
     "omq_attention_bwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P, I64, P, P, I64, P, P, I64,
                                 P]),
+    "omq_qlinear_saved_sizes": (I32, [I64, I64, I64, P, P]),
     "omq_attention_pq_fwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, I32, F32, P, P]),
     "omq_attention_pq_bwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, P, I64, P, I64, P, P, I64, I32, P, P,
                                    P]),
@@ -252,6 +253,12 @@ def omq_attention_bwd(T, n_heads, n_kv, Q, ldq, K, V, ldkv, O, ldo, lse, dO, ldd
     check("omq_attention_bwd", lib().omq_attention_bwd(
         stream_handle(stream), T, n_heads, n_kv, ptr(Q), ldq, ptr(K), ptr(V), ldkv, ptr(O), ldo, ptr(lse), ptr(dO),
         lddo, ptr(D), ptr(dQ), ldg, ptr(dK), ptr(dV), ldgkv, ptr(dev_status)))
+
+
+def omq_qlinear_saved_sizes(T, Cin, Cout, cfg):
+    sizes = (c_int64 * 11)()
+    check("omq_qlinear_saved_sizes", lib().omq_qlinear_saved_sizes(T, Cin, Cout, ctypes.byref(cfg), sizes))
+    return list(sizes)
 
 
 def omq_attention_pq_fwd(T, n_heads, n_kv, Q, ldq, K, V, ldkv, O, ldo, lse, pbits, h_eps, pq_rows,

@@ -670,6 +670,18 @@ omq_status omq_qlinear_fwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t 
                  nullptr, cfg->dev_status);
 }
 
+omq_status omq_qlinear_saved_sizes(int64_t T, int64_t Cin, int64_t Cout, const omq_qcfg* cfg, int64_t* sizes) {
+  OMQ_TRY(omq_check_cfg(cfg));
+  OMQ_REQUIRE(sizes, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(T > 0 && Cin > 0 && Cout > 0, OMQ_ERR_SHAPE);
+  const int64_t g = cfg->group == 0 ? Cin : cfg->group;
+  OMQ_REQUIRE(Cin % g == 0, OMQ_ERR_SHAPE);
+  const int64_t ng = Cout * (Cin / g);
+  const int64_t n[11] = {Cout * Cin, ng, ng, ng, ng, T * Cin, T, T, T, T, Cout};
+  for (int i = 0; i < 11; ++i) sizes[i] = n[i];
+  return OMQ_OK;
+}
+
 size_t omq_qlinear_workspace_size(int64_t T, int64_t Cin, int64_t Cout, const omq_qcfg* cfg) {
   (void)cfg;
   Carve c{nullptr, 0};

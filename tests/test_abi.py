@@ -72,6 +72,16 @@ def test_softmax_quant_argument_errors():
                                   None, None) == 1             # the row records are required
 
 
+def test_qlinear_saved_sizes():
+    """Element counts of the single linear's saved arrays, in the struct's field order."""
+    n = _lib.omq_qlinear_saved_sizes(256, 512, 384, _cfg(group=128))
+    ng = 384 * 4
+    assert n == [384 * 512, ng, ng, ng, ng, 256 * 512, 256, 256, 256, 256, 384]
+    assert _lib.omq_qlinear_saved_sizes(256, 512, 384, _cfg(group=0))[1] == 384
+    with pytest.raises(_lib.OmqError):
+        _lib.omq_qlinear_saved_sizes(256, 512, 384, _cfg(group=96))       # 96 does not divide 512
+
+
 def test_block_workspace_sizes():
     sh = I.SHAPES["llama7b_w4a4"]
     s = _lib.omq_block_shape(sh.T, sh.d, sh.n_heads, sh.n_kv, sh.head_dim, sh.ffn, sh.rms_eps, sh.rope_theta)
