@@ -52,6 +52,26 @@ def _dist():
     return ws, rank, local
 
 
+def replica_seeds(rank: int):
+    """Seeds of rank `rank`'s block replica: every rank calibrates its own block (distinct weights,
+    same shapes), so the ranks share no data and exchange nothing but the timing."""
+    return {"weights": 1 + rank, "theta": 2 + rank}
+
+
+def max_over_ranks(value: float, ws: int, device) -> float:
+    """The largest of every rank's `value` (the slowest rank's time); the value itself alone."""
+    import torch
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    if ws > 1:
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(ws: int, tokens_per_step: int, steps: int, seconds: float) -> float:
+    """Whole-job tokens per second: all ranks' tokens over the slowest rank's time (weak scaling)."""
+    return ws * tokens_per_step * steps / seconds
+
+
 # ------------------------------------------------------------------------------------------------
 # clocks during the timed region
 # ------------------------------------------------------------------------------------------------
@@ -246,10 +266,11 @@ def run_ours(args, shape):
     _lib.lib()
 
     # every rank calibrates its own block: distinct weight seeds, same shapes
-    W = I.make_block_weights(shape, seed=1 + rank)
+    seeds = replica_seeds(rank)
+    W = I.make_block_weights(shape, seed=seeds["weights"])
     n_samples = 4
-    xs = [I.make_block_input(shape, sample=i, weight_seed=1 + rank) for i in range(n_samples)]
-    th = I.make_block_theta(shape, W, xs[0], seed=2 + rank)
+    xs = [I.make_block_input(shape, sample=i, weight_seed=seeds["weights"]) for i in range(n_samples)]
+    th = I.make_block_theta(shape, W, xs[0], seed=seeds["theta"])
     st = BlockState(shape, W, th, pbits=args.pbits)
     xd = [torch.from_numpy(x).cuda() for x in xs]
     yfp = [torch.empty_like(v) for v in xd]
@@ -308,12 +329,9 @@ def run_ours(args, shape):
     launches = int(round(launches_per_step * args.steps))
     gemm_ms, gemm_flops, gemm_launches = (gemm_ms * args.steps / n_prof, gemm_flops * args.steps / n_prof,
                                           gemm_launches * args.steps / n_prof)
-    t = torch.tensor([ms], device="cuda")
-    if ws > 1:
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-    ms_max = float(t.item())
+    ms_max = max_over_ranks(ms, ws, "cuda")
     ms_step = ms_max / args.steps
-    value = ws * shape.T * args.steps / (ms_max / 1e3)
+    value = job_throughput(ws, shape.T, args.steps, ms_max / 1e3)
 
     # ---- end to end through the public API: host buffers in, loss out ----------------------------
     # each step's inputs go host -> device on a copy stream into one of two device buffers while the
@@ -343,6 +361,7 @@ def run_ours(args, shape):
         st.step_adamw_graph(xin[b], yin[b])
         consumed[b].record(main_stream)
     torch.cuda.synchronize()
+    barrier()
     t0 = time.perf_counter()
     enqueue_copy(0)
     for i in range(e2e_steps):
@@ -355,8 +374,8 @@ def run_ours(args, shape):
         loss_h.copy_(st.loss, non_blocking=True)
         main_stream.synchronize()
         _ = float(loss_h[0])
-    e2e_s = time.perf_counter() - t0
-    e2e_value = ws * shape.T * e2e_steps / e2e_s
+    e2e_s = max_over_ranks(time.perf_counter() - t0, ws, "cuda")
+    e2e_value = job_throughput(ws, shape.T, e2e_steps, e2e_s)
 
     peaks = _peaks()
     gemm_flops_step = gemm_flops / args.steps
