@@ -21,6 +21,19 @@ def test_exports_every_declared_function():
     assert _lib.omq_status_string(3).startswith("misaligned")
 
 
+def test_every_exported_function_is_declared():
+    """The reverse direction: no omq_ symbol leaves the library undocumented by the header."""
+    import shutil
+    import subprocess
+    if not shutil.which("nm"):
+        pytest.skip("nm not available")
+    out = subprocess.run(["nm", "-D", "--defined-only", _lib.LIB_PATH], capture_output=True, text=True,
+                         check=True).stdout
+    exported = {f[2] for f in (line.split() for line in out.splitlines())
+                if len(f) == 3 and f[1] == "T" and f[2].startswith("omq_")}
+    assert exported and exported <= set(_lib.header_functions()), sorted(exported - set(_lib.header_functions()))
+
+
 def _cfg(**kw):
     base = dict(wbits=4, abits=16, group=128, let=0, h_eps=1e-5, accumulate=0, dev_status=None, pbits=0)
     base.update(kw)
