@@ -43,7 +43,10 @@ notes of the repository):
  R13 precision policy ("emulate" mode): each operand of every matrix product,
      forward and backward, is rounded to bf16 (nearest, ties to even) right
      before the product; accumulation is exact (fp64 here).  "exact" mode skips
-     the rounding.
+     the rounding.  Nothing else is rounded: every quantizer decision (max/min and
+     their first index, the floor of h, the zero point, every code) is taken in
+     float64 on float64 values, as Eq. 2 states it, and the softmax enters P V
+     normalised (Eq. 5).
  R14 LLaMA blocks have no linear biases (B = 0); the [v, out] LET pair moves
      its transform into v_proj: W_v' = diag(1/s_o) W_v diag(s1),
      b_v' = (W_v delta1 - delta_o) / s_o, and the out_proj input is P V'
@@ -68,20 +71,10 @@ notes of the repository):
      1e-2 for the LET vectors): betas 0.9 / 0.999, eps 1e-8, bias-corrected moments, decoupled
      weight decay; one update after every calibration sample (batch size 1).  Algorithm 1's
      LET statistics (R16) are taken on the fp inputs of each block before they are advanced.
- R15 where floating point decides an integer (a code, a zero point, a max/min
-     index, the floor of h) the decision is taken in the precision of the
-     kernels, IEEE single precision with one rounding per product, difference and
-     quotient, the division by h formed as a product with the correctly rounded
-     reciprocal of h; the clipping strengths entering it are the single-precision sigmoid
-     of `sigmoid_fp32`.  Everything else stays float64.  ("emulate" mode; "exact"
-     mode decides in float64.)
- R19 ("emulate" mode) the unquantized softmax enters the P V product unnormalised: bf16 of
-     2^(S log2(e) - M) with M an integer not below the row maximum of S log2(e) (the rounding is the
-     same for every such M), the product divided by the unrounded row sum afterwards.
  R20 softmax-output quantization (the ablation of Table A7, off by default): the causal softmax
      output is quantized per query row with the MinMax Q_a (gamma = beta = 1, the floor of h
-     included) over the visible keys j <= t only; the masked entries stay 0.  Its decisions are
-     taken on P in single precision (R15) and its backward is the STE of R7.
+     included) over the visible keys j <= t only; the masked entries stay 0.  Its backward is the
+     STE of R7.
 """
 from __future__ import annotations
 
@@ -97,9 +90,10 @@ __all__ = [
     "rne", "to_bf16", "sigmoid", "quant_fwd", "quant_bwd", "quant_ste", "codes_from_scale",
     "lwc_fakequant_fwd", "lwc_fakequant_bwd", "act_quant_per_token", "act_quant_per_token_bwd",
     "let_apply", "block_loss", "qlinear_step", "BlockCfg", "block_forward", "block_step",
-    "rmsnorm", "rope", "silu", "FrozenTape", "use_tape", "block_fp_forward", "sigmoid_fp32",
+    "rmsnorm", "rope", "silu", "FrozenTape", "use_tape", "block_fp_forward",
     "THETA_NAMES_LWC", "THETA_NAMES_LET", "let_init", "pack_codes", "unpack_codes", "block_fold_pack",
-    "folded_forward", "adamw_step", "calibrate_blocks", "softmax_quant", "softmax_pv",
+    "folded_forward", "adamw_step", "calibrate_blocks", "softmax_quant",
+    "stage_attn_in", "stage_attention", "stage_attn_out", "stage_ffn_in", "stage_ffn_out",
 ]
 
 
@@ -125,30 +119,6 @@ def sigmoid(t: torch.Tensor) -> torch.Tensor:
     return 1.0 / (1.0 + torch.exp(-t))
 
 
-_LOG2E32 = 1.44269502162933349609375        # float32 nearest to log2(e)
-_LN2_HI = 0.693145751953125                 # 15-bit head of ln 2: n * head is exact
-_LN2_LO = 1.428606765330187e-06             # float32 tail, head + tail = ln 2 to 5e-14
-_EXP_TAYLOR = [1.98412701138295233249664e-04, 1.38888892251998186111450e-03, 8.33333376795053482055664e-03,
-               4.16666679084300994873047e-02, 1.66666671633720397949219e-01, 0.5, 1.0, 1.0]   # 1/7!, ..., 1/0!
-
-
-def sigmoid_fp32(t: torch.Tensor) -> torch.Tensor:
-    """sigmoid(t) as the kernels evaluate it in single precision (R15), one rounding per
-    operation: exp(-t) by Cody-Waite reduction -t = n ln2 + r, the degree-7 Taylor polynomial of
-    exp(r) in Horner form and an exact scaling by 2^n, then 1 / (1 + exp(-t)); |t| clamped to 80.
-    Returns float32."""
-    f32 = torch.float32
-    x = -torch.clamp(torch.as_tensor(t).to(f32), -80.0, 80.0)
-    n = torch.round(x * _LOG2E32)
-    r = (x - n * _LN2_HI) - n * _LN2_LO
-    p = torch.full_like(r, _EXP_TAYLOR[0])
-    for c in _EXP_TAYLOR[1:]:
-        p = p * r + c
-    two_n = ((n.to(torch.int32) + 127) << 23).view(f32)       # 2^n, exact
-    e = p * two_n
-    return 1.0 / (1.0 + e)
-
-
 def _first_argmax(w: torch.Tensor) -> torch.Tensor:
     """Index of the first maximum along the last axis (R7)."""
     M = w.max(dim=-1, keepdim=True).values
@@ -166,59 +136,25 @@ def _first_argmin(w: torch.Tensor) -> torch.Tensor:
 # Eq. 2, explicit forward and STE backward of one quantizer over groups on the last axis
 # ----------------------------------------------------------------------------------------------
 
-def _decide_fp32(w: torch.Tensor, a, b, Q: float, eps: float, a32=None, b32=None):
-    """The integer decisions of Eq. 2 taken in IEEE single precision (R15).
-
-    Inputs are rounded to fp32 and every product, difference and quotient is rounded to fp32:
-    h = (a*M - b*m)/Q, r = 1/h, u = (b*m)*r, x = w*r; a32, b32 (default: a, b rounded) are the
-    single-precision clipping strengths.  Returns the first argmax/argmin of the fp32 group,
-    the floor flag and h, u, x as fp32 values."""
-    f32 = torch.float32
-    w32 = w.detach().to(f32)
-    a32 = torch.as_tensor(a).detach().to(f32) if a32 is None else torch.as_tensor(a32).to(f32)
-    b32 = torch.as_tensor(b).detach().to(f32) if b32 is None else torch.as_tensor(b32).to(f32)
-    imax = _first_argmax(w32)
-    imin = _first_argmin(w32)
-    M32 = torch.gather(w32, -1, imax[..., None])[..., 0]
-    m32 = torch.gather(w32, -1, imin[..., None])[..., 0]
-    aM = a32 * M32
-    bm = b32 * m32
-    hr = (aM - bm) / Q
-    floored = hr < eps
-    h32 = torch.where(floored, torch.full_like(hr, eps), hr)
-    rh32 = 1.0 / h32                       # correctly rounded reciprocal
-    u32 = bm * rh32
-    x32 = w32 * rh32[..., None]
-    return imax, imin, floored, h32, u32, x32
-
-
-def quant_fwd(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5, decide: str = "fp64",
-              a32=None, b32=None) -> Dict[str, torch.Tensor]:
+def quant_fwd(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5) -> Dict[str, torch.Tensor]:
     """Eq. 2 over groups laid out on the last axis of `w` (shape [..., g]).
 
     a, b are the clipping strengths gamma, beta (tensors of shape [...] or floats; 1.0 gives
-    MinMax, the special case stated after Eq. 2).  decide = "fp64" takes every decision in
-    float64; "fp32" takes max/min, h, z and the codes in IEEE single precision (R15).
+    MinMax, the special case stated after Eq. 2).  Every decision is taken in float64.
     Returns every intermediate."""
     w = w.to(F64)
     Q = float(2 ** nbits - 1)
     a = torch.as_tensor(a, dtype=F64)
     b = torch.as_tensor(b, dtype=F64)
-    if decide == "fp32":
-        imax, imin, floored, h32, u32, x32 = _decide_fp32(w, a, b, Q, eps, a32, b32)
-        M = torch.gather(w, -1, imax[..., None])[..., 0]
-        m = torch.gather(w, -1, imin[..., None])[..., 0]
-        h, u, x = h32.to(F64), u32.to(F64), x32.to(F64)
-    else:
-        imax = _first_argmax(w)
-        imin = _first_argmin(w)
-        M = torch.gather(w, -1, imax[..., None])[..., 0]
-        m = torch.gather(w, -1, imin[..., None])[..., 0]
-        h_raw = (a * M - b * m) / Q
-        floored = h_raw < eps                              # R3
-        h = torch.where(floored, torch.full_like(h_raw, eps), h_raw)
-        u = b * m / h
-        x = w / h[..., None]
+    imax = _first_argmax(w)
+    imin = _first_argmin(w)
+    M = torch.gather(w, -1, imax[..., None])[..., 0]
+    m = torch.gather(w, -1, imin[..., None])[..., 0]
+    h_raw = (a * M - b * m) / Q
+    floored = h_raw < eps                                  # R3
+    h = torch.where(floored, torch.full_like(h_raw, eps), h_raw)
+    u = b * m / h
+    x = w / h[..., None]
     z = -rne(u)
     c = rne(x) + z[..., None]
     q = torch.clamp(c, 0.0, Q)
@@ -305,14 +241,11 @@ class use_tape:
         _TAPE = self.prev
 
 
-def quant_ste(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5, decide: str = "fp64",
-              w_dec: Optional[torch.Tensor] = None, a32=None, b32=None) -> torch.Tensor:
+def quant_ste(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5) -> torch.Tensor:
     """Eq. 2 fake quantization as an autograd graph whose gradient is the STE of R7.
 
     Groups on the last axis; a, b broadcast against w[..., 0] (tensors that may require
-    grad, or floats for Q_a).  With decide = "fp32" the max/min, the floor, the value of h and
-    every round() are taken in IEEE single precision from `w_dec` (default: w rounded to
-    fp32), as the kernels take them (R15); the gradient is the same STE."""
+    grad, or floats for Q_a)."""
     Q = float(2 ** nbits - 1)
     tape = _TAPE
     if tape is not None and tape.mode == "replay":
@@ -326,22 +259,6 @@ def quant_ste(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5, decide: str 
         z = -(u + r["ru"])
         c = w / h[..., None] + r["rx"] + z[..., None]
         q = torch.where(r["inr"], c, torch.where(r["below"], torch.zeros_like(c), torch.full_like(c, Q)))
-        return (q - z[..., None]) * h[..., None]
-    if decide == "fp32":
-        assert tape is None, "the frozen-offset surrogate is defined for float64 decisions"
-        with torch.no_grad():
-            imax, imin, floored, h32, u32, x32 = _decide_fp32(w if w_dec is None else w_dec, a, b, Q, eps,
-                                                              a32, b32)
-        M = torch.gather(w, -1, imax[..., None])[..., 0]
-        m = torch.gather(w, -1, imin[..., None])[..., 0]
-        h_raw = (a * M - b * m) / Q
-        h = torch.where(floored, torch.full_like(h_raw, eps), h_raw)     # R3: no gradient when floored
-        h = h + (h32.to(F64) - h).detach()                                 # value of the fp32 step
-        u = b * m / h
-        z = -(u + (rne(u32.to(F64)) - u).detach())
-        x = w / h[..., None]
-        c = x + (rne(x32.to(F64)) - x).detach() + z[..., None]
-        q = torch.clamp(c, 0.0, Q)
         return (q - z[..., None]) * h[..., None]
     imax = _first_argmax(w.detach())
     imin = _first_argmin(w.detach())
@@ -387,39 +304,23 @@ def _groups(W: torch.Tensor, group: int) -> torch.Tensor:
     return W.reshape(cout, cin // g, g)                    # R6
 
 
-def _wt_fp32(W, s, row_scale):
-    """W~ = fl32(fl32(W * s) * r), the kernels' single-precision quantizer input (R15)."""
-    wt = W.to(torch.float32)
-    if s is not None:
-        wt = wt * s.to(torch.float32)[None, :]
-    if row_scale is not None:
-        wt = wt * row_scale.to(torch.float32)[:, None]
-    return wt
-
-
 def lwc_fakequant_fwd(W, gamma_logit, beta_logit, nbits: int, group: int,
                       s: Optional[torch.Tensor] = None, eps: float = 1e-5,
-                      row_scale: Optional[torch.Tensor] = None, decide: str = "fp64") -> Dict[str, torch.Tensor]:
+                      row_scale: Optional[torch.Tensor] = None) -> Dict[str, torch.Tensor]:
     """LWC of Eq. 2 on W~ = s (.) W (Eq. 3) for W [Cout, Cin].
 
     row_scale (optional, [Cout]) multiplies each output row before quantization; it is how
     the [v, out] LET pair divides v_proj's rows by s_o (R14).  Returns h, z [Cout, ngroups],
     the first argmax/argmin inside each group (as column indices into Cin), integer codes,
-    W_hat [Cout, Cin] and the quantizer input Wt.  decide = "fp32" forms W~ and takes the
-    quantizer's decisions in single precision (R15)."""
+    W_hat [Cout, Cin] and the quantizer input Wt."""
     W = W.to(F64)
-    if decide == "fp32":
-        Wt = _wt_fp32(W, s, row_scale).to(F64)
-    else:
-        Wt = W if s is None else W * s.to(F64)[None, :]
-        if row_scale is not None:
-            Wt = Wt * row_scale.to(F64)[:, None]
+    Wt = W if s is None else W * s.to(F64)[None, :]
+    if row_scale is not None:
+        Wt = Wt * row_scale.to(F64)[:, None]
     G = _groups(Wt, group)
     a = sigmoid(gamma_logit.to(F64))
     b = sigmoid(beta_logit.to(F64))
-    a32 = sigmoid_fp32(gamma_logit) if decide == "fp32" else None
-    b32 = sigmoid_fp32(beta_logit) if decide == "fp32" else None
-    st = quant_fwd(G, a, b, nbits, eps, decide, a32, b32)
+    st = quant_fwd(G, a, b, nbits, eps)
     gsz = G.shape[-1]
     base = torch.arange(G.shape[1], dtype=torch.int64)[None, :] * gsz
     return dict(st=st, Wt=Wt, h=st["h"], z=st["z"], argmax=st["imax"] + base, argmin=st["imin"] + base,
@@ -447,19 +348,15 @@ def lwc_fakequant_bwd(fwd: Dict[str, torch.Tensor], W, dWhat, s: Optional[torch.
 
 
 def act_quant_per_token(X, nbits: int, s: Optional[torch.Tensor] = None,
-                        delta: Optional[torch.Tensor] = None, eps: float = 1e-5,
-                        decide: str = "fp64") -> Dict[str, torch.Tensor]:
+                        delta: Optional[torch.Tensor] = None, eps: float = 1e-5) -> Dict[str, torch.Tensor]:
     """LET on activations (Eq. 3: X~ = (X - delta)/s) followed by Q_a, the per-token MinMax
-    quantizer (gamma = beta = 1 in Eq. 2; one group per token row).  decide = "fp32" forms X~
-    and takes the quantizer's decisions in single precision (R15)."""
-    dt = torch.float32 if decide == "fp32" else F64
-    Xt = X.to(dt)
+    quantizer (gamma = beta = 1 in Eq. 2; one group per token row)."""
+    Xt = X.to(F64)
     if delta is not None:
-        Xt = Xt - delta.to(dt)[None, :]
+        Xt = Xt - delta.to(F64)[None, :]
     if s is not None:
-        Xt = Xt / s.to(dt)[None, :]
-    Xt = Xt.to(F64)
-    st = quant_fwd(Xt, 1.0, 1.0, nbits, eps, decide)
+        Xt = Xt / s.to(F64)[None, :]
+    st = quant_fwd(Xt, 1.0, 1.0, nbits, eps)
     return dict(st=st, Xt=Xt, Xq=st["what"], codes=st["q"].to(torch.int64), h=st["h"], z=st["z"],
                 argmax=st["imax"], argmin=st["imin"])
 
@@ -548,19 +445,10 @@ def qlinear_step(X, W, B, gamma_logit, beta_logit, Yfp, wbits: int, group: int, 
     Bt = (torch.zeros(W.shape[0], dtype=F64) if B is None else B.to(F64))
     if sv is not None:
         Bt = Bt + W @ dv
-    decide = "fp32" if mode == "emulate" else "fp64"
-    with torch.no_grad():
-        xd = X.to(torch.float32)
-        if sv is not None:
-            xd = (xd - dv.detach().to(torch.float32)) / sv.detach().to(torch.float32)
-    Xh = Xt if abits >= 16 else quant_ste(Xt, 1.0, 1.0, abits, eps, decide, xd)
+    Xh = Xt if abits >= 16 else quant_ste(Xt, 1.0, 1.0, abits, eps)
     cout, cin = W.shape
     gsz = cin if group == 0 else group
-    wd = _dec32(W, sv).reshape(cout, cin // gsz, gsz)
-    a32 = sigmoid_fp32(gl.detach()) if decide == "fp32" else None
-    b32 = sigmoid_fp32(bl.detach()) if decide == "fp32" else None
-    Wh = quant_ste(Wt.reshape(cout, cin // gsz, gsz), sigmoid(gl), sigmoid(bl), wbits, eps, decide,
-                   wd, a32, b32).reshape(cout, cin)
+    Wh = quant_ste(Wt.reshape(cout, cin // gsz, gsz), sigmoid(gl), sigmoid(bl), wbits, eps).reshape(cout, cin)
     Y = _mm(Xh, Wh, mode) + Bt
     loss, _ = block_loss(Y, Yfp)
     grads = torch.autograd.grad(loss, leaves)
@@ -629,31 +517,24 @@ def _expand_kv(vec, cfg: BlockCfg):
     return vec.reshape(cfg.n_kv, 1, cfg.head_dim).expand(cfg.n_kv, rep, cfg.head_dim).reshape(-1)
 
 
-def _decide(cfg: BlockCfg) -> str:
-    return "fp32" if cfg.mode == "emulate" else "fp64"
-
-
-def _qw(Wt, gl, bl, cfg: BlockCfg, w_dec=None):
-    """LWC fake quantization of a (LET-scaled) weight; w_dec is its fp32 quantizer input."""
+def _qw(Wt, gl, bl, cfg: BlockCfg):
+    """LWC fake quantization (Eq. 2) of a (LET-scaled) weight [Cout, Cin]."""
     if cfg.wbits >= 16:
         return Wt
     cout, cin = Wt.shape
     gsz = cin if cfg.group == 0 else cfg.group
-    dec = None if w_dec is None else w_dec.reshape(cout, cin // gsz, gsz)
-    fp32 = _decide(cfg) == "fp32"
-    a32 = sigmoid_fp32(gl.detach()) if fp32 else None
-    b32 = sigmoid_fp32(bl.detach()) if fp32 else None
     return quant_ste(Wt.reshape(cout, cin // gsz, gsz), sigmoid(gl), sigmoid(bl),
-                     cfg.wbits, cfg.h_eps, _decide(cfg), dec, a32, b32).reshape(cout, cin)
+                     cfg.wbits, cfg.h_eps).reshape(cout, cin)
 
 
 def _qa(X, cfg: BlockCfg):
+    """Q_a, the per-token MinMax quantizer (R8, R12)."""
     if cfg.abits >= 16:
         return X
-    return quant_ste(X, 1.0, 1.0, cfg.abits, cfg.h_eps, _decide(cfg))
+    return quant_ste(X, 1.0, 1.0, cfg.abits, cfg.h_eps)
 
 
-def softmax_quant(P, nbits: int, eps: float = 1e-5, decide: str = "fp64"):
+def softmax_quant(P, nbits: int, eps: float = 1e-5):
     """Q_p (R20): the causal softmax output P [..., T, T] quantized per query row with the
     MinMax quantizer of Eq. 2 (gamma = beta = 1) over the row's visible keys j <= t, as an
     autograd graph with the STE of R7 (h not detached; max / min pass their gradient to the first
@@ -667,116 +548,92 @@ def softmax_quant(P, nbits: int, eps: float = 1e-5, decide: str = "fp64"):
     # range at an index after every visible key, so max, min and their first indices are unchanged
     diag = torch.diagonal(P, dim1=-2, dim2=-1)[..., :, None]
     Pf = torch.where(causal, P, diag.detach().expand_as(P))
-    return quant_ste(Pf, 1.0, 1.0, nbits, eps, decide).masked_fill(~causal, 0.0)
-
-
-def _qp(P, cfg: BlockCfg):
-    return softmax_quant(P, cfg.pbits, cfg.h_eps, _decide(cfg))
-
-
-LOG2E = 1.0 / math.log(2.0)
-
-
-def softmax_pv(S, Vh, mode: str):
-    """softmax(S) V per head, S [..., T, T] with -inf at masked keys, Vh [..., T, hd] (Sec. 3.3; the
-    softmax output is not quantized, R12).  "emulate" (R19): the value is
-    (bf16(2^(S log2(e) - M)) bf16(V)) / l, with M the row maximum of S log2(e) rounded up to an
-    integer and l the unrounded row sum of 2^(S log2(e) - M): the probabilities enter the product
-    unnormalised and the row sum divides it afterwards.  Rounding to bf16 commutes with scaling by
-    a power of two, so any integer M gives the same value.  The gradient is that of softmax(S) V
-    under R13."""
-    O = _mm(torch.softmax(S, dim=-1), Vh.transpose(-1, -2), mode)
-    if mode != "emulate":
-        return O
-    with torch.no_grad():
-        t = S * LOG2E
-        E = torch.exp2(t - torch.ceil(t.amax(dim=-1, keepdim=True)))
-        On = (to_bf16(E) @ to_bf16(Vh)) / E.sum(dim=-1, keepdim=True)
-    return O + (On - O).detach()
+    return quant_ste(Pf, 1.0, 1.0, nbits, eps).masked_fill(~causal, 0.0)
 
 
 def _attn_pv(S, Vh, cfg: BlockCfg):
-    """The attention output from the masked scores: softmax(S) V (R19), or with the softmax
-    output quantized (R20) the quantized probabilities, rounded to bf16 (R13), times V."""
-    if cfg.pbits >= 16:
-        return softmax_pv(S, Vh, cfg.mode)
-    return _mm(_qp(torch.softmax(S, dim=-1), cfg), Vh.transpose(-1, -2), cfg.mode)
+    """The attention output from the masked scores: softmax(S) (Eq. 5; quantized per query row
+    when the ablation of R20 is on) times V, both operands rounded to bf16 in emulate mode (R13)."""
+    P = torch.softmax(S, dim=-1)
+    if cfg.pbits < 16:
+        P = softmax_quant(P, cfg.pbits, cfg.h_eps)
+    return _mm(P, Vh.transpose(-1, -2), cfg.mode)
 
 
-def _dec32(W, s=None, r=None):
-    """fp32 quantizer input of a scaled weight, formed as the kernels form it (R15)."""
-    with torch.no_grad():
-        return _wt_fp32(W, None if s is None else s.detach(), None if r is None else r.detach())
+# The block forward in five stages; each stage takes its inputs as tensors, so a test can start
+# any stage from another implementation's values of its input (stage-wise comparison).
 
-
-def block_forward(x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], cfg: BlockCfg,
-                  keep: Optional[Dict[str, torch.Tensor]] = None):
-    """Forward of the LET'd, LWC-quantized block (Algorithm 1, LET then
-    Quantization_with_LWC then the block on x_q).  `th` holds the learnable parameters
-    (gamma_*/beta_* logits per linear; s1, d1, so, do, sa, s2, d2 when LET is on).
-    With wbits = abits = 16 and LET off this is the full-precision block F(W, X)."""
+def stage_attn_in(x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], cfg: BlockCfg):
+    """RMSNorm, the [ln1, (q, k, v)] LET pair (Eq. 3) with the [v, out] pair moved into v_proj
+    (R14), Q_a and the three quantized projections (Eq. 4): q, k, v before RoPE, LET biases
+    included."""
     mode = cfg.mode
-    H, Hkv, hd = cfg.n_heads, cfg.n_kv, cfg.head_dim
-    T = x.shape[0]
-    wq, wk, wv, wo = Wd["wq"], Wd["wk"], Wd["wv"], Wd["wo"]
-    wg, wu, wdn = Wd["wg"], Wd["wu"], Wd["wd"]
-    let = cfg.let
-
-    # --- attention half -------------------------------------------------------------------------
+    wq, wk, wv = Wd["wq"], Wd["wk"], Wd["wv"]
     a = rmsnorm(x, cfg.rms_eps)
-    if let:                                               # [ln1, (q, k, v)] pair, Eq. 3
-        s1, d1 = th["s1"], th["d1"]
-        so, do_, sa = th["so"], th["do"], th["sa"]
+    if cfg.let:
+        s1, d1, so, do_ = th["s1"], th["d1"], th["so"], th["do"]
         at = (a - d1) / s1
         wq_t, wk_t = wq * s1, wk * s1
-        wv_t = (wv * s1) / so[:, None]                    # [v, out] pair moved into v_proj (R14)
+        wv_t = (wv * s1) / so[:, None]
         bq, bk = wq @ d1, wk @ d1
         bv = (wv @ d1 - do_) / so
     else:
         at, wq_t, wk_t, wv_t = a, wq, wk, wv
-        bq = bk = bv = None
     ah = _qa(at, cfg)
-    if let:
-        with torch.no_grad():
-            r_o = (1.0 / so.detach().to(torch.float32)).to(F64)
-        dq_, dk_, dv_ = _dec32(wq, s1), _dec32(wk, s1), _dec32(wv, s1, r_o)
-    else:
-        dq_ = dk_ = dv_ = None
-    q = _mm(ah, _qw(wq_t, th.get("gamma_q"), th.get("beta_q"), cfg, dq_), mode)
-    k = _mm(ah, _qw(wk_t, th.get("gamma_k"), th.get("beta_k"), cfg, dk_), mode)
-    v = _mm(ah, _qw(wv_t, th.get("gamma_v"), th.get("beta_v"), cfg, dv_), mode)
-    if let:
+    q = _mm(ah, _qw(wq_t, th.get("gamma_q"), th.get("beta_q"), cfg), mode)
+    k = _mm(ah, _qw(wk_t, th.get("gamma_k"), th.get("beta_k"), cfg), mode)
+    v = _mm(ah, _qw(wv_t, th.get("gamma_v"), th.get("beta_v"), cfg), mode)
+    if cfg.let:
         q, k, v = q + bq, k + bk, v + bv
+    return q, k, v, a
+
+
+def stage_attention(q, k, v, th: Dict[str, torch.Tensor], cfg: BlockCfg):
+    """RoPE, the [Q, K] LET pair after RoPE (Eq. 5, R9), Q_a of Q~, K~, V' (R8, R12) and causal
+    attention with scores scaled by 1/sqrt(head_dim) (R10).  Returns O [T, H * hd] and the
+    post-RoPE q, k."""
+    H, Hkv, hd = cfg.n_heads, cfg.n_kv, cfg.head_dim
+    T = q.shape[0]
     q = rope(q, H, hd, cfg.rope_theta)
     k = rope(k, Hkv, hd, cfg.rope_theta)
-    if let:                                               # [Q, K] pair, Eq. 5, after RoPE (R9)
+    if cfg.let:
+        sa = th["sa"]
         q = q / _expand_kv(sa, cfg)
         k = k * sa
-    qh, kh, vh = _qa(q, cfg), _qa(k, cfg), _qa(v, cfg)    # R8, R12
+    qh, kh, vh = _qa(q, cfg), _qa(k, cfg), _qa(v, cfg)
     rep = H // Hkv
     Qh = qh.reshape(T, H, hd).transpose(0, 1)                            # [H, T, hd]
     Kh = kh.reshape(T, Hkv, hd).transpose(0, 1).repeat_interleave(rep, 0)
     Vh = vh.reshape(T, Hkv, hd).transpose(0, 1).repeat_interleave(rep, 0)
-    S = _mm(Qh, Kh, mode) / math.sqrt(hd)                                # R10
+    S = _mm(Qh, Kh, cfg.mode) / math.sqrt(hd)
     causal = torch.ones(T, T, dtype=torch.bool).tril()
     S = S.masked_fill(~causal, float("-inf"))
-    O = _attn_pv(S, Vh, cfg)                                             # P V, [H, T, hd] (R12, R19, R20)
-    O = O.transpose(0, 1).reshape(T, H * hd)
+    O = _attn_pv(S, Vh, cfg).transpose(0, 1).reshape(T, H * hd)
+    return O, q, k
+
+
+def stage_attn_out(O, x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], cfg: BlockCfg):
+    """Q_a of the attention output and the quantized o_proj with the [v, out] pair's column scale
+    and bias (Eq. 3, Eq. 4, R14), plus the residual: h1 = x + o."""
+    wo = Wd["wo"]
     oh = _qa(O, cfg)
-    if let:
-        wo_t = wo * _expand_kv(so, cfg)[None, :]
-        bo = wo @ _expand_kv(do_, cfg)
+    if cfg.let:
+        wo_t = wo * _expand_kv(th["so"], cfg)[None, :]
+        bo = wo @ _expand_kv(th["do"], cfg)
     else:
         wo_t, bo = wo, None
-    o = _mm(oh, _qw(wo_t, th.get("gamma_o"), th.get("beta_o"), cfg,
-                    _dec32(wo, _expand_kv(so, cfg)) if let else None), mode)
+    o = _mm(oh, _qw(wo_t, th.get("gamma_o"), th.get("beta_o"), cfg), cfg.mode)
     if bo is not None:
         o = o + bo
-    h1 = x + o
+    return x + o
 
-    # --- FFN half -------------------------------------------------------------------------------
+
+def stage_ffn_in(h1, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], cfg: BlockCfg):
+    """RMSNorm, the [ln2, (gate, up)] LET pair, Q_a and the quantized gate and up projections."""
+    mode = cfg.mode
+    wg, wu = Wd["wg"], Wd["wu"]
     b_ = rmsnorm(h1, cfg.rms_eps)
-    if let:                                               # [ln2, (gate, up)] pair
+    if cfg.let:
         s2, d2 = th["s2"], th["d2"]
         bt = (b_ - d2) / s2
         wg_t, wu_t = wg * s2, wu * s2
@@ -784,13 +641,31 @@ def block_forward(x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], c
     else:
         bt, wg_t, wu_t, bg, bu = b_, wg, wu, None, None
     bh = _qa(bt, cfg)
-    gt = _mm(bh, _qw(wg_t, th.get("gamma_g"), th.get("beta_g"), cfg, _dec32(wg, s2) if let else None), mode)
-    up = _mm(bh, _qw(wu_t, th.get("gamma_u"), th.get("beta_u"), cfg, _dec32(wu, s2) if let else None), mode)
-    if let:
+    gt = _mm(bh, _qw(wg_t, th.get("gamma_g"), th.get("beta_g"), cfg), mode)
+    up = _mm(bh, _qw(wu_t, th.get("gamma_u"), th.get("beta_u"), cfg), mode)
+    if cfg.let:
         gt, up = gt + bg, up + bu
+    return gt, up
+
+
+def stage_ffn_out(gt, up, h1, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], cfg: BlockCfg):
+    """SwiGLU, Q_a, the quantized down_proj (no LET on its input, Sec. 3.3) and the residual."""
     m = silu(gt) * up
-    mh = _qa(m, cfg)                                      # down_proj input: no LET (Sec. 3.3)
-    y = h1 + _mm(mh, _qw(wdn, th.get("gamma_d"), th.get("beta_d"), cfg), mode)
+    mh = _qa(m, cfg)
+    return h1 + _mm(mh, _qw(Wd["wd"], th.get("gamma_d"), th.get("beta_d"), cfg), cfg.mode), m
+
+
+def block_forward(x, Wd: Dict[str, torch.Tensor], th: Dict[str, torch.Tensor], cfg: BlockCfg,
+                  keep: Optional[Dict[str, torch.Tensor]] = None):
+    """Forward of the LET'd, LWC-quantized block (Algorithm 1, LET then
+    Quantization_with_LWC then the block on x_q), the five stages in order.  `th` holds the
+    learnable parameters (gamma_*/beta_* logits per linear; s1, d1, so, do, sa, s2, d2 when LET
+    is on).  With wbits = abits = 16 and LET off this is the full-precision block F(W, X)."""
+    q0, k0, v, a = stage_attn_in(x, Wd, th, cfg)
+    O, q, k = stage_attention(q0, k0, v, th, cfg)
+    h1 = stage_attn_out(O, x, Wd, th, cfg)
+    gt, up = stage_ffn_in(h1, Wd, th, cfg)
+    y, m = stage_ffn_out(gt, up, h1, Wd, th, cfg)
     if keep is not None:
         keep.update(dict(a=a, q=q, k=k, v=v, O=O, h1=h1, gate=gt, up=up, m=m))
     return y
@@ -903,13 +778,12 @@ def block_fold_pack(weights: Dict[str, object], theta: Dict[str, object], cfg: B
     Wd = {k: t(v) for k, v in weights.items()}
     th = {k: t(v) for k, v in theta.items()}
     H, Hkv, hd = cfg.n_heads, cfg.n_kv, cfg.head_dim
-    decide = _decide(cfg)
     out: Dict[str, torch.Tensor] = {}
     let = cfg.let
     with torch.no_grad():
         if let:
             s1, d1, so, do_, s2, d2 = th["s1"], th["d1"], th["so"], th["do"], th["s2"], th["d2"]
-            r_o = (1.0 / so.to(torch.float32)).to(F64)
+            r_o = 1.0 / so
             rows = torch.cat([torch.ones(H * hd + Hkv * hd, dtype=F64), r_o])
             so_e, do_e = _expand_kv(so, cfg), _expand_kv(do_, cfg)
         lin = dict(
@@ -920,7 +794,7 @@ def block_fold_pack(weights: Dict[str, object], theta: Dict[str, object], cfg: B
         for name, (Wl, parts, s, r) in lin.items():
             gl = torch.cat([th["gamma_" + p_] for p_ in parts])
             bl = torch.cat([th["beta_" + p_] for p_ in parts])
-            f = lwc_fakequant_fwd(Wl, gl, bl, cfg.wbits, cfg.group, s=s, eps=cfg.h_eps, row_scale=r, decide=decide)
+            f = lwc_fakequant_fwd(Wl, gl, bl, cfg.wbits, cfg.group, s=s, eps=cfg.h_eps, row_scale=r)
             out["codes_" + name] = pack_codes(f["codes"], cfg.wbits)
             out["h_" + name] = f["h"]
             out["z_" + name] = f["z"]

@@ -419,16 +419,16 @@ def test_softmax_quant_hand_example():
     assert float(got[0, 0, 1]) == 0.0 and float(got[0, 1, 2]) == 0.0
 
 
-@pytest.mark.parametrize("nbits,decide", [(8, "fp64"), (6, "fp32"), (4, "fp32"), (3, "fp64")])
-def test_softmax_quant_is_rowwise_minmax_over_visible_keys(nbits, decide):
+@pytest.mark.parametrize("nbits", [8, 6, 4, 3])
+def test_softmax_quant_is_rowwise_minmax_over_visible_keys(nbits):
     """Each query row equals Eq. 2's MinMax quantizer applied to the row's visible slice
     P[t, :t+1] alone (a per-row loop, no filling of the masked part); masked entries are 0."""
     H, T = 2, 9
     P = _causal_probs(H, T, 30 + nbits)
-    got = O.softmax_quant(P, nbits, decide=decide)
+    got = O.softmax_quant(P, nbits)
     for hh in range(H):
         for t in range(T):
-            st = O.quant_fwd(P[hh, t, :t + 1][None], 1.0, 1.0, nbits, decide=decide)
+            st = O.quant_fwd(P[hh, t, :t + 1][None], 1.0, 1.0, nbits)
             assert torch.allclose(got[hh, t, :t + 1], st["what"][0], rtol=0, atol=1e-15)
             assert bool((got[hh, t, t + 1:] == 0).all())
 
@@ -451,52 +451,55 @@ def test_softmax_quant_ste_gradient_is_per_row_quant_bwd(nbits):
             assert bool((dP[hh, t, t + 1:] == 0).all())
 
 
-def test_emulated_softmax_pv():
-    """R19: the emulated P V product rounds the unnormalised probabilities 2^(S log2 e - M) (M an
-    integer) to bf16 and divides by their unrounded sum.  Equal scores make every probability
-    exactly 1: the causal prefix mean of the bf16 values.  Shifting a row's scores by an integer
-    multiple of ln 2 changes nothing (bf16 rounding commutes with powers of two).  Every output is
-    a convex combination with each weight perturbed by at most 2^-9 relative, so it stays within
-    2^-8 max|V| of the exact softmax(S) V on the same bf16 V.  The gradient is that of
-    softmax(S) V with bf16 operands (R13)."""
+def test_sigmoid_silu_hand_values():
+    """sigmoid(t) = 1 / (1 + e^-t) (the footnote to Sec. 3.2): sigmoid(0) = 1/2 and
+    sigmoid(ln 3) = 1 / (1 + 1/3) = 3/4.  SwiGLU's silu(v) = v sigmoid(v): silu(0) = 0,
+    silu(ln 3) = (3/4) ln 3, silu(-ln 3) = -(1/4) ln 3, and silu(v) - silu(-v) = v."""
+    l3 = math.log(3.0)
+    s = O.sigmoid(torch.tensor([0.0, l3, -l3], dtype=F64)).tolist()
+    assert abs(s[0] - 0.5) < 1e-16 and abs(s[1] - 0.75) < 1e-15 and abs(s[2] - 0.25) < 1e-15
+    v = O.silu(torch.tensor([0.0, l3, -l3, 2.5], dtype=F64)).tolist()
+    assert v[0] == 0.0
+    assert abs(v[1] - 0.75 * l3) < 1e-15 and abs(v[2] + 0.25 * l3) < 1e-15
+    w = torch.linspace(-6, 6, 25, dtype=F64)
+    assert torch.allclose(O.silu(w) - O.silu(-w), w, rtol=0, atol=1e-14)
+
+
+def test_rmsnorm_hand_values():
+    """RMSNorm with unit gain: x / sqrt(mean(x^2) + eps) per token.  Row (3, 4) has mean square
+    12.5; with eps = 3.5 the root is sqrt(16) = 4, so the row maps to (0.75, 1.0) (a sum instead
+    of the mean, a variance instead of the mean square, or eps outside the root all give other
+    values).  Row (2, 2, 2, 2) with eps = 0 maps to ones, and every row is scale invariant up to
+    eps."""
+    got = O.rmsnorm(torch.tensor([[3.0, 4.0]], dtype=F64), 3.5)
+    assert torch.allclose(got, torch.tensor([[0.75, 1.0]], dtype=F64), rtol=0, atol=1e-15)
+    assert torch.equal(O.rmsnorm(torch.full((1, 4), 2.0, dtype=F64), 0.0), torch.ones(1, 4, dtype=F64))
+    g = torch.Generator().manual_seed(15)
+    x = torch.randn(3, 16, generator=g, dtype=F64)
+    assert torch.allclose(O.rmsnorm(7.0 * x, 0.0), O.rmsnorm(x, 0.0), rtol=1e-14, atol=0)
+    r = O.rmsnorm(x, 0.0)
+    assert torch.allclose((r * r).mean(-1), torch.ones(3, dtype=F64), rtol=1e-14, atol=0)
+
+
+def test_attention_stage_emulate_rounds_normalised_probabilities():
+    """In emulate mode (R13) the attention's second product takes the normalised softmax output
+    (Eq. 5) rounded to bf16 against bf16(V): equal scores give the causal prefix mean of bf16(V)
+    divided exactly, since 1/n rounds to bf16 exactly only for powers of two; the value is the
+    plain product bf16(softmax(S)) bf16(V)."""
     g = torch.Generator().manual_seed(19)
     H, T, hd = 2, 7, 4
+    cfg = O.BlockCfg(d=H * hd, n_heads=H, n_kv=H, ffn=8, wbits=16, abits=16, group=0, let=False, head_dim=hd)
     V = torch.randn(H, T, hd, generator=g, dtype=F64)
-    Vb = O.to_bf16(V)
     causal = torch.ones(T, T, dtype=torch.bool).tril()
-    S0 = torch.zeros(H, T, T, dtype=F64).masked_fill(~causal, float("-inf"))
-    got = O.softmax_pv(S0, V, "emulate")
-    want = torch.cumsum(Vb, 1) / torch.arange(1, T + 1, dtype=F64)[None, :, None]
-    assert torch.allclose(got, want, rtol=0, atol=1e-14)
     S = (torch.randn(H, T, T, generator=g, dtype=F64) * 3).masked_fill(~causal, float("-inf"))
-    got = O.softmax_pv(S, V, "emulate")
-    shift = torch.randint(-5, 6, (H, T, 1), generator=g).to(F64) * math.log(2.0)
-    assert torch.allclose(O.softmax_pv(S + shift, V, "emulate"), got, rtol=0, atol=1e-13)
-    exact = torch.softmax(S, -1) @ Vb
-    err = float((got - exact).abs().max())
-    assert 0 < err <= 2.0 ** -8 * float(Vb.abs().max())
-    Sg = S.clone().requires_grad_(True)
-    gO = torch.randn(H, T, hd, generator=g, dtype=F64)
-    (gS,) = torch.autograd.grad(O.softmax_pv(Sg, V, "emulate"), [Sg], gO)
-    P = torch.softmax(S, -1)
-    dP = O.to_bf16(gO) @ Vb.transpose(-1, -2)
-    ref = P * (dP - (dP * P).sum(-1, keepdim=True))
-    assert torch.allclose(gS, ref, rtol=1e-12, atol=1e-14)
-
-
-def test_emulated_softmax_pv_integer_reference():
-    """R19's rounding point on a hand-evaluated row: scores with S log2(e) = (0.5, -0.5) and
-    V = (1, 0).  The integer reference is M = 1, so the bf16 operands are bf16(2^-0.5) =
-    0.70703125 and bf16(2^-1.5) = 0.353515625, and the value is 0.70703125 / (2^-0.5 + 2^-1.5)
-    = 0.666595...; subtracting the non-integer maximum 0.5 instead would give exactly 2/3."""
-    ln2 = math.log(2.0)
-    S = torch.tensor([[[0.0, float("-inf")], [0.5 * ln2, -0.5 * ln2]]], dtype=F64)
-    V = torch.tensor([[[1.0], [0.0]]], dtype=F64)
-    got = O.softmax_pv(S, V, "emulate")
-    want = 0.70703125 / (2 ** -0.5 + 2 ** -1.5)
-    assert abs(float(got[0, 1, 0]) - want) < 1e-12
-    assert abs(float(got[0, 1, 0]) - 2 / 3) > 5e-5
-    assert float(got[0, 0, 0]) == 1.0
+    from oracle.omq_oracle import _attn_pv
+    got = _attn_pv(S, V, cfg)
+    want = O.to_bf16(torch.softmax(S, -1)) @ O.to_bf16(V)
+    assert torch.equal(got, want)
+    S0 = torch.zeros(H, T, T, dtype=F64).masked_fill(~causal, float("-inf"))
+    n = torch.arange(1, T + 1, dtype=F64)
+    want0 = (O.to_bf16(1.0 / n)[None, :, None] * torch.cumsum(O.to_bf16(V), 1))
+    assert torch.allclose(_attn_pv(S0, V, cfg), want0, rtol=0, atol=1e-14)
 
 
 def test_rope_properties():
@@ -533,59 +536,6 @@ def test_rope_rotation_direction():
     v = torch.tensor([[1.0, 0.0], [1.0, 0.0]], dtype=F64)
     r = O.rope(v, 1, 2, 10000.0)
     assert torch.allclose(r[1], torch.tensor([math.cos(1.0), math.sin(1.0)], dtype=F64), atol=1e-15)
-
-
-def test_fp32_decisions_match_independent_single_precision():
-    """decide="fp32" equals the same Eq. 2 arithmetic written with numpy float32 scalars, and
-    differs from float64 decisions only at elements within a few fp32 ulps of a .5 boundary."""
-    rng = np.random.default_rng(21)
-    w = (rng.standard_normal((40, 64)) * 0.03).astype(np.float32)
-    gl = rng.normal(1.0, 1.0, 40)
-    bl = rng.normal(1.0, 1.0, 40)
-    st = O.quant_fwd(torch.from_numpy(w).double(), O.sigmoid(torch.from_numpy(gl)), O.sigmoid(torch.from_numpy(bl)),
-                     3, decide="fp32")
-    for o in range(40):
-        a = np.float32(O.sigmoid(torch.tensor(gl[o])))
-        b = np.float32(O.sigmoid(torch.tensor(bl[o])))
-        M, m = np.float32(w[o].max()), np.float32(w[o].min())
-        h = np.float32(np.float32(np.float32(a * M) - np.float32(b * m)) / np.float32(7.0))
-        rh = np.float32(np.float32(1.0) / h)
-        z = -np.rint(np.float32(np.float32(b * m) * rh))
-        codes = np.clip(np.rint(np.float32(w[o] * rh)) + z, 0, 7)
-        assert float(st["h"][o]) == float(h) and float(st["z"][o]) == float(z)
-        assert np.array_equal(st["q"][o].numpy(), codes)
-    st64 = O.quant_fwd(torch.from_numpy(w).double(), O.sigmoid(torch.from_numpy(gl)), O.sigmoid(torch.from_numpy(bl)),
-                       3, decide="fp64")
-    differ = (st["q"] != st64["q"])
-    frac = st64["x"] - torch.floor(st64["x"])
-    assert bool(((frac[differ] - 0.5).abs() < 2e-5).all())
-
-
-def _sigmoid_fp32_scalar(t):
-    """The single-precision sigmoid restated with numpy float32 scalars (one rounding per op)."""
-    f = np.float32
-    x = f(-min(max(f(t), f(-80.0)), f(80.0)))
-    n = f(np.rint(f(x * f(1.44269502162933349609375))))
-    r = f(f(x - f(n * f(0.693145751953125))) - f(n * f(1.428606765330187e-06)))
-    p = f(1.98412701138295233249664e-04)
-    for c in (1.38888892251998186111450e-03, 8.33333376795053482055664e-03, 4.16666679084300994873047e-02,
-              1.66666671633720397949219e-01, 0.5, 1.0, 1.0):
-        p = f(f(p * r) + f(c))
-    e = f(p * f(2.0 ** int(n)))
-    return f(f(1.0) / f(f(1.0) + e))
-
-
-def test_sigmoid_fp32_bitwise_and_error_bound():
-    """The kernels' single-precision sigmoid: the vectorised oracle equals a scalar restatement bit
-    for bit, and stays within 4 ulp of the exact sigmoid over the logits LWC uses."""
-    rng = np.random.default_rng(22)
-    t = np.concatenate([rng.normal(0, 4, 3000), np.linspace(-30, 30, 1001), [0.0, 4.0, -4.0, 80.0, -80.0, 90.0]])
-    v = O.sigmoid_fp32(torch.tensor(t)).numpy()
-    for ti, vi in zip(t[:500], v[:500]):
-        assert vi == _sigmoid_fp32_scalar(ti)
-    exact = 1.0 / (1.0 + np.exp(-np.clip(t.astype(np.float32).astype(np.float64), -80, 80)))
-    ulp = np.spacing(exact.astype(np.float32)).astype(np.float64)
-    assert np.max(np.abs(v.astype(np.float64) - exact) / ulp) <= 4.0
 
 
 @pytest.mark.parametrize("n_kv", [4, 2])
@@ -669,9 +619,7 @@ def test_folded_block_equals_calibrated_block(let, abits, wbits, group, n_kv):
     folded = O.block_fold_pack(W, th, c)
     y_fold = O.folded_forward(folded, x, c)
     y_ref = O.block_forward(torch.as_tensor(x, dtype=F64), _t(W), _t(th), c)
-    # the packed v_proj rows are divided by s_o through the single-precision reciprocal the
-    # kernels use (R14, R15), the calibrated block divides exactly: ~1e-8 relative on h of those rows
-    assert _rel(y_fold, y_ref) < (1e-8 if let else 1e-12)
+    assert _rel(y_fold, y_ref) < 1e-12
     assert folded["codes_qkv"].dtype == torch.uint8
     assert folded["codes_qkv"].shape[1] * 8 == shape.d * wbits
 
