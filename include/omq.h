@@ -147,8 +147,10 @@ size_t omq_loss_workspace_size(int64_t n);
  *   GPU which loads the library holds until the process exits.  No workspace argument, and no
  *   cudaMalloc, cudaFree or allocating routine of any library is called.
  *   Limit: 1 <= n <= OMQ_NOALLOC_LOSS_MAX_N; other sizes return OMQ_ERR_SHAPE before any launch.
- *   Set-up: the first call on a device (with that device current) looks up the array's device
- *   address with cudaGetSymbolAddress; make that first call before any stream capture.
+ *   Set-up: a call looks up the array's device address on the current device with
+ *   cudaGetSymbolAddress whenever its stream is not being captured (so a device reset, which
+ *   reloads the module, leaves no stale address) and otherwise reuses the address of the last
+ *   lookup; make the first call on a device before any stream capture.
  *   Sharing: all calls on a device share the array and it keeps the last call's contents; each
  *   call writes every partial it later reads, so nothing needs clearing.  Calls that overlap on
  *   the GPU (different streams without ordering) race on the array: order them. */
@@ -169,6 +171,19 @@ omq_status omq_gemm_bf16(omq_stream_t stream, int64_t M, int64_t N, int64_t K, i
                          float* Cf, void* Cb, int64_t ldc, int64_t c_bs, float alpha,
                          const float* bias, const float* R, int64_t ldr, float beta_acc,
                          int32_t causal, int32_t* dev_status);
+
+/* Failure-detection self-test (the paper has no counterpart): checks that a device-side wait
+ * that never completes ends with OMQ_ERR_TIMEOUT instead of a hang.  Runs the tensor-core product
+ * of omq_gemm_bf16, C [M, N] fp32 = A [M, K] B [N, K]^T (bf16, both K-major, rows packed; one
+ * CTA: M <= 128, N <= 128, K <= 8192, N and K multiples of 8), with every mbarrier wait bounded
+ * by wait_limit_ns (1e3 .. 1e9) instead of the library's one second.  withhold = 1: the first
+ * operand load is never issued, so the wait for it expires; the kernel then writes
+ * OMQ_ERR_TIMEOUT to *dev_status (if it is still 0), waits (bounded) for the loads it did issue,
+ * releases its tensor memory and returns, leaving C unspecified.  withhold = 0: an ordinary
+ * product.  The return value covers the launch only; read *dev_status with omq_stream_status. */
+omq_status omq_selftest_bounded_wait(omq_stream_t stream, int64_t M, int64_t N, int64_t K, const void* A,
+                                     const void* B, float* C, uint64_t wait_limit_ns, int32_t withhold,
+                                     int32_t* dev_status);
 
 /* ------------------------------------------------------------------------------------------
  * Single quantized linear (Eq. 4): Y = Q_a(X~) Q_w(W~)^T + B~, and its STE backward.
@@ -264,6 +279,40 @@ omq_status omq_block_step(omq_stream_t stream, const omq_block_shape* shape,
                           const float* x, const float* y_fp, float* y, float* loss,
                           const omq_block_params* grads, void* workspace, size_t ws_bytes,
                           const omq_qcfg* cfg);
+
+/* Where omq_block_forward / omq_block_step keep the block's stage values inside the caller's
+ * workspace: byte offsets from the workspace's start (the pointer passed as `workspace`), for a
+ * workspace laid out for `shape` and `cfg`.  They let a caller (a test, a debugger, a profiler)
+ * read the quantizer inputs, stage outputs and intermediate gradients of the last call, e.g. to
+ * compare each stage of the block (Eq. 4 per linear, Eq. 5's attention, Eq. 1's loss) against
+ * another implementation started from the same stage input.  The values stay valid until the
+ * next call that uses the workspace.  Forward entries are written by both calls, backward
+ * entries by omq_block_step only.  Per-token arrays [T] are one step h (fp32) and zero point z
+ * (int32) per token row; qkv_h / qkv_z hold the q, k and v rows one after the other ([3, T]).
+ * Weight entries are indexed 0 = q|k|v, 1 = o, 2 = gate|up, 3 = down: w_hat bf16 [Cout, Cin]
+ * (the fake-quantized LET-scaled weight, Eq. 2 and Eq. 3), w_h fp32 and w_z int32
+ * [Cout, ngroups].  Returns OMQ_ERR_* for a shape or configuration omq_block_workspace_size
+ * rejects. */
+typedef struct {
+  int64_t a_hat;                   /* bf16 [T, d]: Q_a((RMSNorm(x) - d1) / s1), the q|k|v input */
+  int64_t a_h, a_z;
+  int64_t y_qkv;                   /* fp32 [T, nh*128 + 2*nkv*128]: q|k|v before RoPE (+ LET bias) */
+  int64_t qkv_h, qkv_z;            /* of Q~, K~ (after RoPE and s_a) and V' */
+  int64_t q_hat, k_hat, v_hat;     /* bf16 [T, nh*128], [T, nkv*128] x 2: Q_a(Q~), Q_a(K~), Q_a(V') */
+  int64_t o;                       /* fp32 [T, nh*128]: attention output P V */
+  int64_t o_hat, o_h, o_z;         /* bf16 [T, nh*128]: Q_a(O), the o_proj input */
+  int64_t h1;                      /* fp32 [T, d]: x + o_proj output */
+  int64_t b_hat, b_h, b_z;         /* bf16 [T, d]: Q_a((RMSNorm(h1) - d2) / s2) */
+  int64_t y_gu;                    /* fp32 [T, 2 ffn]: gate | up (+ LET bias) */
+  int64_t m_hat, m_h, m_z;         /* bf16 [T, ffn]: Q_a(silu(gate) up), the down_proj input */
+  int64_t w_hat[4], w_h[4], w_z[4];
+  int64_t dy;                      /* fp32 [T, d]: dL/dy */
+  int64_t dy_gu;                   /* fp32 [T, 2 ffn]: dL/d(gate | up) */
+  int64_t dh1;                     /* fp32 [T, d]: dL/dh1 (both paths) */
+  int64_t do_bf16;                 /* bf16 [T, nh*128]: dL/dO through Q_a, the attention backward's operand */
+  int64_t dy_qkv;                  /* fp32 [T, nh*128 + 2*nkv*128]: dL/d(q|k|v before RoPE) */
+} omq_block_saved;
+omq_status omq_block_saved_layout(const omq_block_shape* shape, const omq_qcfg* cfg, omq_block_saved* out);
 
 /* Causal self-attention of the block (Sec. 3.3, Eq. 5 applies LET to Q and K before it; the
  * softmax output is not quantized), computed without storing the [T, T] scores.

@@ -64,6 +64,17 @@ class omq_block_packed(Structure):
     _fields_ = [(n, c_void_p) for n in PACKED_FIELDS]
 
 
+SAVED_FIELDS = ["a_hat", "a_h", "a_z", "y_qkv", "qkv_h", "qkv_z", "q_hat", "k_hat", "v_hat", "o", "o_hat", "o_h", "o_z", "h1", "b_hat", "b_h",
+                "b_z", "y_gu", "m_hat", "m_h", "m_z"]
+SAVED_BWD_FIELDS = ["dy", "dy_gu", "dh1", "do_bf16", "dy_qkv"]
+
+
+class omq_block_saved(Structure):
+    _fields_ = ([(n, c_int64) for n in SAVED_FIELDS] + [("w_hat", c_int64 * 4), ("w_h", c_int64 * 4),
+                                                          ("w_z", c_int64 * 4)] +
+                [(n, c_int64) for n in SAVED_BWD_FIELDS])
+
+
 LET_STATS_FIELDS = ["a_absmax", "a_sum", "q_absmax", "k_absmax", "o_absmax", "o_sum", "b_absmax", "b_sum"]
 
 
@@ -85,12 +96,14 @@ _SIGS = {
     "omq_block_loss_noalloc": (I32, [P, I64, P, P, P, P, P]),
     "omq_gemm_bf16": (I32, [P, I64, I64, I64, I64, P, I64, I64, I32, P, I64, I64, I32, P, P, I64, I64, F32,
                             P, P, I64, F32, I32, P]),
+    "omq_selftest_bounded_wait": (I32, [P, I64, I64, I64, P, P, P, ctypes.c_uint64, I32, P]),
     "omq_qlinear_fwd": (I32, [P, I64, I64, I64, P, P, P, P, P, P, P, P, P, P]),
     "omq_qlinear_bwd": (I32, [P, I64, I64, I64, P, P, P, P, P, P, P, P, P, P, P, P, P, P, SZ, P]),
     "omq_qlinear_workspace_size": (SZ, [I64, I64, I64, P]),
     "omq_block_workspace_size": (SZ, [P, P]),
     "omq_block_forward": (I32, [P, P, P, P, P, P, P, SZ, P]),
     "omq_block_step": (I32, [P, P, P, P, P, P, P, P, P, P, SZ, P]),
+    "omq_block_saved_layout": (I32, [P, P, P]),
     "omq_attention_fwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P]),
     "omq_attention_bwd": (I32, [P, I32, I32, I32, P, I64, P, P, I64, P, I64, P, P, I64, P, P, I64, P, P, I64,
                                 P]),
@@ -325,6 +338,18 @@ def omq_qlinear_bwd(T, Cin, Cout, X, W, s, delta, gamma_logit, beta_logit, saved
 
 def omq_block_workspace_size(shape: omq_block_shape, cfg: omq_qcfg) -> int:
     return lib().omq_block_workspace_size(ctypes.byref(shape), ctypes.byref(cfg))
+
+
+def omq_selftest_bounded_wait(M, N, K, A, B, C, wait_limit_ns, withhold, dev_status, stream=None):
+    check("omq_selftest_bounded_wait", lib().omq_selftest_bounded_wait(
+        stream_handle(stream), M, N, K, ptr(A), ptr(B), ptr(C), int(wait_limit_ns), int(withhold), ptr(dev_status)))
+
+
+def omq_block_saved_layout(shape: omq_block_shape, cfg: omq_qcfg) -> omq_block_saved:
+    out = omq_block_saved()
+    check("omq_block_saved_layout", lib().omq_block_saved_layout(ctypes.byref(shape), ctypes.byref(cfg),
+                                                                 ctypes.byref(out)))
+    return out
 
 
 def omq_block_forward(shape, weights, theta, x, y, workspace, cfg, stream=None):

@@ -104,6 +104,37 @@ class BlockState:
                             self.workspace, self.cfg, stream)
         return self.loss
 
+    def saved(self, backward: bool = True) -> Dict[str, "object"]:
+        """The stage values the last forward / step left in the workspace (omq_block_saved_layout),
+        as device tensor views named like the layout's fields; w_hat, w_h, w_z become lists over
+        q|k|v, o, gate|up, down.  Views, not copies: the next call overwrites them."""
+        torch = self.torch
+        sh = self.shape
+        lay = _lib.omq_block_saved_layout(self.c_shape, self.cfg)
+        T, d, f = sh.T, sh.d, sh.ffn
+        nqkv = sh.dq + 2 * sh.dkv
+        bf, f32, i32 = torch.bfloat16, torch.float32, torch.int32
+        spec = dict(a_hat=(bf, (T, d)), a_h=(f32, (T,)), a_z=(i32, (T,)), y_qkv=(f32, (T, nqkv)),
+                    qkv_h=(f32, (3, T)), qkv_z=(i32, (3, T)), q_hat=(bf, (T, sh.dq)), k_hat=(bf, (T, sh.dkv)),
+                    v_hat=(bf, (T, sh.dkv)), o=(f32, (T, sh.dq)), o_hat=(bf, (T, sh.dq)),
+                    o_h=(f32, (T,)), o_z=(i32, (T,)), h1=(f32, (T, d)), b_hat=(bf, (T, d)), b_h=(f32, (T,)),
+                    b_z=(i32, (T,)), y_gu=(f32, (T, 2 * f)), m_hat=(bf, (T, f)), m_h=(f32, (T,)), m_z=(i32, (T,)))
+        if backward:
+            spec.update(dy=(f32, (T, d)), dy_gu=(f32, (T, 2 * f)), dh1=(f32, (T, d)), do_bf16=(bf, (T, sh.dq)),
+                        dy_qkv=(f32, (T, nqkv)))
+
+        def view(off, dtype, shp):
+            n = int(np.prod(shp)) * torch.empty(0, dtype=dtype).element_size()
+            return self.workspace[off:off + n].view(dtype).view(shp)
+
+        out = {k: view(getattr(lay, k), dt, shp) for k, (dt, shp) in spec.items()}
+        ng = lambda cin: 1 if self.group == 0 else cin // self.group
+        lins = [(nqkv, d), (d, sh.dq), (2 * f, d), (d, f)]
+        out["w_hat"] = [view(lay.w_hat[i], bf, (co, ci)) for i, (co, ci) in enumerate(lins)]
+        out["w_h"] = [view(lay.w_h[i], f32, (co, ng(ci))) for i, (co, ci) in enumerate(lins)]
+        out["w_z"] = [view(lay.w_z[i], i32, (co, ng(ci))) for i, (co, ci) in enumerate(lins)]
+        return out
+
     def adamw(self, lr_lwc: float = 5e-3, lr_let: float = 1e-2, stream=None):
         """AdamW with zero weight decay on both parameter groups (Sec. 4.1 "Training"); the step
         count advances on the device."""

@@ -44,6 +44,9 @@ struct FlashArgs {
   // row statistics (scratch); both 16-byte aligned.
   int pbits; float eps;
   float* pqr; float* pqb;
+  // row stride (in rows) of the per-row arrays lse, D, pqr, pqb: [H, ldl(, 8 | 4)]; 0 = T.  A
+  // multiple of 4 at least T lets the backward fetch them with 16-byte bulk copies for any T.
+  int ldl;
 };
 static inline bool flash_pq_on(int pbits) { return pbits >= 2 && pbits <= 8; }
 omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a);

@@ -114,8 +114,9 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   w.Kh = c.take<bf16>(T * dkv);
   w.Vh = c.take<bf16>(T * dkv);
   w.sqkv = take_qstate(c, 3 * T);
-  w.lse = c.take<float>(H * T);
-  w.pqr = flash_pq_on(cfg.pbits) ? c.take<float>(H * T * 8) : nullptr;
+  const int64_t T4 = (T + 3) / 4 * 4;       // row stride of the attention's per-row arrays
+  w.lse = c.take<float>(H * T4);
+  w.pqr = flash_pq_on(cfg.pbits) ? c.take<float>(H * T4 * 8) : nullptr;
   w.O = c.take<float>(T * dq);
   w.O_h = c.take<bf16>(T * dq);
   w.so = take_qstate(c, T);
@@ -140,8 +141,8 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   w.dh1_b = c.take<bf16>(T * d);
   w.dOh = c.take<float>(T * dq);
   w.dO_b = c.take<bf16>(T * dq);
-  w.Drow = c.take<float>(H * T);
-  w.pqb = flash_pq_on(cfg.pbits) ? c.take<float>(H * T * 4) : nullptr;
+  w.Drow = c.take<float>(H * T4);
+  w.pqb = flash_pq_on(cfg.pbits) ? c.take<float>(H * T4 * 4) : nullptr;
   w.dQKV = c.take<float>(T * nqkv);
   w.dYqkv = c.take<float>(T * nqkv);
   w.dYqkv_b = c.take<bf16>(T * nqkv);
@@ -181,7 +182,7 @@ omq_status check_block(const omq_block_shape* s, const omq_qcfg* cfg) {
   OMQ_REQUIRE(s->T > 0 && s->d > 0 && s->n_heads > 0 && s->n_kv > 0 && s->ffn > 0, OMQ_ERR_SHAPE);
   OMQ_REQUIRE(s->head_dim == 128, OMQ_ERR_UNSUPPORTED);
   OMQ_REQUIRE(s->n_heads % s->n_kv == 0, OMQ_ERR_SHAPE);
-  OMQ_REQUIRE(s->T % 8 == 0 && s->d % 8 == 0 && s->ffn % 8 == 0, OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(s->d % 8 == 0 && s->ffn % 8 == 0, OMQ_ERR_ALIGN);
   if (cfg->group > 0) {
     OMQ_REQUIRE(s->d % cfg->group == 0 && s->ffn % cfg->group == 0 && ((int64_t)s->n_heads * 128) % cfg->group == 0,
                 OMQ_ERR_SHAPE);
@@ -388,7 +389,7 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   fa.T = (int)c.T; fa.H = (int)c.H; fa.Hkv = (int)c.Hkv; fa.hd = (int)c.hd;
   fa.Q = w.Qh; fa.K = w.Kh; fa.V = w.Vh; fa.ldq = c.dq; fa.ldkv = c.dkv;
   fa.O = w.O; fa.ldo = c.dq; fa.lse = w.lse; fa.status = status;
-  fa.pbits = cfg.pbits; fa.eps = cfg.h_eps; fa.pqr = w.pqr;
+  fa.pbits = cfg.pbits; fa.eps = cfg.h_eps; fa.pqr = w.pqr; fa.ldl = (int)((c.T + 3) / 4 * 4);
   OMQ_TRY(flash_fwd_launch(st, fa));
   ActFwdArgs ao{};
   ao.producer = AP_PLAIN; ao.X = w.O; ao.ldx = c.dq; ao.T = c.T; ao.C = c.dq; ao.Xq = w.O_h; ao.ldq = c.dq;
@@ -498,7 +499,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   fa.O = w.O; fa.ldo = c.dq; fa.lse = w.lse; fa.dO = w.dO_b; fa.lddo = c.dq; fa.D = w.Drow;
   fa.dQ = w.dQKV; fa.ldg = c.nqkv; fa.dK = w.dQKV + c.dq; fa.dV = w.dQKV + c.dq + c.dkv; fa.ldgkv = c.nqkv;
   fa.status = status;
-  fa.pbits = cfg.pbits; fa.eps = cfg.h_eps; fa.pqr = w.pqr; fa.pqb = w.pqb;
+  fa.pbits = cfg.pbits; fa.eps = cfg.h_eps; fa.pqr = w.pqr; fa.pqb = w.pqb; fa.ldl = (int)((c.T + 3) / 4 * 4);
   OMQ_TRY(flash_bwd_launch(st, fa));
   QkvArgs qa{};
   qa.T = (int)c.T; qa.H = (int)c.H; qa.Hkv = (int)c.Hkv; qa.hd = (int)c.hd; qa.Y = w.Yqkv; qa.ldy = c.nqkv; qa.cs = w.cs;
@@ -593,6 +594,31 @@ size_t omq_block_workspace_size(const omq_block_shape* shape, const omq_qcfg* cf
   BlockWS tmp;
   carve_block(dry, *shape, *cfg, tmp, true);
   return dry.off + 256;
+}
+
+omq_status omq_block_saved_layout(const omq_block_shape* shape, const omq_qcfg* cfg, omq_block_saved* out) {
+  OMQ_TRY(check_block(shape, cfg));
+  OMQ_REQUIRE(out, OMQ_ERR_INVALID_ARG);
+  // carve against a stand-in base address (never dereferenced) and report offsets from it
+  uint8_t* const base = reinterpret_cast<uint8_t*>(uintptr_t(1) << 20);
+  Carve c{base, 0};
+  BlockWS w;
+  carve_block(c, *shape, *cfg, w, true);
+  auto off = [&](const void* p) -> int64_t { return p ? (int64_t)((const uint8_t*)p - base) : -1; };
+  out->a_hat = off(w.a_h); out->a_h = off(w.sa.h); out->a_z = off(w.sa.z);
+  out->y_qkv = off(w.Yqkv); out->qkv_h = off(w.sqkv.h); out->qkv_z = off(w.sqkv.z);
+  out->q_hat = off(w.Qh); out->k_hat = off(w.Kh); out->v_hat = off(w.Vh);
+  out->o = off(w.O); out->o_hat = off(w.O_h); out->o_h = off(w.so.h); out->o_z = off(w.so.z);
+  out->h1 = off(w.h1); out->b_hat = off(w.b_h); out->b_h = off(w.sb.h); out->b_z = off(w.sb.z);
+  out->y_gu = off(w.Ygu); out->m_hat = off(w.m_h); out->m_h = off(w.sm.h); out->m_z = off(w.sm.z);
+  const bf16* wh[4] = {w.Wqkv_h, w.Wo_h, w.Wgu_h, w.Wd_h};
+  const QState4* sq[4] = {&w.sq_qkv, &w.sq_o, &w.sq_gu, &w.sq_d};
+  for (int i = 0; i < 4; ++i) {
+    out->w_hat[i] = off(wh[i]); out->w_h[i] = off(sq[i]->h); out->w_z[i] = off(sq[i]->z);
+  }
+  out->dy = off(w.dy); out->dy_gu = off(w.dYgu); out->dh1 = off(w.dh1); out->do_bf16 = off(w.dO_b);
+  out->dy_qkv = off(w.dYqkv);
+  return OMQ_OK;
 }
 
 omq_status omq_block_forward(omq_stream_t stream, const omq_block_shape* shape, const omq_block_weights* w,

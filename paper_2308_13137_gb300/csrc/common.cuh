@@ -82,13 +82,13 @@ __device__ __forceinline__ uint4 pack_bf16x8(const float* f) {
 }
 
 // ------------------------------------------------------------------------------------------------
-// Eq. 2 on one element, given the group's h and z (IEEE division, round half to even)
+// Eq. 2 on one element, given the group's h and z
 // ------------------------------------------------------------------------------------------------
 struct QState {          // per-group quantizer state
   float h;               // step, floored at eps
-  float rh;              // 1/h, correctly rounded: w/h is formed as w * rh
-  float z;               // zero point (integer valued)
-  float u;               // beta * min / h
+  float rh;              // 1/h, correctly rounded (a first guess of w/h is w * rh)
+  float z;               // zero point (integer valued): -round(beta * min / h)
+  float u;               // beta * min / h (its value; the rounding is taken exactly, -z)
   float a, b;            // clipping strengths
   float M, m;            // group max / min
   int floored;
@@ -115,43 +115,76 @@ __device__ __forceinline__ float omq_sigmoid(float t) {
   return __fdiv_rn(1.0f, __fadd_rn(1.0f, e));
 }
 
-// h = (a*M - b*m)/Q floored at eps, its reciprocal, u = (b*m) * (1/h) and z = -round(u)
+// round(w / h) of Eq. 2 for the exact quotient of the two single-precision values (h > 0).
+// A first guess k = rint(w * (1/h)) can land on the wrong side of a half when the quotient is
+// within a few ulps of one.  The remainder r = w - k h is exact in single precision (a fused
+// multiply-add; |r| is at most about h / 2 and lies on the grid of the smaller of the two
+// exponents, so it fits in 24 bits), and k moves by rint(r / h), which is 0 or +-1.  The result
+// equals the rounding of the exact quotient except for quotients within about 1e-7 of a half.
+__device__ __forceinline__ float omq_round_quot(float w, float h, float rh) {
+  const float k = rintf(__fmul_rn(w, rh));
+  const float r = __fmaf_rn(-k, h, w);
+  return __fadd_rn(k, rintf(__fmul_rn(r, rh)));
+}
+
+// h = (a*M - b*m)/Q floored at eps, its reciprocal, u = (b*m) / h and z = -round(u).
+// The zero point rounds u written without the rounded h: Q (b m) / (a M - b m), or Q m / (M - m)
+// when a = b (the clipping strengths cancel), or b m / eps when h is floored.  Such a quotient can
+// be exactly a half, which then rounds to even, and often is: with gamma = beta and a group whose
+// max and min are opposite (frequent among bf16 weights) u = -Q/2; rounding u = (b m) (1/h) from
+// the rounded fp32 h would round it by noise instead.  The single-precision u decides unless it lies
+// within its own error bound (eight roundings, times the cancellation factor of a M - b m) of a half;
+// only then is the quotient formed in double precision, where the products by Q and the difference
+// of single-precision values are exact and an exact half stays one.
 __device__ __forceinline__ QState omq_qstate(float M, float m, float a, float b, float Q, float eps) {
   QState s;
   s.a = a; s.b = b; s.M = M; s.m = m;
-  float hr = __fdiv_rn(__fsub_rn(__fmul_rn(a, M), __fmul_rn(b, m)), Q);
+  const float bm = __fmul_rn(b, m);
+  const float aM = __fmul_rn(a, M);
+  const float d = __fsub_rn(aM, bm);
+  float hr = __fdiv_rn(d, Q);
   s.floored = !(hr >= eps);
   s.h = s.floored ? eps : hr;
   s.rh = __frcp_rn(s.h);
-  s.u = __fmul_rn(__fmul_rn(b, m), s.rh);
-  s.z = -rintf(s.u);
+  s.u = __fmul_rn(bm, s.rh);
+  float k = rintf(s.u);
+  const float cancel = s.floored ? 1.f : (fabsf(aM) + fabsf(bm)) / fabsf(d);
+  const float margin = 1e-6f + fabsf(s.u) * 4.76837158203125e-07f * (2.f + cancel);   // 2^-21 = eight ulps
+  if (fabsf(fabsf(s.u - k) - 0.5f) <= margin) {
+    double u64;
+    if (s.floored) u64 = __ddiv_rn((double)bm, (double)eps);
+    else if (a == b) u64 = __ddiv_rn((double)Q * (double)m, (double)M - (double)m);
+    else u64 = __ddiv_rn((double)Q * (double)bm, (double)d);
+    k = (float)rint(u64);
+  }
+  s.z = -k;
   return s;
 }
 
-// code c = round(w/h) + z before the clamp, with w/h formed as w * (1/h)
+// code c = round(w/h) + z before the clamp; *x_out = w/h (value, w * (1/h))
 __device__ __forceinline__ float omq_code_raw(float w, const QState& s, float* x_out) {
-  float x = __fmul_rn(w, s.rh);
-  *x_out = x;
-  return rintf(x) + s.z;
+  *x_out = __fmul_rn(w, s.rh);
+  return omq_round_quot(w, s.h, s.rh) + s.z;
 }
 
-// clamp(rint(w/h) + z, 0, Q) - z formed as clamp(rint(w/h), -z, Q - z): every term is an integer
-// below 2^24 after the clamp, so both forms give the same value
+// clamp(round(w/h) + z, 0, Q) - z formed as clamp(round(w/h), -z, Q - z): every term is an
+// integer below 2^24 after the clamp, so both forms give the same value
 __device__ __forceinline__ float omq_fakequant(float w, const QState& s, float Q, float* code) {
-  const float r = rintf(__fmul_rn(w, s.rh));
+  const float r = omq_round_quot(w, s.h, s.rh);
   const float qz = fminf(fmaxf(r, -s.z), Q - s.z);
   if (code) *code = qz + s.z;
   return __fmul_rn(qz, s.h);
 }
 
-// STE pieces of one element: returns dwhat/dh; *inr = 1 when 0 <= c <= Q
+// STE pieces of one element: returns dwhat/dh; *inr = 1 when 0 <= c <= Q.  round(u) is -z, the
+// zero point's own rounding.
 __device__ __forceinline__ float omq_ste_dh(float w, const QState& s, float Q, int* inr) {
   const float x = __fmul_rn(w, s.rh);
-  const float r = rintf(x);
+  const float r = omq_round_quot(w, s.h, s.rh);
   const float c = r + s.z;
   if (c >= 0.f && c <= Q) { *inr = 1; return r - x; }
   *inr = 0;
-  float ru = rintf(s.u) - s.u;
+  const float ru = -s.z - s.u;
   return (c < 0.f) ? ru : (Q + ru);
 }
 

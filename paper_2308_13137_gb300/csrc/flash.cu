@@ -86,6 +86,7 @@ __device__ __forceinline__ bool waitw(uint64_t* b, uint32_t parity, int32_t* sta
 // ================================================================================================
 struct FwdP {
   int T, H, rep;
+  int ldl;                   // row stride of lse / pqr (>= T)
   float c;                   // log2(e) / sqrt(head_dim)
   float* O; int64_t ldo;     // [T, H*128] fp32
   float* lse;                // [H, T]: m + log2(l) of the scaled base-2 logits
@@ -360,10 +361,10 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
           for (int i = 0; i < 8; ++i) dst[i] = make_float4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
         }
       }
-      if (row < p.T && half == 0) p.lse[(int64_t)h * p.T + row] = mt + log2f(lt);
+      if (row < p.T && half == 0) p.lse[(int64_t)h * p.ldl + row] = mt + log2f(lt);
       if constexpr (PQ) {
         if (row < p.T && half == 0) {
-          float4* d = reinterpret_cast<float4*>(p.pqr + ((int64_t)h * p.T + row) * PQ_N);
+          float4* d = reinterpret_cast<float4*>(p.pqr + ((int64_t)h * p.ldl + row) * PQ_N);
           d[0] = make_float4(qs.h, qs.rh, qs.z, Mp);
           d[1] = make_float4(mp, qs.floored ? 1.f : 0.f, (float)imx, (float)imn);
         }
@@ -573,7 +574,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
                                  fmaf(o0[4 * i + 3], a0, o1[4 * i + 3] * a1));
         }
       }
-      if (row < p.T && half == 0) p.lse[(int64_t)h * p.T + row] = Mt + log2f(lt);
+      if (row < p.T && half == 0) p.lse[(int64_t)h * p.ldl + row] = Mt + log2f(lt);
     }
   }
   tc_fence_before();
@@ -588,7 +589,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
 // backward: D = rowsum(dO * O) per (token, head)
 // ================================================================================================
 __global__ void attn_rowdot_kernel(int T, int H, const __nv_bfloat16* __restrict__ dO, int64_t lddo,
-                                   const float* __restrict__ O, int64_t ldo, float* __restrict__ D) {
+                                   const float* __restrict__ O, int64_t ldo, float* __restrict__ D, int ldl) {
   const int64_t w = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (w >= (int64_t)T * H) return;
@@ -598,7 +599,7 @@ __global__ void attn_rowdot_kernel(int T, int H, const __nv_bfloat16* __restrict
   const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&u);
   const float2 d01 = __bfloat1622float2(b[0]), d23 = __bfloat1622float2(b[1]);
   const float s = warp_sum(o.x * d01.x + o.y * d01.y + o.z * d23.x + o.w * d23.y);
-  if (lane == 0) D[(int64_t)h * T + t] = s;
+  if (lane == 0) D[(int64_t)h * ldl + t] = s;
 }
 
 // ================================================================================================
@@ -606,6 +607,7 @@ __global__ void attn_rowdot_kernel(int T, int H, const __nv_bfloat16* __restrict
 // ================================================================================================
 struct BwdP {
   int T, H, rep;
+  int ldl;                   // row stride of lse / D / pqr / pqb (>= T, a multiple of 4)
   float c;                   // log2(e) / sqrt(head_dim)
   float scale;               // 1 / sqrt(head_dim)
   const float* lse; const float* D;      // [H, T]
@@ -687,8 +689,8 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       const int s = it % B_NQD;
       const int h = g * p.rep + it / niq, qi = i0 + it % niq;
       if (!waitb(&qd_empty[s], ((it / B_NQD) & 1) ^ 1, p.status, abort_flag)) break;
-      const uint32_t nb = (uint32_t)min(64, p.T - qi * 64) * 4;     // lse / D bytes inside [0, T)
-      const int64_t r0 = (int64_t)h * p.T + qi * 64;
+      const uint32_t nb = (uint32_t)min(64, p.ldl - qi * 64) * 4;   // lse / D bytes inside [0, ldl)
+      const int64_t r0 = (int64_t)h * p.ldl + qi * 64;
       float* ld = reinterpret_cast<float*>(smem + B_LD + s * L::RD);  // s: the ring slot
       if constexpr (PQ) {
         mbar_expect_tx(&qd_full[s], 2 * B_QTILE + (1 + PQ_N + PG_N) * nb);
@@ -775,7 +777,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
             const float4 s1 = reinterpret_cast<const float4*>(R8 + qc * PQ_N)[1];   // m, fl, imax, imin
             const float4 gs = *reinterpret_cast<const float4*>(G4 + qc * PG_N);     // D, dM, dm
             const float pv = ex2(fmaf(sv[i], p.c, -Lr[qc]));
-            const float rr = rintf(__fmul_rn(pv, s0.y));
+            const float rr = omq_round_quot(pv, s0.x, s0.y);
             const float cd = rr + s0.z;
             const bool inr = cd >= 0.f && cd <= p.Q;
             float g = inr ? dp[i] : 0.f;
@@ -949,20 +951,20 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     const int row = qb * 128 + r;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     const bool row_ok = row < p.T;
-    const float Lr = row_ok ? p.lse[(int64_t)h * p.T + row] : 0.f;
-    float Dr = (MODE == 0 && row_ok) ? p.D[(int64_t)h * p.T + row] : 0.f;
+    const float Lr = row_ok ? p.lse[(int64_t)h * p.ldl + row] : 0.f;
+    float Dr = (MODE == 0 && row_ok) ? p.D[(int64_t)h * p.ldl + row] : 0.f;
     // PQ: the row's quantizer state (and, for MODE 2, its backward statistics)
-    float q_rh = 0.f, q_z = 0.f, q_ru = 0.f, q_fl = 1.f, q_M = 0.f, q_m = 0.f;
+    float q_h = 1.f, q_rh = 0.f, q_z = 0.f, q_ru = 0.f, q_fl = 1.f, q_M = 0.f, q_m = 0.f;
     int q_imax = -1, q_imin = -1;
     float g_dM = 0.f, g_dm = 0.f;
     if (MODE != 0 && row_ok) {
-      const float4* st = reinterpret_cast<const float4*>(p.pqr + ((int64_t)h * p.T + row) * PQ_N);
+      const float4* st = reinterpret_cast<const float4*>(p.pqr + ((int64_t)h * p.ldl + row) * PQ_N);
       const float4 a0 = st[0], a1 = st[1];
       const float u = __fmul_rn(a1.x, a0.y);        // m / h as the forward formed it
-      q_rh = a0.y; q_z = a0.z; q_M = a0.w; q_m = a1.x; q_ru = rintf(u) - u; q_fl = a1.y;
+      q_h = a0.x; q_rh = a0.y; q_z = a0.z; q_M = a0.w; q_m = a1.x; q_ru = -a0.z - u; q_fl = a1.y;
       q_imax = (int)a1.z; q_imin = (int)a1.w;
       if (MODE == 2) {
-        const float4 gs = *reinterpret_cast<const float4*>(p.pqb + ((int64_t)h * p.T + row) * PG_N);
+        const float4 gs = *reinterpret_cast<const float4*>(p.pqb + ((int64_t)h * p.ldl + row) * PG_N);
         Dr = gs.x; g_dM = gs.y; g_dm = gs.z;
       }
     }
@@ -994,7 +996,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
             const bool vis = !need_mask || (key <= row && row_ok);
             const float pv = ex2(fmaf(sv[i], p.c, -Lr));
             const float x = __fmul_rn(pv, q_rh);
-            const float rr = rintf(x);
+            const float rr = omq_round_quot(pv, q_h, q_rh);
             const float cd = rr + q_z;
             const bool inr = cd >= 0.f && cd <= p.Q;
             if constexpr (MODE == 1) {
@@ -1044,7 +1046,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
         const float Gh = q_fl != 0.f ? 0.f : t[1];    // a floored step has no gradient
         const float dM = Gh / p.Q, dm = t[2] - Gh / p.Q;
         // sum_j P_j dP_j, dP including the totals that reach the max and the min (R7)
-        *reinterpret_cast<float4*>(p.pqb + ((int64_t)h * p.T + row) * PG_N) =
+        *reinterpret_cast<float4*>(p.pqb + ((int64_t)h * p.ldl + row) * PG_N) =
             make_float4(t[0] + q_M * dM + q_m * dm, dM, dm, 0.f);
       }
     } else if (ok) {
@@ -1077,6 +1079,7 @@ bool set_smem(const void* fn, int bytes) {
 
 omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
   OMQ_REQUIRE(a.T > 0 && a.H > 0 && a.Hkv > 0 && a.H % a.Hkv == 0 && a.hd == HD, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(a.ldl == 0 || a.ldl >= a.T, OMQ_ERR_SHAPE);
   OMQ_REQUIRE(a.Q && a.K && a.V && a.O && a.lse, OMQ_ERR_INVALID_ARG);
   OMQ_REQUIRE(a.ldq % 8 == 0 && a.ldkv % 8 == 0 && a.ldo % 4 == 0, OMQ_ERR_ALIGN);
   OMQ_REQUIRE(omq_aligned16(a.Q) && omq_aligned16(a.K) && omq_aligned16(a.V) && omq_aligned16(a.O), OMQ_ERR_ALIGN);
@@ -1099,6 +1102,7 @@ omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
   }
   FwdP p;
   p.T = a.T; p.H = a.H; p.rep = a.H / a.Hkv;
+  p.ldl = a.ldl ? a.ldl : a.T;
   p.c = (float)(1.4426950408889634 / sqrt((double)HD));
   p.O = a.O; p.ldo = a.ldo; p.lse = a.lse; p.status = a.status;
   p.Q = pq ? (float)((1 << a.pbits) - 1) : 0.f; p.eps = a.eps; p.pqr = a.pqr;
@@ -1117,8 +1121,10 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
                   a.ldgkv % 4 == 0,
               OMQ_ERR_ALIGN);
   OMQ_REQUIRE(omq_aligned16(a.dO) && omq_aligned16(a.dQ) && omq_aligned16(a.dK) && omq_aligned16(a.dV), OMQ_ERR_ALIGN);
-  // lse, D and the PQ row data are fetched by 16-byte bulk copies
-  OMQ_REQUIRE(a.T % 4 == 0 && omq_aligned16(a.lse) && (pq || omq_aligned16(a.D)), OMQ_ERR_ALIGN);
+  // lse, D and the PQ row data are fetched by 16-byte bulk copies of whole groups of 4 rows
+  const int ldl = a.ldl ? a.ldl : a.T;
+  OMQ_REQUIRE(ldl >= a.T, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(ldl % 4 == 0 && omq_aligned16(a.lse) && (pq || omq_aligned16(a.D)), OMQ_ERR_ALIGN);
   OMQ_REQUIRE(!pq || (a.pqr && a.pqb), OMQ_ERR_INVALID_ARG);
   OMQ_REQUIRE(!pq || (omq_aligned16(a.pqr) && omq_aligned16(a.pqb)), OMQ_ERR_ALIGN);
   CUtensorMap tq64, tdo64, tk, tv, tq, tdo;
@@ -1143,6 +1149,7 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
   }
   BwdP p;
   p.T = a.T; p.H = a.H; p.rep = a.H / a.Hkv;
+  p.ldl = ldl;
   p.c = (float)(1.4426950408889634 / sqrt((double)HD));
   p.scale = (float)(1.0 / sqrt((double)HD));
   p.lse = a.lse; p.D = a.D;
@@ -1162,7 +1169,7 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
     return OMQ_OK;
   }
   const int64_t rows = (int64_t)a.T * a.H;
-  attn_rowdot_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(a.T, a.H, a.dO, a.lddo, a.O, a.ldo, a.D);
+  attn_rowdot_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(a.T, a.H, a.dO, a.lddo, a.O, a.ldo, a.D, ldl);
   OMQ_LAUNCH_CHECK();
   flash_bwd_dkv_kernel<false><<<g1, FA_THREADS, BL<false>::SMEM, st>>>(tq64, tk, tv, tdo64, p);
   OMQ_LAUNCH_CHECK();

@@ -33,6 +33,8 @@ struct GemmParams {
   GemmLwcEpi lw;             // used by the LWC-epilogue instantiation only
   int32_t* status;
   int pair;                  // 1: CTA pairs, one 256-row tile per pair (cta_group::2)
+  uint64_t wait_ns;          // limit of every mbarrier wait (OMQ_WAIT_LIMIT_NS unless a self-test sets it)
+  int withhold;              // self-test only: the first operand load is never issued, so its wait expires
 };
 
 constexpr int EPI_TILE_BYTES = 32 * 32 * 4;      // one 32 x 32 fp32 block, 128-byte rows
@@ -171,7 +173,7 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
     const uint32_t buf = acc_it & 1;
     bool ok = true;
     if (has_acc) {
-      ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[buf], (acc_it >> 1) & 1));
+      ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[buf], (acc_it >> 1) & 1, p.wait_ns));
       if (!ok) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; }
       tc_fence_after();
     }
@@ -285,6 +287,7 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
   uint64_t* acc_empty = acc_full + 2;      // [2]
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(acc_empty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+  uint64_t* drain = acc_empty + 3;         // after tmem_holder and abort_flag (8 bytes)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bm_tile = PAIR ? 2 * BM : BM;
@@ -300,6 +303,7 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
     constexpr int EPI_WARPS = LWC ? 8 : 4;
     for (int b = 0; b < 2; ++b) { mbar_init(&acc_full[b], 1); mbar_init(&acc_empty[b], (PAIR ? 2 : 1) * EPI_WARPS); }
     *abort_flag = 0;
+    mbar_init(drain, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
@@ -324,9 +328,10 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
       const int nb0 = ti.n0 + rank * BNH;
       for (int kb = 0; kb < ti.nkb; ++kb, ++it) {
         const int s = it % STAGES;
-        if (!mbar_wait(&empty[s], ((it / STAGES) & 1) ^ 1)) {
+        if (!mbar_wait(&empty[s], ((it / STAGES) & 1) ^ 1, p.wait_ns)) {
           omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; break;
         }
+        if (p.withhold && it == 0) continue;      // self-test: the stage's load is never issued
         uint8_t* sa = smem + s * L::STAGE_BYTES;
         uint8_t* sb = sa + L::A_BYTES;
         const int k0 = ti.k_begin + kb * BK;
@@ -365,16 +370,25 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
         }
       }
     }
+    // after an expired wait (or a withheld load) no copy this CTA issued may still be landing in its
+    // shared memory when it exits: wait, bounded, for the last load of every stage (with CTA pairs
+    // the leader's barrier counts both CTAs' bytes, and the peer leaves only after the leader)
+    if ((*abort_flag || p.withhold) && leader) {
+      const uint32_t first = it > (uint32_t)STAGES ? it - STAGES : 0u;
+      for (uint32_t j = first; j < it; ++j)
+        if (!(p.withhold && j == 0)) mbar_wait(&full[j % STAGES], (j / STAGES) & 1, p.wait_ns);
+    }
   } else if (warp == 1 && lane == 0 && leader) {
     // ---------------- MMA issuer (with CTA pairs: the leader CTA only) ----------------
     constexpr uint32_t IDESC_KK = idesc_bf16(PAIR ? 2 * BM : BM, BN, 0, 0);
     const uint32_t idesc = IDESC_KK | ((uint32_t)p.a_mn << 15) | ((uint32_t)p.b_mn << 16);
     uint32_t it = 0, acc_it = 0;
+    bool issued = false;
     for (int t = t_first; t < total && !*abort_flag; t += t_step) {
       const TileInfo ti = tile_info(p, t, BN, rank);
       if (ti.skip || ti.nkb == 0) continue;
       const uint32_t buf = acc_it & 1;
-      if (!mbar_wait(&acc_empty[buf], ((acc_it >> 1) & 1) ^ 1)) {
+      if (!mbar_wait(&acc_empty[buf], ((acc_it >> 1) & 1) ^ 1, p.wait_ns)) {
         omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; break;
       }
       tc_fence_after();
@@ -382,10 +396,11 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
       bool ok = true;
       for (int kb = 0; kb < ti.nkb; ++kb, ++it) {
         const int s = it % STAGES;
-        if (!mbar_wait(&full[s], (it / STAGES) & 1)) {
+        if (!mbar_wait(&full[s], (it / STAGES) & 1, p.wait_ns)) {
           omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; ok = false; break;
         }
         tc_fence_after();
+        issued = true;
         const uint32_t sa = smem_u32(smem + s * L::STAGE_BYTES);
         const uint32_t sb = sa + L::A_BYTES;
 #pragma unroll
@@ -403,6 +418,13 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
       else umma_commit(&acc_full[buf]);
       ++acc_it;
       if (!ok) break;
+    }
+    // after an expired wait, the products already issued must finish before the tensor memory is
+    // released: one more commit, on a barrier of its own, tracks all of them (bounded wait)
+    if (*abort_flag && issued) {
+      if (PAIR) umma_commit_pair(drain, 0x1);
+      else umma_commit(drain);
+      mbar_wait(drain, 0, p.wait_ns);
     }
   } else if (LWC && warp >= 2) {
     lwc_epilogue<BN, PAIR, LWC>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, (warp - 2) >> 2, lane, total, rank);
@@ -424,7 +446,7 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
       const uint32_t buf = acc_it & 1;
       bool ok = true;
       if (has_acc) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[buf], (acc_it >> 1) & 1));  // tcgen05.ld is warp-wide
+        ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[buf], (acc_it >> 1) & 1, p.wait_ns));  // tcgen05.ld is warp-wide
         if (!ok) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; }
         tc_fence_after();
       }
@@ -679,6 +701,7 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
   p.M = (int)M; p.N = (int)N; p.K = (int)K; p.batch = (int)batch;
   p.a_mn = A.kmajor ? 0 : 1; p.b_mn = B.kmajor ? 0 : 1;
   p.causal = causal; p.ep = ep; p.status = status; p.pair = pair ? 1 : 0;
+  p.wait_ns = OMQ_WAIT_LIMIT_NS; p.withhold = 0;
   // stream the larger operand once and keep the smaller one L2-resident: with m fastest, the
   // CTAs working at one time share an N tile of B and sweep A; with n fastest, the reverse
   p.n_fast = ((double)M > 1.5 * (double)N) ? 1 : 0;
@@ -743,6 +766,7 @@ omq_status gemm_launch_lwc(cudaStream_t st, int64_t M, int64_t N, int64_t K, con
   p.M = (int)M; p.N = (int)N; p.K = (int)K; p.batch = 1;
   p.a_mn = A.kmajor ? 0 : 1; p.b_mn = B.kmajor ? 0 : 1;
   p.causal = 0; p.lw = lw; p.status = status; p.pair = pair ? 1 : 0;
+  p.wait_ns = OMQ_WAIT_LIMIT_NS; p.withhold = 0;
   p.n_fast = ((double)M > 1.5 * (double)N) ? 1 : 0;
   cudaEvent_t e0 = nullptr, e1 = nullptr;
   if (g_prof.on) {
@@ -794,4 +818,30 @@ extern "C" omq_status omq_gemm_bf16(omq_stream_t stream, int64_t M, int64_t N, i
   GemmOperand b{B, b_ld, b_bs, b_kmajor ? 1 : 0};
   GemmEpilogue ep{Cf, (__nv_bfloat16*)Cb, ldc, c_bs, alpha, bias, R, ldr, beta_acc};
   return gemm_launch((cudaStream_t)stream, M, N, K, batch, a, b, ep, causal, dev_status);
+}
+
+// Failure-detection self-test: the product above on one CTA with every wait bounded by
+// wait_limit_ns, and optionally without its first operand load, so that the wait for it expires.
+extern "C" omq_status omq_selftest_bounded_wait(omq_stream_t stream, int64_t M, int64_t N, int64_t K, const void* A,
+                                                const void* B, float* C, uint64_t wait_limit_ns, int32_t withhold,
+                                                int32_t* dev_status) {
+  OMQ_REQUIRE(M > 0 && M <= BM && N > 0 && N <= 128 && K > 0 && K <= 8192, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(A && B && C, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(withhold == 0 || withhold == 1, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(wait_limit_ns >= 1000ull && wait_limit_ns <= OMQ_WAIT_LIMIT_NS, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(omq_aligned16(A) && omq_aligned16(B) && omq_aligned16(C), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(K % 8 == 0 && N % 8 == 0, OMQ_ERR_ALIGN);
+  CUtensorMap ta, tb, tc;
+  bool ok = make_map(&ta, A, K, M, 1, K, 0, BM) && make_map(&tb, B, K, N, 1, K, 0, 128) &&
+            make_map_c(&tc, C, N, M, 1, N, 0);
+  if (!ok) return OMQ_ERR_UNSUPPORTED;
+  GemmParams p;
+  memset(&p, 0, sizeof(p));
+  p.M = (int)M; p.N = (int)N; p.K = (int)K; p.batch = 1;
+  p.a_mn = 0; p.b_mn = 0; p.n_fast = 0; p.causal = 0; p.pair = 0;
+  p.ep = GemmEpilogue{C, nullptr, N, 0, 1.f, nullptr, nullptr, 0, 0.f};
+  p.status = dev_status;
+  p.wait_ns = wait_limit_ns;
+  p.withhold = withhold;
+  return launch_cfg<128, 6>((cudaStream_t)stream, ta, tb, tc, p);
 }

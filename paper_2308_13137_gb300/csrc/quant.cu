@@ -1238,15 +1238,23 @@ omq_status omq_block_loss_noalloc(omq_stream_t stream, int64_t n, const float* Y
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return OMQ_ERR_CUDA;
   OMQ_REQUIRE(dev >= 0 && dev < OMQ_NOALLOC_MAX_DEVICES, OMQ_ERR_UNSUPPORTED);
+  // The host-side name of the array is not a device address: ask the runtime for the array's
+  // address on the current device whenever the stream is not being captured, so that a device
+  // reset (which reloads the module) cannot leave a stale address behind; otherwise reuse the
+  // address of the last lookup.
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing((cudaStream_t)stream, &cs) != cudaSuccess) {
+    cudaGetLastError();
+    cs = cudaStreamCaptureStatusActive;
+  }
   float* part = g_noalloc_loss_ptr[dev].load();
-  if (!part) {
-    // first call on this device: the host-side name of the array is not a device address, so
-    // ask the runtime for the array's address on the current device
+  if (cs == cudaStreamCaptureStatusNone) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_noalloc_loss_part) != cudaSuccess || !p) return OMQ_ERR_CUDA;
     part = static_cast<float*>(p);
     g_noalloc_loss_ptr[dev].store(part);
   }
+  if (!part) return OMQ_ERR_CUDA;                 // first call on this device inside a capture
   // every partial the final reduction reads is written by this call, so nothing needs clearing
   return loss_launch((cudaStream_t)stream, n, Yq, Yfp, loss, dY, (__nv_bfloat16*)dY_bf16, part);
 }

@@ -30,15 +30,16 @@ static __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t par
   return ok != 0;
 }
 
-// Bounded wait on a phase parity; false when the time limit expired.
-static __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+// Bounded wait on a phase parity; false when the time limit (default one second) expired.
+static __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
+                                                 uint64_t limit_ns = OMQ_WAIT_LIMIT_NS) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = omq_globaltimer();
   while (true) {
 #pragma unroll 1
     for (int i = 0; i < 32; ++i)
       if (mbar_try_wait(bar, parity)) return true;
-    if (omq_globaltimer() - t0 > OMQ_WAIT_LIMIT_NS) return false;
+    if (omq_globaltimer() - t0 > limit_ns) return false;
   }
 }
 

@@ -38,7 +38,7 @@ def _ref(Q, K, V, dO, H, Hkv, bits, plain_ste=False):
     s = q @ kk.transpose(-1, -2) / math.sqrt(128)
     s = s.masked_fill(~torch.ones(T, T, dtype=torch.bool).tril(), float("-inf"))
     P = torch.softmax(s, -1)
-    Pq = O.softmax_quant(P, bits, EPS, decide="fp32")
+    Pq = O.softmax_quant(P, bits, EPS)
     if plain_ste:              # identity gradient: no clamp mask, no h path (a deliberately wrong backward)
         Pq = P + (Pq - P).detach()
     Pb = Pq + (O.to_bf16(Pq.detach()) - Pq.detach())          # bf16 operand, gradient unchanged

@@ -1,42 +1,33 @@
 """Kernel-level parity of every C-ABI entry point against the fp64 oracle.
 
-Integer decisions (codes, zero points, argmax/argmin) are taken in the kernel's precision on both
-sides: the test re-derives them in IEEE fp32 on the CPU from the same fp32 quantizer input and the
-kernel's own h, so they must match bit for bit; elements whose exact pre-round value lies within
-1e-6 of a .5 boundary are counted and reported.  Real-valued outputs are compared with the fp64
-oracle (h to 1e-6 relative; gradients to 3e-2 relative Frobenius error, the benchmark spec's bound)."""
+Code decisions follow the shared-scale protocol of `_parity`: the codes must equal
+round(w / h) + z, clamped, for the exact quotient of the fp32 quantizer input w (W~ = fl32(s W),
+times fl32 of the row scale; X~ = fl32(fl32(X - delta) / s)) and the kernel's own h and z, except
+elements within 1e-6 of a .5 boundary, which are counted and reported.  h is compared with the
+fp64 oracle (1e-6 relative), z with the oracle's float64 decision (exemptions counted), the
+max/min indices with the first index of the fp32 input's extremes.  Real-valued outputs are
+compared with the fp64 oracle (gradients to 3e-2 relative Frobenius error, the benchmark spec's bound)."""
 import numpy as np
 import pytest
 import torch
 
 import oracle as O
+from _parity import GRAD_TOL, OUT_TOL, check_codes, check_h, check_zero_points, rel as _rel
 from paper_2308_13137_gb300 import _lib, inputs as I
 
 pytestmark = pytest.mark.gpu
 F64 = torch.float64
-GRAD_TOL = 3e-2
-OUT_TOL = 1e-2
-
-
-def _rel(a, b):
-    a, b = torch.as_tensor(a).double().cpu(), torch.as_tensor(b).double().cpu()
-    return float((a - b).norm() / b.norm().clamp_min(1e-300))
 
 
 def _dev(a, dtype=torch.float32):
     return torch.as_tensor(np.asarray(a)).to(dtype).cuda().contiguous()
 
 
-def _fp32_codes(wt32, h32, z32, nbits):
-    """Codes decided in IEEE fp32: clamp(rint(fl32(w/h)) + z, 0, Q); groups on the last axis."""
-    x = wt32 / h32[..., None]
-    c = torch.round(x) + z32[..., None].float()
-    return torch.clamp(c, 0, 2 ** nbits - 1).to(torch.int64)
-
-
-def _near_ties(wt, h, tol=1e-6):
-    x = wt.double() / h.double()[..., None]
-    return ((x - torch.floor(x)) - 0.5).abs() < tol
+def _first_extremes(G32):
+    """First index of the max and of the min along the last axis (R7) of an fp32 tensor."""
+    imax = (G32 == G32.max(-1, keepdim=True).values).int().argmax(-1)
+    imin = (G32 == G32.min(-1, keepdim=True).values).int().argmax(-1)
+    return imax, imin
 
 
 LWC_CASES = [  # Cout, Cin, nbits, group, let, rowscale, perturb
@@ -47,6 +38,7 @@ LWC_CASES = [  # Cout, Cin, nbits, group, let, rowscale, perturb
     (256, 512, 2, 64, False, False, True),
     (192, 512, 4, 0, True, True, True),            # v_proj rows divided by s_o
     (64, 11008, 4, 0, False, False, True),         # down_proj row length
+    (128, 512, 8, 128, True, False, True),         # 8 bits: quotients up to 255
 ]
 
 
@@ -75,44 +67,38 @@ def test_lwc_fwd_bwd(cuda_lib, Cout, Cin, nbits, group, let, rowscale, perturb):
     _lib.omq_lwc_fakequant_fwd(Cout, Cin, Wd, sd, rd, _dev(gl), _dev(bl), Wq, codes, h, z, imax, imin,
                                _dev(delta) if let else None, _dev(shift) if rowscale else None, Bt, cfg)
     torch.cuda.synchronize()
+    tag = f"lwc {Cout}x{Cin} W{nbits} g{group}{' LET' if let else ''}{' rows' if rowscale else ''}"
 
-    # -- integer decisions in fp32 (same precision as the kernel) --
+    # -- the fp32 quantizer input W~ = fl32(fl32(W s) r) (one correctly rounded product each) --
     wt32 = torch.from_numpy(W)
     if let:
         wt32 = wt32 * torch.from_numpy(s)[None, :]
-    wt32 = wt32 * (torch.from_numpy(r)[:, None] if rowscale else 1.0)
+    if rowscale:
+        wt32 = wt32 * torch.from_numpy(r)[:, None]
     gsz = group or Cin
     G32 = wt32.reshape(Cout, ng, gsz)
     hg, zg = h.cpu(), z.cpu()
-    first_max = (G32 == G32.max(-1, keepdim=True).values).int().argmax(-1) + torch.arange(ng) * gsz
-    first_min = (G32 == G32.min(-1, keepdim=True).values).int().argmax(-1) + torch.arange(ng) * gsz
-    assert torch.equal(imax.cpu().long(), first_max) and torch.equal(imin.cpu().long(), first_min)
-    c32 = _fp32_codes(G32, hg, zg, nbits).reshape(Cout, Cin)
-    near = _near_ties(G32, hg).reshape(Cout, Cin)
-    mism = (codes.cpu().long() != c32)
-    assert int(mism.sum()) == 0, f"{int(mism.sum())} code mismatches ({int(near.sum())} near-ties)"
-    what32 = ((c32.float() - zg.float().repeat_interleave(gsz, 1)) * hg.repeat_interleave(gsz, 1)).to(torch.bfloat16)
-    assert torch.equal(Wq.cpu(), what32)
+    fmax, fmin = _first_extremes(G32)
+    base = torch.arange(ng) * gsz
+    assert torch.equal(imax.cpu().long(), fmax + base) and torch.equal(imin.cpu().long(), fmin + base)
+    x = G32.double() / hg.double()[..., None]
+    check_codes(tag, x, codes.cpu().reshape(Cout, ng, gsz), zg, nbits)
+    qz = codes.cpu().reshape(Cout, ng, gsz).float() - zg.float()[..., None]
+    assert torch.equal(Wq.cpu(), (qz * hg[..., None]).reshape(Cout, Cin).to(torch.bfloat16))
 
-    # -- real-valued state against the fp64 oracle --
-    f64 = O.lwc_fakequant_fwd(torch.from_numpy(W), torch.from_numpy(gl), torch.from_numpy(bl), nbits, group,
-                              s=torch.from_numpy(s) if let else None,
-                              row_scale=torch.from_numpy(r) if rowscale else None)
-    assert float(((hg.double() - f64["h"]) / f64["h"]).abs().max()) < 1e-6
-    u_near = ((f64["st"]["u"] - torch.floor(f64["st"]["u"])) - 0.5).abs() < 1e-6
-    assert torch.equal(zg.double()[~u_near], f64["z"][~u_near])
-    # the oracle with its decisions in the kernels' precision: identical integers, same h
+    # -- h and z against the fp64 oracle --
     f = O.lwc_fakequant_fwd(torch.from_numpy(W), torch.from_numpy(gl), torch.from_numpy(bl), nbits, group,
-                            s=torch.from_numpy(s) if let else None, row_scale=torch.from_numpy(r) if rowscale else None,
-                            decide="fp32")
-    assert torch.equal(codes.cpu().long(), f["codes"]) and torch.equal(zg.double(), f["z"])
-    assert torch.equal(hg.double(), f["h"])
+                            s=torch.from_numpy(s) if let else None,
+                            row_scale=torch.from_numpy(r) if rowscale else None)
+    st = f["st"]
+    check_h(tag, hg, f["h"], st["a"] * st["M"], st["b"] * st["m"], 2 ** nbits - 1)
+    check_zero_points(tag, st["u"], zg, f["z"])
     if let:
         ref_B = (torch.from_numpy(W).double() @ torch.from_numpy(delta).double()
                  - (torch.from_numpy(shift).double() if rowscale else 0)) * (torch.from_numpy(r).double() if rowscale else 1)
         assert _rel(Bt.cpu(), ref_B) < 1e-5
 
-    # -- backward --
+    # -- backward against the oracle's own (float64-decided) forward --
     g = np.random.default_rng(7).standard_normal((Cout, Cin)).astype(np.float32)
     dBt = rng.standard_normal(Cout).astype(np.float32) if let else None
     dgl = torch.empty(Cout, ng, device="cuda")
@@ -145,6 +131,7 @@ ACT_CASES = [  # T, C, nbits, let
     (64, 11008, 8, False),
     (128, 1024, 2, True),
     (96, 512, 16, True),
+    (80, 2048, 8, True),
 ]
 
 
@@ -165,24 +152,26 @@ def test_act_quant_fwd_bwd(cuda_lib, T, C, nbits, let):
     sd, dd = (_dev(s), _dev(d)) if let else (None, None)
     _lib.omq_act_quant_per_token(T, C, Xd, sd, dd, Xq, codes, h, z, imax, imin, cfg)
     torch.cuda.synchronize()
+    # the fp32 quantizer input X~ = fl32(fl32(X - delta) / s), each operation correctly rounded
     Xt32 = torch.from_numpy(X)
     if let:
         Xt32 = (Xt32 - torch.from_numpy(d)) / torch.from_numpy(s)
+    tag = f"act {T}x{C} A{nbits}{' LET' if let else ''}"
     if nbits >= 16:
         assert torch.equal(Xq.cpu(), Xt32.to(torch.bfloat16))
+        fa = None
     else:
         hg, zg = h.cpu(), z.cpu()
-        assert torch.equal(imax.cpu().long(), (Xt32 == Xt32.max(-1, keepdim=True).values).int().argmax(-1))
-        assert torch.equal(imin.cpu().long(), (Xt32 == Xt32.min(-1, keepdim=True).values).int().argmax(-1))
-        c32 = _fp32_codes(Xt32, hg, zg, nbits)
-        assert int((codes.cpu().long() != c32).sum()) == 0
-        assert torch.equal(Xq.cpu(), ((c32.float() - zg.float()[:, None]) * hg[:, None]).to(torch.bfloat16))
-        fa64 = O.act_quant_per_token(torch.from_numpy(X), nbits, torch.from_numpy(s) if let else None,
-                                     torch.from_numpy(d) if let else None)
-        assert float(((hg.double() - fa64["h"]) / fa64["h"]).abs().max()) < 1e-6
+        fmax, fmin = _first_extremes(Xt32)
+        assert torch.equal(imax.cpu().long(), fmax) and torch.equal(imin.cpu().long(), fmin)
+        check_codes(tag, Xt32.double() / hg.double()[:, None], codes.cpu(), zg, nbits)
+        qz = codes.cpu().float() - zg.float()[:, None]
+        assert torch.equal(Xq.cpu(), (qz * hg[:, None]).to(torch.bfloat16))
         fa = O.act_quant_per_token(torch.from_numpy(X), nbits, torch.from_numpy(s) if let else None,
-                                   torch.from_numpy(d) if let else None, decide="fp32")
-        assert torch.equal(codes.cpu().long(), fa["codes"]) and torch.equal(hg.double(), fa["h"])
+                                   torch.from_numpy(d) if let else None)
+        st = fa["st"]
+        check_h(tag, hg, fa["h"], st["M"], st["m"], 2 ** nbits - 1)
+        check_zero_points(tag, st["u"], zg, fa["z"])
     # backward
     g = np.random.default_rng(9).standard_normal((T, C)).astype(np.float32)
     dX = torch.empty(T, C, device="cuda")
