@@ -71,6 +71,11 @@ notes of the repository):
      1e-2 for the LET vectors): betas 0.9 / 0.999, eps 1e-8, bias-corrected moments, decoupled
      weight decay; one update after every calibration sample (batch size 1).  Algorithm 1's
      LET statistics (R16) are taken on the fp inputs of each block before they are advanced.
+ R21 the zero point rounds u = beta*min/h with h unfloored written as
+     Q*beta*min / (gamma*max - beta*min), and as Q*min / (max - min) when gamma = beta (the
+     clipping strengths cancel): the same value without the intermediate rounding of h, so a
+     quotient that is exactly a half (gamma = beta and max = -min give u = -Q/2) stays exact
+     and rounds to even (R2).
  R20 softmax-output quantization (the ablation of Table A7, off by default): the causal softmax
      output is quantized per query row with the MinMax Q_a (gamma = beta = 1, the floor of h
      included) over the visible keys j <= t only; the masked entries stay 0.  Its backward is the
@@ -136,6 +141,22 @@ def _first_argmin(w: torch.Tensor) -> torch.Tensor:
 # Eq. 2, explicit forward and STE backward of one quantizer over groups on the last axis
 # ----------------------------------------------------------------------------------------------
 
+def _zero_point_round(a, b, M, m, Q: float, floored, eps: float) -> torch.Tensor:
+    """round(u) for the zero point z = -round(u), u = beta*min/h (Eq. 2), read as R21: with h
+    unfloored, u = Q*beta*min / (gamma*max - beta*min), or Q*min / (max - min) when gamma = beta;
+    with h floored, u = beta*min/eps."""
+    with torch.no_grad():
+        M, m = M.detach(), m.detach()
+        a = torch.as_tensor(a, dtype=F64).detach().expand_as(M)
+        b = torch.as_tensor(b, dtype=F64).detach().expand_as(M)
+        den = a * M - b * m
+        rng_ = M - m
+        u_same = Q * m / torch.where(rng_ == 0, torch.ones_like(rng_), rng_)
+        u_gen = Q * b * m / torch.where(den == 0, torch.ones_like(den), den)
+        u = torch.where(torch.as_tensor(floored), b * m / eps, torch.where(a == b, u_same, u_gen))
+        return rne(u)
+
+
 def quant_fwd(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5) -> Dict[str, torch.Tensor]:
     """Eq. 2 over groups laid out on the last axis of `w` (shape [..., g]).
 
@@ -155,7 +176,7 @@ def quant_fwd(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5) -> Dict[str,
     h = torch.where(floored, torch.full_like(h_raw, eps), h_raw)
     u = b * m / h
     x = w / h[..., None]
-    z = -rne(u)
+    z = -_zero_point_round(a, b, M, m, Q, floored, eps)
     c = rne(x) + z[..., None]
     q = torch.clamp(c, 0.0, Q)
     what = (q - z[..., None]) * h[..., None]               # R1
@@ -179,9 +200,9 @@ def quant_bwd(st: Dict[str, torch.Tensor], g: torch.Tensor) -> Dict[str, torch.T
     a, b, M, m = st["a"], st["b"], st["M"], st["m"]
     inr = (c >= 0) & (c <= Q)
     below = c < 0
+    ru = -st["z"] - u                                      # round(u) is -z
     dh_elem = torch.where(inr, rne(x) - x,
-                          torch.where(below, (rne(u) - u)[..., None],
-                                      (Q + rne(u) - u)[..., None]))
+                          torch.where(below, ru[..., None], (Q + ru)[..., None]))
     G_h = (g * dh_elem).sum(-1)
     G_h = torch.where(st["floored"], torch.zeros_like(G_h), G_h)
     G_bm = (g * (~inr).to(F64)).sum(-1)
@@ -264,8 +285,11 @@ def quant_ste(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5) -> torch.Ten
     imin = _first_argmin(w.detach())
     M = torch.gather(w, -1, imax[..., None])[..., 0]
     m = torch.gather(w, -1, imin[..., None])[..., 0]
-    h = torch.clamp((a * M - b * m) / Q, min=eps)          # R3: gradient 0 when floored
-    z = -_ste_round(b * m / h)
+    h_raw = (a * M - b * m) / Q
+    h = torch.clamp(h_raw, min=eps)                        # R3: gradient 0 when floored
+    u = b * m / h
+    ru = _zero_point_round(a, b, M, m, Q, (h_raw < eps).detach(), eps) - u.detach()
+    z = -(u + ru)                                          # round(u) forward (R21), identity backward
     c = _ste_round(w / h[..., None]) + z[..., None]
     q = torch.clamp(c, 0.0, Q)
     if tape is not None:
@@ -274,7 +298,7 @@ def quant_ste(w: torch.Tensor, a, b, nbits: int, eps: float = 1e-5) -> torch.Ten
             u = b * m / h
             x = w / h[..., None]
             tape.rec.append(dict(imax=imax, imin=imin, floored=torch.as_tensor(h_raw < eps),
-                                 ru=(rne(u) - u).detach(), rx=(rne(x) - x).detach(),
+                                 ru=ru.detach(), rx=(rne(x) - x).detach(),
                                  inr=((c >= 0) & (c <= Q)).detach(), below=(c < 0).detach()))
     return (q - z[..., None]) * h[..., None]
 

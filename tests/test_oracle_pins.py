@@ -451,6 +451,28 @@ def test_softmax_quant_ste_gradient_is_per_row_quant_bwd(nbits):
             assert bool((dP[hh, t, t + 1:] == 0).all())
 
 
+def test_zero_point_exact_halves_round_to_even():
+    """R21 with R2: when gamma = beta the zero point's quotient is u = Q min / (max - min), so a
+    group with max = -min gives u = -Q/2 exactly and one with max = 5 |min| gives u = -Q/6; hand
+    values.  N = 4, group (-1, 0.25, 1): u = 15 (-1) / 2 = -7.5, half to even -8, z = 8; N = 2:
+    u = -1.5 -> -2, z = 2; N = 4, group (-1, 0, 5): u = 15 (-1) / 6 = -2.5 -> -2, z = 2.  The same
+    holds for Q_a (gamma = beta = 1).  With gamma != beta there is no exact half: z = -round(beta
+    min / h) of the plain formula."""
+    t = lambda v: torch.tensor(v, dtype=F64)
+    g4 = t([[-1.0, 0.25, 1.0]])
+    a = O.sigmoid(t([4.0]))
+    assert float(O.quant_fwd(g4, a, a, 4)["z"][0]) == 8.0
+    assert float(O.quant_fwd(g4, a, a, 2)["z"][0]) == 2.0
+    assert float(O.quant_fwd(t([[-1.0, 0.0, 5.0]]), a, a, 4)["z"][0]) == 2.0
+    assert float(O.quant_fwd(g4, 1.0, 1.0, 4)["z"][0]) == 8.0
+    st = O.quant_fwd(t([[-1.0, 0.3, 2.0]]), O.sigmoid(t([3.0])), O.sigmoid(t([1.0])), 4)
+    assert float(st["z"][0]) == -round(float(st["b"][0] * -1.0 / st["h"][0]))
+    # the STE surrogate and the explicit backward see the same zero point
+    w = g4.clone().requires_grad_(True)
+    y = O.quant_ste(w, a, a, 4)
+    assert torch.allclose(y.detach(), O.quant_fwd(g4, a, a, 4)["what"], rtol=0, atol=1e-15)
+
+
 def test_sigmoid_silu_hand_values():
     """sigmoid(t) = 1 / (1 + e^-t) (the footnote to Sec. 3.2): sigmoid(0) = 1/2 and
     sigmoid(ln 3) = 1 / (1 + 1/3) = 3/4.  SwiGLU's silu(v) = v sigmoid(v): silu(0) = 0,
