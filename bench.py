@@ -32,6 +32,8 @@ if ROOT not in sys.path:
 METRIC = "calibration tokens/sec per block (fwd+bwd, fused LWC+LET) and % of step roofline"
 UNIT = "tokens/s"
 DEFAULT_CONFIG = "llama7b_w4a4"
+# configurations whose full oracle step takes over a minute on the host: forward only, extrapolated
+FORWARD_ONLY_BASELINE = ("llama13b_w2a16_g64", "llama2_70b_w4a4_gqa")
 
 
 def _peaks():
@@ -120,88 +122,158 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------------------------------------
-# the oracle on host cores: bounded samples of the same workload
+# the oracle on host cores
 # ------------------------------------------------------------------------------------------------
-def _oracle_sampler(shape, W, th, x):
-    """Yields (seconds, block-equivalent seconds) per sample.  A sample is one oracle calibration
-    step (Eq. 4 quantized linear, LWC + LET where the block has them, MSE to the fp output, STE
-    gradients) of a 128-output-channel slice of one of the block's seven projections, at the full
-    token count, cycling q, k, v, o, gate, up, down; its time is scaled by Cout/128 to the whole
-    projection.  Attention and the norms (about 4% of the step's flops) are not sampled."""
-    import numpy as np
+PIECES = ["fwd q|k|v", "fwd attention", "fwd o_proj", "fwd gate|up", "fwd down_proj", "loss",
+          "bwd down_proj", "bwd gate|up", "bwd o_proj", "bwd attention", "bwd q|k|v"]
+
+
+def _oracle_pieces(shape, W, th, x, yfp, out=None):
+    """Yields (piece name, seconds) forever: the oracle's calibration step (forward of the quantized
+    block, loss against y_fp, straight-through backward to every parameter) cut at the block's
+    five stages, in the order one step runs them (five forward stages, the loss, the five stage
+    backwards), and again for the next step.  One pass over the eleven pieces is exactly one oracle
+    block_step; each piece is a bounded sample of it.  `out` (a dict), when given, receives the
+    step's loss and parameter gradients after every pass."""
     import torch
     import oracle as O
-    torch.manual_seed(0)
-    T, d, f = shape.T, shape.d, shape.ffn
-    x64 = torch.from_numpy(x).double()
-    a = x64 / torch.sqrt((x64 * x64).mean(-1, keepdim=True) + shape.rms_eps)
-    rng = np.random.default_rng(5)
-    m_in = torch.from_numpy(rng.standard_normal((T, f)).astype(np.float32)).double()
-    let = bool(shape.let)
-    lin = [("q", "wq", a, "s1", "d1"), ("k", "wk", a, "s1", "d1"), ("v", "wv", a, "s1", "d1"),
-           ("o", "wo", x64, None, None), ("g", "wg", a, "s2", "d2"), ("u", "wu", a, "s2", "d2"),
-           ("d", "wd", m_in, None, None)]
-    rows = 128
-    i = 0
+    cfg = O.BlockCfg.from_shape(shape)
+    t = lambda v: torch.as_tensor(v).to(torch.float64)
+    Wd = {k: t(v) for k, v in W.items()}
+    names = (O.THETA_NAMES_LWC if shape.wbits < 16 else []) + (O.THETA_NAMES_LET if shape.let else [])
+    dq, dkv, f = shape.dq, shape.dkv, shape.ffn
+    xx, yf = t(x), t(yfp)
+
+    def grad(out, inp, gout):
+        inps = [] if inp is None else (list(inp) if isinstance(inp, (list, tuple)) else [inp])
+        return torch.autograd.grad(out, [leaf[k] for k in names] + inps, gout, allow_unused=True)
+
     while True:
-        name, wn, X, sn, dn = lin[i % 7]
-        Wfull = torch.from_numpy(W[wn])
-        Wsl = Wfull[:rows]
-        gl = torch.from_numpy(th["gamma_" + name][:rows])
-        bl = torch.from_numpy(th["beta_" + name][:rows])
-        s = torch.from_numpy(th[sn]) if (let and sn) else None
-        dl = torch.from_numpy(th[dn]) if (let and dn) else None
-        yfp = X @ Wsl.double().T
-        t0 = time.perf_counter()
-        O.qlinear_step(X, Wsl, None, gl, bl, yfp, shape.wbits, shape.group, shape.abits, s=s, delta=dl,
-                       mode="emulate")
-        dt = time.perf_counter() - t0
-        yield dt, dt * Wfull.shape[0] / rows
-        i += 1
+        leaf = {k: t(th[k]).clone().requires_grad_(True) for k in names}
+        c = time.perf_counter()
+        q, k, v, _ = O.stage_attn_in(xx, Wd, leaf, cfg)
+        qkv = torch.cat([q, k, v], 1)
+        yield PIECES[0], time.perf_counter() - c
+        c = time.perf_counter()
+        qkv_in = qkv.detach().requires_grad_(True)
+        Ob, _, _ = O.stage_attention(qkv_in[:, :dq], qkv_in[:, dq:dq + dkv], qkv_in[:, dq + dkv:], leaf, cfg)
+        yield PIECES[1], time.perf_counter() - c
+        c = time.perf_counter()
+        O_in = Ob.detach().requires_grad_(True)
+        h1 = O.stage_attn_out(O_in, xx, Wd, leaf, cfg)
+        yield PIECES[2], time.perf_counter() - c
+        c = time.perf_counter()
+        h1_in = h1.detach().requires_grad_(True)
+        gt, up = O.stage_ffn_in(h1_in, Wd, leaf, cfg)
+        gu = torch.cat([gt, up], 1)
+        yield PIECES[3], time.perf_counter() - c
+        c = time.perf_counter()
+        gu_in = gu.detach().requires_grad_(True)
+        h1_res = h1_in.detach().requires_grad_(True)
+        y, _ = O.stage_ffn_out(gu_in[:, :f], gu_in[:, f:], h1_res, Wd, leaf, cfg)
+        yield PIECES[4], time.perf_counter() - c
+        c = time.perf_counter()
+        y_in = y.detach().requires_grad_(True)
+        loss, _ = O.block_loss(y_in, yf)
+        (dy,) = torch.autograd.grad(loss, [y_in])
+        yield PIECES[5], time.perf_counter() - c
+        c = time.perf_counter()
+        gE = grad(y, [gu_in, h1_res], dy)
+        yield PIECES[6], time.perf_counter() - c
+        c = time.perf_counter()
+        gD = grad(gu, h1_in, gE[-2])
+        dh1 = gD[-1] + gE[-1]
+        yield PIECES[7], time.perf_counter() - c
+        c = time.perf_counter()
+        gC = grad(h1, O_in, dh1)
+        yield PIECES[8], time.perf_counter() - c
+        c = time.perf_counter()
+        gB = grad(Ob, qkv_in, gC[-1])
+        yield PIECES[9], time.perf_counter() - c
+        c = time.perf_counter()
+        gA = grad(qkv, None, gB[-1]) if names else []
+        dt = time.perf_counter() - c
+        if out is not None:
+            out["loss"] = loss.detach()
+            for i, n in enumerate(names):
+                out["d" + n] = sum(gg[i] for gg in (gA, gB, gC, gD, gE) if gg[i] is not None)
+        yield PIECES[10], dt
+        del q, k, v, qkv, Ob, h1, gt, up, gu, y, gE, gD, gC, gB, gA
 
 
-def _oracle_value(shape, W, th, x, n_samples):
+def _oracle_forward_seconds(shape, W, th, x):
+    """One oracle forward of the quantized block (no autograd), in seconds."""
     import torch
-    it = _oracle_sampler(shape, W, th, x)
-    wall, eq = 0.0, 0.0
-    for _ in range(n_samples):
-        a, b = next(it)
-        wall += a
-        eq += b
-    cycles = n_samples / 7.0
-    return shape.T * cycles / eq, wall, torch.get_num_threads()
+    import oracle as O
+    cfg = O.BlockCfg.from_shape(shape)
+    t = lambda v: torch.as_tensor(v).to(torch.float64)
+    Wd = {k: t(v) for k, v in W.items()}
+    tt = {k: t(v) for k, v in th.items()}
+    with torch.no_grad():
+        c = time.perf_counter()
+        O.block_forward(t(x), Wd, tt, cfg)
+        return time.perf_counter() - c
+
+
+def _oracle_yfp(shape, W, x):
+    import oracle as O
+    return O.block_fp_forward(x, W, O.BlockCfg.from_shape(shape)).float().numpy()
+
+
+def cpu_baseline(shape, W, th, x, full_step: bool):
+    """The oracle on the host cores, timed: one full calibration step (full_step), else one forward
+    with the step's time extrapolated by the ratio of the step's algorithmic flops to the forward's."""
+    import torch
+    if full_step:
+        yfp = _oracle_yfp(shape, W, x)
+        it = _oracle_pieces(shape, W, th, x, yfp)
+        secs = sum(next(it)[1] for _ in PIECES)
+        return dict(value=shape.T / secs, unit=UNIT, cores=torch.get_num_threads(), kind="oracle",
+                    sample="one full fp64 oracle calibration step (forward, loss, STE backward; %.1f s) at %d tokens"
+                           % (secs, shape.T), seconds=secs)
+    secs = _oracle_forward_seconds(shape, W, th, x)
+    ratio = algorithmic_flops(shape) / algorithmic_forward_flops(shape)
+    return dict(value=shape.T / (secs * ratio), unit=UNIT, cores=torch.get_num_threads(), kind="oracle",
+                sample="extrapolated: one fp64 oracle forward of the quantized block (%.1f s) at %d tokens, times the "
+                       "ratio %.2f of the step's algorithmic flops to the forward's" % (secs, shape.T, ratio),
+                seconds=secs * ratio)
 
 
 def run_reference(args, shape):
     ws, rank, _ = _dist()
     if rank != 0:
         return 0
-    import numpy as np
+    import torch
     from paper_2308_13137_gb300 import inputs as I
     W = I.make_block_weights(shape, seed=1)
     x = I.make_block_input(shape, 0, 1)
     th = I.make_block_theta(shape, W, x, seed=2)
-    it = _oracle_sampler(shape, W, th, x)
+    it = _oracle_pieces(shape, W, th, x, _oracle_yfp(shape, W, x))
     for _ in range(args.warmup):
         next(it)
+    per = {p: [] for p in PIECES}
     t0 = time.perf_counter()
-    eq = 0.0
-    for _ in range(args.steps):
-        eq += next(it)[1]
+    k = 0
+    # time K pieces, and at least one of each so that every part of the step is measured
+    while k < args.steps or any(not v for v in per.values()):
+        name, dt = next(it)
+        per[name].append(dt)
+        k += 1
     wall = time.perf_counter() - t0
-    import torch
-    value = shape.T * (args.steps / 7.0) / eq
-    sample = ("each step: one fp64 oracle calibration step of a 128-output-channel slice of one block "
-              "projection (cycling q,k,v,o,gate,up,down) at %d tokens; value scales each slice's time by "
-              "Cout/128 to whole projections (attention and norms not sampled)" % shape.T)
+    step_s = sum(statistics.mean(v) for v in per.values())
+    value = shape.T / step_s
+    sample = ("each step one piece of the fp64 oracle's calibration step (the five forward stages, the loss, the five "
+              "stage backwards, in a step's order); value = %d tokens / the sum of the pieces' mean times (%d pieces "
+              "timed)" % (shape.T, k))
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": 1e3 * wall / args.steps, "higher_is_better": True,
+            "warmup": args.warmup, "ms_per_step": 1e3 * step_s, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": shape.name, "tokens_per_step": shape.T, "wbits": shape.wbits,
                        "abits": shape.abits, "group": shape.group, "let": shape.let},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": torch.get_num_threads(), "kind": "oracle",
                              "sample": sample},
-            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "wall_s": wall}
     print(json.dumps(line), flush=True)
     return 0
 
@@ -234,6 +306,14 @@ def algorithmic_flops(shape) -> float:
     lin = 2 * T * P * 2 + 2 * T * (P if shape.let else P - P_qkv)
     attn = 3 * 2 * shape.head_dim * H * T * (T + 1)
     return float(lin + attn)
+
+
+def algorithmic_forward_flops(shape) -> float:
+    """Flops of one forward of the quantized block: each linear's product (2 T P) and the causal
+    attention's two products (2 * 128 H T (T+1))."""
+    T, d, f, dq, dkv, H = shape.T, shape.d, shape.ffn, shape.dq, shape.dkv, shape.n_heads
+    P = d * (dq + 2 * dkv) + d * dq + 3 * d * f
+    return float(2 * T * P + 2 * shape.head_dim * H * T * (T + 1))
 
 
 def _gemm_traffic():
@@ -270,13 +350,16 @@ def run_ours(args, shape):
     W = I.make_block_weights(shape, seed=seeds["weights"])
     n_samples = 4
     xs = [I.make_block_input(shape, sample=i, weight_seed=seeds["weights"]) for i in range(n_samples)]
-    th = I.make_block_theta(shape, W, xs[0], seed=seeds["theta"])
+    th = I.make_block_theta(shape, W, xs[0], seed=seeds["theta"], weight_seed=seeds["weights"])
     st = BlockState(shape, W, th, pbits=args.pbits)
     xd = [torch.from_numpy(x).cuda() for x in xs]
     yfp = [torch.empty_like(v) for v in xd]
     for v, y in zip(xd, yfp):          # Eq. 1 targets: the full-precision block (not timed)
         st.fp_forward(v, y)
+    if shape.let:                       # Algorithm 1's LET initialisation from the samples (not timed)
+        st.let_init(xd)
     torch.cuda.synchronize()
+    th_host = st.split_theta()          # the parameters the timed steps start from
 
     def step_eager(i):
         st.step(xd[i % n_samples], yfp[i % n_samples])
@@ -420,12 +503,9 @@ def run_ours(args, shape):
                    "samples": clk["samples"]},
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        v, wall, cores = _oracle_value(shape, W, th, xs[0], args.cpu_samples)
-        line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
-                                "sample": "%d oracle calibration steps (%.1f s) of 128-output-channel slices of "
-                                          "the block's projections, cycling q,k,v,o,gate,up,down at %d tokens; each "
-                                          "scaled by Cout/128 (attention and norms not sampled)" % (
-                                              args.cpu_samples, wall, shape.T)}
+        cb = cpu_baseline(shape, W, th_host, xs[0], full_step=shape.name not in FORWARD_ONLY_BASELINE)
+        cb.pop("seconds")
+        line["cpu_baseline"] = cb
     if rank == 0:
         print(json.dumps(line), flush=True)
     if ws > 1:
@@ -441,7 +521,6 @@ def main():
     ap.add_argument("--config", default=DEFAULT_CONFIG)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-samples", type=int, default=14)
     ap.add_argument("--pbits", type=int, default=16,
                     help="softmax-output bits (2..8: the quantized-softmax ablation; 16: not quantized, the default)")
     args = ap.parse_args()

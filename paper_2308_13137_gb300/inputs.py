@@ -18,11 +18,13 @@ same shapes and of the distributions below stand in for them:
   variance and then to std 0.02.
 * LWC logits: gamma_hat = beta_hat = 4.0 (sigmoid ~ 0.982); test cases can
   perturb them so that clipping is active.
-* LET parameters: s and delta of the [ln1,(q,k,v)] and [ln2,(gate,up)] pairs
-  follow the SmoothQuant-style recipe s = max|X|^0.5 / max|W|^0.5 and
-  delta = channel mean, taken over a per-token RMS-normalised copy of the
-  sample's block input (the RMSNorm gain is one).  The [v,o] pair and the Q/K
-  scale start near identity with a small seeded perturbation.
+* LET parameters, drawn rather than computed: per-channel scales exp(N(0, 0.1))
+  times sqrt(outlier factor) on the generator's own outlier channels (the
+  magnitude pattern a smoothing initialisation gives them), shifts N(0, 0.05);
+  the [v, o] pair and the Q/K scale start near identity with a small seeded
+  perturbation.  The method's own initialisation (SmoothQuant-style scales and
+  channel means of the block's statistics) is computed by the library's LET
+  initialisation and by the oracle, not here.
 """
 from __future__ import annotations
 
@@ -176,16 +178,13 @@ def make_block_input(shape: BlockShape, sample: int = 0, weight_seed: int = 1) -
     return x
 
 
-def _rms_normalised(x: np.ndarray, eps: float) -> np.ndarray:
-    x64 = x.astype(np.float64)
-    return x64 / np.sqrt(np.mean(x64 * x64, axis=1, keepdims=True) + eps)
-
-
 def make_block_theta(shape: BlockShape, weights: Dict[str, np.ndarray], x: Optional[np.ndarray] = None,
-                     seed: int = 2, perturb: bool = False) -> Dict[str, np.ndarray]:
-    """Learnable parameters Theta1 (LWC logits per linear) and Theta2 (LET s, delta, s_a).
+                     seed: int = 2, perturb: bool = False, weight_seed: int = 1) -> Dict[str, np.ndarray]:
+    """Learnable parameters Theta1 (LWC logits per linear) and Theta2 (LET s, delta, s_a), drawn.
 
-    `perturb` spreads the LWC logits so that clipping is active in many groups (test cases)."""
+    `perturb` spreads the LWC logits so that clipping is active in many groups (test cases).
+    `x` is not used (kept for call compatibility); `weight_seed` selects the outlier channels that
+    make_block_input scaled."""
     rng = _rng(seed)
     th: Dict[str, np.ndarray] = {}
     for name in ("wq", "wk", "wv", "wo", "wg", "wu", "wd"):
@@ -199,19 +198,13 @@ def make_block_theta(shape: BlockShape, weights: Dict[str, np.ndarray], x: Optio
         th["gamma_" + name[1:]] = g
         th["beta_" + name[1:]] = b
     if shape.let:
-        if x is None:
-            x = make_block_input(shape, 0)
-        a = _rms_normalised(x, shape.rms_eps)
-        xmax = np.maximum(np.abs(a).max(axis=0), 1e-5)
-
-        def smooth(ws):
-            wmax = np.maximum(np.max([np.abs(wi).max(axis=0) for wi in ws], axis=0), 1e-5)
-            return np.maximum(np.sqrt(xmax) / np.sqrt(wmax), 1e-5).astype(np.float32)
-
-        th["s1"] = smooth([weights["wq"], weights["wk"], weights["wv"]])
-        th["d1"] = a.mean(axis=0).astype(np.float32)
-        th["s2"] = smooth([weights["wg"], weights["wu"]])
-        th["d2"] = a.mean(axis=0).astype(np.float32)
+        ch = _outlier_channels(shape, weight_seed)
+        boost = np.ones(shape.d, np.float32)
+        boost[ch] = np.float32(math.sqrt(shape.outlier_scale))
+        th["s1"] = (np.exp(rng.normal(0.0, 0.1, shape.d)) * boost).astype(np.float32)
+        th["d1"] = rng.normal(0.0, 0.05, shape.d).astype(np.float32)
+        th["s2"] = (np.exp(rng.normal(0.0, 0.1, shape.d)) * boost).astype(np.float32)
+        th["d2"] = rng.normal(0.0, 0.05, shape.d).astype(np.float32)
         th["so"] = np.exp(rng.normal(0.0, 0.1, shape.dkv)).astype(np.float32)
         th["do"] = rng.normal(0.0, 0.01, shape.dkv).astype(np.float32)
         th["sa"] = np.exp(rng.normal(0.0, 0.1, shape.dkv)).astype(np.float32)

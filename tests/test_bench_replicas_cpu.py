@@ -64,3 +64,27 @@ def test_job_throughput_and_replicas():
     w1 = I.make_block_weights(shape, seed=bench.replica_seeds(1)["weights"])
     assert w0.keys() == w1.keys()
     assert all(w0[k].shape == w1[k].shape and not np.array_equal(w0[k], w1[k]) for k in w0)
+
+
+def test_oracle_baseline_pieces_are_one_block_step():
+    """The CPU baseline times the oracle's step cut into eleven pieces (five forward stages, the loss,
+    five stage backwards); one pass over them must be exactly the oracle's block_step: same loss,
+    same gradient of every parameter."""
+    import torch
+    import bench
+    import oracle as O
+    from paper_2308_13137_gb300 import inputs as I
+    shape = I.BlockShape("tiny", T=16, d=64, n_heads=2, n_kv=1, ffn=96, wbits=4, abits=4, group=0, let=1,
+                         head_dim=32)
+    W = I.make_block_weights(shape, seed=1)
+    x = I.make_block_input(shape, sample=0, weight_seed=1)
+    th = I.make_block_theta(shape, W, x, seed=2, perturb=True)
+    yfp = bench._oracle_yfp(shape, W, x)
+    out = {}
+    it = bench._oracle_pieces(shape, W, th, x, yfp, out)
+    names = [next(it)[0] for _ in bench.PIECES]
+    assert names == bench.PIECES
+    ref = O.block_step(x, yfp, W, th, O.BlockCfg.from_shape(shape))
+    assert abs(float(out["loss"]) - float(ref["loss"])) <= 1e-12 * float(ref["loss"])
+    for n in O.THETA_NAMES_LWC + O.THETA_NAMES_LET:
+        assert torch.allclose(out["d" + n], ref["d" + n], rtol=1e-9, atol=1e-15), n
