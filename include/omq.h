@@ -307,10 +307,11 @@ typedef struct {
   int64_t m_hat, m_h, m_z;         /* bf16 [T, ffn]: Q_a(silu(gate) up), the down_proj input */
   int64_t w_hat[4], w_h[4], w_z[4];
   int64_t dy;                      /* fp32 [T, d]: dL/dy */
-  int64_t dy_gu;                   /* fp32 [T, 2 ffn]: dL/d(gate | up) */
-  int64_t dh1;                     /* fp32 [T, d]: dL/dh1 (both paths) */
+  /* the intermediate gradients below are bf16, the operand of the products that take them (R13) */
+  int64_t dy_gu;                   /* bf16 [T, 2 ffn]: dL/d(gate | up) */
+  int64_t dh1;                     /* bf16 [T, d]: dL/dh1 (both paths) */
   int64_t do_bf16;                 /* bf16 [T, nh*128]: dL/dO through Q_a, the attention backward's operand */
-  int64_t dy_qkv;                  /* fp32 [T, nh*128 + 2*nkv*128]: dL/d(q|k|v before RoPE) */
+  int64_t dy_qkv;                  /* bf16 [T, nh*128 + 2*nkv*128]: dL/d(q|k|v before RoPE) */
 } omq_block_saved;
 omq_status omq_block_saved_layout(const omq_block_shape* shape, const omq_qcfg* cfg, omq_block_saved* out);
 

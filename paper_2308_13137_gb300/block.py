@@ -120,8 +120,8 @@ class BlockState:
                     o_h=(f32, (T,)), o_z=(i32, (T,)), h1=(f32, (T, d)), b_hat=(bf, (T, d)), b_h=(f32, (T,)),
                     b_z=(i32, (T,)), y_gu=(f32, (T, 2 * f)), m_hat=(bf, (T, f)), m_h=(f32, (T,)), m_z=(i32, (T,)))
         if backward:
-            spec.update(dy=(f32, (T, d)), dy_gu=(f32, (T, 2 * f)), dh1=(f32, (T, d)), do_bf16=(bf, (T, sh.dq)),
-                        dy_qkv=(f32, (T, nqkv)))
+            spec.update(dy=(f32, (T, d)), dy_gu=(bf, (T, 2 * f)), dh1=(bf, (T, d)), do_bf16=(bf, (T, sh.dq)),
+                        dy_qkv=(bf, (T, nqkv)))
 
         def view(off, dtype, shp):
             n = int(np.prod(shp)) * torch.empty(0, dtype=dtype).element_size()

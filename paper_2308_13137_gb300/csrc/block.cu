@@ -68,13 +68,13 @@ struct BlockWS {
   float* dy; bf16* dy_b;
   float* dm;
   float* dW;
-  float* dYgu; bf16* dYgu_b;
+  bf16* dYgu_b;                     // dL/d(gate|up), bf16 (the products' operand; fp32 is not kept)
   float* db;
-  float* dh1; bf16* dh1_b;
+  bf16* dh1_b;
   float* dOh; bf16* dO_b;
   float* Drow;                      // [H, T] rowsum(dO * O)
   float* pqb;                       // [H, T, 4] softmax-output quantizer backward rows (pbits on only)
-  float* dQKV; float* dYqkv; bf16* dYqkv_b;
+  float* dQKV; bf16* dYqkv_b;
   float* da;
   float *dB_qkv, *dB_o, *dB_gu, *dr_qkv;
   float *vtmp0, *vtmp1, *vtmp2;     // [max(d, dq)] scratch vectors
@@ -134,17 +134,14 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   w.dy_b = c.take<bf16>(T * d);
   w.dm = c.take<float>(T * f);
   w.dW = c.take<float>(imax64(imax64(nqkv * d, d * dq), imax64(2 * f * d, d * f)));
-  w.dYgu = c.take<float>(T * 2 * f);
   w.dYgu_b = c.take<bf16>(T * 2 * f);
   w.db = c.take<float>(T * d);
-  w.dh1 = c.take<float>(T * d);
   w.dh1_b = c.take<bf16>(T * d);
   w.dOh = c.take<float>(T * dq);
   w.dO_b = c.take<bf16>(T * dq);
   w.Drow = c.take<float>(H * T4);
   w.pqb = flash_pq_on(cfg.pbits) ? c.take<float>(H * T4 * 4) : nullptr;
   w.dQKV = c.take<float>(T * nqkv);
-  w.dYqkv = c.take<float>(T * nqkv);
   w.dYqkv_b = c.take<bf16>(T * nqkv);
   w.da = c.take<float>(T * d);
   w.dB_qkv = c.take<float>(nqkv);
@@ -449,12 +446,14 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   ActBwdArgs bm{};
   bm.producer = AP_SWIGLU; bm.X = w.Ygu; bm.ldx = 2 * c.f; bm.U = w.Ygu + c.f; bm.ldu = 2 * c.f; bm.T = c.T; bm.C = c.f;
   bm.h = w.sm.h; bm.z = w.sm.z; bm.imax = w.sm.imax; bm.imin = w.sm.imin; bm.dXq = w.dm; bm.lddq = c.f;
-  bm.dX = w.dYgu; bm.lddx = 2 * c.f; bm.dXb = w.dYgu_b; bm.lddxb = 2 * c.f; bm.dU = w.dYgu + c.f; bm.dUb = w.dYgu_b + c.f;
+  bm.dX = nullptr; bm.lddx = 2 * c.f; bm.dXb = w.dYgu_b; bm.lddxb = 2 * c.f; bm.dU = nullptr; bm.dUb = w.dYgu_b + c.f;
   bm.rows_per_cta = 1; bm.abits = cfg.abits; bm.eps = cfg.h_eps;
   OMQ_TRY(act_bwd_launch(st, bm));
 
   // ---- gate / up ----------------------------------------------------------------------------------
-  if (c.let) OMQ_TRY(colsum_rows(st, w.dYgu, c.T, 2 * c.f, 2 * c.f, w.part, w.dB_gu, 1.f, 0));
+  // LET bias gradient dB~ = sum_t dY: the column sums of the bf16 gradient, the operand every product of
+  // this backward takes (R13)
+  if (c.let) OMQ_TRY(colsum_rows_bf16(st, w.dYgu_b, c.T, 2 * c.f, 2 * c.f, w.part, w.dB_gu, 1.f, 0));
   OMQ_TRY(join(st, ax, ev[5]));
   OMQ_TRY(lwc_bwd_dw(ax, c.T, w.dYgu_b, w.b_h, Wgu, 2 * c.f, c.d, cfg, c.let ? th->s2 : nullptr, nullptr,
                      th->gamma_gu, th->beta_gu, w.sq_gu, g->gamma_gu, g->beta_gu, nullptr,
@@ -465,7 +464,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   ActBwdArgs bb{};
   bb.producer = AP_RMS_LET; bb.X = w.h1; bb.ldx = c.d; bb.s = c.let ? th->s2 : nullptr; bb.delta = c.let ? th->d2 : nullptr;
   bb.rstd = w.rstd2; bb.T = c.T; bb.C = c.d; bb.h = w.sb.h; bb.z = w.sb.z; bb.imax = w.sb.imax; bb.imin = w.sb.imin;
-  bb.dXq = w.db; bb.lddq = c.d; bb.dX = w.dh1; bb.lddx = c.d; bb.dXb = w.dh1_b; bb.lddxb = c.d; bb.resid = w.dy;
+  bb.dXq = w.db; bb.lddq = c.d; bb.dX = nullptr; bb.lddx = c.d; bb.dXb = w.dh1_b; bb.lddxb = c.d; bb.resid = w.dy;
   bb.part_s = c.let ? w.part : nullptr; bb.part_d = c.let ? w.part + ((c.T + 3) / 4) * c.d : nullptr;
   bb.rows_per_cta = 4; bb.abits = cfg.abits; bb.eps = cfg.h_eps;
   OMQ_TRY(act_bwd_launch(st, bb));
@@ -476,7 +475,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   }
 
   // ---- o_proj -------------------------------------------------------------------------------------
-  if (c.let) OMQ_TRY(colsum_rows(st, w.dh1, c.T, c.d, c.d, w.part, w.dB_o, 1.f, 0));
+  if (c.let) OMQ_TRY(colsum_rows_bf16(st, w.dh1_b, c.T, c.d, c.d, w.part, w.dB_o, 1.f, 0));
   OMQ_TRY(join(st, ax, ev[7]));
   // ds_o, ddelta_o per query channel; with one query head per kv head straight into the gradients
   const bool fold_o = c.rep > 1;
@@ -505,7 +504,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   qa.T = (int)c.T; qa.H = (int)c.H; qa.Hkv = (int)c.Hkv; qa.hd = (int)c.hd; qa.Y = w.Yqkv; qa.ldy = c.nqkv; qa.cs = w.cs;
   qa.sa_exp = c.let ? sa_e : nullptr; qa.sa = c.let ? th->sa : nullptr;
   qa.h = w.sqkv.h; qa.z = w.sqkv.z; qa.imax = w.sqkv.imax; qa.imin = w.sqkv.imin; qa.abits = cfg.abits; qa.eps = cfg.h_eps;
-  qa.dQKV = w.dQKV; qa.ldd = c.nqkv; qa.dY = w.dYqkv; qa.dYb = w.dYqkv_b;
+  qa.dQKV = w.dQKV; qa.ldd = c.nqkv; qa.dY = nullptr; qa.dYb = w.dYqkv_b;
   const int64_t nsq = qkv_bwd_nslab((int)c.T);
   qa.part_q = c.let ? w.part : nullptr;
   qa.part_k = c.let ? w.part + nsq * c.dq : nullptr;
@@ -527,7 +526,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   }
 
   // ---- q / k / v projections ---------------------------------------------------------------------------
-  if (c.let) OMQ_TRY(colsum_rows(st, w.dYqkv, c.T, c.nqkv, c.nqkv, w.part, w.dB_qkv, 1.f, 0));
+  if (c.let) OMQ_TRY(colsum_rows_bf16(st, w.dYqkv_b, c.T, c.nqkv, c.nqkv, w.part, w.dB_qkv, 1.f, 0));
   OMQ_TRY(join(st, ax, ev[9]));
   OMQ_TRY(lwc_bwd_dw(ax, c.T, w.dYqkv_b, w.a_h, Wqkv, c.nqkv, c.d, cfg, c.let ? th->s1 : nullptr,
                      c.let ? w.r_qkv : nullptr, th->gamma_qkv, th->beta_qkv, w.sq_qkv, g->gamma_qkv, g->beta_qkv,
@@ -616,8 +615,8 @@ omq_status omq_block_saved_layout(const omq_block_shape* shape, const omq_qcfg* 
   for (int i = 0; i < 4; ++i) {
     out->w_hat[i] = off(wh[i]); out->w_h[i] = off(sq[i]->h); out->w_z[i] = off(sq[i]->z);
   }
-  out->dy = off(w.dy); out->dy_gu = off(w.dYgu); out->dh1 = off(w.dh1); out->do_bf16 = off(w.dO_b);
-  out->dy_qkv = off(w.dYqkv);
+  out->dy = off(w.dy); out->dy_gu = off(w.dYgu_b); out->dh1 = off(w.dh1_b); out->do_bf16 = off(w.dO_b);
+  out->dy_qkv = off(w.dYqkv_b);
   return OMQ_OK;
 }
 

@@ -115,9 +115,9 @@ __device__ __forceinline__ void lwc_elems(const uint4 (&wc)[4], const float* s_n
   for (int i = 0; i < 4; ++i) {
     float w8[8], s8[8];
     unpack_bf16x8(wc[i], w8);
-    if (HS) {
-      const float4 a = __ldg(reinterpret_cast<const float4*>(s_nb) + 2 * i);
-      const float4 b = __ldg(reinterpret_cast<const float4*>(s_nb) + 2 * i + 1);
+    if (HS) {                                    // the tile's column scales, staged in shared memory
+      const float4 a = reinterpret_cast<const float4*>(s_nb)[2 * i];
+      const float4 b = reinterpret_cast<const float4*>(s_nb)[2 * i + 1];
       s8[0] = a.x; s8[1] = a.y; s8[2] = a.z; s8[3] = a.w; s8[4] = b.x; s8[5] = b.y; s8[6] = b.z; s8[7] = b.w;
     }
 #pragma unroll
@@ -155,9 +155,13 @@ __device__ __forceinline__ void release_acc(uint64_t* acc_empty, uint32_t buf, i
 
 // Eight epilogue warps: warps w and w+4 drain the same 32 accumulator rows (lane quadrant w % 4),
 // `half` 0 the first BN / 2 columns of the tile, 1 the others; each keeps its own row partials.
+// Each warp stages the LET column scales of its half tile in its own 512 bytes of `s_stage` (the
+// fp32 output staging area, unused here), and issues the loads of its rows' quantizer state and
+// first weight chunk before it waits for the accumulator, so their latency overlaps the mainloop.
 template <int BN, bool PAIR, int FORM>
 __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem, uint64_t* acc_full, uint64_t* acc_empty,
-                                             volatile int* abort_flag, int q, int half, int lane, int total, int rank) {
+                                             volatile int* abort_flag, int q, int half, int lane, int total, int rank,
+                                             float* s_stage) {
   constexpr int HB = BN / 2;                      // columns of a half
   const GemmLwcEpi& L = p.lw;
   const int N = p.N;
@@ -172,11 +176,6 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
     const bool has_acc = ti.nkb > 0;
     const uint32_t buf = acc_it & 1;
     bool ok = true;
-    if (has_acc) {
-      ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[buf], (acc_it >> 1) & 1, p.wait_ns));
-      if (!ok) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; }
-      tc_fence_after();
-    }
     const int row0 = ti.m0 + q * 32;
     const int row = row0 + lane;
     const bool row_ok = row < p.M;
@@ -197,6 +196,21 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
       qs.z = (float)L.z[gk];
       qs.b = L.gb[gk];
       qs.m = L.mv[gk];
+    }
+    if (FORM != 2 && L.s) {                       // this half tile's column scales -> shared memory
+      __syncwarp();                               // the previous tile's reads are done
+      const int c = ti.n0 + jb + 4 * lane;
+      const float4 sv = (4 * lane < HB && c < N) ? __ldg(reinterpret_cast<const float4*>(L.s + c))
+                                                 : make_float4(1.f, 1.f, 1.f, 1.f);
+      if (4 * lane < HB) reinterpret_cast<float4*>(s_stage)[lane] = sv;
+      __syncwarp();
+    }
+    if (has_acc) {
+      ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[buf], (acc_it >> 1) & 1, p.wait_ns));
+      if (!ok) { omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; }
+      tc_fence_after();
+    }
+    if (perch && row_ok) {
       qs.rh = __frcp_rn(qs.h);
       qs.u = __fmul_rn(__fmul_rn(qs.b, qs.m), qs.rh);
     }
@@ -227,8 +241,8 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
         // without LET only the STE part; with it every term (an absent s or r is 1: products by it
         // are exact)
         if (FORM == 2) lwc_elems<false, false, false, false>(wcur, nullptr, rr, dbr, qs, L.Q, g, Gh, Gbm, drm, cs, cd);
-        else if (FORM == 3) lwc_elems<true, false, false, true>(wcur, L.s + nb, rr, dbr, qs, L.Q, g, Gh, Gbm, drm, cs, cd);
-        else if (L.s) lwc_elems<true, true, true, true>(wcur, L.s + nb, rr, dbr, qs, L.Q, g, Gh, Gbm, drm, cs, cd);
+        else if (FORM == 3) lwc_elems<true, false, false, true>(wcur, s_stage + (j0 - jb), rr, dbr, qs, L.Q, g, Gh, Gbm, drm, cs, cd);
+        else if (L.s) lwc_elems<true, true, true, true>(wcur, s_stage + (j0 - jb), rr, dbr, qs, L.Q, g, Gh, Gbm, drm, cs, cd);
         else lwc_elems<false, true, true, true>(wcur, nullptr, rr, dbr, qs, L.Q, g, Gh, Gbm, drm, cs, cd);
         const int64_t prow = (int64_t)(row0 >> 5) * N + nb + lane;
         if (L.part_s) {
@@ -427,7 +441,8 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
       mbar_wait(drain, 0, p.wait_ns);
     }
   } else if (LWC && warp >= 2) {
-    lwc_epilogue<BN, PAIR, LWC>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, (warp - 2) >> 2, lane, total, rank);
+    lwc_epilogue<BN, PAIR, LWC>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, (warp - 2) >> 2, lane, total, rank,
+                                reinterpret_cast<float*>(smem + L::EPI_OFF) + (warp - 2) * (BN / 2));
   } else if (warp >= 2) {
     // ---------------- epilogue ----------------
     // fp32 output leaves through TMA bulk stores: each warp stages its 32 x 32 block in one of two

@@ -913,6 +913,62 @@ __global__ void __launch_bounds__(256) colsum_rows_vec_kernel(const float* __res
 
 int64_t colsum_rows_parts(int64_t T) { return (T + 127) / 128; }
 
+// part[p, c] = sum of the bf16 X[t, c] (in fp32) over the 128 rows t of slab p; each thread sums 8
+// columns (one 16-byte load per row), the eight warps of a CTA stride the slab's rows
+__global__ void __launch_bounds__(256) colsum_rows_bf16_kernel(const __nv_bfloat16* __restrict__ X, int64_t T,
+                                                               int64_t N, int64_t ldx, float* __restrict__ part) {
+  __shared__ float red[8][32][9];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t c = (int64_t)blockIdx.x * 256 + 8 * lane;
+  const int64_t t0 = (int64_t)blockIdx.y * 128, t1 = min(T, t0 + 128);
+  float s[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (c < N) {
+    int64_t t = t0 + w;
+    for (; t + 24 < t1; t += 32) {
+      uint4 v[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) v[i] = __ldg(reinterpret_cast<const uint4*>(X + (t + 8 * i) * ldx + c));
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        float f[8];
+        unpack_bf16x8(v[i], f);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) s[e] += f[e];
+      }
+    }
+    for (; t < t1; t += 8) {
+      float f[8];
+      unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(X + t * ldx + c)), f);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) s[e] += f[e];
+    }
+  }
+#pragma unroll
+  for (int e = 0; e < 8; ++e) red[w][lane][e] = s[e];
+  __syncthreads();
+  if (w == 0 && c < N) {
+    float r[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) r[e] = red[0][lane][e];
+#pragma unroll
+    for (int k = 1; k < 8; ++k)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) r[e] += red[k][lane][e];
+    float4* dst = reinterpret_cast<float4*>(part + (int64_t)blockIdx.y * N + c);
+    dst[0] = make_float4(r[0], r[1], r[2], r[3]);
+    dst[1] = make_float4(r[4], r[5], r[6], r[7]);
+  }
+}
+
+omq_status colsum_rows_bf16(cudaStream_t st, const __nv_bfloat16* X, int64_t T, int64_t N, int64_t ldx, float* part,
+                            float* out, float scale, int accumulate) {
+  OMQ_REQUIRE(N % 8 == 0 && ldx % 8 == 0 && omq_aligned16(X) && omq_aligned16(part), OMQ_ERR_ALIGN);
+  dim3 grid((unsigned)((N + 255) / 256), (unsigned)colsum_rows_parts(T));
+  colsum_rows_bf16_kernel<<<grid, 256, 0, st>>>(X, T, N, ldx, part);
+  OMQ_LAUNCH_CHECK();
+  return omq_colsum_partials(st, part, colsum_rows_parts(T), N, out, scale, accumulate);
+}
+
 omq_status colsum_rows(cudaStream_t st, const float* X, int64_t T, int64_t N, int64_t ldx, float* part,
                        float* out, float scale, int accumulate) {
   if (N % 4 == 0 && ldx % 4 == 0 && omq_aligned16(X) && omq_aligned16(part)) {

@@ -84,6 +84,9 @@ omq_status act_bwd_launch(cudaStream_t st, const ActBwdArgs& a);
 omq_status colsum_rows(cudaStream_t st, const float* X, int64_t T, int64_t N, int64_t ldx,
                        float* part, float* out, float scale, int accumulate);
 int64_t colsum_rows_parts(int64_t T);
+// the same over a bf16 array (each value widened exactly); N and ldx multiples of 8
+omq_status colsum_rows_bf16(cudaStream_t st, const __nv_bfloat16* X, int64_t T, int64_t N, int64_t ldx, float* part,
+                            float* out, float scale, int accumulate);
 
 omq_status loss_launch(cudaStream_t st, int64_t n, const float* Yq, const float* Yfp, float* loss,
                        float* dY, __nv_bfloat16* dYb, float* part);

@@ -994,8 +994,10 @@ __device__ __forceinline__ void qkv_bwd_body(const QkvArgs& a, float* fsm) {
           o1[e] = rope ? d1 * cv[e] + d2 * sv[e] : d1;
           o2[e] = rope ? d2 * cv[e] - d1 * sv[e] : d2;
         }
-        *reinterpret_cast<float4*>(dy + e1) = make_float4(o1[0], o1[1], o1[2], o1[3]);
-        *reinterpret_cast<float4*>(dy + e1 + 64) = make_float4(o2[0], o2[1], o2[2], o2[3]);
+        if (a.dY) {
+          *reinterpret_cast<float4*>(dy + e1) = make_float4(o1[0], o1[1], o1[2], o1[3]);
+          *reinterpret_cast<float4*>(dy + e1 + 64) = make_float4(o2[0], o2[1], o2[2], o2[3]);
+        }
         st_bf16x4(dyb + e1, o1);
         st_bf16x4(dyb + e1 + 64, o2);
       }
@@ -1047,7 +1049,7 @@ __device__ __forceinline__ void qkv_bwd_body(const QkvArgs& a, float* fsm) {
         }
         const float o1 = rope ? d1 * cv + d2 * sv : d1;
         const float o2 = rope ? d2 * cv - d1 * sv : d2;
-        dy[first] = o1; dy[first + 64] = o2;
+        if (a.dY) { dy[first] = o1; dy[first + 64] = o2; }
         dyb[first] = f_to_bf16(o1); dyb[first + 64] = f_to_bf16(o2);
       }
     }
