@@ -33,6 +33,21 @@ def rel(a, b) -> float:
     return float((a - b).norm() / b.norm().clamp_min(1e-300))
 
 
+def grad_errors(got, ref, names):
+    """{d<name>: relative error} over parameter gradients; a gradient that is zero by structure in
+    the reference (one token: the softmax of a single key has no gradient, so d s_a = 0 exactly) is
+    measured by its size against the largest reference gradient instead."""
+    scale = max([float(torch.as_tensor(ref["d" + n]).double().norm()) for n in names] + [1e-300])
+    out = {}
+    for n in names:
+        r = torch.as_tensor(ref["d" + n]).double()
+        if float(r.norm()) > 1e-9 * scale:
+            out["d" + n] = rel(got["d" + n], r)
+        else:
+            out["d" + n] = float(torch.as_tensor(got["d" + n]).double().norm()) / scale
+    return out
+
+
 def fp32_band(mag, h, ulps: float):
     """Rounding band in quotient units of an fp32 value of magnitude `mag` formed with `ulps`
     single-precision roundings (each at most 2^-24 relative), divided by the step h."""

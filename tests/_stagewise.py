@@ -20,7 +20,7 @@ import torch
 import oracle as O
 from oracle.omq_oracle import _expand_kv
 from _parity import (GRAD_TOL, OUT_TOL, add_counts, check_codes, check_h, check_zero_points, code_counts, fp32_band,
-                     record, record_codes, rel)
+                     grad_errors, record, record_codes, rel)
 
 F64 = torch.float64
 
@@ -111,14 +111,7 @@ def compare_step(shape, W: Dict[str, np.ndarray], x: np.ndarray, th: Dict[str, n
     err["loss"] = abs(loss_gpu - float(lref)) / float(lref)
     err["bwd dy"] = rel(G["dy"], dyref)
 
-    # a gradient that is zero by structure (one token: softmax of a single key has no gradient,
-    # so d s_a = 0 exactly) is held to its size against the largest parameter gradient instead
-    gscale = max([float(gsum.norm()) for gsum in total] + [1e-300])
-    for n, gsum in zip(names, total):
-        if float(gsum.norm()) > 1e-9 * gscale:
-            err["d" + n] = rel(grads_gpu["d" + n], gsum)
-        else:
-            err["d" + n] = float(torch.as_tensor(grads_gpu["d" + n]).double().norm()) / gscale
+    err.update(grad_errors(grads_gpu, {"d" + n: gsum for n, gsum in zip(names, total)}, names))
     record("stage-wise", tag, **{k: float(v) for k, v in err.items()})
     bad = {k: v for k, v in err.items() if not v < (OUT_TOL if not (k.startswith("d") or k.startswith("bwd")) else GRAD_TOL)}
     if codes:

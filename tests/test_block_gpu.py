@@ -9,7 +9,7 @@ import pytest
 import torch
 
 import oracle as O
-from _parity import record
+from _parity import grad_errors, record
 from _stagewise import compare_step
 from paper_2308_13137_gb300 import inputs as I
 from paper_2308_13137_gb300.block import BlockState
@@ -72,7 +72,7 @@ def test_block_step_small(cuda_lib, shape):
     compare_step(shape, W, x, th, yfp, got["y"], got["loss"], grads, got["saved"], shape.name)
     errs = dict(y=_rel(got["y"], ref["y"]), loss=abs(got["loss"] - float(ref["loss"])) / float(ref["loss"]))
     names = O.THETA_NAMES_LWC + (O.THETA_NAMES_LET if shape.let else [])
-    errs.update({"d" + n: _rel(got["d" + n], ref["d" + n]) for n in names})
+    errs.update(grad_errors(got, ref, names))
     record("end to end", shape.name, **errs)
     assert errs["y"] < OUT_TOL and errs["loss"] < OUT_TOL, errs
     if shape.abits >= 16:
@@ -102,7 +102,7 @@ def test_block_step_softmax_quant(cuda_lib, shape, pbits):
                  pbits=pbits)
     names = O.THETA_NAMES_LWC + O.THETA_NAMES_LET
     errs = dict(y=_rel(got["y"], ref["y"]), loss=abs(got["loss"] - float(ref["loss"])) / float(ref["loss"]))
-    errs.update({"d" + n: _rel(got["d" + n], ref["d" + n]) for n in names})
+    errs.update(grad_errors(got, ref, names))
     record("end to end", f"{shape.name} softmax {pbits} bits", **errs)
     assert errs["y"] < OUT_TOL and errs["loss"] < OUT_TOL, errs
     if pbits == 2:

@@ -15,7 +15,7 @@ import pytest
 import torch
 
 import oracle as O
-from _parity import GRAD_TOL, OUT_TOL, check_codes, check_h, check_zero_points, record, rel
+from _parity import GRAD_TOL, OUT_TOL, check_codes, check_h, check_zero_points, grad_errors, record, rel
 from _stagewise import compare_step
 from paper_2308_13137_gb300 import _lib, inputs as I
 from paper_2308_13137_gb300.block import BlockState
@@ -204,6 +204,6 @@ def test_block_step_token_counts(cuda_lib, T):
     compare_step(shape, W, x, th, yfp, y.cpu(), float(st.loss.item()), grads, sv, shape.name)
     ref = O.block_step(x, yfp, W, th, cfg)
     errs = dict(y=rel(y.cpu(), ref["y"]), loss=abs(float(st.loss.item()) - float(ref["loss"])) / float(ref["loss"]))
-    errs.update({"d" + n: rel(grads["d" + n], ref["d" + n]) for n in O.THETA_NAMES_LWC + O.THETA_NAMES_LET})
+    errs.update(grad_errors(grads, ref, O.THETA_NAMES_LWC + O.THETA_NAMES_LET))
     record("end to end", shape.name, **errs)
     assert errs["y"] < OUT_TOL and errs["loss"] < OUT_TOL
