@@ -32,8 +32,6 @@ if ROOT not in sys.path:
 METRIC = "calibration tokens/sec per block (fwd+bwd, fused LWC+LET) and % of step roofline"
 UNIT = "tokens/s"
 DEFAULT_CONFIG = "llama7b_w4a4"
-# configurations whose full oracle step takes over a minute on the host: forward only, extrapolated
-FORWARD_ONLY_BASELINE = ("llama13b_w2a16_g64", "llama2_70b_w4a4_gqa")
 
 
 def _peaks():
@@ -201,42 +199,21 @@ def _oracle_pieces(shape, W, th, x, yfp, out=None):
         del q, k, v, qkv, Ob, h1, gt, up, gu, y, gE, gD, gC, gB, gA
 
 
-def _oracle_forward_seconds(shape, W, th, x):
-    """One oracle forward of the quantized block (no autograd), in seconds."""
-    import torch
-    import oracle as O
-    cfg = O.BlockCfg.from_shape(shape)
-    t = lambda v: torch.as_tensor(v).to(torch.float64)
-    Wd = {k: t(v) for k, v in W.items()}
-    tt = {k: t(v) for k, v in th.items()}
-    with torch.no_grad():
-        c = time.perf_counter()
-        O.block_forward(t(x), Wd, tt, cfg)
-        return time.perf_counter() - c
-
-
 def _oracle_yfp(shape, W, x):
     import oracle as O
     return O.block_fp_forward(x, W, O.BlockCfg.from_shape(shape)).float().numpy()
 
 
-def cpu_baseline(shape, W, th, x, full_step: bool):
-    """The oracle on the host cores, timed: one full calibration step (full_step), else one forward
-    with the step's time extrapolated by the ratio of the step's algorithmic flops to the forward's."""
+def cpu_baseline(shape, W, th, x):
+    """The oracle on the host cores, timed: one full calibration step (forward, loss, STE backward)
+    of the block at the workload's token count."""
     import torch
-    if full_step:
-        yfp = _oracle_yfp(shape, W, x)
-        it = _oracle_pieces(shape, W, th, x, yfp)
-        secs = sum(next(it)[1] for _ in PIECES)
-        return dict(value=shape.T / secs, unit=UNIT, cores=torch.get_num_threads(), kind="oracle",
-                    sample="one full fp64 oracle calibration step (forward, loss, STE backward; %.1f s) at %d tokens"
-                           % (secs, shape.T), seconds=secs)
-    secs = _oracle_forward_seconds(shape, W, th, x)
-    ratio = algorithmic_flops(shape) / algorithmic_forward_flops(shape)
-    return dict(value=shape.T / (secs * ratio), unit=UNIT, cores=torch.get_num_threads(), kind="oracle",
-                sample="extrapolated: one fp64 oracle forward of the quantized block (%.1f s) at %d tokens, times the "
-                       "ratio %.2f of the step's algorithmic flops to the forward's" % (secs, shape.T, ratio),
-                seconds=secs * ratio)
+    yfp = _oracle_yfp(shape, W, x)
+    it = _oracle_pieces(shape, W, th, x, yfp)
+    secs = sum(next(it)[1] for _ in PIECES)
+    return dict(value=shape.T / secs, unit=UNIT, cores=torch.get_num_threads(), kind="oracle",
+                sample="one full fp64 oracle calibration step (forward, loss, STE backward; %.1f s) at %d tokens"
+                       % (secs, shape.T), seconds=secs)
 
 
 def run_reference(args, shape):
@@ -308,14 +285,6 @@ def algorithmic_flops(shape) -> float:
     return float(lin + attn)
 
 
-def algorithmic_forward_flops(shape) -> float:
-    """Flops of one forward of the quantized block: each linear's product (2 T P) and the causal
-    attention's two products (2 * 128 H T (T+1))."""
-    T, d, f, dq, dkv, H = shape.T, shape.d, shape.ffn, shape.dq, shape.dkv, shape.n_heads
-    P = d * (dq + 2 * dkv) + d * dq + 3 * d * f
-    return float(2 * T * P + 2 * shape.head_dim * H * T * (T + 1))
-
-
 def _gemm_traffic():
     """DRAM bytes per GEMM launch from the committed ncu capture, if it was taken of this exact
     kernel source (else None)."""
@@ -351,7 +320,7 @@ def run_ours(args, shape):
     n_samples = 4
     xs = [I.make_block_input(shape, sample=i, weight_seed=seeds["weights"]) for i in range(n_samples)]
     th = I.make_block_theta(shape, W, xs[0], seed=seeds["theta"], weight_seed=seeds["weights"])
-    st = BlockState(shape, W, th, pbits=args.pbits)
+    st = BlockState(shape, W, th, pbits=args.pbits, wprep=args.wprep)
     xd = [torch.from_numpy(x).cuda() for x in xs]
     yfp = [torch.empty_like(v) for v in xd]
     for v, y in zip(xd, yfp):          # Eq. 1 targets: the full-precision block (not timed)
@@ -475,6 +444,8 @@ def run_ours(args, shape):
                    "tokens_per_step": shape.T, "hidden": shape.d,
                    "heads": shape.n_heads, "kv_heads": shape.n_kv, "ffn": shape.ffn, "wbits": shape.wbits,
                    "abits": shape.abits, "group": shape.group, "let": shape.let, "softmax_bits": args.pbits,
+                   "qkv_weight_operand": ("fake-quantized tile by tile in the GEMM's shared memory" if args.wprep
+                                          else "W_hat written to HBM by the LWC forward"),
                    "step": "LET+LWC fake-quant, block fwd, MSE loss, STE bwd, AdamW",
                    "launch": "each step replays a CUDA graph of its launches (one graph per input sample)",
                    "l2": "inputs larger than L2 (bf16 weights %.0f MB per block)" % (
@@ -503,9 +474,180 @@ def run_ours(args, shape):
                    "samples": clk["samples"]},
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        cb = cpu_baseline(shape, W, th_host, xs[0], full_step=shape.name not in FORWARD_ONLY_BASELINE)
+        cb = cpu_baseline(shape, W, th_host, xs[0])
         cb.pop("seconds")
         line["cpu_baseline"] = cb
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def run_reference_linear(args, lsh):
+    """The fp64 oracle's step of the single quantized linear on the host cores, one per step."""
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return 0
+    import torch
+    import oracle as O
+    from paper_2308_13137_gb300 import inputs as I
+    tt = {k: torch.from_numpy(v) for k, v in I.make_linear_case(lsh, seed=0).items()}
+    yfp = tt["X"].double() @ tt["W"].double().T
+
+    def one():
+        O.qlinear_step(tt["X"], tt["W"], tt["B"], tt["gamma_logit"], tt["beta_logit"], yfp, lsh.wbits, lsh.group, lsh.abits)
+
+    for _ in range(args.warmup):
+        one()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        one()
+    wall = time.perf_counter() - t0
+    value = lsh.T * args.steps / wall
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * wall / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": lsh.name, "tokens_per_step": lsh.T, "wbits": lsh.wbits, "abits": lsh.abits,
+                       "group": lsh.group, "let": 0},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": torch.get_num_threads(), "kind": "oracle",
+                             "sample": "each step one fp64 oracle calibration step of the linear"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_ours_linear(args, lsh):
+    """The single quantized linear (W4A16 g128, LWC only, Eq. 4 with Eq. 2): one step is the forward,
+    the MSE loss against the full-precision output, the STE backward to gamma_hat, beta_hat and the
+    AdamW update, replayed from a CUDA graph (the step is launch-bound at this size)."""
+    import numpy as np
+    import torch
+    ws, rank, local = _dist()
+    torch.cuda.set_device(local if ws > 1 else 0)
+    from paper_2308_13137_gb300 import _lib, inputs as I
+    _lib.lib()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    case = I.make_linear_case(lsh, seed=rank)
+    T, Cin, Cout = lsh.T, lsh.Cin, lsh.Cout
+    ng = Cin // lsh.group
+    cfg = _lib.make_cfg(wbits=lsh.wbits, abits=lsh.abits, group=lsh.group)
+    f32, bf = dict(device="cuda", dtype=torch.float32), dict(device="cuda", dtype=torch.bfloat16)
+    X = torch.from_numpy(case["X"]).cuda()
+    W = torch.from_numpy(case["W"]).cuda().to(torch.bfloat16)
+    B = torch.from_numpy(case["B"]).cuda()
+    Yfp = X @ W.float().T                       # Eq. 1 target: the full-precision output (not timed)
+    theta = torch.cat([torch.from_numpy(case["gamma_logit"]).reshape(-1), torch.from_numpy(case["beta_logit"]).reshape(-1)]).cuda()
+    grads = torch.zeros_like(theta)
+    m, v = torch.zeros_like(theta), torch.zeros_like(theta)
+    gl, bl = theta[:Cout * ng].view(Cout, ng), theta[Cout * ng:].view(Cout, ng)
+    dgl, dbl = grads[:Cout * ng].view(Cout, ng), grads[Cout * ng:].view(Cout, ng)
+    sv = dict(w_hat=torch.empty(Cout, Cin, **bf), h_w=torch.empty(Cout, ng, **f32),
+              z_w=torch.empty(Cout, ng, device="cuda", dtype=torch.int32),
+              imax_w=torch.empty(Cout, ng, device="cuda", dtype=torch.int32),
+              imin_w=torch.empty(Cout, ng, device="cuda", dtype=torch.int32), x_hat=torch.empty(T, Cin, **bf),
+              h_a=torch.empty(T, **f32), z_a=torch.empty(T, device="cuda", dtype=torch.int32),
+              imax_a=torch.empty(T, device="cuda", dtype=torch.int32), imin_a=torch.empty(T, device="cuda", dtype=torch.int32),
+              b_tilde=torch.empty(Cout, **f32))
+    saved = _lib.omq_qlinear_saved(*[sv[k].data_ptr() for k in ("w_hat", "h_w", "z_w", "imax_w", "imin_w", "x_hat",
+                                                                "h_a", "z_a", "imax_a", "imin_a", "b_tilde")])
+    Y = torch.empty(T, Cout, **f32)
+    dY = torch.empty(T, Cout, **f32)
+    loss = torch.zeros(1, **f32)
+    lws = torch.empty(_lib.omq_loss_workspace_size(T * Cout), device="cuda", dtype=torch.uint8)
+    qws = torch.empty(_lib.omq_qlinear_workspace_size(T, Cin, Cout, cfg), device="cuda", dtype=torch.uint8)
+    step_dev = torch.zeros(1, device="cuda", dtype=torch.int32)
+
+    def step(x):
+        _lib.omq_qlinear_fwd(T, Cin, Cout, x, W, B, None, None, gl, bl, Y, saved, cfg)
+        _lib.omq_block_loss(T * Cout, Y, Yfp, loss, dY, None, lws)
+        _lib.omq_qlinear_bwd(T, Cin, Cout, x, W, None, None, gl, bl, saved, dY, None, dgl, dbl, None, None, qws, cfg)
+        _lib.omq_step_advance(step_dev)
+        _lib.omq_adamw_update_dev(theta.numel(), theta, grads, m, v, 5e-3, 0.9, 0.999, 1e-8, 0.0, step_dev)
+
+    for _ in range(max(3, args.warmup)):
+        step(X)
+    torch.cuda.synchronize()
+    xin = torch.empty_like(X)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step(xin)
+    xin.copy_(X)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    reps = max(20, args.steps)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(0)
+    clocks.start()
+    time.sleep(0.3)
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(reps):
+        g.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms = max_over_ranks(e0.elapsed_time(e1), ws, "cuda")
+    value = job_throughput(ws, T, reps, ms / 1e3)
+    # GEMM rate from ordinary steps
+    _lib.omq_profile_begin()
+    l0 = _lib.omq_launch_count()
+    for _ in range(5):
+        step(X)
+    torch.cuda.synchronize()
+    gemm_ms, gemm_flops, gemm_n = _lib.omq_profile_end()
+    launches = (_lib.omq_launch_count() - l0) / 5
+    # end to end: X from pinned host memory each step, the loss read back
+    xh = torch.from_numpy(case["X"]).pin_memory()
+    lh = torch.zeros(1).pin_memory()
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        xin.copy_(xh, non_blocking=True)
+        g.replay()
+        lh.copy_(loss, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+    e2e_s = max_over_ranks(time.perf_counter() - t0, ws, "cuda")
+    peaks = _peaks()
+    F = 3 * 2.0 * T * Cin * Cout
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": reps, "warmup": args.warmup,
+        "ms_per_step": ms / reps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": lsh.name, "tokens_per_step": T, "Cin": Cin, "Cout": Cout, "wbits": lsh.wbits,
+                   "abits": lsh.abits, "group": lsh.group, "let": 0,
+                   "step": "LWC fake-quant, quantized linear fwd, MSE loss, STE bwd, AdamW",
+                   "launch": "each step replays a CUDA graph of its launches",
+                   "l2": "inputs smaller than L2 (the single-linear case is launch-bound)",
+                   "parallelism": "replicas" if ws > 1 else "single"},
+        "roofline": {"bound": "latency", "kernel": "gemm_bf16_kernel (tcgen05)", "achieved": gemm_flops / (gemm_ms / 1e3) / 1e12,
+                     "peak": peaks["bf16"], "unit": "TFLOP/s", "frac": gemm_flops / (gemm_ms / 1e3) / 1e12 / peaks["bf16"],
+                     "traffic": None, "peak_kind": "%s bf16_tflops burst" % peaks["src"],
+                     "note": "%.2e flop per step: far below what fills the GPU; the step is set by launch latency" % F},
+        "step_roofline": {"flops_per_step": F, "t_roof_ms": F / (peaks["bf16"] * 1e12) * 1e3,
+                          "frac": F / (peaks["bf16"] * 1e12) * 1e3 / (ms / reps)},
+        "e2e": {"value": job_throughput(ws, T, reps, e2e_s), "unit": UNIT, "h2d_bytes_per_step": X.numel() * 4,
+                "d2h_bytes_per_step": 4, "steps": reps},
+        "gpu_launches": int(round(launches * reps)),
+        "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"],
+                   "samples": clk["samples"]},
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        import oracle as O
+        tt = {k: torch.from_numpy(v) for k, v in case.items()}
+        yfp64 = tt["X"].double() @ tt["W"].double().T
+        n_rep, c = 5, time.perf_counter()
+        for _ in range(n_rep):
+            O.qlinear_step(tt["X"], tt["W"], tt["B"], tt["gamma_logit"], tt["beta_logit"], yfp64, lsh.wbits, lsh.group,
+                           lsh.abits)
+        secs = (time.perf_counter() - c) / n_rep
+        line["cpu_baseline"] = {"value": T / secs, "unit": UNIT, "cores": torch.get_num_threads(), "kind": "oracle",
+                                "sample": "fp64 oracle calibration step of the linear, mean of %d (%.3f s each)" % (
+                                    n_rep, secs)}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if ws > 1:
@@ -523,8 +665,14 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--pbits", type=int, default=16,
                     help="softmax-output bits (2..8: the quantized-softmax ablation; 16: not quantized, the default)")
+    ap.add_argument("--wprep", type=int, choices=[0, 1], default=0,
+                    help="q|k|v weight operand: 0 = W_hat materialised in HBM, 1 = fake-quantized inside the GEMM")
     args = ap.parse_args()
     from paper_2308_13137_gb300 import inputs as I
+    if isinstance(I.SHAPES.get(args.config), I.LinearShape):
+        if args.impl == "reference":
+            return run_reference_linear(args, I.SHAPES[args.config])
+        return run_ours_linear(args, I.SHAPES[args.config])
     shape = I.block_shape(args.config)
     if args.impl == "reference":
         return run_reference(args, shape)

@@ -64,6 +64,12 @@ typedef struct {
   int32_t* dev_status; /* optional device int32: 0 = ok, else an omq_status set by a kernel      */
   int32_t pbits;       /* softmax-output bits (the ablation beside Table A7): 2..8, or 0 / 16 = the
                           softmax output is not quantized (the method's default)                  */
+  int32_t wprep;       /* block step / forward only, where the weights are quantized: how the q|k|v
+                          products get W_hat (Eq. 2).  0 = the LWC forward writes W_hat (bf16) to
+                          HBM and the forward and dX products read it; 1 = both products read the
+                          raw bf16 weight and fake-quantize each tile in shared memory with the
+                          quantizer state the LWC forward wrote (W_hat never reaches HBM).  The two
+                          give bit-identical results; other entry points ignore the field.        */
 } omq_qcfg;
 
 /* ------------------------------------------------------------------------------------------
@@ -291,8 +297,8 @@ omq_status omq_block_step(omq_stream_t stream, const omq_block_shape* shape,
  * (int32) per token row; qkv_h / qkv_z hold the q, k and v rows one after the other ([3, T]).
  * Weight entries are indexed 0 = q|k|v, 1 = o, 2 = gate|up, 3 = down: w_hat bf16 [Cout, Cin]
  * (the fake-quantized LET-scaled weight, Eq. 2 and Eq. 3), w_h fp32 and w_z int32
- * [Cout, ngroups].  Returns OMQ_ERR_* for a shape or configuration omq_block_workspace_size
- * rejects. */
+ * [Cout, ngroups]; w_hat[0] is -1 under cfg->wprep = 1 (the q|k|v W_hat is then never formed).
+ * Returns OMQ_ERR_* for a shape or configuration omq_block_workspace_size rejects. */
 typedef struct {
   int64_t a_hat;                   /* bf16 [T, d]: Q_a((RMSNorm(x) - d1) / s1), the q|k|v input */
   int64_t a_h, a_z;

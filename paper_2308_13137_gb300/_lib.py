@@ -30,7 +30,8 @@ class OmqError(RuntimeError):
 
 class omq_qcfg(Structure):
     _fields_ = [("wbits", c_int32), ("abits", c_int32), ("group", c_int32), ("let", c_int32),
-                ("h_eps", c_float), ("accumulate", c_int32), ("dev_status", c_void_p), ("pbits", c_int32)]
+                ("h_eps", c_float), ("accumulate", c_int32), ("dev_status", c_void_p), ("pbits", c_int32),
+                ("wprep", c_int32)]
 
 
 class omq_qlinear_saved(Structure):
@@ -179,8 +180,9 @@ def check(name: str, code: int):
         raise OmqError(name, code)
 
 
-def make_cfg(wbits=4, abits=16, group=0, let=0, h_eps=1e-5, accumulate=0, dev_status=None, pbits=16) -> omq_qcfg:
-    return omq_qcfg(wbits, abits, group, int(let), h_eps, accumulate, ptr(dev_status), pbits)
+def make_cfg(wbits=4, abits=16, group=0, let=0, h_eps=1e-5, accumulate=0, dev_status=None, pbits=16,
+             wprep=0) -> omq_qcfg:
+    return omq_qcfg(wbits, abits, group, int(let), h_eps, accumulate, ptr(dev_status), pbits, int(wprep))
 
 
 # ------------------------------------------------------------------------------------------------

@@ -22,7 +22,7 @@ class BlockState:
 
     def __init__(self, shape, weights: Dict[str, np.ndarray], theta: Dict[str, np.ndarray], device: str = "cuda",
                  wbits: Optional[int] = None, abits: Optional[int] = None, group: Optional[int] = None,
-                 let: Optional[int] = None, pbits: int = 16):
+                 let: Optional[int] = None, pbits: int = 16, wprep: int = 0):
         import torch
         self.torch = torch
         self.shape = shape
@@ -32,6 +32,7 @@ class BlockState:
         self.group = shape.group if group is None else group
         self.let = shape.let if let is None else let
         self.pbits = pbits                 # softmax-output bits; 16 = not quantized (the default)
+        self.wprep = wprep                 # 1: the q|k|v products fake-quantize the raw weight tile by tile
         bf = torch.bfloat16
 
         def dev_bf16(a):
@@ -84,7 +85,8 @@ class BlockState:
         self.c_theta = self._params(self.theta)
         self.c_grads = self._params(self.grads)
         self.status = torch.zeros(1, dtype=torch.int32, device=device)
-        self.cfg = _lib.make_cfg(self.wbits, self.abits, self.group, self.let, 1e-5, 0, self.status, self.pbits)
+        self.cfg = _lib.make_cfg(self.wbits, self.abits, self.group, self.let, 1e-5, 0, self.status, self.pbits,
+                                 self.wprep)
         ws = _lib.omq_block_workspace_size(self.c_shape, self.cfg)
         if ws == 0:
             raise ValueError("block shape or configuration rejected by libomq")
@@ -130,7 +132,7 @@ class BlockState:
         out = {k: view(getattr(lay, k), dt, shp) for k, (dt, shp) in spec.items()}
         ng = lambda cin: 1 if self.group == 0 else cin // self.group
         lins = [(nqkv, d), (d, sh.dq), (2 * f, d), (d, f)]
-        out["w_hat"] = [view(lay.w_hat[i], bf, (co, ci)) for i, (co, ci) in enumerate(lins)]
+        out["w_hat"] = [None if lay.w_hat[i] < 0 else view(lay.w_hat[i], bf, (co, ci)) for i, (co, ci) in enumerate(lins)]
         out["w_h"] = [view(lay.w_h[i], f32, (co, ng(ci))) for i, (co, ci) in enumerate(lins)]
         out["w_z"] = [view(lay.w_z[i], i32, (co, ng(ci))) for i, (co, ci) in enumerate(lins)]
         return out
@@ -148,7 +150,12 @@ class BlockState:
     def step_adamw_graph(self, x, y_fp, lr_lwc: float = 5e-3, lr_let: float = 1e-2):
         """One calibration step and its AdamW update, replayed from a CUDA graph of the same launches
         (one graph per input pair (x, y_fp) and learning rates, captured on first use after one
-        ordinary step has set up the library's state).  The result equals step() + adamw()."""
+        ordinary step has set up the library's state).  The result equals step() + adamw().
+
+        A graph holds the device addresses it was captured with and is looked up by the addresses of
+        x and y_fp: a caller refills the same tensors in place between calls (new tensors, even of
+        equal contents, capture a new graph), and must keep them alive while this state may replay
+        it.  Weights, parameters, gradients and workspace are this object's own buffers."""
         torch = self.torch
         key = (x.data_ptr(), y_fp.data_ptr(), lr_lwc, lr_let)
         g = self._graphs.get(key)

@@ -89,7 +89,7 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   const int64_t T = s.T, d = s.d, hd = s.head_dim, H = s.n_heads, Hkv = s.n_kv, f = s.ffn;
   const int64_t dq = H * hd, dkv = Hkv * hd, nqkv = dq + 2 * dkv;
   auto ng = [&](int64_t cin) { return cfg.group == 0 ? (int64_t)1 : cin / cfg.group; };
-  w.Wqkv_h = c.take<bf16>(nqkv * d);
+  w.Wqkv_h = (cfg.wbits < 16 && cfg.wprep == 1) ? nullptr : c.take<bf16>(nqkv * d);   // wprep: never formed
   w.Wo_h = c.take<bf16>(d * dq);
   w.Wgu_h = c.take<bf16>(2 * f * d);
   w.Wd_h = c.take<bf16>(d * f);
@@ -211,6 +211,17 @@ omq_status gemm_dw(cudaStream_t st, int64_t T, int64_t Cout, int64_t Cin, const 
   return gemm_launch(st, Cout, Cin, T, 1, a, b, ep, 0, status);
 }
 
+// The q|k|v weight operand prepared inside the GEMM (omq_qcfg.wprep = 1): the raw weight with the
+// quantizer state of its LWC forward and, with LET, the column scale s1 and the row scale of the
+// v rows (1 / s_o, Eq. 5's [v, out] pair)
+GemmQuantB qkv_operand(const QState4& q, const omq_qcfg& cfg, int64_t d, const float* s, const float* r) {
+  GemmQuantB qb{};
+  qb.h = q.h; qb.z = q.z; qb.r = r; qb.s = s;
+  qb.group = cfg.group == 0 ? (int)d : cfg.group;
+  qb.Q = (float)((1 << cfg.wbits) - 1);
+  return qb;
+}
+
 LwcFwdArgs lwc_args(const bf16* W, int64_t Cout, int64_t Cin, const omq_qcfg& cfg, const float* s, const float* r,
                     const float* gl, const float* bl, bf16* Wq, const QState4& q, const float* bias_delta,
                     const float* bias_shift, float* Bt) {
@@ -321,8 +332,20 @@ struct Ctx {
   const omq_block_params* th;
   BlockWS ws;
   int64_t T, d, hd, H, Hkv, rep, f, dq, dkv, nqkv;
-  bool let, wq, aq;
+  bool let, wq, aq, wprep;
 };
+
+// da = dY_qkv W_hat_qkv (the gradient reaching the quantized attention input), from W_hat in HBM or
+// from the raw weight prepared tile by tile (omq_qcfg.wprep)
+omq_status qkv_dx(Ctx& c, int32_t* status) {
+  BlockWS& w = c.ws;
+  if (!c.wprep) return gemm_dx(c.st, c.T, c.nqkv, c.d, w.dYqkv_b, w.Wqkv_h, w.da, status);
+  GemmOperand a{w.dYqkv_b, c.nqkv, 0, 1}, b{c.w->wqkv, c.d, 0, 0};
+  GemmEpilogue ep{w.da, nullptr, c.d, 0, 1.f, nullptr, nullptr, 0, 0.f};
+  return gemm_launch_qb(c.st, c.T, c.d, c.nqkv, a, b, ep,
+                        qkv_operand(w.sq_qkv, c.cfg, c.d, c.let ? c.th->s1 : nullptr, c.let ? w.r_qkv : nullptr),
+                        status);
+}
 
 omq_status block_fwd(Ctx& c, const float* x, float* y) {
   cudaStream_t st = c.st;
@@ -354,7 +377,8 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   cudaEvent_t* ev = c.aux->ev;
   OMQ_TRY(join(st, ax, ev[0]));
   OMQ_TRY(lwc_fwd_launch(st, lwc_args(Wqkv, c.nqkv, c.d, cfg, c.let ? th->s1 : nullptr, c.let ? w.r_qkv : nullptr,
-                                      th->gamma_qkv, th->beta_qkv, w.Wqkv_h, w.sq_qkv, c.let ? th->d1 : nullptr,
+                                      th->gamma_qkv, th->beta_qkv, c.wprep ? nullptr : w.Wqkv_h, w.sq_qkv,
+                                      c.let ? th->d1 : nullptr,
                                       c.let ? w.shift_qkv : nullptr, c.let ? w.B_qkv : nullptr)));
   OMQ_TRY(lwc_fwd_launch(ax, lwc_args(Wo, c.d, c.dq, cfg, c.let ? so_e : nullptr, nullptr, th->gamma_o, th->beta_o,
                                       w.Wo_h, w.sq_o, c.let ? do_e : nullptr, nullptr, c.let ? w.B_o : nullptr)));
@@ -374,8 +398,15 @@ omq_status block_fwd(Ctx& c, const float* x, float* y) {
   af.h = w.sa.h; af.z = w.sa.z; af.imax = w.sa.imax; af.imin = w.sa.imin; af.abits = cfg.abits; af.eps = cfg.h_eps;
   af.status = status;
   OMQ_TRY(act_fwd_launch(st, af));
-  OMQ_TRY(gemm_kk(st, c.T, c.nqkv, c.d, w.a_h, c.d, w.Wqkv_h, c.d, w.Yqkv, nullptr, c.nqkv, c.let ? w.B_qkv : nullptr,
-                  nullptr, status));
+  if (c.wprep) {
+    GemmOperand a{w.a_h, c.d, 0, 1}, b{Wqkv, c.d, 0, 1};
+    GemmEpilogue ep{w.Yqkv, nullptr, c.nqkv, 0, 1.f, c.let ? w.B_qkv : nullptr, nullptr, c.nqkv, 0.f};
+    OMQ_TRY(gemm_launch_qb(st, c.T, c.nqkv, c.d, a, b, ep,
+                           qkv_operand(w.sq_qkv, cfg, c.d, c.let ? th->s1 : nullptr, c.let ? w.r_qkv : nullptr), status));
+  } else {
+    OMQ_TRY(gemm_kk(st, c.T, c.nqkv, c.d, w.a_h, c.d, w.Wqkv_h, c.d, w.Yqkv, nullptr, c.nqkv,
+                    c.let ? w.B_qkv : nullptr, nullptr, status));
+  }
   QkvArgs qa{};
   qa.T = (int)c.T; qa.H = (int)c.H; qa.Hkv = (int)c.Hkv; qa.hd = (int)c.hd; qa.Y = w.Yqkv; qa.ldy = c.nqkv; qa.cs = w.cs;
   qa.sa_exp = c.let ? sa_e : nullptr; qa.sa = c.let ? th->sa : nullptr;
@@ -535,7 +566,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   OMQ_REQUIRE(cudaEventRecord(ev[10], ax) == cudaSuccess, OMQ_ERR_CUDA);
   if (c.let) {
     const int64_t off = c.dq + c.dkv;
-    OMQ_TRY(gemm_dx(st, c.T, c.nqkv, c.d, w.dYqkv_b, w.Wqkv_h, w.da, status));
+    OMQ_TRY(qkv_dx(c, status));
     OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[10], 0) == cudaSuccess, OMQ_ERR_CUDA);  // dr of the v rows, ds1, dd1
     OMQ_TRY(let_vo_finalize(st, (int)c.dkv, th->so, w.dr_qkv + off, w.dB_qkv + off, w.B_qkv + off, g->so, g->do_, 1));
     ActBwdArgs ba{};
@@ -579,7 +610,7 @@ omq_status make_ctx(Ctx& c, omq_stream_t stream, const omq_block_shape* shape, c
   carve_block(real, *shape, *cfg, c.ws, bwd);
   c.T = shape->T; c.d = shape->d; c.hd = shape->head_dim; c.H = shape->n_heads; c.Hkv = shape->n_kv;
   c.rep = c.H / c.Hkv; c.f = shape->ffn; c.dq = c.H * c.hd; c.dkv = c.Hkv * c.hd; c.nqkv = c.dq + 2 * c.dkv;
-  c.let = cfg->let != 0; c.wq = cfg->wbits < 16; c.aq = cfg->abits < 16;
+  c.let = cfg->let != 0; c.wq = cfg->wbits < 16; c.aq = cfg->abits < 16; c.wprep = c.wq && cfg->wprep == 1;
   return OMQ_OK;
 }
 

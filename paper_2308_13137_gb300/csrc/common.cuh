@@ -27,6 +27,7 @@ static inline omq_status omq_check_cfg(const omq_qcfg* cfg) {
   if (cfg->group < 0) return OMQ_ERR_SHAPE;
   if (!(cfg->h_eps > 0.f)) return OMQ_ERR_INVALID_ARG;
   if (cfg->pbits != 0 && cfg->pbits != 16 && !(cfg->pbits >= 2 && cfg->pbits <= 8)) return OMQ_ERR_UNSUPPORTED;
+  if (cfg->wprep != 0 && cfg->wprep != 1) return OMQ_ERR_INVALID_ARG;
   return OMQ_OK;
 }
 

@@ -23,6 +23,9 @@ constexpr int BK = 64;          // one 128-byte swizzle row of bf16
 constexpr int UMMA_K = 16;
 constexpr int NUM_THREADS = 192;          // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
 constexpr int NUM_THREADS_LWC = 320;      // LWC epilogue: warps 2..9, two per TMEM lane quadrant
+// LWC = 4: the B operand is the raw weight and warps 6..9 form its fake-quantized bf16 values in
+// shared memory (operand preparation of Eq. 4); warps 2..5 run the plain epilogue
+constexpr int LWC_OPERAND = 4;
 
 struct GemmParams {
   int M, N, K, batch;
@@ -32,6 +35,7 @@ struct GemmParams {
   GemmEpilogue ep;
   GemmLwcEpi lw;             // used by the LWC-epilogue instantiation only
   int32_t* status;
+  GemmQuantB qb;             // used by the operand-preparation instantiation only
   int pair;                  // 1: CTA pairs, one 256-row tile per pair (cta_group::2)
   uint64_t wait_ns;          // limit of every mbarrier wait (OMQ_WAIT_LIMIT_NS unless a self-test sets it)
   int withhold;              // self-test only: the first operand load is never issued, so its wait expires
@@ -276,6 +280,99 @@ __device__ __forceinline__ void lwc_epilogue(const GemmParams& p, uint32_t tmem,
   }
 }
 
+// Operand preparation (LWC = 4): warps 6..9 of each CTA turn the raw weight tile of every stage into
+// its fake-quantized bf16 values in place.  The weight W is [rows, cols] with its quantizer state
+// per (row, group of cols) (GemmQuantB); as a K-major B operand (Y = X W_hat^T) a B row is a weight
+// row, as an MN-major one (dX = dY W_hat) a B row is a K index, i.e. again a weight row.  Either
+// way the tile is a stack of 128-byte swizzled lines of 64 consecutive weight columns of one weight
+// row (logical 16-byte chunk c of line l sits at chunk c ^ (l & 7); the conversion is elementwise,
+// so each chunk is rewritten where it lies), and thread ct owns line ct.  It waits for the tile's
+// own load barrier, converts, makes its writes visible to the tensor core's async proxy and arrives
+// on the leader's `conv` barrier, which the MMA issuer waits for besides `full`.
+template <int BN, int STAGES, bool PAIR>
+__device__ __forceinline__ void operand_prep(const GemmParams& p, uint8_t* smem, uint64_t* bfull, uint64_t* conv,
+                                             volatile int* abort_flag, int ct, int total, int rank) {
+  using L = SmemLayout<BN, STAGES, PAIR>;
+  constexpr int BNH = PAIR ? BN / 2 : BN;
+  static_assert(BNH == 128, "one converter thread per 128-byte line of the B tile");
+  const GemmQuantB& qb = p.qb;
+  const bool mn = p.b_mn != 0;
+  const int lane = ct & 31;
+  const int t_first = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int t_step = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+  const int wcols = mn ? p.N : p.K;                 // weight columns
+  const int wrows = mn ? p.K : p.N;                 // weight rows
+  const int ngroups = wcols / qb.group;
+  uint32_t it = 0;
+  for (int t = t_first; t < total && !*abort_flag; t += t_step) {
+    const TileInfo ti = tile_info(p, t, BN, rank);
+    if (ti.skip) continue;
+    const int nb0 = ti.n0 + rank * BNH;
+    QState qs;
+    qs.h = 1.f; qs.rh = 1.f; qs.z = 0.f; qs.u = 0.f; qs.a = qs.b = qs.M = qs.m = 0.f; qs.floored = 0;
+    int64_t gk_cur = -1;
+    float rr = 1.f;
+    int wr_cur = -1;
+    for (int kb = 0; kb < ti.nkb; ++kb, ++it) {
+      const int s = it % STAGES;
+      if (!mbar_wait(&bfull[s], (it / STAGES) & 1, p.wait_ns)) {
+        omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; break;
+      }
+      const int k0 = ti.k_begin + kb * BK;
+      // this thread's line: weight row wr, weight columns wc0 .. wc0 + 63
+      int wr, wc0;
+      uint32_t line;
+      if (!mn) { wr = nb0 + ct; wc0 = k0; line = smem_u32(smem + s * L::STAGE_BYTES + L::A_BYTES) + ct * 128; }
+      else { wr = k0 + (ct & 63); wc0 = nb0 + 64 * (ct >> 6);
+             line = smem_u32(smem + s * L::STAGE_BYTES + L::A_BYTES) + (ct >> 6) * 64 * BK * 2 + (ct & 63) * 128; }
+      if (wr < wrows) {
+        if (wr != wr_cur) { wr_cur = wr; rr = qb.r ? __ldg(qb.r + wr) : 1.f; gk_cur = -1; }
+        // all eight chunks first (logical chunk c sits at c ^ (line & 7): the eight lines of a
+        // quarter-warp touch eight distinct 16-byte bank groups), then the arithmetic, then the stores
+        uint4 raw[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) raw[c] = lds128(line + ((c ^ (ct & 7)) << 4));
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const int wc = wc0 + 8 * c;
+          if (wc >= wcols) continue;                // beyond the weight the tile holds zeros
+          const int64_t gk = (int64_t)wr * ngroups + wc / qb.group;
+          if (gk != gk_cur) {
+            gk_cur = gk;
+            qs.h = __ldg(qb.h + gk);
+            qs.z = (float)__ldg(qb.z + gk);
+            qs.rh = __frcp_rn(qs.h);
+          }
+          float w[8], o[8];
+          unpack_bf16x8(raw[c], w);
+          if (qb.s) {
+            const float4 s0 = __ldg(reinterpret_cast<const float4*>(qb.s + wc));
+            const float4 s1 = __ldg(reinterpret_cast<const float4*>(qb.s + wc) + 1);
+            const float sv[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) w[e] = __fmul_rn(w[e], sv[e]);
+          }
+          if (qb.r) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) w[e] = __fmul_rn(w[e], rr);
+          }
+#pragma unroll
+          for (int e = 0; e < 8; ++e) o[e] = omq_fakequant(w[e], qs, qb.Q, nullptr);
+          raw[c] = pack_bf16x8(o);
+        }
+#pragma unroll
+        for (int c = 0; c < 8; ++c) sts128(line + ((c ^ (ct & 7)) << 4), raw[c]);
+      }
+      fence_async_smem();                           // the converted tile -> visible to the tensor core
+      __syncwarp();
+      if (lane == 0) {
+        if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&conv[s]), 0));
+        else mbar_arrive(&conv[s]);
+      }
+    }
+  }
+}
+
 // Persistent kernel: one CTA per SM walks tiles blockIdx.x, blockIdx.x + gridDim.x, ...
 // The shared-memory ring runs continuously across tiles; the accumulator is double-buffered
 // in tensor memory (2 x BN columns) so that the epilogue of one tile overlaps the MMAs of
@@ -302,6 +399,10 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(acc_empty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
   uint64_t* drain = acc_empty + 3;         // after tmem_holder and abort_flag (8 bytes)
+  constexpr bool QB = LWC == LWC_OPERAND;
+  constexpr bool EPI_LWC = LWC != 0 && !QB;
+  uint64_t* bfull = drain + 1;             // QB: [STAGES] this CTA's raw B tile landed
+  uint64_t* conv = bfull + STAGES;         // QB: [STAGES] the pair's B tiles prepared (leader's)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bm_tile = PAIR ? 2 * BM : BM;
@@ -314,10 +415,12 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
-    constexpr int EPI_WARPS = LWC ? 8 : 4;
+    constexpr int EPI_WARPS = EPI_LWC ? 8 : 4;
     for (int b = 0; b < 2; ++b) { mbar_init(&acc_full[b], 1); mbar_init(&acc_empty[b], (PAIR ? 2 : 1) * EPI_WARPS); }
     *abort_flag = 0;
     mbar_init(drain, 1);
+    if (QB)
+      for (int s = 0; s < STAGES; ++s) { mbar_init(&bfull[s], 1); mbar_init(&conv[s], (PAIR ? 2 : 1) * 4); }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
@@ -349,7 +452,24 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
         uint8_t* sa = smem + s * L::STAGE_BYTES;
         uint8_t* sb = sa + L::A_BYTES;
         const int k0 = ti.k_begin + kb * BK;
-        if (PAIR) {
+        if (QB) {
+          // A (both CTAs' halves) completes on the leader's full barrier, this CTA's raw B tile on its
+          // own bfull barrier, which its converter warps wait for
+          if (PAIR) {
+            if (leader) mbar_expect_tx(&full[s], 2 * (uint32_t)L::A_BYTES);
+            tma_load_3d_pair(&tmA, mapa_shared(smem_u32(&full[s]), 0), sa, k0, ti.m0, ti.b);
+          } else {
+            mbar_expect_tx(&full[s], (uint32_t)L::A_BYTES);
+            tma_load_3d(&tmA, &full[s], sa, k0, ti.m0, ti.b);
+          }
+          mbar_expect_tx(&bfull[s], (uint32_t)(BNH * BK * 2));
+          if (!p.b_mn) {
+            tma_load_3d(&tmB, &bfull[s], sb, k0, nb0, ti.b);
+          } else {
+#pragma unroll
+            for (int j = 0; j < BNH / 64; ++j) tma_load_3d(&tmB, &bfull[s], sb + j * 64 * BK * 2, nb0 + 64 * j, k0, ti.b);
+          }
+        } else if (PAIR) {
           // both CTAs' loads complete on the leader's barrier, which expects the pair's bytes
           const uint32_t fb = mapa_shared(smem_u32(&full[s]), 0);
           if (leader) mbar_expect_tx(&full[s], 2 * stage_tx);
@@ -392,6 +512,10 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
       for (uint32_t j = first; j < it; ++j)
         if (!(p.withhold && j == 0)) mbar_wait(&full[j % STAGES], (j / STAGES) & 1, p.wait_ns);
     }
+    if (QB && *abort_flag) {                     // this CTA's own B loads
+      const uint32_t first = it > (uint32_t)STAGES ? it - STAGES : 0u;
+      for (uint32_t j = first; j < it; ++j) mbar_wait(&bfull[j % STAGES], (j / STAGES) & 1, p.wait_ns);
+    }
   } else if (warp == 1 && lane == 0 && leader) {
     // ---------------- MMA issuer (with CTA pairs: the leader CTA only) ----------------
     constexpr uint32_t IDESC_KK = idesc_bf16(PAIR ? 2 * BM : BM, BN, 0, 0);
@@ -410,7 +534,9 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
       bool ok = true;
       for (int kb = 0; kb < ti.nkb; ++kb, ++it) {
         const int s = it % STAGES;
-        if (!mbar_wait(&full[s], (it / STAGES) & 1, p.wait_ns)) {
+        if (!mbar_wait(&full[s], (it / STAGES) & 1, p.wait_ns) ||
+            (QB && !(PAIR ? mbar_wait_cluster(&conv[s], (it / STAGES) & 1, p.wait_ns)
+                          : mbar_wait(&conv[s], (it / STAGES) & 1, p.wait_ns)))) {
           omq_set_status(p.status, OMQ_ERR_TIMEOUT); *abort_flag = 1; ok = false; break;
         }
         tc_fence_after();
@@ -440,8 +566,10 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
       else umma_commit(drain);
       mbar_wait(drain, 0, p.wait_ns);
     }
-  } else if (LWC && warp >= 2) {
-    lwc_epilogue<BN, PAIR, LWC>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, (warp - 2) >> 2, lane, total, rank,
+  } else if (QB && warp >= 6) {
+    if constexpr (QB) operand_prep<BN, STAGES, PAIR>(p, smem, bfull, conv, abort_flag, threadIdx.x - 192, total, rank);
+  } else if (EPI_LWC && warp >= 2) {
+    lwc_epilogue<BN, PAIR, (EPI_LWC ? LWC : 1)>(p, tmem, acc_full, acc_empty, abort_flag, warp & 3, (warp - 2) >> 2, lane, total, rank,
                                 reinterpret_cast<float*>(smem + L::EPI_OFF) + (warp - 2) * (BN / 2));
   } else if (warp >= 2) {
     // ---------------- epilogue ----------------
@@ -749,6 +877,46 @@ bool omq_make_map_bf16(CUtensorMap* map, const void* ptr, int64_t inner, int64_t
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+omq_status gemm_launch_qb(cudaStream_t st, int64_t M, int64_t N, int64_t K, const GemmOperand& A, const GemmOperand& B,
+                          const GemmEpilogue& ep, const GemmQuantB& qb, int32_t* status) {
+  OMQ_REQUIRE(M > 0 && N > 0 && K > 0 && M < (1ll << 31) && N < (1ll << 31) && K < (1ll << 31), OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(A.ptr && B.ptr && (ep.Cf || ep.Cb) && qb.h && qb.z, OMQ_ERR_INVALID_ARG);
+  OMQ_REQUIRE(A.kmajor, OMQ_ERR_UNSUPPORTED);
+  const int64_t wcols = B.kmajor ? K : N;            // the weight's own column count
+  OMQ_REQUIRE(qb.group > 0 && qb.group % 8 == 0 && wcols % qb.group == 0 && K % 8 == 0 && N % 8 == 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(omq_aligned16(A.ptr) && omq_aligned16(B.ptr) && A.ld % 8 == 0 && B.ld % 8 == 0, OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(ep.ldc % 8 == 0 && ep.ldc >= N, OMQ_ERR_ALIGN);
+  OMQ_REQUIRE((!ep.Cf || omq_aligned16(ep.Cf)) && (!ep.Cb || omq_aligned16(ep.Cb)), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE(!ep.R || (omq_aligned16(ep.R) && ep.ldr % 4 == 0), OMQ_ERR_ALIGN);
+  OMQ_REQUIRE((!ep.bias || omq_aligned16(ep.bias)) && (!qb.s || omq_aligned16(qb.s)), OMQ_ERR_ALIGN);
+  const bool pair = gemm_n_tile(N) == 256 && M > BM;   // pairs: 128 B rows per CTA; else BN = 128
+  CUtensorMap ta, tb, tc;
+  memset(&tc, 0, sizeof(tc));
+  bool ok = make_map(&ta, A.ptr, K, M, 1, A.ld, 0, BM) &&
+            (B.kmajor ? make_map(&tb, B.ptr, K, N, 1, B.ld, 0, 128) : make_map(&tb, B.ptr, N, K, 1, B.ld, 0, BK));
+  if (ep.Cf) ok = ok && make_map_c(&tc, ep.Cf, N, M, 1, ep.ldc, 0);
+  if (!ok) return OMQ_ERR_UNSUPPORTED;
+  GemmParams p;
+  memset(&p, 0, sizeof(p));
+  p.M = (int)M; p.N = (int)N; p.K = (int)K; p.batch = 1;
+  p.a_mn = 0; p.b_mn = B.kmajor ? 0 : 1; p.causal = 0; p.ep = ep; p.qb = qb; p.status = status; p.pair = pair ? 1 : 0;
+  p.n_fast = ((double)M > 1.5 * (double)N) ? 1 : 0;
+  p.wait_ns = OMQ_WAIT_LIMIT_NS; p.withhold = 0;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  if (g_prof.on) {
+    e0 = prof_event();
+    e1 = prof_event();
+    if (e0 && e1) {
+      cudaEventRecord(e0, st);
+      g_prof.flops += gemm_algorithmic_flops(M, N, K, 1, 0);
+    }
+  }
+  omq_status r = pair ? launch_cfg<256, 6, LWC_OPERAND, true>(st, ta, tb, tc, p)
+                      : launch_cfg<128, 6, LWC_OPERAND>(st, ta, tb, tc, p);
+  if (e0 && e1) cudaEventRecord(e1, st);
+  return r;
 }
 
 omq_status gemm_launch_lwc(cudaStream_t st, int64_t M, int64_t N, int64_t K, const GemmOperand& A,

@@ -42,12 +42,28 @@ struct GemmLwcEpi {
   int want_dr;                    // the row sums for dr (rowpart[2]) are needed
 };
 
+// LWC fake quantization of the B operand inside the GEMM (Eq. 2 and Eq. 4 as operand preparation):
+// B is the raw bf16 weight [N, K] (K-major); after each tile lands in shared memory, four warps
+// replace every element by its fake-quantized value bf16((clamp(round(w~ / h), -z, Q - z)) h) with
+// w~ = fl(fl(w s_k) r_n), exactly the value the LWC forward would have written to HBM.
+struct GemmQuantB {
+  const float* h; const int32_t* z;   // [N, ngroups] step and zero point (ngroups = K / group)
+  const float* r;                     // [N] row scale or null
+  const float* s;                     // [K] LET column scale or null
+  int group;                          // group size along K (a multiple of 8); K = one group per row
+  float Q;                            // 2^N - 1
+};
+
 // N-tile width the GEMM uses for a product with N columns
 int gemm_n_tile(int64_t N);
 
 // C[b] = alpha * A[b] B[b]^T (+bias)(+R)(+beta*C); causal modes as in omq_gemm_bf16
 omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t batch, const GemmOperand& A,
                        const GemmOperand& B, const GemmEpilogue& ep, int causal, int32_t* status);
+
+// C = A B_hat^T with B_hat prepared from the raw weight B in shared memory (GemmQuantB); A, B K-major
+omq_status gemm_launch_qb(cudaStream_t st, int64_t M, int64_t N, int64_t K, const GemmOperand& A, const GemmOperand& B,
+                          const GemmEpilogue& ep, const GemmQuantB& qb, int32_t* status);
 
 // dW_hat = A B^T (K-reduction over tokens) consumed by the fused LWC epilogue above; no C output
 omq_status gemm_launch_lwc(cudaStream_t st, int64_t M, int64_t N, int64_t K, const GemmOperand& A,

@@ -35,10 +35,10 @@ def test_every_exported_function_is_declared():
 
 
 def _cfg(**kw):
-    base = dict(wbits=4, abits=16, group=128, let=0, h_eps=1e-5, accumulate=0, dev_status=None, pbits=0)
+    base = dict(wbits=4, abits=16, group=128, let=0, h_eps=1e-5, accumulate=0, dev_status=None, pbits=0, wprep=0)
     base.update(kw)
     return _lib.omq_qcfg(base["wbits"], base["abits"], base["group"], base["let"], base["h_eps"],
-                         base["accumulate"], base["dev_status"], base["pbits"])
+                         base["accumulate"], base["dev_status"], base["pbits"], base["wprep"])
 
 
 FAKE = 0x10000     # 16-byte aligned dummy address: every call below returns before touching it
@@ -57,6 +57,7 @@ def test_argument_errors_before_launch():
     assert _lwc_fwd(64, 512, _cfg(wbits=1)) == 4               # OMQ_ERR_UNSUPPORTED
     assert _lwc_fwd(64, 512, _cfg(wbits=12)) == 4
     assert _lwc_fwd(64, 512, None) == 1                        # OMQ_ERR_INVALID_ARG
+    assert _lwc_fwd(64, 512, _cfg(wprep=2)) == 1               # operand preparation mode outside {0, 1}
     assert _lwc_fwd(64, 512, _cfg(), W=FAKE + 4) == 3          # misaligned pointer
     L = _lib.lib()
     # workspace too small
