@@ -279,7 +279,13 @@ omq_status omq_block_forward(omq_stream_t stream, const omq_block_shape* shape,
 
 /* One calibration step without the parameter update: forward, loss = mean((y - y_fp)^2) written
  * to the device scalar `loss`, and the STE gradients of every learnable parameter into `grads`.
- * y (NULL = not returned) receives the quantized block output. */
+ * y (NULL = not returned) receives the quantized block output.
+ * The launches go to `stream` and to one auxiliary stream per device owned by the library, joined
+ * back to `stream` by events before the call returns, so the call can be captured into a CUDA
+ * graph on `stream`.  The library keeps no state keyed on the caller's pointers; a captured graph
+ * does: it replays the addresses it was captured with.  A caller that replays (the package's
+ * BlockState looks its graphs up by the addresses of x and y_fp) refills the same buffers in place
+ * between replays and keeps them alive; new buffers need a new capture. */
 omq_status omq_block_step(omq_stream_t stream, const omq_block_shape* shape,
                           const omq_block_weights* w, const omq_block_params* theta,
                           const float* x, const float* y_fp, float* y, float* loss,

@@ -68,9 +68,9 @@ def _compare(shape, seed=0):
     for k, v in ref["saved"].items():
         if isinstance(v, list):
             for i in range(4):
-                if got[("saved")][k][i] is not None:
+                if got["saved"][k][i] is not None:
                     _same(got["saved"][k][i], v[i], f"{k}[{i}]")
-        else:
+        elif shape.abits < 16 or not k.endswith(("_h", "_z")):   # per-token quantizer state exists only with Q_a on
             _same(got["saved"][k], v, k)
 
 
