@@ -79,7 +79,8 @@ struct BlockWS {
   float *dB_qkv, *dB_o, *dB_gu, *dr_qkv;
   float *vtmp0, *vtmp1, *vtmp2;     // [max(d, dq)] scratch vectors
   float* part;                      // shared partial-sum scratch
-  float* part_aux;                  // scratch of the weight-gradient launches on the auxiliary stream
+  float* part_aux;                  // scratch of the launches on the auxiliary stream
+  float* part2;                     // LET column partials of the second RMSNorm backward (reduced on the auxiliary stream)
   size_t part_elems;
 };
 
@@ -170,7 +171,9 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   const int64_t lin[4][2] = {{nqkv, d}, {d, dq}, {2 * f, d}, {d, f}};
   for (const auto& l : lin)
     pa = imax64(pa, imax64(lwc_fused_scratch_elems(l[0], l[1]), (int64_t)lwc_bwd_scratch_bytes(l[0], l[1]) / 4 + 64));
+  pa = imax64(pa, colsum_rows_parts(T) * imax64(imax64(2 * f, nqkv), d));   // the LET bias column sums
   w.part_aux = c.take<float>(pa);
+  w.part2 = c.take<float>(2 * ((T + 3) / 4) * d);
 }
 
 omq_status check_block(const omq_block_shape* s, const omq_qcfg* cfg) {
@@ -483,31 +486,31 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
 
   // ---- gate / up ----------------------------------------------------------------------------------
   // LET bias gradient dB~ = sum_t dY: the column sums of the bf16 gradient, the operand every product of
-  // this backward takes (R13)
-  if (c.let) OMQ_TRY(colsum_rows_bf16(st, w.dYgu_b, c.T, 2 * c.f, 2 * c.f, w.part, w.dB_gu, 1.f, 0));
+  // this backward takes (R13); only the LWC backward of the weight-gradient product reads it, so it is
+  // formed on the auxiliary stream just before that product
   OMQ_TRY(join(st, ax, ev[5]));
+  if (c.let) OMQ_TRY(colsum_rows_bf16(ax, w.dYgu_b, c.T, 2 * c.f, 2 * c.f, w.part_aux, w.dB_gu, 1.f, 0));
   OMQ_TRY(lwc_bwd_dw(ax, c.T, w.dYgu_b, w.b_h, Wgu, 2 * c.f, c.d, cfg, c.let ? th->s2 : nullptr, nullptr,
                      th->gamma_gu, th->beta_gu, w.sq_gu, g->gamma_gu, g->beta_gu, nullptr,
                      c.let ? w.dB_gu : nullptr, c.let ? g->s2 : nullptr, c.let ? g->d2 : nullptr, acc, w.part_aux,
                      w.dW, status));
-  OMQ_REQUIRE(cudaEventRecord(ev[6], ax) == cudaSuccess, OMQ_ERR_CUDA);
   OMQ_TRY(gemm_dx(st, c.T, 2 * c.f, c.d, w.dYgu_b, w.Wgu_h, w.db, status));
   ActBwdArgs bb{};
   bb.producer = AP_RMS_LET; bb.X = w.h1; bb.ldx = c.d; bb.s = c.let ? th->s2 : nullptr; bb.delta = c.let ? th->d2 : nullptr;
   bb.rstd = w.rstd2; bb.T = c.T; bb.C = c.d; bb.h = w.sb.h; bb.z = w.sb.z; bb.imax = w.sb.imax; bb.imin = w.sb.imin;
   bb.dXq = w.db; bb.lddq = c.d; bb.dX = nullptr; bb.lddx = c.d; bb.dXb = w.dh1_b; bb.lddxb = c.d; bb.resid = w.dy;
-  bb.part_s = c.let ? w.part : nullptr; bb.part_d = c.let ? w.part + ((c.T + 3) / 4) * c.d : nullptr;
+  bb.part_s = c.let ? w.part2 : nullptr; bb.part_d = c.let ? w.part2 + ((c.T + 3) / 4) * c.d : nullptr;
   bb.rows_per_cta = 4; bb.abits = cfg.abits; bb.eps = cfg.h_eps;
   OMQ_TRY(act_bwd_launch(st, bb));
-  if (c.let) {
-    OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[6], 0) == cudaSuccess, OMQ_ERR_CUDA);   // LWC part of ds2, dd2
-    OMQ_TRY(omq_colsum_partials2(st, ColsumJob{bb.part_s, (c.T + 3) / 4, c.d, g->s2, 1.f, 1},
-                                 ColsumJob{bb.part_d, (c.T + 3) / 4, c.d, g->d2, 1.f, 1}));
-  }
 
   // ---- o_proj -------------------------------------------------------------------------------------
-  if (c.let) OMQ_TRY(colsum_rows_bf16(st, w.dh1_b, c.T, c.d, c.d, w.part, w.dB_o, 1.f, 0));
   OMQ_TRY(join(st, ax, ev[7]));
+  if (c.let) {
+    // ds2, dd2: the RMSNorm backward's part added after the LWC part (earlier on this stream), then dB~_o
+    OMQ_TRY(omq_colsum_partials2(ax, ColsumJob{bb.part_s, (c.T + 3) / 4, c.d, g->s2, 1.f, 1},
+                                 ColsumJob{bb.part_d, (c.T + 3) / 4, c.d, g->d2, 1.f, 1}));
+    OMQ_TRY(colsum_rows_bf16(ax, w.dh1_b, c.T, c.d, c.d, w.part_aux, w.dB_o, 1.f, 0));
+  }
   // ds_o, ddelta_o per query channel; with one query head per kv head straight into the gradients
   const bool fold_o = c.rep > 1;
   OMQ_TRY(lwc_bwd_dw(ax, c.T, w.dh1_b, w.O_h, Wo, c.d, c.dq, cfg, c.let ? so_e : nullptr, nullptr, th->gamma_o,
@@ -557,8 +560,8 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   }
 
   // ---- q / k / v projections ---------------------------------------------------------------------------
-  if (c.let) OMQ_TRY(colsum_rows_bf16(st, w.dYqkv_b, c.T, c.nqkv, c.nqkv, w.part, w.dB_qkv, 1.f, 0));
   OMQ_TRY(join(st, ax, ev[9]));
+  if (c.let) OMQ_TRY(colsum_rows_bf16(ax, w.dYqkv_b, c.T, c.nqkv, c.nqkv, w.part_aux, w.dB_qkv, 1.f, 0));
   OMQ_TRY(lwc_bwd_dw(ax, c.T, w.dYqkv_b, w.a_h, Wqkv, c.nqkv, c.d, cfg, c.let ? th->s1 : nullptr,
                      c.let ? w.r_qkv : nullptr, th->gamma_qkv, th->beta_qkv, w.sq_qkv, g->gamma_qkv, g->beta_qkv,
                      c.let ? w.dr_qkv : nullptr, c.let ? w.dB_qkv : nullptr, c.let ? g->s1 : nullptr,
