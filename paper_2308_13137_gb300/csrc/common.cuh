@@ -49,6 +49,13 @@ __device__ __forceinline__ void omq_set_status(int32_t* st, int32_t code) {
   if (st) atomicCAS(st, 0, code);
 }
 
+// Bulk prefetch of [p, p + bytes) into L2 (cp.async.bulk.prefetch: no data returned, no completion
+// to wait for); p 16-byte aligned and bytes a multiple of 16, else nothing is issued
+__device__ __forceinline__ void omq_l2_prefetch(const void* p, uint64_t bytes) {
+  if (((uintptr_t)p & 15) != 0 || (bytes & 15) != 0 || bytes == 0) return;
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"((uint32_t)bytes) : "memory");
+}
+
 __device__ __forceinline__ uint64_t omq_globaltimer() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

@@ -440,6 +440,16 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
     for (int k = 0; k < NE; ++k) { acc_s[k] = 0.f; acc_d[k] = 0.f; }
     const int64_t t0 = p * a.rows_per_cta, t1 = min(a.T, t0 + a.rows_per_cta);
     for (int64_t t = t0; t < t1; ++t) {
+      if (tid == 0) {                          // the next row's inputs (and this row's residual) into L2
+        const uint64_t rb = (uint64_t)a.C * 4;
+        if (P == AP_RMS_LET && a.resid) omq_l2_prefetch(a.resid + t * a.lddx, rb);
+        if (t + 1 < t1) {
+          omq_l2_prefetch(a.X + (t + 1) * a.ldx, rb);
+          omq_l2_prefetch(a.dXq + (t + 1) * a.lddq, rb);
+          if (P == AP_SWIGLU) omq_l2_prefetch(a.U + (t + 1) * a.ldu, rb);
+          if (P == AP_RMS_LET && a.resid) omq_l2_prefetch(a.resid + (t + 1) * a.lddx, rb);
+        }
+      }
       ActBwdRow<P> R{a, t, (P == AP_RMS_LET) ? a.rstd[t] : 1.f};
       const float* xr = a.X + t * a.ldx;
       const float* gr = a.dXq + t * a.lddq;
@@ -916,6 +926,10 @@ __device__ __forceinline__ void qkv_bwd_body(const QkvArgs& a, float* fsm) {
       const int Hs = seg == 0 ? a.H : a.Hkv;
       const int np = Hs * 16;
       const int off = seg == 0 ? 0 : (seg == 1 ? dq : dq + dkv);
+      if (tid == 0 && t + 1 < t1) {           // the next row's segment into L2
+        omq_l2_prefetch(a.Y + (int64_t)(t + 1) * a.ldy + off, (uint64_t)Hs * a.hd * 4);
+        omq_l2_prefetch(a.dQKV + (int64_t)(t + 1) * a.ldd + off, (uint64_t)Hs * a.hd * 4);
+      }
       const float* base = a.Y + (int64_t)t * a.ldy + off;
       const float* gsrc = a.dQKV + (int64_t)t * a.ldd + off;
       float* dy = a.dY + (int64_t)t * a.ldy + off;

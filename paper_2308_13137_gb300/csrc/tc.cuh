@@ -30,15 +30,25 @@ static __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t par
   return ok != 0;
 }
 
-// Bounded wait on a phase parity; false when the time limit (default one second) expired.
+// Bounded wait on a phase parity; false when the time limit (default one second) expired.  After a
+// first test the thread waits inside try_wait with a suspend-time hint: the hardware wakes it when
+// the phase completes (or after the hint), instead of the warp spinning on the barrier.
 static __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
                                                  uint64_t limit_ns = OMQ_WAIT_LIMIT_NS) {
   if (mbar_try_wait(bar, parity)) return true;
+  // each try suspends the thread until the phase completes or the hint (ns) elapses
+  const uint32_t hint = limit_ns < 1000000ull ? (uint32_t)limit_ns : 1000000u;
   const uint64_t t0 = omq_globaltimer();
   while (true) {
-#pragma unroll 1
-    for (int i = 0; i < 32; ++i)
-      if (mbar_try_wait(bar, parity)) return true;
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(hint)
+        : "memory");
+    if (ok) return true;
     if (omq_globaltimer() - t0 > limit_ns) return false;
   }
 }
