@@ -86,6 +86,12 @@ struct BlockWS {
 
 int64_t imax64(int64_t a, int64_t b) { return a > b ? a : b; }
 
+// Token rows per CTA of the step's activation-quantizer backward launches (each CTA prefetches its
+// next row into L2 while it works on the current one); the RMSNorm backward's LET column partials
+// have one row per CTA.
+constexpr int kRowsRms = 7, kRowsSwiglu = 1, kRowsPlain = 4;
+int64_t rms_parts(int64_t T) { return (T + kRowsRms - 1) / kRowsRms; }
+
 void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockWS& w, bool with_bwd) {
   const int64_t T = s.T, d = s.d, hd = s.head_dim, H = s.n_heads, Hkv = s.n_kv, f = s.ffn;
   const int64_t dq = H * hd, dkv = Hkv * hd, nqkv = dq + 2 * dkv;
@@ -162,7 +168,7 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
   pe = imax64(pe, lwc_fused_scratch_elems(d, dq));
   pe = imax64(pe, lwc_fused_scratch_elems(2 * f, d));
   pe = imax64(pe, lwc_fused_scratch_elems(d, f));
-  pe = imax64(pe, 2 * ((T + 3) / 4) * imax64(d, dq));
+  pe = imax64(pe, 2 * rms_parts(T) * imax64(d, dq));
   pe = imax64(pe, qkv_bwd_nslab((int)T) * (dq + dkv));
   pe = imax64(pe, colsum_rows_parts(T) * imax64(2 * f, nqkv));
   w.part_elems = (size_t)pe;
@@ -173,7 +179,7 @@ void carve_block(Carve& c, const omq_block_shape& s, const omq_qcfg& cfg, BlockW
     pa = imax64(pa, imax64(lwc_fused_scratch_elems(l[0], l[1]), (int64_t)lwc_bwd_scratch_bytes(l[0], l[1]) / 4 + 64));
   pa = imax64(pa, colsum_rows_parts(T) * imax64(imax64(2 * f, nqkv), d));   // the LET bias column sums
   w.part_aux = c.take<float>(pa);
-  w.part2 = c.take<float>(2 * ((T + 3) / 4) * d);
+  w.part2 = c.take<float>(2 * rms_parts(T) * d);
 }
 
 omq_status check_block(const omq_block_shape* s, const omq_qcfg* cfg) {
@@ -481,7 +487,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   bm.producer = AP_SWIGLU; bm.X = w.Ygu; bm.ldx = 2 * c.f; bm.U = w.Ygu + c.f; bm.ldu = 2 * c.f; bm.T = c.T; bm.C = c.f;
   bm.h = w.sm.h; bm.z = w.sm.z; bm.imax = w.sm.imax; bm.imin = w.sm.imin; bm.dXq = w.dm; bm.lddq = c.f;
   bm.dX = nullptr; bm.lddx = 2 * c.f; bm.dXb = w.dYgu_b; bm.lddxb = 2 * c.f; bm.dU = nullptr; bm.dUb = w.dYgu_b + c.f;
-  bm.rows_per_cta = 1; bm.abits = cfg.abits; bm.eps = cfg.h_eps;
+  bm.rows_per_cta = kRowsSwiglu; bm.abits = cfg.abits; bm.eps = cfg.h_eps;
   OMQ_TRY(act_bwd_launch(st, bm));
 
   // ---- gate / up ----------------------------------------------------------------------------------
@@ -499,16 +505,16 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   bb.producer = AP_RMS_LET; bb.X = w.h1; bb.ldx = c.d; bb.s = c.let ? th->s2 : nullptr; bb.delta = c.let ? th->d2 : nullptr;
   bb.rstd = w.rstd2; bb.T = c.T; bb.C = c.d; bb.h = w.sb.h; bb.z = w.sb.z; bb.imax = w.sb.imax; bb.imin = w.sb.imin;
   bb.dXq = w.db; bb.lddq = c.d; bb.dX = nullptr; bb.lddx = c.d; bb.dXb = w.dh1_b; bb.lddxb = c.d; bb.resid = w.dy;
-  bb.part_s = c.let ? w.part2 : nullptr; bb.part_d = c.let ? w.part2 + ((c.T + 3) / 4) * c.d : nullptr;
-  bb.rows_per_cta = 4; bb.abits = cfg.abits; bb.eps = cfg.h_eps;
+  bb.part_s = c.let ? w.part2 : nullptr; bb.part_d = c.let ? w.part2 + rms_parts(c.T) * c.d : nullptr;
+  bb.rows_per_cta = kRowsRms; bb.abits = cfg.abits; bb.eps = cfg.h_eps;
   OMQ_TRY(act_bwd_launch(st, bb));
 
   // ---- o_proj -------------------------------------------------------------------------------------
   OMQ_TRY(join(st, ax, ev[7]));
   if (c.let) {
     // ds2, dd2: the RMSNorm backward's part added after the LWC part (earlier on this stream), then dB~_o
-    OMQ_TRY(omq_colsum_partials2(ax, ColsumJob{bb.part_s, (c.T + 3) / 4, c.d, g->s2, 1.f, 1},
-                                 ColsumJob{bb.part_d, (c.T + 3) / 4, c.d, g->d2, 1.f, 1}));
+    OMQ_TRY(omq_colsum_partials2(ax, ColsumJob{bb.part_s, rms_parts(c.T), c.d, g->s2, 1.f, 1},
+                                 ColsumJob{bb.part_d, rms_parts(c.T), c.d, g->d2, 1.f, 1}));
     OMQ_TRY(colsum_rows_bf16(ax, w.dh1_b, c.T, c.d, c.d, w.part_aux, w.dB_o, 1.f, 0));
   }
   // ds_o, ddelta_o per query channel; with one query head per kv head straight into the gradients
@@ -522,7 +528,7 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   ActBwdArgs bo{};
   bo.producer = AP_PLAIN; bo.X = w.O; bo.ldx = c.dq; bo.T = c.T; bo.C = c.dq; bo.h = w.so.h; bo.z = w.so.z;
   bo.imax = w.so.imax; bo.imin = w.so.imin; bo.dXq = w.dOh; bo.lddq = c.dq; bo.dX = nullptr; bo.lddx = c.dq;
-  bo.dXb = w.dO_b; bo.lddxb = c.dq; bo.rows_per_cta = 4; bo.abits = cfg.abits; bo.eps = cfg.h_eps;
+  bo.dXb = w.dO_b; bo.lddxb = c.dq; bo.rows_per_cta = kRowsPlain; bo.abits = cfg.abits; bo.eps = cfg.h_eps;
   OMQ_TRY(act_bwd_launch(st, bo));
 
   // ---- attention: dQ, dK, dV from the saved log-sum-exp (scores recomputed, never stored) --------
@@ -575,11 +581,11 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
     ActBwdArgs ba{};
     ba.producer = AP_RMS_LET; ba.X = x; ba.ldx = c.d; ba.s = th->s1; ba.delta = th->d1; ba.rstd = w.rstd1; ba.T = c.T;
     ba.C = c.d; ba.h = w.sa.h; ba.z = w.sa.z; ba.imax = w.sa.imax; ba.imin = w.sa.imin; ba.dXq = w.da; ba.lddq = c.d;
-    ba.dX = nullptr; ba.dXb = nullptr; ba.part_s = w.part; ba.part_d = w.part + ((c.T + 3) / 4) * c.d;
-    ba.rows_per_cta = 4; ba.abits = cfg.abits; ba.eps = cfg.h_eps;
+    ba.dX = nullptr; ba.dXb = nullptr; ba.part_s = w.part; ba.part_d = w.part + rms_parts(c.T) * c.d;
+    ba.rows_per_cta = kRowsRms; ba.abits = cfg.abits; ba.eps = cfg.h_eps;
     OMQ_TRY(act_bwd_launch(st, ba));
-    OMQ_TRY(omq_colsum_partials2(st, ColsumJob{ba.part_s, (c.T + 3) / 4, c.d, g->s1, 1.f, 1},
-                                 ColsumJob{ba.part_d, (c.T + 3) / 4, c.d, g->d1, 1.f, 1}));
+    OMQ_TRY(omq_colsum_partials2(st, ColsumJob{ba.part_s, rms_parts(c.T), c.d, g->s1, 1.f, 1},
+                                 ColsumJob{ba.part_d, rms_parts(c.T), c.d, g->d1, 1.f, 1}));
   }
   OMQ_REQUIRE(cudaStreamWaitEvent(st, ev[10], 0) == cudaSuccess, OMQ_ERR_CUDA);    // every auxiliary launch
   return OMQ_OK;

@@ -57,6 +57,7 @@ struct ActFwdArgs {
   float* h; int32_t* z; int32_t* imax; int32_t* imin;
   int abits; float eps;
   int32_t* status;                   // device status word (timeouts of the staged kernel), nullable
+  int rows_per_cta;                  // set by the launcher
 };
 omq_status act_fwd_launch(cudaStream_t st, const ActFwdArgs& a);
 

@@ -119,13 +119,11 @@ __device__ __forceinline__ void row_ste(const float (&val)[NE], const int (&col)
 // ================================================================================================
 // activation quantizer forward: producer -> (LET) -> Q_a -> bf16
 // ================================================================================================
+// one token row t of the activation quantizer forward, held in registers
 template <int P, int NT, int VPT>
-__global__ void __launch_bounds__(NT) act_fwd_rows(ActFwdArgs a) {
+__device__ __forceinline__ void act_fwd_row(const ActFwdArgs& a, const int64_t t, float* fsm, int* ism) {
   constexpr int NE = 4 * VPT;
-  __shared__ float fsm[64];
-  __shared__ int ism[64];
   const int tid = threadIdx.x;
-  const int64_t t = blockIdx.x;
   const int64_t nv = a.C / 4;
   float val[NE], cd[NE];
   int col[NE];
@@ -195,6 +193,27 @@ __global__ void __launch_bounds__(NT) act_fwd_rows(ActFwdArgs a) {
   }
 }
 
+
+// token rows per CTA of the register-resident forward (rows of up to 4 K columns; the SwiGLU row)
+constexpr int kFwdRows = 2, kFwdRowsSwiglu = 2;
+
+// rows blockIdx.x * R .. + R - 1 (R = a.rows_per_cta, at least 1); the CTA prefetches each next row's
+// inputs into L2 while it works on the current one
+template <int P, int NT, int VPT>
+__global__ void __launch_bounds__(NT) act_fwd_rows(ActFwdArgs a) {
+  __shared__ float fsm[64];
+  __shared__ int ism[64];
+  const int64_t R = a.rows_per_cta > 1 ? a.rows_per_cta : 1;
+  const int64_t t0 = (int64_t)blockIdx.x * R, t1 = t0 + R < a.T ? t0 + R : a.T;
+  for (int64_t t = t0; t < t1; ++t) {
+    if (threadIdx.x == 0 && t + 1 < t1) {
+      omq_l2_prefetch(a.X + (t + 1) * a.ldx, (uint64_t)a.C * 4);
+      if (P == AP_SWIGLU) omq_l2_prefetch(a.U + (t + 1) * a.ldu, (uint64_t)a.C * 4);
+    }
+    act_fwd_row<P, NT, VPT>(a, t, fsm, ism);
+    __syncthreads();                           // the reduction scratch is reused by the next row
+  }
+}
 // ================================================================================================
 // activation quantizer forward, staged: a persistent CTA walks the rows blockIdx.x, + gridDim.x, ...
 // and the bulk-copy engine brings each row's inputs into a ring of `stages` shared-memory buffers
@@ -706,7 +725,9 @@ static omq_status act_fwd_staged_go(cudaStream_t st, const ActFwdArgs& a, int st
 // Rows whose inputs fit two or more times in shared memory take the staged kernel; 16-byte aligned
 // rows of up to 16 K columns.
 template <int PRODUCER>
-static omq_status act_fwd_dispatch(cudaStream_t st, const ActFwdArgs& a) {
+static omq_status act_fwd_dispatch(cudaStream_t st, const ActFwdArgs& a0) {
+  ActFwdArgs a = a0;
+  a.rows_per_cta = 1;
   const int nin = PRODUCER == AP_SWIGLU ? 2 : 1;
   const size_t row_bytes = (size_t)nin * a.C * 4;
   const int stages = (int)std::min<size_t>(3, (200 * 1024) / row_bytes);
@@ -714,12 +735,14 @@ static omq_status act_fwd_dispatch(cudaStream_t st, const ActFwdArgs& a) {
                        (PRODUCER != AP_SWIGLU || (a.ldu % 4 == 0 && omq_aligned16(a.U)));
   const int64_t nv = a.C / 4;
   if (nv <= 128 * 8) {                             // small rows: many CTAs per SM, 32 values per thread
-    act_fwd_rows<PRODUCER, 128, 8><<<(unsigned)a.T, 128, 0, st>>>(a);
+    a.rows_per_cta = kFwdRows;
+    act_fwd_rows<PRODUCER, 128, 8><<<(unsigned)((a.T + kFwdRows - 1) / kFwdRows), 128, 0, st>>>(a);
     OMQ_LAUNCH_CHECK();
     return OMQ_OK;
   }
   if (PRODUCER == AP_SWIGLU && nv <= 256 * 12) {
-    act_fwd_rows<PRODUCER, 256, 12><<<(unsigned)a.T, 256, 0, st>>>(a);
+    a.rows_per_cta = kFwdRowsSwiglu;
+    act_fwd_rows<PRODUCER, 256, 12><<<(unsigned)((a.T + kFwdRowsSwiglu - 1) / kFwdRowsSwiglu), 256, 0, st>>>(a);
     OMQ_LAUNCH_CHECK();
     return OMQ_OK;
   }
@@ -1103,7 +1126,10 @@ __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_seg(QkvArgs a) {
   else qkv_bwd_body<PPT, 2>(a, fsm);
 }
 
-int64_t qkv_bwd_nslab(int T) { return (T + 3) / 4; }
+// token rows per CTA of the q, k, v backward (each CTA prefetches its next row into L2); the ds_a
+// partials have one row per CTA
+constexpr int kQkvBwdRows = 7;
+int64_t qkv_bwd_nslab(int T) { return (T + kQkvBwdRows - 1) / kQkvBwdRows; }
 
 omq_status qkv_fwd_launch(cudaStream_t st, const QkvArgs& a) {
   OMQ_REQUIRE(a.hd == 128, OMQ_ERR_UNSUPPORTED);
@@ -1120,7 +1146,7 @@ omq_status qkv_fwd_launch(cudaStream_t st, const QkvArgs& a) {
 omq_status qkv_bwd_launch(cudaStream_t st, const QkvArgs& a0, int64_t* nslab) {
   QkvArgs a = a0;
   OMQ_REQUIRE(a.hd == 128, OMQ_ERR_UNSUPPORTED);
-  a.rows_per_cta = 4;
+  a.rows_per_cta = kQkvBwdRows;
   const unsigned grid = (unsigned)qkv_bwd_nslab(a.T);
   const int np = a.H * 16;
   if (np <= 256) qkv_bwd_stream<1, 4><<<grid, QKV_BWD_NT, 0, st>>>(a);
