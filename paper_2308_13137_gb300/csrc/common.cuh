@@ -184,6 +184,44 @@ __device__ __forceinline__ float omq_fakequant(float w, const QState& s, float Q
   return __fmul_rn(qz, s.h);
 }
 
+// Paired f32 arithmetic (f32x2: one instruction for two lanes, each rounded to nearest exactly as
+// __fmul_rn / __fmaf_rn / __fadd_rn round one)
+__device__ __forceinline__ uint64_t omq_f2u(float2 v) {
+  return ((uint64_t)__float_as_uint(v.y) << 32) | (uint64_t)__float_as_uint(v.x);
+}
+__device__ __forceinline__ float2 omq_u2f(uint64_t u) {
+  return make_float2(__uint_as_float((uint32_t)u), __uint_as_float((uint32_t)(u >> 32)));
+}
+__device__ __forceinline__ float2 omq_mul2(float2 a, float2 b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(omq_f2u(a)), "l"(omq_f2u(b)));
+  return omq_u2f(d);
+}
+__device__ __forceinline__ float2 omq_fma2(float2 a, float2 b, float2 c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(omq_f2u(a)), "l"(omq_f2u(b)), "l"(omq_f2u(c)));
+  return omq_u2f(d);
+}
+__device__ __forceinline__ float2 omq_add2(float2 a, float2 b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(omq_f2u(a)), "l"(omq_f2u(b)));
+  return omq_u2f(d);
+}
+
+// omq_fakequant of two elements with the paired operations: the same roundings in the same order,
+// so each lane equals the scalar result bit for bit (w - k h as k (-h) + w: the same exact product)
+__device__ __forceinline__ float2 omq_fakequant2(float2 w, const QState& s, float Q, float2* code) {
+  const float2 rh = make_float2(s.rh, s.rh), h = make_float2(s.h, s.h), nh = make_float2(-s.h, -s.h);
+  const float2 x = omq_mul2(w, rh);
+  const float2 k = make_float2(rintf(x.x), rintf(x.y));
+  const float2 r = omq_fma2(k, nh, w);
+  const float2 y = omq_mul2(r, rh);
+  const float2 q = omq_add2(k, make_float2(rintf(y.x), rintf(y.y)));
+  const float2 qz = make_float2(fminf(fmaxf(q.x, -s.z), Q - s.z), fminf(fmaxf(q.y, -s.z), Q - s.z));
+  if (code) *code = omq_add2(qz, make_float2(s.z, s.z));
+  return omq_mul2(qz, h);
+}
+
 // STE pieces of one element: returns dwhat/dh; *inr = 1 when 0 <= c <= Q.  round(u) is -z, the
 // zero point's own rounding.
 __device__ __forceinline__ float omq_ste_dh(float w, const QState& s, float Q, int* inr) {

@@ -46,7 +46,11 @@ __device__ __forceinline__ void lwc_store(const LwcFwdArgs& a, int64_t o, int64_
                                           float Q) {
   float w[8], cd[8];
 #pragma unroll
-  for (int e = 0; e < 8; ++e) w[e] = omq_fakequant(wt[e], qs, Q, &cd[e]);
+  for (int e = 0; e < 8; e += 2) {
+    float2 c2;
+    const float2 v = omq_fakequant2(make_float2(wt[e], wt[e + 1]), qs, Q, &c2);
+    w[e] = v.x; w[e + 1] = v.y; cd[e] = c2.x; cd[e + 1] = c2.y;
+  }
   if (a.Wq) reinterpret_cast<uint4*>(a.Wq + o * a.Cin)[c] = pack_bf16x8(w);
   if (a.codes) {
     uint2 pk;

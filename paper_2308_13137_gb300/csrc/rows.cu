@@ -70,22 +70,30 @@ __device__ __forceinline__ void st_bf16x4(__nv_bfloat16* p, const float* v) {
 template <int NE>
 __device__ __forceinline__ QState row_quantize(float (&val)[NE], const int (&col)[NE], float (&cd)[NE], float Q,
                                                float eps, int* iM_out, int* im_out, float* fsm, int* ism) {
+  static_assert(NE % 2 == 0, "elements are quantized in pairs");
   float M = -INFINITY, m = INFINITY;
 #pragma unroll
   for (int k = 0; k < NE; ++k)
     if (col[k] >= 0) { M = fmaxf(M, val[k]); m = fminf(m, val[k]); }
+  const float lM = M, lm = m;                    // this thread's own extremes
   block_maxmin(M, m, fsm);
   int iM = 0x7fffffff, im = 0x7fffffff;
+  if (lM == M || lm == m) {                      // only the holders of an extreme search its first index
 #pragma unroll
-  for (int k = 0; k < NE; ++k)
-    if (col[k] >= 0) {
-      if (val[k] == M && col[k] < iM) iM = col[k];
-      if (val[k] == m && col[k] < im) im = col[k];
-    }
+    for (int k = 0; k < NE; ++k)
+      if (col[k] >= 0) {
+        if (val[k] == M && col[k] < iM) iM = col[k];
+        if (val[k] == m && col[k] < im) im = col[k];
+      }
+  }
   block_min2i(iM, im, ism);
   const QState qs = omq_qstate(M, m, 1.f, 1.f, Q, eps);
 #pragma unroll
-  for (int k = 0; k < NE; ++k) val[k] = omq_fakequant(val[k], qs, Q, &cd[k]);
+  for (int k = 0; k < NE; k += 2) {
+    float2 c2;
+    const float2 v = omq_fakequant2(make_float2(val[k], val[k + 1]), qs, Q, &c2);
+    val[k] = v.x; val[k + 1] = v.y; cd[k] = c2.x; cd[k + 1] = c2.y;
+  }
   *iM_out = iM;
   *im_out = im;
   return qs;
