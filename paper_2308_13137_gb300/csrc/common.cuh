@@ -234,6 +234,21 @@ __device__ __forceinline__ float omq_ste_dh(float w, const QState& s, float Q, i
   return (c < 0.f) ? ru : (Q + ru);
 }
 
+// omq_ste_dh of two elements with the paired operations (each lane equal to the scalar result)
+__device__ __forceinline__ float2 omq_ste_dh2(float2 w, const QState& s, float Q, int* inr0, int* inr1) {
+  const float2 rh = make_float2(s.rh, s.rh), nh = make_float2(-s.h, -s.h), m1 = make_float2(-1.f, -1.f);
+  const float2 x = omq_mul2(w, rh);
+  const float2 k = make_float2(rintf(x.x), rintf(x.y));
+  const float2 y = omq_mul2(omq_fma2(k, nh, w), rh);
+  const float2 r = omq_add2(k, make_float2(rintf(y.x), rintf(y.y)));
+  const float2 c = omq_add2(r, make_float2(s.z, s.z));
+  const float2 d = omq_fma2(x, m1, r);            // r - x
+  const float ru = -s.z - s.u;
+  const bool in0 = c.x >= 0.f && c.x <= Q, in1 = c.y >= 0.f && c.y <= Q;
+  *inr0 = in0; *inr1 = in1;
+  return make_float2(in0 ? d.x : (c.x < 0.f ? ru : Q + ru), in1 ? d.y : (c.y < 0.f ? ru : Q + ru));
+}
+
 // ------------------------------------------------------------------------------------------------
 // (value, index) reductions with first-index tie break
 // ------------------------------------------------------------------------------------------------

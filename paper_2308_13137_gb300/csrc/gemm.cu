@@ -111,6 +111,20 @@ __device__ __forceinline__ void ldw32(const __nv_bfloat16* p, bool ok, uint4 (&r
 // the code decision, the STE mask and h-path sums, and the LET column terms.  HS / HR: the column
 // scale s / row scale r are present (an absent one is 1, its product skipped, exactly); DR: the row
 // sum for dr is wanted; LET: the column terms for ds (cs) and ddelta (cd).
+// the sums one element adds to, in element order: h path, clamped mass, dr, LET column terms
+template <bool HS, bool HR, bool DR, bool LET>
+__device__ __forceinline__ void lwc_elem(float g, float dh, int inr, float w, float sv, float rr, float dbr, float& Gh,
+                                         float& Gbm, float& drm, float& cs, float& cd) {
+  Gh = fmaf(g, dh, Gh);
+  if (!inr) Gbm += g;
+  const float d = inr ? g : 0.f;
+  if (DR) drm = fmaf(d * w, sv, drm);
+  if (LET) {
+    cs = HR ? (d * w) * rr : d * w;
+    cd = dbr * w;
+  }
+}
+
 template <bool HS, bool HR, bool DR, bool LET>
 __device__ __forceinline__ void lwc_elems(const uint4 (&wc)[4], const float* s_nb, float rr, float dbr, const QState& qs,
                                           float Q, const float (&g)[32], float& Gh, float& Gbm, float& drm,
@@ -125,20 +139,16 @@ __device__ __forceinline__ void lwc_elems(const uint4 (&wc)[4], const float* s_n
       s8[0] = a.x; s8[1] = a.y; s8[2] = a.z; s8[3] = a.w; s8[4] = b.x; s8[5] = b.y; s8[6] = b.z; s8[7] = b.w;
     }
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      const int k = 8 * i + e;
-      float wt = HS ? __fmul_rn(w8[e], s8[e]) : w8[e];
-      if (HR) wt = __fmul_rn(wt, rr);
-      int inr;
-      const float dh = omq_ste_dh(wt, qs, Q, &inr);
-      Gh = fmaf(g[k], dh, Gh);
-      if (!inr) Gbm += g[k];
-      const float d = inr ? g[k] : 0.f;
-      if (DR) drm = fmaf(d * w8[e], HS ? s8[e] : 1.f, drm);
-      if (LET) {
-        cs[k] = HR ? (d * w8[e]) * rr : d * w8[e];
-        cd[k] = dbr * w8[e];
-      }
+    for (int e = 0; e < 8; e += 2) {
+      float2 wt = make_float2(w8[e], w8[e + 1]);
+      if (HS) wt = omq_mul2(wt, make_float2(s8[e], s8[e + 1]));
+      if (HR) wt = omq_mul2(wt, make_float2(rr, rr));
+      int in0, in1;
+      const float2 dh = omq_ste_dh2(wt, qs, Q, &in0, &in1);
+      lwc_elem<HS, HR, DR, LET>(g[8 * i + e], dh.x, in0, w8[e], HS ? s8[e] : 1.f, rr, dbr, Gh, Gbm, drm,
+                                cs[8 * i + e], cd[8 * i + e]);
+      lwc_elem<HS, HR, DR, LET>(g[8 * i + e + 1], dh.y, in1, w8[e + 1], HS ? s8[e + 1] : 1.f, rr, dbr, Gh, Gbm, drm,
+                                cs[8 * i + e + 1], cd[8 * i + e + 1]);
     }
   }
 }
