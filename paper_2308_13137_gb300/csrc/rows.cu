@@ -14,7 +14,10 @@ namespace {
 
 __device__ __forceinline__ float4 ld4(const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); }
 __device__ __forceinline__ float f4get(const float4& v, int e) { return e == 0 ? v.x : (e == 1 ? v.y : (e == 2 ? v.z : v.w)); }
-__device__ __forceinline__ float silu(float g) { return g / (1.f + expf(-g)); }
+// silu(g) = g sigmoid(g); the quotient by the correctly rounded reciprocal (one rounding more than
+// an IEEE division: within 1 ulp of g / (1 + e^-g)); the forward and the backward's recomputation of
+// the quantizer input both use this form
+__device__ __forceinline__ float silu(float g) { return g * __frcp_rn(1.f + expf(-g)); }
 
 // block-wide max and min of values; results in every thread.  smem >= 64 floats.
 __device__ __forceinline__ void block_maxmin(float& M, float& m, float* smem) {
