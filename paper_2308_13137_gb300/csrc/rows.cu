@@ -206,7 +206,8 @@ __device__ __forceinline__ void act_fwd_row(const ActFwdArgs& a, const int64_t t
 
 
 // token rows per CTA of the register-resident forward (rows of up to 4 K columns; the SwiGLU row)
-constexpr int kFwdRows = 2, kFwdRowsSwiglu = 2;
+// and of the q, k, v quantizer forward
+constexpr int kFwdRows = 2, kFwdRowsSwiglu = 2, kQkvFwdRows = 1;
 
 // rows blockIdx.x * R .. + R - 1 (R = a.rows_per_cta, at least 1); the CTA prefetches each next row's
 // inputs into L2 while it works on the current one
@@ -893,8 +894,14 @@ __global__ void __launch_bounds__(NT) qkv_fwd_rows(QkvArgs a) {
   constexpr int NE = 8 * PPT;
   __shared__ float fsm[64];
   __shared__ int ism[64];
-  const int t = blockIdx.x;
   const int dq = a.H * a.hd, dkv = a.Hkv * a.hd;
+  const int t0 = blockIdx.x * kQkvFwdRows, t1 = t0 + kQkvFwdRows < a.T ? t0 + kQkvFwdRows : a.T;
+  for (int t = t0; t < t1; ++t) {
+  if (threadIdx.x == 0 && t + 1 < t1 && gridDim.y != 1) {   // the next row's segment into L2
+    const int sg = (int)blockIdx.y;
+    omq_l2_prefetch(a.Y + (int64_t)(t + 1) * a.ldy + (sg == 0 ? 0 : (sg == 1 ? dq : dq + dkv)),
+                    (uint64_t)(sg == 0 ? dq : dkv) * 4);
+  }
   for (int seg = blockIdx.y; seg < (gridDim.y == 1 ? 3 : (int)blockIdx.y + 1); ++seg) {   // y: one segment per CTA
     QkvRow<PPT> r;
     qkv_load<NT, PPT>(a, seg, t, r);
@@ -916,6 +923,8 @@ __global__ void __launch_bounds__(NT) qkv_fwd_rows(QkvArgs a) {
       }
     }
     (void)W;
+  }
+  __syncthreads();                             // the reduction scratch is reused by the next row
   }
 }
 
@@ -1145,10 +1154,10 @@ int64_t qkv_bwd_nslab(int T) { return (T + kQkvBwdRows - 1) / kQkvBwdRows; }
 omq_status qkv_fwd_launch(cudaStream_t st, const QkvArgs& a) {
   OMQ_REQUIRE(a.hd == 128, OMQ_ERR_UNSUPPORTED);
   const int np = a.H * 16;
-  const dim3 g3((unsigned)a.T, 3);                 // one CTA per (token, q | k | v)
+  const dim3 g3((unsigned)((a.T + kQkvFwdRows - 1) / kQkvFwdRows), 3);   // one CTA per (token rows, q | k | v)
   if (np <= 512) qkv_fwd_rows<128, 4><<<g3, 128, 0, st>>>(a);
-  else if (np <= 1024) qkv_fwd_rows<512, 2><<<a.T, 512, 0, st>>>(a);
-  else if (np <= 2048) qkv_fwd_rows<512, 4><<<a.T, 512, 0, st>>>(a);
+  else if (np <= 1024) qkv_fwd_rows<512, 2><<<g3.x, 512, 0, st>>>(a);
+  else if (np <= 2048) qkv_fwd_rows<512, 4><<<g3.x, 512, 0, st>>>(a);
   else return OMQ_ERR_UNSUPPORTED;
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
