@@ -642,6 +642,7 @@ template <bool PQ>
 __global__ void __launch_bounds__(FA_THREADS, 1)
     flash_bwd_dkv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                          const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
+                         const __grid_constant__ CUtensorMap tmdK, const __grid_constant__ CUtensorMap tmdV,
                          const BwdP p) {
   using L = BL<PQ>;
   constexpr int B_NQD = L::NQD;
@@ -818,22 +819,21 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       ok = waitw(&g_done[b], (last >> 1) & 1, p.status, abort_flag);
     }
     if (ok && nit > 0) {
+      // dV, dK leave through the copy engine: each warp stages its 32 x 32 blocks in two 4 KB slots
+      // of the P^T / dS^T buffers (every product that read them has completed) and stores them
+      // whole; rows past T are clipped by the copy
       tc_fence_after();
+      uint8_t* slots = smem + B_PT + (warp - 2) * 8192;
+      int ns = 0;
 #pragma unroll 1
       for (int c = 2 * half; c < 2 * half + 2; ++c) {
         float dv[32], dk[32];
         tmem_ld32(tmem + 256 + lane_off + 32 * c, dv);
         tmem_ld32(tmem + 384 + lane_off + 32 * c, dk);
-        if (key < p.T) {
-          float4* a = reinterpret_cast<float4*>(p.dV + (int64_t)key * p.ldkv + g * HD + 32 * c);
-          float4* b = reinterpret_cast<float4*>(p.dK + (int64_t)key * p.ldkv + g * HD + 32 * c);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            a[i] = make_float4(dv[4 * i], dv[4 * i + 1], dv[4 * i + 2], dv[4 * i + 3]);
-            b[i] = make_float4(dk[4 * i], dk[4 * i + 1], dk[4 * i + 2], dk[4 * i + 3]);
-          }
-        }
+        store_block32(&tmdV, slots + (ns++ & 1) * 4096, dv, lane, g * HD + 32 * c, kb * 128 + q * 32);
+        store_block32(&tmdK, slots + (ns++ & 1) * 4096, dk, lane, g * HD + 32 * c, kb * 128 + q * 32);
       }
+      if (lane == 0) bulk_wait_all();
     } else if (ok && nit == 0 && key < p.T) {        // keys no query sees (cannot happen for T > 0)
       for (int c = 64 * half; c < 64 * half + 64; ++c) {
         p.dV[(int64_t)key * p.ldkv + g * HD + c] = 0.f;
@@ -865,7 +865,7 @@ template <int MODE>
 __global__ void __launch_bounds__(FA_THREADS, 1)
     flash_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmdO,
-                        const BwdP p) {
+                        const __grid_constant__ CUtensorMap tmdQ, const BwdP p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   Ctl* ctl = reinterpret_cast<Ctl*>(smem + Q_CTL);
@@ -1050,17 +1050,19 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
             make_float4(t[0] + q_M * dM + q_m * dm, dM, dm, 0.f);
       }
     } else if (ok) {
+      // dQ through the copy engine, staged in the Q / dO tiles (every product that read them has
+      // completed): two 4 KB slots per warp, rows past T clipped by the copy
       tc_fence_after();
+      uint8_t* slots = smem + Q_Q + (warp - 2) * 8192;
+      int ns = 0;
 #pragma unroll 1
       for (int c = 2 * half; c < 2 * half + 2; ++c) {
         float o[32];
         tmem_ld32(tmem + 256 + lane_off + 32 * c, o);
-        if (row_ok) {
-          float4* a = reinterpret_cast<float4*>(p.dQ + (int64_t)row * p.ldq + h * HD + 32 * c);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) a[i] = make_float4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
-        }
+        store_block32(&tmdQ, slots + (ns++ & 1) * 4096, o, lane, h * HD + 32 * c, qb * 128 + q * 32);
       }
+      if (lane == 0) bulk_wait_all();
+      (void)row_ok;
     }
   }
   tc_fence_before();
@@ -1137,6 +1139,10 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
   CUtensorMap tk64, tv64;
   ok = ok && omq_make_map_bf16(&tk64, a.K, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
   ok = ok && omq_make_map_bf16(&tv64, a.V, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
+  CUtensorMap tdq, tdk, tdv;                       // fp32 outputs, 32 x 32 store boxes
+  ok = ok && omq_make_map_f32_out(&tdq, a.dQ, (int64_t)a.H * HD, a.T, a.ldg);
+  ok = ok && omq_make_map_f32_out(&tdk, a.dK, (int64_t)a.Hkv * HD, a.T, a.ldgkv);
+  ok = ok && omq_make_map_f32_out(&tdv, a.dV, (int64_t)a.Hkv * HD, a.T, a.ldgkv);
   if (!ok) return OMQ_ERR_UNSUPPORTED;
   static bool attr = false;
   if (!attr) {
@@ -1160,20 +1166,20 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
   dim3 g2((unsigned)a.H, (unsigned)((a.T + 127) / 128));
   if (pq) {
     // row statistics first (they replace D = rowsum(dO * O), which no longer is sum_j P_j dP_j)
-    flash_bwd_dq_kernel<1><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, p);
+    flash_bwd_dq_kernel<1><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, tdq, p);
     OMQ_LAUNCH_CHECK();
-    flash_bwd_dkv_kernel<true><<<g1, FA_THREADS, BL<true>::SMEM, st>>>(tq64, tk, tv, tdo64, p);
+    flash_bwd_dkv_kernel<true><<<g1, FA_THREADS, BL<true>::SMEM, st>>>(tq64, tk, tv, tdo64, tdk, tdv, p);
     OMQ_LAUNCH_CHECK();
-    flash_bwd_dq_kernel<2><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, p);
+    flash_bwd_dq_kernel<2><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, tdq, p);
     OMQ_LAUNCH_CHECK();
     return OMQ_OK;
   }
   const int64_t rows = (int64_t)a.T * a.H;
   attn_rowdot_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(a.T, a.H, a.dO, a.lddo, a.O, a.ldo, a.D, ldl);
   OMQ_LAUNCH_CHECK();
-  flash_bwd_dkv_kernel<false><<<g1, FA_THREADS, BL<false>::SMEM, st>>>(tq64, tk, tv, tdo64, p);
+  flash_bwd_dkv_kernel<false><<<g1, FA_THREADS, BL<false>::SMEM, st>>>(tq64, tk, tv, tdo64, tdk, tdv, p);
   OMQ_LAUNCH_CHECK();
-  flash_bwd_dq_kernel<0><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, p);
+  flash_bwd_dq_kernel<0><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, tdq, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }

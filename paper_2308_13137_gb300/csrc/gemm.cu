@@ -875,6 +875,10 @@ omq_status gemm_launch(cudaStream_t st, int64_t M, int64_t N, int64_t K, int64_t
 
 int gemm_n_tile(int64_t N) { return N % 256 == 0 ? 256 : 128; }
 
+bool omq_make_map_f32_out(CUtensorMap* map, float* ptr, int64_t N, int64_t M, int64_t ld) {
+  return make_map_c(map, ptr, N, M, 1, ld, 0);
+}
+
 bool omq_make_map_bf16(CUtensorMap* map, const void* ptr, int64_t inner, int64_t rows, int64_t batch, int64_t ld,
                        int64_t bs, int box_inner, int box_rows) {
   PFN_encodeTiled_t enc = get_encode();

@@ -264,8 +264,33 @@ static __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// A warp's 32 x 32 fp32 block (lane = row, v = its 32 consecutive columns) to global memory at
+// column c0, row c1 of `map`: staged in a 4 KB 128-byte-swizzled shared-memory slot (16-byte chunk
+// k of row r at chunk k ^ (r & 7)) and stored by the copy engine, which clips rows and columns
+// outside the tensor.  Two slots per warp, used alternately: the store that last read `slot` is
+// waited for first.  The caller waits for all its stores (bulk_wait_all) before exiting.
+static __device__ __forceinline__ void store_block32(const CUtensorMap* map, uint8_t* slot, const float (&v)[32], int lane,
+                                                     int c0, int c1) {
+  if (lane == 0) bulk_wait_read1();
+  __syncwarp();
+  uint8_t* my_row = slot + lane * 128;
+#pragma unroll
+  for (int k = 0; k < 8; ++k)
+    *reinterpret_cast<float4*>(my_row + ((k ^ (lane & 7)) << 4)) = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+  fence_async_smem();                      // generic-proxy writes -> visible to the copy engine
+  __syncwarp();
+  if (lane == 0) {
+    tma_store_3d(map, slot, c0, c1, 0);
+    bulk_commit();
+  }
+}
+
 }  // namespace tc
 
 // Host: 3-D bf16 tensor map {inner, rows, batch}, box {box_inner, box_rows, 1}, 128-byte swizzle.
 bool omq_make_map_bf16(CUtensorMap* map, const void* ptr, int64_t inner, int64_t rows, int64_t batch, int64_t ld,
                        int64_t bs, int box_inner, int box_rows);
+// Host: fp32 output map {N, M, 1} with row stride ld (elements), box {32, 32, 1}, 128-byte swizzle:
+// the layout of a warp's 32 x 32 staging block for tma_store_3d
+bool omq_make_map_f32_out(CUtensorMap* map, float* ptr, int64_t N, int64_t M, int64_t ld);
+
