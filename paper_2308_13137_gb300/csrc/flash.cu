@@ -118,7 +118,7 @@ static_assert(F_SMEM <= 227 * 1024, "forward shared memory");
 template <bool PQ>
 __global__ void __launch_bounds__(FA_THREADS, 1)
     flash_fwd_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                     const __grid_constant__ CUtensorMap tmV, const FwdP p) {
+                     const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO, const FwdP p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   Ctl* ctl = reinterpret_cast<Ctl*>(smem + F_CTL);
@@ -350,17 +350,17 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       if (lane == 0) mbar_arrive(p_full);
     }
     if (ok && waitw(o_done, (nkb - 1) & 1, p.status, abort_flag)) {
+      // O through the copy engine, staged in the K ring (every product that read it has completed)
       tc_fence_after();
+      uint8_t* slots = smem + F_K + (warp - 2) * 8192;
+      int ns = 0;
 #pragma unroll 1
       for (int c = 2 * half; c < 2 * half + 2; ++c) {
         float o[32];
         tmem_ld32(tmem + 256 + lane_off + 32 * c, o);
-        if (row < p.T) {
-          float4* dst = reinterpret_cast<float4*>(p.O + (int64_t)row * p.ldo + h * HD + 32 * c);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) dst[i] = make_float4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
-        }
+        store_block32(&tmO, slots + (ns++ & 1) * 4096, o, lane, h * HD + 32 * c, qb * 128 + q * 32);
       }
+      if (lane == 0) bulk_wait_all();
       if (row < p.T && half == 0) p.lse[(int64_t)h * p.ldl + row] = mt + log2f(lt);
       if constexpr (PQ) {
         if (row < p.T && half == 0) {
@@ -396,7 +396,7 @@ constexpr float F_TAU = 8.f;                          // unnormalised probabilit
 
 __global__ void __launch_bounds__(FA_THREADS, 1)
     flash_fwd1_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                      const __grid_constant__ CUtensorMap tmV, const FwdP p) {
+                      const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO, const FwdP p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   Ctl* ctl = reinterpret_cast<Ctl*>(smem + F_CTL);
@@ -559,21 +559,20 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
     const float lt = l0 * f0 + l1 * f1;
     const float a0 = f0 / lt, a1 = f1 / lt;
     if (ok) {
+      // O through the copy engine, staged in the K ring (every product that read it has completed)
       tc_fence_after();
+      uint8_t* slots = smem + F_K + (warp - 2) * 8192;
+      int ns = 0;
 #pragma unroll 1
       for (int c = 2 * half; c < 2 * half + 2; ++c) {
         float o0[32], o1[32];
         tmem_ld32(tmem + 256 + lane_off + 32 * c, o0);
         tmem_ld32(tmem + 384 + lane_off + 32 * c, o1);
-        if (row < p.T) {
-          float4* dst = reinterpret_cast<float4*>(p.O + (int64_t)row * p.ldo + h * HD + 32 * c);
 #pragma unroll
-          for (int i = 0; i < 8; ++i)
-            dst[i] = make_float4(fmaf(o0[4 * i], a0, o1[4 * i] * a1), fmaf(o0[4 * i + 1], a0, o1[4 * i + 1] * a1),
-                                 fmaf(o0[4 * i + 2], a0, o1[4 * i + 2] * a1),
-                                 fmaf(o0[4 * i + 3], a0, o1[4 * i + 3] * a1));
-        }
+        for (int i = 0; i < 32; ++i) o0[i] = fmaf(o0[i], a0, o1[i] * a1);
+        store_block32(&tmO, slots + (ns++ & 1) * 4096, o0, lane, h * HD + 32 * c, qb * 128 + q * 32);
       }
+      if (lane == 0) bulk_wait_all();
       if (row < p.T && half == 0) p.lse[(int64_t)h * p.ldl + row] = Mt + log2f(lt);
     }
   }
@@ -1095,6 +1094,8 @@ omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
   CUtensorMap tk64, tv64;
   ok = ok && omq_make_map_bf16(&tk64, a.K, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
   ok = ok && omq_make_map_bf16(&tv64, a.V, (int64_t)a.Hkv * HD, a.T, 1, a.ldkv, 0, 64, 64);
+  CUtensorMap to;                                   // fp32 O, 32 x 32 store boxes
+  ok = ok && omq_make_map_f32_out(&to, a.O, (int64_t)a.H * HD, a.T, a.ldo);
   if (!ok) return OMQ_ERR_UNSUPPORTED;
   static bool attr = false;
   if (!attr) {
@@ -1109,8 +1110,8 @@ omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
   p.O = a.O; p.ldo = a.ldo; p.lse = a.lse; p.status = a.status;
   p.Q = pq ? (float)((1 << a.pbits) - 1) : 0.f; p.eps = a.eps; p.pqr = a.pqr;
   dim3 grid((unsigned)a.H, (unsigned)((a.T + 127) / 128));
-  if (pq) flash_fwd_kernel<true><<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, p);
-  else flash_fwd1_kernel<<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, p);
+  if (pq) flash_fwd_kernel<true><<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, to, p);
+  else flash_fwd1_kernel<<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, to, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
