@@ -36,6 +36,7 @@ struct FlashArgs {
   float* lse;
   const __nv_bfloat16* dO; int64_t lddo;
   float* D;
+  int d_ready;            // 1: D already holds rowsum(dO * O) (formed by the producer of dO)
   float* dQ; int64_t ldg;
   float* dK; float* dV; int64_t ldgkv;
   int32_t* status;

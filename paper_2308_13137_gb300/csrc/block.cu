@@ -529,13 +529,15 @@ omq_status block_bwd(Ctx& c, const float* x, const float* y, const float* y_fp, 
   bo.producer = AP_PLAIN; bo.X = w.O; bo.ldx = c.dq; bo.T = c.T; bo.C = c.dq; bo.h = w.so.h; bo.z = w.so.z;
   bo.imax = w.so.imax; bo.imin = w.so.imin; bo.dXq = w.dOh; bo.lddq = c.dq; bo.dX = nullptr; bo.lddx = c.dq;
   bo.dXb = w.dO_b; bo.lddxb = c.dq; bo.rows_per_cta = kRowsPlain; bo.abits = cfg.abits; bo.eps = cfg.h_eps;
+  const bool d_fused = !flash_pq_on(cfg.pbits);   // rowsum(dO * O) of the attention backward, formed here
+  if (d_fused) { bo.rowdot = w.Drow; bo.ldrow = (c.T + 3) / 4 * 4; }
   OMQ_TRY(act_bwd_launch(st, bo));
 
   // ---- attention: dQ, dK, dV from the saved log-sum-exp (scores recomputed, never stored) --------
   FlashArgs fa{};
   fa.T = (int)c.T; fa.H = (int)c.H; fa.Hkv = (int)c.Hkv; fa.hd = (int)c.hd;
   fa.Q = w.Qh; fa.K = w.Kh; fa.V = w.Vh; fa.ldq = c.dq; fa.ldkv = c.dkv;
-  fa.O = w.O; fa.ldo = c.dq; fa.lse = w.lse; fa.dO = w.dO_b; fa.lddo = c.dq; fa.D = w.Drow;
+  fa.O = w.O; fa.ldo = c.dq; fa.lse = w.lse; fa.dO = w.dO_b; fa.lddo = c.dq; fa.D = w.Drow; fa.d_ready = d_fused;
   fa.dQ = w.dQKV; fa.ldg = c.nqkv; fa.dK = w.dQKV + c.dq; fa.dV = w.dQKV + c.dq + c.dkv; fa.ldgkv = c.nqkv;
   fa.status = status;
   fa.pbits = cfg.pbits; fa.eps = cfg.h_eps; fa.pqr = w.pqr; fa.pqb = w.pqb; fa.ldl = (int)((c.T + 3) / 4 * 4);

@@ -1175,9 +1175,11 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
     OMQ_LAUNCH_CHECK();
     return OMQ_OK;
   }
-  const int64_t rows = (int64_t)a.T * a.H;
-  attn_rowdot_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(a.T, a.H, a.dO, a.lddo, a.O, a.ldo, a.D, ldl);
-  OMQ_LAUNCH_CHECK();
+  if (!a.d_ready) {
+    const int64_t rows = (int64_t)a.T * a.H;
+    attn_rowdot_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(a.T, a.H, a.dO, a.lddo, a.O, a.ldo, a.D, ldl);
+    OMQ_LAUNCH_CHECK();
+  }
   flash_bwd_dkv_kernel<false><<<g1, FA_THREADS, BL<false>::SMEM, st>>>(tq64, tk, tv, tdo64, tdk, tdv, p);
   OMQ_LAUNCH_CHECK();
   flash_bwd_dq_kernel<0><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, tdq, p);

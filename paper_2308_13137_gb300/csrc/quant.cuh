@@ -75,6 +75,8 @@ struct ActBwdArgs {
   float* dU; __nv_bfloat16* dUb;     // SWIGLU: d up (same ld as dX / dXb)
   const float* resid;                // RMS: residual gradient added to dX (nullable)
   float* part_s; float* part_d;      // [T / rows_per_cta, C] LET column partials (nullable)
+  float* rowdot; int64_t ldrow;      // PLAIN over [T, heads x 128] rows: D[head, t] = sum of bf16(dX) X over
+                                     // the head's 128 columns, row stride ldrow (nullable; needs dXb)
   int rows_per_cta;
   int abits; float eps;
 };

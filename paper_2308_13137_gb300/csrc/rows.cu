@@ -411,6 +411,11 @@ __device__ __forceinline__ float3 block_sum3(float a, float b, float c, float* s
   return make_float3(warp_sum(x), warp_sum(y), warp_sum(z));
 }
 
+// o . d over one float4 group, in the order of the attention backward's own row dot
+__device__ __forceinline__ float rowdot4(const float4 o, const float (&d)[4]) {
+  return o.x * d[0] + o.y * d[1] + o.z * d[2] + o.w * d[3];
+}
+
 template <int P>
 struct ActBwdRow {
   const ActBwdArgs& a;
@@ -437,7 +442,7 @@ struct ActBwdRow {
   }
 };
 
-template <int P, int VPT, int JB, int MINB, bool SUMS>
+template <int P, int VPT, int JB, int MINB, bool SUMS, bool RD = false>
 __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a) {
   constexpr int NT = ACT_BWD_NT;
   constexpr bool LETP = (P == AP_LET || P == AP_RMS_LET);
@@ -458,6 +463,11 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
   // and the masked gradient of its elements in registers for pass 2
   constexpr bool RS = SUMS && VPT <= 8;
   constexpr bool KEEP = RS && P == AP_RMS_LET;
+  // the plain form with a.rowdot: D[head, t] = the sum of bf16(dX) X over each 128-column head (the
+  // attention backward's rowsum(dO * O)), taken while the row is here; the float4 group j of a warp
+  // is one head (lane L holds its columns 4L .. 4L + 3)
+  static_assert(!RD || (P == AP_PLAIN && !SUMS), "the row dot is a form of the plain producer");
+  float dpart[RD ? VPT : 1];
   __shared__ float4 rs_sm[RS ? VPT * NT : 1];
   float xk[KEEP ? NE : 1], dk[KEEP ? NE : 1];
 #pragma unroll
@@ -554,7 +564,22 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
           } else if (P == AP_PLAIN || P == AP_LET) {
             if (a.dX) *reinterpret_cast<float4*>(a.dX + t * a.lddx + 4 * vi) = make_float4(o1[0], o1[1], o1[2], o1[3]);
             if (a.dXb) st_bf16x4(a.dXb + t * a.lddxb + 4 * vi, o1);
+            if constexpr (RD) {   // C % 128 == 0: the whole warp is here
+              float b4[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) b4[e] = __bfloat162float(__float2bfloat16_rn(o1[e]));
+              dpart[j] = rowdot4(x4[jj], b4);
+            }
           }
+        }
+      }
+      if constexpr (RD) {
+#pragma unroll
+        for (int j = 0; j < VPT; ++j) {
+          const int64_t v0 = (int64_t)j * NT + (tid & ~31);   // the head's first float4 (warp-uniform)
+          if (v0 >= nv) break;
+          const float sd = warp_sum(dpart[j]);
+          if ((tid & 31) == 0) a.rowdot[(v0 >> 5) * a.ldrow + t] = sd;
         }
       }
       if (!quant && !(P == AP_RMS_LET && want_out)) continue;
@@ -601,6 +626,23 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
               if (a.dX) a.dX[t * a.lddx + c] = dn;
               if (a.dXb) a.dXb[t * a.lddxb + c] = f_to_bf16(dn);
             }
+          }
+        }
+        if constexpr (RD) {     // the heads of the routed elements, summed again
+          __syncwarp();                                  // the owner's rewrite, seen by its warp
+#pragma unroll
+          for (int r = 0; r < 2; ++r) {
+            const int64_t c = r == 0 ? iM : im;
+            if (r == 1 && (im >> 7) == (iM >> 7)) break;
+            const int64_t v0 = (c >> 2) & ~(int64_t)31;    // the head's first float4
+            if ((int)((v0 % NT) >> 5) != (tid >> 5)) continue;
+            const int64_t vi = v0 + (tid & 31);
+            const uint2 u = *reinterpret_cast<const uint2*>(a.dXb + t * a.lddxb + 4 * vi);
+            const float2 b01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+            const float2 b23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+            const float b4[4] = {b01.x, b01.y, b23.x, b23.y};
+            const float sd = warp_sum(rowdot4(ld4(xr + 4 * vi), b4));
+            if ((tid & 31) == 0) a.rowdot[(v0 >> 5) * a.ldrow + t] = sd;
           }
         }
       }
@@ -770,10 +812,10 @@ static omq_status act_fwd_dispatch(cudaStream_t st, const ActFwdArgs& a0) {
   return OMQ_OK;
 }
 
-template <int PRODUCER, int VPT, int JB, int MINB, bool SUMS>
+template <int PRODUCER, int VPT, int JB, int MINB, bool SUMS, bool RD = false>
 static omq_status act_bwd_go(cudaStream_t st, const ActBwdArgs& a) {
   const int64_t nparts = (a.T + a.rows_per_cta - 1) / a.rows_per_cta;
-  act_bwd_stream<PRODUCER, VPT, JB, MINB, SUMS><<<(unsigned)nparts, ACT_BWD_NT, 0, st>>>(a);
+  act_bwd_stream<PRODUCER, VPT, JB, MINB, SUMS, RD><<<(unsigned)nparts, ACT_BWD_NT, 0, st>>>(a);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -784,6 +826,16 @@ template <int PRODUCER>
 static omq_status act_bwd_dispatch(cudaStream_t st, const ActBwdArgs& a) {
   const int64_t vpt = (a.C / 4 + ACT_BWD_NT - 1) / ACT_BWD_NT;
   const bool sums = PRODUCER != AP_SWIGLU && a.part_s != nullptr;
+  if constexpr (PRODUCER == AP_PLAIN) {
+    if (a.rowdot) {   // the row dot's partials take registers: loads in pairs to keep four CTAs per SM (two for longer rows)
+      if (sums) return OMQ_ERR_UNSUPPORTED;
+      if (vpt <= 4) return act_bwd_go<PRODUCER, 4, 2, 4, false, true>(st, a);
+      if (vpt <= 8) return act_bwd_go<PRODUCER, 8, 4, 2, false, true>(st, a);
+      if (vpt <= 16) return act_bwd_go<PRODUCER, 16, 4, 2, false, true>(st, a);
+      if (vpt <= 28) return act_bwd_go<PRODUCER, 28, 4, 2, false, true>(st, a);
+      return OMQ_ERR_UNSUPPORTED;
+    }
+  }
   if (!sums) {
     if (vpt <= 4) return act_bwd_go<PRODUCER, 4, 4, 4, false>(st, a);
     if (vpt <= 8) return act_bwd_go<PRODUCER, 8, 4, 4, false>(st, a);
@@ -814,6 +866,7 @@ omq_status act_fwd_launch(cudaStream_t st, const ActFwdArgs& a) {
 omq_status act_bwd_launch(cudaStream_t st, const ActBwdArgs& a0) {
   ActBwdArgs a = a0;
   OMQ_REQUIRE(a.C % 8 == 0 && a.T > 0, OMQ_ERR_SHAPE);
+  OMQ_REQUIRE(!a.rowdot || (a.producer == AP_PLAIN && a.dXb && a.C % 128 == 0 && a.ldrow >= a.T), OMQ_ERR_INVALID_ARG);
   if (a.rows_per_cta <= 0) a.rows_per_cta = 4;
   switch (a.producer) {
     case AP_PLAIN: return act_bwd_dispatch<AP_PLAIN>(st, a);
