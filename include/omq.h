@@ -285,10 +285,7 @@ omq_status omq_block_forward(omq_stream_t stream, const omq_block_shape* shape,
  * graph on `stream`.  The library keeps no state keyed on the caller's pointers; a captured graph
  * does: it replays the addresses it was captured with.  A caller that replays (the package's
  * BlockState looks its graphs up by the addresses of x and y_fp) refills the same buffers in place
- * between replays and keeps them alive; new buffers need a new capture.  Every kernel is launched
- * with programmatic stream serialization and waits (griddepcontrol.wait) for the work before it on
- * its stream before touching global memory, so stream order holds as with plain launches; a
- * captured graph keeps those edges as programmatic ones. */
+ * between replays and keeps them alive; new buffers need a new capture. */
 omq_status omq_block_step(omq_stream_t stream, const omq_block_shape* shape,
                           const omq_block_weights* w, const omq_block_params* theta,
                           const float* x, const float* y_fp, float* y, float* loss,

@@ -10,7 +10,6 @@
 struct RopeFreq { double inv[128]; };
 
 __global__ void rope_table_kernel(int T, int half, RopeFreq f, float* cs) {
-  omq_pdl_enter();
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= (int64_t)T * half) return;
   const int t = (int)(i / half), j = (int)(i % half);
@@ -30,7 +29,7 @@ omq_status rope_table(cudaStream_t st, int T, int hd, float theta, float* cs) {
   const int half = hd / 2;
   for (int j = 0; j < half; ++j) f.inv[j] = std::pow((double)theta, -2.0 * (double)j / (double)hd);
   const int64_t n = (int64_t)T * half;
-  omq_launch(rope_table_kernel, (unsigned)((n + 255) / 256), 256, 0, st, T, half, f, cs);
+  rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(T, half, f, cs);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -39,7 +38,6 @@ omq_status rope_table(cudaStream_t st, int T, int hd, float theta, float* cs) {
 // [v, out] LET pair helpers
 // ------------------------------------------------------------------------------------------------
 __global__ void qkv_row_vectors_kernel(int dq, int dkv, const float* so, const float* do_, float* r, float* shift) {
-  omq_pdl_enter();
   int i = blockIdx.x * blockDim.x + threadIdx.x;
   int n = dq + 2 * dkv;
   if (i >= n) return;
@@ -50,14 +48,13 @@ __global__ void qkv_row_vectors_kernel(int dq, int dkv, const float* so, const f
 
 omq_status qkv_row_vectors(cudaStream_t st, int dq, int dkv, const float* so, const float* do_, float* r, float* shift) {
   int n = dq + 2 * dkv;
-  omq_launch(qkv_row_vectors_kernel, (n + 255) / 256, 256, 0, st, dq, dkv, so, do_, r, shift);
+  qkv_row_vectors_kernel<<<(n + 255) / 256, 256, 0, st>>>(dq, dkv, so, do_, r, shift);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 __global__ void let_vo_finalize_kernel(int dkv, const float* so, const float* dr_v, const float* dBv, const float* Bv,
                                        float* dso, float* ddo, int accumulate) {
-  omq_pdl_enter();
   int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= dkv) return;
   const float s = so[c];
@@ -71,7 +68,7 @@ __global__ void let_vo_finalize_kernel(int dkv, const float* so, const float* dr
 
 omq_status let_vo_finalize(cudaStream_t st, int dkv, const float* so, const float* dr_v, const float* dBv,
                            const float* Bv, float* dso, float* ddo, int accumulate) {
-  omq_launch(let_vo_finalize_kernel, (dkv + 255) / 256, 256, 0, st, dkv, so, dr_v, dBv, Bv, dso, ddo, accumulate);
+  let_vo_finalize_kernel<<<(dkv + 255) / 256, 256, 0, st>>>(dkv, so, dr_v, dBv, Bv, dso, ddo, accumulate);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }

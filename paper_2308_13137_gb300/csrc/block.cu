@@ -695,13 +695,11 @@ omq_status omq_block_step(omq_stream_t stream, const omq_block_shape* shape, con
 // single quantized linear
 // ---------------------------------------------------------------------------------------------------
 __global__ void add_vec_kernel(float* y, const float* x, int64_t n) {
-  omq_pdl_enter();
   int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) y[i] += x[i];
 }
 
 __global__ void f32_to_bf16_kernel(const float* x, __nv_bfloat16* y, int64_t n) {
-  omq_pdl_enter();
   int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) y[i] = __float2bfloat16_rn(x[i]);
 }
@@ -724,7 +722,7 @@ omq_status omq_qlinear_fwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t 
                                       let ? sv->b_tilde : nullptr)));
   const float* bias = nullptr;
   if (let) {
-    if (B) { omq_launch(add_vec_kernel, (unsigned)((Cout + 255) / 256), 256, 0, st, sv->b_tilde, B, Cout); OMQ_LAUNCH_CHECK(); }
+    if (B) { add_vec_kernel<<<(unsigned)((Cout + 255) / 256), 256, 0, st>>>(sv->b_tilde, B, Cout); OMQ_LAUNCH_CHECK(); }
     bias = sv->b_tilde;
   } else if (B) {
     OMQ_TRY(vec_copy(st, sv->b_tilde, B, Cout));
@@ -785,7 +783,7 @@ omq_status omq_qlinear_bwd(omq_stream_t stream, int64_t T, int64_t Cin, int64_t 
   int64_t pe = imax64((int64_t)lwc_bwd_scratch_bytes(Cout, Cin) / 4 + 64, 2 * ((T + 3) / 4) * Cin);
   pe = imax64(pe, colsum_rows_parts(T) * Cout);
   float* part = c.take<float>(pe);
-  omq_launch(f32_to_bf16_kernel, (unsigned)((T * Cout + 255) / 256), 256, 0, st, dY, dYb, T * Cout);
+  f32_to_bf16_kernel<<<(unsigned)((T * Cout + 255) / 256), 256, 0, st>>>(dY, dYb, T * Cout);
   OMQ_LAUNCH_CHECK();
   OMQ_TRY(gemm_dw(st, T, Cout, Cin, dYb, (const bf16*)sv->x_hat, dWh, cfg->dev_status));
   if (let) OMQ_TRY(colsum_rows(st, dY, T, Cout, Cout, part, dB, 1.f, 0));

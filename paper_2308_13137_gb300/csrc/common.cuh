@@ -4,7 +4,6 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 #include <math.h>
-#include <utility>
 
 #include "omq.h"
 
@@ -18,32 +17,6 @@
 void omq_count_launch();
 #define OMQ_LAUNCH_CHECK() do { omq_count_launch(); if (cudaPeekAtLastError() != cudaSuccess) { cudaGetLastError(); return OMQ_ERR_CUDA; } } while (0)
 #define OMQ_TRY(expr) do { omq_status _s = (expr); if (_s != OMQ_OK) return _s; } while (0)
-
-// ------------------------------------------------------------------------------------------------
-// programmatic dependent launch.  Every kernel of the library is launched with programmatic stream
-// serialization, and none of them triggers its successor early: the successor launches as the
-// kernel's last CTAs exit, so its CTAs are placed, and run setup that touches no global memory
-// (mbarrier init, tensor-memory allocation), while the kernel's writes drain, instead of after the
-// whole grid is retired.  Each kernel waits for its predecessor to complete, writes visible
-// (griddepcontrol.wait), before its first global load or store, so a kernel never overlaps data it
-// depends on and a chain of them keeps the stream order.  (Triggering at CTA start instead let the
-// next kernel's waiting CTAs take the SM slots that the auxiliary stream's kernels overlap in, and
-// lost more than it won.)
-// ------------------------------------------------------------------------------------------------
-template <typename... KP, typename... A>
-static inline cudaError_t omq_launch(void (*kernel)(KP...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
-                                     A&&... args) {
-  cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  at[0].val.programmaticStreamSerializationAllowed = 1;
-  cudaLaunchConfig_t c = {};
-  c.gridDim = grid; c.blockDim = block; c.dynamicSmemBytes = smem; c.stream = st;
-  c.attrs = at; c.numAttrs = 1;
-  return cudaLaunchKernelEx(&c, kernel, std::forward<A>(args)...);
-}
-
-// the predecessor on the stream complete and its writes visible (a no-op without the launch attribute)
-__device__ __forceinline__ void omq_pdl_enter() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 static inline bool omq_aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 static inline bool omq_bits_ok(int b) { return (b >= 2 && b <= 8) || b == 16; }

@@ -154,7 +154,6 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = ctl->tmem;           // S buffers at columns 0 / 128, O at 256
-  omq_pdl_enter();                           // setup done: the predecessor's outputs from here on
 
   // iterations 0 .. nkb-1: statistics pass (S only: row max m, row sum l of exp2(c S - m));
   // iterations nkb .. 2 nkb-1: output pass (S again, P = bf16(exp2(c S - m) / l), O += P V)
@@ -432,7 +431,6 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = ctl->tmem;           // S buffers at columns 0 / 128, O_0 at 256, O_1 at 384
-  omq_pdl_enter();                           // setup done: the predecessor's outputs from here on
 
   if (warp == 0 && lane == 0) {
     mbar_expect_tx(q_full, F_TILE);
@@ -591,7 +589,6 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
 // ================================================================================================
 __global__ void attn_rowdot_kernel(int T, int H, const __nv_bfloat16* __restrict__ dO, int64_t lddo,
                                    const float* __restrict__ O, int64_t ldo, float* __restrict__ D, int ldl) {
-  omq_pdl_enter();
   const int64_t w = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (w >= (int64_t)T * H) return;
@@ -683,7 +680,6 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
   tc_fence_after();
   // tensor memory: S^T at 0 / 64, dP^T at 128 / 192 (per buffer), dV at 256, dK at 384
   const uint32_t tmem = ctl->tmem;
-  omq_pdl_enter();                           // setup done: the predecessor's outputs from here on
 
   if (warp == 0 && lane == 0) {
     mbar_expect_tx(kv_full, 2 * F_TILE);
@@ -901,7 +897,6 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = ctl->tmem;       // S at 0 / 64, dP at 128 / 192, dQ at 256
-  omq_pdl_enter();                           // setup done: the predecessor's outputs from here on
 
   if (warp == 0 && lane == 0) {
     mbar_expect_tx(q_full, 2 * F_TILE);
@@ -1115,8 +1110,8 @@ omq_status flash_fwd_launch(cudaStream_t st, const FlashArgs& a) {
   p.O = a.O; p.ldo = a.ldo; p.lse = a.lse; p.status = a.status;
   p.Q = pq ? (float)((1 << a.pbits) - 1) : 0.f; p.eps = a.eps; p.pqr = a.pqr;
   dim3 grid((unsigned)a.H, (unsigned)((a.T + 127) / 128));
-  if (pq) omq_launch(flash_fwd_kernel<true>, grid, FA_THREADS, F_SMEM, st, tq, tk, tv, to, p);
-  else omq_launch(flash_fwd1_kernel, grid, FA_THREADS, F_SMEM, st, tq, tk, tv, to, p);
+  if (pq) flash_fwd_kernel<true><<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, to, p);
+  else flash_fwd1_kernel<<<grid, FA_THREADS, F_SMEM, st>>>(tq, tk, tv, to, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -1172,22 +1167,22 @@ omq_status flash_bwd_launch(cudaStream_t st, const FlashArgs& a) {
   dim3 g2((unsigned)a.H, (unsigned)((a.T + 127) / 128));
   if (pq) {
     // row statistics first (they replace D = rowsum(dO * O), which no longer is sum_j P_j dP_j)
-    omq_launch(flash_bwd_dq_kernel<1>, g2, FA_THREADS, Q_SMEM, st, tq, tk64, tv64, tdo, tdq, p);
+    flash_bwd_dq_kernel<1><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, tdq, p);
     OMQ_LAUNCH_CHECK();
-    omq_launch(flash_bwd_dkv_kernel<true>, g1, FA_THREADS, BL<true>::SMEM, st, tq64, tk, tv, tdo64, tdk, tdv, p);
+    flash_bwd_dkv_kernel<true><<<g1, FA_THREADS, BL<true>::SMEM, st>>>(tq64, tk, tv, tdo64, tdk, tdv, p);
     OMQ_LAUNCH_CHECK();
-    omq_launch(flash_bwd_dq_kernel<2>, g2, FA_THREADS, Q_SMEM, st, tq, tk64, tv64, tdo, tdq, p);
+    flash_bwd_dq_kernel<2><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, tdq, p);
     OMQ_LAUNCH_CHECK();
     return OMQ_OK;
   }
   if (!a.d_ready) {
     const int64_t rows = (int64_t)a.T * a.H;
-    omq_launch(attn_rowdot_kernel, (unsigned)((rows + 7) / 8), 256, 0, st, a.T, a.H, a.dO, a.lddo, a.O, a.ldo, a.D, ldl);
+    attn_rowdot_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(a.T, a.H, a.dO, a.lddo, a.O, a.ldo, a.D, ldl);
     OMQ_LAUNCH_CHECK();
   }
-  omq_launch(flash_bwd_dkv_kernel<false>, g1, FA_THREADS, BL<false>::SMEM, st, tq64, tk, tv, tdo64, tdk, tdv, p);
+  flash_bwd_dkv_kernel<false><<<g1, FA_THREADS, BL<false>::SMEM, st>>>(tq64, tk, tv, tdo64, tdk, tdv, p);
   OMQ_LAUNCH_CHECK();
-  omq_launch(flash_bwd_dq_kernel<0>, g2, FA_THREADS, Q_SMEM, st, tq, tk64, tv64, tdo, tdq, p);
+  flash_bwd_dq_kernel<0><<<g2, FA_THREADS, Q_SMEM, st>>>(tq, tk64, tv64, tdo, tdq, p);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }

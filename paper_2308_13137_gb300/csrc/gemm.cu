@@ -442,7 +442,6 @@ __global__ void __launch_bounds__(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1)
   if (PAIR) cluster_sync();                 // both CTAs' barriers initialised before any remote use
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
-  omq_pdl_enter();                          // setup done: the predecessor's outputs from here on
 
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer ----------------
@@ -762,7 +761,7 @@ omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap&
   const int64_t sms = omq_num_sms();
   if (!PAIR) {
     const unsigned grid = (unsigned)(tiles < sms ? tiles : sms);
-    omq_launch(kern, grid, LWC ? NUM_THREADS_LWC : NUM_THREADS, L::TOTAL, st, ta, tb, tc, p);
+    kern<<<grid, LWC ? NUM_THREADS_LWC : NUM_THREADS, L::TOTAL, st>>>(ta, tb, tc, p);
   } else {
     const int64_t pairs = sms / 2;
     const unsigned grid = (unsigned)(2 * (tiles < pairs ? tiles : pairs));
@@ -771,15 +770,13 @@ omq_status launch_cfg(cudaStream_t st, const CUtensorMap& ta, const CUtensorMap&
     cfg.blockDim = dim3(LWC ? NUM_THREADS_LWC : NUM_THREADS, 1, 1);
     cfg.dynamicSmemBytes = L::TOTAL;
     cfg.stream = st;
-    cudaLaunchAttribute attr[2];
+    cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
-    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 2;
+    cfg.numAttrs = 1;
     if (cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, p) != cudaSuccess) return OMQ_ERR_CUDA;
   }
   OMQ_LAUNCH_CHECK();

@@ -17,7 +17,6 @@ __global__ void __launch_bounds__(LI_THREADS) colstats_kernel(const TX* __restri
                                                               int64_t ldx, const float* __restrict__ rstd,
                                                               float* __restrict__ absmax, float* __restrict__ sum,
                                                               int first) {
-  omq_pdl_enter();
   __shared__ float rm[8][33], rs[8][33];
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
   const int64_t c = (int64_t)blockIdx.x * 32 + tx;
@@ -44,7 +43,6 @@ __global__ void __launch_bounds__(LI_THREADS) colstats_kernel(const TX* __restri
 // max over output rows of |W[o, c]| for a bf16 [Cout, Cin] weight
 __global__ void __launch_bounds__(LI_THREADS) weight_colmax_kernel(const __nv_bfloat16* __restrict__ W, int64_t Cout,
                                                                    int64_t Cin, float* __restrict__ out, int first) {
-  omq_pdl_enter();
   __shared__ float rm[8][33];
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
   const int64_t c = (int64_t)blockIdx.x * 32 + tx;
@@ -69,7 +67,6 @@ __device__ __forceinline__ float smooth_scale(float xmax, float wmax, float alph
 // s, delta of a [norm, linears] pair: one thread per channel
 __global__ void smooth_pair_kernel(int64_t C, const float* xmax, const float* xsum, const float* wmax, double ntok,
                                    float alpha, float floor, float* s, float* delta) {
-  omq_pdl_enter();
   const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= C) return;
   s[c] = smooth_scale(xmax[c], wmax[c], alpha, floor);
@@ -81,7 +78,6 @@ __global__ void smooth_pair_kernel(int64_t C, const float* xmax, const float* xs
 __global__ void kv_pairs_kernel(int Hkv, int rep, int hd, const float* omax, const float* osum, const float* womax,
                                 const float* qmax, const float* kmax, double ntok, float alpha, float floor,
                                 float* so, float* do_, float* sa) {
-  omq_pdl_enter();
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= Hkv * hd) return;
   const int g = c / hd, e = c % hd;
@@ -104,28 +100,28 @@ __global__ void kv_pairs_kernel(int Hkv, int rep, int hd, const float* omax, con
 
 omq_status let_colstats(cudaStream_t st, const float* X, int64_t n, int64_t C, int64_t ldx, const float* rstd,
                         float* absmax, float* sum, int first) {
-  omq_launch(colstats_kernel<float>, (unsigned)((C + 31) / 32), LI_THREADS, 0, st, X, n, C, ldx, rstd, absmax, sum, first);
+  colstats_kernel<float><<<(unsigned)((C + 31) / 32), LI_THREADS, 0, st>>>(X, n, C, ldx, rstd, absmax, sum, first);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 omq_status let_colstats_bf16(cudaStream_t st, const __nv_bfloat16* X, int64_t n, int64_t C, int64_t ldx,
                              float* absmax, int first) {
-  omq_launch(colstats_kernel<__nv_bfloat16>, (unsigned)((C + 31) / 32), LI_THREADS, 0, st, X, n, C, ldx, nullptr, absmax,
+  colstats_kernel<__nv_bfloat16><<<(unsigned)((C + 31) / 32), LI_THREADS, 0, st>>>(X, n, C, ldx, nullptr, absmax,
                                                                                    nullptr, first);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 omq_status let_weight_colmax(cudaStream_t st, const __nv_bfloat16* W, int64_t Cout, int64_t Cin, float* out, int first) {
-  omq_launch(weight_colmax_kernel, (unsigned)((Cin + 31) / 32), LI_THREADS, 0, st, W, Cout, Cin, out, first);
+  weight_colmax_kernel<<<(unsigned)((Cin + 31) / 32), LI_THREADS, 0, st>>>(W, Cout, Cin, out, first);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 omq_status let_smooth_pair(cudaStream_t st, int64_t C, const float* xmax, const float* xsum, const float* wmax,
                            double ntok, float alpha, float floor, float* s, float* delta) {
-  omq_launch(smooth_pair_kernel, (unsigned)((C + 255) / 256), 256, 0, st, C, xmax, xsum, wmax, ntok, alpha, floor, s, delta);
+  smooth_pair_kernel<<<(unsigned)((C + 255) / 256), 256, 0, st>>>(C, xmax, xsum, wmax, ntok, alpha, floor, s, delta);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -134,7 +130,7 @@ omq_status let_kv_pairs(cudaStream_t st, int Hkv, int rep, int hd, const float* 
                         const float* womax, const float* qmax, const float* kmax, double ntok, float alpha, float floor,
                         float* so, float* do_, float* sa) {
   const int n = Hkv * hd;
-  omq_launch(kv_pairs_kernel, (unsigned)((n + 255) / 256), 256, 0, st, Hkv, rep, hd, omax, osum, womax, qmax, kmax, ntok, alpha,
+  kv_pairs_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(Hkv, rep, hd, omax, osum, womax, qmax, kmax, ntok, alpha,
                                                                floor, so, do_, sa);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;

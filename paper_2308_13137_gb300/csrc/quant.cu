@@ -73,7 +73,6 @@ __device__ __forceinline__ float dot8(const uint4& raw, const float* d, int64_t 
 // MODE 0: quantization off; 1: one group per row; 2: groups of <= 256 columns
 template <int MODE>
 __global__ void __launch_bounds__(256, 4) lwc_fwd_kernel(LwcFwdArgs a) {
-  omq_pdl_enter();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t o = (int64_t)blockIdx.x * 8 + warp;
   if (o >= a.Cout) return;                       // whole warp leaves; no block-level barrier below
@@ -234,7 +233,6 @@ __global__ void __launch_bounds__(256, 4) lwc_fwd_kernel(LwcFwdArgs a) {
 // bit except the LET bias dot, whose summation order differs.
 template <int NT, int CPT>
 __global__ void __launch_bounds__(NT) lwc_fwd_row_kernel(LwcFwdArgs a) {
-  omq_pdl_enter();
   constexpr int NW = NT / 32;
   __shared__ float red[3][NW];
   __shared__ int sidx[2];
@@ -332,10 +330,10 @@ __global__ void __launch_bounds__(NT) lwc_fwd_row_kernel(LwcFwdArgs a) {
 template <int NT>
 static void lwc_fwd_row_go(cudaStream_t st, const LwcFwdArgs& a, int64_t cpt) {
   const unsigned grid = (unsigned)a.Cout;
-  if (cpt <= 2) omq_launch(lwc_fwd_row_kernel<NT, 2>, grid, NT, 0, st, a);
-  else if (cpt <= 4) omq_launch(lwc_fwd_row_kernel<NT, 4>, grid, NT, 0, st, a);
-  else if (cpt <= 6) omq_launch(lwc_fwd_row_kernel<NT, 6>, grid, NT, 0, st, a);
-  else omq_launch(lwc_fwd_row_kernel<NT, 8>, grid, NT, 0, st, a);
+  if (cpt <= 2) lwc_fwd_row_kernel<NT, 2><<<grid, NT, 0, st>>>(a);
+  else if (cpt <= 4) lwc_fwd_row_kernel<NT, 4><<<grid, NT, 0, st>>>(a);
+  else if (cpt <= 6) lwc_fwd_row_kernel<NT, 6><<<grid, NT, 0, st>>>(a);
+  else lwc_fwd_row_kernel<NT, 8><<<grid, NT, 0, st>>>(a);
 }
 
 static bool lwc_group_ok(int64_t Cin, int g) {
@@ -349,12 +347,12 @@ omq_status lwc_fwd_launch(cudaStream_t st, const LwcFwdArgs& a) {
   OMQ_REQUIRE(lwc_group_ok(a.Cin, a.group), OMQ_ERR_UNSUPPORTED);
   const unsigned grid = (unsigned)((a.Cout + 7) / 8);
   const int64_t nchunk = a.Cin / 8;
-  if (a.wbits >= 16) omq_launch(lwc_fwd_kernel<0>, grid, 256, 0, st, a);
+  if (a.wbits >= 16) lwc_fwd_kernel<0><<<grid, 256, 0, st>>>(a);
   else if (a.group == a.Cin && nchunk <= 128 * 8) lwc_fwd_row_go<128>(st, a, (nchunk + 127) / 128);
   else if (a.group == a.Cin && nchunk <= 256 * 8) lwc_fwd_row_go<256>(st, a, (nchunk + 255) / 256);
   else if (a.group == a.Cin && nchunk <= 512 * 8) lwc_fwd_row_go<512>(st, a, (nchunk + 511) / 512);
-  else if (a.group == a.Cin) omq_launch(lwc_fwd_kernel<1>, grid, 256, 0, st, a);
-  else omq_launch(lwc_fwd_kernel<2>, grid, 256, 0, st, a);
+  else if (a.group == a.Cin) lwc_fwd_kernel<1><<<grid, 256, 0, st>>>(a);
+  else lwc_fwd_kernel<2><<<grid, 256, 0, st>>>(a);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -410,7 +408,6 @@ size_t lwc_bwd_scratch_bytes(int64_t Cout, int64_t Cin) {
 }
 
 __global__ void sigmoid_pair_kernel(const float* gl, const float* bl, int64_t n, float* ga, float* gb) {
-  omq_pdl_enter();
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) { ga[i] = omq_sigmoid(gl[i]); gb[i] = omq_sigmoid(bl[i]); }
 }
@@ -423,7 +420,6 @@ __device__ __forceinline__ float lwc_sig(const float* saved, const float* logit,
 #define LWC_BWD_RB 1          // rows whose loads are issued together
 
 __global__ void __launch_bounds__(LWC_BWD_THREADS, 3) lwc_bwd_tile_kernel(LwcBwdArgs a, LwcBwdScratch sc) {
-  omq_pdl_enter();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t nchunk = a.Cin / 8;
   const int64_t c = (int64_t)blockIdx.x * LWC_BWD_THREADS + tid;     // this thread's chunk
@@ -580,7 +576,6 @@ __global__ void __launch_bounds__(LWC_BWD_THREADS, 3) lwc_bwd_tile_kernel(LwcBwd
 // of dW~ to the row's max / min element.  The routing's share of ds is written to route[o] =
 // (max column, value, min column, value) and added to the column partials by lwc_route_kernel.
 __global__ void __launch_bounds__(256) lwc_bwd_finalize_kernel(LwcBwdArgs a, LwcBwdScratch sc, float4* route) {
-  omq_pdl_enter();
   const int lane = threadIdx.x & 31;
   const int64_t o = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   if (o >= a.Cout) return;
@@ -644,7 +639,6 @@ __device__ __forceinline__ void route_add(float* prow, int col, float v, int lan
 // so that ds does not depend on the order in which warps run.
 __global__ void __launch_bounds__(256) lwc_route_kernel(const float4* __restrict__ route, int64_t Cout, int64_t R,
                                                         float* __restrict__ part_s, int64_t Cin) {
-  omq_pdl_enter();
   const int lane = threadIdx.x & 31;
   const int64_t pidx = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   if (pidx * R >= Cout) return;                       // whole warp
@@ -670,22 +664,22 @@ omq_status lwc_bwd_launch(cudaStream_t st, const LwcBwdArgs& a0, void* scratch) 
   LwcBwdScratch sc = lwc_bwd_carve(scratch, a.Cout, a.Cin, ng, nullptr);
   if (a.lwc && (!a.ga || !a.gb)) {           // one sigmoid per group, not one per element
     const int64_t n = a.Cout * ng;
-    omq_launch(sigmoid_pair_kernel, (unsigned)((n + 255) / 256), 256, 0, st, a.gl, a.bl, n, sc.sig, sc.sig + n);
+    sigmoid_pair_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(a.gl, a.bl, n, sc.sig, sc.sig + n);
     OMQ_LAUNCH_CHECK();
     a.ga = sc.sig;
     a.gb = sc.sig + n;
   }
   const int64_t ncol = (a.Cin / 8 + LWC_BWD_THREADS - 1) / LWC_BWD_THREADS;
   dim3 grid((unsigned)ncol, (unsigned)sc.nrt);
-  omq_launch(lwc_bwd_tile_kernel, grid, LWC_BWD_THREADS, 0, st, a, sc);
+  lwc_bwd_tile_kernel<<<grid, LWC_BWD_THREADS, 0, st>>>(a, sc);
   OMQ_LAUNCH_CHECK();
   // the finalize and the routing of ds into the partial rows, then the partial rows are reduced
   if (perch || a.dr) {
-    omq_launch(lwc_bwd_finalize_kernel, (unsigned)((a.Cout + 7) / 8), 256, 0, st, a, sc, reinterpret_cast<float4*>(sc.route));
+    lwc_bwd_finalize_kernel<<<(unsigned)((a.Cout + 7) / 8), 256, 0, st>>>(a, sc, reinterpret_cast<float4*>(sc.route));
     OMQ_LAUNCH_CHECK();
   }
   if (perch && a.ds) {
-    omq_launch(lwc_route_kernel, (unsigned)((sc.nrt + 7) / 8), 256, 0, st, reinterpret_cast<const float4*>(sc.route), a.Cout,
+    lwc_route_kernel<<<(unsigned)((sc.nrt + 7) / 8), 256, 0, st>>>(reinterpret_cast<const float4*>(sc.route), a.Cout,
                                                                     sc.rows, sc.part_s, a.Cin);
     OMQ_LAUNCH_CHECK();
   }
@@ -710,10 +704,10 @@ omq_status lwc_bwd_fused_finish(cudaStream_t st, const LwcBwdArgs& a0, float* ro
     sc.rowpart = rowpart;
     sc.ncw = ntn;
     sc.ng = a.Cin / a.group;
-    omq_launch(lwc_bwd_finalize_kernel, (unsigned)((a.Cout + 7) / 8), 256, 0, st, a, sc, reinterpret_cast<float4*>(route));
+    lwc_bwd_finalize_kernel<<<(unsigned)((a.Cout + 7) / 8), 256, 0, st>>>(a, sc, reinterpret_cast<float4*>(route));
     OMQ_LAUNCH_CHECK();
     if (perch && want_s) {
-      omq_launch(lwc_route_kernel, (unsigned)((nparts + 7) / 8), 256, 0, st, reinterpret_cast<const float4*>(route), a.Cout,
+      lwc_route_kernel<<<(unsigned)((nparts + 7) / 8), 256, 0, st>>>(reinterpret_cast<const float4*>(route), a.Cout,
                                                                       32, part_s, a.Cin);
       OMQ_LAUNCH_CHECK();
     }
@@ -734,7 +728,6 @@ omq_status lwc_bwd_fused_finish(cudaStream_t st, const LwcBwdArgs& a0, float* ro
 // ================================================================================================
 __global__ void pack_codes_kernel(const uint8_t* __restrict__ codes, int64_t Cout, int64_t Cin, int nbits,
                                   uint8_t* __restrict__ out) {
-  omq_pdl_enter();
   const int64_t nchunk = Cin / 8;
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;     // one 8-code chunk
   if (i >= Cout * nchunk) return;
@@ -751,13 +744,12 @@ __global__ void pack_codes_kernel(const uint8_t* __restrict__ codes, int64_t Cou
 omq_status pack_codes_launch(cudaStream_t st, const uint8_t* codes, int64_t Cout, int64_t Cin, int nbits, uint8_t* out) {
   OMQ_REQUIRE(Cin % 8 == 0 && nbits >= 1 && nbits <= 8, OMQ_ERR_SHAPE);
   const int64_t n = Cout * (Cin / 8);
-  omq_launch(pack_codes_kernel, (unsigned)((n + 255) / 256), 256, 0, st, codes, Cout, Cin, nbits, out);
+  pack_codes_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(codes, Cout, Cin, nbits, out);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 __global__ void norm_fold_kernel(int64_t n, const float* s, const float* d, float* gain, float* bias) {
-  omq_pdl_enter();
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   gain[i] = 1.0f / s[i];
@@ -765,7 +757,7 @@ __global__ void norm_fold_kernel(int64_t n, const float* s, const float* d, floa
 }
 
 omq_status norm_fold_launch(cudaStream_t st, int64_t n, const float* s, const float* d, float* gain, float* bias) {
-  omq_launch(norm_fold_kernel, (unsigned)((n + 255) / 256), 256, 0, st, n, s, d, gain, bias);
+  norm_fold_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(n, s, d, gain, bias);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -777,7 +769,6 @@ omq_status norm_fold_launch(cudaStream_t st, int64_t n, const float* s, const fl
 // Used when the column count or a pointer does not allow 16-byte accesses.
 __global__ void omq_colsum_partials_kernel(const float* __restrict__ part, int64_t P, int64_t C,
                                            float* __restrict__ out, float scale, int accumulate) {
-  omq_pdl_enter();
   __shared__ float red[8][33];
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
   const int64_t c = (int64_t)blockIdx.x * 32 + tx;
@@ -805,7 +796,6 @@ __device__ __forceinline__ void add4(float4& a, const float4 b) { a.x += b.x; a.
 // blockIdx.z selects one of two independent reductions of one launch
 __global__ void __cluster_dims__(1, COLSUM_CLUSTER, 1) __launch_bounds__(256)
     colsum_cluster_kernel(ColsumJob j0, ColsumJob j1) {
-  omq_pdl_enter();
   const ColsumJob& J = blockIdx.z == 0 ? j0 : j1;
   const float* __restrict__ part = J.part;
   const int64_t P = J.P, C = J.C;
@@ -865,7 +855,7 @@ omq_status omq_colsum_partials2(cudaStream_t st, const ColsumJob& a, const Colsu
   }
   const int64_t C = a.C > b.C ? a.C : b.C;
   dim3 grid((unsigned)((C / 4 + 31) / 32), COLSUM_CLUSTER, 2);
-  omq_launch(colsum_cluster_kernel, grid, 256, 0, st, a, b);
+  colsum_cluster_kernel<<<grid, 256, 0, st>>>(a, b);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -875,9 +865,9 @@ omq_status omq_colsum_partials(cudaStream_t st, const float* part, int64_t P, in
   ColsumJob j{part, P, C, out, scale, accumulate};
   if (colsum_vec_ok(j)) {
     dim3 grid((unsigned)((C / 4 + 31) / 32), COLSUM_CLUSTER);
-    omq_launch(colsum_cluster_kernel, grid, 256, 0, st, j, j);
+    colsum_cluster_kernel<<<grid, 256, 0, st>>>(j, j);
   } else {
-    omq_launch(omq_colsum_partials_kernel, (unsigned)((C + 31) / 32), 256, 0, st, part, P, C, out, scale, accumulate);
+    omq_colsum_partials_kernel<<<(unsigned)((C + 31) / 32), 256, 0, st>>>(part, P, C, out, scale, accumulate);
   }
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
@@ -886,7 +876,6 @@ omq_status omq_colsum_partials(cudaStream_t st, const float* part, int64_t P, in
 // stage 1 of a column sum over rows: part[blockIdx.y, n] = sum of X[t, n] over 128 rows
 __global__ void colsum_rows_kernel(const float* __restrict__ X, int64_t T, int64_t N, int64_t ldx,
                                    float* __restrict__ part) {
-  omq_pdl_enter();
   int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (n >= N) return;
   int64_t t0 = (int64_t)blockIdx.y * 128, t1 = min(T, t0 + 128);
@@ -900,7 +889,6 @@ __global__ void colsum_rows_kernel(const float* __restrict__ X, int64_t T, int64
 // in warp order
 __global__ void __launch_bounds__(256) colsum_rows_vec_kernel(const float* __restrict__ X, int64_t T, int64_t N,
                                                               int64_t ldx, float* __restrict__ part) {
-  omq_pdl_enter();
   __shared__ float4 red[8][32];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int64_t c = (int64_t)blockIdx.x * 128 + 4 * lane;
@@ -933,7 +921,6 @@ int64_t colsum_rows_parts(int64_t T) { return (T + 127) / 128; }
 // columns (one 16-byte load per row), the eight warps of a CTA stride the slab's rows
 __global__ void __launch_bounds__(256) colsum_rows_bf16_kernel(const __nv_bfloat16* __restrict__ X, int64_t T,
                                                                int64_t N, int64_t ldx, float* __restrict__ part) {
-  omq_pdl_enter();
   __shared__ float red[8][32][9];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int64_t c = (int64_t)blockIdx.x * 256 + 8 * lane;
@@ -981,7 +968,7 @@ omq_status colsum_rows_bf16(cudaStream_t st, const __nv_bfloat16* X, int64_t T, 
                             float* out, float scale, int accumulate) {
   OMQ_REQUIRE(N % 8 == 0 && ldx % 8 == 0 && omq_aligned16(X) && omq_aligned16(part), OMQ_ERR_ALIGN);
   dim3 grid((unsigned)((N + 255) / 256), (unsigned)colsum_rows_parts(T));
-  omq_launch(colsum_rows_bf16_kernel, grid, 256, 0, st, X, T, N, ldx, part);
+  colsum_rows_bf16_kernel<<<grid, 256, 0, st>>>(X, T, N, ldx, part);
   OMQ_LAUNCH_CHECK();
   return omq_colsum_partials(st, part, colsum_rows_parts(T), N, out, scale, accumulate);
 }
@@ -990,10 +977,10 @@ omq_status colsum_rows(cudaStream_t st, const float* X, int64_t T, int64_t N, in
                        float* out, float scale, int accumulate) {
   if (N % 4 == 0 && ldx % 4 == 0 && omq_aligned16(X) && omq_aligned16(part)) {
     dim3 grid((unsigned)((N + 127) / 128), (unsigned)colsum_rows_parts(T));
-    omq_launch(colsum_rows_vec_kernel, grid, 256, 0, st, X, T, N, ldx, part);
+    colsum_rows_vec_kernel<<<grid, 256, 0, st>>>(X, T, N, ldx, part);
   } else {
     dim3 grid((unsigned)((N + 255) / 256), (unsigned)colsum_rows_parts(T));
-    omq_launch(colsum_rows_kernel, grid, 256, 0, st, X, T, N, ldx, part);
+    colsum_rows_kernel<<<grid, 256, 0, st>>>(X, T, N, ldx, part);
   }
   OMQ_LAUNCH_CHECK();
   return omq_colsum_partials(st, part, colsum_rows_parts(T), N, out, scale, accumulate);
@@ -1002,7 +989,6 @@ omq_status colsum_rows(cudaStream_t st, const float* X, int64_t T, int64_t N, in
 __global__ void loss_partial_kernel(int64_t n, const float* __restrict__ Yq, const float* __restrict__ Yfp,
                                     float* __restrict__ dY, __nv_bfloat16* __restrict__ dYb,
                                     float* __restrict__ part) {
-  omq_pdl_enter();
   __shared__ float red_f[64];
   float s = 0.f;
   const float g = 2.0f / (float)n;
@@ -1018,7 +1004,6 @@ __global__ void loss_partial_kernel(int64_t n, const float* __restrict__ Yq, con
 }
 
 __global__ void loss_final_kernel(const float* __restrict__ part, int P, int64_t n, float* loss) {
-  omq_pdl_enter();
   __shared__ float red_f[64];
   float s = 0.f;
   for (int i = threadIdx.x; i < P; i += blockDim.x) s += part[i];
@@ -1034,37 +1019,34 @@ int64_t loss_parts(int64_t n) {
 omq_status loss_launch(cudaStream_t st, int64_t n, const float* Yq, const float* Yfp, float* loss,
                        float* dY, __nv_bfloat16* dYb, float* part) {
   int P = (int)loss_parts(n);
-  omq_launch(loss_partial_kernel, P, 256, 0, st, n, Yq, Yfp, dY, dYb, part);
+  loss_partial_kernel<<<P, 256, 0, st>>>(n, Yq, Yfp, dY, dYb, part);
   OMQ_LAUNCH_CHECK();
-  omq_launch(loss_final_kernel, 1, 256, 0, st, part, P, n, loss);
+  loss_final_kernel<<<1, 256, 0, st>>>(part, P, n, loss);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 __global__ void vec_fill_kernel(float* p, int64_t n, float v) {
-  omq_pdl_enter();
   int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) p[i] = v;
 }
 omq_status vec_fill(cudaStream_t st, float* p, int64_t n, float v) {
-  omq_launch(vec_fill_kernel, (unsigned)((n + 255) / 256), 256, 0, st, p, n, v);
+  vec_fill_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(p, n, v);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 __global__ void vec_copy_kernel(float* d, const float* s, int64_t n) {
-  omq_pdl_enter();
   int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) d[i] = s[i];
 }
 omq_status vec_copy(cudaStream_t st, float* dst, const float* src, int64_t n) {
-  omq_launch(vec_copy_kernel, (unsigned)((n + 255) / 256), 256, 0, st, dst, src, n);
+  vec_copy_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(dst, src, n);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 __global__ void gqa_expand_kernel(const float* src, float* dst, int n_kv, int rep, int hd, int op) {
-  omq_pdl_enter();
   int i = blockIdx.x * blockDim.x + threadIdx.x;
   int n = n_kv * rep * hd;
   if (i >= n) return;
@@ -1074,13 +1056,12 @@ __global__ void gqa_expand_kernel(const float* src, float* dst, int n_kv, int re
 }
 omq_status gqa_expand(cudaStream_t st, const float* src, float* dst, int n_kv, int rep, int hd, int op) {
   int n = n_kv * rep * hd;
-  omq_launch(gqa_expand_kernel, (n + 255) / 256, 256, 0, st, src, dst, n_kv, rep, hd, op);
+  gqa_expand_kernel<<<(n + 255) / 256, 256, 0, st>>>(src, dst, n_kv, rep, hd, op);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
 
 __global__ void gqa_fold_kernel(const float* src, float* dst, int n_kv, int rep, int hd, int accumulate) {
-  omq_pdl_enter();
   int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= n_kv * hd) return;
   int kv = c / hd, j = c % hd;
@@ -1090,7 +1071,7 @@ __global__ void gqa_fold_kernel(const float* src, float* dst, int n_kv, int rep,
 }
 omq_status gqa_fold(cudaStream_t st, const float* src, float* dst, int n_kv, int rep, int hd, int accumulate) {
   int n = n_kv * hd;
-  omq_launch(gqa_fold_kernel, (n + 255) / 256, 256, 0, st, src, dst, n_kv, rep, hd, accumulate);
+  gqa_fold_kernel<<<(n + 255) / 256, 256, 0, st>>>(src, dst, n_kv, rep, hd, accumulate);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -1099,7 +1080,6 @@ omq_status gqa_fold(cudaStream_t st, const float* src, float* dst, int n_kv, int
 // LET apply (Eq. 3) as a standalone operation
 // ================================================================================================
 __global__ void let_x_kernel(const float* X, int64_t T, int64_t C, const float* s, const float* d, float* Xt) {
-  omq_pdl_enter();
   int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= T * C) return;
   int64_t c = i % C;
@@ -1107,14 +1087,12 @@ __global__ void let_x_kernel(const float* X, int64_t T, int64_t C, const float* 
 }
 
 __global__ void let_w_kernel(const __nv_bfloat16* W, int64_t Cout, int64_t Cin, const float* s, float* Wt) {
-  omq_pdl_enter();
   int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= Cout * Cin) return;
   Wt[i] = __fmul_rn(bf16_to_f(W[i]), s[i % Cin]);
 }
 
 __global__ void let_b_kernel(const __nv_bfloat16* W, int64_t Cout, int64_t Cin, const float* B, const float* d, float* Bt) {
-  omq_pdl_enter();
   __shared__ float red_f[64];
   int64_t o = blockIdx.x;
   float acc = 0.f;
@@ -1128,7 +1106,6 @@ __global__ void let_b_kernel(const __nv_bfloat16* W, int64_t Cout, int64_t Cin, 
 // ================================================================================================
 __global__ void adamw_kernel(int64_t n, float* p, const float* g, float* m, float* v, float lr, float b1, float b2,
                              float eps, float wd, float bc1, float bc2) {
-  omq_pdl_enter();
   int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   float gi = g[i];
@@ -1143,7 +1120,6 @@ __global__ void adamw_kernel(int64_t n, float* p, const float* g, float* m, floa
 // the same, t read from device memory; bias corrections formed once per CTA
 __global__ void adamw_dev_kernel(int64_t n, float* p, const float* g, float* m, float* v, float lr, float b1, float b2,
                                  float eps, float wd, const int32_t* step) {
-  omq_pdl_enter();
   __shared__ float bc[2];
   if (threadIdx.x == 0) {
     const float t = (float)*step;
@@ -1162,8 +1138,7 @@ __global__ void adamw_dev_kernel(int64_t n, float* p, const float* g, float* m, 
   p[i] = pi - lr * (mi / bc[0]) / (sqrtf(vi / bc[1]) + eps) - lr * wd * pi;
 }
 
-__global__ void step_advance_kernel(int32_t* step) {
-  omq_pdl_enter(); *step += 1; }
+__global__ void step_advance_kernel(int32_t* step) { *step += 1; }
 
 // ================================================================================================
 // C ABI: kernel-level entry points
@@ -1180,17 +1155,17 @@ omq_status omq_let_apply(omq_stream_t stream, int64_t T, int64_t Cin, int64_t Co
   OMQ_REQUIRE(Cin % 8 == 0, OMQ_ERR_ALIGN);
   if (Xt) {
     OMQ_REQUIRE(X, OMQ_ERR_INVALID_ARG);
-    omq_launch(let_x_kernel, (unsigned)((T * Cin + 255) / 256), 256, 0, st, X, T, Cin, s, delta, Xt);
+    let_x_kernel<<<(unsigned)((T * Cin + 255) / 256), 256, 0, st>>>(X, T, Cin, s, delta, Xt);
     OMQ_LAUNCH_CHECK();
   }
   if (Wt) {
     OMQ_REQUIRE(W, OMQ_ERR_INVALID_ARG);
-    omq_launch(let_w_kernel, (unsigned)((Cout * Cin + 255) / 256), 256, 0, st, (const __nv_bfloat16*)W, Cout, Cin, s, Wt);
+    let_w_kernel<<<(unsigned)((Cout * Cin + 255) / 256), 256, 0, st>>>((const __nv_bfloat16*)W, Cout, Cin, s, Wt);
     OMQ_LAUNCH_CHECK();
   }
   if (Bt) {
     OMQ_REQUIRE(W, OMQ_ERR_INVALID_ARG);
-    omq_launch(let_b_kernel, (unsigned)Cout, 256, 0, st, (const __nv_bfloat16*)W, Cout, Cin, B, delta, Bt);
+    let_b_kernel<<<(unsigned)Cout, 256, 0, st>>>((const __nv_bfloat16*)W, Cout, Cin, B, delta, Bt);
     OMQ_LAUNCH_CHECK();
   }
   return OMQ_OK;
@@ -1349,7 +1324,7 @@ omq_status omq_adamw_update(omq_stream_t stream, int64_t n, float* p, const floa
   OMQ_REQUIRE(n > 0, OMQ_ERR_SHAPE);
   OMQ_REQUIRE(p && g && m && v && step >= 1, OMQ_ERR_INVALID_ARG);
   float bc1 = 1.f - powf(beta1, (float)step), bc2 = 1.f - powf(beta2, (float)step);
-  omq_launch(adamw_kernel, (unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream, n, p, g, m, v, lr, beta1, beta2, eps,
+  adamw_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(n, p, g, m, v, lr, beta1, beta2, eps,
                                                                               weight_decay, bc1, bc2);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
@@ -1360,7 +1335,7 @@ omq_status omq_adamw_update_dev(omq_stream_t stream, int64_t n, float* p, const 
                                 const int32_t* step_dev) {
   OMQ_REQUIRE(n > 0, OMQ_ERR_SHAPE);
   OMQ_REQUIRE(p && g && m && v && step_dev, OMQ_ERR_INVALID_ARG);
-  omq_launch(adamw_dev_kernel, (unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream, n, p, g, m, v, lr, beta1, beta2,
+  adamw_dev_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(n, p, g, m, v, lr, beta1, beta2,
                                                                                   eps, weight_decay, step_dev);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
@@ -1368,7 +1343,7 @@ omq_status omq_adamw_update_dev(omq_stream_t stream, int64_t n, float* p, const 
 
 omq_status omq_step_advance(omq_stream_t stream, int32_t* step_dev) {
   OMQ_REQUIRE(step_dev, OMQ_ERR_INVALID_ARG);
-  omq_launch(step_advance_kernel, 1, 1, 0, (cudaStream_t)stream, step_dev);
+  step_advance_kernel<<<1, 1, 0, (cudaStream_t)stream>>>(step_dev);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }

@@ -213,7 +213,6 @@ constexpr int kFwdRows = 2, kFwdRowsSwiglu = 2, kQkvFwdRows = 1;
 // inputs into L2 while it works on the current one
 template <int P, int NT, int VPT>
 __global__ void __launch_bounds__(NT) act_fwd_rows(ActFwdArgs a) {
-  omq_pdl_enter();
   __shared__ float fsm[64];
   __shared__ int ism[64];
   const int64_t R = a.rows_per_cta > 1 ? a.rows_per_cta : 1;
@@ -237,7 +236,6 @@ __global__ void __launch_bounds__(NT) act_fwd_rows(ActFwdArgs a) {
 // ================================================================================================
 template <int P, int NT, int VPT>
 __global__ void __launch_bounds__(NT) act_fwd_staged(ActFwdArgs a, int stages) {
-  omq_pdl_enter();
   constexpr int NE = 4 * VPT, NW = NT / 32, MAXS = 4;
   constexpr int NIN = P == AP_SWIGLU ? 2 : 1;
   extern __shared__ float4 stg4[];                 // [stages][NIN][C / 4]
@@ -446,7 +444,6 @@ struct ActBwdRow {
 
 template <int P, int VPT, int JB, int MINB, bool SUMS, bool RD = false>
 __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a) {
-  omq_pdl_enter();
   constexpr int NT = ACT_BWD_NT;
   constexpr bool LETP = (P == AP_LET || P == AP_RMS_LET);
   static_assert(!(SUMS && P == AP_SWIGLU), "SwiGLU has no LET column sums");
@@ -752,10 +749,10 @@ __global__ void __launch_bounds__(ACT_BWD_NT, MINB) act_bwd_stream(ActBwdArgs a)
 #define ACT_DISPATCH(KERNEL, ARGS, GRID, C)                                                          \
   do {                                                                                               \
     const int64_t nv_ = (C) / 4;                                                                     \
-    if (nv_ <= 512 * 2) omq_launch(KERNEL<PRODUCER, 512, 2>, (GRID), 512, 0, st, ARGS);                      \
-    else if (nv_ <= 512 * 4) omq_launch(KERNEL<PRODUCER, 512, 4>, (GRID), 512, 0, st, ARGS);                 \
-    else if (nv_ <= 1024 * 4) omq_launch(KERNEL<PRODUCER, 1024, 4>, (GRID), 1024, 0, st, ARGS);              \
-    else if (nv_ <= 1024 * 8) omq_launch(KERNEL<PRODUCER, 1024, 8>, (GRID), 1024, 0, st, ARGS);              \
+    if (nv_ <= 512 * 2) KERNEL<PRODUCER, 512, 2><<<(GRID), 512, 0, st>>>(ARGS);                      \
+    else if (nv_ <= 512 * 4) KERNEL<PRODUCER, 512, 4><<<(GRID), 512, 0, st>>>(ARGS);                 \
+    else if (nv_ <= 1024 * 4) KERNEL<PRODUCER, 1024, 4><<<(GRID), 1024, 0, st>>>(ARGS);              \
+    else if (nv_ <= 1024 * 8) KERNEL<PRODUCER, 1024, 8><<<(GRID), 1024, 0, st>>>(ARGS);              \
     else return OMQ_ERR_UNSUPPORTED;                                                                 \
   } while (0)
 
@@ -774,7 +771,7 @@ static omq_status act_fwd_staged_go(cudaStream_t st, const ActFwdArgs& a, int st
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, kern, NT, smem) != cudaSuccess || bps < 1) return OMQ_ERR_CUDA;
   (void)per_sm;
   const int64_t grid = std::min<int64_t>(a.T, (int64_t)omq_num_sms() * bps);
-  omq_launch(kern, (unsigned)grid, NT, smem, st, a, stages);
+  kern<<<(unsigned)grid, NT, smem, st>>>(a, stages);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -793,13 +790,13 @@ static omq_status act_fwd_dispatch(cudaStream_t st, const ActFwdArgs& a0) {
   const int64_t nv = a.C / 4;
   if (nv <= 128 * 8) {                             // small rows: many CTAs per SM, 32 values per thread
     a.rows_per_cta = kFwdRows;
-    omq_launch(act_fwd_rows<PRODUCER, 128, 8>, (unsigned)((a.T + kFwdRows - 1) / kFwdRows), 128, 0, st, a);
+    act_fwd_rows<PRODUCER, 128, 8><<<(unsigned)((a.T + kFwdRows - 1) / kFwdRows), 128, 0, st>>>(a);
     OMQ_LAUNCH_CHECK();
     return OMQ_OK;
   }
   if (PRODUCER == AP_SWIGLU && nv <= 256 * 12) {
     a.rows_per_cta = kFwdRowsSwiglu;
-    omq_launch(act_fwd_rows<PRODUCER, 256, 12>, (unsigned)((a.T + kFwdRowsSwiglu - 1) / kFwdRowsSwiglu), 256, 0, st, a);
+    act_fwd_rows<PRODUCER, 256, 12><<<(unsigned)((a.T + kFwdRowsSwiglu - 1) / kFwdRowsSwiglu), 256, 0, st>>>(a);
     OMQ_LAUNCH_CHECK();
     return OMQ_OK;
   }
@@ -818,7 +815,7 @@ static omq_status act_fwd_dispatch(cudaStream_t st, const ActFwdArgs& a0) {
 template <int PRODUCER, int VPT, int JB, int MINB, bool SUMS, bool RD = false>
 static omq_status act_bwd_go(cudaStream_t st, const ActBwdArgs& a) {
   const int64_t nparts = (a.T + a.rows_per_cta - 1) / a.rows_per_cta;
-  omq_launch(act_bwd_stream<PRODUCER, VPT, JB, MINB, SUMS, RD>, (unsigned)nparts, ACT_BWD_NT, 0, st, a);
+  act_bwd_stream<PRODUCER, VPT, JB, MINB, SUMS, RD><<<(unsigned)nparts, ACT_BWD_NT, 0, st>>>(a);
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
 }
@@ -947,7 +944,6 @@ __device__ __forceinline__ void qkv_load(const QkvArgs& a, int seg, int t, QkvRo
 
 template <int NT, int PPT>
 __global__ void __launch_bounds__(NT) qkv_fwd_rows(QkvArgs a) {
-  omq_pdl_enter();
   constexpr int NE = 8 * PPT;
   __shared__ float fsm[64];
   __shared__ int ism[64];
@@ -1190,7 +1186,6 @@ __device__ __forceinline__ void qkv_bwd_body(const QkvArgs& a, float* fsm) {
 
 template <int PPT, int MINB>
 __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
-  omq_pdl_enter();
   __shared__ float fsm[96];
   qkv_bwd_body<PPT, -1>(a, fsm);
 }
@@ -1198,7 +1193,6 @@ __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_stream(QkvArgs a) {
 // one CTA per (row slab, segment): blockIdx.y picks q, k or v
 template <int PPT, int MINB>
 __global__ void __launch_bounds__(QKV_BWD_NT, MINB) qkv_bwd_seg(QkvArgs a) {
-  omq_pdl_enter();
   __shared__ float fsm[96];
   if (blockIdx.y == 0) qkv_bwd_body<PPT, 0>(a, fsm);
   else if (blockIdx.y == 1) qkv_bwd_body<PPT, 1>(a, fsm);
@@ -1214,9 +1208,9 @@ omq_status qkv_fwd_launch(cudaStream_t st, const QkvArgs& a) {
   OMQ_REQUIRE(a.hd == 128, OMQ_ERR_UNSUPPORTED);
   const int np = a.H * 16;
   const dim3 g3((unsigned)((a.T + kQkvFwdRows - 1) / kQkvFwdRows), 3);   // one CTA per (token rows, q | k | v)
-  if (np <= 512) omq_launch(qkv_fwd_rows<128, 4>, g3, 128, 0, st, a);
-  else if (np <= 1024) omq_launch(qkv_fwd_rows<512, 2>, g3.x, 512, 0, st, a);
-  else if (np <= 2048) omq_launch(qkv_fwd_rows<512, 4>, g3.x, 512, 0, st, a);
+  if (np <= 512) qkv_fwd_rows<128, 4><<<g3, 128, 0, st>>>(a);
+  else if (np <= 1024) qkv_fwd_rows<512, 2><<<g3.x, 512, 0, st>>>(a);
+  else if (np <= 2048) qkv_fwd_rows<512, 4><<<g3.x, 512, 0, st>>>(a);
   else return OMQ_ERR_UNSUPPORTED;
   OMQ_LAUNCH_CHECK();
   return OMQ_OK;
@@ -1228,10 +1222,10 @@ omq_status qkv_bwd_launch(cudaStream_t st, const QkvArgs& a0, int64_t* nslab) {
   a.rows_per_cta = kQkvBwdRows;
   const unsigned grid = (unsigned)qkv_bwd_nslab(a.T);
   const int np = a.H * 16;
-  if (np <= 256) omq_launch(qkv_bwd_stream<1, 4>, grid, QKV_BWD_NT, 0, st, a);
-  else if (np <= 512) omq_launch(qkv_bwd_seg<2, 2>, dim3(grid, 3), QKV_BWD_NT, 0, st, a);
-  else if (np <= 1024) omq_launch(qkv_bwd_stream<4, 1>, grid, QKV_BWD_NT, 0, st, a);
-  else if (np <= 2048) omq_launch(qkv_bwd_stream<8, 1>, grid, QKV_BWD_NT, 0, st, a);
+  if (np <= 256) qkv_bwd_stream<1, 4><<<grid, QKV_BWD_NT, 0, st>>>(a);
+  else if (np <= 512) qkv_bwd_seg<2, 2><<<dim3(grid, 3), QKV_BWD_NT, 0, st>>>(a);
+  else if (np <= 1024) qkv_bwd_stream<4, 1><<<grid, QKV_BWD_NT, 0, st>>>(a);
+  else if (np <= 2048) qkv_bwd_stream<8, 1><<<grid, QKV_BWD_NT, 0, st>>>(a);
   else return OMQ_ERR_UNSUPPORTED;
   OMQ_LAUNCH_CHECK();
   if (nslab) *nslab = qkv_bwd_nslab(a.T);
